@@ -1,0 +1,481 @@
+"""Plain fp64 CPU oracle of the candidate-scoring path of SCOOT.
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, the smoke check and the
+benchmark's CPU-baseline leg may import this module.  It shares no code
+with the CUDA path: it takes the same seeded inputs (raw configuration words,
+observed values, hyperparameters, forest nodes, base samples) and computes
+every step on its own, slowly and directly, in float64.
+
+Steps, in the order of one suggestion round (Section 4, Algorithm 1):
+
+1. known-constraint pruning, Eq. (2) and the appendix on known constraints;
+2. random-forest probability of feasibility, Eq. (3) (Section 4.6);
+3. GP posterior mean and variance, the two equations of Section 4.3;
+4. acquisition: EI, Eq. (6), or Monte-Carlo EHVI, Eq. (7), with the
+   hypervolume of Section 4.4 (Fig. 4);
+5. top-q selection for parallel suggestion (Section 4.7);
+6. sequential picks with kriging-believer fantasies (not in the paper; the
+   refit form is used here: each pick is appended to the observations with
+   its posterior mean as value and the GP is conditioned again).
+
+Readings of points the paper leaves open are marked "Reading:".
+Every function is pinned by the not-gpu tests against closed forms,
+invariants, brute force or library routines; nothing here is "parity
+unpinned".
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import scipy.linalg as sla
+from scipy.special import erfc
+
+INT_UNIFORM, INT_LOG, CATEGORICAL, CONTINUOUS = 0, 1, 2, 3
+MATERN52, MATERN32 = 0, 1
+NODE_LEAF = 1
+
+
+# --------------------------------------------------------------------------
+# decoding
+
+def decode(space, words: np.ndarray, n: int | None = None) -> np.ndarray:
+    """Stored values of candidates as float64 [n][d].
+
+    Integers and category indices are int32 words; continuous values are
+    float32 bit patterns (Section 3's mixed space of int / enum / float /
+    bool parameters).
+    """
+    n = words.shape[1] if n is None else n
+    cols = []
+    for i in range(len(space)):
+        w = np.ascontiguousarray(words[i, :n])
+        if int(space[i]["kind"]) == CONTINUOUS:
+            cols.append(w.view(np.float32).astype(np.float64))
+        else:
+            cols.append(w.view(np.int32).astype(np.float64))
+    return np.stack(cols, axis=1) if cols else np.zeros((n, 0))
+
+
+# --------------------------------------------------------------------------
+# 1. known constraints, Eq. (2)
+
+def prune_mask(space, clauses, words: np.ndarray, n: int) -> np.ndarray:
+    """mask[i] = every clause c of C holds for candidate i (Eq. 2).
+
+    Reading: a clause is "all guards hold => sum_t coef_t x[param_t] >= rhs",
+    evaluated in exact integer arithmetic; the inclusive ">=" follows the
+    appendix ("greater than or equal to").  The example constraint of
+    Section 3 ("x[1] < x[3] if x[4] is False") is a clause with one guard.
+    """
+    x = decode(space, words, n)
+    mask = np.ones(n, dtype=bool)
+    for c in clauses:
+        guard = np.ones(n, dtype=bool)
+        for g in range(int(c["n_guard"])):
+            p = int(c["guard_param"][g])
+            guard &= x[:, p].astype(np.int64) == int(c["guard_value"][g])
+        lhs = np.zeros(n, dtype=object)
+        for t in range(int(c["n_term"])):
+            p = int(c["term_param"][t])
+            lhs = lhs + int(c["coef"][t]) * x[:, p].astype(np.int64).astype(object)
+        holds = np.array([int(v) >= int(c["rhs"]) for v in lhs], dtype=bool) if n else np.zeros(0, bool)
+        mask &= (~guard) | holds
+    return mask
+
+
+# --------------------------------------------------------------------------
+# 2. random-forest probability of feasibility, Eq. (3)
+
+def tree_walk(nodes: np.ndarray, base: int, x: np.ndarray) -> float:
+    """Leaf value of the regression tree whose root is nodes[base], for one
+    configuration x, by recursion from the root.
+
+    Reading: an internal node sends x to its left child when x[feat] <= thr;
+    the right child sits right after the left one; child indices are
+    relative to the tree's root.
+    """
+    return _walk_from(nodes, base, 0, x)
+
+
+def _walk_from(nodes, tree_base, idx, x):
+    nd = nodes[tree_base + idx]
+    if int(nd["flags"]) & NODE_LEAF:
+        return float(nd["val"])
+    left = int(nd["left"])
+    return _walk_from(nodes, tree_base, left if x[int(nd["feat"])] <= float(nd["val"]) else left + 1, x)
+
+
+def rf_votes_one(nodes, tree_offset, x: np.ndarray) -> int:
+    """Sum over trees of the integer leaf votes for one configuration."""
+    total = 0
+    for t in range(len(tree_offset) - 1):
+        total += int(_walk_from(nodes, int(tree_offset[t]), 0, x))
+    return total
+
+
+def rf_votes(nodes, tree_offset, space, words, n: int) -> np.ndarray:
+    """Votes for all n candidates: the same tree walk, vectorised over candidates."""
+    x = decode(space, words, n)
+    votes = np.zeros(n, dtype=np.int64)
+    for t in range(len(tree_offset) - 1):
+        base = int(tree_offset[t])
+        size = int(tree_offset[t + 1]) - base
+        tree = nodes[base:base + size]
+        idx = np.zeros(n, dtype=np.int64)
+        for _ in range(size + 1):
+            leaf = (tree["flags"][idx] & NODE_LEAF) != 0
+            if leaf.all():
+                break
+            feat = tree["feat"][idx].astype(np.int64)
+            thr = tree["val"][idx].astype(np.float64)
+            left = tree["left"][idx].astype(np.int64)
+            xv = x[np.arange(n), feat]
+            nxt = np.where(xv <= thr, left, left + 1)
+            idx = np.where(leaf, idx, nxt)
+        votes += tree["val"][idx].astype(np.float64).astype(np.int64)
+    return votes
+
+
+def pof_feasible(votes, n_trees: int, leaf_scale: int, delta_num: int, delta_den: int):
+    """POF(x) >= Delta (Eq. 3) with POF = votes / (leaf_scale * T), Delta = num / den.
+
+    Reading: the forest regresses a 0/1 feasibility label; each leaf stores
+    round(leaf_scale * mean label) so POF is an exact rational and the
+    test is the exact integer comparison den * votes >= num * scale * T.
+    """
+    v = np.asarray(votes, dtype=object)
+    lhs = v * int(delta_den)
+    rhs = int(delta_num) * int(leaf_scale) * int(n_trees)
+    return np.array([int(a) >= rhs for a in lhs], dtype=bool)
+
+
+# --------------------------------------------------------------------------
+# 3. GP posterior (Section 4.3)
+
+def gp_features(space, x: np.ndarray):
+    """Coordinates on which the covariance acts.
+
+    Reading (the paper does not say): integer log-uniform parameters on a log
+    scale, (ln v - ln lo) / (ln hi - ln lo); integer uniform and continuous
+    ones linearly, (v - lo) / (hi - lo); categoricals by their index, compared
+    for equality only.
+    """
+    u = np.array(x, dtype=np.float64, copy=True)
+    is_cat = np.zeros(len(space), dtype=bool)
+    for i in range(len(space)):
+        kind = int(space[i]["kind"])
+        lo, hi = float(space[i]["lo"]), float(space[i]["hi"])
+        if kind == INT_LOG:
+            u[:, i] = (np.log(x[:, i]) - math.log(lo)) / (math.log(hi) - math.log(lo))
+        elif kind in (INT_UNIFORM, CONTINUOUS):
+            u[:, i] = (x[:, i] - lo) / (hi - lo) if hi > lo else 0.0
+        else:
+            is_cat[i] = True
+    return u, is_cat
+
+
+def scaled_distance(ua, ub, is_cat, lengthscale) -> np.ndarray:
+    """r[a, b] with r^2 = sum_c ((ua_c - ub_c) / l_c)^2 over ordinal dims plus
+    sum_c [ua_c != ub_c] / l_c^2 over categorical dims (ARD lengthscales)."""
+    r2 = np.zeros((ua.shape[0], ub.shape[0]))
+    for c in range(ua.shape[1]):
+        ell = float(lengthscale[c])
+        if is_cat[c]:
+            r2 += (ua[:, c][:, None] != ub[:, c][None, :]).astype(np.float64) / (ell * ell)
+        else:
+            diff = (ua[:, c][:, None] - ub[:, c][None, :]) / ell
+            r2 += diff * diff
+    return np.sqrt(r2)
+
+
+def matern(r, signal_var: float, kernel: int = MATERN52):
+    """Matern covariance of smoothness 5/2 (default) or 3/2.
+
+    k_{5/2}(r) = s (1 + sqrt5 r + 5 r^2 / 3) exp(-sqrt5 r);
+    k_{3/2}(r) = s (1 + sqrt3 r) exp(-sqrt3 r)  (the paper's kernel, Section 4.3).
+    """
+    r = np.asarray(r, dtype=np.float64)
+    if kernel == MATERN52:
+        a = math.sqrt(5.0) * r
+        return signal_var * (1.0 + a + a * a / 3.0) * np.exp(-a)
+    if kernel == MATERN32:
+        a = math.sqrt(3.0) * r
+        return signal_var * (1.0 + a) * np.exp(-a)
+    raise ValueError(kernel)
+
+
+class GP:
+    """One objective's GP conditioned on the observations (Section 4.3)."""
+
+    def __init__(self, space, x_obs_words, y, lengthscale, signal_var, noise_var,
+                 kernel: int = MATERN52):
+        self.space = space
+        self.kernel = kernel
+        self.lengthscale = np.asarray(lengthscale, np.float64)
+        self.signal_var = float(signal_var)
+        self.noise_var = float(noise_var)
+        x = decode(space, x_obs_words)
+        self.u_obs, self.is_cat = gp_features(space, x)
+        self.y = np.asarray(y, np.float64)
+        self._factor()
+
+    def _factor(self):
+        n = len(self.y)
+        K = self.cov(self.u_obs, self.u_obs) + self.noise_var * np.eye(n)
+        self.chol = np.linalg.cholesky(K)            # K + tau^2 I = L L^T
+        self.alpha = sla.cho_solve((self.chol, True), self.y)  # (K + tau^2 I)^{-1} Y
+
+    def cov(self, ua, ub):
+        return matern(scaled_distance(ua, ub, self.is_cat, self.lengthscale),
+                      self.signal_var, self.kernel)
+
+    def add_observations(self, u_new, y_new):
+        """Condition again with extra (feature, value) pairs (plain refit)."""
+        self.u_obs = np.concatenate([self.u_obs, u_new], axis=0)
+        self.y = np.concatenate([self.y, np.asarray(y_new, np.float64)])
+        self._factor()
+
+    def posterior_u(self, u):
+        """mu = k(x, X)(K + tau^2 I)^{-1} Y and
+        sigma^2 = k(x, x) - k(x, X)(K + tau^2 I)^{-1} k(X, x), clamped at 0.
+
+        Reading: sigma^2 is the variance of the latent f (tau^2 appears only
+        inside the inverse, as printed)."""
+        kstar = self.cov(u, self.u_obs)                      # [N][n]
+        mu = kstar @ self.alpha
+        v = sla.solve_triangular(self.chol, kstar.T, lower=True)   # L v = k*
+        var = self.signal_var - np.sum(v * v, axis=0)
+        return mu, np.maximum(var, 0.0)
+
+    def posterior(self, words, n=None):
+        u, _ = gp_features(self.space, decode(self.space, words, n))
+        return self.posterior_u(u)
+
+    def mean_condition(self, words, n=None):
+        """sum_j |k(x, X_j) alpha_j|: the scale of the rounding error of any
+        evaluation of mu as a dot product (used by the tests' tolerance)."""
+        u, _ = gp_features(self.space, decode(self.space, words, n))
+        return np.abs(self.cov(u, self.u_obs)) @ np.abs(self.alpha)
+
+
+# --------------------------------------------------------------------------
+# 4a. expected improvement, Eq. (6)
+
+def norm_cdf(z):
+    return 0.5 * erfc(-np.asarray(z, np.float64) / math.sqrt(2.0))
+
+
+def norm_pdf(z):
+    z = np.asarray(z, np.float64)
+    return np.exp(-0.5 * z * z) / math.sqrt(2.0 * math.pi)
+
+
+def expected_improvement(mu, var, y_best: float, xi: float = 1e-4):
+    """EI(x) = E[max(0, f(x) + xi - f(x+))] for f(x) ~ N(mu, sigma^2).
+
+    Closed form: with a = mu - y+ + xi and z = a / sigma,
+    EI = a Phi(z) + sigma phi(z); EI = max(0, a) when sigma = 0.
+    Reading: xi enters with the sign printed in Eq. (6); xi = 1e-4 (Section 4.5).
+    """
+    mu = np.asarray(mu, np.float64)
+    sd = np.sqrt(np.maximum(np.asarray(var, np.float64), 0.0))
+    a = mu - y_best + xi
+    out = np.maximum(a, 0.0)
+    pos = sd > 0
+    z = np.where(pos, a / np.where(pos, sd, 1.0), 0.0)
+    return np.where(pos, a * norm_cdf(z) + sd * norm_pdf(z), out)
+
+
+# --------------------------------------------------------------------------
+# 4b. hypervolume (Section 4.4) and Monte-Carlo EHVI, Eq. (7)
+
+def pareto_front(Y: np.ndarray, ref: np.ndarray) -> np.ndarray:
+    """Non-dominated points of Y (rows, maximised) that strictly dominate r.
+
+    Points that do not lie strictly above r in every objective enclose no
+    volume with r, so they are left out (they add 0, cf. Eq. 8)."""
+    Y = np.asarray(Y, np.float64)
+    ref = np.asarray(ref, np.float64)
+    cand = [y for y in Y if np.all(y > ref)]
+    front = []
+    for i, y in enumerate(cand):
+        dominated = False
+        for j, z in enumerate(cand):
+            if j != i and np.all(z >= y) and (np.any(z > y) or j < i):
+                dominated = True   # a strictly better point, or an earlier duplicate
+                break
+        if not dominated:
+            front.append(y)
+    return np.array(front).reshape(-1, len(ref))
+
+
+def nondominated_cells(front: np.ndarray, ref: np.ndarray):
+    """The region {z >= r : no front point dominates z} as grid cells.
+
+    The grid's coordinates on axis j are r_j, every front coordinate, and
+    +inf.  Domination is constant inside a cell, so the region is exactly the
+    union of the cells whose upper corner no front point weakly dominates
+    (cells reaching +inf on some axis are never dominated).  Returns the
+    cells' lower and upper corners, each [C][M].
+    """
+    front = np.asarray(front, np.float64).reshape(-1, len(ref))
+    ref = np.asarray(ref, np.float64)
+    M = len(ref)
+    axes = []
+    for j in range(M):
+        c = np.unique(np.concatenate([[ref[j]], front[:, j]]))
+        axes.append(np.concatenate([c, [np.inf]]))
+    grids_lo = np.meshgrid(*[a[:-1] for a in axes], indexing="ij")
+    grids_hi = np.meshgrid(*[a[1:] for a in axes], indexing="ij")
+    lo = np.stack([g.ravel() for g in grids_lo], axis=1)
+    hi = np.stack([g.ravel() for g in grids_hi], axis=1)
+    if len(front):
+        dom = np.zeros(len(lo), dtype=bool)
+        for p in front:
+            dom |= np.all(p[None, :] >= hi, axis=1)
+        lo, hi = lo[~dom], hi[~dom]
+    return lo, hi
+
+
+def hypervolume(points: np.ndarray, ref: np.ndarray) -> float:
+    """HV(P): volume dominated by P and dominating r (Section 4.4), by
+    summing the grid cells whose upper corner some point dominates."""
+    P = pareto_front(points, ref)
+    if len(P) == 0:
+        return 0.0
+    ref = np.asarray(ref, np.float64)
+    M = len(ref)
+    axes = [np.unique(np.concatenate([[ref[j]], P[:, j]])) for j in range(M)]
+    lo = np.stack([g.ravel() for g in np.meshgrid(*[a[:-1] for a in axes], indexing="ij")], 1)
+    hi = np.stack([g.ravel() for g in np.meshgrid(*[a[1:] for a in axes], indexing="ij")], 1)
+    dom = np.zeros(len(lo), dtype=bool)
+    for p in P:
+        dom |= np.all(p[None, :] >= hi, axis=1)
+    return float(np.sum(np.prod(hi[dom] - lo[dom], axis=1)))
+
+
+def hvi_cells(y: np.ndarray, lo: np.ndarray, hi: np.ndarray) -> np.ndarray:
+    """HV(P u {y}) - HV(P) for rows y [K][M]: the volume of [r, y] that lies in
+    the non-dominated region, sum_c prod_j max(0, min(y_j, hi_cj) - lo_cj)."""
+    y = np.atleast_2d(np.asarray(y, np.float64))
+    ext = np.minimum(y[:, None, :], hi[None, :, :]) - lo[None, :, :]
+    return np.sum(np.prod(np.maximum(ext, 0.0), axis=2), axis=1)
+
+
+def ehvi_mc(mu: np.ndarray, var: np.ndarray, eps: np.ndarray, front, ref) -> np.ndarray:
+    """Monte-Carlo EHVI (Eq. 7) with common base samples.
+
+    Reading: the expectation of Eq. (7) over the independent per-objective
+    posteriors (Section 4.3: outputs modelled independently) is estimated with
+    fixed base samples eps[S][M]: y_s = mu + sigma * eps_s, EHVI = mean_s HVI(y_s).
+    mu, var: [N][M].
+    """
+    lo, hi = nondominated_cells(front, ref)
+    mu = np.asarray(mu, np.float64)
+    sd = np.sqrt(np.maximum(np.asarray(var, np.float64), 0.0))
+    eps = np.asarray(eps, np.float64)
+    out = np.empty(len(mu))
+    for i in range(len(mu)):
+        ys = mu[i][None, :] + sd[i][None, :] * eps
+        out[i] = np.mean(hvi_cells(ys, lo, hi))
+    return out
+
+
+# --------------------------------------------------------------------------
+# 5. top-q selection (Section 4.7)
+
+def select_topq(acq, mask, q: int):
+    """The q largest acquisition values among feasible candidates.
+
+    Reading: order is value descending, then index ascending (lowest index
+    wins a tie); candidates that are masked out, -inf or NaN are never
+    selected; fewer than q eligible candidates return them all (the
+    shortfall is filled by Sobol sampling outside this step, Section 4.6)."""
+    acq = np.asarray(acq, np.float64)
+    n = len(acq)
+    ok = np.isfinite(acq) | (acq == np.inf)
+    ok &= ~np.isnan(acq)
+    if mask is not None:
+        ok &= np.asarray(mask, bool)
+    idx = np.nonzero(ok)[0]
+    keys = sorted(idx.tolist(), key=lambda i: (-acq[i], i))
+    take = keys[:q]
+    return np.array(take, np.int64), acq[take], len(take)
+
+
+# --------------------------------------------------------------------------
+# whole round
+
+def score_round(inst, acq_kind: str, xi: float = 1e-4, kernel: int = MATERN52,
+                subset: np.ndarray | None = None):
+    """One suggestion round on an instance: masks, votes, posterior, acquisition.
+
+    ``subset`` restricts the GP/acquisition work to those candidate indices
+    (masks and votes are still computed for all of them)."""
+    w = inst.workload
+    n = inst.n_cand
+    words = inst.cand
+    mask_k = prune_mask(inst.space, inst.clauses, words, n)
+    votes = rf_votes(inst.nodes, inst.tree_offset, inst.space, words, n)
+    feas = mask_k & pof_feasible(votes, inst.n_trees, w.leaf_scale, w.delta_num, w.delta_den)
+    sel = np.arange(n) if subset is None else np.asarray(subset)
+    gps = [GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m],
+              inst.signal_var[m], inst.noise_var[m], kernel) for m in range(inst.n_obj)]
+    sub_words = words[:, sel]
+    mv = [gp.posterior(sub_words) for gp in gps]
+    mu = np.stack([m for m, _ in mv], axis=1)
+    var = np.stack([v for _, v in mv], axis=1)
+    if acq_kind == "ei":
+        a = expected_improvement(mu[:, 0], var[:, 0], float(np.max(inst.y_obs[0])), xi)
+    else:
+        front = pareto_front(inst.y_obs.T, inst.ref)
+        a = ehvi_mc(mu, var, inst.eps, front, inst.ref)
+    a = np.where(feas[sel], a, -np.inf)
+    return dict(mask_known=mask_k, votes=votes, feasible=feas, index=sel, mu=mu, var=var, acq=a)
+
+
+# --------------------------------------------------------------------------
+# 6. sequential picks with fantasies
+
+def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
+                  forced: list | None = None):
+    """q sequential EHVI picks with kriging-believer fantasies (refit form).
+
+    After each pick p the GP of every objective is conditioned again on the
+    observations plus (x_p, mu(x_p)) with noise tau^2, the front is rebuilt
+    with mu(x_p) added, and EHVI is recomputed over the pool with the picked
+    candidates excluded.  ``forced`` replays a given pick sequence (to follow
+    another implementation's choices step by step) instead of taking argmax.
+    Returns the picks and the acquisition array of each step.
+    """
+    n = inst.n_cand
+    words = inst.cand[:, :n]
+    gps = [GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m],
+              inst.signal_var[m], inst.noise_var[m], kernel) for m in range(inst.n_obj)]
+    u_pool, _ = gp_features(inst.space, decode(inst.space, words, n))
+    mu0 = np.stack([gp.posterior_u(u_pool)[0] for gp in gps], axis=1)
+    Yf = inst.y_obs.T.astype(np.float64)
+    picks, acqs, mus, vars_ = [], [], [], []
+    eligible = np.asarray(feasible, bool).copy()
+    for j in range(q):
+        var = np.stack([gp.posterior_u(u_pool)[1] for gp in gps], axis=1)
+        front = pareto_front(Yf, inst.ref)
+        a = ehvi_mc(mu0, var, inst.eps, front, inst.ref)
+        a = np.where(eligible, a, -np.inf)
+        if forced is not None:
+            p = int(forced[j])
+        else:
+            idx, _, cnt = select_topq(a, None, 1)
+            if cnt == 0:
+                break
+            p = int(idx[0])
+        picks.append(p)
+        acqs.append(a)
+        vars_.append(var)
+        mus.append(mu0)
+        eligible[p] = False
+        for m, gp in enumerate(gps):
+            gp.add_observations(u_pool[p:p + 1], [mu0[p, m]])
+        Yf = np.concatenate([Yf, mu0[p:p + 1]], axis=0)
+    return dict(picks=picks, acq=acqs, var=vars_, mu=mus)

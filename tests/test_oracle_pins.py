@@ -1,0 +1,505 @@
+"""Pins of the fp64 oracle against closed forms, invariants, brute force and
+library routines (no GPU).  Each group names the equation or passage of the
+paper it checks."""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy import integrate, special
+
+import oracle as O
+from workloads import (CATEGORICAL, CLAUSE_DTYPE, CONTINUOUS, INT_LOG, INT_UNIFORM, NODE_DTYPE,
+                       PARAM_DTYPE, Stream, make_instance, seeds, WORKLOADS)
+
+
+def _space(*params):
+    a = np.zeros(len(params), PARAM_DTYPE)
+    for i, p in enumerate(params):
+        a[i] = p
+    return a
+
+
+def _clause(guards=(), terms=(), rhs=0):
+    c = np.zeros(1, CLAUSE_DTYPE)
+    c[0]["n_guard"] = len(guards)
+    for g, (p, v) in enumerate(guards):
+        c[0]["guard_param"][g] = p
+        c[0]["guard_value"][g] = v
+    c[0]["n_term"] = len(terms)
+    for t, (p, k) in enumerate(terms):
+        c[0]["term_param"][t] = p
+        c[0]["coef"][t] = k
+    c[0]["rhs"] = rhs
+    return c
+
+
+def _words_int(cols):
+    return np.stack([np.asarray(c, np.int32).view(np.uint32) for c in cols])
+
+
+# ------------------------------------------------------------------ Eq. (2)
+
+@pytest.mark.parametrize("K", [1, 2, 7, 33])
+def test_prune_closed_form_counts(K):
+    """#{(a, b) in [1..K]^2 : a >= b} = K(K+1)/2; #{a + b >= K + 1} = K(K+1)/2."""
+    a, b = np.meshgrid(np.arange(1, K + 1), np.arange(1, K + 1), indexing="ij")
+    words = _words_int([a.ravel(), b.ravel()])
+    sp = _space((INT_UNIFORM, 0, 1, K), (INT_UNIFORM, 0, 1, K))
+    n = K * K
+    m = O.prune_mask(sp, _clause(terms=((0, 1), (1, -1)), rhs=0), words, n)
+    assert m.sum() == K * (K + 1) // 2
+    m = O.prune_mask(sp, _clause(terms=((0, 1), (1, 1)), rhs=K + 1), words, n)
+    assert m.sum() == K * (K + 1) // 2
+    # strict a > b via rhs 1: K(K-1)/2
+    m = O.prune_mask(sp, _clause(terms=((0, 1), (1, -1)), rhs=1), words, n)
+    assert m.sum() == K * (K - 1) // 2
+
+
+def test_prune_guards_and_degenerate_clauses():
+    K = 6
+    a, b, c = np.meshgrid(np.arange(1, K + 1), np.arange(1, K + 1), np.arange(3), indexing="ij")
+    words = _words_int([a.ravel(), b.ravel(), c.ravel()])
+    sp = _space((INT_UNIFORM, 0, 1, K), (INT_UNIFORM, 0, 1, K), (CATEGORICAL, 3, 0, 0))
+    n = words.shape[1]
+    # guard c == 1 => a >= b : the two other categories pass untouched
+    m = O.prune_mask(sp, _clause(guards=((2, 1),), terms=((0, 1), (1, -1))), words, n)
+    assert m.sum() == 2 * K * K + K * (K + 1) // 2
+    # a guard no candidate meets (category 5 of 3) leaves everything feasible
+    m = O.prune_mask(sp, _clause(guards=((2, 5),), terms=((0, 1),), rhs=10 ** 9), words, n)
+    assert m.all()
+    # two guards must both hold
+    m = O.prune_mask(sp, _clause(guards=((2, 0), (0, 1)), terms=((1, 1),), rhs=K + 1), words, n)
+    assert m.sum() == n - K
+    # empty sum: 0 >= 0 holds, 0 >= 1 fails everywhere
+    assert O.prune_mask(sp, _clause(rhs=0), words, n).all()
+    assert not O.prune_mask(sp, _clause(rhs=1), words, n).any()
+    # several clauses AND together
+    cl = np.concatenate([_clause(terms=((0, 1), (1, -1))), _clause(terms=((1, 1),), rhs=K)])
+    m = O.prune_mask(sp, cl, words, n)
+    assert m.sum() == 3 * 1  # only a = b = K survives, for each category
+
+
+def test_prune_exact_with_large_coefficients():
+    """Exact integer arithmetic: 2^40 a - 2^40 b - 1 >= 0 iff a > b (float64 would not tell)."""
+    vals = np.array([[2 ** 20, 2 ** 20], [2 ** 20 + 1, 2 ** 20], [5, 7]]).T
+    words = _words_int(vals)
+    sp = _space((INT_UNIFORM, 0, 1, 2 ** 21), (INT_UNIFORM, 0, 1, 2 ** 21))
+    m = O.prune_mask(sp, _clause(terms=((0, 2 ** 40), (1, -(2 ** 40))), rhs=1), words, 3)
+    assert m.tolist() == [False, True, False]
+
+
+def test_prune_fail_fraction_of_ten_parameter_space():
+    """The ten-parameter vLLM space loses about 40% of a uniform pool."""
+    inst = make_instance("d10-ei", seeds("d10-ei")[0], n_cand=1 << 16)
+    m = O.prune_mask(inst.space, inst.clauses, inst.cand, inst.n_cand)
+    assert abs((1.0 - m.mean()) - 0.40) <= 0.03
+
+
+# ------------------------------------------------------------------ Eq. (3)
+
+def _load_forest(path):
+    trees = {}
+    cases = []
+    for line in open(path):
+        f = line.split()
+        if not f or f[0].startswith("#"):
+            continue
+        if f[0] == "node":
+            t, i = int(f[1]), int(f[2])
+            if f[3] == "split":
+                trees.setdefault(t, {})[i] = (float(f[5]), int(f[6]), int(f[4]), 0)
+            else:
+                trees.setdefault(t, {})[i] = (float(f[4]), 0, 0, O.NODE_LEAF)
+        elif f[0] == "case":
+            cases.append((float(f[1]), float(f[2]), int(f[3])))
+    nodes, offs = [], [0]
+    for t in sorted(trees):
+        for i in sorted(trees[t]):
+            nodes.append(trees[t][i])
+        offs.append(len(nodes))
+    arr = np.zeros(len(nodes), NODE_DTYPE)
+    for j, nd in enumerate(nodes):
+        arr[j] = nd
+    return arr, np.array(offs, np.int32), cases
+
+
+def test_forest_hand_built(golden_dir):
+    nodes, offs, cases = _load_forest(os.path.join(golden_dir, "forest_hand.txt"))
+    sp = _space((CONTINUOUS, 0, 0, 100), (CONTINUOUS, 0, 0, 100))
+    x = np.array([[c[0], c[1]] for c in cases], np.float32)
+    words = np.ascontiguousarray(x.T).view(np.uint32)
+    want = [c[2] for c in cases]
+    assert O.rf_votes(nodes, offs, sp, words, len(cases)).tolist() == want
+    assert [O.rf_votes_one(nodes, offs, xi.astype(np.float64)) for xi in x] == want
+
+
+def test_forest_constant_leaves_and_tree_order():
+    rng = Stream(7, "forest-test")
+    inst = make_instance("tiny", 1001, n_cand=512)
+    # constant forest: every leaf votes c => votes = T c
+    nodes = inst.nodes.copy()
+    leaf = (nodes["flags"] & O.NODE_LEAF) != 0
+    nodes["val"][leaf] = 17
+    v = O.rf_votes(nodes, inst.tree_offset, inst.space, inst.cand, inst.n_cand)
+    assert (v == 17 * inst.n_trees).all()
+    # reversing the tree order does not change the votes
+    T = inst.n_trees
+    perm = np.array(rng.integers(0, 1000, T).argsort())
+    parts = [inst.nodes[inst.tree_offset[t]:inst.tree_offset[t + 1]] for t in perm]
+    offs = np.zeros(T + 1, np.int32)
+    offs[1:] = np.cumsum([len(p) for p in parts])
+    v1 = O.rf_votes(inst.nodes, inst.tree_offset, inst.space, inst.cand, inst.n_cand)
+    v2 = O.rf_votes(np.concatenate(parts), offs, inst.space, inst.cand, inst.n_cand)
+    assert (v1 == v2).all()
+    # the recursive walk agrees with the vectorised one
+    x = O.decode(inst.space, inst.cand, 64)
+    assert [O.rf_votes_one(inst.nodes, inst.tree_offset, xi) for xi in x] == v1[:64].tolist()
+
+
+def test_tree_grown_to_purity_reproduces_labels():
+    """A single CART tree without bootstrap, grown without a depth limit on
+    distinct points, sends every training point to a leaf of its own label."""
+    from workloads.generate import _grow, _layout
+    w = WORKLOADS["d8-ehvi2"]
+    st = Stream(11, "purity")
+    from workloads.generate import draw_configs, stored_values
+    X = stored_values(w, draw_configs(w, st, 64))
+    lab = (st.uniform(64) < 0.5).astype(np.float64)
+    tree = _layout(_grow(X, lab, 0, 64, 255))
+    offs = np.array([0, len(tree)], np.int32)
+    words = draw_configs(w, Stream(11, "purity"), 64)
+    sp = np.zeros(w.d, PARAM_DTYPE)
+    for i, p in enumerate(w.params):
+        sp[i] = (p.kind, p.n_choices, p.lo, p.hi)
+    v = O.rf_votes(tree, offs, sp, words, 64)
+    assert (v == 255 * lab).all()
+
+
+def test_pof_threshold_inclusive():
+    T, V = 100, 255
+    thr = 10 * V * T // 20  # Delta = 0.5 -> votes >= 12750
+    v = np.array([thr - 1, thr, thr + 1, 0, V * T])
+    assert O.pof_feasible(v, T, V, 10, 20).tolist() == [False, True, True, False, True]
+    # Delta = 0.25 and 0.75 (the bounds of Algorithm 1)
+    assert O.pof_feasible(np.array([V * T // 4]), T, V, 5, 20).tolist() == [True]
+    assert O.pof_feasible(np.array([3 * V * T // 4 - 1]), T, V, 15, 20).tolist() == [False]
+
+
+# ------------------------------------------------------------------ GP, Section 4.3
+
+@pytest.mark.parametrize("nu,kernel", [(2.5, O.MATERN52), (1.5, O.MATERN32)])
+def test_matern_matches_bessel_form(nu, kernel):
+    """k(r) = s 2^(1-nu)/Gamma(nu) (sqrt(2 nu) r)^nu K_nu(sqrt(2 nu) r)."""
+    r = np.linspace(1e-3, 8.0, 400)
+    z = math.sqrt(2 * nu) * r
+    ref = 1.7 * 2 ** (1 - nu) / special.gamma(nu) * z ** nu * special.kv(nu, z)
+    assert np.allclose(O.matern(r, 1.7, kernel), ref, rtol=1e-12, atol=1e-14)
+    assert O.matern(0.0, 1.7, kernel) == pytest.approx(1.7)
+    assert np.all(np.diff(O.matern(r, 1.0, kernel)) < 0)
+
+
+def test_features_and_distance():
+    sp = _space((INT_LOG, 0, 4, 4096), (INT_UNIFORM, 0, 2, 10), (CONTINUOUS, 0, 0.5, 1.0),
+                (CATEGORICAL, 3, 0, 0))
+    x = np.array([[4, 2, 0.5, 0], [4096, 10, 1.0, 2], [128, 6, 0.75, 1]], np.float64)
+    u, cat = O.gp_features(sp, x)
+    assert np.allclose(u[:, :3], [[0, 0, 0], [1, 1, 1], [0.5, 0.5, 0.5]])
+    assert cat.tolist() == [False, False, False, True]
+    ell = np.array([0.5, 1.0, 2.0, 0.25])
+    r = O.scaled_distance(u, u, cat, ell)
+    # rows 0 and 1: (1/0.5)^2 + 1 + (1/2)^2 + categorical 1/0.0625
+    assert r[0, 1] ** 2 == pytest.approx(4 + 1 + 0.25 + 16)
+    assert np.allclose(r, r.T) and np.allclose(np.diag(r), 0)
+
+
+def _toy_gp(n, seed=3, noise=1e-3, ell=0.4, d=3):
+    st = Stream(seed, "toy-gp")
+    sp = _space(*[(CONTINUOUS, 0, 0.0, 1.0)] * d)
+    X = st.uniform(n * d).reshape(d, n).astype(np.float32)
+    y = st.normal(n).astype(np.float32)
+    gp = O.GP(sp, X.view(np.uint32), y, np.full(d, ell), 1.0, noise)
+    return sp, X, y, gp
+
+
+def test_gp_single_observation_closed_form():
+    """n = 1: mu = k y / (s + tau^2), sigma^2 = s - k^2 / (s + tau^2)."""
+    sp, X, y, gp = _toy_gp(1, noise=0.3)
+    st = Stream(5, "cands")
+    C = st.uniform(3 * 50).reshape(3, 50).astype(np.float32)
+    mu, var = gp.posterior(C.view(np.uint32))
+    k = gp.cov(O.gp_features(sp, O.decode(sp, C.view(np.uint32)))[0], gp.u_obs)[:, 0]
+    assert np.allclose(mu, k * y[0] / 1.3, rtol=1e-12)
+    assert np.allclose(var, 1.0 - k * k / 1.3, rtol=1e-12)
+
+
+def test_gp_interpolates_as_noise_vanishes():
+    sp, X, y, gp = _toy_gp(12, noise=1e-10)
+    mu, var = gp.posterior(X.view(np.uint32))
+    assert np.allclose(mu, y, atol=1e-5)
+    assert np.all(var < 1e-6)
+
+
+def test_gp_far_field_and_bounds():
+    sp, X, y, gp = _toy_gp(20, ell=0.05)
+    st = Stream(9, "far")
+    C = st.uniform(3 * 200).reshape(3, 200).astype(np.float32)
+    far = (C + 5.0).astype(np.float32)  # 100 lengthscales from every observation
+    mu, var = gp.posterior(far.view(np.uint32))
+    assert np.all(np.abs(mu) < 1e-12) and np.allclose(var, 1.0, atol=1e-12)
+    sp, X, y, gp = _toy_gp(40, ell=0.3)
+    mu, var = gp.posterior(C.view(np.uint32))
+    assert np.all(var >= 0) and np.all(var <= 1.0 + 1e-12)
+
+
+def test_gp_permutation_invariant():
+    sp, X, y, gp = _toy_gp(25)
+    perm = np.array(Stream(2, "perm").integers(0, 10 ** 6, 25).argsort())
+    gp2 = O.GP(sp, np.ascontiguousarray(X[:, perm]).view(np.uint32), y[perm], np.full(3, 0.4), 1.0, 1e-3)
+    C = Stream(4, "c").uniform(300).reshape(3, 100).astype(np.float32).view(np.uint32)
+    m1, v1 = gp.posterior(C)
+    m2, v2 = gp2.posterior(C)
+    assert np.allclose(m1, m2, rtol=1e-10, atol=1e-12) and np.allclose(v1, v2, rtol=1e-10, atol=1e-12)
+
+
+def _gauss_jordan_inverse(A):
+    A = np.array(A, np.float64)
+    n = len(A)
+    M = np.concatenate([A, np.eye(n)], axis=1)
+    for c in range(n):
+        p = c + int(np.argmax(np.abs(M[c:, c])))
+        M[[c, p]] = M[[p, c]]
+        M[c] /= M[c, c]
+        for r in range(n):
+            if r != c:
+                M[r] -= M[r, c] * M[c]
+    return M[:, n:]
+
+
+@pytest.mark.parametrize("n", [2, 5, 8])
+def test_gp_matches_explicit_inverse(n):
+    """The Cholesky route equals the printed formulas with an explicit inverse."""
+    sp, X, y, gp = _toy_gp(n, noise=0.05)
+    C = Stream(8, "c").uniform(3 * 40).reshape(3, 40).astype(np.float32).view(np.uint32)
+    u, _ = O.gp_features(sp, O.decode(sp, C))
+    Kinv = _gauss_jordan_inverse(gp.cov(gp.u_obs, gp.u_obs) + 0.05 * np.eye(n))
+    ks = gp.cov(u, gp.u_obs)
+    mu_ref = ks @ Kinv @ y.astype(np.float64)
+    var_ref = 1.0 - np.einsum("ij,jk,ik->i", ks, Kinv, ks)
+    mu, var = gp.posterior(C)
+    assert np.allclose(mu, mu_ref, rtol=1e-10, atol=1e-12)
+    assert np.allclose(var, var_ref, rtol=1e-9, atol=1e-12)
+
+
+# ------------------------------------------------------------------ EI, Eq. (6)
+
+def test_ei_closed_form_matches_quadrature():
+    xi = 1e-4
+    for mu, sd, yb in [(0.0, 1.0, 0.0), (-1.3, 0.2, 0.5), (2.0, 0.5, 1.0), (0.3, 3.0, 2.0), (-4, 0.7, 0.0)]:
+        f = lambda t: max(0.0, mu + sd * t + xi - yb) * math.exp(-0.5 * t * t) / math.sqrt(2 * math.pi)
+        lo = (yb - xi - mu) / sd
+        q, _ = integrate.quad(f, max(lo, -12.0), 12.0, epsabs=1e-13, epsrel=1e-12, limit=200)
+        assert O.expected_improvement(mu, sd * sd, yb, xi) == pytest.approx(q, rel=1e-9, abs=1e-12)
+
+
+def test_ei_limits_and_monotonicity():
+    a = np.array([-1.0, 0.0, 0.5])
+    assert np.allclose(O.expected_improvement(a, 0.0, 0.0, 0.0), np.maximum(a, 0))
+    assert np.allclose(O.expected_improvement(a, 1e-24, 0.0, 0.0), np.maximum(a, 0), atol=1e-11)
+    mus = np.linspace(-3, 3, 50)
+    assert np.all(np.diff(O.expected_improvement(mus, 0.25, 0.0)) > 0)
+    sds = np.linspace(0.01, 3, 50)
+    assert np.all(np.diff(O.expected_improvement(0.2, sds ** 2, 0.5)) > 0)
+
+
+# ------------------------------------------------------------------ HV, EHVI, Eq. (7), Eq. (8)
+
+def _hv2d_rectangles(points, ref):
+    """Section 4.4: sum of rectangles between the sorted front and r."""
+    P = [p for p in points if p[0] > ref[0] and p[1] > ref[1]]
+    P.sort(key=lambda p: -p[0])
+    hv, top = 0.0, ref[1]
+    for x, y in P:
+        if y > top:
+            hv += (x - ref[0]) * (y - top)
+            top = y
+    return hv
+
+
+def _hv_lattice(points, ref, top):
+    """Brute force on integers: count unit cells [z, z+1) dominated by some point."""
+    M = len(ref)
+    count = 0
+    for z in itertools.product(*[range(ref[j], top) for j in range(M)]):
+        if any(all(p[j] >= z[j] + 1 for j in range(M)) for p in points):
+            count += 1
+    return count
+
+
+def test_hv_worked_example(golden_dir):
+    pts, hvis = [], []
+    for line in open(os.path.join(golden_dir, "hv_2d_worked.txt")):
+        f = line.split()
+        if not f or f[0].startswith("#"):
+            continue
+        if f[0] == "ref":
+            ref = np.array([float(f[1]), float(f[2])])
+        elif f[0] == "point":
+            pts.append([float(f[1]), float(f[2])])
+        elif f[0] == "hv":
+            hv = float(f[1])
+        elif f[0] == "hvi":
+            hvis.append(([float(f[1]), float(f[2])], float(f[3])))
+    pts = np.array(pts)
+    assert O.hypervolume(pts, ref) == pytest.approx(hv)
+    front = O.pareto_front(pts, ref)
+    assert len(front) == 3
+    lo, hi = O.nondominated_cells(front, ref)
+    for y, want in hvis:
+        assert O.hvi_cells(np.array([y]), lo, hi)[0] == pytest.approx(want)
+
+
+def test_single_point_hv_eq8(golden_dir):
+    for line in open(os.path.join(golden_dir, "hv_single_point.txt")):
+        f = line.split()
+        if not f or f[0].startswith("#"):
+            continue
+        y1, y2, r1, r2, want = map(float, f)
+        assert O.hypervolume(np.array([[y1, y2]]), np.array([r1, r2])) == pytest.approx(want)
+
+
+@pytest.mark.parametrize("M,top,npts", [(2, 12, 9), (3, 7, 8)])
+def test_hv_lattice_brute_force(M, top, npts):
+    st = Stream(M, "lattice")
+    for trial in range(4):
+        pts = st.integers(1, top, npts * M).reshape(npts, M)
+        ref = np.zeros(M, np.int64)
+        want = _hv_lattice(pts.tolist(), ref.tolist(), top)
+        assert O.hypervolume(pts.astype(float), ref.astype(float)) == pytest.approx(want)
+        if M == 2:
+            assert _hv2d_rectangles(pts.astype(float).tolist(), [0.0, 0.0]) == pytest.approx(want)
+
+
+@pytest.mark.parametrize("M", [2, 3])
+def test_hvi_by_cells_equals_hv_difference(M):
+    st = Stream(40 + M, "hvi")
+    ref = np.zeros(M)
+    pts = st.uniform(10 * M).reshape(10, M) * 4.0
+    front = O.pareto_front(pts, ref)
+    base = O.hypervolume(front, ref)
+    lo, hi = O.nondominated_cells(front, ref)
+    ys = st.uniform(60 * M).reshape(60, M) * 5.0 - 0.5
+    got = O.hvi_cells(ys, lo, hi)
+    want = [O.hypervolume(np.vstack([front, y]), ref) - base for y in ys]
+    assert np.allclose(got, want, rtol=1e-12, atol=1e-12)
+    # permuting the points leaves HV unchanged
+    perm = np.array(st.integers(0, 10 ** 6, len(pts)).argsort())
+    assert O.hypervolume(pts[perm], ref) == pytest.approx(O.hypervolume(pts, ref), rel=1e-14)
+    # a dominated point improves nothing
+    assert O.hvi_cells(front[:1] * 0.999, lo, hi)[0] == pytest.approx(0.0, abs=1e-14)
+    # cells clipped to a bounding box plus HV fill the box
+    box = np.full(M, 6.0)
+    clipped = np.prod(np.maximum(np.minimum(hi, box) - lo, 0), axis=1).sum()
+    assert clipped + base == pytest.approx(np.prod(box - ref), rel=1e-12)
+
+
+def test_empty_front_single_cell():
+    ref = np.array([0.5, -1.0])
+    lo, hi = O.nondominated_cells(np.zeros((0, 2)), ref)
+    assert len(lo) == 1
+    y = np.array([[1.5, 2.0], [0.0, 3.0]])
+    assert np.allclose(O.hvi_cells(y, lo, hi), [3.0, 0.0])
+
+
+def _ehvi_analytic(mu, sd, lo, hi):
+    """Independent Gaussians: E prod_j clip_j = prod_j E clip_j per cell, with
+    E[max(0, min(Y, u) - l)] = int_l^u P(Y > t) dt in closed form."""
+    def g(t, m, s):  # int_{-inf}^{t} Phi((x - m)/s) dx
+        z = (t - m) / s
+        return s * (z * O.norm_cdf(z) + O.norm_pdf(z))
+    tot = 0.0
+    for l, u in zip(lo, hi):
+        prod = 1.0
+        for j in range(len(mu)):
+            inner = (u[j] - l[j]) if np.isfinite(u[j]) else None
+            # int_l^u (1 - Phi) = (u - l) - [G(u) - G(l)], G = int Phi
+            if np.isfinite(u[j]):
+                val = (u[j] - l[j]) - (g(u[j], mu[j], sd[j]) - g(l[j], mu[j], sd[j]))
+            else:
+                # int_l^inf (1 - Phi((t-m)/s)) dt = s psi((m - l)/s)
+                z = (mu[j] - l[j]) / sd[j]
+                val = sd[j] * (z * O.norm_cdf(z) + O.norm_pdf(z))
+            prod *= val
+        tot += prod
+    return tot
+
+
+@pytest.mark.parametrize("M", [2, 3])
+def test_mc_ehvi_converges_to_analytic(M):
+    st = Stream(60 + M, "ehvi-conv")
+    ref = np.zeros(M)
+    front = O.pareto_front(st.uniform(8 * M).reshape(8, M) * 2.0, ref)
+    lo, hi = O.nondominated_cells(front, ref)
+    mu = np.full(M, 1.2)
+    sd = np.array([0.5, 0.8, 0.3][:M])
+    S = 40000
+    eps = st.normal(S * M).reshape(S, M)
+    vals = O.hvi_cells(mu + sd * eps, lo, hi)
+    est = vals.mean()
+    se = vals.std() / math.sqrt(S)
+    assert abs(est - _ehvi_analytic(mu, sd, lo, hi)) < 4 * se
+    # the oracle's MC EHVI is that mean
+    e = O.ehvi_mc(mu[None, :], (sd ** 2)[None, :], eps, front, ref)[0]
+    assert e == pytest.approx(est, rel=1e-12)
+
+
+# ------------------------------------------------------------------ top-q, Section 4.7
+
+def test_topq_against_repeated_argmax():
+    st = Stream(77, "topq")
+    for trial in range(20):
+        n = int(st.integers(1, 300, 1)[0])
+        acq = np.round(st.normal(n), 1)  # many ties
+        acq[st.uniform(n) < 0.1] = -np.inf
+        acq[st.uniform(n) < 0.05] = np.nan
+        mask = st.uniform(n) < 0.8
+        q = int(st.integers(1, 40, 1)[0])
+        idx, val, cnt = O.select_topq(acq, mask, q)
+        # brute force: q rounds of "largest value, lowest index" over the eligible set
+        alive = [i for i in range(n) if mask[i] and not np.isnan(acq[i]) and acq[i] > -np.inf]
+        want = []
+        for _ in range(q):
+            if not alive:
+                break
+            best = alive[0]
+            for i in alive:
+                if acq[i] > acq[best]:
+                    best = i
+            want.append(best)
+            alive.remove(best)
+        assert idx.tolist() == want and cnt == len(want)
+
+
+# ------------------------------------------------------------------ fantasies (refit form)
+
+def test_fantasy_refit_properties():
+    """Kriging believer: conditioning on y_p = mu(x_p) leaves mu unchanged;
+    sigma^2(x_p) becomes s t / (s + t) (s = sigma^2(x_p), t = tau^2); the
+    refit variance equals the rank-1 downdate sigma^2 - c(x)^2 with
+    c(x) = k_post(x, x_p) / sqrt(s + t)."""
+    sp, X, y, gp = _toy_gp(30, noise=2e-3)
+    C = Stream(12, "c").uniform(3 * 300).reshape(3, 300).astype(np.float32).view(np.uint32)
+    u, _ = O.gp_features(sp, O.decode(sp, C))
+    mu0, var0 = gp.posterior_u(u)
+    p = 17
+    kstar = gp.cov(u, gp.u_obs)
+    Kn = gp.cov(gp.u_obs, gp.u_obs) + 2e-3 * np.eye(30)
+    kpost = gp.cov(u, u[p:p + 1])[:, 0] - kstar @ np.linalg.solve(Kn, kstar[p])
+    c = kpost / math.sqrt(var0[p] + 2e-3)
+    gp.add_observations(u[p:p + 1], [mu0[p]])
+    mu1, var1 = gp.posterior_u(u)
+    assert np.allclose(mu1, mu0, rtol=1e-9, atol=1e-11)
+    s, t = var0[p], 2e-3
+    assert var1[p] == pytest.approx(s * t / (s + t), rel=1e-8)
+    assert np.allclose(var1, np.maximum(var0 - c * c, 0), rtol=1e-8, atol=1e-11)
