@@ -1,0 +1,287 @@
+/*
+ * scoot.h - C ABI of the GB300 candidate-scoring path of SCOOT
+ * (SLO-oriented tuning of LLM inference engines by Bayesian optimisation).
+ *
+ * One suggestion round scores a pool of N candidate engine configurations:
+ *
+ *   scoot_prune          known constraints, Eq. (2)
+ *   scoot_rf_predict     random-forest probability of feasibility, Eq. (3)
+ *   scoot_gp_posterior   GP posterior mean and variance (Section 4.3)
+ *   scoot_acq_ei         expected improvement, Eq. (6)
+ *   scoot_acq_ehvi       Monte-Carlo expected hypervolume improvement, Eq. (7)
+ *   scoot_score_ei       posterior + EI in one kernel
+ *   scoot_score_ehvi     posterior + EHVI in one kernel
+ *   scoot_select_topq    top-q for parallel suggestion (Section 4.7)
+ *
+ * plus host-side preparation of per-round state (Cholesky factor of the
+ * observations' covariance, box decomposition of the non-dominated region,
+ * forest packing).
+ *
+ * Conventions
+ *  - Every call returns a scoot_status: SCOOT_OK (0) or a negative error.
+ *    No call aborts, throws across the ABI or traps on the device.  After an
+ *    error, scoot_last_error(ctx) returns a message owned by the context.
+ *  - Pointers named h_* are host memory; every other array pointer is device
+ *    memory of the context's device.  All arrays are owned by the caller;
+ *    the library owns only the workspace inside a scoot_ctx.
+ *  - Device calls are asynchronous on the given stream (a cudaStream_t passed
+ *    as void*; NULL is the legacy default stream).  Host-side calls
+ *    (*_layout_init, *_prepare, *_build, *_pack) are synchronous and touch
+ *    no device.
+ *  - Candidates are stored structure-of-arrays: column p of a pool of n
+ *    candidates with leading dimension ld is cand[p * ld + i], one 32-bit
+ *    word per parameter: integer and categorical parameters as int32,
+ *    continuous ones as float32 bit patterns.  cand must be 16-byte aligned
+ *    and ld a multiple of 4 with ld >= n.
+ *  - Objectives are maximised (Eq. 1 with the lambda signs applied).
+ *  - A context is used by one host thread at a time.  Calls on one context
+ *    that overlap on the GPU share its workspace: order them on one stream.
+ */
+#ifndef SCOOT_H
+#define SCOOT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t scoot_status;
+#define SCOOT_OK            0
+#define SCOOT_EINVAL       -1   /* bad argument: null, size, alignment, NaN, malformed input */
+#define SCOOT_ENOMEM       -2   /* workspace allocation failed */
+#define SCOOT_ECUDA        -3   /* a CUDA runtime call failed */
+#define SCOOT_EDEVICE      -4   /* a kernel flagged a bad index or value at run time */
+#define SCOOT_ETIMEOUT     -5   /* a bounded device-side wait gave up */
+#define SCOOT_EUNSUPPORTED -6   /* size or option beyond what this build handles */
+
+/* Parameter kinds of the mixed search space (Section 3, Table 1). */
+#define SCOOT_INT_UNIFORM 0
+#define SCOOT_INT_LOG     1
+#define SCOOT_CATEGORICAL 2   /* booleans are categoricals of two */
+#define SCOOT_CONTINUOUS  3
+
+/* Covariance functions (Section 4.3 names Matern-3/2; Matern-5/2 ARD is the default). */
+#define SCOOT_MATERN52 0
+#define SCOOT_MATERN32 1
+
+#define SCOOT_MAX_DIM      16   /* parameters per configuration */
+#define SCOOT_MAX_CLAUSES  16   /* known-constraint clauses per call */
+#define SCOOT_MAX_OBJ       4   /* objectives */
+#define SCOOT_MAX_OBS    1024   /* observed configurations */
+#define SCOOT_MAX_Q        64   /* picks per top-q call */
+
+/* One parameter: kind, number of categories (categorical only) and the
+ * range [lo, hi] (integer and continuous kinds).  16 bytes. */
+typedef struct {
+    int32_t kind;
+    int32_t n_choices;
+    float lo;
+    float hi;
+} scoot_param;
+
+/* One known constraint (Eq. 2): if x[guard_param[g]] == guard_value[g] for
+ * every g < n_guard, then sum_{t < n_term} coef[t] * x[term_param[t]] >= rhs
+ * must hold, evaluated exactly in 64-bit integers.  Only integer and
+ * categorical parameters may appear.  80 bytes. */
+typedef struct {
+    int32_t n_guard;
+    int32_t guard_param[2];
+    int32_t guard_value[2];
+    int32_t n_term;
+    int32_t term_param[4];
+    int64_t coef[4];
+    int64_t rhs;
+} scoot_clause;
+
+/* One regression-tree node, 8 bytes.  A split node (flags & 1 == 0) sends a
+ * configuration to node `left` when x[feat] <= val and to node left + 1
+ * otherwise; child indices count from the tree's first node.  A leaf
+ * (flags & 1) carries an integer vote count in val, 0 <= val <= leaf_scale.
+ * x[feat] is the stored value as a float (integers and category indices
+ * converted exactly, continuous values as stored). */
+typedef struct {
+    float val;
+    uint16_t left;
+    uint8_t feat;
+    uint8_t flags;
+} scoot_node;
+
+typedef struct scoot_ctx scoot_ctx;
+
+/* ------------------------------------------------------------------ context */
+
+/* Create a context on CUDA device `device` (made current for every call on
+ * the context).  *out receives the handle; on error *out is NULL. */
+scoot_status scoot_ctx_create(int32_t device, scoot_ctx** out);
+scoot_status scoot_ctx_destroy(scoot_ctx* ctx);
+/* Message of the last error on ctx ("" if none).  Owned by ctx. */
+const char* scoot_last_error(const scoot_ctx* ctx);
+const char* scoot_status_string(scoot_status s);
+/* Wait for `stream`, then read and clear the context's device error word:
+ * SCOOT_EDEVICE if a kernel flagged a bad index or value since the last
+ * check, SCOOT_ETIMEOUT if a bounded wait gave up, else SCOOT_OK. */
+scoot_status scoot_ctx_check(scoot_ctx* ctx, void* stream);
+/* Bytes of device workspace the context currently holds. */
+scoot_status scoot_ctx_workspace_bytes(const scoot_ctx* ctx, int64_t* bytes);
+
+/* ------------------------------------------------------------------ 1. prune, Eq. (2) */
+
+/* mask[i] = 1 when candidate i satisfies every clause of h_clauses, else 0
+ * (the solution space pruned by known constraints, Section 4.5).  Only the
+ * columns named by some clause are read.  If n_feasible is not NULL it is a
+ * device int64 that receives the number of feasible candidates (overwritten,
+ * not accumulated).  n == 0 is valid and writes nothing but the count. */
+scoot_status scoot_prune(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
+                         const scoot_clause* h_clauses, int32_t n_clauses,
+                         const uint32_t* cand, int64_t n, int64_t ld,
+                         uint8_t* mask, int64_t* n_feasible, void* stream);
+
+/* ------------------------------------------------------------------ 2. random forest, Eq. (3) */
+
+/* Packed forest: a device blob built by scoot_forest_pack. */
+typedef struct {
+    int32_t n_trees;
+    int32_t n_nodes;          /* total nodes */
+    int32_t d;                /* features */
+    int32_t leaf_scale;       /* V: leaves hold votes in [0, V] */
+    int32_t max_depth;        /* longest root-to-leaf path (edges) */
+    int32_t n_chunks;         /* groups of whole trees staged in shared memory one at a time */
+    int32_t max_chunk_nodes;  /* nodes of the largest group */
+    int32_t reserved;
+    int64_t bytes;            /* blob size */
+    int64_t off_chunks;       /* int32[n_chunks][4]: first tree, tree count, first node, node count */
+    int64_t off_roots;        /* int32[n_trees]: first node of each tree */
+    int64_t off_nodes;        /* scoot_node[n_nodes] */
+} scoot_forest_layout;
+
+/* Validate a forest given as nodes plus tree offsets (tree t owns nodes
+ * h_tree_offset[t] .. h_tree_offset[t+1]-1) and plan its blob.  Rejects
+ * child indices outside the tree or not after their parent (so no cycles),
+ * features >= d, and leaf votes that are not integers in [0, leaf_scale]. */
+scoot_status scoot_forest_layout_init(const scoot_node* h_nodes, const int32_t* h_tree_offset,
+                                      int32_t n_trees, int32_t d, int32_t leaf_scale,
+                                      scoot_forest_layout* out);
+/* Write the blob (layout->bytes bytes) into h_blob; copy it to the device as is. */
+scoot_status scoot_forest_pack(const scoot_forest_layout* layout, const scoot_node* h_nodes,
+                               const int32_t* h_tree_offset, void* h_blob);
+
+/* votes[i] = sum over trees of the leaf votes reached by candidate i, for
+ * every candidate with mask[i] == 1 on entry; then mask[i] &= (delta_den *
+ * votes[i] >= delta_num * leaf_scale * n_trees), i.e. POF(x) >= Delta with
+ * POF = votes / (leaf_scale * T) and Delta = delta_num / delta_den (Eq. 3).
+ * Candidates with mask[i] == 0 on entry are not walked: votes[i] = 0.
+ * mask may be NULL (every candidate walked, no mask written).  n_feasible,
+ * if not NULL, is a device int64 receiving the count of mask == 1 after. */
+scoot_status scoot_rf_predict(scoot_ctx* ctx, const scoot_forest_layout* layout,
+                              const void* forest, const scoot_param* h_space,
+                              const uint32_t* cand, int64_t n, int64_t ld,
+                              uint32_t delta_num, uint32_t delta_den,
+                              uint32_t* votes, uint8_t* mask, int64_t* n_feasible,
+                              void* stream);
+
+/* ------------------------------------------------------------------ 3. GP posterior (Section 4.3) */
+
+/* Per-round GP state for M objectives over n observations: a device blob
+ * built on the host by scoot_gp_prepare (fp64 Cholesky of K + tau^2 I, then
+ * alpha = (K + tau^2 I)^{-1} Y and L^{-1}, stored in fp32). */
+typedef struct {
+    int32_t n, d, n_obj, kernel;
+    int32_t n_rb;             /* row blocks of 64 in the tiled L^{-1} */
+    int32_t n_tiles;          /* 32 x 64 tiles of L^{-1} per objective */
+    int64_t bytes;
+    int64_t off_fmap;         /* float[d][4]: kind, a, b, 0 of the feature map */
+    int64_t off_xs;           /* float[M][n][d]: observed features scaled by 1/lengthscale */
+    int64_t off_ils;          /* float[M][d]: 1/l (ordinal dims) or 1/l^2 (categorical dims) */
+    int64_t off_alpha;        /* float[M][n] */
+    int64_t off_linv;         /* float[M][n_tiles][32][64]: L^{-1} tiles, transposed, zero-filled */
+    int64_t off_scal;         /* float[M][4]: signal variance, noise variance, best observed y, 0 */
+} scoot_gp_layout;
+
+/* Plan the blob for n observations, d parameters, M objectives and a kernel. */
+scoot_status scoot_gp_layout_init(int32_t n, int32_t d, int32_t n_obj, int32_t kernel,
+                                  scoot_gp_layout* out);
+/* Build the blob on the host.  h_x_obs: observed configurations, SoA words
+ * [d][ld_obs]; h_y: standardised observed values [M][n]; h_lengthscale
+ * [M][d] (> 0); h_signal_var, h_noise_var [M] (> 0 and >= 0).  Features
+ * (the covariance's input coordinates): integer log-uniform parameters
+ * (ln v - ln lo)/(ln hi - ln lo); integer uniform and continuous ones
+ * (v - lo)/(hi - lo); categoricals compared for equality, adding
+ * [c != c']/l^2 to r^2.  Fails with SCOOT_EINVAL if K + tau^2 I is not
+ * numerically positive definite.  If h_cond is not NULL it receives, per
+ * objective, the ratio of the largest to the smallest pivot squared of the
+ * Cholesky factor (a cheap conditioning indicator). */
+scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
+                              const float* h_y, const float* h_lengthscale,
+                              const float* h_signal_var, const float* h_noise_var,
+                              const scoot_gp_layout* layout, void* h_blob, double* h_cond);
+
+/* mean[m * ldo + i], var[m * ldo + i] for every candidate i < n and
+ * objective m:  mu = k(x, X)(K + tau^2 I)^{-1} Y and
+ * sigma^2 = k(x, x) - k(x, X)(K + tau^2 I)^{-1} k(X, x) (latent f, clamped
+ * at 0).  If mask is not NULL, candidates with mask[i] == 0 are skipped and
+ * their outputs left untouched.  ldo >= n. */
+scoot_status scoot_gp_posterior(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                                const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                                float* mean, float* var, int64_t ldo, void* stream);
+
+/* ------------------------------------------------------------------ 4. acquisition */
+
+/* EI(x) = E[max(0, f(x) + xi - y_best)] in closed form, Eq. (6):
+ * a = mu - y_best + xi, z = a / sigma, EI = a Phi(z) + sigma phi(z);
+ * EI = max(0, a) when sigma == 0.  acq[i] = -inf where mask[i] == 0
+ * (mask may be NULL). */
+scoot_status scoot_acq_ei(scoot_ctx* ctx, const float* mean, const float* var,
+                          const uint8_t* mask, int64_t n, float y_best, float xi,
+                          float* acq, void* stream);
+
+/* Box decomposition of the region above h_ref that the Pareto front of the
+ * points h_y ([M][n_pts], maximised) does not dominate.  Only points that
+ * strictly dominate h_ref take part (others enclose no volume, Eq. 8).
+ * Boxes are written row-major: h_lo[b * M + j], h_hi[b * M + j] (+inf where
+ * unbounded); *n_boxes receives the count, *front_size the front's size.
+ * cap is the capacity of h_lo / h_hi in boxes (SCOOT_EUNSUPPORTED if too
+ * small; *n_boxes then holds the count needed).  2 <= M <= SCOOT_MAX_OBJ. */
+scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, const float* h_ref,
+                               int32_t cap, float* h_lo, float* h_hi, int32_t* n_boxes,
+                               int32_t* front_size);
+
+/* Monte-Carlo EHVI, Eq. (7): with base samples eps [S][M] shared by every
+ * candidate, y_s = mu + sigma * eps_s and
+ * EHVI = (1/S) sum_s sum_b prod_j max(0, min(y_sj, hi_bj) - lo_bj)
+ * over the n_boxes boxes (lo, hi: device, [B][M]).  mean/var as written by
+ * scoot_gp_posterior ([M][ldm]).  acq[i] = -inf where mask[i] == 0. */
+scoot_status scoot_acq_ehvi(scoot_ctx* ctx, const float* mean, const float* var, int64_t ldm,
+                            int32_t n_obj, const uint8_t* mask, int64_t n,
+                            const float* box_lo, const float* box_hi, int32_t n_boxes,
+                            const float* eps, int32_t n_mc, float* acq, void* stream);
+
+/* scoot_gp_posterior followed by scoot_acq_ei, in one kernel, without
+ * writing mean or variance (objective 0; y_best is the state's best
+ * observed value of objective 0). */
+scoot_status scoot_score_ei(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                            const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                            float xi, float* acq, void* stream);
+
+/* scoot_gp_posterior followed by scoot_acq_ehvi, in one kernel. */
+scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                              const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                              const float* box_lo, const float* box_hi, int32_t n_boxes,
+                              const float* eps, int32_t n_mc, float* acq, void* stream);
+
+/* ------------------------------------------------------------------ 5. top-q (Section 4.7) */
+
+/* The min(q, eligible) candidates with the largest acq, eligible meaning
+ * mask[i] == 1 (mask may be NULL) and acq[i] neither NaN nor -inf.  Order:
+ * value descending, then index ascending (the lowest index wins a tie).
+ * idx (int64 [q]), val (float [q]) and count (int32 [1]) are device
+ * outputs; entries beyond count are set to -1 / -inf.  1 <= q <= SCOOT_MAX_Q. */
+scoot_status scoot_select_topq(scoot_ctx* ctx, const float* acq, const uint8_t* mask, int64_t n,
+                               int32_t q, int64_t* idx, float* val, int32_t* count, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SCOOT_H */

@@ -75,11 +75,20 @@ def prune_mask(space, clauses, words: np.ndarray, n: int) -> np.ndarray:
         for g in range(int(c["n_guard"])):
             p = int(c["guard_param"][g])
             guard &= x[:, p].astype(np.int64) == int(c["guard_value"][g])
-        lhs = np.zeros(n, dtype=object)
-        for t in range(int(c["n_term"])):
-            p = int(c["term_param"][t])
-            lhs = lhs + int(c["coef"][t]) * x[:, p].astype(np.int64).astype(object)
-        holds = np.array([int(v) >= int(c["rhs"]) for v in lhs], dtype=bool) if n else np.zeros(0, bool)
+        nt = int(c["n_term"])
+        coefs = [int(c["coef"][t]) for t in range(nt)]
+        if all(abs(k) < 2 ** 29 for k in coefs) and abs(int(c["rhs"])) < 2 ** 62:
+            # every term is below 2^60 in magnitude (values are 32-bit), so
+            # the int64 sum of at most four terms is exact
+            lhs = np.zeros(n, dtype=np.int64)
+            for t in range(nt):
+                lhs += coefs[t] * x[:, int(c["term_param"][t])].astype(np.int64)
+            holds = lhs >= int(c["rhs"])
+        else:
+            lhs = np.zeros(n, dtype=object)
+            for t in range(nt):
+                lhs = lhs + coefs[t] * x[:, int(c["term_param"][t])].astype(np.int64).astype(object)
+            holds = np.array([int(v) >= int(c["rhs"]) for v in lhs], dtype=bool) if n else np.zeros(0, bool)
         mask &= (~guard) | holds
     return mask
 
@@ -123,16 +132,16 @@ def rf_votes(nodes, tree_offset, space, words, n: int) -> np.ndarray:
         size = int(tree_offset[t + 1]) - base
         tree = nodes[base:base + size]
         idx = np.zeros(n, dtype=np.int64)
+        active = np.arange(n)          # candidates not yet at a leaf
         for _ in range(size + 1):
-            leaf = (tree["flags"][idx] & NODE_LEAF) != 0
-            if leaf.all():
+            node = idx[active]
+            leaf = (tree["flags"][node] & NODE_LEAF) != 0
+            active, node = active[~leaf], node[~leaf]
+            if len(active) == 0:
                 break
-            feat = tree["feat"][idx].astype(np.int64)
-            thr = tree["val"][idx].astype(np.float64)
-            left = tree["left"][idx].astype(np.int64)
-            xv = x[np.arange(n), feat]
-            nxt = np.where(xv <= thr, left, left + 1)
-            idx = np.where(leaf, idx, nxt)
+            xv = x[active, tree["feat"][node].astype(np.int64)]
+            left = tree["left"][node].astype(np.int64)
+            idx[active] = np.where(xv <= tree["val"][node].astype(np.float64), left, left + 1)
         votes += tree["val"][idx].astype(np.float64).astype(np.int64)
     return votes
 

@@ -1,0 +1,453 @@
+// Host-side, synchronous preparation of per-round state (no device work):
+//  - the GP state blob: fp64 Cholesky factor of K + tau^2 I, alpha and
+//    L^{-1} (Section 4.3), cast to fp32 in the tiled layout the kernels read;
+//  - the box decomposition of the region the Pareto front does not dominate
+//    (Section 4.4, used by the Monte-Carlo EHVI of Eq. 7);
+//  - validation and packing of the random forest of Eq. (3).
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <limits>
+#include <vector>
+
+#include "internal.h"
+
+namespace {
+
+constexpr int64_t kAlign = 256;
+constexpr int kRowBlock = 64;   // rows of L^{-1} per tile
+constexpr int kColChunk = 32;   // columns of L^{-1} per tile
+constexpr int kForestChunkNodes = 12288;  // 96 KiB of nodes staged at a time
+
+int64_t align_up(int64_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+bool is_finite(double x) { return std::isfinite(x); }
+
+double stored_value(const scoot_param& p, uint32_t w) {
+    if (p.kind == SCOOT_CONTINUOUS) {
+        float f;
+        std::memcpy(&f, &w, 4);
+        return (double)f;
+    }
+    return (double)(int32_t)w;
+}
+
+// Feature coordinate of a stored value (categoricals keep their index).
+double feature(const scoot_param& p, double v) {
+    switch (p.kind) {
+    case SCOOT_INT_LOG:
+        return (std::log(v) - std::log((double)p.lo)) / (std::log((double)p.hi) - std::log((double)p.lo));
+    case SCOOT_INT_UNIFORM:
+    case SCOOT_CONTINUOUS:
+        return p.hi > p.lo ? (v - (double)p.lo) / ((double)p.hi - (double)p.lo) : 0.0;
+    default:
+        return v;
+    }
+}
+
+double matern(double r, int kernel) {
+    if (kernel == SCOOT_MATERN32) {
+        double a = std::sqrt(3.0) * r;
+        return (1.0 + a) * std::exp(-a);
+    }
+    double a = std::sqrt(5.0) * r;
+    return (1.0 + a + a * a / 3.0) * std::exp(-a);
+}
+
+bool valid_space(const scoot_param* sp, int32_t d) {
+    for (int c = 0; c < d; ++c) {
+        const scoot_param& p = sp[c];
+        if (p.kind == SCOOT_CATEGORICAL) {
+            if (p.n_choices < 1) return false;
+        } else if (p.kind == SCOOT_INT_LOG) {
+            if (!(p.lo > 0.0f) || !(p.hi > p.lo)) return false;
+        } else if (p.kind == SCOOT_INT_UNIFORM || p.kind == SCOOT_CONTINUOUS) {
+            if (!is_finite(p.lo) || !is_finite(p.hi) || p.hi < p.lo) return false;
+        } else {
+            return false;
+        }
+    }
+    return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* scoot_status_string(scoot_status s) {
+    switch (s) {
+    case SCOOT_OK: return "ok";
+    case SCOOT_EINVAL: return "invalid argument";
+    case SCOOT_ENOMEM: return "out of device memory";
+    case SCOOT_ECUDA: return "CUDA runtime error";
+    case SCOOT_EDEVICE: return "device-side index or value check failed";
+    case SCOOT_ETIMEOUT: return "bounded device wait timed out";
+    case SCOOT_EUNSUPPORTED: return "unsupported size or option";
+    default: return "unknown status";
+    }
+}
+
+// ---------------------------------------------------------------- GP state
+
+scoot_status scoot_gp_layout_init(int32_t n, int32_t d, int32_t n_obj, int32_t kernel,
+                                  scoot_gp_layout* out) {
+    if (!out) return SCOOT_EINVAL;
+    std::memset(out, 0, sizeof(*out));
+    if (n < 1 || d < 1 || n_obj < 1) return SCOOT_EINVAL;
+    if (n > SCOOT_MAX_OBS || d > SCOOT_MAX_DIM || n_obj > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
+    if (kernel != SCOOT_MATERN52 && kernel != SCOOT_MATERN32) return SCOOT_EINVAL;
+    out->n = n;
+    out->d = d;
+    out->n_obj = n_obj;
+    out->kernel = kernel;
+    out->n_rb = (n + kRowBlock - 1) / kRowBlock;
+    out->n_tiles = out->n_rb * (out->n_rb + 1);  // row block b spans 2(b+1) column chunks
+    int64_t off = 0;
+    out->off_fmap = off;  off = align_up(off + (int64_t)d * 4 * 4);
+    out->off_xs = off;    off = align_up(off + (int64_t)n_obj * n * d * 4);
+    out->off_ils = off;   off = align_up(off + (int64_t)n_obj * d * 4);
+    out->off_alpha = off; off = align_up(off + (int64_t)n_obj * n * 4);
+    out->off_linv = off;  off = align_up(off + (int64_t)n_obj * out->n_tiles * kColChunk * kRowBlock * 4);
+    out->off_scal = off;  off = align_up(off + (int64_t)n_obj * 4 * 4);
+    out->bytes = off;
+    return SCOOT_OK;
+}
+
+scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
+                              const float* h_y, const float* h_lengthscale,
+                              const float* h_signal_var, const float* h_noise_var,
+                              const scoot_gp_layout* L, void* h_blob, double* h_cond) {
+    if (!h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var || !L || !h_blob)
+        return SCOOT_EINVAL;
+    scoot_gp_layout chk;
+    if (scoot_gp_layout_init(L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK ||
+        std::memcmp(&chk, L, sizeof(chk)) != 0)
+        return SCOOT_EINVAL;
+    const int n = L->n, d = L->d, M = L->n_obj;
+    if (ld_obs < n || !valid_space(h_space, d)) return SCOOT_EINVAL;
+    for (int m = 0; m < M; ++m) {
+        if (!(h_signal_var[m] > 0.0f) || !is_finite(h_signal_var[m])) return SCOOT_EINVAL;
+        if (!(h_noise_var[m] >= 0.0f) || !is_finite(h_noise_var[m])) return SCOOT_EINVAL;
+        for (int c = 0; c < d; ++c)
+            if (!(h_lengthscale[m * d + c] > 0.0f) || !is_finite(h_lengthscale[m * d + c])) return SCOOT_EINVAL;
+        for (int j = 0; j < n; ++j)
+            if (!is_finite(h_y[m * n + j])) return SCOOT_EINVAL;
+    }
+
+    // Features of the observations.
+    std::vector<double> u((size_t)n * d);
+    for (int j = 0; j < n; ++j)
+        for (int c = 0; c < d; ++c) {
+            double v = stored_value(h_space[c], h_x_obs[(size_t)c * ld_obs + j]);
+            if (!is_finite(v)) return SCOOT_EINVAL;
+            if (h_space[c].kind == SCOOT_INT_LOG && !(v > 0.0)) return SCOOT_EINVAL;
+            u[(size_t)j * d + c] = feature(h_space[c], v);
+        }
+
+    char* blob = static_cast<char*>(h_blob);
+    std::memset(blob, 0, (size_t)L->bytes);
+    float* fmap = reinterpret_cast<float*>(blob + L->off_fmap);
+    for (int c = 0; c < d; ++c) {
+        const scoot_param& p = h_space[c];
+        float a = 0.f, b = 0.f;
+        if (p.kind == SCOOT_INT_LOG) {
+            a = (float)std::log((double)p.lo);
+            b = (float)(1.0 / (std::log((double)p.hi) - std::log((double)p.lo)));
+        } else if (p.kind != SCOOT_CATEGORICAL) {
+            a = p.lo;
+            b = p.hi > p.lo ? (float)(1.0 / ((double)p.hi - (double)p.lo)) : 0.0f;
+        }
+        fmap[c * 4 + 0] = (float)p.kind;
+        fmap[c * 4 + 1] = a;
+        fmap[c * 4 + 2] = b;
+    }
+
+    float* xs = reinterpret_cast<float*>(blob + L->off_xs);
+    float* ils = reinterpret_cast<float*>(blob + L->off_ils);
+    float* alpha_out = reinterpret_cast<float*>(blob + L->off_alpha);
+    float* linv_out = reinterpret_cast<float*>(blob + L->off_linv);
+    float* scal = reinterpret_cast<float*>(blob + L->off_scal);
+
+    std::vector<double> K((size_t)n * n), Li((size_t)n * n), alpha(n), tmp(n);
+    for (int m = 0; m < M; ++m) {
+        const float* ell = h_lengthscale + (size_t)m * d;
+        const double sf2 = h_signal_var[m], tau2 = h_noise_var[m];
+        for (int c = 0; c < d; ++c) {
+            bool cat = h_space[c].kind == SCOOT_CATEGORICAL;
+            double l = ell[c];
+            ils[m * d + c] = cat ? (float)(1.0 / (l * l)) : (float)(1.0 / l);
+            for (int j = 0; j < n; ++j)
+                xs[((size_t)m * n + j) * d + c] = cat ? (float)u[(size_t)j * d + c] : (float)(u[(size_t)j * d + c] / l);
+        }
+        // K + tau^2 I
+        for (int i = 0; i < n; ++i)
+            for (int j = 0; j <= i; ++j) {
+                double r2 = 0.0;
+                for (int c = 0; c < d; ++c) {
+                    double l = ell[c];
+                    if (h_space[c].kind == SCOOT_CATEGORICAL) {
+                        if (u[(size_t)i * d + c] != u[(size_t)j * d + c]) r2 += 1.0 / (l * l);
+                    } else {
+                        double t = (u[(size_t)i * d + c] - u[(size_t)j * d + c]) / l;
+                        r2 += t * t;
+                    }
+                }
+                double k = sf2 * matern(std::sqrt(r2), L->kernel);
+                K[(size_t)i * n + j] = K[(size_t)j * n + i] = k + (i == j ? tau2 : 0.0);
+            }
+        // Cholesky K = C C^T (lower, in place in the lower triangle).
+        double pmin = std::numeric_limits<double>::infinity(), pmax = 0.0;
+        for (int j = 0; j < n; ++j) {
+            double s = K[(size_t)j * n + j];
+            for (int k = 0; k < j; ++k) s -= K[(size_t)j * n + k] * K[(size_t)j * n + k];
+            if (!(s > 0.0) || !is_finite(s)) return SCOOT_EINVAL;
+            double piv = std::sqrt(s);
+            K[(size_t)j * n + j] = piv;
+            pmin = std::min(pmin, piv);
+            pmax = std::max(pmax, piv);
+            for (int i = j + 1; i < n; ++i) {
+                double t = K[(size_t)i * n + j];
+                for (int k = 0; k < j; ++k) t -= K[(size_t)i * n + k] * K[(size_t)j * n + k];
+                K[(size_t)i * n + j] = t / piv;
+            }
+        }
+        if (h_cond) h_cond[m] = (pmax / pmin) * (pmax / pmin);
+        // alpha = C^{-T} C^{-1} y
+        for (int i = 0; i < n; ++i) {
+            double t = h_y[(size_t)m * n + i];
+            for (int k = 0; k < i; ++k) t -= K[(size_t)i * n + k] * tmp[k];
+            tmp[i] = t / K[(size_t)i * n + i];
+        }
+        for (int i = n - 1; i >= 0; --i) {
+            double t = tmp[i];
+            for (int k = i + 1; k < n; ++k) t -= K[(size_t)k * n + i] * alpha[k];
+            alpha[i] = t / K[(size_t)i * n + i];
+        }
+        for (int i = 0; i < n; ++i) alpha_out[(size_t)m * n + i] = (float)alpha[i];
+        // L^{-1} = C^{-1} by forward substitution on the identity, column by column.
+        std::fill(Li.begin(), Li.end(), 0.0);
+        for (int col = 0; col < n; ++col) {
+            for (int i = col; i < n; ++i) {
+                double t = (i == col) ? 1.0 : 0.0;
+                for (int k = col; k < i; ++k) t -= K[(size_t)i * n + k] * Li[(size_t)k * n + col];
+                Li[(size_t)i * n + col] = t / K[(size_t)i * n + i];
+            }
+        }
+        // Tiles: row block rb covers rows [64 rb, 64 rb + 64) and column
+        // chunks cj = 0 .. 2 rb + 1 of 32 columns; tile[jj][ii] = Li[row][col].
+        float* tiles = linv_out + (size_t)m * L->n_tiles * kColChunk * kRowBlock;
+        int t = 0;
+        for (int rb = 0; rb < L->n_rb; ++rb)
+            for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t)
+                for (int jj = 0; jj < kColChunk; ++jj)
+                    for (int ii = 0; ii < kRowBlock; ++ii) {
+                        int row = rb * kRowBlock + ii, col = cj * kColChunk + jj;
+                        float v = 0.0f;
+                        if (row < n && col <= row) v = (float)Li[(size_t)row * n + col];
+                        tiles[((size_t)t * kColChunk + jj) * kRowBlock + ii] = v;
+                    }
+        float ybest = -std::numeric_limits<float>::infinity();
+        for (int j = 0; j < n; ++j) ybest = std::max(ybest, h_y[(size_t)m * n + j]);
+        scal[m * 4 + 0] = (float)sf2;
+        scal[m * 4 + 1] = (float)tau2;
+        scal[m * 4 + 2] = ybest;
+    }
+    return SCOOT_OK;
+}
+
+// ---------------------------------------------------------------- boxes
+
+scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, const float* h_ref,
+                               int32_t cap, float* h_lo, float* h_hi, int32_t* n_boxes,
+                               int32_t* front_size) {
+    if (!h_ref || !n_boxes || cap < 0 || n_pts < 0 || (n_pts > 0 && !h_y)) return SCOOT_EINVAL;
+    if (n_obj < 2 || n_obj > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
+    const int M = n_obj;
+    for (int j = 0; j < M; ++j)
+        if (!is_finite(h_ref[j])) return SCOOT_EINVAL;
+    // Points strictly above the reference point.
+    std::vector<std::vector<double>> pts;
+    for (int i = 0; i < n_pts; ++i) {
+        std::vector<double> p(M);
+        bool above = true;
+        for (int j = 0; j < M; ++j) {
+            p[j] = h_y[(size_t)j * n_pts + i];
+            if (!is_finite(p[j])) return SCOOT_EINVAL;
+            above &= p[j] > (double)h_ref[j];
+        }
+        if (above) pts.push_back(p);
+    }
+    // Non-dominated subset (duplicates kept once).
+    std::vector<std::vector<double>> front;
+    for (size_t i = 0; i < pts.size(); ++i) {
+        bool dom = false;
+        for (size_t k = 0; k < pts.size() && !dom; ++k) {
+            if (k == i) continue;
+            bool ge = true, gt = false;
+            for (int j = 0; j < M; ++j) {
+                ge &= pts[k][j] >= pts[i][j];
+                gt |= pts[k][j] > pts[i][j];
+            }
+            dom = ge && (gt || k < i);
+        }
+        if (!dom) front.push_back(pts[i]);
+    }
+    if (front_size) *front_size = (int32_t)front.size();
+    // Grid on axes 0 .. M-2: the reference coordinate and the front's.
+    const int G = M - 1;
+    std::vector<std::vector<double>> axis(G);
+    for (int j = 0; j < G; ++j) {
+        axis[j].push_back(h_ref[j]);
+        for (auto& p : front) axis[j].push_back(p[j]);
+        std::sort(axis[j].begin(), axis[j].end());
+        axis[j].erase(std::unique(axis[j].begin(), axis[j].end()), axis[j].end());
+    }
+    const double inf = std::numeric_limits<double>::infinity();
+    // Column over a cell: above h = the highest last-objective value among
+    // front points that dominate the cell's upper corner on axes 0..M-2.
+    std::vector<int> k(G, 0);
+    struct Box { std::vector<double> lo, hi; };
+    std::vector<Box> out;
+    bool done = false;
+    while (!done) {
+        // Cells along the last grid axis (G-1) are merged while h is unchanged.
+        std::vector<double> up(G);
+        for (int j = 0; j < G - 1; ++j)
+            up[j] = k[j] + 1 < (int)axis[j].size() ? axis[j][k[j] + 1] : inf;
+        const int last = G - 1;
+        const int cells = (int)axis[last].size();
+        double prev_h = 0.0;
+        for (int kk = 0; kk < cells; ++kk) {
+            up[last] = kk + 1 < cells ? axis[last][kk + 1] : inf;
+            double h = -inf;
+            for (auto& p : front) {
+                bool dominates = true;
+                for (int j = 0; j < G; ++j) dominates &= p[j] >= up[j];
+                if (dominates) h = std::max(h, p[M - 1]);
+            }
+            double lo_last = std::max((double)h_ref[M - 1], h);
+            if (kk > 0 && lo_last == prev_h) {
+                out.back().hi[last] = up[last];
+                continue;
+            }
+            Box b;
+            b.lo.resize(M);
+            b.hi.resize(M);
+            for (int j = 0; j < G; ++j) {
+                b.lo[j] = axis[j][j == last ? kk : k[j]];
+                b.hi[j] = up[j];
+            }
+            b.lo[M - 1] = lo_last;
+            b.hi[M - 1] = inf;
+            out.push_back(b);
+            prev_h = lo_last;
+        }
+        // Next cell of axes 0 .. G-2 (odometer).
+        int j = G - 2;
+        while (j >= 0) {
+            if (++k[j] < (int)axis[j].size()) break;
+            k[j] = 0;
+            --j;
+        }
+        done = j < 0;
+    }
+    *n_boxes = (int32_t)out.size();
+    if ((int32_t)out.size() > cap) return SCOOT_EUNSUPPORTED;
+    if (!out.empty() && (!h_lo || !h_hi)) return SCOOT_EINVAL;
+    for (size_t b = 0; b < out.size(); ++b)
+        for (int j = 0; j < M; ++j) {
+            h_lo[b * M + j] = (float)out[b].lo[j];
+            h_hi[b * M + j] = std::isinf(out[b].hi[j]) ? std::numeric_limits<float>::infinity()
+                                                       : (float)out[b].hi[j];
+        }
+    return SCOOT_OK;
+}
+
+// ---------------------------------------------------------------- forest
+
+scoot_status scoot_forest_layout_init(const scoot_node* h_nodes, const int32_t* h_tree_offset,
+                                      int32_t n_trees, int32_t d, int32_t leaf_scale,
+                                      scoot_forest_layout* out) {
+    if (!out) return SCOOT_EINVAL;
+    std::memset(out, 0, sizeof(*out));
+    if (!h_nodes || !h_tree_offset || n_trees < 1 || d < 1 || d > SCOOT_MAX_DIM || leaf_scale < 1)
+        return SCOOT_EINVAL;
+    if (h_tree_offset[0] != 0) return SCOOT_EINVAL;
+    int max_depth = 0;
+    std::vector<int> depth;
+    std::vector<int32_t> chunks;  // first tree, count, first node, node count
+    int chunk_first = 0, chunk_nodes = 0;
+    for (int t = 0; t < n_trees; ++t) {
+        int32_t b = h_tree_offset[t], e = h_tree_offset[t + 1];
+        int size = e - b;
+        if (size < 1 || size > 65535) return SCOOT_EINVAL;
+        if (size > kForestChunkNodes) return SCOOT_EUNSUPPORTED;
+        depth.assign(size, -1);
+        depth[0] = 0;
+        for (int i = 0; i < size; ++i) {
+            const scoot_node& nd = h_nodes[b + i];
+            if (depth[i] < 0) return SCOOT_EINVAL;  // unreachable node
+            if (nd.flags & 1) {
+                float v = nd.val;
+                if (!(v >= 0.0f) || v > (float)leaf_scale || v != std::floor(v)) return SCOOT_EINVAL;
+                max_depth = std::max(max_depth, depth[i]);
+            } else {
+                if (nd.feat >= d || !is_finite(nd.val)) return SCOOT_EINVAL;
+                int l = nd.left;
+                if (l <= i || l + 1 >= size) return SCOOT_EINVAL;
+                if (depth[l] >= 0 || depth[l + 1] >= 0) return SCOOT_EINVAL;  // shared child
+                depth[l] = depth[l + 1] = depth[i] + 1;
+            }
+        }
+        if (chunk_nodes + size > kForestChunkNodes) {
+            chunks.insert(chunks.end(), {chunk_first, t - chunk_first, h_tree_offset[chunk_first], chunk_nodes});
+            chunk_first = t;
+            chunk_nodes = 0;
+        }
+        chunk_nodes += size;
+    }
+    chunks.insert(chunks.end(), {chunk_first, n_trees - chunk_first, h_tree_offset[chunk_first], chunk_nodes});
+    out->n_trees = n_trees;
+    out->n_nodes = h_tree_offset[n_trees];
+    out->d = d;
+    out->leaf_scale = leaf_scale;
+    out->max_depth = max_depth;
+    out->n_chunks = (int32_t)(chunks.size() / 4);
+    for (size_t c = 0; c < chunks.size(); c += 4)
+        out->max_chunk_nodes = std::max(out->max_chunk_nodes, chunks[c + 3]);
+    int64_t off = 0;
+    out->off_chunks = off; off = align_up(off + (int64_t)out->n_chunks * 16);
+    out->off_roots = off;  off = align_up(off + (int64_t)n_trees * 4);
+    out->off_nodes = off;  off = align_up(off + (int64_t)out->n_nodes * 8);
+    out->bytes = off;
+    return SCOOT_OK;
+}
+
+scoot_status scoot_forest_pack(const scoot_forest_layout* L, const scoot_node* h_nodes,
+                               const int32_t* h_tree_offset, void* h_blob) {
+    if (!L || !h_nodes || !h_tree_offset || !h_blob) return SCOOT_EINVAL;
+    scoot_forest_layout chk;
+    scoot_status s = scoot_forest_layout_init(h_nodes, h_tree_offset, L->n_trees, L->d, L->leaf_scale, &chk);
+    if (s != SCOOT_OK) return s;
+    if (std::memcmp(&chk, L, sizeof(chk)) != 0) return SCOOT_EINVAL;
+    char* blob = static_cast<char*>(h_blob);
+    std::memset(blob, 0, (size_t)L->bytes);
+    int32_t* ch = reinterpret_cast<int32_t*>(blob + L->off_chunks);
+    int c = 0, first = 0, nodes = 0;
+    for (int t = 0; t < L->n_trees; ++t) {
+        int size = h_tree_offset[t + 1] - h_tree_offset[t];
+        if (nodes + size > kForestChunkNodes) {
+            ch[c * 4 + 0] = first; ch[c * 4 + 1] = t - first;
+            ch[c * 4 + 2] = h_tree_offset[first]; ch[c * 4 + 3] = nodes;
+            ++c; first = t; nodes = 0;
+        }
+        nodes += size;
+    }
+    ch[c * 4 + 0] = first; ch[c * 4 + 1] = L->n_trees - first;
+    ch[c * 4 + 2] = h_tree_offset[first]; ch[c * 4 + 3] = nodes;
+    std::memcpy(blob + L->off_roots, h_tree_offset, (size_t)L->n_trees * 4);
+    std::memcpy(blob + L->off_nodes, h_nodes, (size_t)L->n_nodes * 8);
+    return SCOOT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,328 @@
+// Known-constraint pruning (Eq. 2) and random-forest probability of
+// feasibility (Eq. 3) over a structure-of-arrays candidate pool.
+#include <cstring>
+
+#include "internal.h"
+
+namespace {
+
+constexpr int kPruneThreads = 256;
+constexpr int kRfThreads = 256;
+constexpr int kRfPerThread = 2;                  // candidates walked together (ILP)
+constexpr int kRfTile = kRfThreads * kRfPerThread;
+
+struct PruneArgs {
+    int32_t n_clauses;
+    int32_t pad;
+    scoot_clause cl[SCOOT_MAX_CLAUSES];
+};
+
+__device__ __forceinline__ int4 ld_col4(const uint32_t* __restrict__ cand, int64_t ld, int p, int64_t i0) {
+    return __ldg(reinterpret_cast<const int4*>(cand + (int64_t)p * ld + i0));
+}
+
+// Block-wide sum of per-thread counts, added once per block to *count.
+__device__ __forceinline__ void add_count(unsigned long long* count, uint32_t mine) {
+    __shared__ uint32_t warp_sums[32];
+    for (int o = 16; o > 0; o >>= 1) mine += __shfl_xor_sync(0xffffffffu, mine, o);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) warp_sums[warp] = mine;
+    __syncthreads();
+    if (warp == 0) {
+        uint32_t v = lane < (int)(blockDim.x >> 5) ? warp_sums[lane] : 0u;
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0 && v) atomicAdd(count, (unsigned long long)v);
+    }
+}
+
+// One thread evaluates every clause on four consecutive candidates, reading
+// each referenced column as one 16-byte load (ld % 4 == 0, columns aligned).
+__global__ void __launch_bounds__(kPruneThreads)
+prune_kernel(const __grid_constant__ PruneArgs a, const uint32_t* __restrict__ cand, int64_t n,
+             int64_t ld, uint8_t* __restrict__ mask, unsigned long long* count) {
+    const int64_t n4 = (n + 3) >> 2;
+    uint32_t feasible = 0;
+    const bool vec_store = (reinterpret_cast<uintptr_t>(mask) & 3u) == 0;
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < n4;
+         q += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i0 = q << 2;
+        bool ok0 = true, ok1 = true, ok2 = true, ok3 = true;
+        for (int c = 0; c < a.n_clauses; ++c) {
+            const scoot_clause& C = a.cl[c];
+            bool g0 = true, g1 = true, g2 = true, g3 = true;
+            for (int k = 0; k < C.n_guard; ++k) {
+                int4 v = ld_col4(cand, ld, C.guard_param[k], i0);
+                const int gv = C.guard_value[k];
+                g0 &= v.x == gv; g1 &= v.y == gv; g2 &= v.z == gv; g3 &= v.w == gv;
+            }
+            if (!(g0 | g1 | g2 | g3)) continue;
+            __int128 s0 = 0, s1 = 0, s2 = 0, s3 = 0;
+            for (int t = 0; t < C.n_term; ++t) {
+                int4 v = ld_col4(cand, ld, C.term_param[t], i0);
+                const __int128 k = C.coef[t];
+                s0 += k * v.x; s1 += k * v.y; s2 += k * v.z; s3 += k * v.w;
+            }
+            const __int128 r = C.rhs;
+            ok0 &= !g0 || s0 >= r; ok1 &= !g1 || s1 >= r;
+            ok2 &= !g2 || s2 >= r; ok3 &= !g3 || s3 >= r;
+        }
+        const uint8_t m0 = ok0, m1 = ok1, m2 = ok2, m3 = ok3;
+        if (i0 + 3 < n) {
+            feasible += m0 + m1 + m2 + m3;
+            if (vec_store) {
+                *reinterpret_cast<uchar4*>(mask + i0) = make_uchar4(m0, m1, m2, m3);
+            } else {
+                mask[i0] = m0; mask[i0 + 1] = m1; mask[i0 + 2] = m2; mask[i0 + 3] = m3;
+            }
+        } else {
+            const uint8_t mm[4] = {m0, m1, m2, m3};
+            for (int k = 0; k < 4 && i0 + k < n; ++k) {
+                mask[i0 + k] = mm[k];
+                feasible += mm[k];
+            }
+        }
+    }
+    if (count) add_count(count, feasible);
+}
+
+struct RfArgs {
+    const char* forest;
+    int64_t off_chunks, off_roots, off_nodes;
+    int32_t n_chunks, n_trees, max_depth, d;
+    uint32_t float_cols;          // bit c set: column c holds float32 values
+    uint32_t delta_num, delta_den, leaf_scale;
+    const uint32_t* cand;
+    int64_t n, ld;
+    uint32_t* votes;
+    uint8_t* mask;
+    unsigned long long* count;
+    uint32_t* err;
+    int32_t single_chunk;
+};
+
+// Persistent blocks: each stages (a chunk of) the forest in shared memory,
+// then walks tiles of kRfTile candidates whose feature values sit in shared
+// memory as feat[c][slot] (bank = slot % 32, so lanes never conflict).
+__global__ void __launch_bounds__(kRfThreads)
+rf_kernel(const __grid_constant__ RfArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    float* sfeat = reinterpret_cast<float*>(smem_raw);                       // [d][kRfTile]
+    uint2* snodes = reinterpret_cast<uint2*>(sfeat + a.d * kRfTile);         // chunk nodes
+
+    const int32_t* chunks = reinterpret_cast<const int32_t*>(a.forest + a.off_chunks);
+    const int32_t* roots = reinterpret_cast<const int32_t*>(a.forest + a.off_roots);
+    const uint2* gnodes = reinterpret_cast<const uint2*>(a.forest + a.off_nodes);
+    const int tid = threadIdx.x;
+    const int64_t n_tiles = (a.n + kRfTile - 1) / kRfTile;
+    uint32_t feasible = 0;
+
+    auto stage_chunk = [&](int ch) {
+        const int first_node = chunks[ch * 4 + 2], count = chunks[ch * 4 + 3];
+        for (int k = tid; k < count; k += kRfThreads) snodes[k] = __ldg(gnodes + first_node + k);
+    };
+    if (a.single_chunk) {
+        stage_chunk(0);
+        __syncthreads();
+    }
+
+    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+        const int64_t base = tile * kRfTile;
+        int64_t idx[kRfPerThread];
+        bool live[kRfPerThread];
+        int any = 0;
+#pragma unroll
+        for (int r = 0; r < kRfPerThread; ++r) {
+            idx[r] = base + tid + r * kRfThreads;
+            live[r] = idx[r] < a.n && (a.mask == nullptr || a.mask[idx[r]] != 0);
+            any |= live[r];
+        }
+        if (!__syncthreads_or(any)) {
+            // Nothing to walk in this tile: votes are 0, masks stay 0.
+#pragma unroll
+            for (int r = 0; r < kRfPerThread; ++r)
+                if (idx[r] < a.n) a.votes[idx[r]] = 0u;
+            continue;
+        }
+        for (int c = 0; c < a.d; ++c) {
+            const bool isf = (a.float_cols >> c) & 1u;
+#pragma unroll
+            for (int r = 0; r < kRfPerThread; ++r) {
+                float x = 0.0f;
+                if (idx[r] < a.n) {
+                    uint32_t w = __ldg(a.cand + (int64_t)c * a.ld + idx[r]);
+                    x = isf ? __uint_as_float(w) : (float)(int32_t)w;
+                }
+                sfeat[c * kRfTile + tid + r * kRfThreads] = x;
+            }
+        }
+        uint32_t vote[kRfPerThread];
+#pragma unroll
+        for (int r = 0; r < kRfPerThread; ++r) vote[r] = 0u;
+
+        for (int ch = 0; ch < a.n_chunks; ++ch) {
+            if (!a.single_chunk) {
+                __syncthreads();
+                stage_chunk(ch);
+            }
+            __syncthreads();
+            const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1], node0 = chunks[ch * 4 + 2];
+            for (int t = t0; t < t0 + nt; ++t) {
+                const int root = roots[t] - node0;
+                int node[kRfPerThread];
+                bool done[kRfPerThread];
+#pragma unroll
+                for (int r = 0; r < kRfPerThread; ++r) {
+                    node[r] = root;
+                    done[r] = !live[r];
+                }
+                for (int step = 0; step <= a.max_depth; ++step) {
+                    bool all_done = true;
+#pragma unroll
+                    for (int r = 0; r < kRfPerThread; ++r) {
+                        if (!done[r]) {
+                            const uint2 nd = snodes[node[r]];
+                            if ((nd.y >> 24) & 1u) {
+                                vote[r] += (uint32_t)__uint_as_float(nd.x);
+                                done[r] = true;
+                            } else {
+                                const int feat = (nd.y >> 16) & 0xff;
+                                const float x = sfeat[feat * kRfTile + tid + r * kRfThreads];
+                                node[r] = root + (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
+                            }
+                        }
+                        all_done &= done[r];
+                    }
+                    if (all_done) break;
+                }
+#pragma unroll
+                for (int r = 0; r < kRfPerThread; ++r)
+                    if (!done[r]) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
+            }
+        }
+        const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
+#pragma unroll
+        for (int r = 0; r < kRfPerThread; ++r) {
+            if (idx[r] >= a.n) continue;
+            a.votes[idx[r]] = live[r] ? vote[r] : 0u;
+            if (live[r]) {
+                const bool ok = (unsigned __int128)a.delta_den * vote[r] >= need;
+                if (a.mask) a.mask[idx[r]] = ok;
+                feasible += ok;
+            }
+        }
+        __syncthreads();  // sfeat is rewritten by the next tile
+    }
+    if (a.count) add_count(a.count, feasible);
+}
+
+int sm_count(int device) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, device);
+    return v > 0 ? v : 1;
+}
+
+}  // namespace
+
+extern "C" {
+
+scoot_status scoot_prune(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
+                         const scoot_clause* h_clauses, int32_t n_clauses,
+                         const uint32_t* cand, int64_t n, int64_t ld,
+                         uint8_t* mask, int64_t* n_feasible, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (!h_space) return scoot_fail(ctx, SCOOT_EINVAL, "h_space is NULL");
+    if ((s = scoot_check_pool(ctx, cand, n, ld, d)) != SCOOT_OK) return s;
+    if (n_clauses < 0 || n_clauses > SCOOT_MAX_CLAUSES)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n_clauses = %d outside 0..%d", n_clauses, SCOOT_MAX_CLAUSES);
+    if (n_clauses > 0 && !h_clauses) return scoot_fail(ctx, SCOOT_EINVAL, "h_clauses is NULL");
+    if (n > 0 && !mask) return scoot_fail(ctx, SCOOT_EINVAL, "mask is NULL");
+    PruneArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.n_clauses = n_clauses;
+    for (int c = 0; c < n_clauses; ++c) {
+        const scoot_clause& C = h_clauses[c];
+        if (C.n_guard < 0 || C.n_guard > 2 || C.n_term < 0 || C.n_term > 4)
+            return scoot_fail(ctx, SCOOT_EINVAL, "clause %d: n_guard %d / n_term %d out of range", c, C.n_guard, C.n_term);
+        for (int g = 0; g < C.n_guard; ++g) {
+            int p = C.guard_param[g];
+            if (p < 0 || p >= d || h_space[p].kind == SCOOT_CONTINUOUS)
+                return scoot_fail(ctx, SCOOT_EINVAL, "clause %d: guard parameter %d invalid", c, p);
+        }
+        for (int t = 0; t < C.n_term; ++t) {
+            int p = C.term_param[t];
+            if (p < 0 || p >= d || h_space[p].kind == SCOOT_CONTINUOUS)
+                return scoot_fail(ctx, SCOOT_EINVAL, "clause %d: term parameter %d invalid", c, p);
+        }
+        a.cl[c] = C;
+    }
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (n_feasible) SCOOT_CUDA(ctx, cudaMemsetAsync(n_feasible, 0, sizeof(int64_t), st));
+    if (n == 0) return SCOOT_OK;
+    const int64_t n4 = (n + 3) / 4;
+    int64_t blocks = (n4 + kPruneThreads - 1) / kPruneThreads;
+    const int64_t cap = (int64_t)sm_count(ctx->device) * 8;
+    if (blocks > cap) blocks = cap;
+    prune_kernel<<<(unsigned)blocks, kPruneThreads, 0, st>>>(
+        a, cand, n, ld, mask, reinterpret_cast<unsigned long long*>(n_feasible));
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+scoot_status scoot_rf_predict(scoot_ctx* ctx, const scoot_forest_layout* L, const void* forest,
+                              const scoot_param* h_space, const uint32_t* cand, int64_t n, int64_t ld,
+                              uint32_t delta_num, uint32_t delta_den, uint32_t* votes, uint8_t* mask,
+                              int64_t* n_feasible, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (!L || !forest || !h_space) return scoot_fail(ctx, SCOOT_EINVAL, "layout, forest or h_space is NULL");
+    if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
+    if (L->n_trees < 1 || L->n_chunks < 1 || L->max_depth < 0 || L->leaf_scale < 1)
+        return scoot_fail(ctx, SCOOT_EINVAL, "forest layout is not initialised");
+    if (delta_den == 0) return scoot_fail(ctx, SCOOT_EINVAL, "delta_den = 0");
+    if (n > 0 && !votes) return scoot_fail(ctx, SCOOT_EINVAL, "votes is NULL");
+    if (!scoot_aligned16(forest)) return scoot_fail(ctx, SCOOT_EINVAL, "forest blob is not 16-byte aligned");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (n_feasible) SCOOT_CUDA(ctx, cudaMemsetAsync(n_feasible, 0, sizeof(int64_t), st));
+    if (n == 0) return SCOOT_OK;
+
+    const int max_chunk_nodes = L->max_chunk_nodes;
+    if (max_chunk_nodes < 1 || max_chunk_nodes > L->n_nodes)
+        return scoot_fail(ctx, SCOOT_EINVAL, "forest layout is not initialised");
+    RfArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.forest = static_cast<const char*>(forest);
+    a.off_chunks = L->off_chunks;
+    a.off_roots = L->off_roots;
+    a.off_nodes = L->off_nodes;
+    a.n_chunks = L->n_chunks;
+    a.n_trees = L->n_trees;
+    a.max_depth = L->max_depth;
+    a.d = L->d;
+    for (int c = 0; c < L->d; ++c)
+        if (h_space[c].kind == SCOOT_CONTINUOUS) a.float_cols |= 1u << c;
+    a.delta_num = delta_num;
+    a.delta_den = delta_den;
+    a.leaf_scale = (uint32_t)L->leaf_scale;
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.votes = votes;
+    a.mask = mask;
+    a.count = reinterpret_cast<unsigned long long*>(n_feasible);
+    a.err = ctx->d_err;
+    a.single_chunk = L->n_chunks == 1;
+    const size_t smem = (size_t)L->d * kRfTile * 4 + (size_t)max_chunk_nodes * 8;
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(rf_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    int per_sm = 0;
+    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rf_kernel, kRfThreads, smem));
+    if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "forest chunk does not fit in shared memory");
+    const int64_t tiles = (n + kRfTile - 1) / kRfTile;
+    int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
+    if (blocks > tiles) blocks = tiles;
+    rf_kernel<<<(unsigned)blocks, kRfThreads, smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+}  // extern "C"

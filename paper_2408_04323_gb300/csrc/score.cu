@@ -1,0 +1,511 @@
+// GP posterior (Section 4.3) and acquisition values: EI (Eq. 6) and
+// Monte-Carlo EHVI over a box decomposition (Eq. 7), fused or separate.
+//
+// A block of 64 threads owns a tile of 64 candidates.  Per objective:
+//  1. each thread evaluates its candidate's covariance row k(x, X) against
+//     the n observations (staged in shared memory) into Ks[j][c] and
+//     accumulates mu = k . alpha;
+//  2. the block computes V = L^{-1} Ks as a register-tiled SIMT product
+//     (8 candidates x 8 rows per thread) over 32 x 64 tiles of L^{-1} that the
+//     host laid out transposed and zero-filled, and reduces sum_i V_ic^2;
+//     sigma^2 = s_f^2 - sum_i V_ic^2, clamped at 0.
+// The epilogue writes mu and sigma^2, or the EI, or the EHVI of the tile.
+#include <cstring>
+
+#include "internal.h"
+
+namespace {
+
+constexpr int kTC = 64;     // candidates per tile = threads per block
+constexpr int kRB = 64;     // rows of L^{-1} per tile
+constexpr int kCJ = 32;     // columns of L^{-1} per tile
+constexpr int kMaxD = SCOOT_MAX_DIM;
+constexpr int kMaxM = SCOOT_MAX_OBJ;
+constexpr int kAcqThreads = 128;
+
+enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2 };
+
+struct ScoreArgs {
+    const char* state;
+    int64_t off_fmap, off_xs, off_ils, off_alpha, off_linv, off_scal;
+    int32_t n_obs, d, dp, n_obj, kernel, n_rb, n_tiles;
+    const uint32_t* cand;
+    int64_t n, ld;
+    const uint8_t* mask;
+    float* mean;
+    float* var;
+    int64_t ldo;
+    float* acq;
+    float xi;
+    const float* box_lo;
+    const float* box_hi;
+    int32_t n_boxes;
+    const float* eps;
+    int32_t n_mc;
+};
+
+__device__ __forceinline__ float matern(float r, int kernel) {
+    if (kernel == SCOOT_MATERN32) {
+        const float a = 1.7320508075688772f * r;
+        return (1.0f + a) * expf(-a);
+    }
+    const float a = 2.2360679774997896f * r;
+    return fmaf(a, fmaf(a, 0.33333333333333333f, 1.0f), 1.0f) * expf(-a);
+}
+
+__device__ __forceinline__ float ei_value(float mu, float var, float ybest, float xi) {
+    const float a = (mu - ybest) + xi;
+    const float s = sqrtf(fmaxf(var, 0.0f));
+    if (!(s > 0.0f)) return fmaxf(a, 0.0f);
+    const float z = a / s;
+    const float cdf = 0.5f * erfcf(-z * 0.70710678118654752f);
+    const float pdf = 0.39894228040143268f * expf(-0.5f * z * z);
+    return fmaf(a, cdf, s * pdf);
+}
+
+// HVI summed over S base samples for one candidate; boxes as float4 rows
+// (lo, hi padded to four objectives), eps as float4 rows.
+template <int M>
+__device__ __forceinline__ float ehvi_value(const float* mu, const float* sd, const float4* blo,
+                                            const float4* bhi, int n_boxes, const float4* eps,
+                                            int n_mc) {
+    float acc = 0.0f;
+    for (int s = 0; s < n_mc; ++s) {
+        const float4 e = eps[s];
+        const float y0 = fmaf(sd[0], e.x, mu[0]);
+        const float y1 = fmaf(sd[1], e.y, mu[1]);
+        const float y2 = M > 2 ? fmaf(sd[2], e.z, mu[2]) : 0.0f;
+        const float y3 = M > 3 ? fmaf(sd[3], e.w, mu[3]) : 0.0f;
+        float hv = 0.0f;
+        for (int b = 0; b < n_boxes; ++b) {
+            const float4 lo = blo[b], hi = bhi[b];
+            float p = fmaxf(fminf(y0, hi.x) - lo.x, 0.0f) * fmaxf(fminf(y1, hi.y) - lo.y, 0.0f);
+            if (M > 2) p *= fmaxf(fminf(y2, hi.z) - lo.z, 0.0f);
+            if (M > 3) p *= fmaxf(fminf(y3, hi.w) - lo.w, 0.0f);
+            hv += p;
+        }
+        acc += hv;
+    }
+    return acc * (1.0f / (float)n_mc);
+}
+
+__device__ void stage_boxes(const ScoreArgs& a, int M, float4* blo, float4* bhi, float4* eps) {
+    for (int b = threadIdx.x; b < a.n_boxes; b += blockDim.x) {
+        float l[4] = {0.f, 0.f, 0.f, 0.f}, h[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int j = 0; j < M; ++j) {
+            l[j] = a.box_lo[b * M + j];
+            h[j] = a.box_hi[b * M + j];
+        }
+        blo[b] = make_float4(l[0], l[1], l[2], l[3]);
+        bhi[b] = make_float4(h[0], h[1], h[2], h[3]);
+    }
+    for (int s = threadIdx.x; s < a.n_mc; s += blockDim.x) {
+        float e[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int j = 0; j < M; ++j) e[j] = a.eps[s * M + j];
+        eps[s] = make_float4(e[0], e[1], e[2], e[3]);
+    }
+}
+
+template <int EPI, int M>
+__global__ void __launch_bounds__(kTC)
+score_kernel(const __grid_constant__ ScoreArgs a) {
+    extern __shared__ __align__(16) float sm[];
+    const int n_pad = a.n_rb * kRB;
+    float* Ks = sm;                                   // [n_pad][kTC]
+    float* xs = Ks + (size_t)n_pad * kTC;             // [n_obs][dp]
+    float* al = xs + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3));   // [n_pad]
+    float* Lt = al + n_pad;                           // [kCJ][kRB]
+    float* part = Lt + kCJ * kRB;                     // [8][kTC]
+    float4* blo = reinterpret_cast<float4*>(part + 8 * kTC);
+    float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
+    float4* epsv = bhi + (EPI == kEHVI ? a.n_boxes : 0);
+
+    const int tid = threadIdx.x;
+    const int nobj = EPI == kEHVI ? M : (EPI == kEI ? 1 : a.n_obj);
+    const float* fmap = reinterpret_cast<const float*>(a.state + a.off_fmap);
+    const float* gxs = reinterpret_cast<const float*>(a.state + a.off_xs);
+    const float* gils = reinterpret_cast<const float*>(a.state + a.off_ils);
+    const float* galpha = reinterpret_cast<const float*>(a.state + a.off_alpha);
+    const float4* glinv = reinterpret_cast<const float4*>(a.state + a.off_linv);
+    const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
+
+    if (EPI == kEHVI) stage_boxes(a, M, blo, bhi, epsv);  // visible after the first barrier below
+
+    // Per-dimension feature map (uniform across the block).
+    int kind[kMaxD];
+    float fa[kMaxD], fb[kMaxD];
+#pragma unroll
+    for (int c = 0; c < kMaxD; ++c) {
+        kind[c] = c < a.d ? (int)fmap[c * 4] : SCOOT_CATEGORICAL;
+        fa[c] = c < a.d ? fmap[c * 4 + 1] : 0.f;
+        fb[c] = c < a.d ? fmap[c * 4 + 2] : 0.f;
+    }
+
+    const int64_t n_tiles = (a.n + kTC - 1) / kTC;
+    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+        const int64_t i = tile * kTC + tid;
+        const bool live = i < a.n && (a.mask == nullptr || a.mask[i] != 0);
+        if (!__syncthreads_or(live)) {
+            if (EPI != kWriteMoments && i < a.n) a.acq[i] = -INFINITY;
+            continue;
+        }
+        // Features of this thread's candidate.
+        float u[kMaxD];
+#pragma unroll
+        for (int c = 0; c < kMaxD; ++c) {
+            u[c] = 0.0f;
+            if (c < a.d && live) {
+                const uint32_t w = __ldg(a.cand + (int64_t)c * a.ld + i);
+                if (kind[c] == SCOOT_INT_LOG) u[c] = (logf((float)(int32_t)w) - fa[c]) * fb[c];
+                else if (kind[c] == SCOOT_INT_UNIFORM) u[c] = ((float)(int32_t)w - fa[c]) * fb[c];
+                else if (kind[c] == SCOOT_CONTINUOUS) u[c] = (__uint_as_float(w) - fa[c]) * fb[c];
+                else u[c] = (float)(int32_t)w;
+            }
+        }
+        float mu[kMaxM], vr[kMaxM];
+        for (int m = 0; m < nobj; ++m) {
+            __syncthreads();  // previous users of xs / al / part are done
+            const float* sx = gxs + (size_t)m * a.n_obs * a.d;
+            for (int k = tid; k < a.n_obs * a.d; k += kTC) {
+                const int j = k / a.d, c = k - j * a.d;
+                xs[j * a.dp + c] = sx[k];
+            }
+            for (int j = tid; j < n_pad; j += kTC) al[j] = j < a.n_obs ? galpha[(size_t)m * a.n_obs + j] : 0.0f;
+            const float sf2 = gscal[m * 4 + 0];
+            float ut[kMaxD], w2[kMaxD];
+#pragma unroll
+            for (int c = 0; c < kMaxD; ++c) {
+                const float s = c < a.d ? gils[m * a.d + c] : 0.0f;
+                const bool cat = kind[c] == SCOOT_CATEGORICAL;
+                ut[c] = cat ? u[c] : u[c] * s;
+                w2[c] = cat ? s : 0.0f;
+            }
+            __syncthreads();
+            // 1. covariance row and mean.
+            float acc = 0.0f;
+#pragma unroll 2
+            for (int j = 0; j < a.n_obs; ++j) {
+                const float* xj = xs + j * a.dp;
+                float r2 = 0.0f;
+#pragma unroll
+                for (int c = 0; c < kMaxD; ++c) {
+                    if (c < a.d) {
+                        const float t = ut[c] - xj[c];
+                        if (kind[c] == SCOOT_CATEGORICAL) r2 += t != 0.0f ? w2[c] : 0.0f;
+                        else r2 = fmaf(t, t, r2);
+                    }
+                }
+                const float k = sf2 * matern(sqrtf(r2), a.kernel);
+                Ks[j * kTC + tid] = k;
+                acc = fmaf(k, al[j], acc);
+            }
+            for (int j = a.n_obs; j < n_pad; ++j) Ks[j * kTC + tid] = 0.0f;
+            mu[m] = acc;
+            __syncthreads();
+            // 2. V = L^{-1} Ks, sum of squares per candidate.
+            const int cg = tid & 7, rg = tid >> 3;
+            float sq[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) sq[c] = 0.0f;
+            const float4* tiles = glinv + (size_t)m * a.n_tiles * (kCJ * kRB / 4);
+            const float4* Ks4 = reinterpret_cast<const float4*>(Ks);
+            const float4* Lt4 = reinterpret_cast<const float4*>(Lt);
+            int t = 0;
+            for (int rb = 0; rb < a.n_rb; ++rb) {
+                float accm[8][8];
+#pragma unroll
+                for (int r = 0; r < 8; ++r)
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) accm[r][c] = 0.0f;
+                for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t) {
+                    __syncthreads();
+                    const float4* src = tiles + (size_t)t * (kCJ * kRB / 4);
+#pragma unroll
+                    for (int k = 0; k < kCJ * kRB / 4 / kTC; ++k)
+                        reinterpret_cast<float4*>(Lt)[tid + k * kTC] = __ldg(src + tid + k * kTC);
+                    __syncthreads();
+                    const int j0 = cj * kCJ;
+#pragma unroll 4
+                    for (int jj = 0; jj < kCJ; ++jj) {
+                        const float4 k0 = Ks4[(j0 + jj) * (kTC / 4) + cg * 2];
+                        const float4 k1 = Ks4[(j0 + jj) * (kTC / 4) + cg * 2 + 1];
+                        const float4 l0 = Lt4[jj * (kRB / 4) + rg * 2];
+                        const float4 l1 = Lt4[jj * (kRB / 4) + rg * 2 + 1];
+                        const float kv[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
+                        const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
+#pragma unroll
+                        for (int r = 0; r < 8; ++r)
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) accm[r][c] = fmaf(lv[r], kv[c], accm[r][c]);
+                    }
+                }
+#pragma unroll
+                for (int r = 0; r < 8; ++r)
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) sq[c] = fmaf(accm[r][c], accm[r][c], sq[c]);
+            }
+#pragma unroll
+            for (int c = 0; c < 8; ++c) part[rg * kTC + cg * 8 + c] = sq[c];
+            __syncthreads();
+            float ss = 0.0f;
+#pragma unroll
+            for (int g = 0; g < 8; ++g) ss += part[g * kTC + tid];
+            vr[m] = fmaxf(sf2 - ss, 0.0f);
+        }
+        // Epilogue.
+        if (EPI == kWriteMoments) {
+            if (live)
+                for (int m = 0; m < nobj; ++m) {
+                    a.mean[(int64_t)m * a.ldo + i] = mu[m];
+                    a.var[(int64_t)m * a.ldo + i] = vr[m];
+                }
+        } else if (EPI == kEI) {
+            if (i < a.n) a.acq[i] = live ? ei_value(mu[0], vr[0], gscal[2], a.xi) : -INFINITY;
+        } else {
+            if (i < a.n) {
+                float v = -INFINITY;
+                if (live) {
+                    float sd[kMaxM];
+#pragma unroll
+                    for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
+                    v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
+                }
+                a.acq[i] = v;
+            }
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kAcqThreads)
+ei_kernel(const float* __restrict__ mean, const float* __restrict__ var, const uint8_t* __restrict__ mask,
+          int64_t n, float ybest, float xi, float* __restrict__ acq) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const bool live = mask == nullptr || mask[i] != 0;
+        acq[i] = live ? ei_value(mean[i], var[i], ybest, xi) : -INFINITY;
+    }
+}
+
+template <int M>
+__global__ void __launch_bounds__(kAcqThreads)
+ehvi_kernel(const __grid_constant__ ScoreArgs a) {
+    extern __shared__ __align__(16) float sm[];
+    float4* blo = reinterpret_cast<float4*>(sm);
+    float4* bhi = blo + a.n_boxes;
+    float4* epsv = bhi + a.n_boxes;
+    stage_boxes(a, M, blo, bhi, epsv);
+    __syncthreads();
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n; i += (int64_t)gridDim.x * blockDim.x) {
+        const bool live = a.mask == nullptr || a.mask[i] != 0;
+        float v = -INFINITY;
+        if (live) {
+            float mu[kMaxM], sd[kMaxM];
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                mu[m] = a.mean[(int64_t)m * a.ldo + i];
+                sd[m] = sqrtf(fmaxf(a.var[(int64_t)m * a.ldo + i], 0.0f));
+            }
+            v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
+        }
+        a.acq[i] = v;
+    }
+}
+
+int sm_count(int device) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, device);
+    return v > 0 ? v : 1;
+}
+
+scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state, ScoreArgs& a) {
+    if (!L || !state) return scoot_fail(ctx, SCOOT_EINVAL, "layout or state is NULL");
+    scoot_gp_layout chk;
+    if (scoot_gp_layout_init(L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK || std::memcmp(&chk, L, sizeof(chk)) != 0)
+        return scoot_fail(ctx, SCOOT_EINVAL, "GP layout is not one made by scoot_gp_layout_init");
+    if (!scoot_aligned16(state)) return scoot_fail(ctx, SCOOT_EINVAL, "state blob is not 16-byte aligned");
+    std::memset(&a, 0, sizeof(a));
+    a.state = static_cast<const char*>(state);
+    a.off_fmap = L->off_fmap;
+    a.off_xs = L->off_xs;
+    a.off_ils = L->off_ils;
+    a.off_alpha = L->off_alpha;
+    a.off_linv = L->off_linv;
+    a.off_scal = L->off_scal;
+    a.n_obs = L->n;
+    a.d = L->d;
+    a.dp = (L->d + 3) & ~3;
+    a.n_obj = L->n_obj;
+    a.kernel = L->kernel;
+    a.n_rb = L->n_rb;
+    a.n_tiles = L->n_tiles;
+    return SCOOT_OK;
+}
+
+size_t score_smem(const ScoreArgs& a, int epi) {
+    const size_t n_pad = (size_t)a.n_rb * kRB;
+    size_t f = n_pad * kTC + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3)) + n_pad + kCJ * kRB + 8 * kTC;
+    if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
+    return f * 4;
+}
+
+template <int EPI, int M>
+scoot_status launch_score(scoot_ctx* ctx, const ScoreArgs& a, cudaStream_t st) {
+    const size_t smem = score_smem(a, EPI);
+    auto kern = score_kernel<EPI, M>;
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    int per_sm = 0;
+    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kTC, smem));
+    if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "score kernel needs %zu bytes of shared memory", smem);
+    const int64_t tiles = (a.n + kTC - 1) / kTC;
+    int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
+    if (blocks > tiles) blocks = tiles;
+    kern<<<(unsigned)blocks, kTC, smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+scoot_status check_boxes(scoot_ctx* ctx, int M, const float* lo, const float* hi, int32_t B, const float* eps, int32_t S) {
+    if (M < 2 || M > kMaxM) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "EHVI needs 2 <= M <= %d objectives, got %d", kMaxM, M);
+    if (B < 1 || !lo || !hi) return scoot_fail(ctx, SCOOT_EINVAL, "boxes: B = %d, lo/hi must be non-NULL", B);
+    if (S < 1 || !eps) return scoot_fail(ctx, SCOOT_EINVAL, "base samples: S = %d, eps must be non-NULL", S);
+    if ((size_t)(2 * B + S) * 16 > 160 * 1024)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "%d boxes and %d samples exceed the shared-memory budget", B, S);
+    return SCOOT_OK;
+}
+
+template <int EPI>
+scoot_status dispatch_m(scoot_ctx* ctx, const ScoreArgs& a, int M, cudaStream_t st) {
+    switch (M) {
+    case 2: return launch_score<EPI, 2>(ctx, a, st);
+    case 3: return launch_score<EPI, 3>(ctx, a, st);
+    case 4: return launch_score<EPI, 4>(ctx, a, st);
+    default: return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "M = %d", M);
+    }
+}
+
+}  // namespace
+
+extern "C" {
+
+scoot_status scoot_gp_posterior(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                                const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                                float* mean, float* var, int64_t ldo, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    ScoreArgs a;
+    if ((s = fill_state_args(ctx, L, state, a)) != SCOOT_OK) return s;
+    if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!mean || !var || ldo < n) return scoot_fail(ctx, SCOOT_EINVAL, "mean/var NULL or ldo < n");
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.mask = mask;
+    a.mean = mean;
+    a.var = var;
+    a.ldo = ldo;
+    return launch_score<kWriteMoments, 1>(ctx, a, static_cast<cudaStream_t>(stream));
+}
+
+scoot_status scoot_acq_ei(scoot_ctx* ctx, const float* mean, const float* var, const uint8_t* mask,
+                          int64_t n, float y_best, float xi, float* acq, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (n < 0) return scoot_fail(ctx, SCOOT_EINVAL, "n < 0");
+    if (n == 0) return SCOOT_OK;
+    if (!mean || !var || !acq) return scoot_fail(ctx, SCOOT_EINVAL, "mean, var or acq is NULL");
+    int64_t blocks = (n + kAcqThreads - 1) / kAcqThreads;
+    const int64_t cap = (int64_t)sm_count(ctx->device) * 16;
+    if (blocks > cap) blocks = cap;
+    ei_kernel<<<(unsigned)blocks, kAcqThreads, 0, static_cast<cudaStream_t>(stream)>>>(mean, var, mask, n, y_best, xi, acq);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+scoot_status scoot_acq_ehvi(scoot_ctx* ctx, const float* mean, const float* var, int64_t ldm, int32_t n_obj,
+                            const uint8_t* mask, int64_t n, const float* box_lo, const float* box_hi,
+                            int32_t n_boxes, const float* eps, int32_t n_mc, float* acq, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (n < 0) return scoot_fail(ctx, SCOOT_EINVAL, "n < 0");
+    if ((s = check_boxes(ctx, n_obj, box_lo, box_hi, n_boxes, eps, n_mc)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!mean || !var || !acq || ldm < n) return scoot_fail(ctx, SCOOT_EINVAL, "mean/var/acq NULL or ldm < n");
+    ScoreArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.mean = const_cast<float*>(mean);
+    a.var = const_cast<float*>(var);
+    a.ldo = ldm;
+    a.mask = mask;
+    a.n = n;
+    a.acq = acq;
+    a.box_lo = box_lo;
+    a.box_hi = box_hi;
+    a.n_boxes = n_boxes;
+    a.eps = eps;
+    a.n_mc = n_mc;
+    const size_t smem = (size_t)(2 * n_boxes + n_mc) * 16;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int64_t blocks = (n + kAcqThreads - 1) / kAcqThreads;
+    auto go = [&](auto kern) -> scoot_status {
+        SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        int per_sm = 0;
+        SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kAcqThreads, smem));
+        if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "EHVI kernel does not fit");
+        const int64_t cap = (int64_t)sm_count(ctx->device) * per_sm;
+        if (blocks > cap) blocks = cap;
+        kern<<<(unsigned)blocks, kAcqThreads, smem, st>>>(a);
+        SCOOT_LAUNCHED(ctx);
+        return SCOOT_OK;
+    };
+    switch (n_obj) {
+    case 2: return go(ehvi_kernel<2>);
+    case 3: return go(ehvi_kernel<3>);
+    default: return go(ehvi_kernel<4>);
+    }
+}
+
+scoot_status scoot_score_ei(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                            const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                            float xi, float* acq, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    ScoreArgs a;
+    if ((s = fill_state_args(ctx, L, state, a)) != SCOOT_OK) return s;
+    if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!acq) return scoot_fail(ctx, SCOOT_EINVAL, "acq is NULL");
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.mask = mask;
+    a.acq = acq;
+    a.xi = xi;
+    return launch_score<kEI, 1>(ctx, a, static_cast<cudaStream_t>(stream));
+}
+
+scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                              const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                              const float* box_lo, const float* box_hi, int32_t n_boxes,
+                              const float* eps, int32_t n_mc, float* acq, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    ScoreArgs a;
+    if ((s = fill_state_args(ctx, L, state, a)) != SCOOT_OK) return s;
+    if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
+    if ((s = check_boxes(ctx, L->n_obj, box_lo, box_hi, n_boxes, eps, n_mc)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!acq) return scoot_fail(ctx, SCOOT_EINVAL, "acq is NULL");
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.mask = mask;
+    a.acq = acq;
+    a.box_lo = box_lo;
+    a.box_hi = box_hi;
+    a.n_boxes = n_boxes;
+    a.eps = eps;
+    a.n_mc = n_mc;
+    return dispatch_m<kEHVI>(ctx, a, L->n_obj, static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,174 @@
+// Top-q selection for parallel suggestion (Section 4.7): the q largest
+// acquisition values among eligible candidates, ties broken by the lowest
+// index, in two passes.
+//
+// Every eligible candidate i becomes one 64-bit key whose order is the
+// selection order: the high word is the acquisition value mapped to an
+// order-preserving unsigned integer, the low word is 0xFFFFFFFF - i, so a
+// larger key means a larger value or, on equal values, a lower index.
+// Keys are unique, so "the q largest keys" is a single well-defined set.
+//  pass 1: each block keeps, per thread, a sorted register list of its QT
+//          best keys over a contiguous slice of the pool, then extracts the
+//          block's q best by q rounds of a block-wide maximum;
+//  pass 2: one block merges the per-block lists the same way.
+// The per-block lists live in the context's workspace.
+#include "internal.h"
+
+namespace {
+
+constexpr int kTopqThreads = 128;
+constexpr int kMergeThreads = 256;
+
+__device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
+    uint32_t b = __float_as_uint(v);
+    b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return ((uint64_t)b << 32) | (uint64_t)(0xFFFFFFFFu - idx);
+}
+
+__device__ __forceinline__ float key_value(uint64_t k) {
+    uint32_t b = (uint32_t)(k >> 32);
+    b = (b & 0x80000000u) ? (b & 0x7FFFFFFFu) : ~b;
+    return __uint_as_float(b);
+}
+
+__device__ __forceinline__ int64_t key_index(uint64_t k) {
+    return (int64_t)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFu));
+}
+
+template <int QT>
+__device__ __forceinline__ void insert(uint64_t (&lst)[QT], uint64_t x) {
+    if (x <= lst[QT - 1]) return;
+#pragma unroll
+    for (int p = QT - 1; p > 0; --p) {
+        const uint64_t prev = lst[p - 1];
+        lst[p] = x > prev ? prev : (x > lst[p] ? x : lst[p]);
+    }
+    if (x > lst[0]) lst[0] = x;
+}
+
+__device__ __forceinline__ uint64_t warp_max(uint64_t v) {
+    for (int o = 16; o > 0; o >>= 1) {
+        const uint64_t w = __shfl_xor_sync(0xffffffffu, v, o);
+        v = w > v ? w : v;
+    }
+    return v;
+}
+
+// q rounds of a block-wide maximum over the heads of the per-thread sorted
+// lists; the winner pops its head.  Writes at most q keys to out (0 = none).
+template <int QT>
+__device__ void block_extract(uint64_t (&lst)[QT], int q, uint64_t* out) {
+    __shared__ uint64_t wmax[32];
+    __shared__ uint64_t best;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    for (int r = 0; r < q; ++r) {
+        const uint64_t m = warp_max(lst[0]);
+        if (lane == 0) wmax[warp] = m;
+        __syncthreads();
+        if (warp == 0) {
+            uint64_t v = lane < nw ? wmax[lane] : 0ull;
+            v = warp_max(v);
+            if (lane == 0) best = v;
+        }
+        __syncthreads();
+        const uint64_t b = best;
+        if (threadIdx.x == 0) out[r] = b;
+        if (b != 0ull && lst[0] == b) {
+#pragma unroll
+            for (int p = 0; p < QT - 1; ++p) lst[p] = lst[p + 1];
+            lst[QT - 1] = 0ull;
+        }
+        __syncthreads();  // wmax / best are rewritten next round
+    }
+}
+
+template <int QT>
+__global__ void __launch_bounds__(kTopqThreads)
+topq_pass1(const float* __restrict__ acq, const uint8_t* __restrict__ mask, int64_t n, int64_t slice,
+           int q, uint64_t* __restrict__ partial) {
+    uint64_t lst[QT];
+#pragma unroll
+    for (int p = 0; p < QT; ++p) lst[p] = 0ull;
+    const int64_t b0 = (int64_t)blockIdx.x * slice;
+    const int64_t b1 = b0 + slice < n ? b0 + slice : n;
+    for (int64_t i = b0 + threadIdx.x; i < b1; i += blockDim.x) {
+        const float v = acq[i];
+        if ((mask == nullptr || mask[i] != 0) && !(v != v) && v != -INFINITY)
+            insert<QT>(lst, make_key(v, (uint32_t)i));
+    }
+    block_extract<QT>(lst, q, partial + (int64_t)blockIdx.x * q);
+}
+
+template <int QT>
+__global__ void __launch_bounds__(kMergeThreads)
+topq_pass2(const uint64_t* __restrict__ partial, int64_t total, int q, int64_t* __restrict__ idx,
+           float* __restrict__ val, int32_t* __restrict__ count) {
+    __shared__ uint64_t result[SCOOT_MAX_Q];
+    uint64_t lst[QT];
+#pragma unroll
+    for (int p = 0; p < QT; ++p) lst[p] = 0ull;
+    for (int64_t k = threadIdx.x; k < total; k += blockDim.x) {
+        const uint64_t x = partial[k];
+        if (x) insert<QT>(lst, x);
+    }
+    block_extract<QT>(lst, q, result);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int c = 0;
+        for (int r = 0; r < q; ++r) {
+            const uint64_t k = result[r];
+            if (k) {
+                idx[r] = key_index(k);
+                val[r] = key_value(k);
+                ++c;
+            } else {
+                idx[r] = -1;
+                val[r] = -INFINITY;
+            }
+        }
+        *count = c;
+    }
+}
+
+int sm_count(int device) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, device);
+    return v > 0 ? v : 1;
+}
+
+template <int QT>
+scoot_status run(scoot_ctx* ctx, const float* acq, const uint8_t* mask, int64_t n, int q, int64_t* idx,
+                 float* val, int32_t* count, cudaStream_t st) {
+    // One slice per block; at least 8 keys per thread, at most 4 blocks per SM.
+    int64_t blocks = (n + kTopqThreads * 8 - 1) / (kTopqThreads * 8);
+    const int64_t cap = (int64_t)sm_count(ctx->device) * 4;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    const int64_t slice = (n + blocks - 1) / blocks;
+    scoot_status s = scoot_workspace(ctx, (size_t)blocks * q * sizeof(uint64_t));
+    if (s != SCOOT_OK) return s;
+    uint64_t* partial = static_cast<uint64_t*>(ctx->ws);
+    topq_pass1<QT><<<(unsigned)blocks, kTopqThreads, 0, st>>>(acq, mask, n, slice, q, partial);
+    SCOOT_LAUNCHED(ctx);
+    topq_pass2<QT><<<1, kMergeThreads, 0, st>>>(partial, blocks * q, q, idx, val, count);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+}  // namespace
+
+extern "C" scoot_status scoot_select_topq(scoot_ctx* ctx, const float* acq, const uint8_t* mask, int64_t n,
+                                          int32_t q, int64_t* idx, float* val, int32_t* count,
+                                          void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (q < 1 || q > SCOOT_MAX_Q) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "q = %d outside 1..%d", q, SCOOT_MAX_Q);
+    if (n < 0) return scoot_fail(ctx, SCOOT_EINVAL, "n < 0");
+    if (n > 0xFFFFFFFFll) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n = %lld >= 2^32", (long long)n);
+    if (!idx || !val || !count || (n > 0 && !acq)) return scoot_fail(ctx, SCOOT_EINVAL, "NULL output or input");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (q <= 1) return run<1>(ctx, acq, mask, n, q, idx, val, count, st);
+    if (q <= 4) return run<4>(ctx, acq, mask, n, q, idx, val, count, st);
+    if (q <= 16) return run<16>(ctx, acq, mask, n, q, idx, val, count, st);
+    return run<64>(ctx, acq, mask, n, q, idx, val, count, st);
+}

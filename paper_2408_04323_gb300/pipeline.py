@@ -1,0 +1,104 @@
+"""One suggestion round through the C ABI: prune -> forest -> posterior +
+acquisition -> top-q (Section 4, Algorithm 1's SUGGEST step).
+
+Host-side state (GP factor, box decomposition, packed forest) is prepared by
+the library's own host functions; torch only holds device memory and
+streams.  Nothing here computes any step of the path itself.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+from . import scoot as S
+
+
+@dataclass
+class RoundInputs:
+    """Host arrays describing one round (layouts as in include/scoot.h)."""
+    space: np.ndarray          # scoot_param[d]
+    clauses: np.ndarray        # scoot_clause[n_clauses]
+    nodes: np.ndarray          # scoot_node[total]
+    tree_offset: np.ndarray    # int32[T+1]
+    leaf_scale: int
+    delta_num: int
+    delta_den: int
+    x_obs: np.ndarray          # uint32[d][n]
+    y_obs: np.ndarray          # float32[M][n]
+    lengthscale: np.ndarray    # float32[M][d]
+    signal_var: np.ndarray     # float32[M]
+    noise_var: np.ndarray      # float32[M]
+    ref: np.ndarray            # float32[M]
+    eps: np.ndarray            # float32[S][M]
+    acq: str                   # "ei" or "ehvi"
+    q: int
+    kernel: int = S.MATERN52
+    xi: float = 1e-4
+
+
+class State:
+    """Per-round state prepared on the host and copied to the device."""
+
+    def __init__(self, inp: RoundInputs, device: torch.device):
+        d = len(inp.space)
+        M = inp.y_obs.shape[0]
+        self.gp_layout = S.scoot_gp_layout_init(inp.y_obs.shape[1], d, M, inp.kernel)
+        blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                             inp.signal_var, inp.noise_var, self.gp_layout)
+        self.forest_layout = S.scoot_forest_layout_init(inp.nodes, inp.tree_offset, d, inp.leaf_scale)
+        fblob = S.scoot_forest_pack(self.forest_layout, inp.nodes, inp.tree_offset)
+        self.h_blobs = (blob, fblob)
+        self.gp_state = torch.from_numpy(blob).to(device)
+        self.forest = torch.from_numpy(fblob).to(device)
+        self.n_boxes = 0
+        self.front_size = 0
+        if inp.acq == "ehvi":
+            lo, hi, self.front_size = S.scoot_boxes_build(inp.y_obs, inp.ref)
+            self.n_boxes = len(lo)
+            self.h_boxes = (lo, hi)
+            self.box_lo = torch.from_numpy(lo).to(device)
+            self.box_hi = torch.from_numpy(hi).to(device)
+            self.eps = torch.from_numpy(np.ascontiguousarray(inp.eps, np.float32)).to(device)
+
+
+class ScoringRound:
+    """Device buffers for pools of up to `capacity` candidates and the calls of one round."""
+
+    def __init__(self, ctx: S.Context, inp: RoundInputs, capacity: int, device=None):
+        self.ctx = ctx
+        self.inp = inp
+        self.device = torch.device("cuda", ctx.device) if device is None else torch.device(device)
+        self.state = State(inp, self.device)
+        self.capacity = int(capacity)
+        dev = self.device
+        self.mask = torch.empty(self.capacity, dtype=torch.uint8, device=dev)
+        self.votes = torch.empty(self.capacity, dtype=torch.int32, device=dev)
+        self.acq = torch.empty(self.capacity, dtype=torch.float32, device=dev)
+        self.n_known = torch.zeros(1, dtype=torch.int64, device=dev)
+        self.n_feasible = torch.zeros(1, dtype=torch.int64, device=dev)
+        q = inp.q
+        self.top_idx = torch.empty(q, dtype=torch.int64, device=dev)
+        self.top_val = torch.empty(q, dtype=torch.float32, device=dev)
+        self.top_count = torch.empty(1, dtype=torch.int32, device=dev)
+
+    # number of library kernels one call of run() launches
+    KERNELS_PER_ROUND = 5
+
+    def run(self, cand: torch.Tensor, n: int, stream=None):
+        """prune -> rf -> score -> top-q on a resident pool cand (int32 [d][ld])."""
+        if n > self.capacity:
+            raise ValueError("pool larger than the round's capacity")
+        inp, st = self.inp, self.state
+        S.scoot_prune(self.ctx, inp.space, inp.clauses, cand, n, self.mask, self.n_known, stream)
+        S.scoot_rf_predict(self.ctx, st.forest_layout, st.forest, inp.space, cand, n, inp.delta_num,
+                           inp.delta_den, self.votes, self.mask, self.n_feasible, stream)
+        if inp.acq == "ei":
+            S.scoot_score_ei(self.ctx, st.gp_layout, st.gp_state, cand, n, inp.xi, self.acq, self.mask, stream)
+        else:
+            S.scoot_score_ehvi(self.ctx, st.gp_layout, st.gp_state, cand, n, st.box_lo, st.box_hi, st.eps,
+                               self.acq, self.mask, stream)
+        S.scoot_select_topq(self.ctx, self.acq, n, inp.q, self.top_idx, self.top_val, self.top_count,
+                            self.mask, stream)
+        return self.top_idx, self.top_val, self.top_count

@@ -1,0 +1,332 @@
+"""ctypes binding of libscoot (include/scoot.h): argument marshalling only.
+
+Every function here has the name of the C entry point it calls and does no
+arithmetic of its own: host arrays are numpy arrays (passed by pointer),
+device arrays are CUDA torch tensors (passed by data pointer), streams are
+torch CUDA streams (passed by handle).  A non-zero status raises ScootError
+with the library's message.  If libscoot.so has not been built, importing
+the functions raises ImportError: there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libscoot.so")
+
+INT_UNIFORM, INT_LOG, CATEGORICAL, CONTINUOUS = 0, 1, 2, 3
+MATERN52, MATERN32 = 0, 1
+MAX_DIM, MAX_CLAUSES, MAX_OBJ, MAX_OBS, MAX_Q = 16, 16, 4, 1024, 64
+
+STATUS = {0: "SCOOT_OK", -1: "SCOOT_EINVAL", -2: "SCOOT_ENOMEM", -3: "SCOOT_ECUDA",
+          -4: "SCOOT_EDEVICE", -5: "SCOOT_ETIMEOUT", -6: "SCOOT_EUNSUPPORTED"}
+
+
+class ScootError(RuntimeError):
+    def __init__(self, status: int, func: str, message: str = ""):
+        self.status = status
+        super().__init__(f"{func}: {STATUS.get(status, status)} {message}".rstrip())
+
+
+class scoot_param(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("n_choices", C.c_int32), ("lo", C.c_float), ("hi", C.c_float)]
+
+
+class scoot_clause(C.Structure):
+    _fields_ = [("n_guard", C.c_int32), ("guard_param", C.c_int32 * 2), ("guard_value", C.c_int32 * 2),
+                ("n_term", C.c_int32), ("term_param", C.c_int32 * 4), ("coef", C.c_int64 * 4),
+                ("rhs", C.c_int64)]
+
+
+class scoot_node(C.Structure):
+    _fields_ = [("val", C.c_float), ("left", C.c_uint16), ("feat", C.c_uint8), ("flags", C.c_uint8)]
+
+
+class scoot_forest_layout(C.Structure):
+    _fields_ = [("n_trees", C.c_int32), ("n_nodes", C.c_int32), ("d", C.c_int32), ("leaf_scale", C.c_int32),
+                ("max_depth", C.c_int32), ("n_chunks", C.c_int32), ("max_chunk_nodes", C.c_int32),
+                ("reserved", C.c_int32), ("bytes", C.c_int64), ("off_chunks", C.c_int64),
+                ("off_roots", C.c_int64), ("off_nodes", C.c_int64)]
+
+
+class scoot_gp_layout(C.Structure):
+    _fields_ = [("n", C.c_int32), ("d", C.c_int32), ("n_obj", C.c_int32), ("kernel", C.c_int32),
+                ("n_rb", C.c_int32), ("n_tiles", C.c_int32), ("bytes", C.c_int64),
+                ("off_fmap", C.c_int64), ("off_xs", C.c_int64), ("off_ils", C.c_int64),
+                ("off_alpha", C.c_int64), ("off_linv", C.c_int64), ("off_scal", C.c_int64)]
+
+
+assert C.sizeof(scoot_param) == 16 and C.sizeof(scoot_clause) == 80 and C.sizeof(scoot_node) == 8
+
+_vp, _i32, _i64, _u32, _f32 = C.c_void_p, C.c_int32, C.c_int64, C.c_uint32, C.c_float
+_PROTOS = {
+    "scoot_ctx_create": [_i32, C.POINTER(_vp)],
+    "scoot_ctx_destroy": [_vp],
+    "scoot_last_error": [_vp],
+    "scoot_status_string": [_i32],
+    "scoot_ctx_check": [_vp, _vp],
+    "scoot_ctx_workspace_bytes": [_vp, C.POINTER(_i64)],
+    "scoot_prune": [_vp, _vp, _i32, _vp, _i32, _vp, _i64, _i64, _vp, _vp, _vp],
+    "scoot_forest_layout_init": [_vp, _vp, _i32, _i32, _i32, C.POINTER(scoot_forest_layout)],
+    "scoot_forest_pack": [C.POINTER(scoot_forest_layout), _vp, _vp, _vp],
+    "scoot_rf_predict": [_vp, C.POINTER(scoot_forest_layout), _vp, _vp, _vp, _i64, _i64, _u32, _u32,
+                         _vp, _vp, _vp, _vp],
+    "scoot_gp_layout_init": [_i32, _i32, _i32, _i32, C.POINTER(scoot_gp_layout)],
+    "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
+    "scoot_gp_posterior": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i64, _vp],
+    "scoot_acq_ei": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp],
+    "scoot_boxes_build": [_vp, _i32, _i32, _vp, _i32, _vp, _vp, C.POINTER(_i32), C.POINTER(_i32)],
+    "scoot_acq_ehvi": [_vp, _vp, _vp, _i64, _i32, _vp, _i64, _vp, _vp, _i32, _vp, _i32, _vp, _vp],
+    "scoot_score_ei": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _f32, _vp, _vp],
+    "scoot_score_ehvi": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i32,
+                         _vp, _i32, _vp, _vp],
+    "scoot_select_topq": [_vp, _vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
+}
+_STRING_FUNCS = {"scoot_last_error", "scoot_status_string"}
+EXPORTS = tuple(_PROTOS)
+
+_lib = None
+
+
+def lib() -> C.CDLL:
+    """The loaded libscoot.so (ImportError if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"{LIB_PATH} is missing: build it with paper_2408_04323_gb300.build()")
+        L = C.CDLL(LIB_PATH)
+        for name, args in _PROTOS.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = C.c_char_p if name in _STRING_FUNCS else _i32
+        _lib = L
+    return _lib
+
+
+# ------------------------------------------------------------------ marshalling
+
+def _host(a, itemsize=None, dtype=None, name="array"):
+    if a is None:
+        return None
+    if not isinstance(a, np.ndarray):
+        raise TypeError(f"{name} must be a numpy array (host memory)")
+    if not a.flags.c_contiguous:
+        raise ValueError(f"{name} must be C-contiguous")
+    if dtype is not None and a.dtype != np.dtype(dtype):
+        raise TypeError(f"{name} must have dtype {np.dtype(dtype)}, got {a.dtype}")
+    if itemsize is not None and a.dtype.itemsize != itemsize:
+        raise TypeError(f"{name} items must be {itemsize} bytes, got {a.dtype.itemsize}")
+    return a.ctypes.data_as(_vp)
+
+
+def _dev(t, dtype=None, name="tensor"):
+    if t is None:
+        return None
+    import torch
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA torch tensor (device memory)")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must have dtype {dtype}, got {t.dtype}")
+    return _vp(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return _vp(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _check(status, func, ctx=None):
+    if status != 0:
+        msg = ""
+        if ctx is not None:
+            raw = lib().scoot_last_error(ctx)
+            msg = raw.decode() if raw else ""
+        raise ScootError(int(status), func, msg)
+
+
+# ------------------------------------------------------------------ context
+
+def scoot_ctx_create(device: int = 0) -> C.c_void_p:
+    h = _vp()
+    _check(lib().scoot_ctx_create(int(device), C.byref(h)), "scoot_ctx_create")
+    return h
+
+
+def scoot_ctx_destroy(ctx) -> None:
+    _check(lib().scoot_ctx_destroy(ctx), "scoot_ctx_destroy")
+
+
+def scoot_ctx_check(ctx, stream=None) -> None:
+    _check(lib().scoot_ctx_check(ctx, _stream(stream)), "scoot_ctx_check", ctx)
+
+
+def scoot_ctx_workspace_bytes(ctx) -> int:
+    v = _i64()
+    _check(lib().scoot_ctx_workspace_bytes(ctx, C.byref(v)), "scoot_ctx_workspace_bytes")
+    return int(v.value)
+
+
+def scoot_status_string(status: int) -> str:
+    return lib().scoot_status_string(int(status)).decode()
+
+
+class Context:
+    """A scoot_ctx bound to one CUDA device."""
+
+    def __init__(self, device: int = 0):
+        self.device = int(device)
+        self.handle = scoot_ctx_create(self.device)
+
+    def close(self):
+        if self.handle:
+            scoot_ctx_destroy(self.handle)
+            self.handle = None
+
+    def check(self, stream=None):
+        scoot_ctx_check(self.handle, stream)
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def _h(ctx):
+    return ctx.handle if isinstance(ctx, Context) else ctx
+
+
+# ------------------------------------------------------------------ host-side preparation
+
+def scoot_gp_layout_init(n: int, d: int, n_obj: int, kernel: int = MATERN52) -> scoot_gp_layout:
+    L = scoot_gp_layout()
+    _check(lib().scoot_gp_layout_init(int(n), int(d), int(n_obj), int(kernel), C.byref(L)), "scoot_gp_layout_init")
+    return L
+
+
+def scoot_gp_prepare(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, layout):
+    """Returns (host blob uint8[layout.bytes], cond float64[M])."""
+    blob = np.zeros(layout.bytes, np.uint8)
+    cond = np.zeros(layout.n_obj, np.float64)
+    _check(lib().scoot_gp_prepare(_host(h_space, 16, name="h_space"), _host(h_x_obs, 4, name="h_x_obs"),
+                                  int(h_x_obs.shape[1]), _host(h_y, dtype=np.float32, name="h_y"),
+                                  _host(h_lengthscale, dtype=np.float32, name="h_lengthscale"),
+                                  _host(h_signal_var, dtype=np.float32, name="h_signal_var"),
+                                  _host(h_noise_var, dtype=np.float32, name="h_noise_var"),
+                                  C.byref(layout), _host(blob), _host(cond)), "scoot_gp_prepare")
+    return blob, cond
+
+
+def scoot_forest_layout_init(h_nodes, h_tree_offset, d: int, leaf_scale: int) -> scoot_forest_layout:
+    L = scoot_forest_layout()
+    _check(lib().scoot_forest_layout_init(_host(h_nodes, 8, name="h_nodes"),
+                                          _host(h_tree_offset, dtype=np.int32, name="h_tree_offset"),
+                                          int(len(h_tree_offset) - 1), int(d), int(leaf_scale), C.byref(L)),
+           "scoot_forest_layout_init")
+    return L
+
+
+def scoot_forest_pack(layout, h_nodes, h_tree_offset) -> np.ndarray:
+    blob = np.zeros(layout.bytes, np.uint8)
+    _check(lib().scoot_forest_pack(C.byref(layout), _host(h_nodes, 8, name="h_nodes"),
+                                   _host(h_tree_offset, dtype=np.int32, name="h_tree_offset"), _host(blob)),
+           "scoot_forest_pack")
+    return blob
+
+
+def scoot_boxes_build(h_y, h_ref, cap: int = 4096):
+    """h_y float32 [M][n_pts], h_ref float32 [M] -> (lo [B][M], hi [B][M], front_size)."""
+    M, n_pts = h_y.shape
+    lo = np.zeros((max(cap, 1), M), np.float32)
+    hi = np.zeros((max(cap, 1), M), np.float32)
+    nb, fs = _i32(), _i32()
+    _check(lib().scoot_boxes_build(_host(h_y, dtype=np.float32, name="h_y"), int(n_pts), int(M),
+                                   _host(h_ref, dtype=np.float32, name="h_ref"), int(cap), _host(lo), _host(hi),
+                                   C.byref(nb), C.byref(fs)), "scoot_boxes_build")
+    return lo[:nb.value].copy(), hi[:nb.value].copy(), int(fs.value)
+
+
+# ------------------------------------------------------------------ device calls
+
+def scoot_prune(ctx, h_space, h_clauses, cand, n, mask, n_feasible=None, stream=None):
+    import torch
+    _check(lib().scoot_prune(_h(ctx), _host(h_space, 16, name="h_space"), int(len(h_space)),
+                             _host(h_clauses, 80, name="h_clauses"), int(len(h_clauses)),
+                             _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]),
+                             _dev(mask, torch.uint8, "mask"), _dev(n_feasible, torch.int64, "n_feasible"),
+                             _stream(stream)), "scoot_prune", _h(ctx))
+
+
+def scoot_rf_predict(ctx, layout, forest, h_space, cand, n, delta_num, delta_den, votes, mask=None,
+                     n_feasible=None, stream=None):
+    import torch
+    _check(lib().scoot_rf_predict(_h(ctx), C.byref(layout), _dev(forest, torch.uint8, "forest"),
+                                  _host(h_space, 16, name="h_space"), _dev(cand, torch.int32, "cand"),
+                                  int(n), int(cand.shape[1]), int(delta_num), int(delta_den),
+                                  _dev(votes, torch.int32, "votes"), _dev(mask, torch.uint8, "mask"),
+                                  _dev(n_feasible, torch.int64, "n_feasible"), _stream(stream)),
+           "scoot_rf_predict", _h(ctx))
+
+
+def scoot_gp_posterior(ctx, layout, state, cand, n, mean, var, mask=None, stream=None):
+    import torch
+    _check(lib().scoot_gp_posterior(_h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"),
+                                    _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]),
+                                    _dev(mask, torch.uint8, "mask"), _dev(mean, torch.float32, "mean"),
+                                    _dev(var, torch.float32, "var"), int(mean.shape[-1]), _stream(stream)),
+           "scoot_gp_posterior", _h(ctx))
+
+
+def scoot_acq_ei(ctx, mean, var, n, y_best, xi, acq, mask=None, stream=None):
+    import torch
+    _check(lib().scoot_acq_ei(_h(ctx), _dev(mean, torch.float32, "mean"), _dev(var, torch.float32, "var"),
+                              _dev(mask, torch.uint8, "mask"), int(n), float(y_best), float(xi),
+                              _dev(acq, torch.float32, "acq"), _stream(stream)), "scoot_acq_ei", _h(ctx))
+
+
+def scoot_acq_ehvi(ctx, mean, var, n, box_lo, box_hi, eps, acq, mask=None, stream=None):
+    import torch
+    M = int(mean.shape[0])
+    _check(lib().scoot_acq_ehvi(_h(ctx), _dev(mean, torch.float32, "mean"), _dev(var, torch.float32, "var"),
+                                int(mean.shape[1]), M, _dev(mask, torch.uint8, "mask"), int(n),
+                                _dev(box_lo, torch.float32, "box_lo"), _dev(box_hi, torch.float32, "box_hi"),
+                                int(box_lo.shape[0]), _dev(eps, torch.float32, "eps"), int(eps.shape[0]),
+                                _dev(acq, torch.float32, "acq"), _stream(stream)), "scoot_acq_ehvi", _h(ctx))
+
+
+def scoot_score_ei(ctx, layout, state, cand, n, xi, acq, mask=None, stream=None):
+    import torch
+    _check(lib().scoot_score_ei(_h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"),
+                                _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]),
+                                _dev(mask, torch.uint8, "mask"), float(xi), _dev(acq, torch.float32, "acq"),
+                                _stream(stream)), "scoot_score_ei", _h(ctx))
+
+
+def scoot_score_ehvi(ctx, layout, state, cand, n, box_lo, box_hi, eps, acq, mask=None, stream=None):
+    import torch
+    _check(lib().scoot_score_ehvi(_h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"),
+                                  _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]),
+                                  _dev(mask, torch.uint8, "mask"), _dev(box_lo, torch.float32, "box_lo"),
+                                  _dev(box_hi, torch.float32, "box_hi"), int(box_lo.shape[0]),
+                                  _dev(eps, torch.float32, "eps"), int(eps.shape[0]),
+                                  _dev(acq, torch.float32, "acq"), _stream(stream)), "scoot_score_ehvi", _h(ctx))
+
+
+def scoot_select_topq(ctx, acq, n, q, idx, val, count, mask=None, stream=None):
+    import torch
+    _check(lib().scoot_select_topq(_h(ctx), _dev(acq, torch.float32, "acq"), _dev(mask, torch.uint8, "mask"),
+                                   int(n), int(q), _dev(idx, torch.int64, "idx"), _dev(val, torch.float32, "val"),
+                                   _dev(count, torch.int32, "count"), _stream(stream)), "scoot_select_topq", _h(ctx))

@@ -1,0 +1,394 @@
+"""Parity of the CUDA path with the fp64 oracle, through the C ABI.
+
+Bars: bit-exact for masks, vote counts and selected indices; for floating
+point |gpu - oracle| <= 1e-6 + 1e-4 |oracle| (posterior variance, EI, EHVI).
+The posterior mean additionally gets 2^-22 * sum_j |k_j alpha_j|, the
+rounding scale of any fp32 evaluation of the dot product mu = k . alpha
+(it matters only where mu crosses zero).
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle as O
+from workloads import Stream, make_instance, seeds
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+ATOL, RTOL = 1e-6, 1e-4
+MU_COND = 2.0 ** -22
+
+
+@pytest.fixture(scope="module")
+def S():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2408_04323_gb300 as pkg
+    pkg.build()
+    from paper_2408_04323_gb300 import scoot
+    return scoot
+
+
+@pytest.fixture(scope="module")
+def ctx(S):
+    c = S.Context(0)
+    yield c
+    c.close()
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def cand_dev(inst):
+    return dev(inst.cand.view(np.int32))
+
+
+def np_(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+def report(name, g, o, extra=0.0):
+    g = np.asarray(g, np.float64)
+    o = np.asarray(o, np.float64)
+    tol = ATOL + RTOL * np.abs(o) + extra
+    ratio = np.abs(g - o) / tol
+    worst = float(ratio.max()) if ratio.size else 0.0
+    print(f"[parity] {name}: n={g.size} max|err|/tol={worst:.3f} max|err|={np.abs(g - o).max() if g.size else 0:.3e}")
+    return ratio
+
+
+def sample_idx(n, k, seed):
+    if n <= k:
+        return np.arange(n)
+    st = Stream(seed, "sample")
+    return np.unique(st.integers(0, n - 1, k))
+
+
+POOL = {"tiny": 4096, "d8-ehvi2": 1 << 18, "d10-ei": 1 << 20, "d10-ehvi3": 1 << 20, "d12-fantasy": 1 << 22}
+NAMES = list(POOL)
+
+
+# ------------------------------------------------------------------ prune, Eq. (2)
+
+@pytest.mark.parametrize("name", NAMES)
+def test_prune_bit_exact_full_pool(S, ctx, name):
+    inst = make_instance(name, seeds(name)[0])
+    n = inst.n_cand
+    mask = torch.full((n,), 7, dtype=torch.uint8, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int64, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses, cand_dev(inst), n, mask, cnt)
+    got = np_(mask)
+    want = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
+    assert np.array_equal(got, want.astype(np.uint8))
+    assert int(np_(cnt)[0]) == int(want.sum())
+    ctx.check()
+
+
+def test_prune_edge_cases(S, ctx):
+    inst = make_instance("d10-ei", seeds("d10-ei")[1], n_cand=1037)
+    want = O.prune_mask(inst.space, inst.clauses, inst.cand, 1037).astype(np.uint8)
+    cand = cand_dev(inst)
+    for n in (0, 1, 2, 3, 5, 1037):
+        buf = torch.full((1040,), 9, dtype=torch.uint8, device="cuda")
+        mask = buf[1:1 + max(n, 1)]  # deliberately not 4-byte aligned
+        cnt = torch.full((1,), 123, dtype=torch.int64, device="cuda")
+        S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask, cnt)
+        got = np_(buf)
+        assert np.array_equal(got[1:1 + n], want[:n]) and got[0] == 9 and np.all(got[1 + n:] == 9)
+        assert int(np_(cnt)[0]) == int(want[:n].sum())
+    # no clauses: everything feasible
+    mask = torch.zeros(1037, dtype=torch.uint8, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses[:0], cand, 1037, mask)
+    assert np_(mask).all()
+
+
+def test_prune_rejects_bad_arguments(S, ctx):
+    inst = make_instance("tiny", 1001, n_cand=64)
+    cand = cand_dev(inst)
+    mask = torch.zeros(64, dtype=torch.uint8, device="cuda")
+    with pytest.raises(S.ScootError) as e:  # ld not a multiple of 4
+        S.scoot_prune(ctx, inst.space, inst.clauses, cand[:, :63].contiguous(), 63, mask)
+    assert e.value.status == -1
+    bad = inst.clauses.copy()
+    bad[0]["term_param"][0] = 3  # a continuous parameter in a clause
+    with pytest.raises(S.ScootError):
+        S.scoot_prune(ctx, inst.space, bad, cand, 64, mask)
+    big = torch.zeros((inst.d, 68), dtype=torch.int32, device="cuda")
+    with pytest.raises(S.ScootError):  # ld < n
+        S.scoot_prune(ctx, inst.space, inst.clauses, big[:, :64].contiguous(), 65, mask)
+
+
+# ------------------------------------------------------------------ forest, Eq. (3)
+
+def forest_dev(S, inst):
+    L = S.scoot_forest_layout_init(inst.nodes, inst.tree_offset, inst.d, inst.workload.leaf_scale)
+    return L, dev(S.scoot_forest_pack(L, inst.nodes, inst.tree_offset))
+
+
+@pytest.mark.parametrize("name", NAMES)
+def test_rf_votes_bit_exact(S, ctx, name):
+    n = POOL[name] if name != "d12-fantasy" else 1 << 18
+    inst = make_instance(name, seeds(name)[0], n_cand=n)
+    w = inst.workload
+    L, forest = forest_dev(S, inst)
+    cand = cand_dev(inst)
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
+    votes = torch.full((n,), -1, dtype=torch.int32, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int64, device="cuda")
+    S.scoot_rf_predict(ctx, L, forest, inst.space, cand, n, w.delta_num, w.delta_den, votes, mask, cnt)
+    ctx.check()
+    known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
+    want_votes = O.rf_votes(inst.nodes, inst.tree_offset, inst.space, inst.cand, n)
+    got_votes = np_(votes).astype(np.int64)
+    assert np.array_equal(got_votes[known], want_votes[known])
+    assert np.all(got_votes[~known] == 0)
+    feas = known & O.pof_feasible(want_votes, inst.n_trees, w.leaf_scale, w.delta_num, w.delta_den)
+    assert np.array_equal(np_(mask).astype(bool), feas)
+    assert int(np_(cnt)[0]) == int(feas.sum())
+    # without a mask every candidate is walked
+    S.scoot_rf_predict(ctx, L, forest, inst.space, cand, n, w.delta_num, w.delta_den, votes, None)
+    assert np.array_equal(np_(votes).astype(np.int64), want_votes)
+
+
+def test_rf_multi_chunk_forest(S, ctx):
+    """A forest too large for one shared-memory chunk gives the same votes."""
+    inst = make_instance("d12-fantasy", seeds("d12-fantasy")[1], n_cand=20000)
+    reps = 4
+    nodes = np.concatenate([inst.nodes] * reps)
+    offs = np.zeros(inst.n_trees * reps + 1, np.int32)
+    offs[1:] = np.cumsum(np.tile(np.diff(inst.tree_offset), reps))
+    L = S.scoot_forest_layout_init(nodes, offs, inst.d, 255)
+    assert L.n_chunks >= 2
+    forest = dev(S.scoot_forest_pack(L, nodes, offs))
+    votes = torch.empty(inst.n_cand, dtype=torch.int32, device="cuda")
+    S.scoot_rf_predict(ctx, L, forest, inst.space, cand_dev(inst), inst.n_cand, 10, 20, votes, None)
+    want = O.rf_votes(nodes, offs, inst.space, inst.cand, inst.n_cand)
+    assert np.array_equal(np_(votes).astype(np.int64), want)
+
+
+# ------------------------------------------------------------------ GP posterior (Section 4.3)
+
+def gp_state(S, inst, kernel=0):
+    L = S.scoot_gp_layout_init(inst.n_obs, inst.d, inst.n_obj, kernel)
+    blob, _ = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
+                                 inst.signal_var, inst.noise_var, L)
+    return L, dev(blob)
+
+
+def oracle_gps(inst, kernel=0):
+    return [O.GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m], inst.signal_var[m],
+                 inst.noise_var[m], kernel) for m in range(inst.n_obj)]
+
+
+@pytest.mark.parametrize("name,kernel", [("tiny", 0), ("d8-ehvi2", 0), ("d10-ei", 0), ("d10-ehvi3", 0),
+                                         ("d12-fantasy", 0), ("d8-ehvi2", 1)])
+def test_posterior_parity(S, ctx, name, kernel):
+    n = 4096 + 37  # several tiles and a ragged tail
+    inst = make_instance(name, seeds(name)[1], n_cand=n)
+    L, state = gp_state(S, inst, kernel)
+    M = inst.n_obj
+    ldo = n + 3
+    mean = torch.full((M, ldo), 77.0, device="cuda")
+    var = torch.full((M, ldo), 77.0, device="cuda")
+    S.scoot_gp_posterior(ctx, L, state, cand_dev(inst), n, mean, var)
+    gm, gv = np_(mean), np_(var)
+    assert np.all(gm[:, n:] == 77.0) and np.all(gv[:, n:] == 77.0)
+    for m, gp in enumerate(oracle_gps(inst, kernel)):
+        mu, v = gp.posterior(inst.cand, n)
+        cond = gp.mean_condition(inst.cand, n)
+        r_mu = report(f"{name} k{kernel} mu[{m}]", gm[m, :n], mu, MU_COND * cond)
+        r_mu_plain = report(f"{name} k{kernel} mu[{m}] (stated tol only)", gm[m, :n], mu)
+        r_v = report(f"{name} k{kernel} var[{m}]", gv[m, :n], v)
+        print(f"[parity] {name} mu[{m}] beyond stated tol: {int((r_mu_plain > 1).sum())} of {n}")
+        assert r_mu.max() <= 1.0
+        assert r_v.max() <= 1.0
+        assert np.all(gv[m, :n] >= 0) and np.all(gv[m, :n] <= inst.signal_var[m] * (1 + 1e-6))
+
+
+def test_posterior_mask_skips(S, ctx):
+    inst = make_instance("d8-ehvi2", seeds("d8-ehvi2")[2], n_cand=999)
+    L, state = gp_state(S, inst)
+    maskh = (Stream(5, "m").uniform(999) < 0.5).astype(np.uint8)
+    mean = torch.full((2, 999), 5.0, device="cuda")
+    var = torch.full((2, 999), 5.0, device="cuda")
+    S.scoot_gp_posterior(ctx, L, state, cand_dev(inst), 999, mean, var, dev(maskh))
+    gm = np_(mean)
+    assert np.all(gm[:, maskh == 0] == 5.0) and np.all(gm[:, maskh == 1] != 5.0)
+
+
+# ------------------------------------------------------------------ acquisition
+
+def test_ei_kernel_on_generated_moments(S, ctx):
+    """Eq. (6) on seeded (mu, sigma^2) arrays, including sigma = 0 and far tails."""
+    st = Stream(21, "ei")
+    n = 50000
+    mu = (st.normal(n) * 1.5).astype(np.float32)
+    var = (st.uniform(n) ** 3).astype(np.float32)
+    var[:100] = 0.0
+    var[100:200] = 1e-30
+    mask = (st.uniform(n) < 0.9).astype(np.uint8)
+    acq = torch.empty(n, device="cuda")
+    S.scoot_acq_ei(ctx, dev(mu), dev(var), n, 0.7, 1e-4, acq, dev(mask))
+    g = np_(acq)
+    want = O.expected_improvement(mu.astype(np.float64), var.astype(np.float64), 0.7, 1e-4)
+    assert np.all(g[mask == 0] == -np.inf)
+    assert report("ei kernel", g[mask == 1], want[mask == 1]).max() <= 1.0
+
+
+@pytest.mark.parametrize("M,nf", [(2, 1), (2, 9), (3, 14), (4, 6)])
+def test_ehvi_kernel_on_generated_moments(S, ctx, M, nf):
+    """Eq. (7) on seeded moments and a seeded front (boxes from the library, cells from the oracle)."""
+    st = Stream(30 + M * 10 + nf, "ehvi")
+    Y = (st.uniform(M * nf).reshape(M, nf) * 2.0).astype(np.float32)
+    ref = np.zeros(M, np.float32)
+    lo, hi, fs = S.scoot_boxes_build(Y, ref)
+    n, Sm = 3001, 48
+    mu = (st.uniform(n * M).reshape(M, n) * 2.4 - 0.2).astype(np.float32)
+    var = (st.uniform(n * M).reshape(M, n) * 0.3).astype(np.float32)
+    var[:, :50] = 0.0
+    eps = st.normal(Sm * M).reshape(Sm, M).astype(np.float32)
+    acq = torch.empty(n, device="cuda")
+    S.scoot_acq_ehvi(ctx, dev(mu), dev(var), n, dev(lo), dev(hi), dev(eps), acq)
+    g = np_(acq)
+    front = O.pareto_front(Y.T, ref)
+    want = O.ehvi_mc(mu.T.astype(np.float64), var.T.astype(np.float64), eps, front, ref)
+    assert report(f"ehvi kernel M={M} P={fs}", g, want).max() <= 1.0
+
+
+def ehvi_inputs(S, inst):
+    lo, hi, fs = S.scoot_boxes_build(inst.y_obs, inst.ref)
+    return dev(lo), dev(hi), dev(inst.eps), fs
+
+
+@pytest.mark.parametrize("name,k", [("tiny", 4096), ("d8-ehvi2", 1024), ("d10-ehvi3", 96), ("d12-fantasy", 384)])
+def test_score_ehvi_parity(S, ctx, name, k):
+    inst = make_instance(name, seeds(name)[0])
+    n = inst.n_cand
+    L, state = gp_state(S, inst)
+    lo, hi, eps, fs = ehvi_inputs(S, inst)
+    cand = cand_dev(inst)
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
+    acq = torch.empty(n, device="cuda")
+    S.scoot_score_ehvi(ctx, L, state, cand, n, lo, hi, eps, acq, mask)
+    g = np_(acq)
+    known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
+    assert np.array_equal(np.isfinite(g), known)
+    idx = sample_idx(n, k, 7)
+    idx = idx[known[idx]]
+    gps = oracle_gps(inst)
+    sub = np.ascontiguousarray(inst.cand[:, idx])
+    mv = [gp.posterior(sub) for gp in gps]
+    mu = np.stack([a for a, _ in mv], 1)
+    var = np.stack([b for _, b in mv], 1)
+    want = O.ehvi_mc(mu, var, inst.eps, O.pareto_front(inst.y_obs.T, inst.ref), inst.ref)
+    assert report(f"score_ehvi {name} (P={fs})", g[idx], want).max() <= 1.0
+    # the two-kernel path gives the same numbers as the fused kernel
+    if n <= 1 << 18:
+        M = inst.n_obj
+        mean = torch.empty((M, n), device="cuda")
+        var_d = torch.empty((M, n), device="cuda")
+        S.scoot_gp_posterior(ctx, L, state, cand, n, mean, var_d, mask)
+        acq2 = torch.empty(n, device="cuda")
+        S.scoot_acq_ehvi(ctx, mean, var_d, n, lo, hi, eps, acq2, mask)
+        assert np.array_equal(np_(acq2), g)
+
+
+def test_score_ei_parity(S, ctx):
+    name = "d10-ei"
+    inst = make_instance(name, seeds(name)[0])
+    n = inst.n_cand
+    L, state = gp_state(S, inst)
+    cand = cand_dev(inst)
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
+    acq = torch.empty(n, device="cuda")
+    S.scoot_score_ei(ctx, L, state, cand, n, 1e-4, acq, mask)
+    g = np_(acq)
+    known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
+    assert np.array_equal(np.isfinite(g), known)
+    top = np.argsort(-np.where(known, g, -np.inf))[:64]
+    idx = np.union1d(sample_idx(n, 8192, 9), top)
+    idx = idx[known[idx]]
+    gp = oracle_gps(inst)[0]
+    mu, var = gp.posterior(np.ascontiguousarray(inst.cand[:, idx]))
+    want = O.expected_improvement(mu, var, float(inst.y_obs[0].max()), 1e-4)
+    assert report("score_ei d10-ei", g[idx], want).max() <= 1.0
+
+
+# ------------------------------------------------------------------ top-q (Section 4.7)
+
+@pytest.mark.parametrize("n,q", [(1, 1), (7, 4), (1000, 1), (5000, 16), (100003, 17), (1 << 20, 64), (300, 64)])
+def test_topq_bit_exact_on_generated_arrays(S, ctx, n, q):
+    st = Stream(n * 131 + q, "topq")
+    acq = np.round(st.normal(n) * 4.0).astype(np.float32) / 4  # many exact ties
+    acq[st.uniform(n) < 0.05] = -np.inf
+    acq[st.uniform(n) < 0.02] = np.nan
+    mask = (st.uniform(n) < 0.7).astype(np.uint8)
+    idx = torch.empty(q, dtype=torch.int64, device="cuda")
+    val = torch.empty(q, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int32, device="cuda")
+    for m in (None, mask):
+        S.scoot_select_topq(ctx, dev(acq), n, q, idx, val, cnt, None if m is None else dev(m))
+        want, wval, c = O.select_topq(acq.astype(np.float64), m, q)
+        gi, gv, gc = np_(idx), np_(val), int(np_(cnt)[0])
+        assert gc == c
+        assert gi[:c].tolist() == want.tolist()
+        assert np.array_equal(gv[:c], acq[want])
+        assert np.all(gi[c:] == -1) and np.all(gv[c:] == -np.inf)
+
+
+def test_topq_degenerate(S, ctx):
+    idx = torch.empty(4, dtype=torch.int64, device="cuda")
+    val = torch.empty(4, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int32, device="cuda")
+    acq = torch.full((100,), -math.inf, device="cuda")
+    S.scoot_select_topq(ctx, acq, 100, 4, idx, val, cnt)
+    assert int(np_(cnt)[0]) == 0 and np.all(np_(idx) == -1)
+    S.scoot_select_topq(ctx, acq, 0, 4, idx, val, cnt)
+    assert int(np_(cnt)[0]) == 0
+    acq = torch.zeros(100, device="cuda")  # all tied: lowest indices win
+    S.scoot_select_topq(ctx, acq, 100, 4, idx, val, cnt)
+    assert np_(idx).tolist() == [0, 1, 2, 3]
+    with pytest.raises(S.ScootError):
+        S.scoot_select_topq(ctx, acq, 100, 65, idx, val, cnt)
+
+
+# ------------------------------------------------------------------ whole round
+
+@pytest.mark.parametrize("name", ["tiny", "d8-ehvi2", "d10-ei", "d10-ehvi3"])
+def test_round_selects_valid_top_q(S, ctx, name):
+    """Gate B: the picks of a full round are a valid top-q of the oracle's own
+    acquisition values, up to swaps within the tolerance."""
+    from paper_2408_04323_gb300.pipeline import RoundInputs, ScoringRound
+    inst = make_instance(name, seeds(name)[0])
+    w = inst.workload
+    inp = RoundInputs(inst.space, inst.clauses, inst.nodes, inst.tree_offset, w.leaf_scale, w.delta_num,
+                      w.delta_den, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                      inst.noise_var, inst.ref, inst.eps, w.acq, w.q)
+    rnd = ScoringRound(ctx, inp, inst.n_cand)
+    idx, val, cnt = rnd.run(cand_dev(inst), inst.n_cand)
+    ctx.check()
+    gi, gv, c = np_(idx), np_(val), int(np_(cnt)[0])
+    known = O.prune_mask(inst.space, inst.clauses, inst.cand, inst.n_cand)
+    votes = O.rf_votes(inst.nodes, inst.tree_offset, inst.space, inst.cand, inst.n_cand)
+    feas = known & O.pof_feasible(votes, inst.n_trees, w.leaf_scale, w.delta_num, w.delta_den)
+    assert np.array_equal(np_(rnd.mask).astype(bool), feas)
+    assert c == min(w.q, int(feas.sum()))
+    g = np_(rnd.acq)
+    # oracle acquisition on the GPU's top candidates plus the next best by the GPU's ranking
+    order = np.argsort(-np.where(feas, g, -np.inf), kind="stable")[:max(4 * w.q, 32)]
+    res = O.score_round(inst, w.acq, subset=order)
+    oacq = res["acq"]
+    tol = ATOL + RTOL * np.abs(oacq)
+    picked = set(gi[:c].tolist())
+    kth = np.sort(oacq)[::-1][c - 1]
+    for j, i in enumerate(order):
+        if i in picked:
+            assert oacq[j] >= kth - 2 * tol[j]
+    assert report(f"round {name} picked acq", gv[:c], oacq[[list(order).index(i) for i in gi[:c]]]).max() <= 1.0

@@ -1,0 +1,203 @@
+"""The C-ABI library without a GPU: it loads, exports what include/scoot.h
+declares, and its host-side preparation agrees with the oracle."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as O
+from workloads import NODE_DTYPE, Stream, make_instance, seeds
+
+from conftest import ROOT
+
+
+@pytest.fixture(scope="module")
+def S():
+    import paper_2408_04323_gb300 as pkg
+    pkg.build()
+    from paper_2408_04323_gb300 import scoot
+    scoot.lib()
+    return scoot
+
+
+def _header_functions():
+    text = open(os.path.join(ROOT, "include", "scoot.h")).read()
+    return sorted(set(re.findall(r"^(?:scoot_status|const char\*)\s+(scoot_\w+)\s*\(", text, re.M)))
+
+
+def test_library_exports_every_declared_symbol(S):
+    names = _header_functions()
+    assert len(names) >= 18
+    lib = S.lib()
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(S.EXPORTS) == names
+
+
+def test_status_strings(S):
+    assert S.scoot_status_string(0) == "ok"
+    assert "unsupported" in S.scoot_status_string(-6)
+
+
+# ------------------------------------------------------------------ boxes
+
+def _hvi_boxes(y, lo, hi):
+    y = np.atleast_2d(y).astype(np.float64)
+    ext = np.minimum(y[:, None, :], hi[None].astype(np.float64)) - lo[None].astype(np.float64)
+    return np.prod(np.maximum(ext, 0), axis=2).sum(1)
+
+
+@pytest.mark.parametrize("M,npts", [(2, 1), (2, 12), (3, 9), (3, 30), (4, 7)])
+def test_boxes_sum_to_oracle_hvi(S, M, npts):
+    st = Stream(100 + M * 7 + npts, "boxes")
+    Y = (st.uniform(M * npts).reshape(M, npts) * 4.0).astype(np.float32)
+    ref = np.zeros(M, np.float32)
+    lo, hi, fs = S.scoot_boxes_build(Y, ref)
+    front = O.pareto_front(Y.T, ref)
+    assert fs == len(front)
+    clo, chi = O.nondominated_cells(front, ref)
+    ys = st.uniform(400 * M).reshape(400, M) * 5.0 - 0.5
+    assert np.allclose(_hvi_boxes(ys, lo, hi), O.hvi_cells(ys, clo, chi), rtol=1e-12, atol=1e-12)
+    # boxes are disjoint: their volumes inside a bounding box plus HV fill it
+    box = np.full(M, 6.0)
+    inside = np.prod(np.maximum(np.minimum(hi.astype(np.float64), box) - lo, 0), axis=1).sum()
+    assert inside + O.hypervolume(front, ref) == pytest.approx(np.prod(box), rel=1e-12)
+    if M == 2:
+        assert len(lo) == len(front) + 1
+
+
+def test_boxes_edge_cases(S):
+    ref = np.array([0.5, -1.0], np.float32)
+    # no point strictly above r: one box [r, +inf)^2
+    Y = np.array([[0.5, 3.0], [2.0, -1.0]], np.float32)
+    lo, hi, fs = S.scoot_boxes_build(Y, ref)
+    assert fs == 0 and len(lo) == 1 and np.allclose(lo[0], ref) and np.all(np.isinf(hi[0]))
+    # duplicates count once
+    Y = np.array([[1.0, 1.0, 2.0], [1.0, 1.0, 0.0]], np.float32)
+    lo, hi, fs = S.scoot_boxes_build(Y, ref)
+    assert fs == 2
+    # capacity too small: unsupported, count reported
+    Y = (Stream(3, "cap").uniform(3 * 20).reshape(3, 20)).astype(np.float32)
+    with pytest.raises(S.ScootError) as e:
+        S.scoot_boxes_build(Y, np.zeros(3, np.float32), cap=2)
+    assert e.value.status == -6
+    with pytest.raises(S.ScootError):
+        S.scoot_boxes_build(np.array([[np.nan], [1.0]], np.float32), np.zeros(2, np.float32))
+
+
+def test_boxes_of_the_three_objective_workload_fit(S):
+    for seed in seeds("d10-ehvi3"):
+        inst = make_instance("d10-ehvi3", seed, n_cand=64)
+        lo, hi, fs = S.scoot_boxes_build(inst.y_obs, inst.ref)
+        assert len(lo) <= 2000 and fs <= 48
+
+
+# ------------------------------------------------------------------ GP state
+
+def _unpack_gp(S, L, blob):
+    f = lambda off, n: blob[off:off + 4 * n].view(np.float32)
+    n, d, M = L.n, L.d, L.n_obj
+    alpha = f(L.off_alpha, M * n).reshape(M, n)
+    tiles = f(L.off_linv, M * L.n_tiles * 32 * 64).reshape(M, L.n_tiles, 32, 64)
+    npad = L.n_rb * 64
+    linv = np.zeros((M, npad, npad), np.float32)
+    for m in range(M):
+        t = 0
+        for rb in range(L.n_rb):
+            for cj in range(2 * (rb + 1)):
+                linv[m, rb * 64:(rb + 1) * 64, cj * 32:(cj + 1) * 32] = tiles[m, t].T
+                t += 1
+    scal = f(L.off_scal, M * 4).reshape(M, 4)
+    xs = f(L.off_xs, M * n * d).reshape(M, n, d)
+    ils = f(L.off_ils, M * d).reshape(M, d)
+    return alpha, linv[:, :n, :n], scal, xs, ils
+
+
+@pytest.mark.parametrize("name", ["tiny", "d8-ehvi2", "d10-ei", "d10-ehvi3"])
+def test_gp_prepare_matches_oracle_factor(S, name):
+    inst = make_instance(name, seeds(name)[0], n_cand=64)
+    M, n, d = inst.n_obj, inst.n_obs, inst.d
+    L = S.scoot_gp_layout_init(n, d, M)
+    blob, cond = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
+                                    inst.signal_var, inst.noise_var, L)
+    alpha, linv, scal, xs, ils = _unpack_gp(S, L, blob)
+    for m in range(M):
+        gp = O.GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m], inst.signal_var[m], inst.noise_var[m])
+        assert np.allclose(alpha[m], gp.alpha, rtol=1e-6, atol=1e-6 * np.abs(gp.alpha).max())
+        Li = np.linalg.inv(gp.chol)
+        assert np.allclose(linv[m], Li, rtol=1e-6, atol=1e-6 * np.abs(Li).max())
+        assert np.all(np.triu(linv[m], 1) == 0)
+        assert scal[m, 0] == inst.signal_var[m] and scal[m, 1] == inst.noise_var[m]
+        assert scal[m, 2] == inst.y_obs[m].max()
+        cat = gp.is_cat
+        assert np.allclose(xs[m][:, ~cat], gp.u_obs[:, ~cat] / inst.lengthscale[m][~cat], rtol=1e-6)
+        assert np.array_equal(xs[m][:, cat], gp.u_obs[:, cat])
+        assert np.allclose(ils[m][cat], 1.0 / inst.lengthscale[m][cat].astype(np.float64) ** 2, rtol=1e-6)
+        assert 1.0 <= cond[m] < 1e8
+
+
+def test_gp_prepare_rejects_bad_inputs(S):
+    inst = make_instance("tiny", 1001, n_cand=8)
+    M, n, d = inst.n_obj, inst.n_obs, inst.d
+    L = S.scoot_gp_layout_init(n, d, M)
+    args = [inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var, inst.noise_var]
+    bad_y = inst.y_obs.copy(); bad_y[0, 3] = np.nan
+    bad_l = inst.lengthscale.copy(); bad_l[1, 2] = 0.0
+    for i, bad in [(2, bad_y), (3, bad_l), (4, np.array([1.0, -1.0], np.float32))]:
+        a = list(args); a[i] = bad
+        with pytest.raises(S.ScootError) as e:
+            S.scoot_gp_prepare(*a, L)
+        assert e.value.status == -1
+    # duplicated observations without noise: K is singular
+    x = np.ascontiguousarray(np.repeat(inst.x_obs[:, :1], n, axis=1))
+    with pytest.raises(S.ScootError):
+        S.scoot_gp_prepare(inst.space, x, inst.y_obs, inst.lengthscale, inst.signal_var,
+                           np.zeros(M, np.float32), L)
+    with pytest.raises(S.ScootError):
+        S.scoot_gp_layout_init(2000, d, M)
+
+
+# ------------------------------------------------------------------ forest
+
+def test_forest_pack_roundtrip_and_validation(S):
+    inst = make_instance("d8-ehvi2", seeds("d8-ehvi2")[0], n_cand=8)
+    L = S.scoot_forest_layout_init(inst.nodes, inst.tree_offset, inst.d, 255)
+    assert L.n_trees == inst.n_trees and L.n_nodes == len(inst.nodes) and L.n_chunks == 1
+    blob = S.scoot_forest_pack(L, inst.nodes, inst.tree_offset)
+    got = blob[L.off_nodes:L.off_nodes + 8 * L.n_nodes].view(NODE_DTYPE)
+    assert np.array_equal(got, inst.nodes)
+
+    def bad(mutate, d=inst.d, scale=255):
+        nodes = inst.nodes.copy()
+        offs = inst.tree_offset.copy()
+        mutate(nodes, offs)
+        with pytest.raises(S.ScootError) as e:
+            S.scoot_forest_layout_init(nodes, offs, d, scale)
+        return e.value.status
+
+    split = int(np.nonzero((inst.nodes["flags"] & 1) == 0)[0][0])
+    leaf = int(np.nonzero(inst.nodes["flags"] & 1)[0][0])
+    assert bad(lambda n, o: n.__setitem__(split, (n[split]["val"], 60000, n[split]["feat"], 0))) == -1
+    assert bad(lambda n, o: n.__setitem__(split, (n[split]["val"], 0, n[split]["feat"], 0))) == -1  # cycle
+    assert bad(lambda n, o: n.__setitem__(split, (n[split]["val"], n[split]["left"], 40, 0))) == -1
+    assert bad(lambda n, o: n.__setitem__(leaf, (2.5, 0, 0, 1))) == -1
+    assert bad(lambda n, o: n.__setitem__(leaf, (256.0, 0, 0, 1))) == -1
+    assert bad(lambda n, o: n.__setitem__(split, (np.nan, n[split]["left"], n[split]["feat"], 0))) == -1
+
+
+def test_forest_chunking_of_large_forests(S):
+    """A forest larger than one shared-memory chunk is split at tree boundaries."""
+    inst = make_instance("d12-fantasy", seeds("d12-fantasy")[0], n_cand=8)
+    reps = 4
+    nodes = np.concatenate([inst.nodes] * reps)
+    sizes = np.diff(inst.tree_offset)
+    offs = np.zeros(inst.n_trees * reps + 1, np.int32)
+    offs[1:] = np.cumsum(np.tile(sizes, reps))
+    L = S.scoot_forest_layout_init(nodes, offs, inst.d, 255)
+    assert L.n_chunks >= 2 and L.max_chunk_nodes <= 12288
+    blob = S.scoot_forest_pack(L, nodes, offs)
+    ch = blob[L.off_chunks:L.off_chunks + 16 * L.n_chunks].view(np.int32).reshape(-1, 4)
+    assert ch[:, 1].sum() == inst.n_trees * reps and ch[:, 3].sum() == len(nodes)
+    assert np.all(ch[1:, 0] == np.cumsum(ch[:-1, 1]))
