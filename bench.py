@@ -1,0 +1,407 @@
+#!/usr/bin/env python
+"""Benchmark of one SCOOT suggestion round on GB300.
+
+A step is one pass of the whole scoring path over a resident candidate
+pool: known-constraint pruning (Eq. 2) -> random-forest POF (Eq. 3) -> GP
+posterior + acquisition (Section 4.3, Eq. 6 / Eq. 7, fused) -> top-q
+(Section 4.7).  The default workload is the 8-parameter, 2-objective EHVI
+configuration: d=8, n=64 observations, N=2^18 candidates, S=64 base
+samples, 100 trees of depth <= 10, q=4.
+
+Prints one JSON line.  `value` is candidates/s with the pool resident in HBM
+(CUDA events on the launching stream, L2 flushed between steps); `e2e` is the
+same metric through the C ABI from pinned host buffers (state preparation,
+host->device copies and the read-back of the picks inside the timed
+region); `roofline` is the dominant kernel's algorithmic work per launch
+over its measured launch time; `cpu_baseline` is the fp64 oracle timed on a
+bounded sample of the same workload on the host.
+
+`--impl reference` times the oracle itself (the only reference this path
+has: the paper ships no code) on bounded samples of the same workload.
+Under torchrun (--gpus N > 1) each rank scores its own pool of N candidates
+(weak scaling) and the ranks' top-q lists are all-gathered and merged.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "candidate configs scored/sec (prune+RF+GP+acq+top-q) and % FP32/HBM roofline"
+UNIT = "candidates/s"
+DEFAULT_WORKLOAD = "d8-ehvi2"
+FLUSH_BYTES = 256 << 20   # > 129 MB of L2
+FP32_LANES_PER_SM = 128
+
+# DRAM bytes per launch from ncu (dram__bytes_read.sum + dram__bytes_write.sum),
+# keyed by (kernel, workload), valid only while the kernel's source file is
+# unchanged (sha256 prefix of the file when the counters were taken).
+TRAFFIC = {}
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the cpu_baseline sample")
+    p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def workload_config(w, extra=None):
+    desc = (f"{w.name}: d={w.d}, n={w.n_obs}, N={w.n_cand}, M={w.n_obj} {w.acq.upper()}"
+            + (f" S={w.n_mc}" if w.acq == "ehvi" else "")
+            + f", RF {w.n_trees} trees depth<={w.max_depth}, q={w.q}")
+    cfg = {"workload": desc, "pool": w.n_cand, "observations": w.n_obs, "objectives": w.n_obj,
+           "acquisition": w.acq, "trees": w.n_trees, "q": w.q,
+           "l2": "flushed between steps (256 MiB write)", "inputs": "seeded synthetic pool, resident in HBM"}
+    if extra:
+        cfg.update(extra)
+    return cfg
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+def referenced_columns(inst):
+    cols = set()
+    for c in inst.clauses:
+        cols.update(int(c["guard_param"][g]) for g in range(int(c["n_guard"])))
+        cols.update(int(c["term_param"][t]) for t in range(int(c["n_term"])))
+    return len(cols)
+
+
+def work_model(inst, n_boxes):
+    """Algorithmic work per candidate of each stage (bytes or flops)."""
+    w = inst.workload
+    d, n = inst.d, inst.n_obs
+    m_eff = 1 if w.acq == "ei" else inst.n_obj
+    post = m_eff * (n * (3 * d + 12) + 2 * n + n * (n + 1) + 2 * n)
+    acq = 30 if w.acq == "ei" else w.n_mc * n_boxes * 4 * inst.n_obj
+    return {
+        "prune": ("hbm", 4 * referenced_columns(inst) + 1),
+        "rf": ("hbm", 4 * d + 1 + 1 + 4),
+        "score": ("alu", post + acq),
+        "topq": ("hbm", 4 + 1),
+    }
+
+
+def sha_of(relpath):
+    with open(os.path.join(ROOT, relpath), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+class ClockSampler:
+    QUERY = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap,utilization.gpu")
+
+    def __init__(self):
+        self.proc = None
+        idx = os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0].strip() or "0"
+        self.gpu = idx if idx.isdigit() else "0"
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-i", self.gpu, "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        rows = []
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                rows.append((float(f[0]), float(f[1]), f[3:7], float(f[7]) if f[7] not in ("", "[N/A]") else 0.0))
+            except ValueError:
+                continue
+        loaded = [r for r in rows if r[3] > 0] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in loaded for i, v in enumerate(r[2]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in loaded) if loaded else None,
+                "sm_max_mhz": max(r[1] for r in loaded) if loaded else None,
+                "reasons": reasons, "samples": len(loaded)}
+
+
+def cpu_oracle_sample(name, seed, n_sample, threads=1):
+    """Time the oracle on n_sample candidates of the workload in a fresh process."""
+    env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
+               MKL_NUM_THREADS=str(threads))
+    code = (
+        "import sys, time, json; sys.path.insert(0, %r)\n"
+        "import numpy as np, oracle\n"
+        "from workloads import make_instance\n"
+        "inst = make_instance(%r, %d, n_cand=%d)\n"
+        "t = time.perf_counter()\n"
+        "r = oracle.score_round(inst, inst.workload.acq)\n"
+        "oracle.select_topq(r['acq'], r['feasible'], inst.workload.q)\n"
+        "print(json.dumps({'seconds': time.perf_counter() - t}))\n" % (ROOT, name, seed, n_sample))
+    p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    if p.returncode != 0:
+        raise RuntimeError(p.stderr[-2000:])
+    return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
+
+
+def calibrate_sample(name, seed, budget_s):
+    """Largest sample whose oracle round fits the budget (scaled from a probe)."""
+    probe = 64
+    t = cpu_oracle_sample(name, seed, probe)
+    per = max(t / probe, 1e-6)
+    return max(16, int(budget_s / per))
+
+
+def run_reference(args):
+    from workloads import WORKLOADS, seeds
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = WORKLOADS[args.workload]
+    seed = seeds(w.name)[0]
+    per_step = max(0.05, 120.0 / max(1, args.steps + args.warmup))
+    sample = calibrate_sample(w.name, seed, per_step)
+    for _ in range(args.warmup):
+        cpu_oracle_sample(w.name, seed, sample)
+    times = [cpu_oracle_sample(w.name, seed, sample) for _ in range(args.steps)]
+    ms = 1e3 * statistics.mean(times)
+    value = sample / (ms / 1e3)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(w, {"reference": "fp64 CPU oracle (the paper ships no code)",
+                                          "sample_per_step": sample}),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{sample} candidates of the {w.name} pool per step, all five steps"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import numpy as np
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(device)
+
+    import paper_2408_04323_gb300 as pkg
+    pkg.build()
+    from paper_2408_04323_gb300 import scoot as S
+    from paper_2408_04323_gb300.pipeline import RoundInputs, ScoringRound, State
+    from paper_2408_04323_gb300.shard import gather_topq
+    from workloads import WORKLOADS, Stream, draw_configs, make_instance, seeds
+
+    w = WORKLOADS[args.workload]
+    seed = seeds(w.name)[0]
+    inst = make_instance(w.name, seed)
+    cand_np = inst.cand
+    if rank > 0:  # each rank scores a pool of its own; the round state is shared
+        cand_np = draw_configs(w, Stream(seed, f"pool-rank{rank}"), inst.n_cand, inst.ld)
+    N = inst.n_cand
+    inp = RoundInputs(inst.space, inst.clauses, inst.nodes, inst.tree_offset, w.leaf_scale, w.delta_num,
+                      w.delta_den, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                      inst.noise_var, inst.ref, inst.eps, w.acq, w.q)
+    ctx = S.Context(device.index)
+    rnd = ScoringRound(ctx, inp, N, device)
+    cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
+    stream = torch.cuda.current_stream(device)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
+    st = rnd.state
+
+    def step(evs=None):
+        sp = S.scoot_prune
+        if evs:
+            evs[0].record(stream)
+        sp(ctx, inp.space, inp.clauses, cand, N, rnd.mask, rnd.n_known, stream)
+        if evs:
+            evs[1].record(stream)
+        S.scoot_rf_predict(ctx, st.forest_layout, st.forest, inp.space, cand, N, inp.delta_num,
+                           inp.delta_den, rnd.votes, rnd.mask, rnd.n_feasible, stream)
+        if evs:
+            evs[2].record(stream)
+        if inp.acq == "ei":
+            S.scoot_score_ei(ctx, st.gp_layout, st.gp_state, cand, N, inp.xi, rnd.acq, rnd.mask, stream)
+        else:
+            S.scoot_score_ehvi(ctx, st.gp_layout, st.gp_state, cand, N, st.box_lo, st.box_hi, st.eps,
+                               rnd.acq, rnd.mask, stream)
+        if evs:
+            evs[3].record(stream)
+        S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask, stream)
+        if evs:
+            evs[4].record(stream)
+
+    sampler = ClockSampler()
+    sampler.start()
+    # warm-up: at least W steps and at least one second of load
+    t_end = time.perf_counter() + args.warmup_seconds
+    k = 0
+    while k < max(3, args.warmup) or time.perf_counter() < t_end:
+        flush.fill_(k & 0xFF)
+        step()
+        k += 1
+        if k % 50 == 0:
+            torch.cuda.synchronize(device)
+    torch.cuda.synchronize(device)
+    ctx.check(stream)
+    n_feasible = int(rnd.n_feasible.item())
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(device)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    for kk in range(args.steps):
+        flush.fill_(kk & 0xFF)
+        step(evs[kk])
+        if dist:
+            gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
+    torch.cuda.synchronize(device)
+    if dist:
+        dist.barrier()
+    clocks = sampler.stop()
+    ctx.check(stream)
+
+    stage_names = ["prune", "rf", "score", "topq"]
+    stage_ms = {s: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, s in enumerate(stage_names)}
+    step_ms = statistics.mean(e[0].elapsed_time(e[4]) for e in evs)
+    if dist:
+        t = torch.tensor([step_ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        step_ms = float(t.item())
+    value = world * N / (step_ms / 1e3)
+
+    # roofline of the dominant stage
+    peaks, peak_src = measured_peaks()
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    fp32_peak = sms * FP32_LANES_PER_SM * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # TFLOP/s
+    work = work_model(inst, st.n_boxes)
+    dom = max(stage_names, key=lambda s: stage_ms[s])
+    kind, per_cand = work[dom]
+    units = n_feasible if dom == "score" else N
+    launch_s = stage_ms[dom] / 1e3
+    kernel_file = {"prune": "prune_rf.cu", "rf": "prune_rf.cu", "score": "score.cu", "topq": "topq.cu"}[dom]
+    tr = TRAFFIC.get((dom, w.name))
+    traffic = None
+    if tr and tr["sha"] == sha_of(os.path.join("paper_2408_04323_gb300", "csrc", kernel_file)):
+        traffic = tr["bytes"]
+    if kind == "hbm":
+        achieved = per_cand * units / launch_s / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"], "traffic": traffic}
+    else:
+        achieved = per_cand * units / launch_s / 1e12
+        roof = {"bound": "alu", "achieved": achieved, "peak": fp32_peak, "unit": "TFLOP/s",
+                "frac": achieved / fp32_peak, "traffic": traffic}
+    roof.update({"kernel": dom, "peak_source": f"{peak_src}; FP32 = SMs x 128 lanes x 2 x max SM clock",
+                 "work_per_unit": per_cand, "units_per_launch": units})
+    stage_roofs = {}
+    for s in stage_names:
+        k_, pc = work[s]
+        u = n_feasible if s == "score" else N
+        if k_ == "hbm":
+            stage_roofs[s] = round(pc * u / (stage_ms[s] / 1e3) / 1e9 / peaks["hbm_gbs"], 4)
+        else:
+            stage_roofs[s] = round(pc * u / (stage_ms[s] / 1e3) / 1e12 / fp32_peak, 4)
+
+    # end to end through the C ABI from pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        host_pool = torch.from_numpy(cand_np.view(np.int32)).pin_memory()
+        cand_e2e = torch.empty_like(cand)
+        h2d = host_pool.numel() * 4
+        times = []
+        for kk in range(args.warmup + args.steps):
+            flush.fill_(kk & 0xFF)
+            torch.cuda.synchronize(device)
+            t0 = time.perf_counter()
+            state = State(inp, device)  # host preparation through the C ABI + copies
+            cand_e2e.copy_(host_pool, non_blocking=True)
+            S.scoot_prune(ctx, inp.space, inp.clauses, cand_e2e, N, rnd.mask, None, stream)
+            S.scoot_rf_predict(ctx, state.forest_layout, state.forest, inp.space, cand_e2e, N, inp.delta_num,
+                               inp.delta_den, rnd.votes, rnd.mask, None, stream)
+            if inp.acq == "ei":
+                S.scoot_score_ei(ctx, state.gp_layout, state.gp_state, cand_e2e, N, inp.xi, rnd.acq, rnd.mask, stream)
+            else:
+                S.scoot_score_ehvi(ctx, state.gp_layout, state.gp_state, cand_e2e, N, state.box_lo, state.box_hi,
+                                   state.eps, rnd.acq, rnd.mask, stream)
+            S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask, stream)
+            picks = (rnd.top_idx.cpu(), rnd.top_val.cpu(), rnd.top_count.cpu())
+            if dist:
+                gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
+            torch.cuda.synchronize(device)
+            if kk >= args.warmup:
+                times.append(time.perf_counter() - t0)
+        state_bytes = sum(b.nbytes for b in state.h_blobs)
+        if inp.acq == "ehvi":
+            state_bytes += sum(b.nbytes for b in state.h_boxes) + inp.eps.nbytes
+        e2e_s = statistics.mean(times)
+        if dist:
+            t = torch.tensor([e2e_s], device=device)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        e2e = {"value": world * N / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d + state_bytes),
+               "d2h_bytes_per_step": int(sum(p.numel() * p.element_size() for p in picks)),
+               "ms_per_step": 1e3 * e2e_s}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = calibrate_sample(w.name, seed, args.cpu_seconds)
+        secs = cpu_oracle_sample(w.name, seed, sample)
+        cpu = {"value": sample / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"{sample} candidates of the {w.name} pool (same round state), all five steps, "
+                         f"fp64 numpy, one thread"}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+                "config": workload_config(w, {"feasible": n_feasible, "boxes": st.n_boxes,
+                                              "front": st.front_size, "parallelism": f"pool shards x{world}"}),
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": args.steps * ScoringRound.KERNELS_PER_ROUND,
+                "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},
+                "stage_roofline_frac": stage_roofs}
+        print(json.dumps(line), flush=True)
+    ctx.close()
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
