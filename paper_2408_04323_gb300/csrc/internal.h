@@ -38,6 +38,16 @@ static inline bool scoot_aligned16(const void* p) {
 scoot_status scoot_check_pool(scoot_ctx* ctx, const uint32_t* cand, int64_t n, int64_t ld, int32_t d);
 
 #ifdef __CUDACC__
+// Index list of live candidates built by scoot_compact in the context workspace.
+struct ScootList {
+    int32_t* list;
+    unsigned int* count;
+};
+// Compacts the indices i < n with mask[i] != 0 into out->list (count on the
+// device); where mask[i] == 0, fill[i] = fill_bits if fill is not NULL.
+scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint32_t* fill, uint32_t fill_bits,
+                           cudaStream_t st, ScootList* out);
+
 #define SCOOT_CUDA(ctx, call)                                                          \
     do {                                                                               \
         cudaError_t e_ = (call);                                                       \

@@ -98,6 +98,8 @@ struct RfArgs {
     unsigned long long* count;
     uint32_t* err;
     int32_t single_chunk;
+    const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
+    const unsigned int* n_list;
 };
 
 // Persistent blocks: each stages (a chunk of) the forest in shared memory,
@@ -113,7 +115,8 @@ rf_kernel(const __grid_constant__ RfArgs a) {
     const int32_t* roots = reinterpret_cast<const int32_t*>(a.forest + a.off_roots);
     const uint2* gnodes = reinterpret_cast<const uint2*>(a.forest + a.off_nodes);
     const int tid = threadIdx.x;
-    const int64_t n_tiles = (a.n + kRfTile - 1) / kRfTile;
+    const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
+    const int64_t n_tiles = (n_work + kRfTile - 1) / kRfTile;
     uint32_t feasible = 0;
 
     auto stage_chunk = [&](int ch) {
@@ -129,26 +132,18 @@ rf_kernel(const __grid_constant__ RfArgs a) {
         const int64_t base = tile * kRfTile;
         int64_t idx[kRfPerThread];
         bool live[kRfPerThread];
-        int any = 0;
 #pragma unroll
         for (int r = 0; r < kRfPerThread; ++r) {
-            idx[r] = base + tid + r * kRfThreads;
-            live[r] = idx[r] < a.n && (a.mask == nullptr || a.mask[idx[r]] != 0);
-            any |= live[r];
-        }
-        if (!__syncthreads_or(any)) {
-            // Nothing to walk in this tile: votes are 0, masks stay 0.
-#pragma unroll
-            for (int r = 0; r < kRfPerThread; ++r)
-                if (idx[r] < a.n) a.votes[idx[r]] = 0u;
-            continue;
+            const int64_t pos = base + tid + r * kRfThreads;
+            live[r] = pos < n_work;
+            idx[r] = live[r] ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
         }
         for (int c = 0; c < a.d; ++c) {
             const bool isf = (a.float_cols >> c) & 1u;
 #pragma unroll
             for (int r = 0; r < kRfPerThread; ++r) {
                 float x = 0.0f;
-                if (idx[r] < a.n) {
+                if (live[r]) {
                     uint32_t w = __ldg(a.cand + (int64_t)c * a.ld + idx[r]);
                     x = isf ? __uint_as_float(w) : (float)(int32_t)w;
                 }
@@ -202,13 +197,11 @@ rf_kernel(const __grid_constant__ RfArgs a) {
         const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
 #pragma unroll
         for (int r = 0; r < kRfPerThread; ++r) {
-            if (idx[r] >= a.n) continue;
-            a.votes[idx[r]] = live[r] ? vote[r] : 0u;
-            if (live[r]) {
-                const bool ok = (unsigned __int128)a.delta_den * vote[r] >= need;
-                if (a.mask) a.mask[idx[r]] = ok;
-                feasible += ok;
-            }
+            if (!live[r]) continue;
+            a.votes[idx[r]] = vote[r];
+            const bool ok = (unsigned __int128)a.delta_den * vote[r] >= need;
+            if (a.mask) a.mask[idx[r]] = ok;
+            feasible += ok;
         }
         __syncthreads();  // sfeat is rewritten by the next tile
     }
@@ -312,6 +305,13 @@ scoot_status scoot_rf_predict(scoot_ctx* ctx, const scoot_forest_layout* L, cons
     a.count = reinterpret_cast<unsigned long long*>(n_feasible);
     a.err = ctx->d_err;
     a.single_chunk = L->n_chunks == 1;
+    if (mask) {
+        // Walk only the candidates still in play; the others get 0 votes.
+        ScootList lst;
+        if ((s = scoot_compact(ctx, mask, n, votes, 0u, st, &lst)) != SCOOT_OK) return s;
+        a.list = lst.list;
+        a.n_list = lst.count;
+    }
     const size_t smem = (size_t)L->d * kRfTile * 4 + (size_t)max_chunk_nodes * 8;
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(rf_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;

@@ -42,6 +42,8 @@ struct ScoreArgs {
     int32_t n_boxes;
     const float* eps;
     int32_t n_mc;
+    const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
+    const unsigned int* n_list;
 };
 
 __device__ __forceinline__ float matern(float r, int kernel) {
@@ -63,30 +65,44 @@ __device__ __forceinline__ float ei_value(float mu, float var, float ybest, floa
     return fmaf(a, cdf, s * pdf);
 }
 
-// HVI summed over S base samples for one candidate; boxes as float4 rows
-// (lo, hi padded to four objectives), eps as float4 rows.
+// EHVI of one candidate: the mean over the S base samples of the hypervolume
+// improvement, summed over boxes.  Boxes are float4 rows (lo, hi padded to
+// four objectives), base samples float4 rows.  Samples are taken eight at a
+// time so that each box is read from shared memory once per eight samples;
+// padding samples sit at -inf and add nothing.
 template <int M>
 __device__ __forceinline__ float ehvi_value(const float* mu, const float* sd, const float4* blo,
                                             const float4* bhi, int n_boxes, const float4* eps,
                                             int n_mc) {
-    float acc = 0.0f;
-    for (int s = 0; s < n_mc; ++s) {
-        const float4 e = eps[s];
-        const float y0 = fmaf(sd[0], e.x, mu[0]);
-        const float y1 = fmaf(sd[1], e.y, mu[1]);
-        const float y2 = M > 2 ? fmaf(sd[2], e.z, mu[2]) : 0.0f;
-        const float y3 = M > 3 ? fmaf(sd[3], e.w, mu[3]) : 0.0f;
-        float hv = 0.0f;
-        for (int b = 0; b < n_boxes; ++b) {
-            const float4 lo = blo[b], hi = bhi[b];
-            float p = fmaxf(fminf(y0, hi.x) - lo.x, 0.0f) * fmaxf(fminf(y1, hi.y) - lo.y, 0.0f);
-            if (M > 2) p *= fmaxf(fminf(y2, hi.z) - lo.z, 0.0f);
-            if (M > 3) p *= fmaxf(fminf(y3, hi.w) - lo.w, 0.0f);
-            hv += p;
+    constexpr int kCh = 8;
+    float total = 0.0f;
+    for (int s0 = 0; s0 < n_mc; s0 += kCh) {
+        float y[kCh][M], acc[kCh];
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) {
+            acc[k] = 0.0f;
+            const bool in = s0 + k < n_mc;
+            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float ev[4] = {e.x, e.y, e.z, e.w};
+#pragma unroll
+            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
         }
-        acc += hv;
+        for (int b = 0; b < n_boxes; ++b) {
+            const float4 lo4 = blo[b], hi4 = bhi[b];
+            const float lo[4] = {lo4.x, lo4.y, lo4.z, lo4.w};
+            const float hi[4] = {hi4.x, hi4.y, hi4.z, hi4.w};
+#pragma unroll
+            for (int k = 0; k < kCh; ++k) {
+                float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+#pragma unroll
+                for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
+                acc[k] += p;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) total += acc[k];
     }
-    return acc * (1.0f / (float)n_mc);
+    return total * (1.0f / (float)n_mc);
 }
 
 __device__ void stage_boxes(const ScoreArgs& a, int M, float4* blo, float4* bhi, float4* eps) {
@@ -141,14 +157,12 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
         fb[c] = c < a.d ? fmap[c * 4 + 2] : 0.f;
     }
 
-    const int64_t n_tiles = (a.n + kTC - 1) / kTC;
+    const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
+    const int64_t n_tiles = (n_work + kTC - 1) / kTC;
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-        const int64_t i = tile * kTC + tid;
-        const bool live = i < a.n && (a.mask == nullptr || a.mask[i] != 0);
-        if (!__syncthreads_or(live)) {
-            if (EPI != kWriteMoments && i < a.n) a.acq[i] = -INFINITY;
-            continue;
-        }
+        const int64_t pos = tile * kTC + tid;
+        const bool live = pos < n_work;
+        const int64_t i = live ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
         // Features of this thread's candidate.
         float u[kMaxD];
 #pragma unroll
@@ -260,18 +274,13 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                     a.var[(int64_t)m * a.ldo + i] = vr[m];
                 }
         } else if (EPI == kEI) {
-            if (i < a.n) a.acq[i] = live ? ei_value(mu[0], vr[0], gscal[2], a.xi) : -INFINITY;
+            if (live) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
         } else {
-            if (i < a.n) {
-                float v = -INFINITY;
-                if (live) {
-                    float sd[kMaxM];
+            float sd[kMaxM];
 #pragma unroll
-                    for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
-                    v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
-                }
-                a.acq[i] = v;
-            }
+            for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
+            const float v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
+            if (live) a.acq[i] = v;
         }
     }
 }
@@ -294,19 +303,17 @@ ehvi_kernel(const __grid_constant__ ScoreArgs a) {
     float4* epsv = bhi + a.n_boxes;
     stage_boxes(a, M, blo, bhi, epsv);
     __syncthreads();
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < a.n; i += (int64_t)gridDim.x * blockDim.x) {
-        const bool live = a.mask == nullptr || a.mask[i] != 0;
-        float v = -INFINITY;
-        if (live) {
-            float mu[kMaxM], sd[kMaxM];
+    const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
+    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < n_work;
+         pos += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+        float mu[kMaxM], sd[kMaxM];
 #pragma unroll
-            for (int m = 0; m < M; ++m) {
-                mu[m] = a.mean[(int64_t)m * a.ldo + i];
-                sd[m] = sqrtf(fmaxf(a.var[(int64_t)m * a.ldo + i], 0.0f));
-            }
-            v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
+        for (int m = 0; m < M; ++m) {
+            mu[m] = a.mean[(int64_t)m * a.ldo + i];
+            sd[m] = sqrtf(fmaxf(a.var[(int64_t)m * a.ldo + i], 0.0f));
         }
-        a.acq[i] = v;
+        a.acq[i] = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
     }
 }
 
@@ -348,7 +355,17 @@ size_t score_smem(const ScoreArgs& a, int epi) {
 }
 
 template <int EPI, int M>
-scoot_status launch_score(scoot_ctx* ctx, const ScoreArgs& a, cudaStream_t st) {
+scoot_status launch_score(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
+    if (a.mask) {
+        // Score only the candidates still in play; the acquisition of the
+        // others is -inf (their moments are left untouched).
+        ScootList lst;
+        scoot_status s = scoot_compact(ctx, a.mask, a.n, EPI == kWriteMoments ? nullptr : reinterpret_cast<uint32_t*>(a.acq),
+                                       0xFF800000u, st, &lst);
+        if (s != SCOOT_OK) return s;
+        a.list = lst.list;
+        a.n_list = lst.count;
+    }
     const size_t smem = score_smem(a, EPI);
     auto kern = score_kernel<EPI, M>;
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
@@ -445,6 +462,13 @@ scoot_status scoot_acq_ehvi(scoot_ctx* ctx, const float* mean, const float* var,
     a.n_mc = n_mc;
     const size_t smem = (size_t)(2 * n_boxes + n_mc) * 16;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (mask) {
+        ScootList lst;
+        if ((s = scoot_compact(ctx, mask, n, reinterpret_cast<uint32_t*>(acq), 0xFF800000u, st, &lst)) != SCOOT_OK)
+            return s;
+        a.list = lst.list;
+        a.n_list = lst.count;
+    }
     int64_t blocks = (n + kAcqThreads - 1) / kAcqThreads;
     auto go = [&](auto kern) -> scoot_status {
         SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
