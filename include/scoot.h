@@ -280,6 +280,27 @@ scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* layout, con
 scoot_status scoot_select_topq(scoot_ctx* ctx, const float* acq, const uint8_t* mask, int64_t n,
                                int32_t q, int64_t* idx, float* val, int32_t* count, void* stream);
 
+/* scoot_select_topq without a context and without allocating.  The paper
+ * has no counterpart: this is a convenience of this library for callers that
+ * cannot allocate device memory at selection time (an allocator that forbids
+ * allocations while it is active, a process whose device memory is sized up
+ * front, or code that cannot create a scoot_ctx because creating one
+ * allocates).  Same arguments, semantics and results as scoot_select_topq,
+ * on the current CUDA device.  The per-block partial lists live in one
+ * fixed 256 KiB device array (32768 keys) that every device which loads the
+ * library keeps until the process exits; a call uses at most blocks * q <=
+ * 32768 keys, so no pool size overflows it.  The first call on a device
+ * looks up the array's device address (make that first call before any
+ * stream capture).  All calls share the array: calls that overlap on the GPU
+ * (different streams, or different host threads) race and must not be
+ * issued; calls ordered on one stream are safe.  Nothing needs clearing
+ * between calls: every entry read is written by the same call.  Errors:
+ * SCOOT_EUNSUPPORTED for q outside 1..SCOOT_MAX_Q or n >= 2^32,
+ * SCOOT_EINVAL for bad pointers or n < 0, SCOOT_ECUDA for runtime failures
+ * (there is no context, so no message). */
+scoot_status scoot_select_topq_static(const float* acq, const uint8_t* mask, int64_t n, int32_t q,
+                                      int64_t* idx, float* val, int32_t* count, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -12,6 +12,8 @@
 //          block's q best by q rounds of a block-wide maximum;
 //  pass 2: one block merges the per-block lists the same way.
 // The per-block lists live in the context's workspace.
+#include <mutex>
+
 #include "internal.h"
 
 namespace {
@@ -171,4 +173,70 @@ extern "C" scoot_status scoot_select_topq(scoot_ctx* ctx, const float* acq, cons
     if (q <= 4) return run<4>(ctx, acq, mask, n, q, idx, val, count, st);
     if (q <= 16) return run<16>(ctx, acq, mask, n, q, idx, val, count, st);
     return run<64>(ctx, acq, mask, n, q, idx, val, count, st);
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant.
+//
+// Some callers cannot allocate device memory when they select: code running
+// under an allocator that forbids new allocations while it is active (for
+// example a caching allocator in the middle of a stream capture, or an
+// embedding process whose memory pool is sized up front), or callers that
+// hold no scoot_ctx because creating one allocates.  For them the per-block
+// partial lists live in this fixed device array instead of a workspace.  The
+// array exists once per device for as long as the library is loaded.
+
+namespace {
+
+constexpr int kStaticKeys = 32768;  // 256 KiB of 64-bit keys
+static __device__ __align__(256) uint64_t g_topq_scratch[kStaticKeys];
+
+constexpr int kMaxDevices = 64;
+std::once_flag g_scratch_once[kMaxDevices];
+uint64_t* g_scratch_ptr[kMaxDevices];
+cudaError_t g_scratch_err[kMaxDevices];
+
+}  // namespace
+
+extern "C" scoot_status scoot_select_topq_static(const float* acq, const uint8_t* mask, int64_t n, int32_t q,
+                                                 int64_t* idx, float* val, int32_t* count, void* stream) {
+    if (q < 1 || q > SCOOT_MAX_Q) return SCOOT_EUNSUPPORTED;
+    if (n < 0) return SCOOT_EINVAL;
+    if (n > 0xFFFFFFFFll) return SCOOT_EUNSUPPORTED;
+    if (!idx || !val || !count || (n > 0 && !acq)) return SCOOT_EINVAL;
+    int device = 0;
+    if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices) {
+        cudaGetLastError();
+        return SCOOT_ECUDA;
+    }
+    // First call on a device: look up the device address of the scratch
+    // array with that device current (host code cannot use the symbol's
+    // name as a device pointer).
+    std::call_once(g_scratch_once[device], [device] {
+        void* p = nullptr;
+        g_scratch_err[device] = cudaGetSymbolAddress(&p, g_topq_scratch);
+        g_scratch_ptr[device] = static_cast<uint64_t*>(p);
+    });
+    if (g_scratch_err[device] != cudaSuccess || !g_scratch_ptr[device]) return SCOOT_ECUDA;
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) return SCOOT_ECUDA;
+    // Blocks are capped so that blocks * q keys fit the array; every key pass
+    // 2 reads is written by pass 1 of the same call, so nothing needs clearing.
+    int64_t blocks = (n + kTopqThreads * 8 - 1) / (kTopqThreads * 8);
+    int64_t cap = (int64_t)(sms > 0 ? sms : 1) * 4;
+    if (cap > kStaticKeys / q) cap = kStaticKeys / q;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    const int64_t slice = (n + blocks - 1) / blocks;
+    uint64_t* partial = g_scratch_ptr[device];
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    auto go = [&](auto p1, auto p2) {
+        p1<<<(unsigned)blocks, kTopqThreads, 0, st>>>(acq, mask, n, slice, q, partial);
+        p2<<<1, kMergeThreads, 0, st>>>(partial, blocks * q, q, idx, val, count);
+    };
+    if (q <= 1) go(topq_pass1<1>, topq_pass2<1>);
+    else if (q <= 4) go(topq_pass1<4>, topq_pass2<4>);
+    else if (q <= 16) go(topq_pass1<16>, topq_pass2<16>);
+    else go(topq_pass1<64>, topq_pass2<64>);
+    return cudaGetLastError() == cudaSuccess ? SCOOT_OK : SCOOT_ECUDA;
 }

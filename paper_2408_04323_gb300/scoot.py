@@ -84,6 +84,7 @@ _PROTOS = {
     "scoot_score_ehvi": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i32,
                          _vp, _i32, _vp, _vp],
     "scoot_select_topq": [_vp, _vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
+    "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
 }
 _STRING_FUNCS = {"scoot_last_error", "scoot_status_string"}
 EXPORTS = tuple(_PROTOS)
@@ -330,3 +331,14 @@ def scoot_select_topq(ctx, acq, n, q, idx, val, count, mask=None, stream=None):
     _check(lib().scoot_select_topq(_h(ctx), _dev(acq, torch.float32, "acq"), _dev(mask, torch.uint8, "mask"),
                                    int(n), int(q), _dev(idx, torch.int64, "idx"), _dev(val, torch.float32, "val"),
                                    _dev(count, torch.int32, "count"), _stream(stream)), "scoot_select_topq", _h(ctx))
+
+
+def scoot_select_topq_static(acq, n, q, idx, val, count, mask=None, stream=None):
+    """Top-q without a context and without allocating (see include/scoot.h):
+    for callers that cannot allocate device memory when they select.  Calls
+    that overlap on the GPU share one scratch array and must not be issued."""
+    import torch
+    _check(lib().scoot_select_topq_static(_dev(acq, torch.float32, "acq"), _dev(mask, torch.uint8, "mask"),
+                                          int(n), int(q), _dev(idx, torch.int64, "idx"),
+                                          _dev(val, torch.float32, "val"), _dev(count, torch.int32, "count"),
+                                          _stream(stream)), "scoot_select_topq_static")
