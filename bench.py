@@ -238,7 +238,7 @@ def main():
     N = inst.n_cand
     inp = RoundInputs(inst.space, inst.clauses, inst.nodes, inst.tree_offset, w.leaf_scale, w.delta_num,
                       w.delta_den, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
-                      inst.noise_var, inst.ref, inst.eps, w.acq, w.q)
+                      inst.noise_var, inst.ref, inst.eps, w.acq, w.q, fantasy=w.fantasy)
     ctx = S.Context(device.index)
     rnd = ScoringRound(ctx, inp, N, device)
     cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
@@ -257,6 +257,14 @@ def main():
                            inp.delta_den, rnd.votes, rnd.mask, rnd.n_feasible, stream)
         if evs:
             evs[2].record(stream)
+        if inp.fantasy:
+            S.scoot_suggest_fantasy(ctx, st.gp_layout, st.gp_state, inp.space, inp.x_obs, inp.y_obs,
+                                    inp.lengthscale, inp.signal_var, inp.noise_var, cand, N, inp.ref, st.eps,
+                                    inp.q, rnd.work, mask=rnd.mask, stream=stream)
+            if evs:
+                evs[3].record(stream)
+                evs[4].record(stream)
+            return
         if inp.acq == "ei":
             S.scoot_score_ei(ctx, st.gp_layout, st.gp_state, cand, N, inp.xi, rnd.acq, rnd.mask, stream)
         else:
@@ -355,12 +363,20 @@ def main():
             S.scoot_prune(ctx, inp.space, inp.clauses, cand_e2e, N, rnd.mask, None, stream)
             S.scoot_rf_predict(ctx, state.forest_layout, state.forest, inp.space, cand_e2e, N, inp.delta_num,
                                inp.delta_den, rnd.votes, rnd.mask, None, stream)
-            if inp.acq == "ei":
+            if inp.fantasy:
+                idx_h, val_h = S.scoot_suggest_fantasy(ctx, state.gp_layout, state.gp_state, inp.space, inp.x_obs,
+                                                       inp.y_obs, inp.lengthscale, inp.signal_var, inp.noise_var,
+                                                       cand_e2e, N, inp.ref, state.eps, inp.q, rnd.work,
+                                                       mask=rnd.mask, stream=stream)
+                rnd.top_idx[:len(idx_h)].copy_(torch.from_numpy(idx_h))
+            elif inp.acq == "ei":
                 S.scoot_score_ei(ctx, state.gp_layout, state.gp_state, cand_e2e, N, inp.xi, rnd.acq, rnd.mask, stream)
             else:
                 S.scoot_score_ehvi(ctx, state.gp_layout, state.gp_state, cand_e2e, N, state.box_lo, state.box_hi,
                                    state.eps, rnd.acq, rnd.mask, stream)
-            S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask, stream)
+            if not inp.fantasy:
+                S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask,
+                                    stream)
             picks = (rnd.top_idx.cpu(), rnd.top_val.cpu(), rnd.top_count.cpu())
             if dist:
                 gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
@@ -394,7 +410,7 @@ def main():
                 "config": workload_config(w, {"feasible": n_feasible, "boxes": st.n_boxes,
                                               "front": st.front_size, "parallelism": f"pool shards x{world}"}),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": args.steps * ScoringRound.KERNELS_PER_ROUND,
+                "gpu_launches": args.steps * rnd.kernels_per_round(),
                 "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},
                 "stage_roofline_frac": stage_roofs}
         print(json.dumps(line), flush=True)

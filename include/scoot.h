@@ -280,6 +280,39 @@ scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* layout, con
 scoot_status scoot_select_topq(scoot_ctx* ctx, const float* acq, const uint8_t* mask, int64_t n,
                                int32_t q, int64_t* idx, float* val, int32_t* count, void* stream);
 
+/* ------------------------------------------------------------------ 6. sequential fantasised picks */
+
+/* Bytes of the caller-owned device work buffer scoot_suggest_fantasy needs
+ * for a pool of n candidates and q picks (about 4 n (M (2 + 64 n_rb + q) + 1)
+ * bytes: moments, whitened covariance rows and downdate factors of every
+ * candidate). */
+scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* layout, int64_t n, int32_t q, int64_t* bytes);
+
+/* q sequential EHVI picks with kriging-believer fantasies (a variant of the
+ * parallel suggestion of Section 4.7, whose picks are plain top-k): pick 1 is
+ * the EHVI argmax (Eq. 7) over the candidates with mask[i] == 1 (mask may be
+ * NULL); after each pick p every objective's value at x_p is fantasised as
+ * its posterior mean, the GP is conditioned on it with noise tau^2 (means
+ * unchanged, variances lowered by a rank-1 term), the fantasised point joins
+ * the Pareto front above h_ref (boxes rebuilt on the host), and the next
+ * pick is the EHVI argmax among the candidates not yet picked.  Ties go to
+ * the lowest index.  The GP host inputs (h_x_obs [d][ld_obs], h_y [M][n],
+ * h_lengthscale, h_signal_var, h_noise_var) must be those the state blob was
+ * prepared from; the per-pick rank-1 terms are computed from them in fp64.
+ * eps: device base samples [S][M].  work: device buffer of at least
+ * scoot_fantasy_work_bytes bytes, 256-byte aligned.  Outputs: h_idx, h_val
+ * (host, [q]) and *h_count (fewer than q when the candidates run out); if
+ * var_out is not NULL (device [M][n]) it receives the variances after the
+ * last downdate for candidates with mask[i] == 1.  Synchronous: returns after
+ * the picks are on the host.  2 <= M <= 4, 1 <= q <= SCOOT_MAX_Q. */
+scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                                   const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
+                                   const float* h_y, const float* h_lengthscale, const float* h_signal_var,
+                                   const float* h_noise_var, const uint32_t* cand, int64_t n, int64_t ld,
+                                   const uint8_t* mask, const float* h_ref, const float* eps, int32_t n_mc,
+                                   int32_t q, void* work, int64_t work_bytes, int64_t* h_idx, float* h_val,
+                                   int32_t* h_count, float* var_out, void* stream);
+
 /* scoot_select_topq without a context and without allocating.  The paper
  * has no counterpart: this is a convenience of this library for callers that
  * cannot allocate device memory at selection time (an allocator that forbids

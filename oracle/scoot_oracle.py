@@ -465,11 +465,12 @@ def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
     u_pool, _ = gp_features(inst.space, decode(inst.space, words, n))
     mu0 = np.stack([gp.posterior_u(u_pool)[0] for gp in gps], axis=1)
     Yf = inst.y_obs.T.astype(np.float64)
-    picks, acqs, mus, vars_ = [], [], [], []
+    picks, acqs, mus, vars_, fronts = [], [], [], [], []
     eligible = np.asarray(feasible, bool).copy()
     for j in range(q):
         var = np.stack([gp.posterior_u(u_pool)[1] for gp in gps], axis=1)
         front = pareto_front(Yf, inst.ref)
+        fronts.append(front)
         a = ehvi_mc(mu0, var, inst.eps, front, inst.ref)
         a = np.where(eligible, a, -np.inf)
         if forced is not None:
@@ -487,4 +488,4 @@ def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
         for m, gp in enumerate(gps):
             gp.add_observations(u_pool[p:p + 1], [mu0[p, m]])
         Yf = np.concatenate([Yf, mu0[p:p + 1]], axis=0)
-    return dict(picks=picks, acq=acqs, var=vars_, mu=mus)
+    return dict(picks=picks, acq=acqs, var=vars_, mu=mus, fronts=fronts)

@@ -15,7 +15,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libscoot.so")
-SOURCES = ["context.cu", "host_prep.cpp", "compact.cu", "prune_rf.cu", "score.cu", "topq.cu"]
+SOURCES = ["context.cu", "host_prep.cpp", "compact.cu", "prune_rf.cu", "score.cu", "topq.cu", "fantasy.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall"]
 
@@ -36,8 +36,8 @@ def _stale(obj: str, deps: list[str]) -> bool:
 
 def build(force: bool = False, verbose: bool = False, extra: list[str] | None = None) -> str:
     os.makedirs(BUILD, exist_ok=True)
-    headers = [os.path.join(CSRC, "internal.h"),
-               os.path.join(os.path.dirname(PKG), "include", "scoot.h")]
+    headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
+    headers.append(os.path.join(os.path.dirname(PKG), "include", "scoot.h"))
     cc = nvcc()
     jobs = []
     for src in SOURCES:

@@ -1,0 +1,120 @@
+// Device helpers shared by the scoring kernels (score.cu) and the fantasy
+// kernels (fantasy.cu).
+#pragma once
+
+#include "internal.h"
+
+namespace scoot_dev {
+
+__device__ __forceinline__ float matern(float r, int kernel) {
+    if (kernel == SCOOT_MATERN32) {
+        const float a = 1.7320508075688772f * r;
+        return (1.0f + a) * expf(-a);
+    }
+    const float a = 2.2360679774997896f * r;
+    return fmaf(a, fmaf(a, 0.33333333333333333f, 1.0f), 1.0f) * expf(-a);
+}
+
+__device__ __forceinline__ float ei_value(float mu, float var, float ybest, float xi) {
+    const float a = (mu - ybest) + xi;
+    const float s = sqrtf(fmaxf(var, 0.0f));
+    if (!(s > 0.0f)) return fmaxf(a, 0.0f);
+    const float z = a / s;
+    const float cdf = 0.5f * erfcf(-z * 0.70710678118654752f);
+    const float pdf = 0.39894228040143268f * expf(-0.5f * z * z);
+    return fmaf(a, cdf, s * pdf);
+}
+
+// EHVI of one candidate: the mean over the S base samples of the hypervolume
+// improvement, summed over boxes.  Boxes are float4 rows (lo, hi padded to
+// four objectives), base samples float4 rows.  Samples are taken eight at a
+// time so that each box is read from shared memory once per eight samples;
+// padding samples sit at -inf and add nothing.
+template <int M>
+__device__ __forceinline__ float ehvi_value(const float* mu, const float* sd, const float4* blo,
+                                            const float4* bhi, int n_boxes, const float4* eps,
+                                            int n_mc) {
+    constexpr int kCh = 8;
+    float total = 0.0f;
+    for (int s0 = 0; s0 < n_mc; s0 += kCh) {
+        float y[kCh][M], acc[kCh];
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) {
+            acc[k] = 0.0f;
+            const bool in = s0 + k < n_mc;
+            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float ev[4] = {e.x, e.y, e.z, e.w};
+#pragma unroll
+            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
+        }
+        for (int b = 0; b < n_boxes; ++b) {
+            const float4 lo4 = blo[b], hi4 = bhi[b];
+            const float lo[4] = {lo4.x, lo4.y, lo4.z, lo4.w};
+            const float hi[4] = {hi4.x, hi4.y, hi4.z, hi4.w};
+#pragma unroll
+            for (int k = 0; k < kCh; ++k) {
+                float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+#pragma unroll
+                for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
+                acc[k] += p;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) total += acc[k];
+    }
+    return total * (1.0f / (float)n_mc);
+}
+
+// Boxes ([B][M] lower and upper bounds) and base samples ([S][M]) into shared
+// memory as float4 rows padded to four objectives.
+__device__ __forceinline__ void stage_boxes(const float* box_lo, const float* box_hi, int n_boxes, const float* eps_in,
+                                            int n_mc, int M, float4* blo, float4* bhi, float4* eps) {
+    for (int b = threadIdx.x; b < n_boxes; b += blockDim.x) {
+        float l[4] = {0.f, 0.f, 0.f, 0.f}, h[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int j = 0; j < M; ++j) {
+            l[j] = box_lo[b * M + j];
+            h[j] = box_hi[b * M + j];
+        }
+        blo[b] = make_float4(l[0], l[1], l[2], l[3]);
+        bhi[b] = make_float4(h[0], h[1], h[2], h[3]);
+    }
+    for (int s = threadIdx.x; s < n_mc; s += blockDim.x) {
+        float e[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int j = 0; j < M; ++j) e[j] = eps_in[s * M + j];
+        eps[s] = make_float4(e[0], e[1], e[2], e[3]);
+    }
+}
+
+// Covariance-input coordinate of one stored parameter value (Section 4.3 with
+// the feature map of include/scoot.h): log scale for integer log-uniform
+// parameters, linear for integer uniform and continuous ones, the category
+// index for categoricals; a and b are the offset and scale of the map.
+__device__ __forceinline__ float feature_of(uint32_t w, int kind, float a, float b) {
+    if (kind == SCOOT_INT_LOG) return (logf((float)(int32_t)w) - a) * b;
+    if (kind == SCOOT_INT_UNIFORM) return ((float)(int32_t)w - a) * b;
+    if (kind == SCOOT_CONTINUOUS) return (__uint_as_float(w) - a) * b;
+    return (float)(int32_t)w;
+}
+
+
+// Selection key of a candidate (Section 4.7 order): the high word is the
+// value mapped to an order-preserving unsigned integer, the low word is
+// 0xFFFFFFFF - index, so a larger key is a larger value or, on equal
+// values, a lower index.  0 is never a key of an eligible candidate.
+__device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
+    uint32_t b = __float_as_uint(v);
+    b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return ((uint64_t)b << 32) | (uint64_t)(0xFFFFFFFFu - idx);
+}
+
+__device__ __forceinline__ float key_value(uint64_t k) {
+    uint32_t b = (uint32_t)(k >> 32);
+    b = (b & 0x80000000u) ? (b & 0x7FFFFFFFu) : ~b;
+    return __uint_as_float(b);
+}
+
+__device__ __forceinline__ int64_t key_index(uint64_t k) {
+    return (int64_t)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFu));
+}
+
+}  // namespace scoot_dev

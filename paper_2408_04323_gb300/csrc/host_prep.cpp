@@ -72,6 +72,98 @@ bool valid_space(const scoot_param* sp, int32_t d) {
 
 }  // namespace
 
+double HostGP::cov(const double* ua, const double* ub) const {
+    double r2 = 0.0;
+    for (int c = 0; c < d; ++c) {
+        if (cat[c]) {
+            if (ua[c] != ub[c]) r2 += 1.0 / (ell[c] * ell[c]);
+        } else {
+            const double t = (ua[c] - ub[c]) / ell[c];
+            r2 += t * t;
+        }
+    }
+    return sf2 * matern(std::sqrt(r2), kernel);
+}
+
+void HostGP::kstar(const double* ux, double* k) const {
+    for (int j = 0; j < n; ++j) k[j] = cov(ux, &u[(size_t)j * d]);
+}
+
+void HostGP::solve_lower(const double* b, double* x) const {
+    for (int i = 0; i < n; ++i) {
+        double t = b[i];
+        for (int k = 0; k < i; ++k) t -= chol[(size_t)i * n + k] * x[k];
+        x[i] = t / chol[(size_t)i * n + i];
+    }
+}
+
+bool scoot_host_features(const scoot_param* sp, int d, const uint32_t* words, int64_t ld, int64_t j, double* u) {
+    for (int c = 0; c < d; ++c) {
+        const double v = stored_value(sp[c], words[(size_t)c * ld + j]);
+        if (!is_finite(v)) return false;
+        if (sp[c].kind == SCOOT_INT_LOG && !(v > 0.0)) return false;
+        u[c] = feature(sp[c], v);
+    }
+    return true;
+}
+
+scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, int64_t ld_obs, int n,
+                           const float* y, const float* lengthscale, float signal_var, float noise_var,
+                           int kernel, HostGP* g, double* cond) {
+    if (!(signal_var > 0.0f) || !is_finite(signal_var) || !(noise_var >= 0.0f) || !is_finite(noise_var))
+        return SCOOT_EINVAL;
+    g->n = n;
+    g->d = d;
+    g->kernel = kernel;
+    g->sf2 = signal_var;
+    g->tau2 = noise_var;
+    g->u.assign((size_t)n * d, 0.0);
+    g->cat.assign(d, 0);
+    g->ell.assign(d, 1.0);
+    for (int c = 0; c < d; ++c) {
+        if (!(lengthscale[c] > 0.0f) || !is_finite(lengthscale[c])) return SCOOT_EINVAL;
+        g->ell[c] = lengthscale[c];
+        g->cat[c] = sp[c].kind == SCOOT_CATEGORICAL;
+    }
+    for (int j = 0; j < n; ++j) {
+        if (!is_finite(y[j])) return SCOOT_EINVAL;
+        if (!scoot_host_features(sp, d, x_obs, ld_obs, j, &g->u[(size_t)j * d])) return SCOOT_EINVAL;
+    }
+    std::vector<double>& K = g->chol;
+    K.assign((size_t)n * n, 0.0);
+    for (int i = 0; i < n; ++i)
+        for (int j = 0; j <= i; ++j)
+            K[(size_t)i * n + j] = g->cov(&g->u[(size_t)i * d], &g->u[(size_t)j * d]) + (i == j ? g->tau2 : 0.0);
+    double pmin = std::numeric_limits<double>::infinity(), pmax = 0.0;
+    for (int j = 0; j < n; ++j) {
+        double s = K[(size_t)j * n + j];
+        for (int k = 0; k < j; ++k) s -= K[(size_t)j * n + k] * K[(size_t)j * n + k];
+        if (!(s > 0.0) || !is_finite(s)) return SCOOT_EINVAL;
+        const double piv = std::sqrt(s);
+        K[(size_t)j * n + j] = piv;
+        pmin = std::min(pmin, piv);
+        pmax = std::max(pmax, piv);
+        for (int i = j + 1; i < n; ++i) {
+            double t = K[(size_t)i * n + j];
+            for (int k = 0; k < j; ++k) t -= K[(size_t)i * n + k] * K[(size_t)j * n + k];
+            K[(size_t)i * n + j] = t / piv;
+        }
+        for (int i = 0; i < j; ++i) K[(size_t)i * n + j] = 0.0;  // keep the upper triangle zero
+    }
+    if (cond) *cond = (pmax / pmin) * (pmax / pmin);
+    // alpha = C^{-T} C^{-1} y
+    std::vector<double> tmp(n), yd(n);
+    for (int j = 0; j < n; ++j) yd[j] = y[j];
+    g->solve_lower(yd.data(), tmp.data());
+    g->alpha.assign(n, 0.0);
+    for (int i = n - 1; i >= 0; --i) {
+        double t = tmp[i];
+        for (int k = i + 1; k < n; ++k) t -= K[(size_t)k * n + i] * g->alpha[k];
+        g->alpha[i] = t / K[(size_t)i * n + i];
+    }
+    return SCOOT_OK;
+}
+
 extern "C" {
 
 const char* scoot_status_string(scoot_status s) {
@@ -134,16 +226,6 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
             if (!is_finite(h_y[m * n + j])) return SCOOT_EINVAL;
     }
 
-    // Features of the observations.
-    std::vector<double> u((size_t)n * d);
-    for (int j = 0; j < n; ++j)
-        for (int c = 0; c < d; ++c) {
-            double v = stored_value(h_space[c], h_x_obs[(size_t)c * ld_obs + j]);
-            if (!is_finite(v)) return SCOOT_EINVAL;
-            if (h_space[c].kind == SCOOT_INT_LOG && !(v > 0.0)) return SCOOT_EINVAL;
-            u[(size_t)j * d + c] = feature(h_space[c], v);
-        }
-
     char* blob = static_cast<char*>(h_blob);
     std::memset(blob, 0, (size_t)L->bytes);
     float* fmap = reinterpret_cast<float*>(blob + L->off_fmap);
@@ -168,70 +250,27 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
     float* linv_out = reinterpret_cast<float*>(blob + L->off_linv);
     float* scal = reinterpret_cast<float*>(blob + L->off_scal);
 
-    std::vector<double> K((size_t)n * n), Li((size_t)n * n), alpha(n), tmp(n);
+    std::vector<double> Li((size_t)n * n), e(n), col(n);
+    HostGP g;
     for (int m = 0; m < M; ++m) {
-        const float* ell = h_lengthscale + (size_t)m * d;
-        const double sf2 = h_signal_var[m], tau2 = h_noise_var[m];
+        scoot_status s = scoot_host_gp(h_space, d, h_x_obs, ld_obs, n, h_y + (size_t)m * n,
+                                       h_lengthscale + (size_t)m * d, h_signal_var[m], h_noise_var[m],
+                                       L->kernel, &g, h_cond ? &h_cond[m] : nullptr);
+        if (s != SCOOT_OK) return s;
         for (int c = 0; c < d; ++c) {
-            bool cat = h_space[c].kind == SCOOT_CATEGORICAL;
-            double l = ell[c];
-            ils[m * d + c] = cat ? (float)(1.0 / (l * l)) : (float)(1.0 / l);
+            const double l = g.ell[c];
+            ils[m * d + c] = g.cat[c] ? (float)(1.0 / (l * l)) : (float)(1.0 / l);
             for (int j = 0; j < n; ++j)
-                xs[((size_t)m * n + j) * d + c] = cat ? (float)u[(size_t)j * d + c] : (float)(u[(size_t)j * d + c] / l);
+                xs[((size_t)m * n + j) * d + c] = g.cat[c] ? (float)g.u[(size_t)j * d + c]
+                                                           : (float)(g.u[(size_t)j * d + c] / l);
         }
-        // K + tau^2 I
-        for (int i = 0; i < n; ++i)
-            for (int j = 0; j <= i; ++j) {
-                double r2 = 0.0;
-                for (int c = 0; c < d; ++c) {
-                    double l = ell[c];
-                    if (h_space[c].kind == SCOOT_CATEGORICAL) {
-                        if (u[(size_t)i * d + c] != u[(size_t)j * d + c]) r2 += 1.0 / (l * l);
-                    } else {
-                        double t = (u[(size_t)i * d + c] - u[(size_t)j * d + c]) / l;
-                        r2 += t * t;
-                    }
-                }
-                double k = sf2 * matern(std::sqrt(r2), L->kernel);
-                K[(size_t)i * n + j] = K[(size_t)j * n + i] = k + (i == j ? tau2 : 0.0);
-            }
-        // Cholesky K = C C^T (lower, in place in the lower triangle).
-        double pmin = std::numeric_limits<double>::infinity(), pmax = 0.0;
-        for (int j = 0; j < n; ++j) {
-            double s = K[(size_t)j * n + j];
-            for (int k = 0; k < j; ++k) s -= K[(size_t)j * n + k] * K[(size_t)j * n + k];
-            if (!(s > 0.0) || !is_finite(s)) return SCOOT_EINVAL;
-            double piv = std::sqrt(s);
-            K[(size_t)j * n + j] = piv;
-            pmin = std::min(pmin, piv);
-            pmax = std::max(pmax, piv);
-            for (int i = j + 1; i < n; ++i) {
-                double t = K[(size_t)i * n + j];
-                for (int k = 0; k < j; ++k) t -= K[(size_t)i * n + k] * K[(size_t)j * n + k];
-                K[(size_t)i * n + j] = t / piv;
-            }
-        }
-        if (h_cond) h_cond[m] = (pmax / pmin) * (pmax / pmin);
-        // alpha = C^{-T} C^{-1} y
-        for (int i = 0; i < n; ++i) {
-            double t = h_y[(size_t)m * n + i];
-            for (int k = 0; k < i; ++k) t -= K[(size_t)i * n + k] * tmp[k];
-            tmp[i] = t / K[(size_t)i * n + i];
-        }
-        for (int i = n - 1; i >= 0; --i) {
-            double t = tmp[i];
-            for (int k = i + 1; k < n; ++k) t -= K[(size_t)k * n + i] * alpha[k];
-            alpha[i] = t / K[(size_t)i * n + i];
-        }
-        for (int i = 0; i < n; ++i) alpha_out[(size_t)m * n + i] = (float)alpha[i];
-        // L^{-1} = C^{-1} by forward substitution on the identity, column by column.
-        std::fill(Li.begin(), Li.end(), 0.0);
-        for (int col = 0; col < n; ++col) {
-            for (int i = col; i < n; ++i) {
-                double t = (i == col) ? 1.0 : 0.0;
-                for (int k = col; k < i; ++k) t -= K[(size_t)i * n + k] * Li[(size_t)k * n + col];
-                Li[(size_t)i * n + col] = t / K[(size_t)i * n + i];
-            }
+        for (int i = 0; i < n; ++i) alpha_out[(size_t)m * n + i] = (float)g.alpha[i];
+        // L^{-1}: column by column, C col = e_col.
+        for (int c = 0; c < n; ++c) {
+            std::fill(e.begin(), e.end(), 0.0);
+            e[c] = 1.0;
+            g.solve_lower(e.data(), col.data());
+            for (int i = 0; i < n; ++i) Li[(size_t)i * n + c] = i >= c ? col[i] : 0.0;
         }
         // Tiles: row block rb covers rows [64 rb, 64 rb + 64) and column
         // chunks cj = 0 .. 2 rb + 1 of 32 columns; tile[jj][ii] = Li[row][col].
@@ -241,15 +280,15 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
             for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t)
                 for (int jj = 0; jj < kColChunk; ++jj)
                     for (int ii = 0; ii < kRowBlock; ++ii) {
-                        int row = rb * kRowBlock + ii, col = cj * kColChunk + jj;
+                        const int row = rb * kRowBlock + ii, c = cj * kColChunk + jj;
                         float v = 0.0f;
-                        if (row < n && col <= row) v = (float)Li[(size_t)row * n + col];
+                        if (row < n && c <= row) v = (float)Li[(size_t)row * n + c];
                         tiles[((size_t)t * kColChunk + jj) * kRowBlock + ii] = v;
                     }
         float ybest = -std::numeric_limits<float>::infinity();
         for (int j = 0; j < n; ++j) ybest = std::max(ybest, h_y[(size_t)m * n + j]);
-        scal[m * 4 + 0] = (float)sf2;
-        scal[m * 4 + 1] = (float)tau2;
+        scal[m * 4 + 0] = h_signal_var[m];
+        scal[m * 4 + 1] = h_noise_var[m];
         scal[m * 4 + 2] = ybest;
     }
     return SCOOT_OK;

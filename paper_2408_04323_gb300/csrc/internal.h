@@ -5,6 +5,7 @@
 #include <cstdint>
 #include <cstdio>
 #include <string>
+#include <vector>
 
 #include "../../include/scoot.h"
 
@@ -34,6 +35,28 @@ static inline bool scoot_aligned16(const void* p) {
     return (reinterpret_cast<uintptr_t>(p) & 15u) == 0;
 }
 
+// fp64 GP of one objective over the observations (Section 4.3), host side:
+// K + tau^2 I = C C^T, alpha = (K + tau^2 I)^{-1} y.
+struct HostGP {
+    int n = 0, d = 0, kernel = SCOOT_MATERN52;
+    double sf2 = 1.0, tau2 = 0.0;
+    std::vector<double> u;        // [n][d] features of the observations
+    std::vector<uint8_t> cat;     // [d] 1 for categorical dimensions
+    std::vector<double> ell;      // [d] lengthscales
+    std::vector<double> chol;     // [n][n], lower triangle
+    std::vector<double> alpha;    // [n]
+    double cov(const double* ua, const double* ub) const;       // k(a, b)
+    void kstar(const double* ux, double* k) const;              // k(x, X_j), j < n
+    void solve_lower(const double* b, double* x) const;         // C x = b
+};
+// Features of configuration j of a SoA word array (ld = leading dimension).
+bool scoot_host_features(const scoot_param* sp, int d, const uint32_t* words, int64_t ld, int64_t j, double* u);
+// Factor objective m; SCOOT_EINVAL on bad inputs or a matrix that is not
+// numerically positive definite.  cond (optional) receives (max/min pivot)^2.
+scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, int64_t ld_obs, int n,
+                           const float* y, const float* lengthscale, float signal_var, float noise_var,
+                           int kernel, HostGP* out, double* cond);
+
 // Checks shared by the device entry points.
 scoot_status scoot_check_pool(scoot_ctx* ctx, const uint32_t* cand, int64_t n, int64_t ld, int32_t d);
 
@@ -47,6 +70,14 @@ struct ScootList {
 // device); where mask[i] == 0, fill[i] = fill_bits if fill is not NULL.
 scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint32_t* fill, uint32_t fill_bits,
                            cudaStream_t st, ScootList* out);
+
+// Posterior of the listed candidates into list-position order: mean and var
+// [M][ldc], and the whitened rows V = L^{-1} k(X, x) [M][n_rb * 64][ldc]
+// (rows >= n left unwritten).  ldc >= the list length.
+scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                                      const uint32_t* cand, int64_t n, int64_t ld, const int32_t* list,
+                                      const unsigned int* n_list, float* mean, float* var, float* V, int64_t ldc,
+                                      cudaStream_t st);
 
 #define SCOOT_CUDA(ctx, call)                                                          \
     do {                                                                               \

@@ -12,9 +12,12 @@
 // The epilogue writes mu and sigma^2, or the EI, or the EHVI of the tile.
 #include <cstring>
 
+#include "device_common.cuh"
 #include "internal.h"
 
 namespace {
+
+using namespace scoot_dev;
 
 constexpr int kTC = 64;     // candidates per tile = threads per block
 constexpr int kRB = 64;     // rows of L^{-1} per tile
@@ -23,7 +26,7 @@ constexpr int kMaxD = SCOOT_MAX_DIM;
 constexpr int kMaxM = SCOOT_MAX_OBJ;
 constexpr int kAcqThreads = 128;
 
-enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2 };
+enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3 };
 
 struct ScoreArgs {
     const char* state;
@@ -44,83 +47,9 @@ struct ScoreArgs {
     int32_t n_mc;
     const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
     const unsigned int* n_list;
+    float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad][ldv] by list position
+    int64_t ldv;
 };
-
-__device__ __forceinline__ float matern(float r, int kernel) {
-    if (kernel == SCOOT_MATERN32) {
-        const float a = 1.7320508075688772f * r;
-        return (1.0f + a) * expf(-a);
-    }
-    const float a = 2.2360679774997896f * r;
-    return fmaf(a, fmaf(a, 0.33333333333333333f, 1.0f), 1.0f) * expf(-a);
-}
-
-__device__ __forceinline__ float ei_value(float mu, float var, float ybest, float xi) {
-    const float a = (mu - ybest) + xi;
-    const float s = sqrtf(fmaxf(var, 0.0f));
-    if (!(s > 0.0f)) return fmaxf(a, 0.0f);
-    const float z = a / s;
-    const float cdf = 0.5f * erfcf(-z * 0.70710678118654752f);
-    const float pdf = 0.39894228040143268f * expf(-0.5f * z * z);
-    return fmaf(a, cdf, s * pdf);
-}
-
-// EHVI of one candidate: the mean over the S base samples of the hypervolume
-// improvement, summed over boxes.  Boxes are float4 rows (lo, hi padded to
-// four objectives), base samples float4 rows.  Samples are taken eight at a
-// time so that each box is read from shared memory once per eight samples;
-// padding samples sit at -inf and add nothing.
-template <int M>
-__device__ __forceinline__ float ehvi_value(const float* mu, const float* sd, const float4* blo,
-                                            const float4* bhi, int n_boxes, const float4* eps,
-                                            int n_mc) {
-    constexpr int kCh = 8;
-    float total = 0.0f;
-    for (int s0 = 0; s0 < n_mc; s0 += kCh) {
-        float y[kCh][M], acc[kCh];
-#pragma unroll
-        for (int k = 0; k < kCh; ++k) {
-            acc[k] = 0.0f;
-            const bool in = s0 + k < n_mc;
-            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float ev[4] = {e.x, e.y, e.z, e.w};
-#pragma unroll
-            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
-        }
-        for (int b = 0; b < n_boxes; ++b) {
-            const float4 lo4 = blo[b], hi4 = bhi[b];
-            const float lo[4] = {lo4.x, lo4.y, lo4.z, lo4.w};
-            const float hi[4] = {hi4.x, hi4.y, hi4.z, hi4.w};
-#pragma unroll
-            for (int k = 0; k < kCh; ++k) {
-                float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
-#pragma unroll
-                for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
-                acc[k] += p;
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < kCh; ++k) total += acc[k];
-    }
-    return total * (1.0f / (float)n_mc);
-}
-
-__device__ void stage_boxes(const ScoreArgs& a, int M, float4* blo, float4* bhi, float4* eps) {
-    for (int b = threadIdx.x; b < a.n_boxes; b += blockDim.x) {
-        float l[4] = {0.f, 0.f, 0.f, 0.f}, h[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int j = 0; j < M; ++j) {
-            l[j] = a.box_lo[b * M + j];
-            h[j] = a.box_hi[b * M + j];
-        }
-        blo[b] = make_float4(l[0], l[1], l[2], l[3]);
-        bhi[b] = make_float4(h[0], h[1], h[2], h[3]);
-    }
-    for (int s = threadIdx.x; s < a.n_mc; s += blockDim.x) {
-        float e[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int j = 0; j < M; ++j) e[j] = a.eps[s * M + j];
-        eps[s] = make_float4(e[0], e[1], e[2], e[3]);
-    }
-}
 
 template <int EPI, int M>
 __global__ void __launch_bounds__(kTC)
@@ -138,6 +67,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
 
     const int tid = threadIdx.x;
     const int nobj = EPI == kEHVI ? M : (EPI == kEI ? 1 : a.n_obj);
+    const int64_t n_pad64 = n_pad;
     const float* fmap = reinterpret_cast<const float*>(a.state + a.off_fmap);
     const float* gxs = reinterpret_cast<const float*>(a.state + a.off_xs);
     const float* gils = reinterpret_cast<const float*>(a.state + a.off_ils);
@@ -145,7 +75,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     const float4* glinv = reinterpret_cast<const float4*>(a.state + a.off_linv);
     const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
 
-    if (EPI == kEHVI) stage_boxes(a, M, blo, bhi, epsv);  // visible after the first barrier below
+    if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);  // visible after the first barrier below
 
     // Per-dimension feature map (uniform across the block).
     int kind[kMaxD];
@@ -169,11 +99,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
         for (int c = 0; c < kMaxD; ++c) {
             u[c] = 0.0f;
             if (c < a.d && live) {
-                const uint32_t w = __ldg(a.cand + (int64_t)c * a.ld + i);
-                if (kind[c] == SCOOT_INT_LOG) u[c] = (logf((float)(int32_t)w) - fa[c]) * fb[c];
-                else if (kind[c] == SCOOT_INT_UNIFORM) u[c] = ((float)(int32_t)w - fa[c]) * fb[c];
-                else if (kind[c] == SCOOT_CONTINUOUS) u[c] = (__uint_as_float(w) - fa[c]) * fb[c];
-                else u[c] = (float)(int32_t)w;
+                u[c] = feature_of(__ldg(a.cand + (int64_t)c * a.ld + i), kind[c], fa[c], fb[c]);
             }
         }
         float mu[kMaxM], vr[kMaxM];
@@ -257,6 +183,20 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 for (int r = 0; r < 8; ++r)
 #pragma unroll
                     for (int c = 0; c < 8; ++c) sq[c] = fmaf(accm[r][c], accm[r][c], sq[c]);
+                if (EPI == kWriteWhitened) {
+                    // Rows of V for the fantasy downdates, indexed by list position.
+#pragma unroll
+                    for (int r = 0; r < 8; ++r) {
+                        const int row = rb * kRB + rg * 8 + r;
+                        if (row >= a.n_obs) continue;
+                        float* dst = a.vout + ((int64_t)m * n_pad64 + row) * a.ldv;
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            const int64_t p = tile * kTC + cg * 8 + c;
+                            if (p < n_work) dst[p] = accm[r][c];
+                        }
+                    }
+                }
             }
 #pragma unroll
             for (int c = 0; c < 8; ++c) part[rg * kTC + cg * 8 + c] = sq[c];
@@ -272,6 +212,12 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 for (int m = 0; m < nobj; ++m) {
                     a.mean[(int64_t)m * a.ldo + i] = mu[m];
                     a.var[(int64_t)m * a.ldo + i] = vr[m];
+                }
+        } else if (EPI == kWriteWhitened) {
+            if (live)
+                for (int m = 0; m < nobj; ++m) {
+                    a.mean[(int64_t)m * a.ldo + pos] = mu[m];
+                    a.var[(int64_t)m * a.ldo + pos] = vr[m];
                 }
         } else if (EPI == kEI) {
             if (live) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
@@ -301,7 +247,7 @@ ehvi_kernel(const __grid_constant__ ScoreArgs a) {
     float4* blo = reinterpret_cast<float4*>(sm);
     float4* bhi = blo + a.n_boxes;
     float4* epsv = bhi + a.n_boxes;
-    stage_boxes(a, M, blo, bhi, epsv);
+    stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
     __syncthreads();
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
     for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < n_work;
@@ -400,6 +346,26 @@ scoot_status dispatch_m(scoot_ctx* ctx, const ScoreArgs& a, int M, cudaStream_t 
 }
 
 }  // namespace
+
+scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                                      const uint32_t* cand, int64_t n, int64_t ld, const int32_t* list,
+                                      const unsigned int* n_list, float* mean, float* var, float* V, int64_t ldc,
+                                      cudaStream_t st) {
+    ScoreArgs a;
+    scoot_status s = fill_state_args(ctx, L, state, a);
+    if (s != SCOOT_OK) return s;
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.list = list;
+    a.n_list = n_list;
+    a.mean = mean;
+    a.var = var;
+    a.ldo = ldc;
+    a.vout = V;
+    a.ldv = ldc;
+    return launch_score<kWriteWhitened, 1>(ctx, a, st);
+}
 
 extern "C" {
 

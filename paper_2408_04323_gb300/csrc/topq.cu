@@ -14,28 +14,15 @@
 // The per-block lists live in the context's workspace.
 #include <mutex>
 
+#include "device_common.cuh"
 #include "internal.h"
 
 namespace {
 
+using namespace scoot_dev;
+
 constexpr int kTopqThreads = 128;
 constexpr int kMergeThreads = 256;
-
-__device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
-    uint32_t b = __float_as_uint(v);
-    b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-    return ((uint64_t)b << 32) | (uint64_t)(0xFFFFFFFFu - idx);
-}
-
-__device__ __forceinline__ float key_value(uint64_t k) {
-    uint32_t b = (uint32_t)(k >> 32);
-    b = (b & 0x80000000u) ? (b & 0x7FFFFFFFu) : ~b;
-    return __uint_as_float(b);
-}
-
-__device__ __forceinline__ int64_t key_index(uint64_t k) {
-    return (int64_t)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFu));
-}
 
 template <int QT>
 __device__ __forceinline__ void insert(uint64_t (&lst)[QT], uint64_t x) {

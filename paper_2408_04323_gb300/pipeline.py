@@ -36,6 +36,7 @@ class RoundInputs:
     q: int
     kernel: int = S.MATERN52
     xi: float = 1e-4
+    fantasy: bool = False      # q sequential picks with kriging-believer fantasies
 
 
 class State:
@@ -82,9 +83,23 @@ class ScoringRound:
         self.top_idx = torch.empty(q, dtype=torch.int64, device=dev)
         self.top_val = torch.empty(q, dtype=torch.float32, device=dev)
         self.top_count = torch.empty(1, dtype=torch.int32, device=dev)
+        self.work = None
+        if inp.fantasy:
+            nbytes = S.scoot_fantasy_work_bytes(self.state.gp_layout, self.capacity, q)
+            self.work = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        self.picks = None
 
-    # number of library kernels one call of run() launches
-    KERNELS_PER_ROUND = 5
+    # number of library kernels one call of run() launches (plain top-q rounds)
+    KERNELS_PER_ROUND = 7
+
+    def kernels_per_round(self):
+        """Library kernel launches of one run(): prune, compaction, forest walk, then
+        either compaction + fused score + two top-q passes, or (fantasies)
+        compaction + posterior + per pick EHVI, two argmax passes and a downdate
+        (the last pick skips the downdate)."""
+        if not self.inp.fantasy:
+            return 7
+        return 3 + 2 + 4 * self.inp.q - 1
 
     def run(self, cand: torch.Tensor, n: int, stream=None):
         """prune -> rf -> score -> top-q on a resident pool cand (int32 [d][ld])."""
@@ -94,6 +109,16 @@ class ScoringRound:
         S.scoot_prune(self.ctx, inp.space, inp.clauses, cand, n, self.mask, self.n_known, stream)
         S.scoot_rf_predict(self.ctx, st.forest_layout, st.forest, inp.space, cand, n, inp.delta_num,
                            inp.delta_den, self.votes, self.mask, self.n_feasible, stream)
+        if inp.fantasy:
+            idx, val = S.scoot_suggest_fantasy(self.ctx, st.gp_layout, st.gp_state, inp.space, inp.x_obs, inp.y_obs,
+                                               inp.lengthscale, inp.signal_var, inp.noise_var, cand, n, inp.ref,
+                                               st.eps, inp.q, self.work, mask=self.mask, stream=stream)
+            self.picks = (idx, val)
+            k = len(idx)
+            self.top_idx[:k].copy_(torch.from_numpy(idx))
+            self.top_val[:k].copy_(torch.from_numpy(val))
+            self.top_count.fill_(k)
+            return self.top_idx, self.top_val, self.top_count
         if inp.acq == "ei":
             S.scoot_score_ei(self.ctx, st.gp_layout, st.gp_state, cand, n, inp.xi, self.acq, self.mask, stream)
         else:

@@ -85,6 +85,9 @@ _PROTOS = {
                          _vp, _i32, _vp, _vp],
     "scoot_select_topq": [_vp, _vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
     "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
+    "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, C.POINTER(_i64)],
+    "scoot_suggest_fantasy": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _vp, _i64, _vp, _vp, _vp, _vp,
+                              _vp, _i64, _i64, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _vp, _vp, _vp, _vp, _vp],
 }
 _STRING_FUNCS = {"scoot_last_error", "scoot_status_string"}
 EXPORTS = tuple(_PROTOS)
@@ -342,3 +345,29 @@ def scoot_select_topq_static(acq, n, q, idx, val, count, mask=None, stream=None)
                                           int(n), int(q), _dev(idx, torch.int64, "idx"),
                                           _dev(val, torch.float32, "val"), _dev(count, torch.int32, "count"),
                                           _stream(stream)), "scoot_select_topq_static")
+
+
+def scoot_fantasy_work_bytes(layout, n: int, q: int) -> int:
+    v = _i64()
+    _check(lib().scoot_fantasy_work_bytes(C.byref(layout), int(n), int(q), C.byref(v)), "scoot_fantasy_work_bytes")
+    return int(v.value)
+
+
+def scoot_suggest_fantasy(ctx, layout, state, h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var,
+                          cand, n, h_ref, eps, q, work, mask=None, var_out=None, stream=None):
+    """Returns (idx int64[count], val float32[count]) of q sequential fantasised picks."""
+    import torch
+    idx = np.full(q, -1, np.int64)
+    val = np.full(q, -np.inf, np.float32)
+    cnt = _i32()
+    _check(lib().scoot_suggest_fantasy(
+        _h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"), _host(h_space, 16, name="h_space"),
+        _host(h_x_obs, 4, name="h_x_obs"), int(h_x_obs.shape[1]), _host(h_y, dtype=np.float32, name="h_y"),
+        _host(h_lengthscale, dtype=np.float32, name="h_lengthscale"),
+        _host(h_signal_var, dtype=np.float32, name="h_signal_var"),
+        _host(h_noise_var, dtype=np.float32, name="h_noise_var"), _dev(cand, torch.int32, "cand"), int(n),
+        int(cand.shape[1]), _dev(mask, torch.uint8, "mask"), _host(h_ref, dtype=np.float32, name="h_ref"),
+        _dev(eps, torch.float32, "eps"), int(eps.shape[0]), int(q), _vp(work.data_ptr()), int(work.numel()),
+        _host(idx), _host(val), C.byref(cnt), _dev(var_out, torch.float32, "var_out"), _stream(stream)),
+        "scoot_suggest_fantasy", _h(ctx))
+    return idx[:cnt.value], val[:cnt.value]

@@ -1,0 +1,93 @@
+"""Sequential fantasised picks (the q = 16 parallel-suggestion workload):
+the GPU's rank-1 downdates against the oracle's refit of the GP with the
+picked points appended, pick by pick."""
+import numpy as np
+import pytest
+
+import oracle as O
+from workloads import make_instance, seeds
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from parity_tol import ATOL, RTOL, posterior_tols, propagated_tol  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def S():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2408_04323_gb300 as pkg
+    pkg.build()
+    from paper_2408_04323_gb300 import scoot
+    return scoot
+
+
+@pytest.mark.parametrize("seed_i,n,q", [(0, 2048, 16), (1, 1500, 6)])
+def test_fantasy_picks_follow_the_refit_oracle(S, seed_i, n, q):
+    name = "d12-fantasy"
+    inst = make_instance(name, seeds(name)[seed_i], n_cand=n)
+    w = inst.workload
+    ctx = S.Context(0)
+    try:
+        cand = torch.from_numpy(inst.cand.view(np.int32)).cuda()
+        mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+        S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
+        L = S.scoot_forest_layout_init(inst.nodes, inst.tree_offset, inst.d, w.leaf_scale)
+        forest = torch.from_numpy(S.scoot_forest_pack(L, inst.nodes, inst.tree_offset)).cuda()
+        votes = torch.empty(n, dtype=torch.int32, device="cuda")
+        S.scoot_rf_predict(ctx, L, forest, inst.space, cand, n, w.delta_num, w.delta_den, votes, mask)
+        G = S.scoot_gp_layout_init(inst.n_obs, inst.d, inst.n_obj)
+        blob, _ = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                     inst.noise_var, G)
+        state = torch.from_numpy(blob).cuda()
+        work = torch.empty(S.scoot_fantasy_work_bytes(G, n, q), dtype=torch.uint8, device="cuda")
+        var_out = torch.full((inst.n_obj, n), -1.0, device="cuda")
+        eps = torch.from_numpy(inst.eps).cuda()
+        idx, val = S.scoot_suggest_fantasy(ctx, G, state, inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
+                                           inst.signal_var, inst.noise_var, cand, n, inst.ref, eps, q, work,
+                                           mask=mask, var_out=var_out)
+        ctx.check()
+        feas_gpu = mask.cpu().numpy().astype(bool)
+    finally:
+        ctx.close()
+
+    known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
+    v = O.rf_votes(inst.nodes, inst.tree_offset, inst.space, inst.cand, n)
+    feas = known & O.pof_feasible(v, inst.n_trees, w.leaf_scale, w.delta_num, w.delta_den)
+    assert np.array_equal(feas_gpu, feas)
+    ref = O.fantasy_picks(inst, q, feas)
+    assert len(idx) == len(ref["picks"]) == min(q, int(feas.sum()))
+    gps = [O.GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m], inst.signal_var[m],
+                inst.noise_var[m]) for m in range(inst.n_obj)]
+
+    def value_tol(j, i):
+        """The oracle's step-j EHVI of candidate i and its propagated tolerance."""
+        _, _, e_mu, _ = posterior_tols(gps, np.ascontiguousarray(inst.cand[:, [i]]))
+        mu = ref["mu"][j][[i]]
+        var = ref["var"][j][[i]]
+        f = lambda a_, b_: O.ehvi_mc(a_, b_, inst.eps, ref["fronts"][j], inst.ref)
+        return propagated_tol(f, mu, var, e_mu, ATOL + RTOL * var)
+
+    same = 0
+    for j, (g, o) in enumerate(zip(idx.tolist(), ref["picks"])):
+        want_g, tol_g = value_tol(j, g)
+        print(f"[fantasy] pick {j}: gpu {g} ({val[j]:.7g}) oracle {o} ({ref['acq'][j][o]:.7g}) "
+              f"|err|/tol={abs(float(val[j]) - want_g[0]) / tol_g[0]:.3f}")
+        # the GPU's value at its pick is the oracle's value there, within tolerance
+        assert abs(float(val[j]) - want_g[0]) <= tol_g[0]
+        if g != o:
+            # a different pick is only allowed on a near-tie of the oracle's values
+            want_o, tol_o = value_tol(j, o)
+            assert want_g[0] >= want_o[0] - tol_g[0] - tol_o[0]
+            break
+        same += 1
+    print(f"[fantasy] {same} of {len(idx)} picks identical")
+    if same == len(idx) and len(idx) > 1:
+        # variances after the downdates of picks 0 .. q-2, against the refit
+        gv = var_out.cpu().numpy().astype(np.float64)[:, feas].T
+        ov = ref["var"][-1][feas]
+        err = np.abs(gv - ov) / (ATOL + RTOL * np.abs(ov))
+        print(f"[fantasy] variance after {len(idx) - 1} fantasies: max|err|/tol={err.max():.3f} "
+              f"max|err|={np.abs(gv - ov).max():.3e}")
+        assert err.max() <= 1.0

@@ -22,8 +22,7 @@ from workloads import Stream, make_instance, seeds
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-ATOL, RTOL = 1e-6, 1e-4
-MU_COND = 2.0 ** -22
+from parity_tol import ATOL, MU_COND, RTOL, posterior_tols, propagated_tol  # noqa: E402
 
 
 @pytest.fixture(scope="module")
@@ -64,29 +63,6 @@ def report(name, g, o, extra=0.0):
     worst = float(ratio.max()) if ratio.size else 0.0
     print(f"[parity] {name}: n={g.size} max|err|/tol={worst:.3f} max|err|={np.abs(g - o).max() if g.size else 0:.3e}")
     return ratio
-
-
-def posterior_tols(gps, words):
-    """Oracle mu, var [K][M] and the tolerances of the GPU's mu and var."""
-    mv = [gp.posterior(words) for gp in gps]
-    mu = np.stack([a for a, _ in mv], 1)
-    var = np.stack([b for _, b in mv], 1)
-    cond = np.stack([gp.mean_condition(words) for gp in gps], 1)
-    e_mu = ATOL + RTOL * np.abs(mu) + MU_COND * cond
-    e_var = ATOL + RTOL * var
-    return mu, var, e_mu, e_var
-
-
-def propagated_tol(f, mu, var, e_mu, e_var):
-    """1e-6 + 1e-4 |f| plus |f(mu +- e_mu)| and |f(var +- e_var)| half-differences."""
-    base = f(mu, var)
-    tol = ATOL + RTOL * np.abs(base)
-    for m in range(mu.shape[1]):
-        d = np.zeros_like(mu); d[:, m] = e_mu[:, m]
-        tol = tol + 0.5 * np.abs(f(mu + d, var) - f(mu - d, var))
-        d = np.zeros_like(var); d[:, m] = e_var[:, m]
-        tol = tol + 0.5 * np.abs(f(mu, var + d) - f(mu, np.maximum(var - d, 0.0)))
-    return base, tol
 
 
 def report_tol(name, g, o, tol):
