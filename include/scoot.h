@@ -191,9 +191,11 @@ typedef struct {
     int32_t n_rb;             /* row blocks of 64 in the tiled L^{-1} */
     int32_t n_tiles;          /* 32 x 64 tiles of L^{-1} per objective */
     int64_t bytes;
-    int64_t off_fmap;         /* float[d][4]: kind, a, b, 0 of the feature map */
-    int64_t off_xs;           /* float[M][n][d]: observed features scaled by 1/lengthscale */
-    int64_t off_ils;          /* float[M][d]: 1/l (ordinal dims) or 1/l^2 (categorical dims) */
+    int64_t off_fmap;         /* float[d][4]: kind, a, b, source parameter of each feature, ordinal
+                                 parameters first, then categorical ones ("feature order") */
+    int64_t off_xs;           /* float[M][n][d]: observed features in feature order, ordinal ones
+                                 scaled by 1/lengthscale, categorical ones as the category index */
+    int64_t off_ils;          /* float[M][d]: 1/l (ordinal) or 1/l^2 (categorical), feature order */
     int64_t off_alpha;        /* float[M][n] */
     int64_t off_linv;         /* float[M][n_tiles][32][64]: L^{-1} tiles, transposed, zero-filled */
     int64_t off_scal;         /* float[M][4]: signal variance, noise variance, best observed y, 0 */

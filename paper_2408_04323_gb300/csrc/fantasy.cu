@@ -143,8 +143,9 @@ __global__ void __launch_bounds__(kFThreads) fant_update(const __grid_constant__
         for (int m = 0; m < M; ++m) r2[m] = 0.0f;
         for (int c = 0; c < a.d; ++c) {
             const int kind = (int)fmap[c * 4];
-            const float ux = feature_of(__ldg(a.cand + (int64_t)c * a.ld + i), kind, fmap[c * 4 + 1], fmap[c * 4 + 2]);
-            const float up = feature_of(__ldg(a.cand + (int64_t)c * a.ld + a.p), kind, fmap[c * 4 + 1], fmap[c * 4 + 2]);
+            const int64_t col = (int64_t)fmap[c * 4 + 3];  // features are in feature order
+            const float ux = feature_of(__ldg(a.cand + col * a.ld + i), kind, fmap[c * 4 + 1], fmap[c * 4 + 2]);
+            const float up = feature_of(__ldg(a.cand + col * a.ld + a.p), kind, fmap[c * 4 + 1], fmap[c * 4 + 2]);
 #pragma unroll
             for (int m = 0; m < M; ++m) {
                 const float s = gils[m * a.d + c];

@@ -228,8 +228,16 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
 
     char* blob = static_cast<char*>(h_blob);
     std::memset(blob, 0, (size_t)L->bytes);
+    // Feature order: ordinal parameters first, then categorical ones, so the
+    // kernels' distance loops need no per-dimension branch on the kind.
+    std::vector<int> order;
+    for (int c = 0; c < d; ++c)
+        if (h_space[c].kind != SCOOT_CATEGORICAL) order.push_back(c);
+    for (int c = 0; c < d; ++c)
+        if (h_space[c].kind == SCOOT_CATEGORICAL) order.push_back(c);
     float* fmap = reinterpret_cast<float*>(blob + L->off_fmap);
-    for (int c = 0; c < d; ++c) {
+    for (int f = 0; f < d; ++f) {
+        const int c = order[f];
         const scoot_param& p = h_space[c];
         float a = 0.f, b = 0.f;
         if (p.kind == SCOOT_INT_LOG) {
@@ -239,9 +247,10 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
             a = p.lo;
             b = p.hi > p.lo ? (float)(1.0 / ((double)p.hi - (double)p.lo)) : 0.0f;
         }
-        fmap[c * 4 + 0] = (float)p.kind;
-        fmap[c * 4 + 1] = a;
-        fmap[c * 4 + 2] = b;
+        fmap[f * 4 + 0] = (float)p.kind;
+        fmap[f * 4 + 1] = a;
+        fmap[f * 4 + 2] = b;
+        fmap[f * 4 + 3] = (float)c;
     }
 
     float* xs = reinterpret_cast<float*>(blob + L->off_xs);
@@ -257,11 +266,12 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
                                        h_lengthscale + (size_t)m * d, h_signal_var[m], h_noise_var[m],
                                        L->kernel, &g, h_cond ? &h_cond[m] : nullptr);
         if (s != SCOOT_OK) return s;
-        for (int c = 0; c < d; ++c) {
+        for (int f = 0; f < d; ++f) {
+            const int c = order[f];
             const double l = g.ell[c];
-            ils[m * d + c] = g.cat[c] ? (float)(1.0 / (l * l)) : (float)(1.0 / l);
+            ils[m * d + f] = g.cat[c] ? (float)(1.0 / (l * l)) : (float)(1.0 / l);
             for (int j = 0; j < n; ++j)
-                xs[((size_t)m * n + j) * d + c] = g.cat[c] ? (float)g.u[(size_t)j * d + c]
+                xs[((size_t)m * n + j) * d + f] = g.cat[c] ? (float)g.u[(size_t)j * d + c]
                                                            : (float)(g.u[(size_t)j * d + c] / l);
         }
         for (int i = 0; i < n; ++i) alpha_out[(size_t)m * n + i] = (float)g.alpha[i];

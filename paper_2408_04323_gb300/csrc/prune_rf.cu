@@ -8,18 +8,14 @@ namespace {
 
 constexpr int kPruneThreads = 256;
 constexpr int kRfThreads = 256;
-constexpr int kRfPerThread = 2;                  // candidates walked together (ILP)
-constexpr int kRfTile = kRfThreads * kRfPerThread;
+constexpr int kRfGroups = 4;                     // threads (tree groups) per candidate
+constexpr int kRfCand = kRfThreads / kRfGroups;  // candidates per tile
 
 struct PruneArgs {
     int32_t n_clauses;
     int32_t pad;
     scoot_clause cl[SCOOT_MAX_CLAUSES];
 };
-
-__device__ __forceinline__ int4 ld_col4(const uint32_t* __restrict__ cand, int64_t ld, int p, int64_t i0) {
-    return __ldg(reinterpret_cast<const int4*>(cand + (int64_t)p * ld + i0));
-}
 
 // Block-wide sum of per-thread counts, added once per block to *count.
 __device__ __forceinline__ void add_count(unsigned long long* count, uint32_t mine) {
@@ -35,52 +31,31 @@ __device__ __forceinline__ void add_count(unsigned long long* count, uint32_t mi
     }
 }
 
-// One thread evaluates every clause on four consecutive candidates, reading
-// each referenced column as one 16-byte load (ld % 4 == 0, columns aligned).
+// One thread per candidate: every clause is evaluated with exact 128-bit
+// integer sums; column reads are coalesced 4-byte loads (repeated columns hit
+// L1).  One candidate per thread keeps enough warps in flight to cover the
+// load latency even for pools of a few hundred thousand candidates.
 __global__ void __launch_bounds__(kPruneThreads)
 prune_kernel(const __grid_constant__ PruneArgs a, const uint32_t* __restrict__ cand, int64_t n,
              int64_t ld, uint8_t* __restrict__ mask, unsigned long long* count) {
-    const int64_t n4 = (n + 3) >> 2;
     uint32_t feasible = 0;
-    const bool vec_store = (reinterpret_cast<uintptr_t>(mask) & 3u) == 0;
-    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < n4;
-         q += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t i0 = q << 2;
-        bool ok0 = true, ok1 = true, ok2 = true, ok3 = true;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        bool ok = true;
         for (int c = 0; c < a.n_clauses; ++c) {
             const scoot_clause& C = a.cl[c];
-            bool g0 = true, g1 = true, g2 = true, g3 = true;
-            for (int k = 0; k < C.n_guard; ++k) {
-                int4 v = ld_col4(cand, ld, C.guard_param[k], i0);
-                const int gv = C.guard_value[k];
-                g0 &= v.x == gv; g1 &= v.y == gv; g2 &= v.z == gv; g3 &= v.w == gv;
-            }
-            if (!(g0 | g1 | g2 | g3)) continue;
-            __int128 s0 = 0, s1 = 0, s2 = 0, s3 = 0;
-            for (int t = 0; t < C.n_term; ++t) {
-                int4 v = ld_col4(cand, ld, C.term_param[t], i0);
-                const __int128 k = C.coef[t];
-                s0 += k * v.x; s1 += k * v.y; s2 += k * v.z; s3 += k * v.w;
-            }
-            const __int128 r = C.rhs;
-            ok0 &= !g0 || s0 >= r; ok1 &= !g1 || s1 >= r;
-            ok2 &= !g2 || s2 >= r; ok3 &= !g3 || s3 >= r;
+            bool g = true;
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+                if (k < C.n_guard) g &= (int32_t)__ldg(cand + (int64_t)C.guard_param[k] * ld + i) == C.guard_value[k];
+            if (!g) continue;
+            __int128 sum = 0;
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+                if (t < C.n_term) sum += (__int128)C.coef[t] * (int32_t)__ldg(cand + (int64_t)C.term_param[t] * ld + i);
+            ok &= sum >= (__int128)C.rhs;
         }
-        const uint8_t m0 = ok0, m1 = ok1, m2 = ok2, m3 = ok3;
-        if (i0 + 3 < n) {
-            feasible += m0 + m1 + m2 + m3;
-            if (vec_store) {
-                *reinterpret_cast<uchar4*>(mask + i0) = make_uchar4(m0, m1, m2, m3);
-            } else {
-                mask[i0] = m0; mask[i0 + 1] = m1; mask[i0 + 2] = m2; mask[i0 + 3] = m3;
-            }
-        } else {
-            const uint8_t mm[4] = {m0, m1, m2, m3};
-            for (int k = 0; k < 4 && i0 + k < n; ++k) {
-                mask[i0 + k] = mm[k];
-                feasible += mm[k];
-            }
-        }
+        mask[i] = ok;
+        feasible += ok;
     }
     if (count) add_count(count, feasible);
 }
@@ -102,58 +77,53 @@ struct RfArgs {
     const unsigned int* n_list;
 };
 
-// Persistent blocks: each stages (a chunk of) the forest in shared memory,
-// then walks tiles of kRfTile candidates whose feature values sit in shared
-// memory as feat[c][slot] (bank = slot % 32, so lanes never conflict).
+// Persistent blocks of 256 threads score tiles of 64 candidates; thread t
+// serves candidate slot t / 4 and walks the trees of group t % 4 (trees
+// g, g + 4, ...), so a block has four independent walks per candidate and a
+// pool of ~10^5 live candidates still fills every SM.  The forest (or one
+// chunk of whole trees at a time) sits in shared memory; each tile's feature
+// values sit in shared memory as feat[slot][f] with an odd row stride.  The
+// four partial vote counts of a candidate are added with warp shuffles.
 __global__ void __launch_bounds__(kRfThreads)
 rf_kernel(const __grid_constant__ RfArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    float* sfeat = reinterpret_cast<float*>(smem_raw);                       // [d][kRfTile]
-    uint2* snodes = reinterpret_cast<uint2*>(sfeat + a.d * kRfTile);         // chunk nodes
+    const int fs = a.d | 1;                                                   // odd row stride
+    float* sfeat = reinterpret_cast<float*>(smem_raw);                        // [kRfCand][fs]
+    uint2* snodes = reinterpret_cast<uint2*>(sfeat + ((kRfCand * fs + 1) & ~1));  // chunk nodes
 
     const int32_t* chunks = reinterpret_cast<const int32_t*>(a.forest + a.off_chunks);
     const int32_t* roots = reinterpret_cast<const int32_t*>(a.forest + a.off_roots);
     const uint2* gnodes = reinterpret_cast<const uint2*>(a.forest + a.off_nodes);
     const int tid = threadIdx.x;
+    const int slot = tid / kRfGroups, grp = tid % kRfGroups;
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
-    const int64_t n_tiles = (n_work + kRfTile - 1) / kRfTile;
+    const int64_t n_tiles = (n_work + kRfCand - 1) / kRfCand;
     uint32_t feasible = 0;
 
     auto stage_chunk = [&](int ch) {
         const int first_node = chunks[ch * 4 + 2], count = chunks[ch * 4 + 3];
         for (int k = tid; k < count; k += kRfThreads) snodes[k] = __ldg(gnodes + first_node + k);
     };
-    if (a.single_chunk) {
-        stage_chunk(0);
-        __syncthreads();
-    }
+    if (a.single_chunk) stage_chunk(0);  // visible after the first barrier below
 
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-        const int64_t base = tile * kRfTile;
-        int64_t idx[kRfPerThread];
-        bool live[kRfPerThread];
-#pragma unroll
-        for (int r = 0; r < kRfPerThread; ++r) {
-            const int64_t pos = base + tid + r * kRfThreads;
-            live[r] = pos < n_work;
-            idx[r] = live[r] ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
-        }
-        for (int c = 0; c < a.d; ++c) {
-            const bool isf = (a.float_cols >> c) & 1u;
-#pragma unroll
-            for (int r = 0; r < kRfPerThread; ++r) {
-                float x = 0.0f;
-                if (live[r]) {
-                    uint32_t w = __ldg(a.cand + (int64_t)c * a.ld + idx[r]);
-                    x = isf ? __uint_as_float(w) : (float)(int32_t)w;
-                }
-                sfeat[c * kRfTile + tid + r * kRfThreads] = x;
+        const int64_t base = tile * kRfCand;
+        __syncthreads();  // the previous tile's features are no longer read
+        for (int k = tid; k < kRfCand * a.d; k += kRfThreads) {
+            const int f = k / kRfCand, c = k - f * kRfCand;
+            const int64_t pos = base + c;
+            float x = 0.0f;
+            if (pos < n_work) {
+                const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+                const uint32_t w = __ldg(a.cand + (int64_t)f * a.ld + i);
+                x = ((a.float_cols >> f) & 1u) ? __uint_as_float(w) : (float)(int32_t)w;
             }
+            sfeat[c * fs + f] = x;
         }
-        uint32_t vote[kRfPerThread];
-#pragma unroll
-        for (int r = 0; r < kRfPerThread; ++r) vote[r] = 0u;
-
+        const int64_t pos = base + slot;
+        const bool live = pos < n_work;
+        const float* my = sfeat + slot * fs;
+        uint32_t vote = 0;
         for (int ch = 0; ch < a.n_chunks; ++ch) {
             if (!a.single_chunk) {
                 __syncthreads();
@@ -161,49 +131,35 @@ rf_kernel(const __grid_constant__ RfArgs a) {
             }
             __syncthreads();
             const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1], node0 = chunks[ch * 4 + 2];
-            for (int t = t0; t < t0 + nt; ++t) {
+            if (!live) continue;
+            for (int t = t0 + grp; t < t0 + nt; t += kRfGroups) {
                 const int root = roots[t] - node0;
-                int node[kRfPerThread];
-                bool done[kRfPerThread];
-#pragma unroll
-                for (int r = 0; r < kRfPerThread; ++r) {
-                    node[r] = root;
-                    done[r] = !live[r];
-                }
+                int node = root;
+                bool done = false;
                 for (int step = 0; step <= a.max_depth; ++step) {
-                    bool all_done = true;
-#pragma unroll
-                    for (int r = 0; r < kRfPerThread; ++r) {
-                        if (!done[r]) {
-                            const uint2 nd = snodes[node[r]];
-                            if ((nd.y >> 24) & 1u) {
-                                vote[r] += (uint32_t)__uint_as_float(nd.x);
-                                done[r] = true;
-                            } else {
-                                const int feat = (nd.y >> 16) & 0xff;
-                                const float x = sfeat[feat * kRfTile + tid + r * kRfThreads];
-                                node[r] = root + (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
-                            }
-                        }
-                        all_done &= done[r];
+                    const uint2 nd = snodes[node];
+                    if ((nd.y >> 24) & 1u) {
+                        vote += (uint32_t)__uint_as_float(nd.x);
+                        done = true;
+                        break;
                     }
-                    if (all_done) break;
+                    const float x = my[(nd.y >> 16) & 0xff];
+                    node = root + (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
                 }
-#pragma unroll
-                for (int r = 0; r < kRfPerThread; ++r)
-                    if (!done[r]) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
+                if (!done) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
             }
         }
-        const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
-#pragma unroll
-        for (int r = 0; r < kRfPerThread; ++r) {
-            if (!live[r]) continue;
-            a.votes[idx[r]] = vote[r];
-            const bool ok = (unsigned __int128)a.delta_den * vote[r] >= need;
-            if (a.mask) a.mask[idx[r]] = ok;
+        // add the group partials (the four threads of a slot are adjacent lanes)
+        vote += __shfl_xor_sync(0xffffffffu, vote, 1);
+        vote += __shfl_xor_sync(0xffffffffu, vote, 2);
+        if (live && grp == 0) {
+            const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+            const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
+            a.votes[i] = vote;
+            const bool ok = (unsigned __int128)a.delta_den * vote >= need;
+            if (a.mask) a.mask[i] = ok;
             feasible += ok;
         }
-        __syncthreads();  // sfeat is rewritten by the next tile
     }
     if (a.count) add_count(a.count, feasible);
 }
@@ -252,9 +208,8 @@ scoot_status scoot_prune(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (n_feasible) SCOOT_CUDA(ctx, cudaMemsetAsync(n_feasible, 0, sizeof(int64_t), st));
     if (n == 0) return SCOOT_OK;
-    const int64_t n4 = (n + 3) / 4;
-    int64_t blocks = (n4 + kPruneThreads - 1) / kPruneThreads;
-    const int64_t cap = (int64_t)sm_count(ctx->device) * 8;
+    int64_t blocks = (n + kPruneThreads - 1) / kPruneThreads;
+    const int64_t cap = (int64_t)sm_count(ctx->device) * 16;
     if (blocks > cap) blocks = cap;
     prune_kernel<<<(unsigned)blocks, kPruneThreads, 0, st>>>(
         a, cand, n, ld, mask, reinterpret_cast<unsigned long long*>(n_feasible));
@@ -312,12 +267,12 @@ scoot_status scoot_rf_predict(scoot_ctx* ctx, const scoot_forest_layout* L, cons
         a.list = lst.list;
         a.n_list = lst.count;
     }
-    const size_t smem = (size_t)L->d * kRfTile * 4 + (size_t)max_chunk_nodes * 8;
+    const size_t smem = (size_t)((kRfCand * (L->d | 1) + 1) & ~1) * 4 + (size_t)max_chunk_nodes * 8;
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(rf_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;
     SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rf_kernel, kRfThreads, smem));
     if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "forest chunk does not fit in shared memory");
-    const int64_t tiles = (n + kRfTile - 1) / kRfTile;
+    const int64_t tiles = (n + kRfCand - 1) / kRfCand;
     int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
     if (blocks > tiles) blocks = tiles;
     rf_kernel<<<(unsigned)blocks, kRfThreads, smem, st>>>(a);

@@ -19,7 +19,8 @@ namespace {
 
 using namespace scoot_dev;
 
-constexpr int kTC = 64;     // candidates per tile = threads per block
+constexpr int kTC = 64;     // candidates per tile
+constexpr int kThreads = 128;  // two threads per candidate
 constexpr int kRB = 64;     // rows of L^{-1} per tile
 constexpr int kCJ = 32;     // columns of L^{-1} per tile
 constexpr int kMaxD = SCOOT_MAX_DIM;
@@ -51,138 +52,185 @@ struct ScoreArgs {
     int64_t ldv;
 };
 
-template <int EPI, int M>
-__global__ void __launch_bounds__(kTC)
+// Partial EHVI sum of one candidate over the sample chunks first, first +
+// stride, ... (chunks of eight samples, padding samples at -inf).
+template <int M>
+__device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, const float4* blo, const float4* bhi,
+                                             int n_boxes, const float4* eps, int n_mc, int first, int stride) {
+    constexpr int kCh = 8;
+    float total = 0.0f;
+    for (int s0 = first * kCh; s0 < n_mc; s0 += stride * kCh) {
+        float y[kCh][M], acc[kCh];
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) {
+            acc[k] = 0.0f;
+            const bool in = s0 + k < n_mc;
+            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float ev[4] = {e.x, e.y, e.z, e.w};
+#pragma unroll
+            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
+        }
+        for (int b = 0; b < n_boxes; ++b) {
+            const float4 lo4 = blo[b], hi4 = bhi[b];
+            const float lo[4] = {lo4.x, lo4.y, lo4.z, lo4.w};
+            const float hi[4] = {hi4.x, hi4.y, hi4.z, hi4.w};
+#pragma unroll
+            for (int k = 0; k < kCh; ++k) {
+                float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+#pragma unroll
+                for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
+                acc[k] += p;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) total += acc[k];
+    }
+    return total;
+}
+
+// One block of 128 threads scores a tile of 64 candidates; thread t works on
+// candidate slot t % 64 with its partner t +- 64 ("half" t / 64):
+//  1. both halves compute the candidate's features; for each objective the
+//     halves split the covariance row k(x, X_j) (j even / odd) into Ks[j][slot]
+//     and the partial sums of mu = k . alpha;
+//  2. all 128 threads compute V = L^{-1} Ks over 32 x 64 tiles of L^{-1} with a
+//     4-candidate x 8-row register tile each; a warp whose 16 rows lie wholly
+//     above a tile's columns (upper triangle, all zero) skips that tile;
+//     sigma^2 = s_f^2 - sum_i V_i^2;
+//  3. the epilogue (EI on one half, EHVI with the halves splitting the
+//     sample chunks, or the moments / whitened rows) writes the tile.
+// DM >= d bounds the per-dimension register arrays; features come in feature
+// order (ordinal parameters first), so the distance loop has no kind branch.
+template <int EPI, int M, int DM>
+__global__ void __launch_bounds__(kThreads)
 score_kernel(const __grid_constant__ ScoreArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
-    float* Ks = sm;                                   // [n_pad][kTC]
-    float* xs = Ks + (size_t)n_pad * kTC;             // [n_obs][dp]
-    float* al = xs + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3));   // [n_pad]
-    float* Lt = al + n_pad;                           // [kCJ][kRB]
-    float* part = Lt + kCJ * kRB;                     // [8][kTC]
-    float4* blo = reinterpret_cast<float4*>(part + 8 * kTC);
+    float* Ks = sm;                                                   // [n_pad][kTC]
+    float* xs = Ks + (size_t)n_pad * kTC;                             // [n_obs][dp]
+    float* al = xs + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3));     // [n_pad]
+    float* Lt = al + n_pad;                                           // [kCJ][kRB]
+    float* part = Lt + kCJ * kRB;                                     // [8][kTC]
+    float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [DM] feature map
+    float4* blo = fm + DM;
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
     float4* epsv = bhi + (EPI == kEHVI ? a.n_boxes : 0);
 
     const int tid = threadIdx.x;
+    const int slot = tid & (kTC - 1), half = tid >> 6;
+    const int warp = tid >> 5;
     const int nobj = EPI == kEHVI ? M : (EPI == kEI ? 1 : a.n_obj);
     const int64_t n_pad64 = n_pad;
-    const float* fmap = reinterpret_cast<const float*>(a.state + a.off_fmap);
+    const float4* gfmap = reinterpret_cast<const float4*>(a.state + a.off_fmap);
     const float* gxs = reinterpret_cast<const float*>(a.state + a.off_xs);
     const float* gils = reinterpret_cast<const float*>(a.state + a.off_ils);
     const float* galpha = reinterpret_cast<const float*>(a.state + a.off_alpha);
     const float4* glinv = reinterpret_cast<const float4*>(a.state + a.off_linv);
     const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
 
-    if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);  // visible after the first barrier below
-
-    // Per-dimension feature map (uniform across the block).
-    int kind[kMaxD];
-    float fa[kMaxD], fb[kMaxD];
+    if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
+    if (tid < DM) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
+    __syncthreads();
+    int n_ord = 0;
 #pragma unroll
-    for (int c = 0; c < kMaxD; ++c) {
-        kind[c] = c < a.d ? (int)fmap[c * 4] : SCOOT_CATEGORICAL;
-        fa[c] = c < a.d ? fmap[c * 4 + 1] : 0.f;
-        fb[c] = c < a.d ? fmap[c * 4 + 2] : 0.f;
-    }
+    for (int q = 0; q < DM; ++q) n_ord += (q < a.d && (int)fm[q].x != SCOOT_CATEGORICAL) ? 1 : 0;
 
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
     const int64_t n_tiles = (n_work + kTC - 1) / kTC;
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-        const int64_t pos = tile * kTC + tid;
+        const int64_t pos = tile * kTC + slot;
         const bool live = pos < n_work;
         const int64_t i = live ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
-        // Features of this thread's candidate.
-        float u[kMaxD];
+        float u[DM];
 #pragma unroll
-        for (int c = 0; c < kMaxD; ++c) {
-            u[c] = 0.0f;
-            if (c < a.d && live) {
-                u[c] = feature_of(__ldg(a.cand + (int64_t)c * a.ld + i), kind[c], fa[c], fb[c]);
+        for (int q = 0; q < DM; ++q) {
+            u[q] = 0.0f;
+            if (q < a.d && live) {
+                const float4 f = fm[q];
+                u[q] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + i), (int)f.x, f.y, f.z);
             }
         }
         float mu[kMaxM], vr[kMaxM];
         for (int m = 0; m < nobj; ++m) {
             __syncthreads();  // previous users of xs / al / part are done
             const float* sx = gxs + (size_t)m * a.n_obs * a.d;
-            for (int k = tid; k < a.n_obs * a.d; k += kTC) {
-                const int j = k / a.d, c = k - j * a.d;
-                xs[j * a.dp + c] = sx[k];
+            for (int k = tid; k < a.n_obs * a.d; k += kThreads) {
+                const int j = k / a.d, q = k - j * a.d;
+                xs[j * a.dp + q] = sx[k];
             }
-            for (int j = tid; j < n_pad; j += kTC) al[j] = j < a.n_obs ? galpha[(size_t)m * a.n_obs + j] : 0.0f;
+            for (int j = tid; j < n_pad; j += kThreads) al[j] = j < a.n_obs ? galpha[(size_t)m * a.n_obs + j] : 0.0f;
             const float sf2 = gscal[m * 4 + 0];
-            float ut[kMaxD], w2[kMaxD];
+            float ut[DM], w2[DM];
 #pragma unroll
-            for (int c = 0; c < kMaxD; ++c) {
-                const float s = c < a.d ? gils[m * a.d + c] : 0.0f;
-                const bool cat = kind[c] == SCOOT_CATEGORICAL;
-                ut[c] = cat ? u[c] : u[c] * s;
-                w2[c] = cat ? s : 0.0f;
+            for (int q = 0; q < DM; ++q) {
+                const float sc = q < a.d ? gils[m * a.d + q] : 0.0f;
+                ut[q] = q < n_ord ? u[q] * sc : u[q];
+                w2[q] = q < n_ord ? 0.0f : sc;
             }
             __syncthreads();
-            // 1. covariance row and mean.
+            // 1. covariance row (this half's j) and the partial mean.
             float acc = 0.0f;
 #pragma unroll 2
-            for (int j = 0; j < a.n_obs; ++j) {
+            for (int j = half; j < a.n_obs; j += 2) {
                 const float* xj = xs + j * a.dp;
                 float r2 = 0.0f;
 #pragma unroll
-                for (int c = 0; c < kMaxD; ++c) {
-                    if (c < a.d) {
-                        const float t = ut[c] - xj[c];
-                        if (kind[c] == SCOOT_CATEGORICAL) r2 += t != 0.0f ? w2[c] : 0.0f;
-                        else r2 = fmaf(t, t, r2);
+                for (int q = 0; q < DM; ++q)
+                    if (q < n_ord) {
+                        const float t = ut[q] - xj[q];
+                        r2 = fmaf(t, t, r2);
                     }
-                }
+#pragma unroll
+                for (int q = 0; q < DM; ++q)
+                    if (q >= n_ord && q < a.d) r2 += ut[q] != xj[q] ? w2[q] : 0.0f;
                 const float k = sf2 * matern(sqrtf(r2), a.kernel);
-                Ks[j * kTC + tid] = k;
+                Ks[j * kTC + slot] = k;
                 acc = fmaf(k, al[j], acc);
             }
-            for (int j = a.n_obs; j < n_pad; ++j) Ks[j * kTC + tid] = 0.0f;
-            mu[m] = acc;
+            for (int j = a.n_obs + half; j < n_pad; j += 2) Ks[j * kTC + slot] = 0.0f;
+            part[half * kTC + slot] = acc;
             __syncthreads();
-            // 2. V = L^{-1} Ks, sum of squares per candidate.
-            const int cg = tid & 7, rg = tid >> 3;
-            float sq[8];
-#pragma unroll
-            for (int c = 0; c < 8; ++c) sq[c] = 0.0f;
+            mu[m] = part[slot] + part[kTC + slot];
+            // 2. V = L^{-1} Ks and the sum of squares per candidate.
+            const int cg = tid & 15, rg = tid >> 4;
+            float sq[4] = {0.f, 0.f, 0.f, 0.f};
             const float4* tiles = glinv + (size_t)m * a.n_tiles * (kCJ * kRB / 4);
             const float4* Ks4 = reinterpret_cast<const float4*>(Ks);
             const float4* Lt4 = reinterpret_cast<const float4*>(Lt);
             int t = 0;
             for (int rb = 0; rb < a.n_rb; ++rb) {
-                float accm[8][8];
+                float accm[8][4];
 #pragma unroll
                 for (int r = 0; r < 8; ++r)
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) accm[r][c] = 0.0f;
+                    for (int c = 0; c < 4; ++c) accm[r][c] = 0.0f;
                 for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t) {
                     __syncthreads();
                     const float4* src = tiles + (size_t)t * (kCJ * kRB / 4);
 #pragma unroll
-                    for (int k = 0; k < kCJ * kRB / 4 / kTC; ++k)
-                        reinterpret_cast<float4*>(Lt)[tid + k * kTC] = __ldg(src + tid + k * kTC);
+                    for (int k = 0; k < kCJ * kRB / 4 / kThreads; ++k)
+                        reinterpret_cast<float4*>(Lt)[tid + k * kThreads] = __ldg(src + tid + k * kThreads);
                     __syncthreads();
+                    // rows of this warp: rb*64 + 16*warp .. +15; columns cj*32 .. +31
+                    if (cj * kCJ > rb * kRB + 16 * warp + 15) continue;
                     const int j0 = cj * kCJ;
 #pragma unroll 4
                     for (int jj = 0; jj < kCJ; ++jj) {
-                        const float4 k0 = Ks4[(j0 + jj) * (kTC / 4) + cg * 2];
-                        const float4 k1 = Ks4[(j0 + jj) * (kTC / 4) + cg * 2 + 1];
+                        const float4 k4 = Ks4[(j0 + jj) * (kTC / 4) + cg];
                         const float4 l0 = Lt4[jj * (kRB / 4) + rg * 2];
                         const float4 l1 = Lt4[jj * (kRB / 4) + rg * 2 + 1];
-                        const float kv[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
+                        const float kv[4] = {k4.x, k4.y, k4.z, k4.w};
                         const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
 #pragma unroll
                         for (int r = 0; r < 8; ++r)
 #pragma unroll
-                            for (int c = 0; c < 8; ++c) accm[r][c] = fmaf(lv[r], kv[c], accm[r][c]);
+                            for (int c = 0; c < 4; ++c) accm[r][c] = fmaf(lv[r], kv[c], accm[r][c]);
                     }
                 }
 #pragma unroll
                 for (int r = 0; r < 8; ++r)
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) sq[c] = fmaf(accm[r][c], accm[r][c], sq[c]);
+                    for (int c = 0; c < 4; ++c) sq[c] = fmaf(accm[r][c], accm[r][c], sq[c]);
                 if (EPI == kWriteWhitened) {
                     // Rows of V for the fantasy downdates, indexed by list position.
 #pragma unroll
@@ -191,42 +239,46 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                         if (row >= a.n_obs) continue;
                         float* dst = a.vout + ((int64_t)m * n_pad64 + row) * a.ldv;
 #pragma unroll
-                        for (int c = 0; c < 8; ++c) {
-                            const int64_t p = tile * kTC + cg * 8 + c;
+                        for (int c = 0; c < 4; ++c) {
+                            const int64_t p = tile * kTC + cg * 4 + c;
                             if (p < n_work) dst[p] = accm[r][c];
                         }
                     }
                 }
             }
+            __syncthreads();  // every thread has read its mean halves from part
 #pragma unroll
-            for (int c = 0; c < 8; ++c) part[rg * kTC + cg * 8 + c] = sq[c];
+            for (int c = 0; c < 4; ++c) part[rg * kTC + cg * 4 + c] = sq[c];
             __syncthreads();
             float ss = 0.0f;
 #pragma unroll
-            for (int g = 0; g < 8; ++g) ss += part[g * kTC + tid];
+            for (int g = 0; g < 8; ++g) ss += part[g * kTC + slot];
             vr[m] = fmaxf(sf2 - ss, 0.0f);
         }
-        // Epilogue.
+        // 3. epilogue.
         if (EPI == kWriteMoments) {
-            if (live)
+            if (live && half == 0)
                 for (int m = 0; m < nobj; ++m) {
                     a.mean[(int64_t)m * a.ldo + i] = mu[m];
                     a.var[(int64_t)m * a.ldo + i] = vr[m];
                 }
         } else if (EPI == kWriteWhitened) {
-            if (live)
+            if (live && half == 0)
                 for (int m = 0; m < nobj; ++m) {
                     a.mean[(int64_t)m * a.ldo + pos] = mu[m];
                     a.var[(int64_t)m * a.ldo + pos] = vr[m];
                 }
         } else if (EPI == kEI) {
-            if (live) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
+            if (live && half == 0) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
         } else {
             float sd[kMaxM];
 #pragma unroll
             for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
-            const float v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
-            if (live) a.acq[i] = v;
+            const float v = ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2);
+            __syncthreads();  // part is free again
+            part[half * kTC + slot] = v;
+            __syncthreads();
+            if (live && half == 0) a.acq[i] = (part[slot] + part[kTC + slot]) * (1.0f / (float)a.n_mc);
         }
     }
 }
@@ -295,9 +347,25 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
 
 size_t score_smem(const ScoreArgs& a, int epi) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
-    size_t f = n_pad * kTC + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3)) + n_pad + kCJ * kRB + 8 * kTC;
+    size_t f = n_pad * kTC + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3)) + n_pad + kCJ * kRB + 8 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
     return f * 4;
+}
+
+template <int EPI, int M, int DM>
+scoot_status launch_score_dm(scoot_ctx* ctx, const ScoreArgs& a, cudaStream_t st) {
+    const size_t smem = score_smem(a, EPI);
+    auto kern = score_kernel<EPI, M, DM>;
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    int per_sm = 0;
+    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));
+    if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "score kernel needs %zu bytes of shared memory", smem);
+    const int64_t tiles = (a.n + kTC - 1) / kTC;
+    int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
+    if (blocks > tiles) blocks = tiles;
+    kern<<<(unsigned)blocks, kThreads, smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
 }
 
 template <int EPI, int M>
@@ -312,18 +380,10 @@ scoot_status launch_score(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
         a.list = lst.list;
         a.n_list = lst.count;
     }
-    const size_t smem = score_smem(a, EPI);
-    auto kern = score_kernel<EPI, M>;
-    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    int per_sm = 0;
-    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kTC, smem));
-    if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "score kernel needs %zu bytes of shared memory", smem);
-    const int64_t tiles = (a.n + kTC - 1) / kTC;
-    int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
-    if (blocks > tiles) blocks = tiles;
-    kern<<<(unsigned)blocks, kTC, smem, st>>>(a);
-    SCOOT_LAUNCHED(ctx);
-    return SCOOT_OK;
+    if (a.d <= 4) return launch_score_dm<EPI, M, 4>(ctx, a, st);
+    if (a.d <= 8) return launch_score_dm<EPI, M, 8>(ctx, a, st);
+    if (a.d <= 12) return launch_score_dm<EPI, M, 12>(ctx, a, st);
+    return launch_score_dm<EPI, M, 16>(ctx, a, st);
 }
 
 scoot_status check_boxes(scoot_ctx* ctx, int M, const float* lo, const float* hi, int32_t B, const float* eps, int32_t S) {

@@ -309,7 +309,11 @@ def test_score_ehvi_parity(S, ctx, name, k):
         S.scoot_gp_posterior(ctx, L, state, cand, n, mean, var_d, mask)
         acq2 = torch.empty(n, device="cuda")
         S.scoot_acq_ehvi(ctx, mean, var_d, n, lo, hi, eps, acq2, mask)
-        assert np.array_equal(np_(acq2), g)
+        g2 = np_(acq2)
+        # same arithmetic, only the order of the sample sum differs
+        assert np.array_equal(np.isfinite(g2), np.isfinite(g))
+        fin = np.isfinite(g)
+        assert np.all(np.abs(g2[fin] - g[fin]) <= 1e-6 + 1e-5 * np.abs(g[fin]))
 
 
 def test_score_ei_parity(S, ctx):

@@ -110,9 +110,12 @@ def _unpack_gp(S, L, blob):
                 linv[m, rb * 64:(rb + 1) * 64, cj * 32:(cj + 1) * 32] = tiles[m, t].T
                 t += 1
     scal = f(L.off_scal, M * 4).reshape(M, 4)
-    xs = f(L.off_xs, M * n * d).reshape(M, n, d)
-    ils = f(L.off_ils, M * d).reshape(M, d)
-    return alpha, linv[:, :n, :n], scal, xs, ils
+    src = f(L.off_fmap, d * 4).reshape(d, 4)[:, 3].astype(int)  # feature order -> parameter
+    xs = np.zeros((M, n, d), np.float32)
+    ils = np.zeros((M, d), np.float32)
+    xs[:, :, src] = f(L.off_xs, M * n * d).reshape(M, n, d)
+    ils[:, src] = f(L.off_ils, M * d).reshape(M, d)
+    return alpha, linv[:, :n, :n], scal, xs, ils, src
 
 
 @pytest.mark.parametrize("name", ["tiny", "d8-ehvi2", "d10-ei", "d10-ehvi3"])
@@ -122,7 +125,10 @@ def test_gp_prepare_matches_oracle_factor(S, name):
     L = S.scoot_gp_layout_init(n, d, M)
     blob, cond = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
                                     inst.signal_var, inst.noise_var, L)
-    alpha, linv, scal, xs, ils = _unpack_gp(S, L, blob)
+    alpha, linv, scal, xs, ils, src = _unpack_gp(S, L, blob)
+    kinds = inst.space["kind"][src]
+    assert sorted(src.tolist()) == list(range(d))
+    assert np.all(np.diff((kinds == 2).astype(int)) >= 0)  # ordinal parameters come first
     for m in range(M):
         gp = O.GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m], inst.signal_var[m], inst.noise_var[m])
         assert np.allclose(alpha[m], gp.alpha, rtol=1e-6, atol=1e-6 * np.abs(gp.alpha).max())
