@@ -42,9 +42,16 @@ FLUSH_BYTES = 256 << 20   # > 129 MB of L2
 FP32_LANES_PER_SM = 128
 
 # DRAM bytes per launch from ncu (dram__bytes_read.sum + dram__bytes_write.sum),
-# keyed by (kernel, workload), valid only while the kernel's source file is
-# unchanged (sha256 prefix of the file when the counters were taken).
-TRAFFIC = {}
+# keyed by (stage, workload), valid only while the stage kernel's sources are
+# unchanged (sha256 prefix of their contents when the counters were taken);
+# the captures are summarised in profiles/kernels_full_<workload>.md.
+KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["score.cu", "device_common.cuh"],
+                "topq": ["topq.cu", "device_common.cuh"]}
+TRAFFIC = {
+    ("prune", "d8-ehvi2"): {"bytes": 3153152, "sha": "1eeab4bef935f295"},
+    ("rf", "d8-ehvi2"): {"bytes": 8805376, "sha": "1eeab4bef935f295"},
+    ("score", "d8-ehvi2"): {"bytes": 8834304, "sha": "a979d1e56ce96aee"},
+}
 
 
 def parse_args():
@@ -105,9 +112,12 @@ def work_model(inst, n_boxes):
     }
 
 
-def sha_of(relpath):
-    with open(os.path.join(ROOT, relpath), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+def sources_sha(stage):
+    h = hashlib.sha256()
+    for f in KERNEL_FILES[stage]:
+        with open(os.path.join(ROOT, "paper_2408_04323_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
 
 
 class ClockSampler:
@@ -323,11 +333,8 @@ def main():
     kind, per_cand = work[dom]
     units = n_feasible if dom == "score" else N
     launch_s = stage_ms[dom] / 1e3
-    kernel_file = {"prune": "prune_rf.cu", "rf": "prune_rf.cu", "score": "score.cu", "topq": "topq.cu"}[dom]
     tr = TRAFFIC.get((dom, w.name))
-    traffic = None
-    if tr and tr["sha"] == sha_of(os.path.join("paper_2408_04323_gb300", "csrc", kernel_file)):
-        traffic = tr["bytes"]
+    traffic = tr["bytes"] if tr and tr["sha"] == sources_sha(dom) else None
     if kind == "hbm":
         achieved = per_cand * units / launch_s / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
