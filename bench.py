@@ -256,7 +256,7 @@ def main():
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
     st = rnd.state
 
-    def step(evs=None):
+    def step(evs=None, stream=stream):
         sp = S.scoot_prune
         if evs:
             evs[0].record(stream)
@@ -303,10 +303,49 @@ def main():
     if dist:
         dist.barrier()
     torch.cuda.synchronize(device)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
-    for kk in range(args.steps):
+    # Per-stage times from eagerly launched steps (diagnostic; they feed the roofline).
+    n_diag = min(args.steps, 50)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n_diag)]
+    for kk in range(n_diag):
         flush.fill_(kk & 0xFF)
         step(evs[kk])
+    torch.cuda.synchronize(device)
+    stage_names = ["prune", "rf", "score", "topq"]
+    stage_ms = {s: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, s in enumerate(stage_names)}
+    eager_ms = statistics.mean(e[0].elapsed_time(e[4]) for e in evs)
+
+    # The step as one CUDA graph (its launches and memsets replayed without
+    # host gaps); the fantasy round synchronises with the host and stays eager.
+    graph = None
+    if not inp.fantasy:
+        try:
+            cap = torch.cuda.Stream(device)
+            cap.wait_stream(stream)
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=cap, capture_error_mode="thread_local"):
+                step(stream=cap)
+            torch.cuda.synchronize(device)
+            for _ in range(3):
+                graph.replay()
+            torch.cuda.synchronize(device)
+        except Exception as e:  # capture refused: time eager launches instead
+            graph = None
+            print(f"# CUDA graph capture unavailable ({e}); timing eager launches", file=sys.stderr)
+            torch.cuda.synchronize(device)
+
+    # The timed K steps.
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(device)
+    tev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    for kk in range(args.steps):
+        flush.fill_(kk & 0xFF)
+        tev[kk][0].record(stream)
+        if graph is not None:
+            graph.replay()
+        else:
+            step()
+        tev[kk][1].record(stream)
         if dist:
             gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
     torch.cuda.synchronize(device)
@@ -314,10 +353,7 @@ def main():
         dist.barrier()
     clocks = sampler.stop()
     ctx.check(stream)
-
-    stage_names = ["prune", "rf", "score", "topq"]
-    stage_ms = {s: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, s in enumerate(stage_names)}
-    step_ms = statistics.mean(e[0].elapsed_time(e[4]) for e in evs)
+    step_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in tev)
     if dist:
         t = torch.tensor([step_ms], device=device)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -415,7 +451,10 @@ def main():
                 "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic",
                 "config": workload_config(w, {"feasible": n_feasible, "boxes": st.n_boxes,
-                                              "front": st.front_size, "parallelism": f"pool shards x{world}"}),
+                                              "front": st.front_size, "parallelism": f"pool shards x{world}",
+                                              "launch": "CUDA graph of the step" if graph is not None
+                                              else "eager launches",
+                                              "eager_ms_per_step": round(eager_ms, 5)}),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps * rnd.kernels_per_round(),
                 "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},

@@ -153,7 +153,8 @@ typedef struct {
     int64_t bytes;            /* blob size */
     int64_t off_chunks;       /* int32[n_chunks][4]: first tree, tree count, first node, node count */
     int64_t off_roots;        /* int32[n_trees]: first node of each tree */
-    int64_t off_nodes;        /* scoot_node[n_nodes] */
+    int64_t off_nodes;        /* scoot_node[n_nodes], split nodes' left child counted from the
+                                 first node of their chunk */
 } scoot_forest_layout;
 
 /* Validate a forest given as nodes plus tree offsets (tree t owns nodes
@@ -190,19 +191,26 @@ typedef struct {
     int32_t n, d, n_obj, kernel;
     int32_t n_rb;             /* row blocks of 64 in the tiled L^{-1} */
     int32_t n_tiles;          /* 32 x 64 tiles of L^{-1} per objective */
+    int32_t n_ord;            /* ordinal (integer or continuous) parameters */
+    int32_t n_pat;            /* joint category patterns: product of the categoricals' n_choices (1 if none) */
     int64_t bytes;
     int64_t off_fmap;         /* float[d][4]: kind, a, b, source parameter of each feature, ordinal
-                                 parameters first, then categorical ones ("feature order") */
+                                 parameters first, then categorical ones ("feature order"); for a
+                                 categorical feature a = n_choices and b = its mixed-radix stride */
     int64_t off_xs;           /* float[M][n][d]: observed features in feature order, ordinal ones
                                  scaled by 1/lengthscale, categorical ones as the category index */
     int64_t off_ils;          /* float[M][d]: 1/l (ordinal) or 1/l^2 (categorical), feature order */
     int64_t off_alpha;        /* float[M][n] */
     int64_t off_linv;         /* float[M][n_tiles][32][64]: L^{-1} tiles, transposed, zero-filled */
     int64_t off_scal;         /* float[M][4]: signal variance, noise variance, best observed y, 0 */
+    int64_t off_cat;          /* float[M][n][n_pat]: for each category pattern p (mixed radix over the
+                                 categorical parameters in feature order), sum_c [p_c != X_jc] / l_c^2 */
 } scoot_gp_layout;
 
-/* Plan the blob for n observations, d parameters, M objectives and a kernel. */
-scoot_status scoot_gp_layout_init(int32_t n, int32_t d, int32_t n_obj, int32_t kernel,
+/* Plan the blob for n observations of the d-parameter space h_space, M
+ * objectives and a covariance kernel.  SCOOT_EUNSUPPORTED if the categorical
+ * parameters have more than 4096 joint patterns. */
+scoot_status scoot_gp_layout_init(const scoot_param* h_space, int32_t n, int32_t d, int32_t n_obj, int32_t kernel,
                                   scoot_gp_layout* out);
 /* Build the blob on the host.  h_x_obs: observed configurations, SoA words
  * [d][ld_obs]; h_y: standardised observed values [M][n]; h_lengthscale

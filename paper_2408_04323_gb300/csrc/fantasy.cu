@@ -353,8 +353,7 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
         !h_ref || !eps || !h_idx || !h_val || !h_count || !work)
         return scoot_fail(ctx, SCOOT_EINVAL, "a required pointer is NULL");
     *h_count = 0;
-    scoot_gp_layout chk;
-    if (scoot_gp_layout_init(L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK || std::memcmp(&chk, L, sizeof(chk)) != 0)
+    if (!scoot_gp_layout_valid(L))
         return scoot_fail(ctx, SCOOT_EINVAL, "GP layout is not one made by scoot_gp_layout_init");
     const int M = L->n_obj;
     if (M < 2 || M > 4) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "fantasy picks need 2 <= M <= 4, got %d", M);

@@ -18,6 +18,7 @@ constexpr int64_t kAlign = 256;
 constexpr int kRowBlock = 64;   // rows of L^{-1} per tile
 constexpr int kColChunk = 32;   // columns of L^{-1} per tile
 constexpr int kForestChunkNodes = 12288;  // 96 KiB of nodes staged at a time
+constexpr int kMaxPatterns = 4096;        // joint category patterns of the GP's categorical table
 
 int64_t align_up(int64_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
@@ -181,19 +182,25 @@ const char* scoot_status_string(scoot_status s) {
 
 // ---------------------------------------------------------------- GP state
 
-scoot_status scoot_gp_layout_init(int32_t n, int32_t d, int32_t n_obj, int32_t kernel,
-                                  scoot_gp_layout* out) {
-    if (!out) return SCOOT_EINVAL;
+}  // extern "C"
+
+namespace {
+
+scoot_status gp_layout_compute(int32_t n, int32_t d, int32_t n_obj, int32_t kernel, int32_t n_ord, int32_t n_pat,
+                               scoot_gp_layout* out) {
     std::memset(out, 0, sizeof(*out));
     if (n < 1 || d < 1 || n_obj < 1) return SCOOT_EINVAL;
     if (n > SCOOT_MAX_OBS || d > SCOOT_MAX_DIM || n_obj > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
     if (kernel != SCOOT_MATERN52 && kernel != SCOOT_MATERN32) return SCOOT_EINVAL;
+    if (n_ord < 0 || n_ord > d || n_pat < 1 || n_pat > kMaxPatterns) return SCOOT_EINVAL;
     out->n = n;
     out->d = d;
     out->n_obj = n_obj;
     out->kernel = kernel;
     out->n_rb = (n + kRowBlock - 1) / kRowBlock;
     out->n_tiles = out->n_rb * (out->n_rb + 1);  // row block b spans 2(b+1) column chunks
+    out->n_ord = n_ord;
+    out->n_pat = n_pat;
     int64_t off = 0;
     out->off_fmap = off;  off = align_up(off + (int64_t)d * 4 * 4);
     out->off_xs = off;    off = align_up(off + (int64_t)n_obj * n * d * 4);
@@ -201,8 +208,40 @@ scoot_status scoot_gp_layout_init(int32_t n, int32_t d, int32_t n_obj, int32_t k
     out->off_alpha = off; off = align_up(off + (int64_t)n_obj * n * 4);
     out->off_linv = off;  off = align_up(off + (int64_t)n_obj * out->n_tiles * kColChunk * kRowBlock * 4);
     out->off_scal = off;  off = align_up(off + (int64_t)n_obj * 4 * 4);
+    out->off_cat = off;   off = align_up(off + (int64_t)n_obj * n * n_pat * 4);
     out->bytes = off;
     return SCOOT_OK;
+}
+
+}  // namespace
+
+bool scoot_gp_layout_valid(const scoot_gp_layout* L) {
+    if (!L) return false;
+    scoot_gp_layout chk;
+    if (gp_layout_compute(L->n, L->d, L->n_obj, L->kernel, L->n_ord, L->n_pat, &chk) != SCOOT_OK) return false;
+    return std::memcmp(&chk, L, sizeof(chk)) == 0;
+}
+
+extern "C" {
+
+scoot_status scoot_gp_layout_init(const scoot_param* h_space, int32_t n, int32_t d, int32_t n_obj, int32_t kernel,
+                                  scoot_gp_layout* out) {
+    if (!out) return SCOOT_EINVAL;
+    std::memset(out, 0, sizeof(*out));
+    if (!h_space || d < 1) return SCOOT_EINVAL;
+    if (d > SCOOT_MAX_DIM) return SCOOT_EUNSUPPORTED;
+    if (!valid_space(h_space, d)) return SCOOT_EINVAL;
+    int32_t n_ord = 0;
+    int64_t n_pat = 1;
+    for (int c = 0; c < d; ++c) {
+        if (h_space[c].kind == SCOOT_CATEGORICAL) {
+            n_pat *= h_space[c].n_choices;
+            if (n_pat > kMaxPatterns) return SCOOT_EUNSUPPORTED;
+        } else {
+            ++n_ord;
+        }
+    }
+    return gp_layout_compute(n, d, n_obj, kernel, n_ord, (int32_t)n_pat, out);
 }
 
 scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
@@ -212,7 +251,7 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
     if (!h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var || !L || !h_blob)
         return SCOOT_EINVAL;
     scoot_gp_layout chk;
-    if (scoot_gp_layout_init(L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK ||
+    if (scoot_gp_layout_init(h_space, L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK ||
         std::memcmp(&chk, L, sizeof(chk)) != 0)
         return SCOOT_EINVAL;
     const int n = L->n, d = L->d, M = L->n_obj;
@@ -252,6 +291,17 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
         fmap[f * 4 + 2] = b;
         fmap[f * 4 + 3] = (float)c;
     }
+    // Categorical features: n_choices and the mixed-radix stride of the pattern id.
+    {
+        int stride = 1;
+        for (int f = L->n_ord; f < d; ++f) {
+            const scoot_param& p = h_space[order[f]];
+            fmap[f * 4 + 1] = (float)p.n_choices;
+            fmap[f * 4 + 2] = (float)stride;
+            stride *= p.n_choices;
+        }
+    }
+    float* cat = reinterpret_cast<float*>(blob + L->off_cat);
 
     float* xs = reinterpret_cast<float*>(blob + L->off_xs);
     float* ils = reinterpret_cast<float*>(blob + L->off_ils);
@@ -295,6 +345,19 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
                         if (row < n && c <= row) v = (float)Li[(size_t)row * n + c];
                         tiles[((size_t)t * kColChunk + jj) * kRowBlock + ii] = v;
                     }
+        // Categorical part of r^2 for every (observation, category pattern).
+        for (int j = 0; j < n; ++j)
+            for (int pat = 0; pat < L->n_pat; ++pat) {
+                double r2 = 0.0;
+                int rest = pat;
+                for (int f = L->n_ord; f < d; ++f) {
+                    const int c = order[f];
+                    const int v = rest % h_space[c].n_choices;
+                    rest /= h_space[c].n_choices;
+                    if ((double)v != g.u[(size_t)j * d + c]) r2 += 1.0 / (g.ell[c] * g.ell[c]);
+                }
+                cat[((size_t)m * n + j) * L->n_pat + pat] = (float)r2;
+            }
         float ybest = -std::numeric_limits<float>::infinity();
         for (int j = 0; j < n; ++j) ybest = std::max(ybest, h_y[(size_t)m * n + j]);
         scal[m * 4 + 0] = h_signal_var[m];
@@ -495,7 +558,18 @@ scoot_status scoot_forest_pack(const scoot_forest_layout* L, const scoot_node* h
     ch[c * 4 + 0] = first; ch[c * 4 + 1] = L->n_trees - first;
     ch[c * 4 + 2] = h_tree_offset[first]; ch[c * 4 + 3] = nodes;
     std::memcpy(blob + L->off_roots, h_tree_offset, (size_t)L->n_trees * 4);
-    std::memcpy(blob + L->off_nodes, h_nodes, (size_t)L->n_nodes * 8);
+    // Nodes with the left child counted from the first node of the node's
+    // chunk, so a walk in shared memory needs no per-tree offset.
+    scoot_node* out = reinterpret_cast<scoot_node*>(blob + L->off_nodes);
+    for (int k = 0; k < L->n_chunks; ++k) {
+        const int first = ch[k * 4 + 0], count = ch[k * 4 + 1], node0 = ch[k * 4 + 2];
+        for (int t = first; t < first + count; ++t)
+            for (int i = h_tree_offset[t]; i < h_tree_offset[t + 1]; ++i) {
+                out[i] = h_nodes[i];
+                if (!(h_nodes[i].flags & 1))
+                    out[i].left = (uint16_t)(h_tree_offset[t] - node0 + h_nodes[i].left);
+            }
+    }
     return SCOOT_OK;
 }
 

@@ -57,6 +57,9 @@ scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, 
                            const float* y, const float* lengthscale, float signal_var, float noise_var,
                            int kernel, HostGP* out, double* cond);
 
+// Consistency of a GP layout's offsets with its own sizes.
+bool scoot_gp_layout_valid(const scoot_gp_layout* L);
+
 // Checks shared by the device entry points.
 scoot_status scoot_check_pool(scoot_ctx* ctx, const uint32_t* cand, int64_t n, int64_t ld, int32_t d);
 

@@ -8,8 +8,8 @@ namespace {
 
 constexpr int kPruneThreads = 256;
 constexpr int kRfThreads = 256;
-constexpr int kRfGroups = 4;                     // threads (tree groups) per candidate
-constexpr int kRfCand = kRfThreads / kRfGroups;  // candidates per tile
+constexpr int kRfCand = 32;                      // candidates per tile (one per lane)
+constexpr int kRfGroups = kRfThreads / kRfCand;  // warps = tree groups
 
 struct PruneArgs {
     int32_t n_clauses;
@@ -75,40 +75,47 @@ struct RfArgs {
     int32_t single_chunk;
     const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
     const unsigned int* n_list;
+    int32_t max_chunk_nodes;
 };
 
-// Persistent blocks of 256 threads score tiles of 64 candidates; thread t
-// serves candidate slot t / 4 and walks the trees of group t % 4 (trees
-// g, g + 4, ...), so a block has four independent walks per candidate and a
-// pool of ~10^5 live candidates still fills every SM.  The forest (or one
-// chunk of whole trees at a time) sits in shared memory; each tile's feature
-// values sit in shared memory as feat[slot][f] with an odd row stride.  The
-// four partial vote counts of a candidate are added with warp shuffles.
+// Persistent blocks of 256 threads score tiles of 32 candidates: lane l of
+// warp g serves candidate slot l and walks trees g, g + 8, g + 16, ... of the
+// forest, so the 32 lanes of a warp walk the same tree for 32 candidates
+// (the upper levels are broadcast loads) and each candidate has eight
+// independent walks in flight.  The forest (or one chunk of whole trees at a
+// time) sits in shared memory with chunk-relative child indices; the tile's
+// feature values sit in shared memory as feat[slot][f] with an odd row
+// stride (conflict-free when a warp reads one feature).  The eight partial
+// vote counts of a candidate are added through shared memory.
 __global__ void __launch_bounds__(kRfThreads)
 rf_kernel(const __grid_constant__ RfArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    const int fs = a.d | 1;                                                   // odd row stride
-    float* sfeat = reinterpret_cast<float*>(smem_raw);                        // [kRfCand][fs]
-    uint2* snodes = reinterpret_cast<uint2*>(sfeat + ((kRfCand * fs + 1) & ~1));  // chunk nodes
+    const int fs = a.d | 1;                                                       // odd row stride
+    uint2* snodes = reinterpret_cast<uint2*>(smem_raw);                           // chunk nodes
+    float* sfeat = reinterpret_cast<float*>(snodes + a.max_chunk_nodes);          // [kRfCand][fs]
+    uint32_t* svote = reinterpret_cast<uint32_t*>(sfeat + kRfCand * fs);          // [kRfGroups][kRfCand]
+    int32_t* sroot = reinterpret_cast<int32_t*>(svote + kRfGroups * kRfCand);      // [n_trees]
 
     const int32_t* chunks = reinterpret_cast<const int32_t*>(a.forest + a.off_chunks);
     const int32_t* roots = reinterpret_cast<const int32_t*>(a.forest + a.off_roots);
     const uint2* gnodes = reinterpret_cast<const uint2*>(a.forest + a.off_nodes);
     const int tid = threadIdx.x;
-    const int slot = tid / kRfGroups, grp = tid % kRfGroups;
+    const int slot = tid & (kRfCand - 1), grp = tid / kRfCand;
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
     const int64_t n_tiles = (n_work + kRfCand - 1) / kRfCand;
     uint32_t feasible = 0;
 
     auto stage_chunk = [&](int ch) {
+        const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
         const int first_node = chunks[ch * 4 + 2], count = chunks[ch * 4 + 3];
         for (int k = tid; k < count; k += kRfThreads) snodes[k] = __ldg(gnodes + first_node + k);
+        for (int k = tid; k < nt; k += kRfThreads) sroot[t0 + k] = roots[t0 + k] - first_node;
     };
     if (a.single_chunk) stage_chunk(0);  // visible after the first barrier below
 
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
         const int64_t base = tile * kRfCand;
-        __syncthreads();  // the previous tile's features are no longer read
+        __syncthreads();  // the previous tile's features and votes are no longer read
         for (int k = tid; k < kRfCand * a.d; k += kRfThreads) {
             const int f = k / kRfCand, c = k - f * kRfCand;
             const int64_t pos = base + c;
@@ -130,11 +137,10 @@ rf_kernel(const __grid_constant__ RfArgs a) {
                 stage_chunk(ch);
             }
             __syncthreads();
-            const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1], node0 = chunks[ch * 4 + 2];
+            const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
             if (!live) continue;
             for (int t = t0 + grp; t < t0 + nt; t += kRfGroups) {
-                const int root = roots[t] - node0;
-                int node = root;
+                int node = sroot[t];
                 bool done = false;
                 for (int step = 0; step <= a.max_depth; ++step) {
                     const uint2 nd = snodes[node];
@@ -144,19 +150,21 @@ rf_kernel(const __grid_constant__ RfArgs a) {
                         break;
                     }
                     const float x = my[(nd.y >> 16) & 0xff];
-                    node = root + (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
+                    node = (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
                 }
                 if (!done) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
             }
         }
-        // add the group partials (the four threads of a slot are adjacent lanes)
-        vote += __shfl_xor_sync(0xffffffffu, vote, 1);
-        vote += __shfl_xor_sync(0xffffffffu, vote, 2);
-        if (live && grp == 0) {
+        svote[grp * kRfCand + slot] = vote;
+        __syncthreads();
+        if (grp == 0 && live) {
+            uint32_t v = 0;
+#pragma unroll
+            for (int g = 0; g < kRfGroups; ++g) v += svote[g * kRfCand + slot];
             const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
             const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
-            a.votes[i] = vote;
-            const bool ok = (unsigned __int128)a.delta_den * vote >= need;
+            a.votes[i] = v;
+            const bool ok = (unsigned __int128)a.delta_den * v >= need;
             if (a.mask) a.mask[i] = ok;
             feasible += ok;
         }
@@ -267,7 +275,9 @@ scoot_status scoot_rf_predict(scoot_ctx* ctx, const scoot_forest_layout* L, cons
         a.list = lst.list;
         a.n_list = lst.count;
     }
-    const size_t smem = (size_t)((kRfCand * (L->d | 1) + 1) & ~1) * 4 + (size_t)max_chunk_nodes * 8;
+    a.max_chunk_nodes = max_chunk_nodes;
+    const size_t smem = (size_t)max_chunk_nodes * 8 + (size_t)kRfCand * (L->d | 1) * 4 +
+                        (size_t)kRfGroups * kRfCand * 4 + (size_t)L->n_trees * 4;
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(rf_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;
     SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rf_kernel, kRfThreads, smem));

@@ -31,8 +31,8 @@ enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3 };
 
 struct ScoreArgs {
     const char* state;
-    int64_t off_fmap, off_xs, off_ils, off_alpha, off_linv, off_scal;
-    int32_t n_obs, d, dp, n_obj, kernel, n_rb, n_tiles;
+    int64_t off_fmap, off_xs, off_ils, off_alpha, off_linv, off_scal, off_cat;
+    int32_t n_obs, d, dp, n_obj, kernel, n_rb, n_tiles, n_ord, n_pat;
     const uint32_t* cand;
     int64_t n, ld;
     const uint8_t* mask;
@@ -50,11 +50,14 @@ struct ScoreArgs {
     const unsigned int* n_list;
     float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad][ldv] by list position
     int64_t ldv;
+    uint32_t* err;                // device error word
 };
 
 // Partial EHVI sum of one candidate over the sample chunks first, first +
-// stride, ... (chunks of eight samples, padding samples at -inf).
-template <int M>
+// stride, ... (chunks of eight samples, padding samples at -inf).  FAST: the
+// boxes are open (+inf) on the last objective, as scoot_boxes_build emits
+// them; then the last factor needs no min and the product folds into an FMA.
+template <int M, bool FAST>
 __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, const float4* blo, const float4* bhi,
                                              int n_boxes, const float4* eps, int n_mc, int first, int stride) {
     constexpr int kCh = 8;
@@ -76,16 +79,33 @@ __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, 
             const float hi[4] = {hi4.x, hi4.y, hi4.z, hi4.w};
 #pragma unroll
             for (int k = 0; k < kCh; ++k) {
-                float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+                if (FAST) {
+                    float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
 #pragma unroll
-                for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
-                acc[k] += p;
+                    for (int j = 1; j < M - 1; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
+                    acc[k] = fmaf(p, fmaxf(y[k][M - 1] - lo[M - 1], 0.0f), acc[k]);
+                } else {
+                    float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+#pragma unroll
+                    for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
+                    acc[k] += p;
+                }
             }
         }
 #pragma unroll
         for (int k = 0; k < kCh; ++k) total += acc[k];
     }
     return total;
+}
+
+// True (in every thread) when every staged box is open on the last objective.
+__device__ __forceinline__ bool boxes_fast(const float4* bhi, int n_boxes, int M) {
+    int ok = 1;
+    for (int b = threadIdx.x; b < n_boxes; b += blockDim.x) {
+        const float4 h = bhi[b];
+        ok &= (M == 2 ? h.y : (M == 3 ? h.z : h.w)) == INFINITY;
+    }
+    return __syncthreads_and(ok) != 0;
 }
 
 // One block of 128 threads scores a tile of 64 candidates; thread t works on
@@ -99,20 +119,23 @@ __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, 
 //     sigma^2 = s_f^2 - sum_i V_i^2;
 //  3. the epilogue (EI on one half, EHVI with the halves splitting the
 //     sample chunks, or the moments / whitened rows) writes the tile.
-// DM >= d bounds the per-dimension register arrays; features come in feature
-// order (ordinal parameters first), so the distance loop has no kind branch.
-template <int EPI, int M, int DM>
-__global__ void __launch_bounds__(kThreads)
+// Features come in feature order (ordinal parameters first).  DO >= n_ord
+// bounds the ordinal register arrays; padded ordinal dimensions are zero on
+// both sides and add nothing, so the distance loop has no per-dimension
+// branch.  The categorical part of r^2 depends only on the candidate's joint
+// category pattern and is read from the host-built table (one load).
+template <int EPI, int M, int DO>
+__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO <= 8) ? 6 : 1)
 score_kernel(const __grid_constant__ ScoreArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
     float* Ks = sm;                                                   // [n_pad][kTC]
-    float* xs = Ks + (size_t)n_pad * kTC;                             // [n_obs][dp]
-    float* al = xs + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3));     // [n_pad]
+    float* xs = Ks + (size_t)n_pad * kTC;                             // [n_obs][DO] ordinal features
+    float* al = xs + (size_t)a.n_obs * DO;                            // [n_pad]
     float* Lt = al + n_pad;                                           // [kCJ][kRB]
     float* part = Lt + kCJ * kRB;                                     // [8][kTC]
-    float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [DM] feature map
-    float4* blo = fm + DM;
+    float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [kMaxD] feature map
+    float4* blo = fm + kMaxD;
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
     float4* epsv = bhi + (EPI == kEHVI ? a.n_boxes : 0);
 
@@ -127,13 +150,13 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     const float* galpha = reinterpret_cast<const float*>(a.state + a.off_alpha);
     const float4* glinv = reinterpret_cast<const float4*>(a.state + a.off_linv);
     const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
+    const float* gcat = reinterpret_cast<const float*>(a.state + a.off_cat);
 
     if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
-    if (tid < DM) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
+    if (tid < kMaxD) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
     __syncthreads();
-    int n_ord = 0;
-#pragma unroll
-    for (int q = 0; q < DM; ++q) n_ord += (q < a.d && (int)fm[q].x != SCOOT_CATEGORICAL) ? 1 : 0;
+    const bool fast = EPI == kEHVI ? boxes_fast(bhi, a.n_boxes, M) : false;
+    const int n_ord = a.n_ord;
 
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
     const int64_t n_tiles = (n_work + kTC - 1) / kTC;
@@ -141,48 +164,59 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
         const int64_t pos = tile * kTC + slot;
         const bool live = pos < n_work;
         const int64_t i = live ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
-        float u[DM];
+        float u[DO];
 #pragma unroll
-        for (int q = 0; q < DM; ++q) {
+        for (int q = 0; q < DO; ++q) {
             u[q] = 0.0f;
-            if (q < a.d && live) {
+            if (q < n_ord && live) {
                 const float4 f = fm[q];
                 u[q] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + i), (int)f.x, f.y, f.z);
             }
+        }
+        // Joint category pattern (mixed radix); out-of-range categories are
+        // clamped and flagged.
+        int pid = 0;
+        for (int q = n_ord; q < a.d && live; ++q) {
+            const float4 f = fm[q];
+            const int nc = (int)f.y;
+            int v = (int)__ldg(a.cand + (int64_t)f.w * a.ld + i);
+            if (v < 0 || v >= nc) {
+                atomicOr(a.err, SCOOT_DEVERR_INDEX);
+                v = v < 0 ? 0 : nc - 1;
+            }
+            pid += v * (int)f.z;
         }
         float mu[kMaxM], vr[kMaxM];
         for (int m = 0; m < nobj; ++m) {
             __syncthreads();  // previous users of xs / al / part are done
             const float* sx = gxs + (size_t)m * a.n_obs * a.d;
-            for (int k = tid; k < a.n_obs * a.d; k += kThreads) {
-                const int j = k / a.d, q = k - j * a.d;
-                xs[j * a.dp + q] = sx[k];
+            for (int e = tid; e < a.n_obs * DO; e += kThreads) {
+                const int j = e / DO, q = e - j * DO;
+                xs[e] = q < n_ord ? sx[j * a.d + q] : 0.0f;
             }
             for (int j = tid; j < n_pad; j += kThreads) al[j] = j < a.n_obs ? galpha[(size_t)m * a.n_obs + j] : 0.0f;
             const float sf2 = gscal[m * 4 + 0];
-            float ut[DM], w2[DM];
+            const float* catrow = gcat + (size_t)m * a.n_obs * a.n_pat + pid;
+            float ut[DO];
 #pragma unroll
-            for (int q = 0; q < DM; ++q) {
-                const float sc = q < a.d ? gils[m * a.d + q] : 0.0f;
-                ut[q] = q < n_ord ? u[q] * sc : u[q];
-                w2[q] = q < n_ord ? 0.0f : sc;
-            }
+            for (int q = 0; q < DO; ++q) ut[q] = q < n_ord ? u[q] * gils[m * a.d + q] : 0.0f;
             __syncthreads();
             // 1. covariance row (this half's j) and the partial mean.
             float acc = 0.0f;
 #pragma unroll 2
             for (int j = half; j < a.n_obs; j += 2) {
-                const float* xj = xs + j * a.dp;
-                float r2 = 0.0f;
+                const float4* xj4 = reinterpret_cast<const float4*>(xs + j * DO);
+                float r2 = __ldg(catrow + (size_t)j * a.n_pat);  // categorical part
 #pragma unroll
-                for (int q = 0; q < DM; ++q)
-                    if (q < n_ord) {
-                        const float t = ut[q] - xj[q];
-                        r2 = fmaf(t, t, r2);
-                    }
-#pragma unroll
-                for (int q = 0; q < DM; ++q)
-                    if (q >= n_ord && q < a.d) r2 += ut[q] != xj[q] ? w2[q] : 0.0f;
+                for (int q4 = 0; q4 < DO / 4; ++q4) {
+                    const float4 v = xj4[q4];
+                    const float t0 = ut[q4 * 4] - v.x, t1 = ut[q4 * 4 + 1] - v.y;
+                    const float t2 = ut[q4 * 4 + 2] - v.z, t3 = ut[q4 * 4 + 3] - v.w;
+                    r2 = fmaf(t0, t0, r2);
+                    r2 = fmaf(t1, t1, r2);
+                    r2 = fmaf(t2, t2, r2);
+                    r2 = fmaf(t3, t3, r2);
+                }
                 const float k = sf2 * matern(sqrtf(r2), a.kernel);
                 Ks[j * kTC + slot] = k;
                 acc = fmaf(k, al[j], acc);
@@ -274,7 +308,8 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             float sd[kMaxM];
 #pragma unroll
             for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
-            const float v = ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2);
+            const float v = fast ? ehvi_partial<M, true>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2)
+                                 : ehvi_partial<M, false>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2);
             __syncthreads();  // part is free again
             part[half * kTC + slot] = v;
             __syncthreads();
@@ -323,8 +358,7 @@ int sm_count(int device) {
 
 scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state, ScoreArgs& a) {
     if (!L || !state) return scoot_fail(ctx, SCOOT_EINVAL, "layout or state is NULL");
-    scoot_gp_layout chk;
-    if (scoot_gp_layout_init(L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK || std::memcmp(&chk, L, sizeof(chk)) != 0)
+    if (!scoot_gp_layout_valid(L))
         return scoot_fail(ctx, SCOOT_EINVAL, "GP layout is not one made by scoot_gp_layout_init");
     if (!scoot_aligned16(state)) return scoot_fail(ctx, SCOOT_EINVAL, "state blob is not 16-byte aligned");
     std::memset(&a, 0, sizeof(a));
@@ -335,6 +369,9 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
     a.off_alpha = L->off_alpha;
     a.off_linv = L->off_linv;
     a.off_scal = L->off_scal;
+    a.off_cat = L->off_cat;
+    a.n_ord = L->n_ord;
+    a.n_pat = L->n_pat;
     a.n_obs = L->n;
     a.d = L->d;
     a.dp = (L->d + 3) & ~3;
@@ -345,17 +382,17 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
     return SCOOT_OK;
 }
 
-size_t score_smem(const ScoreArgs& a, int epi) {
+size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
-    size_t f = n_pad * kTC + (((size_t)a.n_obs * a.dp + 3) & ~size_t(3)) + n_pad + kCJ * kRB + 8 * kTC + 4 * kMaxD;
+    size_t f = n_pad * kTC + (size_t)a.n_obs * DO + n_pad + kCJ * kRB + 8 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
     return f * 4;
 }
 
-template <int EPI, int M, int DM>
+template <int EPI, int M, int DO>
 scoot_status launch_score_dm(scoot_ctx* ctx, const ScoreArgs& a, cudaStream_t st) {
-    const size_t smem = score_smem(a, EPI);
-    auto kern = score_kernel<EPI, M, DM>;
+    const size_t smem = score_smem(a, EPI, DO);
+    auto kern = score_kernel<EPI, M, DO>;
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;
     SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));
@@ -380,9 +417,10 @@ scoot_status launch_score(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
         a.list = lst.list;
         a.n_list = lst.count;
     }
-    if (a.d <= 4) return launch_score_dm<EPI, M, 4>(ctx, a, st);
-    if (a.d <= 8) return launch_score_dm<EPI, M, 8>(ctx, a, st);
-    if (a.d <= 12) return launch_score_dm<EPI, M, 12>(ctx, a, st);
+    a.err = ctx->d_err;
+    if (a.n_ord <= 4) return launch_score_dm<EPI, M, 4>(ctx, a, st);
+    if (a.n_ord <= 8) return launch_score_dm<EPI, M, 8>(ctx, a, st);
+    if (a.n_ord <= 12) return launch_score_dm<EPI, M, 12>(ctx, a, st);
     return launch_score_dm<EPI, M, 16>(ctx, a, st);
 }
 

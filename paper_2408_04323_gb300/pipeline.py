@@ -45,7 +45,7 @@ class State:
     def __init__(self, inp: RoundInputs, device: torch.device):
         d = len(inp.space)
         M = inp.y_obs.shape[0]
-        self.gp_layout = S.scoot_gp_layout_init(inp.y_obs.shape[1], d, M, inp.kernel)
+        self.gp_layout = S.scoot_gp_layout_init(inp.space, inp.y_obs.shape[1], M, inp.kernel)
         blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
                                              inp.signal_var, inp.noise_var, self.gp_layout)
         self.forest_layout = S.scoot_forest_layout_init(inp.nodes, inp.tree_offset, d, inp.leaf_scale)

@@ -54,9 +54,10 @@ class scoot_forest_layout(C.Structure):
 
 class scoot_gp_layout(C.Structure):
     _fields_ = [("n", C.c_int32), ("d", C.c_int32), ("n_obj", C.c_int32), ("kernel", C.c_int32),
-                ("n_rb", C.c_int32), ("n_tiles", C.c_int32), ("bytes", C.c_int64),
-                ("off_fmap", C.c_int64), ("off_xs", C.c_int64), ("off_ils", C.c_int64),
-                ("off_alpha", C.c_int64), ("off_linv", C.c_int64), ("off_scal", C.c_int64)]
+                ("n_rb", C.c_int32), ("n_tiles", C.c_int32), ("n_ord", C.c_int32), ("n_pat", C.c_int32),
+                ("bytes", C.c_int64), ("off_fmap", C.c_int64), ("off_xs", C.c_int64), ("off_ils", C.c_int64),
+                ("off_alpha", C.c_int64), ("off_linv", C.c_int64), ("off_scal", C.c_int64),
+                ("off_cat", C.c_int64)]
 
 
 assert C.sizeof(scoot_param) == 16 and C.sizeof(scoot_clause) == 80 and C.sizeof(scoot_node) == 8
@@ -74,7 +75,7 @@ _PROTOS = {
     "scoot_forest_pack": [C.POINTER(scoot_forest_layout), _vp, _vp, _vp],
     "scoot_rf_predict": [_vp, C.POINTER(scoot_forest_layout), _vp, _vp, _vp, _i64, _i64, _u32, _u32,
                          _vp, _vp, _vp, _vp],
-    "scoot_gp_layout_init": [_i32, _i32, _i32, _i32, C.POINTER(scoot_gp_layout)],
+    "scoot_gp_layout_init": [_vp, _i32, _i32, _i32, _i32, C.POINTER(scoot_gp_layout)],
     "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_posterior": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i64, _vp],
     "scoot_acq_ei": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp],
@@ -215,9 +216,10 @@ def _h(ctx):
 
 # ------------------------------------------------------------------ host-side preparation
 
-def scoot_gp_layout_init(n: int, d: int, n_obj: int, kernel: int = MATERN52) -> scoot_gp_layout:
+def scoot_gp_layout_init(h_space, n: int, n_obj: int, kernel: int = MATERN52) -> scoot_gp_layout:
     L = scoot_gp_layout()
-    _check(lib().scoot_gp_layout_init(int(n), int(d), int(n_obj), int(kernel), C.byref(L)), "scoot_gp_layout_init")
+    _check(lib().scoot_gp_layout_init(_host(h_space, 16, name="h_space"), int(n), int(len(h_space)), int(n_obj),
+                                      int(kernel), C.byref(L)), "scoot_gp_layout_init")
     return L
 
 

@@ -37,7 +37,7 @@ def test_fantasy_picks_follow_the_refit_oracle(S, seed_i, n, q):
         forest = torch.from_numpy(S.scoot_forest_pack(L, inst.nodes, inst.tree_offset)).cuda()
         votes = torch.empty(n, dtype=torch.int32, device="cuda")
         S.scoot_rf_predict(ctx, L, forest, inst.space, cand, n, w.delta_num, w.delta_den, votes, mask)
-        G = S.scoot_gp_layout_init(inst.n_obs, inst.d, inst.n_obj)
+        G = S.scoot_gp_layout_init(inst.space, inst.n_obs, inst.n_obj)
         blob, _ = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
                                      inst.noise_var, G)
         state = torch.from_numpy(blob).cuda()

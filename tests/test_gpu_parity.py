@@ -187,7 +187,7 @@ def test_rf_multi_chunk_forest(S, ctx):
 # ------------------------------------------------------------------ GP posterior (Section 4.3)
 
 def gp_state(S, inst, kernel=0):
-    L = S.scoot_gp_layout_init(inst.n_obs, inst.d, inst.n_obj, kernel)
+    L = S.scoot_gp_layout_init(inst.space, inst.n_obs, inst.n_obj, kernel)
     blob, _ = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
                                  inst.signal_var, inst.noise_var, L)
     return L, dev(blob)

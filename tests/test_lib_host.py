@@ -122,7 +122,7 @@ def _unpack_gp(S, L, blob):
 def test_gp_prepare_matches_oracle_factor(S, name):
     inst = make_instance(name, seeds(name)[0], n_cand=64)
     M, n, d = inst.n_obj, inst.n_obs, inst.d
-    L = S.scoot_gp_layout_init(n, d, M)
+    L = S.scoot_gp_layout_init(inst.space, n, M)
     blob, cond = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
                                     inst.signal_var, inst.noise_var, L)
     alpha, linv, scal, xs, ils, src = _unpack_gp(S, L, blob)
@@ -147,7 +147,7 @@ def test_gp_prepare_matches_oracle_factor(S, name):
 def test_gp_prepare_rejects_bad_inputs(S):
     inst = make_instance("tiny", 1001, n_cand=8)
     M, n, d = inst.n_obj, inst.n_obs, inst.d
-    L = S.scoot_gp_layout_init(n, d, M)
+    L = S.scoot_gp_layout_init(inst.space, n, M)
     args = [inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var, inst.noise_var]
     bad_y = inst.y_obs.copy(); bad_y[0, 3] = np.nan
     bad_l = inst.lengthscale.copy(); bad_l[1, 2] = 0.0
@@ -162,7 +162,7 @@ def test_gp_prepare_rejects_bad_inputs(S):
         S.scoot_gp_prepare(inst.space, x, inst.y_obs, inst.lengthscale, inst.signal_var,
                            np.zeros(M, np.float32), L)
     with pytest.raises(S.ScootError):
-        S.scoot_gp_layout_init(2000, d, M)
+        S.scoot_gp_layout_init(inst.space, 2000, M)
 
 
 # ------------------------------------------------------------------ forest
@@ -173,7 +173,12 @@ def test_forest_pack_roundtrip_and_validation(S):
     assert L.n_trees == inst.n_trees and L.n_nodes == len(inst.nodes) and L.n_chunks == 1
     blob = S.scoot_forest_pack(L, inst.nodes, inst.tree_offset)
     got = blob[L.off_nodes:L.off_nodes + 8 * L.n_nodes].view(NODE_DTYPE)
-    assert np.array_equal(got, inst.nodes)
+    for f in ("val", "feat", "flags"):
+        assert np.array_equal(got[f], inst.nodes[f])
+    # split nodes point at their left child counted from the chunk's first node (one chunk here)
+    base = np.repeat(inst.tree_offset[:-1], np.diff(inst.tree_offset))
+    split = (inst.nodes["flags"] & 1) == 0
+    assert np.array_equal(got["left"][split].astype(int), (base + inst.nodes["left"].astype(int))[split])
 
     def bad(mutate, d=inst.d, scale=255):
         nodes = inst.nodes.copy()
