@@ -105,10 +105,17 @@ rf_kernel(const __grid_constant__ RfArgs a) {
     const int64_t n_tiles = (n_work + kRfCand - 1) / kRfCand;
     uint32_t feasible = 0;
 
+    // Staged node word: x = threshold bits (split) or vote count as a float
+    // (leaf); y = chunk-relative left child in bits 0..15, the feature's byte
+    // offset in a feature row in bits 16..30, bit 31 set for a leaf.
     auto stage_chunk = [&](int ch) {
         const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
         const int first_node = chunks[ch * 4 + 2], count = chunks[ch * 4 + 3];
-        for (int k = tid; k < count; k += kRfThreads) snodes[k] = __ldg(gnodes + first_node + k);
+        for (int k = tid; k < count; k += kRfThreads) {
+            const uint2 g = __ldg(gnodes + first_node + k);
+            const uint32_t leaf = (g.y >> 24) & 1u, feat = (g.y >> 16) & 0xffu;
+            snodes[k] = make_uint2(g.x, leaf ? 0x80000000u : ((feat * 4u) << 16) | (g.y & 0xffffu));
+        }
         for (int k = tid; k < nt; k += kRfThreads) sroot[t0 + k] = roots[t0 + k] - first_node;
     };
     if (a.single_chunk) stage_chunk(0);  // visible after the first barrier below
@@ -129,7 +136,7 @@ rf_kernel(const __grid_constant__ RfArgs a) {
         }
         const int64_t pos = base + slot;
         const bool live = pos < n_work;
-        const float* my = sfeat + slot * fs;
+        const char* my = reinterpret_cast<const char*>(sfeat + slot * fs);
         uint32_t vote = 0;
         for (int ch = 0; ch < a.n_chunks; ++ch) {
             if (!a.single_chunk) {
@@ -142,14 +149,15 @@ rf_kernel(const __grid_constant__ RfArgs a) {
             for (int t = t0 + grp; t < t0 + nt; t += kRfGroups) {
                 int node = sroot[t];
                 bool done = false;
+#pragma unroll 2
                 for (int step = 0; step <= a.max_depth; ++step) {
                     const uint2 nd = snodes[node];
-                    if ((nd.y >> 24) & 1u) {
+                    if ((int)nd.y < 0) {
                         vote += (uint32_t)__uint_as_float(nd.x);
                         done = true;
                         break;
                     }
-                    const float x = my[(nd.y >> 16) & 0xff];
+                    const float x = *reinterpret_cast<const float*>(my + (nd.y >> 16));
                     node = (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
                 }
                 if (!done) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth

@@ -245,11 +245,15 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                     for (int k = 0; k < kCJ * kRB / 4 / kThreads; ++k)
                         reinterpret_cast<float4*>(Lt)[tid + k * kThreads] = __ldg(src + tid + k * kThreads);
                     __syncthreads();
-                    // rows of this warp: rb*64 + 16*warp .. +15; columns cj*32 .. +31
-                    if (cj * kCJ > rb * kRB + 16 * warp + 15) continue;
+                    // rows of this warp: rb*64 + 16*warp .. +15; columns cj*32 .. +31;
+                    // L^{-1} is zero right of the diagonal, so a warp stops at its
+                    // last row (in steps of 16 columns).
                     const int j0 = cj * kCJ;
+                    const int last_row = rb * kRB + 16 * warp + 15;
+                    if (j0 > last_row) continue;
+                    const int jj_end = last_row - j0 + 1 >= kCJ ? kCJ : 16;
 #pragma unroll 4
-                    for (int jj = 0; jj < kCJ; ++jj) {
+                    for (int jj = 0; jj < jj_end; ++jj) {
                         const float4 k4 = Ks4[(j0 + jj) * (kTC / 4) + cg];
                         const float4 l0 = Lt4[jj * (kRB / 4) + rg * 2];
                         const float4 l1 = Lt4[jj * (kRB / 4) + rg * 2 + 1];
