@@ -54,10 +54,9 @@ struct ScoreArgs {
 };
 
 // Partial EHVI sum of one candidate over the sample chunks first, first +
-// stride, ... (chunks of eight samples, padding samples at -inf).  FAST: the
-// boxes are open (+inf) on the last objective, as scoot_boxes_build emits
-// them; then the last factor needs no min and the product folds into an FMA.
-template <int M, bool FAST>
+// stride, ... (chunks of eight samples, padding samples at -inf); boxes as
+// staged by stage_boxes.
+template <int M>
 __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, const float4* blo, const float4* bhi,
                                              int n_boxes, const float4* eps, int n_mc, int first, int stride) {
     constexpr int kCh = 8;
@@ -79,17 +78,75 @@ __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, 
             const float hi[4] = {hi4.x, hi4.y, hi4.z, hi4.w};
 #pragma unroll
             for (int k = 0; k < kCh; ++k) {
-                if (FAST) {
-                    float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+                float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
 #pragma unroll
-                    for (int j = 1; j < M - 1; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
-                    acc[k] = fmaf(p, fmaxf(y[k][M - 1] - lo[M - 1], 0.0f), acc[k]);
-                } else {
-                    float p = fmaxf(fminf(y[k][0], hi[0]) - lo[0], 0.0f);
+                for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
+                acc[k] += p;
+            }
+        }
 #pragma unroll
-                    for (int j = 1; j < M; ++j) p *= fmaxf(fminf(y[k][j], hi[j]) - lo[j], 0.0f);
-                    acc[k] += p;
-                }
+        for (int k = 0; k < kCh; ++k) total += acc[k];
+    }
+    return total;
+}
+
+// Width that stands in for an unbounded side of a box on the first M-1
+// objectives: a power of two, so scaling by it and by its inverse is exact;
+// valid while every sample lies within 2^40 of the box's lower corner.
+constexpr float kOpenWidth = 1099511627776.0f;  // 2^40
+
+// Boxes open on the last objective in "saturated" form: for the first M-1
+// objectives a_j = 1/w_j and b_j = -l_j/w_j (w_j the box width), and for the
+// last one W = prod_j w_j and C = -l_last * W, so that a box's HVI term is
+//   prod_{j<M-1} sat(y_j a_j + b_j) * max(y_last W + C, 0)
+// (sat clamps to [0, 1]): one saturated FMA per bounded objective.
+// Row b holds (a_0, b_0, a_1, b_1) and (a_2, b_2, W, C) as two float4.
+__device__ __forceinline__ void stage_boxes_sat(const float* box_lo, const float* box_hi, int n_boxes, int M,
+                                                float4* bs) {
+    for (int b = threadIdx.x; b < n_boxes; b += blockDim.x) {
+        float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        float W = 1.0f;
+        for (int j = 0; j < M - 1; ++j) {
+            const float l = box_lo[b * M + j], h = box_hi[b * M + j];
+            const float w = h == INFINITY ? kOpenWidth : h - l;
+            v[2 * j] = 1.0f / w;
+            v[2 * j + 1] = -l / w;
+            W *= w;
+        }
+        v[6] = W;
+        v[7] = -box_lo[b * M + M - 1] * W;
+        bs[2 * b] = make_float4(v[0], v[1], v[2], v[3]);
+        bs[2 * b + 1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+
+template <int M>
+__device__ __forceinline__ float ehvi_partial_sat(const float* mu, const float* sd, const float4* bs, int n_boxes,
+                                                 const float4* eps, int n_mc, int first, int stride) {
+    constexpr int kCh = 8;
+    float total = 0.0f;
+    for (int s0 = first * kCh; s0 < n_mc; s0 += stride * kCh) {
+        float y[kCh][M], acc[kCh];
+#pragma unroll
+        for (int k = 0; k < kCh; ++k) {
+            acc[k] = 0.0f;
+            const bool in = s0 + k < n_mc;
+            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float ev[4] = {e.x, e.y, e.z, e.w};
+#pragma unroll
+            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
+        }
+        for (int b = 0; b < n_boxes; ++b) {
+            const float4 q0 = bs[2 * b];
+            const float4 q1 = (M > 2) ? bs[2 * b + 1] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float W = M > 2 ? q1.z : bs[2 * b + 1].z;
+            const float Cc = M > 2 ? q1.w : bs[2 * b + 1].w;
+#pragma unroll
+            for (int k = 0; k < kCh; ++k) {
+                float p = __saturatef(fmaf(y[k][0], q0.x, q0.y));
+                if (M > 2) p *= __saturatef(fmaf(y[k][1], q0.z, q0.w));
+                if (M > 3) p *= __saturatef(fmaf(y[k][2], q1.x, q1.y));
+                acc[k] = fmaf(p, fmaxf(fmaf(y[k][M - 1], W, Cc), 0.0f), acc[k]);
             }
         }
 #pragma unroll
@@ -125,7 +182,7 @@ __device__ __forceinline__ bool boxes_fast(const float4* bhi, int n_boxes, int M
 // branch.  The categorical part of r^2 depends only on the candidate's joint
 // category pattern and is read from the host-built table (one load).
 template <int EPI, int M, int DO>
-__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO <= 8) ? 6 : 1)
+__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 6 : 1)
 score_kernel(const __grid_constant__ ScoreArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
@@ -135,7 +192,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     float* Lt = al + n_pad;                                           // [kCJ][kRB]
     float* part = Lt + kCJ * kRB;                                     // [8][kTC]
     float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [kMaxD] feature map
-    float4* blo = fm + kMaxD;
+    float4* blo = fm + kMaxD;                          // [B] (general boxes) or [2B] (saturated form)
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
     float4* epsv = bhi + (EPI == kEHVI ? a.n_boxes : 0);
 
@@ -155,7 +212,13 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
     if (tid < kMaxD) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
     __syncthreads();
+    // Boxes open on the last objective (as scoot_boxes_build makes them) are
+    // restaged in saturated form over the same storage (2 float4 per box).
     const bool fast = EPI == kEHVI ? boxes_fast(bhi, a.n_boxes, M) : false;
+    if (EPI == kEHVI && fast) {
+        stage_boxes_sat(a.box_lo, a.box_hi, a.n_boxes, M, blo);
+        __syncthreads();
+    }
     const int n_ord = a.n_ord;
 
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
@@ -312,8 +375,8 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             float sd[kMaxM];
 #pragma unroll
             for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
-            const float v = fast ? ehvi_partial<M, true>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2)
-                                 : ehvi_partial<M, false>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2);
+            const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, a.n_boxes, epsv, a.n_mc, half, 2)
+                                 : ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2);
             __syncthreads();  // part is free again
             part[half * kTC + slot] = v;
             __syncthreads();

@@ -414,3 +414,22 @@ def test_round_selects_valid_top_q(S, ctx, name):
     # every pick is within tolerance of the oracle's c-th best value among these candidates
     kth = np.sort(oacq)[::-1][c - 1]
     assert np.all(oacq[pos] >= kth - tol[pos] - tol[np.argsort(oacq)[::-1][c - 1]])
+
+
+def test_out_of_range_category_is_reported_not_read(S, ctx):
+    """A category index outside 0..n_choices-1 is clamped inside the kernel
+    (no read outside the state) and reported as SCOOT_EDEVICE by the next
+    context check; the check clears the flag."""
+    inst = make_instance("d8-ehvi2", seeds("d8-ehvi2")[2], n_cand=256)
+    cat_cols = [c for c in range(inst.d) if inst.space[c]["kind"] == 2]
+    words = inst.cand.copy()
+    words[cat_cols[0], 5] = np.uint32(7)
+    L, state = gp_state(S, inst)
+    mean = torch.empty((2, 256), device="cuda")
+    var = torch.empty((2, 256), device="cuda")
+    S.scoot_gp_posterior(ctx, L, state, dev(words.view(np.int32)), 256, mean, var)
+    with pytest.raises(S.ScootError) as e:
+        ctx.check()
+    assert e.value.status == -4
+    ctx.check()  # cleared
+    assert np.all(np.isfinite(np_(mean)))
