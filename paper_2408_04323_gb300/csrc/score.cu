@@ -182,7 +182,7 @@ __device__ __forceinline__ bool boxes_fast(const float4* bhi, int n_boxes, int M
 // branch.  The categorical part of r^2 depends only on the candidate's joint
 // category pattern and is read from the host-built table (one load).
 template <int EPI, int M, int DO>
-__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 6 : 1)
+__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 5 : 1)
 score_kernel(const __grid_constant__ ScoreArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
