@@ -50,7 +50,7 @@ KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["scor
 TRAFFIC = {
     ("prune", "d8-ehvi2"): {"bytes": 3152896, "sha": "8774c0f1248b1325"},
     ("rf", "d8-ehvi2"): {"bytes": 8809984, "sha": "8774c0f1248b1325"},
-    ("score", "d8-ehvi2"): {"bytes": 8839424, "sha": "64abd094c32aaec2"},
+    ("score", "d8-ehvi2"): {"bytes": 8843520, "sha": "28fc276540321214"},
 }
 
 

@@ -1,14 +1,16 @@
 // GP posterior (Section 4.3) and acquisition values: EI (Eq. 6) and
 // Monte-Carlo EHVI over a box decomposition (Eq. 7), fused or separate.
 //
-// A block of 64 threads owns a tile of 64 candidates.  Per objective:
-//  1. each thread evaluates its candidate's covariance row k(x, X) against
-//     the n observations (staged in shared memory) into Ks[j][c] and
-//     accumulates mu = k . alpha;
+// A block of 128 threads (two per candidate) owns a tile of 64 candidates.
+// Per objective:
+//  1. the two threads of a candidate evaluate its covariance row k(x, X)
+//     against the n observations (staged in shared memory) into Ks[j][c],
+//     splitting j by parity, and accumulate mu = k . alpha;
 //  2. the block computes V = L^{-1} Ks as a register-tiled SIMT product
-//     (8 candidates x 8 rows per thread) over 32 x 64 tiles of L^{-1} that the
-//     host laid out transposed and zero-filled, and reduces sum_i V_ic^2;
-//     sigma^2 = s_f^2 - sum_i V_ic^2, clamped at 0.
+//     (4 candidates x 8 rows per thread) over 32 x 64 tiles of L^{-1} that the
+//     host laid out transposed and zero-filled; the tiles are double-buffered
+//     in shared memory by cp.async, so the next tile streams in while the
+//     current one is multiplied; sigma^2 = s_f^2 - sum_i V_ic^2, clamped at 0.
 // The epilogue writes mu and sigma^2, or the EI, or the EHVI of the tile.
 #include <cstring>
 
@@ -165,6 +167,21 @@ __device__ __forceinline__ bool boxes_fast(const float4* bhi, int n_boxes, int M
     return __syncthreads_and(ok) != 0;
 }
 
+// Asynchronous copy of one 32 x 64 tile of L^{-1} (8 KiB, 16-byte aligned at
+// both ends) into shared memory: each of the 128 threads moves four 16-byte
+// pieces with cp.async and commits them as one group.
+__device__ __forceinline__ void stage_tile_async(float* dst, const float4* src, int tid) {
+#pragma unroll
+    for (int k = 0; k < kCJ * kRB / 4 / kThreads; ++k) {
+        const unsigned s = (unsigned)__cvta_generic_to_shared(dst + 4 * (tid + k * kThreads));
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(src + tid + k * kThreads) : "memory");
+    }
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+
+// Waits until every cp.async group this thread committed has landed.
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
+
 // One block of 128 threads scores a tile of 64 candidates; thread t works on
 // candidate slot t % 64 with its partner t +- 64 ("half" t / 64):
 //  1. both halves compute the candidate's features; for each objective the
@@ -189,8 +206,8 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     float* Ks = sm;                                                   // [n_pad][kTC]
     float* xs = Ks + (size_t)n_pad * kTC;                             // [n_obs][DO] ordinal features
     float* al = xs + (size_t)a.n_obs * DO;                            // [n_pad]
-    float* Lt = al + n_pad;                                           // [kCJ][kRB]
-    float* part = Lt + kCJ * kRB;                                     // [8][kTC]
+    float* Lt = al + n_pad;                                           // [2][kCJ][kRB] double buffer
+    float* part = Lt + 2 * kCJ * kRB;                                 // [8][kTC]
     float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [kMaxD] feature map
     float4* blo = fm + kMaxD;                          // [B] (general boxes) or [2B] (saturated form)
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
@@ -251,7 +268,9 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
         }
         float mu[kMaxM], vr[kMaxM];
         for (int m = 0; m < nobj; ++m) {
-            __syncthreads();  // previous users of xs / al / part are done
+            __syncthreads();  // previous users of xs / al / part / Lt are done
+            const float4* tiles = glinv + (size_t)m * a.n_tiles * (kCJ * kRB / 4);
+            stage_tile_async(Lt, tiles, tid);  // tile 0 lands while the covariance row is computed
             const float* sx = gxs + (size_t)m * a.n_obs * a.d;
             for (int e = tid; e < a.n_obs * DO; e += kThreads) {
                 const int j = e / DO, q = e - j * DO;
@@ -291,9 +310,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             // 2. V = L^{-1} Ks and the sum of squares per candidate.
             const int cg = tid & 15, rg = tid >> 4;
             float sq[4] = {0.f, 0.f, 0.f, 0.f};
-            const float4* tiles = glinv + (size_t)m * a.n_tiles * (kCJ * kRB / 4);
             const float4* Ks4 = reinterpret_cast<const float4*>(Ks);
-            const float4* Lt4 = reinterpret_cast<const float4*>(Lt);
             int t = 0;
             for (int rb = 0; rb < a.n_rb; ++rb) {
                 float accm[8][4];
@@ -302,12 +319,14 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
 #pragma unroll
                     for (int c = 0; c < 4; ++c) accm[r][c] = 0.0f;
                 for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t) {
+                    // Tile t has landed in buffer t&1 and every thread is done
+                    // with tile t-1, so tile t+1 may overwrite buffer (t+1)&1
+                    // while tile t is multiplied.
+                    cp_async_wait_all();
                     __syncthreads();
-                    const float4* src = tiles + (size_t)t * (kCJ * kRB / 4);
-#pragma unroll
-                    for (int k = 0; k < kCJ * kRB / 4 / kThreads; ++k)
-                        reinterpret_cast<float4*>(Lt)[tid + k * kThreads] = __ldg(src + tid + k * kThreads);
-                    __syncthreads();
+                    if (t + 1 < a.n_tiles)
+                        stage_tile_async(Lt + ((t + 1) & 1) * (kCJ * kRB), tiles + (size_t)(t + 1) * (kCJ * kRB / 4), tid);
+                    const float4* Lt4 = reinterpret_cast<const float4*>(Lt + (t & 1) * (kCJ * kRB));
                     // rows of this warp: rb*64 + 16*warp .. +15; columns cj*32 .. +31;
                     // L^{-1} is zero right of the diagonal, so a warp stops at its
                     // last row (in steps of 16 columns).
@@ -451,7 +470,7 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
 
 size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
-    size_t f = n_pad * kTC + (size_t)a.n_obs * DO + n_pad + kCJ * kRB + 8 * kTC + 4 * kMaxD;
+    size_t f = n_pad * kTC + (size_t)a.n_obs * DO + n_pad + 2 * kCJ * kRB + 8 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
     return f * 4;
 }
