@@ -16,7 +16,9 @@ Steps, in the order of one suggestion round (Section 4, Algorithm 1):
 5. top-q selection for parallel suggestion (Section 4.7);
 6. sequential picks with kriging-believer fantasies (not in the paper; the
    refit form is used here: each pick is appended to the observations with
-   its posterior mean as value and the GP is conditioned again).
+   its posterior mean as value and the GP is conditioned again);
+7. MACE for single-objective suggestion (Sections 4.5 and 4.7): UCB, PI and
+   EI on the same posterior, their Pareto front, and a random k-subset of it.
 
 Readings of points the paper leaves open are marked "Reading:".
 Every function is pinned by the not-gpu tests against closed forms,
@@ -489,3 +491,95 @@ def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
             gp.add_observations(u_pool[p:p + 1], [mu0[p, m]])
         Yf = np.concatenate([Yf, mu0[p:p + 1]], axis=0)
     return dict(picks=picks, acq=acqs, var=vars_, mu=mus, fronts=fronts)
+
+
+# --------------------------------------------------------------------------
+# 7. MACE for single-objective suggestion (Sections 4.5 and 4.7)
+
+def upper_confidence_bound(mu, var, kappa: float):
+    """UCB(x) = mu(x) + beta * sigma(x), the UCB equation of Section 4.5.
+
+    Reading: the coefficient multiplies sigma as printed; its value for
+    tuning iteration t (beta_t of Section 4.5) is computed by the caller
+    and passed in as ``kappa``."""
+    sd = np.sqrt(np.maximum(np.asarray(var, np.float64), 0.0))
+    return np.asarray(mu, np.float64) + float(kappa) * sd
+
+
+def probability_of_improvement(mu, var, y_best: float, xi: float = 1e-4):
+    """PI(x) = P(f(x) + xi > f(x+)) for f(x) ~ N(mu, sigma^2), the PI equation
+    of Section 4.5: Phi((mu + xi - y+) / sigma).
+
+    Reading: with sigma = 0 the event is certain when mu + xi > y+ and
+    impossible otherwise (strict inequality, as printed)."""
+    mu = np.asarray(mu, np.float64)
+    sd = np.sqrt(np.maximum(np.asarray(var, np.float64), 0.0))
+    a = mu - y_best + xi
+    pos = sd > 0
+    z = np.where(pos, a / np.where(pos, sd, 1.0), 0.0)
+    return np.where(pos, norm_cdf(z), (a > 0).astype(np.float64))
+
+
+def mace_acquisitions(mu, var, y_best: float, xi: float, kappa: float) -> np.ndarray:
+    """The three acquisition values MACE ranks candidates by (Section 4.5):
+    rows UCB, PI, EI, each to be maximised."""
+    return np.stack([upper_confidence_bound(mu, var, kappa),
+                     probability_of_improvement(mu, var, y_best, xi),
+                     expected_improvement(mu, var, y_best, xi)])
+
+
+def nondominated(Y) -> np.ndarray:
+    """Boolean mask of the rows of Y (points, maximised) that no other row
+    dominates: row j dominates row i when Y_j >= Y_i in every column and
+    Y_j > Y_i in at least one.  Equal rows do not dominate each other, so
+    duplicates of a front point are all on the front.  Straight from the
+    definition: every pair is compared (in blocks of rows)."""
+    Y = np.asarray(Y, np.float64)
+    n = len(Y)
+    out = np.ones(n, bool)
+    for s in range(0, n, 256):
+        blk = Y[s:s + 256]
+        ge = np.all(Y[None, :, :] >= blk[:, None, :], axis=2)
+        gt = np.any(Y[None, :, :] > blk[:, None, :], axis=2)
+        out[s:s + 256] = ~np.any(ge & gt, axis=1)
+    return out
+
+
+_SM_GAMMA = 0x9E3779B97F4A7C15
+_SM_MASK = (1 << 64) - 1
+
+
+def splitmix64(seed: int, i: int) -> int:
+    """Output i (0-based) of the SplitMix64 generator seeded with ``seed``
+    (Steele, Lea and Flood, OOPSLA 2014, in the form Vigna publishes): the
+    state after i + 1 steps is seed + (i + 1) * 0x9E3779B97F4A7C15, passed
+    through the generator's 64-bit finaliser."""
+    z = (seed + (i + 1) * _SM_GAMMA) & _SM_MASK
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _SM_MASK
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _SM_MASK
+    return z ^ (z >> 31)
+
+
+def mace_select(acq3, mask, k: int, seed: int):
+    """k candidates drawn at random from the Pareto front of (UCB, PI, EI)
+    (Section 4.7: for SOBO, the k suggestions are picked at random from the
+    front of the three acquisition functions).
+
+    Reading: eligible candidates are those with mask set whose three values
+    are neither NaN nor -inf; the front is taken over eligible candidates
+    only.  The random draw gives candidate i the key splitmix64(seed, i) and
+    takes the k front members with the smallest keys (the lower index on
+    equal keys), in that order: a uniformly random k-subset in random order.
+    A front smaller than k is returned whole.
+
+    Returns (picks, front indices in ascending order, number of picks)."""
+    A = np.asarray(acq3, np.float64)
+    n = A.shape[1]
+    ok = ~np.any(np.isnan(A) | (A == -np.inf), axis=0)
+    if mask is not None:
+        ok &= np.asarray(mask, bool)[:n]
+    idx = np.nonzero(ok)[0]
+    front = idx[nondominated(A[:, idx].T)] if len(idx) else idx
+    order = sorted(front.tolist(), key=lambda i: (splitmix64(seed, i), i))
+    picks = np.array(order[:k], np.int64)
+    return picks, np.sort(front).astype(np.int64), len(picks)

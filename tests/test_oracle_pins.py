@@ -503,3 +503,127 @@ def test_fantasy_refit_properties():
     s, t = var0[p], 2e-3
     assert var1[p] == pytest.approx(s * t / (s + t), rel=1e-8)
     assert np.allclose(var1, np.maximum(var0 - c * c, 0), rtol=1e-8, atol=1e-11)
+
+
+# ------------------------------------------------------------------ MACE (Sections 4.5 and 4.7)
+
+def test_pi_closed_form_matches_quadrature():
+    """PI = P(f + xi > y+) is the Gaussian density integrated above y+ - xi."""
+    xi = 1e-4
+    for mu, sd, yb in [(0.0, 1.0, 0.0), (-1.3, 0.2, 0.5), (2.0, 0.5, 1.0), (0.3, 3.0, 2.0), (-4, 0.7, 0.0)]:
+        pdf = lambda y: math.exp(-0.5 * ((y - mu) / sd) ** 2) / (sd * math.sqrt(2 * math.pi))
+        lo = yb - xi
+        q, _ = integrate.quad(pdf, lo, mu + 14 * sd, epsabs=1e-14, epsrel=1e-12, limit=200) if lo < mu + 14 * sd else (0.0, 0)
+        assert O.probability_of_improvement(mu, sd * sd, yb, xi) == pytest.approx(q, rel=1e-9, abs=1e-13)
+
+
+def test_pi_is_the_mean_derivative_of_ei():
+    """d EI / d mu = Phi(z) = PI: ties the two closed forms to each other."""
+    h = 1e-6
+    for mu, var, yb in [(0.1, 0.3, 0.4), (-2.0, 1.5, 0.0), (1.2, 0.01, 1.0)]:
+        d = (O.expected_improvement(mu + h, var, yb) - O.expected_improvement(mu - h, var, yb)) / (2 * h)
+        assert float(d) == pytest.approx(float(O.probability_of_improvement(mu, var, yb)), abs=1e-8)
+
+
+def test_pi_and_ucb_limits():
+    # sigma = 0: a certain event exactly when mu + xi > y+ (strict)
+    assert np.array_equal(O.probability_of_improvement(np.array([0.5, 1.0, 1.5]), 0.0, 1.0, 0.0), [0.0, 0.0, 1.0])
+    assert np.allclose(O.upper_confidence_bound(np.array([0.5, -2.0]), 0.0, 7.0), [0.5, -2.0])
+    # mu + kappa sigma is the Phi(kappa) quantile of N(mu, sigma^2) (library quantile)
+    from scipy.stats import norm
+    for mu, sd, kappa in [(0.3, 0.2, 1.5), (-1.0, 2.0, 0.5), (2.0, 0.1, 3.0)]:
+        want = norm.ppf(norm.cdf(kappa), loc=mu, scale=sd)
+        assert O.upper_confidence_bound(mu, sd * sd, kappa) == pytest.approx(want, rel=1e-9)
+    mus = np.linspace(-3, 3, 40)
+    assert np.all(np.diff(O.probability_of_improvement(mus, 0.3, 0.0)) > 0)
+    A = O.mace_acquisitions(np.array([0.1]), np.array([0.04]), 0.2, 1e-4, 2.0)
+    assert A.shape == (3, 1) and A[0, 0] == pytest.approx(0.5)
+
+
+def _front_2d_sweep(P):
+    """Textbook 2-D maxima: sort by x descending (y descending on ties) and
+    keep a point when its y is at least the best y seen among points with a
+    strictly larger x, and it equals the previous kept point or beats every
+    y seen so far."""
+    order = sorted(range(len(P)), key=lambda i: (-P[i][0], -P[i][1]))
+    keep, best_y, prev = [], -math.inf, None
+    for i in order:
+        x, y = P[i]
+        if y > best_y or (prev is not None and (x, y) == prev):
+            keep.append(i)
+            prev = (x, y)
+        best_y = max(best_y, y)
+    return sorted(keep)
+
+
+def test_nondominated_matches_2d_sweep():
+    st = Stream(41, "front2d")
+    for trial in range(20):
+        n = 1 + trial * 7
+        P = np.floor(st.uniform(2 * n).reshape(n, 2) * (3 + trial)).tolist()
+        got = np.nonzero(O.nondominated(np.array(P)))[0].tolist()
+        assert got == _front_2d_sweep([tuple(p) for p in P])
+
+
+@pytest.mark.parametrize("M", [3, 4])
+def test_nondominated_is_the_maxima_set(M):
+    """The unique set that is mutually non-dominating and dominates every
+    other point; permutation-invariant; unchanged by a dominated point;
+    duplicates of front points all kept."""
+    st = Stream(42 + M, "frontMd")
+    dom = lambda a, b: all(x >= y for x, y in zip(a, b)) and any(x > y for x, y in zip(a, b))
+    for trial in range(12):
+        n = 5 + 9 * trial
+        Y = np.floor(st.uniform(M * n).reshape(n, M) * 4)
+        f = O.nondominated(Y)
+        F = [tuple(Y[i]) for i in np.nonzero(f)[0]]
+        assert f.any()
+        for i in range(n):
+            dominated = any(dom(tuple(Y[j]), tuple(Y[i])) for j in range(n))
+            assert f[i] == (not dominated)
+            if not f[i]:
+                assert any(dom(p, tuple(Y[i])) for p in F)
+        perm = np.argsort(st.uniform(n))
+        assert np.array_equal(O.nondominated(Y[perm]), f[perm])
+        worst = Y.min(axis=0) - 1
+        assert np.array_equal(O.nondominated(np.vstack([Y, worst]))[:n], f)
+        i0 = int(np.nonzero(f)[0][0])
+        f2 = O.nondominated(np.vstack([Y, Y[i0]]))
+        assert f2[-1] and np.array_equal(f2[:n], f)
+
+
+def test_splitmix64_published_outputs(golden_dir):
+    lines = [l for l in open(os.path.join(golden_dir, "splitmix64_seed0.txt")) if not l.startswith("#")]
+    assert lines[0].split() == ["seed", "0"]
+    want = [int(l, 16) for l in lines[1:]]
+    assert [O.splitmix64(0, i) for i in range(len(want))] == want
+
+
+def test_mace_select_draws_from_the_front():
+    st = Stream(44, "mace")
+    n = 400
+    A = np.floor(st.uniform(3 * n).reshape(3, n) * 6)
+    mask = st.uniform(n) < 0.8
+    A[0, 5] = np.nan
+    A[1, 6] = -np.inf
+    picks, front, cnt = O.mace_select(A, mask, 4, seed=7)
+    ok = mask.copy()
+    ok[[5, 6]] = False
+    idx = np.nonzero(ok)[0]
+    assert np.array_equal(front, idx[O.nondominated(A[:, idx].T)])
+    assert cnt == min(4, len(front)) and set(picks) <= set(front) and len(set(picks)) == cnt
+    keys = [O.splitmix64(7, int(i)) for i in picks]
+    assert keys == sorted(keys)
+    assert all(O.splitmix64(7, int(i)) > keys[-1] for i in set(front) - set(picks))
+    # a front smaller than k comes back whole; nothing eligible gives nothing
+    p2, f2, c2 = O.mace_select(A, mask, len(front) + 3, seed=1)
+    assert c2 == len(front) and sorted(p2) == sorted(front)
+    p3, f3, c3 = O.mace_select(A, np.zeros(n, bool), 4, seed=1)
+    assert c3 == 0 and len(p3) == 0 and len(f3) == 0
+    # over many seeds every front member is drawn about k / F of the time
+    F = len(front)
+    counts = np.zeros(n)
+    for s in range(2000):
+        counts[O.mace_select(A, mask, 2, seed=s)[0]] += 1
+    freq = counts[front] / 2000
+    assert np.all(np.abs(freq - 2 / F) < 5 * math.sqrt((2 / F) * (1 - 2 / F) / 2000) + 1e-9)
