@@ -46,7 +46,7 @@ FP32_LANES_PER_SM = 128
 # unchanged (sha256 prefix of their contents when the counters were taken);
 # the captures are summarised in profiles/kernels_full_<workload>.md.
 KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["score.cu", "device_common.cuh"],
-                "topq": ["topq.cu", "device_common.cuh"]}
+                "topq": ["topq.cu", "device_common.cuh"], "pareto": ["pareto.cu"]}
 TRAFFIC = {
     ("prune", "d8-ehvi2"): {"bytes": 3152896, "sha": "8774c0f1248b1325"},
     ("rf", "d8-ehvi2"): {"bytes": 8809984, "sha": "8774c0f1248b1325"},
@@ -61,6 +61,8 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--acq", choices=["default", "mace"], default="default",
+                   help="mace: UCB/PI/EI and a random subset of their Pareto front (one objective)")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the cpu_baseline sample")
     p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -68,12 +70,13 @@ def parse_args():
     return p.parse_args()
 
 
-def workload_config(w, extra=None):
-    desc = (f"{w.name}: d={w.d}, n={w.n_obs}, N={w.n_cand}, M={w.n_obj} {w.acq.upper()}"
+def workload_config(w, extra=None, acq=None):
+    acq = acq or w.acq
+    desc = (f"{w.name}: d={w.d}, n={w.n_obs}, N={w.n_cand}, M={w.n_obj} {acq.upper()}"
             + (f" S={w.n_mc}" if w.acq == "ehvi" else "")
             + f", RF {w.n_trees} trees depth<={w.max_depth}, q={w.q}")
     cfg = {"workload": desc, "pool": w.n_cand, "observations": w.n_obs, "objectives": w.n_obj,
-           "acquisition": w.acq, "trees": w.n_trees, "q": w.q,
+           "acquisition": acq, "trees": w.n_trees, "q": w.q,
            "l2": "flushed between steps (256 MiB write)", "inputs": "seeded synthetic pool, resident in HBM"}
     if extra:
         cfg.update(extra)
@@ -97,18 +100,21 @@ def referenced_columns(inst):
     return len(cols)
 
 
-def work_model(inst, n_boxes):
+def work_model(inst, n_boxes, acq_kind=None):
     """Algorithmic work per candidate of each stage (bytes or flops)."""
     w = inst.workload
+    acq_kind = acq_kind or w.acq
     d, n = inst.d, inst.n_obs
-    m_eff = 1 if w.acq == "ei" else inst.n_obj
+    m_eff = inst.n_obj if acq_kind == "ehvi" else 1
     post = m_eff * (n * (3 * d + 12) + 2 * n + n * (n + 1) + 2 * n)
-    acq = 30 if w.acq == "ei" else w.n_mc * n_boxes * 4 * inst.n_obj
+    # EI ~30 flops; MACE adds PI (~15) and UCB (2)
+    acq = {"ei": 30, "mace": 47}.get(acq_kind, w.n_mc * n_boxes * 4 * inst.n_obj)
     return {
         "prune": ("hbm", 4 * referenced_columns(inst) + 1),
         "rf": ("hbm", 4 * d + 1 + 1 + 4),
         "score": ("alu", post + acq),
         "topq": ("hbm", 4 + 1),
+        "pareto": ("hbm", 12 + 1),
     }
 
 
@@ -161,29 +167,38 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(loaded)}
 
 
-def cpu_oracle_sample(name, seed, n_sample, threads=1):
-    """Time the oracle on n_sample candidates of the workload in a fresh process."""
+def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None):
+    """Time the oracle on n_sample candidates of the workload in a fresh process
+    (with mace_kappa set: the MACE round, UCB coefficient mace_kappa)."""
     env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
                MKL_NUM_THREADS=str(threads))
+    if mace_kappa is None:
+        select = ("r = oracle.score_round(inst, inst.workload.acq)\n"
+                  "oracle.select_topq(r['acq'], r['feasible'], inst.workload.q)\n")
+    else:
+        select = ("r = oracle.score_round(inst, 'ei')\n"
+                  "A = oracle.mace_acquisitions(r['mu'][:, 0], r['var'][:, 0], float(inst.y_obs[0].max()), "
+                  "1e-4, %r)\n"
+                  "A[:, ~r['feasible']] = -np.inf\n"
+                  "oracle.mace_select(A, r['feasible'], inst.workload.q, 0)\n" % float(mace_kappa))
     code = (
         "import sys, time, json; sys.path.insert(0, %r)\n"
         "import numpy as np, oracle\n"
         "from workloads import make_instance\n"
         "inst = make_instance(%r, %d, n_cand=%d)\n"
-        "t = time.perf_counter()\n"
-        "r = oracle.score_round(inst, inst.workload.acq)\n"
-        "oracle.select_topq(r['acq'], r['feasible'], inst.workload.q)\n"
-        "print(json.dumps({'seconds': time.perf_counter() - t}))\n" % (ROOT, name, seed, n_sample))
+        "t = time.perf_counter()\n" % (ROOT, name, seed, n_sample)
+        + select
+        + "print(json.dumps({'seconds': time.perf_counter() - t}))\n")
     p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
     if p.returncode != 0:
         raise RuntimeError(p.stderr[-2000:])
     return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
 
 
-def calibrate_sample(name, seed, budget_s):
+def calibrate_sample(name, seed, budget_s, mace_kappa=None):
     """Largest sample whose oracle round fits the budget (scaled from a probe)."""
     probe = 64
-    t = cpu_oracle_sample(name, seed, probe)
+    t = cpu_oracle_sample(name, seed, probe, mace_kappa=mace_kappa)
     per = max(t / probe, 1e-6)
     return max(16, int(budget_s / per))
 
@@ -195,18 +210,23 @@ def run_reference(args):
         return
     w = WORKLOADS[args.workload]
     seed = seeds(w.name)[0]
+    kappa = None
+    if args.acq == "mace":
+        from paper_2408_04323_gb300.pipeline import mace_beta
+        kappa = mace_beta(w.n_obs)
     per_step = max(0.05, 120.0 / max(1, args.steps + args.warmup))
-    sample = calibrate_sample(w.name, seed, per_step)
+    sample = calibrate_sample(w.name, seed, per_step, kappa)
     for _ in range(args.warmup):
-        cpu_oracle_sample(w.name, seed, sample)
-    times = [cpu_oracle_sample(w.name, seed, sample) for _ in range(args.steps)]
+        cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa)
+    times = [cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa) for _ in range(args.steps)]
     ms = 1e3 * statistics.mean(times)
     value = sample / (ms / 1e3)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(w, {"reference": "fp64 CPU oracle (the paper ships no code)",
-                                          "sample_per_step": sample}),
+                                          "sample_per_step": sample},
+                                      acq=None if args.acq == "default" else args.acq),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{sample} candidates of the {w.name} pool per step, all five steps"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -240,6 +260,11 @@ def main():
     from workloads import WORKLOADS, Stream, draw_configs, make_instance, seeds
 
     w = WORKLOADS[args.workload]
+    acq_kind = w.acq if args.acq == "default" else args.acq
+    if acq_kind == "mace" and (w.n_obj != 1 or w.fantasy):
+        raise SystemExit("--acq mace needs a one-objective workload")
+    if acq_kind == "mace" and world > 1:
+        raise SystemExit("--acq mace runs on one GPU: its front is not merged across ranks")
     seed = seeds(w.name)[0]
     inst = make_instance(w.name, seed)
     cand_np = inst.cand
@@ -248,7 +273,7 @@ def main():
     N = inst.n_cand
     inp = RoundInputs(inst.space, inst.clauses, inst.nodes, inst.tree_offset, w.leaf_scale, w.delta_num,
                       w.delta_den, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
-                      inst.noise_var, inst.ref, inst.eps, w.acq, w.q, fantasy=w.fantasy)
+                      inst.noise_var, inst.ref, inst.eps, acq_kind, w.q, fantasy=w.fantasy)
     ctx = S.Context(device.index)
     rnd = ScoringRound(ctx, inp, N, device)
     cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
@@ -277,12 +302,20 @@ def main():
             return
         if inp.acq == "ei":
             S.scoot_score_ei(ctx, st.gp_layout, st.gp_state, cand, N, inp.xi, rnd.acq, rnd.mask, stream)
+        elif inp.acq == "mace":
+            S.scoot_score_mace(ctx, st.gp_layout, st.gp_state, cand, N, inp.xi, rnd.kappa, rnd.acq3, rnd.mask,
+                               stream)
         else:
             S.scoot_score_ehvi(ctx, st.gp_layout, st.gp_state, cand, N, st.box_lo, st.box_hi, st.eps,
                                rnd.acq, rnd.mask, stream)
         if evs:
             evs[3].record(stream)
-        S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask, stream)
+        if inp.acq == "mace":
+            S.scoot_select_pareto(ctx, rnd.acq3, N, inp.q, rnd.seed, rnd.top_idx, rnd.top_count, rnd.mask,
+                                  rnd.front, stream)
+        else:
+            S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask,
+                                stream)
         if evs:
             evs[4].record(stream)
 
@@ -310,7 +343,7 @@ def main():
         flush.fill_(kk & 0xFF)
         step(evs[kk])
     torch.cuda.synchronize(device)
-    stage_names = ["prune", "rf", "score", "topq"]
+    stage_names = ["prune", "rf", "score", "pareto" if inp.acq == "mace" else "topq"]
     stage_ms = {s: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, s in enumerate(stage_names)}
     eager_ms = statistics.mean(e[0].elapsed_time(e[4]) for e in evs)
 
@@ -364,12 +397,12 @@ def main():
     peaks, peak_src = measured_peaks()
     sms = torch.cuda.get_device_properties(device).multi_processor_count
     fp32_peak = sms * FP32_LANES_PER_SM * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # TFLOP/s
-    work = work_model(inst, st.n_boxes)
+    work = work_model(inst, st.n_boxes, inp.acq)
     dom = max(stage_names, key=lambda s: stage_ms[s])
     kind, per_cand = work[dom]
     units = n_feasible if dom == "score" else N
     launch_s = stage_ms[dom] / 1e3
-    tr = TRAFFIC.get((dom, w.name))
+    tr = TRAFFIC.get((dom, w.name if inp.acq == w.acq else f"{w.name}/{inp.acq}"))
     traffic = tr["bytes"] if tr and tr["sha"] == sources_sha(dom) else None
     if kind == "hbm":
         achieved = per_cand * units / launch_s / 1e9
@@ -414,10 +447,15 @@ def main():
                 rnd.top_idx[:len(idx_h)].copy_(torch.from_numpy(idx_h))
             elif inp.acq == "ei":
                 S.scoot_score_ei(ctx, state.gp_layout, state.gp_state, cand_e2e, N, inp.xi, rnd.acq, rnd.mask, stream)
+            elif inp.acq == "mace":
+                S.scoot_score_mace(ctx, state.gp_layout, state.gp_state, cand_e2e, N, inp.xi, rnd.kappa, rnd.acq3,
+                                   rnd.mask, stream)
+                S.scoot_select_pareto(ctx, rnd.acq3, N, inp.q, rnd.seed, rnd.top_idx, rnd.top_count, rnd.mask,
+                                      rnd.front, stream)
             else:
                 S.scoot_score_ehvi(ctx, state.gp_layout, state.gp_state, cand_e2e, N, state.box_lo, state.box_hi,
                                    state.eps, rnd.acq, rnd.mask, stream)
-            if not inp.fantasy:
+            if not inp.fantasy and inp.acq != "mace":
                 S.scoot_select_topq(ctx, rnd.acq, N, inp.q, rnd.top_idx, rnd.top_val, rnd.top_count, rnd.mask,
                                     stream)
             picks = (rnd.top_idx.cpu(), rnd.top_val.cpu(), rnd.top_count.cpu())
@@ -440,8 +478,9 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        sample = calibrate_sample(w.name, seed, args.cpu_seconds)
-        secs = cpu_oracle_sample(w.name, seed, sample)
+        kappa = rnd.kappa if inp.acq == "mace" else None
+        sample = calibrate_sample(w.name, seed, args.cpu_seconds, kappa)
+        secs = cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa)
         cpu = {"value": sample / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"{sample} candidates of the {w.name} pool (same round state), all five steps, "
                          f"fp64 numpy, one thread"}
@@ -454,7 +493,7 @@ def main():
                                               "front": st.front_size, "parallelism": f"pool shards x{world}",
                                               "launch": "CUDA graph of the step" if graph is not None
                                               else "eager launches",
-                                              "eager_ms_per_step": round(eager_ms, 5)}),
+                                              "eager_ms_per_step": round(eager_ms, 5)}, acq=inp.acq),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps * rnd.kernels_per_round(),
                 "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},

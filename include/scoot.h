@@ -12,6 +12,8 @@
  *   scoot_score_ei       posterior + EI in one kernel
  *   scoot_score_ehvi     posterior + EHVI in one kernel
  *   scoot_select_topq    top-q for parallel suggestion (Section 4.7)
+ *   scoot_score_mace     posterior + UCB, PI, EI for MACE (Section 4.5)
+ *   scoot_select_pareto  random k-subset of the (UCB, PI, EI) front (Section 4.7)
  *
  * plus host-side preparation of per-round state (Cholesky factor of the
  * observations' covariance, box decomposition of the non-dominated region,
@@ -121,7 +123,8 @@ const char* scoot_last_error(const scoot_ctx* ctx);
 const char* scoot_status_string(scoot_status s);
 /* Wait for `stream`, then read and clear the context's device error word:
  * SCOOT_EDEVICE if a kernel flagged a bad index or value since the last
- * check, SCOOT_ETIMEOUT if a bounded wait gave up, else SCOOT_OK. */
+ * check, SCOOT_ETIMEOUT if a bounded wait gave up, SCOOT_EUNSUPPORTED if a
+ * Pareto filter ran out of survivor capacity, else SCOOT_OK. */
 scoot_status scoot_ctx_check(scoot_ctx* ctx, void* stream);
 /* Bytes of device workspace the context currently holds. */
 scoot_status scoot_ctx_workspace_bytes(const scoot_ctx* ctx, int64_t* bytes);
@@ -322,6 +325,57 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* layout
                                    const uint8_t* mask, const float* h_ref, const float* eps, int32_t n_mc,
                                    int32_t q, void* work, int64_t work_bytes, int64_t* h_idx, float* h_val,
                                    int32_t* h_count, float* var_out, void* stream);
+
+/* ------------------------------------------------------------------ 7. MACE (Sections 4.5 and 4.7) */
+
+/* Candidates that may survive the pivot stage of scoot_select_pareto (see
+ * there). */
+#define SCOOT_PARETO_CAP 65536
+
+/* The three acquisition values MACE ranks single-objective candidates by
+ * (Section 4.5), from the posterior of objective 0:
+ *   UCB = mu + kappa * sigma                  (the UCB equation; kappa is the
+ *                                              coefficient beta_t, given by
+ *                                              the caller)
+ *   PI  = Phi((mu + xi - y_best) / sigma)     (the PI equation; with sigma = 0,
+ *                                              1 if mu + xi > y_best, else 0)
+ *   EI  as in scoot_acq_ei                    (Eq. 6)
+ * acq is [3][lda] (rows UCB, PI, EI; lda >= n); where mask[i] == 0 (mask may
+ * be NULL) all three are -inf.  mean/var: objective 0's rows as written by
+ * scoot_gp_posterior. */
+scoot_status scoot_acq_mace(scoot_ctx* ctx, const float* mean, const float* var, const uint8_t* mask,
+                            int64_t n, float y_best, float xi, float kappa, float* acq, int64_t lda,
+                            void* stream);
+
+/* scoot_gp_posterior followed by scoot_acq_mace, in one kernel (objective 0;
+ * y_best is the state's best observed value of objective 0). */
+scoot_status scoot_score_mace(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                              const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                              float xi, float kappa, float* acq, int64_t lda, void* stream);
+
+/* Parallel suggestion for one objective (Section 4.7): k candidates drawn at
+ * random from the Pareto front of the three rows of acq ([3][lda], each
+ * maximised, e.g. as written by scoot_score_mace).  Eligible candidates have
+ * mask[i] == 1 (mask may be NULL) and no row NaN or -inf; candidate j
+ * dominates i when it is >= in every row and > in one; the front is the
+ * eligible candidates no eligible candidate dominates (equal triples are all
+ * on it).  The draw gives candidate i the key SplitMix64(seed, i) (output i
+ * of the SplitMix64 generator seeded with seed) and takes the k front members
+ * with the smallest keys (lower index on equal keys), in that order: a
+ * uniformly random k-subset.  Outputs (device): idx (int64 [k], -1 beyond
+ * the picks), count (int32 [2]: the number of picks min(k, front size), then
+ * the front size) and, if front is not NULL, the first min(front size,
+ * front_cap) front members in no particular order.
+ * The filter is exact and runs in stages: the front of a strided sample of
+ * at most 16384 candidates serves as pivots; every candidate that no pivot
+ * dominates is kept, and the kept candidates are filtered against each
+ * other.  If more than SCOOT_PARETO_CAP candidates are kept (a front of that
+ * size, or pivots that dominate too little), count is {-1, -1}, no pick is
+ * made and scoot_ctx_check reports SCOOT_EUNSUPPORTED.
+ * 1 <= k <= SCOOT_MAX_Q, n < 2^31. */
+scoot_status scoot_select_pareto(scoot_ctx* ctx, const float* acq, int64_t lda, const uint8_t* mask,
+                                 int64_t n, int32_t k, uint64_t seed, int64_t* idx, int32_t* count,
+                                 int64_t* front, int64_t front_cap, void* stream);
 
 /* scoot_select_topq without a context and without allocating.  The paper
  * has no counterpart: this is a convenience of this library for callers that

@@ -11,7 +11,8 @@ constexpr int kCompactThreads = 256;
 
 __global__ void __launch_bounds__(kCompactThreads)
 compact_kernel(const uint8_t* __restrict__ mask, int64_t n, int32_t* __restrict__ list,
-               unsigned int* __restrict__ count, uint32_t* __restrict__ fill, uint32_t fill_bits) {
+               unsigned int* __restrict__ count, uint32_t* __restrict__ fill, uint32_t fill_bits, int fill_rows,
+               int64_t fill_ld) {
     __shared__ unsigned int warp_count[kCompactThreads / 32];
     __shared__ unsigned int block_base;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -20,7 +21,8 @@ compact_kernel(const uint8_t* __restrict__ mask, int64_t n, int32_t* __restrict_
         const int64_t i = i0 + threadIdx.x;
         const bool in = i < n;
         const bool live = in && mask[i] != 0;
-        if (in && !live && fill) fill[i] = fill_bits;
+        if (in && !live && fill)
+            for (int r = 0; r < fill_rows; ++r) fill[r * fill_ld + i] = fill_bits;
         const unsigned int ballot = __ballot_sync(0xffffffffu, live);
         if (lane == 0) warp_count[warp] = __popc(ballot);
         __syncthreads();
@@ -45,7 +47,7 @@ compact_kernel(const uint8_t* __restrict__ mask, int64_t n, int32_t* __restrict_
 }  // namespace
 
 scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint32_t* fill, uint32_t fill_bits,
-                           cudaStream_t st, ScootList* out) {
+                           cudaStream_t st, ScootList* out, int fill_rows, int64_t fill_ld) {
     if (n > 0x7FFFFFFFll) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "compaction of %lld > 2^31 candidates", (long long)n);
     const size_t bytes = 256 + (size_t)n * sizeof(int32_t);
     scoot_status s = scoot_workspace(ctx, bytes);
@@ -59,7 +61,8 @@ scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint3
     int64_t blocks = (n + kCompactThreads - 1) / kCompactThreads;
     const int64_t cap = (int64_t)(sms > 0 ? sms : 1) * 8;
     if (blocks > cap) blocks = cap;
-    compact_kernel<<<(unsigned)blocks, kCompactThreads, 0, st>>>(mask, n, out->list, out->count, fill, fill_bits);
+    compact_kernel<<<(unsigned)blocks, kCompactThreads, 0, st>>>(mask, n, out->list, out->count, fill, fill_bits,
+                                                                 fill_rows, fill_ld);
     SCOOT_LAUNCHED(ctx);
     return SCOOT_OK;
 }

@@ -25,6 +25,19 @@ __device__ __forceinline__ float ei_value(float mu, float var, float ybest, floa
     return fmaf(a, cdf, s * pdf);
 }
 
+// PI = P(f + xi > y+) = Phi((mu + xi - y+) / sigma); a step at sigma = 0.
+__device__ __forceinline__ float pi_value(float mu, float var, float ybest, float xi) {
+    const float a = (mu - ybest) + xi;
+    const float s = sqrtf(fmaxf(var, 0.0f));
+    if (!(s > 0.0f)) return a > 0.0f ? 1.0f : 0.0f;
+    return 0.5f * erfcf(-(a / s) * 0.70710678118654752f);
+}
+
+// UCB = mu + kappa * sigma.
+__device__ __forceinline__ float ucb_value(float mu, float var, float kappa) {
+    return fmaf(kappa, sqrtf(fmaxf(var, 0.0f)), mu);
+}
+
 // EHVI of one candidate: the mean over the S base samples of the hypervolume
 // improvement, summed over boxes.  Boxes are float4 rows (lo, hi padded to
 // four objectives), base samples float4 rows.  Samples are taken eight at a

@@ -16,6 +16,7 @@
 // Bits of the device error word.
 #define SCOOT_DEVERR_INDEX   1u   // a node, feature or box index out of range
 #define SCOOT_DEVERR_TIMEOUT 2u   // a bounded wait gave up
+#define SCOOT_DEVERR_CAPACITY 4u  // a Pareto filter had more survivors than it can hold
 
 struct scoot_ctx {
     int32_t device = 0;
@@ -70,9 +71,10 @@ struct ScootList {
     unsigned int* count;
 };
 // Compacts the indices i < n with mask[i] != 0 into out->list (count on the
-// device); where mask[i] == 0, fill[i] = fill_bits if fill is not NULL.
+// device); where mask[i] == 0, fill[r * fill_ld + i] = fill_bits for the
+// fill_rows rows of fill, if fill is not NULL.
 scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint32_t* fill, uint32_t fill_bits,
-                           cudaStream_t st, ScootList* out);
+                           cudaStream_t st, ScootList* out, int fill_rows = 1, int64_t fill_ld = 0);
 
 // Posterior of the listed candidates into list-position order: mean and var
 // [M][ldc], and the whitened rows V = L^{-1} k(X, x) [M][n_rb * 64][ldc]

@@ -29,7 +29,7 @@ constexpr int kMaxD = SCOOT_MAX_DIM;
 constexpr int kMaxM = SCOOT_MAX_OBJ;
 constexpr int kAcqThreads = 128;
 
-enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3 };
+enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3, kMACE = 4 };
 
 struct ScoreArgs {
     const char* state;
@@ -42,7 +42,9 @@ struct ScoreArgs {
     float* var;
     int64_t ldo;
     float* acq;
+    int64_t lda;                  // kMACE: rows UCB, PI, EI of acq, lda apart
     float xi;
+    float kappa;                  // kMACE: UCB coefficient
     const float* box_lo;
     const float* box_hi;
     int32_t n_boxes;
@@ -216,7 +218,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     const int tid = threadIdx.x;
     const int slot = tid & (kTC - 1), half = tid >> 6;
     const int warp = tid >> 5;
-    const int nobj = EPI == kEHVI ? M : (EPI == kEI ? 1 : a.n_obj);
+    const int nobj = EPI == kEHVI ? M : ((EPI == kEI || EPI == kMACE) ? 1 : a.n_obj);
     const int64_t n_pad64 = n_pad;
     const float4* gfmap = reinterpret_cast<const float4*>(a.state + a.off_fmap);
     const float* gxs = reinterpret_cast<const float*>(a.state + a.off_xs);
@@ -390,6 +392,12 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 }
         } else if (EPI == kEI) {
             if (live && half == 0) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
+        } else if (EPI == kMACE) {
+            if (live && half == 0) {
+                a.acq[i] = ucb_value(mu[0], vr[0], a.kappa);
+                a.acq[a.lda + i] = pi_value(mu[0], vr[0], gscal[2], a.xi);
+                a.acq[2 * a.lda + i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
+            }
         } else {
             float sd[kMaxM];
 #pragma unroll
@@ -401,6 +409,18 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             __syncthreads();
             if (live && half == 0) a.acq[i] = (part[slot] + part[kTC + slot]) * (1.0f / (float)a.n_mc);
         }
+    }
+}
+
+__global__ void __launch_bounds__(kAcqThreads)
+mace_kernel(const float* __restrict__ mean, const float* __restrict__ var, const uint8_t* __restrict__ mask,
+            int64_t n, float ybest, float xi, float kappa, float* __restrict__ acq, int64_t lda) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const bool live = mask == nullptr || mask[i] != 0;
+        const float mu = live ? mean[i] : 0.0f, vr = live ? var[i] : 0.0f;
+        acq[i] = live ? ucb_value(mu, vr, kappa) : -INFINITY;
+        acq[lda + i] = live ? pi_value(mu, vr, ybest, xi) : -INFINITY;
+        acq[2 * lda + i] = live ? ei_value(mu, vr, ybest, xi) : -INFINITY;
     }
 }
 
@@ -498,7 +518,7 @@ scoot_status launch_score(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
         // others is -inf (their moments are left untouched).
         ScootList lst;
         scoot_status s = scoot_compact(ctx, a.mask, a.n, EPI == kWriteMoments ? nullptr : reinterpret_cast<uint32_t*>(a.acq),
-                                       0xFF800000u, st, &lst);
+                                       0xFF800000u, st, &lst, EPI == kMACE ? 3 : 1, a.lda);
         if (s != SCOOT_OK) return s;
         a.list = lst.list;
         a.n_list = lst.count;
@@ -588,6 +608,23 @@ scoot_status scoot_acq_ei(scoot_ctx* ctx, const float* mean, const float* var, c
     return SCOOT_OK;
 }
 
+scoot_status scoot_acq_mace(scoot_ctx* ctx, const float* mean, const float* var, const uint8_t* mask,
+                            int64_t n, float y_best, float xi, float kappa, float* acq, int64_t lda, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (n < 0) return scoot_fail(ctx, SCOOT_EINVAL, "n < 0");
+    if (n == 0) return SCOOT_OK;
+    if (!mean || !var || !acq) return scoot_fail(ctx, SCOOT_EINVAL, "mean, var or acq is NULL");
+    if (lda < n) return scoot_fail(ctx, SCOOT_EINVAL, "lda = %lld < n", (long long)lda);
+    int64_t blocks = (n + kAcqThreads - 1) / kAcqThreads;
+    const int64_t cap = (int64_t)sm_count(ctx->device) * 16;
+    if (blocks > cap) blocks = cap;
+    mace_kernel<<<(unsigned)blocks, kAcqThreads, 0, static_cast<cudaStream_t>(stream)>>>(mean, var, mask, n, y_best,
+                                                                                          xi, kappa, acq, lda);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
 scoot_status scoot_acq_ehvi(scoot_ctx* ctx, const float* mean, const float* var, int64_t ldm, int32_t n_obj,
                             const uint8_t* mask, int64_t n, const float* box_lo, const float* box_hi,
                             int32_t n_boxes, const float* eps, int32_t n_mc, float* acq, void* stream) {
@@ -655,6 +692,28 @@ scoot_status scoot_score_ei(scoot_ctx* ctx, const scoot_gp_layout* L, const void
     a.acq = acq;
     a.xi = xi;
     return launch_score<kEI, 1>(ctx, a, static_cast<cudaStream_t>(stream));
+}
+
+scoot_status scoot_score_mace(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                              const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                              float xi, float kappa, float* acq, int64_t lda, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    ScoreArgs a;
+    if ((s = fill_state_args(ctx, L, state, a)) != SCOOT_OK) return s;
+    if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!acq) return scoot_fail(ctx, SCOOT_EINVAL, "acq is NULL");
+    if (lda < n) return scoot_fail(ctx, SCOOT_EINVAL, "lda = %lld < n", (long long)lda);
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.mask = mask;
+    a.acq = acq;
+    a.lda = lda;
+    a.xi = xi;
+    a.kappa = kappa;
+    return launch_score<kMACE, 1>(ctx, a, static_cast<cudaStream_t>(stream));
 }
 
 scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,

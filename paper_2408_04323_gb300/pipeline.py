@@ -1,5 +1,7 @@
 """One suggestion round through the C ABI: prune -> forest -> posterior +
-acquisition -> top-q (Section 4, Algorithm 1's SUGGEST step).
+acquisition -> top-q (Section 4, Algorithm 1's SUGGEST step), or, for one
+objective with MACE, posterior + (UCB, PI, EI) -> random k-subset of their
+Pareto front (Sections 4.5 and 4.7).
 
 Host-side state (GP factor, box decomposition, packed forest) is prepared by
 the library's own host functions; torch only holds device memory and
@@ -7,6 +9,7 @@ streams.  Nothing here computes any step of the path itself.
 """
 from __future__ import annotations
 
+import math
 from dataclasses import dataclass
 
 import numpy as np
@@ -32,11 +35,22 @@ class RoundInputs:
     noise_var: np.ndarray      # float32[M]
     ref: np.ndarray            # float32[M]
     eps: np.ndarray            # float32[S][M]
-    acq: str                   # "ei" or "ehvi"
+    acq: str                   # "ei", "ehvi" or "mace"
     q: int
     kernel: int = S.MATERN52
     xi: float = 1e-4
     fantasy: bool = False      # q sequential picks with kriging-believer fantasies
+    kappa: float | None = None  # MACE: UCB coefficient (None: mace_beta(n_obs))
+    seed: int = 0               # MACE: seed of the random draw from the front
+
+
+def mace_beta(t: int) -> float:
+    """UCB coefficient for tuning iteration t (Section 4.5):
+    beta_t = 2 log(t^2 pi^2 / (6 delta)) with delta = 1 / t^2, taken as the
+    factor of sigma in UCB = mu + beta sigma as printed."""
+    t = max(int(t), 1)
+    delta = 1.0 / (t * t)
+    return 2.0 * math.log(t * t * math.pi ** 2 / (6.0 * delta))
 
 
 class State:
@@ -88,6 +102,16 @@ class ScoringRound:
             nbytes = S.scoot_fantasy_work_bytes(self.state.gp_layout, self.capacity, q)
             self.work = torch.empty(nbytes, dtype=torch.uint8, device=dev)
         self.picks = None
+        self.acq3 = self.front = None
+        if inp.acq == "mace":
+            if inp.y_obs.shape[0] != 1:
+                raise ValueError("MACE scores one objective")
+            self.acq3 = torch.empty((3, self.capacity), dtype=torch.float32, device=dev)
+            self.front_cap = 4096
+            self.front = torch.empty(self.front_cap, dtype=torch.int64, device=dev)
+            self.top_count = torch.empty(2, dtype=torch.int32, device=dev)
+            self.kappa = float(mace_beta(inp.y_obs.shape[1]) if inp.kappa is None else inp.kappa)
+            self.seed = int(inp.seed)
 
     # number of library kernels one call of run() launches (plain top-q rounds)
     KERNELS_PER_ROUND = 7
@@ -97,12 +121,18 @@ class ScoringRound:
         either compaction + fused score + two top-q passes, or (fantasies)
         compaction + posterior + per pick EHVI, two argmax passes and a downdate
         (the last pick skips the downdate)."""
+        if self.inp.acq == "mace":
+            return 10  # prune, compaction, forest, compaction, score, five Pareto kernels
         if not self.inp.fantasy:
             return 7
         return 3 + 2 + 4 * self.inp.q - 1
 
     def run(self, cand: torch.Tensor, n: int, stream=None):
-        """prune -> rf -> score -> top-q on a resident pool cand (int32 [d][ld])."""
+        """prune -> rf -> score -> top-q on a resident pool cand (int32 [d][ld]).
+
+        Returns (idx, val, count).  With MACE, idx holds the random picks from
+        the front, count is (picks, front size), val is not written and the
+        front itself is in self.front (first front_cap members)."""
         if n > self.capacity:
             raise ValueError("pool larger than the round's capacity")
         inp, st = self.inp, self.state
@@ -118,6 +148,12 @@ class ScoringRound:
             self.top_idx[:k].copy_(torch.from_numpy(idx))
             self.top_val[:k].copy_(torch.from_numpy(val))
             self.top_count.fill_(k)
+            return self.top_idx, self.top_val, self.top_count
+        if inp.acq == "mace":
+            S.scoot_score_mace(self.ctx, st.gp_layout, st.gp_state, cand, n, inp.xi, self.kappa, self.acq3,
+                               self.mask, stream)
+            S.scoot_select_pareto(self.ctx, self.acq3, n, inp.q, self.seed, self.top_idx, self.top_count,
+                                  self.mask, self.front, stream)
             return self.top_idx, self.top_val, self.top_count
         if inp.acq == "ei":
             S.scoot_score_ei(self.ctx, st.gp_layout, st.gp_state, cand, n, inp.xi, self.acq, self.mask, stream)

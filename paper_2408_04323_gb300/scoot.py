@@ -85,6 +85,9 @@ _PROTOS = {
     "scoot_score_ehvi": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i32,
                          _vp, _i32, _vp, _vp],
     "scoot_select_topq": [_vp, _vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
+    "scoot_acq_mace": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _f32, _vp, _i64, _vp],
+    "scoot_score_mace": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _f32, _f32, _vp, _i64, _vp],
+    "scoot_select_pareto": [_vp, _vp, _i64, _vp, _i64, _i32, C.c_uint64, _vp, _vp, _vp, _i64, _vp],
     "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
     "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, C.POINTER(_i64)],
     "scoot_suggest_fantasy": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _vp, _i64, _vp, _vp, _vp, _vp,
@@ -336,6 +339,36 @@ def scoot_select_topq(ctx, acq, n, q, idx, val, count, mask=None, stream=None):
     _check(lib().scoot_select_topq(_h(ctx), _dev(acq, torch.float32, "acq"), _dev(mask, torch.uint8, "mask"),
                                    int(n), int(q), _dev(idx, torch.int64, "idx"), _dev(val, torch.float32, "val"),
                                    _dev(count, torch.int32, "count"), _stream(stream)), "scoot_select_topq", _h(ctx))
+
+
+def scoot_acq_mace(ctx, mean, var, n, y_best, xi, kappa, acq, mask=None, stream=None):
+    """acq: float32 [3][lda] (rows UCB, PI, EI)."""
+    import torch
+    _check(lib().scoot_acq_mace(_h(ctx), _dev(mean, torch.float32, "mean"), _dev(var, torch.float32, "var"),
+                                _dev(mask, torch.uint8, "mask"), int(n), float(y_best), float(xi), float(kappa),
+                                _dev(acq, torch.float32, "acq"), int(acq.shape[-1]), _stream(stream)),
+           "scoot_acq_mace", _h(ctx))
+
+
+def scoot_score_mace(ctx, layout, state, cand, n, xi, kappa, acq, mask=None, stream=None):
+    """acq: float32 [3][lda] (rows UCB, PI, EI)."""
+    import torch
+    _check(lib().scoot_score_mace(_h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"),
+                                  _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]),
+                                  _dev(mask, torch.uint8, "mask"), float(xi), float(kappa),
+                                  _dev(acq, torch.float32, "acq"), int(acq.shape[-1]), _stream(stream)),
+           "scoot_score_mace", _h(ctx))
+
+
+def scoot_select_pareto(ctx, acq, n, k, seed, idx, count, mask=None, front=None, stream=None):
+    """idx: int64 [k]; count: int32 [2] (picks, front size); front: optional int64 [cap]."""
+    import torch
+    _check(lib().scoot_select_pareto(_h(ctx), _dev(acq, torch.float32, "acq"), int(acq.shape[-1]),
+                                     _dev(mask, torch.uint8, "mask"), int(n), int(k),
+                                     C.c_uint64(int(seed) & 0xFFFFFFFFFFFFFFFF), _dev(idx, torch.int64, "idx"),
+                                     _dev(count, torch.int32, "count"), _dev(front, torch.int64, "front"),
+                                     int(front.shape[0]) if front is not None else 0, _stream(stream)),
+           "scoot_select_pareto", _h(ctx))
 
 
 def scoot_select_topq_static(acq, n, q, idx, val, count, mask=None, stream=None):
