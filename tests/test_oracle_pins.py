@@ -449,9 +449,45 @@ def test_mc_ehvi_converges_to_analytic(M):
     est = vals.mean()
     se = vals.std() / math.sqrt(S)
     assert abs(est - _ehvi_analytic(mu, sd, lo, hi)) < 4 * se
-    # the oracle's MC EHVI is that mean
+    # the oracle's MC EHVI is that mean, and its exact EHVI is the test's own closed form
     e = O.ehvi_mc(mu[None, :], (sd ** 2)[None, :], eps, front, ref)[0]
     assert e == pytest.approx(est, rel=1e-12)
+    x = O.ehvi_analytic(mu[None, :], (sd ** 2)[None, :], front, ref)[0]
+    assert x == pytest.approx(_ehvi_analytic(mu, sd, lo, hi), rel=1e-10)
+    assert abs(est - x) < 4 * se
+
+
+def test_exact_ehvi_limits_and_quadrature():
+    """sigma -> 0 gives the deterministic HVI(mu); for M = 2 the exact EHVI
+    equals 2-D quadrature of HVI(y) against the product density."""
+    st = Stream(71, "ehvi-exact")
+    ref = np.zeros(2)
+    front = O.pareto_front(st.uniform(12).reshape(6, 2) * 2.0, ref)
+    lo, hi = O.nondominated_cells(front, ref)
+    for mu in ([1.1, 0.7], [2.5, 0.1], [-0.3, 1.9]):
+        mu = np.array(mu)
+        got = O.ehvi_analytic(mu[None, :], np.zeros((1, 2)), front, ref)[0]
+        assert got == pytest.approx(O.hvi_cells(mu, lo, hi)[0], rel=1e-12, abs=1e-14)
+    mu, sd = np.array([1.0, 0.8]), np.array([0.4, 0.25])
+    dens = lambda y, m, s: math.exp(-0.5 * ((y - m) / s) ** 2) / (s * math.sqrt(2 * math.pi))
+    # HVI is piecewise bilinear with kinks on the grid lines: nested quad with those breakpoints
+    kinks = [np.unique(np.concatenate([[0.0], front[:, j]])) for j in range(2)]
+    box = [(mu[j] - 9 * sd[j], mu[j] + 9 * sd[j]) for j in range(2)]
+
+    def inner(y1):
+        g = lambda y0: O.hvi_cells(np.array([y0, y1]), lo, hi)[0] * dens(y0, mu[0], sd[0])
+        pts = [k for k in kinks[0] if box[0][0] < k < box[0][1]]
+        return integrate.quad(g, *box[0], points=pts, epsabs=1e-12, epsrel=1e-10, limit=200)[0]
+
+    pts = [k for k in kinks[1] if box[1][0] < k < box[1][1]]
+    q, _ = integrate.quad(lambda y1: inner(y1) * dens(y1, mu[1], sd[1]), *box[1], points=pts,
+                          epsabs=1e-11, epsrel=1e-9, limit=200)
+    got = O.ehvi_analytic(mu[None, :], (sd ** 2)[None, :], front, ref)[0]
+    assert got == pytest.approx(q, rel=1e-6, abs=1e-9)
+    # psi(a) = E[max(0, Y - a)] against quadrature
+    for m, s_, a in [(0.3, 0.7, 0.1), (-1.0, 0.2, 0.5), (2.0, 1.5, -1.0)]:
+        qq, _ = integrate.quad(lambda y: max(0.0, y - a) * dens(y, m, s_), a, m + 14 * s_, epsabs=1e-13, limit=200)
+        assert float(O.expected_excess(m, s_, a)) == pytest.approx(qq, rel=1e-9, abs=1e-13)
 
 
 # ------------------------------------------------------------------ top-q, Section 4.7
