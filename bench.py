@@ -61,8 +61,9 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    p.add_argument("--acq", choices=["default", "mace"], default="default",
-                   help="mace: UCB/PI/EI and a random subset of their Pareto front (one objective)")
+    p.add_argument("--acq", choices=["default", "mace", "ehvi-exact"], default="default",
+                   help="mace: UCB/PI/EI and a random subset of their Pareto front (one objective); "
+                        "ehvi-exact: EHVI as the exact expectation (several objectives)")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the cpu_baseline sample")
     p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -100,15 +101,19 @@ def referenced_columns(inst):
     return len(cols)
 
 
-def work_model(inst, n_boxes, acq_kind=None):
+def work_model(inst, n_boxes, acq_kind=None, n_grid=None):
     """Algorithmic work per candidate of each stage (bytes or flops)."""
     w = inst.workload
     acq_kind = acq_kind or w.acq
     d, n = inst.d, inst.n_obs
-    m_eff = inst.n_obj if acq_kind == "ehvi" else 1
+    m_eff = inst.n_obj if acq_kind in ("ehvi", "ehvi-exact") else 1
     post = m_eff * (n * (3 * d + 12) + 2 * n + n * (n + 1) + 2 * n)
-    # EI ~30 flops; MACE adds PI (~15) and UCB (2)
-    acq = {"ei": 30, "mace": 47}.get(acq_kind, w.n_mc * n_boxes * 4 * inst.n_obj)
+    # EI ~30 flops; MACE adds PI (~15) and UCB (2); exact EHVI: ~12 flops per psi at each grid
+    # coordinate and 2M per box
+    if acq_kind == "ehvi-exact":
+        acq = 12 * int(sum(n_grid)) + 2 * inst.n_obj * n_boxes
+    else:
+        acq = {"ei": 30, "mace": 47}.get(acq_kind, w.n_mc * n_boxes * 4 * inst.n_obj)
     return {
         "prune": ("hbm", 4 * referenced_columns(inst) + 1),
         "rf": ("hbm", 4 * d + 1 + 1 + 4),
@@ -167,13 +172,14 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(loaded)}
 
 
-def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None):
+def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None):
     """Time the oracle on n_sample candidates of the workload in a fresh process
-    (with mace_kappa set: the MACE round, UCB coefficient mace_kappa)."""
+    (with mace_kappa set: the MACE round, UCB coefficient mace_kappa; acq
+    overrides the workload's acquisition)."""
     env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
                MKL_NUM_THREADS=str(threads))
     if mace_kappa is None:
-        select = ("r = oracle.score_round(inst, inst.workload.acq)\n"
+        select = ("r = oracle.score_round(inst, %s)\n" % (repr(acq) if acq else "inst.workload.acq") +
                   "oracle.select_topq(r['acq'], r['feasible'], inst.workload.q)\n")
     else:
         select = ("r = oracle.score_round(inst, 'ei')\n"
@@ -195,10 +201,10 @@ def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None):
     return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
 
 
-def calibrate_sample(name, seed, budget_s, mace_kappa=None):
+def calibrate_sample(name, seed, budget_s, mace_kappa=None, acq=None):
     """Largest sample whose oracle round fits the budget (scaled from a probe)."""
     probe = 64
-    t = cpu_oracle_sample(name, seed, probe, mace_kappa=mace_kappa)
+    t = cpu_oracle_sample(name, seed, probe, mace_kappa=mace_kappa, acq=acq)
     per = max(t / probe, 1e-6)
     return max(16, int(budget_s / per))
 
@@ -214,11 +220,12 @@ def run_reference(args):
     if args.acq == "mace":
         from paper_2408_04323_gb300.pipeline import mace_beta
         kappa = mace_beta(w.n_obs)
+    acq = "ehvi-exact" if args.acq == "ehvi-exact" else None
     per_step = max(0.05, 120.0 / max(1, args.steps + args.warmup))
-    sample = calibrate_sample(w.name, seed, per_step, kappa)
+    sample = calibrate_sample(w.name, seed, per_step, kappa, acq)
     for _ in range(args.warmup):
-        cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa)
-    times = [cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa) for _ in range(args.steps)]
+        cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq)
+    times = [cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq) for _ in range(args.steps)]
     ms = 1e3 * statistics.mean(times)
     value = sample / (ms / 1e3)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -263,6 +270,8 @@ def main():
     acq_kind = w.acq if args.acq == "default" else args.acq
     if acq_kind == "mace" and (w.n_obj != 1 or w.fantasy):
         raise SystemExit("--acq mace needs a one-objective workload")
+    if acq_kind == "ehvi-exact" and (w.n_obj < 2 or w.fantasy):
+        raise SystemExit("--acq ehvi-exact needs a multi-objective workload without fantasies")
     if acq_kind == "mace" and world > 1:
         raise SystemExit("--acq mace runs on one GPU: its front is not merged across ranks")
     seed = seeds(w.name)[0]
@@ -305,6 +314,9 @@ def main():
         elif inp.acq == "mace":
             S.scoot_score_mace(ctx, st.gp_layout, st.gp_state, cand, N, inp.xi, rnd.kappa, rnd.acq3, rnd.mask,
                                stream)
+        elif inp.acq == "ehvi-exact":
+            S.scoot_score_ehvi_exact(ctx, st.gp_layout, st.gp_state, cand, N, st.grid, st.n_grid, st.corner,
+                                     rnd.acq, rnd.mask, stream)
         else:
             S.scoot_score_ehvi(ctx, st.gp_layout, st.gp_state, cand, N, st.box_lo, st.box_hi, st.eps,
                                rnd.acq, rnd.mask, stream)
@@ -397,7 +409,7 @@ def main():
     peaks, peak_src = measured_peaks()
     sms = torch.cuda.get_device_properties(device).multi_processor_count
     fp32_peak = sms * FP32_LANES_PER_SM * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # TFLOP/s
-    work = work_model(inst, st.n_boxes, inp.acq)
+    work = work_model(inst, st.n_boxes, inp.acq, getattr(st, "n_grid", None))
     dom = max(stage_names, key=lambda s: stage_ms[s])
     kind, per_cand = work[dom]
     units = n_feasible if dom == "score" else N
@@ -452,6 +464,9 @@ def main():
                                    rnd.mask, stream)
                 S.scoot_select_pareto(ctx, rnd.acq3, N, inp.q, rnd.seed, rnd.top_idx, rnd.top_count, rnd.mask,
                                       rnd.front, stream)
+            elif inp.acq == "ehvi-exact":
+                S.scoot_score_ehvi_exact(ctx, state.gp_layout, state.gp_state, cand_e2e, N, state.grid, state.n_grid,
+                                         state.corner, rnd.acq, rnd.mask, stream)
             else:
                 S.scoot_score_ehvi(ctx, state.gp_layout, state.gp_state, cand_e2e, N, state.box_lo, state.box_hi,
                                    state.eps, rnd.acq, rnd.mask, stream)
@@ -465,7 +480,7 @@ def main():
             if kk >= args.warmup:
                 times.append(time.perf_counter() - t0)
         state_bytes = sum(b.nbytes for b in state.h_blobs)
-        if inp.acq == "ehvi":
+        if inp.acq in ("ehvi", "ehvi-exact"):
             state_bytes += sum(b.nbytes for b in state.h_boxes) + inp.eps.nbytes
         e2e_s = statistics.mean(times)
         if dist:
@@ -479,8 +494,9 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         kappa = rnd.kappa if inp.acq == "mace" else None
-        sample = calibrate_sample(w.name, seed, args.cpu_seconds, kappa)
-        secs = cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa)
+        acq = "ehvi-exact" if inp.acq == "ehvi-exact" else None
+        sample = calibrate_sample(w.name, seed, args.cpu_seconds, kappa, acq)
+        secs = cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq)
         cpu = {"value": sample / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"{sample} candidates of the {w.name} pool (same round state), all five steps, "
                          f"fp64 numpy, one thread"}

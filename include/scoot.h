@@ -11,6 +11,7 @@
  *   scoot_acq_ehvi       Monte-Carlo expected hypervolume improvement, Eq. (7)
  *   scoot_score_ei       posterior + EI in one kernel
  *   scoot_score_ehvi     posterior + EHVI in one kernel
+ *   scoot_score_ehvi_exact  posterior + exact EHVI (independent Gaussians)
  *   scoot_select_topq    top-q for parallel suggestion (Section 4.7)
  *   scoot_score_mace     posterior + UCB, PI, EI for MACE (Section 4.5)
  *   scoot_select_pareto  random k-subset of the (UCB, PI, EI) front (Section 4.7)
@@ -260,6 +261,18 @@ scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, c
                                int32_t cap, float* h_lo, float* h_hi, int32_t* n_boxes,
                                int32_t* front_size);
 
+/* Corner indices of boxes for the exact EHVI (scoot_acq_ehvi_exact,
+ * scoot_score_ehvi_exact).  h_lo, h_hi: n_boxes boxes [B][M] as written by
+ * scoot_boxes_build.  For each objective j, h_grid[j * grid_cap + g]
+ * (g < h_n_grid[j]) receives the distinct finite box coordinates on that axis
+ * in increasing order, and h_corner[b * M + j] = lo | hi << 16, the indices of
+ * box b's lower and upper coordinates in that list (h_n_grid[j] standing for
+ * +inf).  Host only.  SCOOT_EINVAL for a NaN, an infinite lower corner or
+ * hi <= lo; SCOOT_EUNSUPPORTED if an axis has more than grid_cap (or 65535)
+ * coordinates (h_n_grid then holds the counts found so far). */
+scoot_status scoot_boxes_index(const float* h_lo, const float* h_hi, int32_t n_boxes, int32_t n_obj,
+                               int32_t grid_cap, float* h_grid, int32_t* h_n_grid, uint32_t* h_corner);
+
 /* Monte-Carlo EHVI, Eq. (7): with base samples eps [S][M] shared by every
  * candidate, y_s = mu + sigma * eps_s and
  * EHVI = (1/S) sum_s sum_b prod_j max(0, min(y_sj, hi_bj) - lo_bj)
@@ -282,6 +295,30 @@ scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* layout, con
                               const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
                               const float* box_lo, const float* box_hi, int32_t n_boxes,
                               const float* eps, int32_t n_mc, float* acq, void* stream);
+
+/* EHVI (Eq. 7) as the exact expectation over independent Gaussian
+ * objectives Y_j ~ N(mu_j, sigma_j^2), the closed form behind the paper's
+ * EHVI reference (Yang et al.):
+ *   EHVI = sum_b prod_j [psi_j(lo_bj) - psi_j(hi_bj)],
+ *   psi_j(a) = E[max(0, Y_j - a)] = sigma_j phi(z) + (mu_j - a) Phi(z),
+ *   z = (mu_j - a) / sigma_j  (max(0, mu_j - a) when sigma_j = 0; 0 at +inf),
+ * over boxes given as scoot_boxes_index writes them: grid (device
+ * [M][grid_cap]), h_n_grid (host [M]), corner (device [B][M]).  psi is
+ * evaluated once per grid coordinate and candidate.  mean/var as written by
+ * scoot_gp_posterior ([M][ldm]); acq[i] = -inf where mask[i] == 0.
+ * SCOOT_EUNSUPPORTED when sum_j (h_n_grid[j] + 1) > 320.  A corner index
+ * beyond h_n_grid is clamped and flagged (SCOOT_EDEVICE from
+ * scoot_ctx_check). */
+scoot_status scoot_acq_ehvi_exact(scoot_ctx* ctx, const float* mean, const float* var, int64_t ldm,
+                                  int32_t n_obj, const uint8_t* mask, int64_t n, const float* grid,
+                                  int32_t grid_cap, const int32_t* h_n_grid, const uint32_t* corner,
+                                  int32_t n_boxes, float* acq, void* stream);
+
+/* scoot_gp_posterior followed by scoot_acq_ehvi_exact, in one kernel. */
+scoot_status scoot_score_ehvi_exact(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                                    const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                                    const float* grid, int32_t grid_cap, const int32_t* h_n_grid,
+                                    const uint32_t* corner, int32_t n_boxes, float* acq, void* stream);
 
 /* ------------------------------------------------------------------ 5. top-q (Section 4.7) */
 

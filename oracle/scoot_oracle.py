@@ -472,6 +472,8 @@ def score_round(inst, acq_kind: str, xi: float = 1e-4, kernel: int = MATERN52,
     var = np.stack([v for _, v in mv], axis=1)
     if acq_kind == "ei":
         a = expected_improvement(mu[:, 0], var[:, 0], float(np.max(inst.y_obs[0])), xi)
+    elif acq_kind == "ehvi-exact":
+        a = ehvi_analytic(mu, var, pareto_front(inst.y_obs.T, inst.ref), inst.ref)
     else:
         front = pareto_front(inst.y_obs.T, inst.ref)
         a = ehvi_mc(mu, var, inst.eps, front, inst.ref)

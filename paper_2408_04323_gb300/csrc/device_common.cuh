@@ -33,6 +33,39 @@ __device__ __forceinline__ float pi_value(float mu, float var, float ybest, floa
     return 0.5f * erfcf(-(a / s) * 0.70710678118654752f);
 }
 
+// psi(a) = E[max(0, Y - a)] for Y ~ N(mu, sd^2), a finite:
+// sd phi(z) + (mu - a) Phi(z) with z = (mu - a) / sd; max(0, mu - a) at sd = 0.
+__device__ __forceinline__ float expected_excess(float mu, float sd, float a) {
+    const float d = mu - a;
+    if (!(sd > 0.0f)) return fmaxf(d, 0.0f);
+    const float z = d / sd;
+    const float cdf = 0.5f * erfcf(-z * 0.70710678118654752f);
+    const float pdf = 0.39894228040143268f * expf(-0.5f * z * z);
+    return fmaf(sd, pdf, d * cdf);
+}
+
+// Staging of the exact-EHVI boxes: the per-axis grids (axis j at
+// grid_s[goff_j ..]) and the boxes' corner indices, validated against the
+// grid sizes (an index beyond n_grid[j] is clamped and flagged).
+__device__ __forceinline__ void stage_box_grid(const float* grid, int grid_cap, const int* n_grid, const uint32_t* corner,
+                                               int n_boxes, int M, float* grid_s, uint32_t* corner_s, uint32_t* err) {
+    int goff = 0;
+    for (int j = 0; j < M; ++j) {
+        for (int g = threadIdx.x; g < n_grid[j]; g += blockDim.x) grid_s[goff + g] = grid[j * grid_cap + g];
+        goff += n_grid[j];
+    }
+    for (int e = threadIdx.x; e < n_boxes * M; e += blockDim.x) {
+        const int j = e % M;
+        uint32_t c = corner[e];
+        const uint32_t lo = c & 0xFFFFu, hi = c >> 16, G = (uint32_t)n_grid[j];
+        if (lo > G || hi > G) {
+            atomicOr(err, 1u);  // SCOOT_DEVERR_INDEX
+            c = (lo > G ? G : lo) | ((hi > G ? G : hi) << 16);
+        }
+        corner_s[e] = c;
+    }
+}
+
 // UCB = mu + kappa * sigma.
 __device__ __forceinline__ float ucb_value(float mu, float var, float kappa) {
     return fmaf(kappa, sqrtf(fmaxf(var, 0.0f)), mu);

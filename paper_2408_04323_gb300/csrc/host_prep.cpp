@@ -475,6 +475,36 @@ scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, c
     return SCOOT_OK;
 }
 
+scoot_status scoot_boxes_index(const float* h_lo, const float* h_hi, int32_t n_boxes, int32_t n_obj,
+                               int32_t grid_cap, float* h_grid, int32_t* h_n_grid, uint32_t* h_corner) {
+    if (n_boxes < 0 || grid_cap < 0 || !h_n_grid) return SCOOT_EINVAL;
+    if (n_obj < 2 || n_obj > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
+    if (n_boxes > 0 && (!h_lo || !h_hi || !h_corner)) return SCOOT_EINVAL;
+    const int M = n_obj;
+    for (int j = 0; j < M; ++j) {
+        std::vector<float> axis;
+        for (int b = 0; b < n_boxes; ++b) {
+            const float lo = h_lo[(size_t)b * M + j], hi = h_hi[(size_t)b * M + j];
+            if (!std::isfinite(lo) || std::isnan(hi) || !(hi > lo)) return SCOOT_EINVAL;
+            axis.push_back(lo);
+            if (std::isfinite(hi)) axis.push_back(hi);
+        }
+        std::sort(axis.begin(), axis.end());
+        axis.erase(std::unique(axis.begin(), axis.end()), axis.end());
+        h_n_grid[j] = (int32_t)axis.size();
+        if ((int64_t)axis.size() > grid_cap || axis.size() > 65535) return SCOOT_EUNSUPPORTED;
+        if (!axis.empty() && !h_grid) return SCOOT_EINVAL;
+        std::copy(axis.begin(), axis.end(), h_grid + (size_t)j * grid_cap);
+        auto index = [&](float v) -> uint32_t {
+            if (std::isinf(v)) return (uint32_t)axis.size();
+            return (uint32_t)(std::lower_bound(axis.begin(), axis.end(), v) - axis.begin());
+        };
+        for (int b = 0; b < n_boxes; ++b)
+            h_corner[(size_t)b * M + j] = index(h_lo[(size_t)b * M + j]) | (index(h_hi[(size_t)b * M + j]) << 16);
+    }
+    return SCOOT_OK;
+}
+
 // ---------------------------------------------------------------- forest
 
 scoot_status scoot_forest_layout_init(const scoot_node* h_nodes, const int32_t* h_tree_offset,

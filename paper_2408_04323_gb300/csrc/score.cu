@@ -29,7 +29,7 @@ constexpr int kMaxD = SCOOT_MAX_DIM;
 constexpr int kMaxM = SCOOT_MAX_OBJ;
 constexpr int kAcqThreads = 128;
 
-enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3, kMACE = 4 };
+enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3, kMACE = 4, kEHVIX = 5 };
 
 struct ScoreArgs {
     const char* state;
@@ -50,6 +50,11 @@ struct ScoreArgs {
     int32_t n_boxes;
     const float* eps;
     int32_t n_mc;
+    const float* grid;            // kEHVIX: per-axis box coordinates [M][grid_cap]
+    const uint32_t* corner;       // kEHVIX: box corner indices [B][M]
+    int32_t grid_cap;
+    int32_t n_grid[kMaxM];
+    int32_t psi_rows;             // kEHVIX: sum_j (n_grid[j] + 1), rows of the psi table
     const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
     const unsigned int* n_list;
     float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad][ldv] by list position
@@ -205,8 +210,10 @@ __global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) 
 score_kernel(const __grid_constant__ ScoreArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
+    // Ks, and after the posterior the exact-EHVI psi table [psi_rows][kTC]
+    const int ks_rows = EPI == kEHVIX && a.psi_rows > n_pad ? a.psi_rows : n_pad;
     float* Ks = sm;                                                   // [n_pad][kTC]
-    float* xs = Ks + (size_t)n_pad * kTC;                             // [n_obs][DO] ordinal features
+    float* xs = Ks + (size_t)ks_rows * kTC;                           // [n_obs][DO] ordinal features
     float* al = xs + (size_t)a.n_obs * DO;                            // [n_pad]
     float* Lt = al + n_pad;                                           // [2][kCJ][kRB] double buffer
     float* part = Lt + 2 * kCJ * kRB;                                 // [8][kTC]
@@ -214,11 +221,13 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     float4* blo = fm + kMaxD;                          // [B] (general boxes) or [2B] (saturated form)
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
     float4* epsv = bhi + (EPI == kEHVI ? a.n_boxes : 0);
+    float* grid_s = reinterpret_cast<float*>(fm + kMaxD);             // kEHVIX: [sum n_grid] (padded to 4)
+    uint32_t* corner_s = reinterpret_cast<uint32_t*>(grid_s + ((a.psi_rows + 3) & ~3));  // [B][M]
 
     const int tid = threadIdx.x;
     const int slot = tid & (kTC - 1), half = tid >> 6;
     const int warp = tid >> 5;
-    const int nobj = EPI == kEHVI ? M : ((EPI == kEI || EPI == kMACE) ? 1 : a.n_obj);
+    const int nobj = (EPI == kEHVI || EPI == kEHVIX) ? M : ((EPI == kEI || EPI == kMACE) ? 1 : a.n_obj);
     const int64_t n_pad64 = n_pad;
     const float4* gfmap = reinterpret_cast<const float4*>(a.state + a.off_fmap);
     const float* gxs = reinterpret_cast<const float*>(a.state + a.off_xs);
@@ -229,6 +238,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     const float* gcat = reinterpret_cast<const float*>(a.state + a.off_cat);
 
     if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
+    if (EPI == kEHVIX) stage_box_grid(a.grid, a.grid_cap, a.n_grid, a.corner, a.n_boxes, M, grid_s, corner_s, a.err);
     if (tid < kMaxD) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
     __syncthreads();
     // Boxes open on the last objective (as scoot_boxes_build makes them) are
@@ -392,6 +402,39 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 }
         } else if (EPI == kEI) {
             if (live && half == 0) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
+        } else if (EPI == kEHVIX) {
+            // psi table: row poff_j + g holds psi_j(grid_j[g]) (the row past
+            // the last grid coordinate, +inf, holds 0).  Every thread read its
+            // last Ks value before the barriers that ended the posterior.
+            float sd[kMaxM];
+#pragma unroll
+            for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
+            int goff = 0, poff = 0;
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                for (int g = half; g < a.n_grid[m]; g += 2)
+                    Ks[(poff + g) * kTC + slot] = expected_excess(mu[m], sd[m], grid_s[goff + g]);
+                if (half == 0) Ks[(poff + a.n_grid[m]) * kTC + slot] = 0.0f;
+                goff += a.n_grid[m];
+                poff += a.n_grid[m] + 1;
+            }
+            __syncthreads();
+            float v = 0.0f;
+            for (int b = half; b < a.n_boxes; b += 2) {
+                float p = 1.0f;
+                int po = 0;
+#pragma unroll
+                for (int m = 0; m < M; ++m) {
+                    const uint32_t c = corner_s[b * M + m];
+                    p *= Ks[(po + (int)(c & 0xFFFFu)) * kTC + slot] - Ks[(po + (int)(c >> 16)) * kTC + slot];
+                    po += a.n_grid[m] + 1;
+                }
+                v += p;
+            }
+            __syncthreads();  // part is free again; the psi table is read
+            part[half * kTC + slot] = v;
+            __syncthreads();
+            if (live && half == 0) a.acq[i] = part[slot] + part[kTC + slot];
         } else if (EPI == kMACE) {
             if (live && half == 0) {
                 a.acq[i] = ucb_value(mu[0], vr[0], a.kappa);
@@ -456,10 +499,76 @@ ehvi_kernel(const __grid_constant__ ScoreArgs a) {
     }
 }
 
+// Exact EHVI on given moments: one thread per candidate with its own column
+// of the psi table in shared memory.
+template <int M>
+__global__ void __launch_bounds__(kAcqThreads)
+ehvix_kernel(const __grid_constant__ ScoreArgs a) {
+    extern __shared__ __align__(16) float sm[];
+    float* psi = sm;                                                    // [psi_rows][kAcqThreads]
+    float* grid_s = psi + (size_t)a.psi_rows * kAcqThreads;
+    uint32_t* corner_s = reinterpret_cast<uint32_t*>(grid_s + ((a.psi_rows + 3) & ~3));
+    stage_box_grid(a.grid, a.grid_cap, a.n_grid, a.corner, a.n_boxes, M, grid_s, corner_s, a.err);
+    __syncthreads();
+    const int t = threadIdx.x;
+    const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
+    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + t; pos < n_work; pos += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+        int goff = 0, poff = 0;
+#pragma unroll
+        for (int m = 0; m < M; ++m) {
+            const float mu = a.mean[(int64_t)m * a.ldo + i];
+            const float sd = sqrtf(fmaxf(a.var[(int64_t)m * a.ldo + i], 0.0f));
+            for (int g = 0; g < a.n_grid[m]; ++g)
+                psi[(poff + g) * kAcqThreads + t] = expected_excess(mu, sd, grid_s[goff + g]);
+            psi[(poff + a.n_grid[m]) * kAcqThreads + t] = 0.0f;
+            goff += a.n_grid[m];
+            poff += a.n_grid[m] + 1;
+        }
+        float v = 0.0f;
+        for (int b = 0; b < a.n_boxes; ++b) {
+            float p = 1.0f;
+            int po = 0;
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                const uint32_t c = corner_s[b * M + m];
+                p *= psi[(po + (int)(c & 0xFFFFu)) * kAcqThreads + t] - psi[(po + (int)(c >> 16)) * kAcqThreads + t];
+                po += a.n_grid[m] + 1;
+            }
+            v += p;
+        }
+        a.acq[i] = v;
+    }
+}
+
 int sm_count(int device) {
     int v = 0;
     cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, device);
     return v > 0 ? v : 1;
+}
+
+// Arguments of the exact-EHVI calls: the box grid and the psi-table height.
+scoot_status fill_box_grid(scoot_ctx* ctx, int M, const float* grid, int32_t grid_cap, const int32_t* h_n_grid,
+                           const uint32_t* corner, int32_t n_boxes, ScoreArgs& a) {
+    if (M < 2 || M > kMaxM) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "EHVI needs 2 <= M <= %d objectives, got %d", kMaxM, M);
+    if (n_boxes < 1 || !corner || !h_n_grid || !grid)
+        return scoot_fail(ctx, SCOOT_EINVAL, "boxes: B = %d, grid / n_grid / corner must be non-NULL", n_boxes);
+    int rows = 0;
+    for (int j = 0; j < M; ++j) {
+        if (h_n_grid[j] < 0 || h_n_grid[j] > grid_cap || h_n_grid[j] > 65535)
+            return scoot_fail(ctx, SCOOT_EINVAL, "n_grid[%d] = %d outside 0..min(grid_cap, 65535)", j, h_n_grid[j]);
+        a.n_grid[j] = h_n_grid[j];
+        rows += h_n_grid[j] + 1;
+    }
+    if (rows > 320) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "%d grid rows exceed the psi table (320)", rows);
+    if ((size_t)n_boxes * M * 4 > 64 * 1024)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "%d boxes exceed the shared-memory budget", n_boxes);
+    a.grid = grid;
+    a.grid_cap = grid_cap;
+    a.corner = corner;
+    a.n_boxes = n_boxes;
+    a.psi_rows = rows;
+    return SCOOT_OK;
 }
 
 scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state, ScoreArgs& a) {
@@ -490,8 +599,10 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
 
 size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
-    size_t f = n_pad * kTC + (size_t)a.n_obs * DO + n_pad + 2 * kCJ * kRB + 8 * kTC + 4 * kMaxD;
+    const size_t ks_rows = epi == kEHVIX && (size_t)a.psi_rows > n_pad ? (size_t)a.psi_rows : n_pad;
+    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + 2 * kCJ * kRB + 8 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
+    if (epi == kEHVIX) f += (size_t)((a.psi_rows + 3) & ~3) + (size_t)a.n_boxes * kMaxM;
     return f * 4;
 }
 
@@ -673,6 +784,73 @@ scoot_status scoot_acq_ehvi(scoot_ctx* ctx, const float* mean, const float* var,
     case 3: return go(ehvi_kernel<3>);
     default: return go(ehvi_kernel<4>);
     }
+}
+
+scoot_status scoot_acq_ehvi_exact(scoot_ctx* ctx, const float* mean, const float* var, int64_t ldm, int32_t n_obj,
+                                  const uint8_t* mask, int64_t n, const float* grid, int32_t grid_cap,
+                                  const int32_t* h_n_grid, const uint32_t* corner, int32_t n_boxes, float* acq,
+                                  void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (n < 0) return scoot_fail(ctx, SCOOT_EINVAL, "n < 0");
+    ScoreArgs a;
+    std::memset(&a, 0, sizeof(a));
+    if ((s = fill_box_grid(ctx, n_obj, grid, grid_cap, h_n_grid, corner, n_boxes, a)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!mean || !var || !acq || ldm < n) return scoot_fail(ctx, SCOOT_EINVAL, "mean/var/acq NULL or ldm < n");
+    a.mean = const_cast<float*>(mean);
+    a.var = const_cast<float*>(var);
+    a.ldo = ldm;
+    a.mask = mask;
+    a.n = n;
+    a.acq = acq;
+    a.err = ctx->d_err;
+    const size_t smem = ((size_t)a.psi_rows * kAcqThreads + ((a.psi_rows + 3) & ~3) + (size_t)n_boxes * n_obj) * 4;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (mask) {
+        ScootList lst;
+        if ((s = scoot_compact(ctx, mask, n, reinterpret_cast<uint32_t*>(acq), 0xFF800000u, st, &lst)) != SCOOT_OK)
+            return s;
+        a.list = lst.list;
+        a.n_list = lst.count;
+    }
+    int64_t blocks = (n + kAcqThreads - 1) / kAcqThreads;
+    auto go = [&](auto kern) -> scoot_status {
+        SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        int per_sm = 0;
+        SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kAcqThreads, smem));
+        if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "exact EHVI kernel does not fit");
+        const int64_t cap = (int64_t)sm_count(ctx->device) * per_sm;
+        if (blocks > cap) blocks = cap;
+        kern<<<(unsigned)blocks, kAcqThreads, smem, st>>>(a);
+        SCOOT_LAUNCHED(ctx);
+        return SCOOT_OK;
+    };
+    switch (n_obj) {
+    case 2: return go(ehvix_kernel<2>);
+    case 3: return go(ehvix_kernel<3>);
+    default: return go(ehvix_kernel<4>);
+    }
+}
+
+scoot_status scoot_score_ehvi_exact(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                                    const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                                    const float* grid, int32_t grid_cap, const int32_t* h_n_grid,
+                                    const uint32_t* corner, int32_t n_boxes, float* acq, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    ScoreArgs a;
+    if ((s = fill_state_args(ctx, L, state, a)) != SCOOT_OK) return s;
+    if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
+    if ((s = fill_box_grid(ctx, L->n_obj, grid, grid_cap, h_n_grid, corner, n_boxes, a)) != SCOOT_OK) return s;
+    if (n == 0) return SCOOT_OK;
+    if (!acq) return scoot_fail(ctx, SCOOT_EINVAL, "acq is NULL");
+    a.cand = cand;
+    a.n = n;
+    a.ld = ld;
+    a.mask = mask;
+    a.acq = acq;
+    return dispatch_m<kEHVIX>(ctx, a, L->n_obj, static_cast<cudaStream_t>(stream));
 }
 
 scoot_status scoot_score_ei(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,

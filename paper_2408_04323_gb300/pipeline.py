@@ -35,7 +35,7 @@ class RoundInputs:
     noise_var: np.ndarray      # float32[M]
     ref: np.ndarray            # float32[M]
     eps: np.ndarray            # float32[S][M]
-    acq: str                   # "ei", "ehvi" or "mace"
+    acq: str                   # "ei", "ehvi", "ehvi-exact" or "mace"
     q: int
     kernel: int = S.MATERN52
     xi: float = 1e-4
@@ -69,13 +69,18 @@ class State:
         self.forest = torch.from_numpy(fblob).to(device)
         self.n_boxes = 0
         self.front_size = 0
-        if inp.acq == "ehvi":
+        if inp.acq in ("ehvi", "ehvi-exact"):
             lo, hi, self.front_size = S.scoot_boxes_build(inp.y_obs, inp.ref)
             self.n_boxes = len(lo)
             self.h_boxes = (lo, hi)
             self.box_lo = torch.from_numpy(lo).to(device)
             self.box_hi = torch.from_numpy(hi).to(device)
             self.eps = torch.from_numpy(np.ascontiguousarray(inp.eps, np.float32)).to(device)
+        if inp.acq == "ehvi-exact":
+            grid, self.n_grid, corner = S.scoot_boxes_index(lo, hi)
+            self.h_boxes = (lo, hi, grid, corner)
+            self.grid = torch.from_numpy(grid).to(device)
+            self.corner = torch.from_numpy(corner.view(np.int32)).to(device)
 
 
 class ScoringRound:
@@ -157,6 +162,9 @@ class ScoringRound:
             return self.top_idx, self.top_val, self.top_count
         if inp.acq == "ei":
             S.scoot_score_ei(self.ctx, st.gp_layout, st.gp_state, cand, n, inp.xi, self.acq, self.mask, stream)
+        elif inp.acq == "ehvi-exact":
+            S.scoot_score_ehvi_exact(self.ctx, st.gp_layout, st.gp_state, cand, n, st.grid, st.n_grid, st.corner,
+                                     self.acq, self.mask, stream)
         else:
             S.scoot_score_ehvi(self.ctx, st.gp_layout, st.gp_state, cand, n, st.box_lo, st.box_hi, st.eps,
                                self.acq, self.mask, stream)

@@ -81,6 +81,10 @@ _PROTOS = {
     "scoot_acq_ei": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp],
     "scoot_boxes_build": [_vp, _i32, _i32, _vp, _i32, _vp, _vp, C.POINTER(_i32), C.POINTER(_i32)],
     "scoot_acq_ehvi": [_vp, _vp, _vp, _i64, _i32, _vp, _i64, _vp, _vp, _i32, _vp, _i32, _vp, _vp],
+    "scoot_boxes_index": [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp],
+    "scoot_acq_ehvi_exact": [_vp, _vp, _vp, _i64, _i32, _vp, _i64, _vp, _i32, _vp, _vp, _i32, _vp, _vp],
+    "scoot_score_ehvi_exact": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _i32, _vp, _vp,
+                               _i32, _vp, _vp],
     "scoot_score_ei": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _f32, _vp, _vp],
     "scoot_score_ehvi": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i32,
                          _vp, _i32, _vp, _vp],
@@ -268,6 +272,18 @@ def scoot_boxes_build(h_y, h_ref, cap: int = 4096):
     return lo[:nb.value].copy(), hi[:nb.value].copy(), int(fs.value)
 
 
+def scoot_boxes_index(h_lo, h_hi, grid_cap: int = 256):
+    """Boxes [B][M] -> (grid float32 [M][grid_cap], n_grid int32 [M], corner uint32 [B][M])."""
+    B, M = h_lo.shape
+    grid = np.zeros((M, max(grid_cap, 1)), np.float32)
+    n_grid = np.zeros(M, np.int32)
+    corner = np.zeros((max(B, 1), M), np.uint32)
+    _check(lib().scoot_boxes_index(_host(np.ascontiguousarray(h_lo), dtype=np.float32, name="h_lo"),
+                                   _host(np.ascontiguousarray(h_hi), dtype=np.float32, name="h_hi"), int(B), int(M),
+                                   int(grid_cap), _host(grid), _host(n_grid), _host(corner)), "scoot_boxes_index")
+    return grid, n_grid, corner[:B].copy()
+
+
 # ------------------------------------------------------------------ device calls
 
 def scoot_prune(ctx, h_space, h_clauses, cand, n, mask, n_feasible=None, stream=None):
@@ -314,6 +330,29 @@ def scoot_acq_ehvi(ctx, mean, var, n, box_lo, box_hi, eps, acq, mask=None, strea
                                 _dev(box_lo, torch.float32, "box_lo"), _dev(box_hi, torch.float32, "box_hi"),
                                 int(box_lo.shape[0]), _dev(eps, torch.float32, "eps"), int(eps.shape[0]),
                                 _dev(acq, torch.float32, "acq"), _stream(stream)), "scoot_acq_ehvi", _h(ctx))
+
+
+def scoot_acq_ehvi_exact(ctx, mean, var, n, grid, h_n_grid, corner, acq, mask=None, stream=None):
+    """grid: float32 [M][grid_cap], h_n_grid: host int32 [M], corner: [B][M] (int32 view of uint32)."""
+    import torch
+    M = int(mean.shape[0])
+    n_grid = np.ascontiguousarray(h_n_grid, np.int32)
+    _check(lib().scoot_acq_ehvi_exact(_h(ctx), _dev(mean, torch.float32, "mean"), _dev(var, torch.float32, "var"),
+                                      int(mean.shape[1]), M, _dev(mask, torch.uint8, "mask"), int(n),
+                                      _dev(grid, torch.float32, "grid"), int(grid.shape[1]), _host(n_grid),
+                                      _dev(corner, torch.int32, "corner"), int(corner.shape[0]),
+                                      _dev(acq, torch.float32, "acq"), _stream(stream)), "scoot_acq_ehvi_exact", _h(ctx))
+
+
+def scoot_score_ehvi_exact(ctx, layout, state, cand, n, grid, h_n_grid, corner, acq, mask=None, stream=None):
+    import torch
+    n_grid = np.ascontiguousarray(h_n_grid, np.int32)
+    _check(lib().scoot_score_ehvi_exact(_h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"),
+                                        _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]),
+                                        _dev(mask, torch.uint8, "mask"), _dev(grid, torch.float32, "grid"),
+                                        int(grid.shape[1]), _host(n_grid), _dev(corner, torch.int32, "corner"),
+                                        int(corner.shape[0]), _dev(acq, torch.float32, "acq"), _stream(stream)),
+           "scoot_score_ehvi_exact", _h(ctx))
 
 
 def scoot_score_ei(ctx, layout, state, cand, n, xi, acq, mask=None, stream=None):

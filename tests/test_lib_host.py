@@ -212,3 +212,25 @@ def test_forest_chunking_of_large_forests(S):
     ch = blob[L.off_chunks:L.off_chunks + 16 * L.n_chunks].view(np.int32).reshape(-1, 4)
     assert ch[:, 1].sum() == inst.n_trees * reps and ch[:, 3].sum() == len(nodes)
     assert np.all(ch[1:, 0] == np.cumsum(ch[:-1, 1]))
+
+
+@pytest.mark.parametrize("M,npts", [(2, 1), (2, 12), (3, 9), (3, 30), (4, 7)])
+def test_boxes_index_reproduces_the_boxes(S, M, npts):
+    st = Stream(300 + M * 7 + npts, "boxidx")
+    Y = (st.uniform(M * npts).reshape(M, npts) * 4.0).astype(np.float32)
+    lo, hi, _ = S.scoot_boxes_build(Y, np.zeros(M, np.float32))
+    grid, n_grid, corner = S.scoot_boxes_index(lo, hi)
+    for j in range(M):
+        g = grid[j, :n_grid[j]]
+        assert np.all(np.diff(g) > 0)
+        ext = np.concatenate([g, [np.inf]]).astype(np.float32)
+        assert np.array_equal(ext[corner[:, j] & 0xFFFF], lo[:, j])
+        assert np.array_equal(ext[corner[:, j] >> 16], hi[:, j])
+    with pytest.raises(S.ScootError) as e:
+        S.scoot_boxes_index(lo, hi, grid_cap=1)
+    assert e.value.status == -6
+    bad = hi.copy()
+    bad[0, 0] = lo[0, 0]
+    with pytest.raises(S.ScootError) as e:
+        S.scoot_boxes_index(lo, bad)
+    assert e.value.status == -1
