@@ -217,12 +217,23 @@ def matern(r, signal_var: float, kernel: int = MATERN52):
     raise ValueError(kernel)
 
 
+def kumaraswamy_cdf(u, a, b):
+    """Input warping of Section 4.3 (the Kumaraswamy CDF of the warping work
+    the paper cites): w(u) = 1 - (1 - u^a)^b on [0, 1], a, b > 0."""
+    u = np.clip(np.asarray(u, np.float64), 0.0, 1.0)
+    return 1.0 - (1.0 - u ** a) ** b
+
+
 class GP:
-    """One objective's GP conditioned on the observations (Section 4.3)."""
+    """One objective's GP conditioned on the observations (Section 4.3).
+
+    ``warp`` ([d][2], optional) gives each parameter's Kumaraswamy (a, b);
+    ordinal features are warped before the distance, categoricals never."""
 
     def __init__(self, space, x_obs_words, y, lengthscale, signal_var, noise_var,
-                 kernel: int = MATERN52):
+                 kernel: int = MATERN52, warp=None):
         self.space = space
+        self.warp = None if warp is None else np.asarray(warp, np.float64)
         self.kernel = kernel
         self.lengthscale = np.asarray(lengthscale, np.float64)
         self.signal_var = float(signal_var)
@@ -238,8 +249,17 @@ class GP:
         self.chol = np.linalg.cholesky(K)            # K + tau^2 I = L L^T
         self.alpha = sla.cho_solve((self.chol, True), self.y)  # (K + tau^2 I)^{-1} Y
 
+    def warped(self, u):
+        """Features with the ordinal coordinates warped (identity without warp)."""
+        if self.warp is None:
+            return u
+        w = np.array(u, np.float64, copy=True)
+        for c in np.nonzero(~self.is_cat)[0]:
+            w[:, c] = kumaraswamy_cdf(u[:, c], self.warp[c, 0], self.warp[c, 1])
+        return w
+
     def cov(self, ua, ub):
-        return matern(scaled_distance(ua, ub, self.is_cat, self.lengthscale),
+        return matern(scaled_distance(self.warped(ua), self.warped(ub), self.is_cat, self.lengthscale),
                       self.signal_var, self.kernel)
 
     def add_observations(self, u_new, y_new):

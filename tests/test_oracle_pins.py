@@ -663,3 +663,48 @@ def test_mace_select_draws_from_the_front():
         counts[O.mace_select(A, mask, 2, seed=s)[0]] += 1
     freq = counts[front] / 2000
     assert np.all(np.abs(freq - 2 / F) < 5 * math.sqrt((2 / F) * (1 - 2 / F) / 2000) + 1e-9)
+
+
+# ------------------------------------------------------------------ input warping (Section 4.3)
+
+def test_kumaraswamy_cdf_is_the_integral_of_its_density():
+    for a, b in [(0.5, 2.0), (1.7, 0.6), (3.0, 3.0), (1.0, 1.0)]:
+        pdf = lambda x: a * b * x ** (a - 1) * (1 - x ** a) ** (b - 1)
+        for u in (0.05, 0.3, 0.77, 0.999):
+            q, _ = integrate.quad(pdf, 0.0, u, epsabs=1e-13, epsrel=1e-11, limit=200)
+            assert float(O.kumaraswamy_cdf(u, a, b)) == pytest.approx(q, rel=1e-8, abs=1e-12)
+    u = np.linspace(0, 1, 101)
+    assert np.allclose(O.kumaraswamy_cdf(u, 1.0, 1.0), u, atol=1e-15)
+    w = O.kumaraswamy_cdf(u, 2.3, 0.4)
+    assert w[0] == 0.0 and w[-1] == 1.0 and np.all(np.diff(w) > 0)
+
+
+def test_warped_gp_is_the_plain_gp_on_warped_features():
+    """The warp acts once on both the observations and the candidates."""
+    sp, X, y, gp = _toy_gp(20, noise=1e-3)
+    st = Stream(81, "warp")
+    warp = np.exp(st.normal(2 * len(sp)).reshape(len(sp), 2) * 0.4)
+    Xw = X.view(np.uint32)
+    gw = O.GP(sp, Xw, y, gp.lengthscale, gp.signal_var, gp.noise_var, gp.kernel, warp=warp)
+    C = st.uniform(3 * 200).reshape(3, 200).astype(np.float32).view(np.uint32)
+    u, cat = O.gp_features(sp, O.decode(sp, C))
+    plain = O.GP(sp, Xw, y, gp.lengthscale, gp.signal_var, gp.noise_var, gp.kernel)
+    plain.u_obs = gw.warped(plain.u_obs)
+    plain._factor()
+    m1, v1 = gw.posterior_u(u)
+    m2, v2 = plain.posterior_u(gw.warped(u))
+    assert np.allclose(m1, m2, rtol=1e-12, atol=1e-13) and np.allclose(v1, v2, rtol=1e-12, atol=1e-13)
+    # one observation, one ordinal dimension: the closed form on warped coordinates
+    sp1 = sp[:1]
+    x1 = np.ascontiguousarray(Xw[:1, :1])
+    g1 = O.GP(sp1, x1, y[:1], gp.lengthscale[:1], 1.0, 0.1, O.MATERN52, warp=warp[:1])
+    c1 = np.ascontiguousarray(C[:1, :5])
+    uc, _ = O.gp_features(sp1, O.decode(sp1, c1))
+    uo, _ = O.gp_features(sp1, O.decode(sp1, x1))
+    a_, b_ = warp[0]
+    wc = 1 - (1 - uc[:, 0] ** a_) ** b_
+    wo = 1 - (1 - uo[0, 0] ** a_) ** b_
+    r = np.abs(wc - wo) / gp.lengthscale[0]
+    k = (1 + math.sqrt(5) * r + 5 * r * r / 3) * np.exp(-math.sqrt(5) * r)
+    mu, var = g1.posterior_u(uc)
+    assert np.allclose(mu, k * y[0] / 1.1, rtol=1e-12) and np.allclose(var, 1 - k * k / 1.1, rtol=1e-10, atol=1e-14)

@@ -247,6 +247,17 @@ def train_forest(w: Workload, st: Stream, feats: np.ndarray, labels: np.ndarray)
 
 # ---------------------------------------------------------------- instance
 
+def warp_params(w: Workload | str, seed: int) -> np.ndarray:
+    """Input-warping parameters for the workload's GPs: float32 [M][d][2] of
+    Kumaraswamy (a, b), each lognormal(0, 0.4) (hyperparameters are inputs of
+    the path; the tuner would fit them).  Categorical entries are drawn too
+    and ignored by both sides."""
+    if isinstance(w, str):
+        w = WORKLOADS[w]
+    st = Stream(seed, "warp")
+    return np.exp(st.normal(w.n_obj * w.d * 2) * 0.4).reshape(w.n_obj, w.d, 2).astype(np.float32)
+
+
 def make_instance(w: Workload | str, seed: int, n_cand: int | None = None,
                   ld_pad: int = 4) -> Instance:
     """Build one seeded instance; ``n_cand`` overrides the pool size."""
