@@ -61,6 +61,9 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--kernel", choices=["matern52", "matern32"], default="matern52",
+                   help="covariance (matern32 with --warp is the paper's own kernel)")
+    p.add_argument("--warp", action="store_true", help="Kumaraswamy input warping of ordinal features")
     p.add_argument("--acq", choices=["default", "mace", "ehvi-exact"], default="default",
                    help="mace: UCB/PI/EI and a random subset of their Pareto front (one objective); "
                         "ehvi-exact: EHVI as the exact expectation (several objectives)")
@@ -172,17 +175,18 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(loaded)}
 
 
-def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None):
+def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None, kernel=0, warp=False):
     """Time the oracle on n_sample candidates of the workload in a fresh process
     (with mace_kappa set: the MACE round, UCB coefficient mace_kappa; acq
     overrides the workload's acquisition)."""
     env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
                MKL_NUM_THREADS=str(threads))
+    gp_opts = "kernel=%d, warp=%s" % (kernel, "warp_params(%r, %d)" % (name, seed) if warp else "None")
     if mace_kappa is None:
-        select = ("r = oracle.score_round(inst, %s)\n" % (repr(acq) if acq else "inst.workload.acq") +
+        select = ("r = oracle.score_round(inst, %s, %s)\n" % (repr(acq) if acq else "inst.workload.acq", gp_opts) +
                   "oracle.select_topq(r['acq'], r['feasible'], inst.workload.q)\n")
     else:
-        select = ("r = oracle.score_round(inst, 'ei')\n"
+        select = ("r = oracle.score_round(inst, 'ei', %s)\n" % gp_opts +
                   "A = oracle.mace_acquisitions(r['mu'][:, 0], r['var'][:, 0], float(inst.y_obs[0].max()), "
                   "1e-4, %r)\n"
                   "A[:, ~r['feasible']] = -np.inf\n"
@@ -190,7 +194,7 @@ def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None
     code = (
         "import sys, time, json; sys.path.insert(0, %r)\n"
         "import numpy as np, oracle\n"
-        "from workloads import make_instance\n"
+        "from workloads import make_instance, warp_params\n"
         "inst = make_instance(%r, %d, n_cand=%d)\n"
         "t = time.perf_counter()\n" % (ROOT, name, seed, n_sample)
         + select
@@ -201,10 +205,10 @@ def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None
     return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
 
 
-def calibrate_sample(name, seed, budget_s, mace_kappa=None, acq=None):
+def calibrate_sample(name, seed, budget_s, mace_kappa=None, acq=None, kernel=0, warp=False):
     """Largest sample whose oracle round fits the budget (scaled from a probe)."""
     probe = 64
-    t = cpu_oracle_sample(name, seed, probe, mace_kappa=mace_kappa, acq=acq)
+    t = cpu_oracle_sample(name, seed, probe, mace_kappa=mace_kappa, acq=acq, kernel=kernel, warp=warp)
     per = max(t / probe, 1e-6)
     return max(16, int(budget_s / per))
 
@@ -221,18 +225,21 @@ def run_reference(args):
         from paper_2408_04323_gb300.pipeline import mace_beta
         kappa = mace_beta(w.n_obs)
     acq = "ehvi-exact" if args.acq == "ehvi-exact" else None
+    kern = 1 if args.kernel == "matern32" else 0
+    opts = dict(mace_kappa=kappa, acq=acq, kernel=kern, warp=args.warp)
     per_step = max(0.05, 120.0 / max(1, args.steps + args.warmup))
-    sample = calibrate_sample(w.name, seed, per_step, kappa, acq)
+    sample = calibrate_sample(w.name, seed, per_step, kappa, acq, kern, args.warp)
     for _ in range(args.warmup):
-        cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq)
-    times = [cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq) for _ in range(args.steps)]
+        cpu_oracle_sample(w.name, seed, sample, **opts)
+    times = [cpu_oracle_sample(w.name, seed, sample, **opts) for _ in range(args.steps)]
     ms = 1e3 * statistics.mean(times)
     value = sample / (ms / 1e3)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(w, {"reference": "fp64 CPU oracle (the paper ships no code)",
-                                          "sample_per_step": sample},
+                                          "sample_per_step": sample, "kernel": args.kernel,
+                                          "warp": bool(args.warp)},
                                       acq=None if args.acq == "default" else args.acq),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{sample} candidates of the {w.name} pool per step, all five steps"},
@@ -264,7 +271,7 @@ def main():
     from paper_2408_04323_gb300 import scoot as S
     from paper_2408_04323_gb300.pipeline import RoundInputs, ScoringRound, State
     from paper_2408_04323_gb300.shard import gather_topq
-    from workloads import WORKLOADS, Stream, draw_configs, make_instance, seeds
+    from workloads import WORKLOADS, Stream, draw_configs, make_instance, seeds, warp_params
 
     w = WORKLOADS[args.workload]
     acq_kind = w.acq if args.acq == "default" else args.acq
@@ -282,7 +289,11 @@ def main():
     N = inst.n_cand
     inp = RoundInputs(inst.space, inst.clauses, inst.nodes, inst.tree_offset, w.leaf_scale, w.delta_num,
                       w.delta_den, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
-                      inst.noise_var, inst.ref, inst.eps, acq_kind, w.q, fantasy=w.fantasy)
+                      inst.noise_var, inst.ref, inst.eps, acq_kind, w.q, fantasy=w.fantasy,
+                      kernel=S.MATERN32 if args.kernel == "matern32" else S.MATERN52,
+                      warp=warp_params(w, seed) if args.warp else None)
+    if args.warp and w.fantasy:
+        raise SystemExit("--warp: fantasy picks take unwarped GP states")
     ctx = S.Context(device.index)
     rnd = ScoringRound(ctx, inp, N, device)
     cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
@@ -495,8 +506,8 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         kappa = rnd.kappa if inp.acq == "mace" else None
         acq = "ehvi-exact" if inp.acq == "ehvi-exact" else None
-        sample = calibrate_sample(w.name, seed, args.cpu_seconds, kappa, acq)
-        secs = cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq)
+        sample = calibrate_sample(w.name, seed, args.cpu_seconds, kappa, acq, inp.kernel, args.warp)
+        secs = cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq, kernel=inp.kernel, warp=args.warp)
         cpu = {"value": sample / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"{sample} candidates of the {w.name} pool (same round state), all five steps, "
                          f"fp64 numpy, one thread"}
@@ -509,7 +520,8 @@ def main():
                                               "front": st.front_size, "parallelism": f"pool shards x{world}",
                                               "launch": "CUDA graph of the step" if graph is not None
                                               else "eager launches",
-                                              "eager_ms_per_step": round(eager_ms, 5)}, acq=inp.acq),
+                                              "eager_ms_per_step": round(eager_ms, 5),
+                                              "kernel": args.kernel, "warp": bool(args.warp)}, acq=inp.acq),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps * rnd.kernels_per_round(),
                 "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},

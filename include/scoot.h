@@ -206,9 +206,12 @@ typedef struct {
     int64_t off_ils;          /* float[M][d]: 1/l (ordinal) or 1/l^2 (categorical), feature order */
     int64_t off_alpha;        /* float[M][n] */
     int64_t off_linv;         /* float[M][n_tiles][32][64]: L^{-1} tiles, transposed, zero-filled */
-    int64_t off_scal;         /* float[M][4]: signal variance, noise variance, best observed y, 0 */
+    int64_t off_scal;         /* float[M][4]: signal variance, noise variance, best observed y,
+                                 1 if the objective's ordinal features are warped else 0 */
     int64_t off_cat;          /* float[M][n][n_pat]: for each category pattern p (mixed radix over the
                                  categorical parameters in feature order), sum_c [p_c != X_jc] / l_c^2 */
+    int64_t off_warp;         /* float[M][d][2]: Kumaraswamy (a, b) per feature, feature order
+                                 (1, 1 when not warped) */
 } scoot_gp_layout;
 
 /* Plan the blob for n observations of the d-parameter space h_space, M
@@ -230,6 +233,20 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
                               const float* h_y, const float* h_lengthscale,
                               const float* h_signal_var, const float* h_noise_var,
                               const scoot_gp_layout* layout, void* h_blob, double* h_cond);
+
+/* scoot_gp_prepare with input warping (the kernel of Section 4.3 is Matérn
+ * with input warping): every ordinal feature u of objective m is replaced by
+ * the Kumaraswamy CDF w(u) = 1 - (1 - u^a)^b before distances are taken, for
+ * the observations here and for the candidates inside the posterior and
+ * scoring kernels.  h_warp: [M][d][2] = (a, b) per parameter (source order,
+ * a, b > 0 and finite; entries of categorical parameters are ignored).  The
+ * kernels evaluate w as -expm1(b log1p(-u^a)).  scoot_suggest_fantasy does
+ * not take warped states (SCOOT_EUNSUPPORTED). */
+scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
+                                     const float* h_y, const float* h_lengthscale,
+                                     const float* h_signal_var, const float* h_noise_var,
+                                     const float* h_warp, const scoot_gp_layout* layout, void* h_blob,
+                                     double* h_cond);
 
 /* mean[m * ldo + i], var[m * ldo + i] for every candidate i < n and
  * objective m:  mu = k(x, X)(K + tau^2 I)^{-1} Y and

@@ -472,7 +472,7 @@ def select_topq(acq, mask, q: int):
 # whole round
 
 def score_round(inst, acq_kind: str, xi: float = 1e-4, kernel: int = MATERN52,
-                subset: np.ndarray | None = None):
+                subset: np.ndarray | None = None, warp=None):
     """One suggestion round on an instance: masks, votes, posterior, acquisition.
 
     ``subset`` restricts the GP/acquisition work to those candidate indices
@@ -484,8 +484,8 @@ def score_round(inst, acq_kind: str, xi: float = 1e-4, kernel: int = MATERN52,
     votes = rf_votes(inst.nodes, inst.tree_offset, inst.space, words, n)
     feas = mask_k & pof_feasible(votes, inst.n_trees, w.leaf_scale, w.delta_num, w.delta_den)
     sel = np.arange(n) if subset is None else np.asarray(subset)
-    gps = [GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m],
-              inst.signal_var[m], inst.noise_var[m], kernel) for m in range(inst.n_obj)]
+    gps = [GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m], inst.signal_var[m],
+              inst.noise_var[m], kernel, warp=None if warp is None else warp[m]) for m in range(inst.n_obj)]
     sub_words = words[:, sel]
     mv = [gp.posterior(sub_words) for gp in gps]
     mu = np.stack([m for m, _ in mv], axis=1)

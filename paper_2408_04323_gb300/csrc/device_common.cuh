@@ -25,6 +25,16 @@ __device__ __forceinline__ float ei_value(float mu, float var, float ybest, floa
     return fmaf(a, cdf, s * pdf);
 }
 
+// Kumaraswamy CDF w(u) = 1 - (1 - u^a)^b (input warping), evaluated as
+// -expm1(b log1p(-u^a)) so that small u^a keeps its relative accuracy.  Not
+// inlined: the scoring kernels call it only for warped states, and inlining
+// it raised the register pressure of their common, unwarped path.
+static __device__ __noinline__ float kumaraswamy_cdf(float u, float a, float b) {
+    u = fminf(fmaxf(u, 0.0f), 1.0f);
+    const float ua = u > 0.0f ? exp2f(a * log2f(u)) : 0.0f;
+    return -expm1f(b * log1pf(-ua));
+}
+
 // PI = P(f + xi > y+) = Phi((mu + xi - y+) / sigma); a step at sigma = 0.
 __device__ __forceinline__ float pi_value(float mu, float var, float ybest, float xi) {
     const float a = (mu - ybest) + xi;

@@ -86,8 +86,19 @@ double HostGP::cov(const double* ua, const double* ub) const {
     return sf2 * matern(std::sqrt(r2), kernel);
 }
 
+void HostGP::warp_features(double* uf) const {
+    if (warp.empty()) return;
+    for (int c = 0; c < d; ++c) {
+        if (cat[c]) continue;
+        const double x = std::min(std::max(uf[c], 0.0), 1.0);
+        uf[c] = 1.0 - std::pow(1.0 - std::pow(x, warp[2 * c]), warp[2 * c + 1]);
+    }
+}
+
 void HostGP::kstar(const double* ux, double* k) const {
-    for (int j = 0; j < n; ++j) k[j] = cov(ux, &u[(size_t)j * d]);
+    std::vector<double> w(ux, ux + d);
+    warp_features(w.data());
+    for (int j = 0; j < n; ++j) k[j] = cov(w.data(), &u[(size_t)j * d]);
 }
 
 void HostGP::solve_lower(const double* b, double* x) const {
@@ -110,7 +121,7 @@ bool scoot_host_features(const scoot_param* sp, int d, const uint32_t* words, in
 
 scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, int64_t ld_obs, int n,
                            const float* y, const float* lengthscale, float signal_var, float noise_var,
-                           int kernel, HostGP* g, double* cond) {
+                           int kernel, HostGP* g, double* cond, const float* warp) {
     if (!(signal_var > 0.0f) || !is_finite(signal_var) || !(noise_var >= 0.0f) || !is_finite(noise_var))
         return SCOOT_EINVAL;
     g->n = n;
@@ -121,14 +132,26 @@ scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, 
     g->u.assign((size_t)n * d, 0.0);
     g->cat.assign(d, 0);
     g->ell.assign(d, 1.0);
+    g->warp.clear();
     for (int c = 0; c < d; ++c) {
         if (!(lengthscale[c] > 0.0f) || !is_finite(lengthscale[c])) return SCOOT_EINVAL;
         g->ell[c] = lengthscale[c];
         g->cat[c] = sp[c].kind == SCOOT_CATEGORICAL;
     }
+    if (warp) {
+        g->warp.assign(2 * (size_t)d, 1.0);
+        for (int c = 0; c < d; ++c) {
+            if (g->cat[c]) continue;
+            for (int t = 0; t < 2; ++t) {
+                if (!(warp[2 * c + t] > 0.0f) || !is_finite(warp[2 * c + t])) return SCOOT_EINVAL;
+                g->warp[2 * c + t] = warp[2 * c + t];
+            }
+        }
+    }
     for (int j = 0; j < n; ++j) {
         if (!is_finite(y[j])) return SCOOT_EINVAL;
         if (!scoot_host_features(sp, d, x_obs, ld_obs, j, &g->u[(size_t)j * d])) return SCOOT_EINVAL;
+        g->warp_features(&g->u[(size_t)j * d]);
     }
     std::vector<double>& K = g->chol;
     K.assign((size_t)n * n, 0.0);
@@ -209,6 +232,7 @@ scoot_status gp_layout_compute(int32_t n, int32_t d, int32_t n_obj, int32_t kern
     out->off_linv = off;  off = align_up(off + (int64_t)n_obj * out->n_tiles * kColChunk * kRowBlock * 4);
     out->off_scal = off;  off = align_up(off + (int64_t)n_obj * 4 * 4);
     out->off_cat = off;   off = align_up(off + (int64_t)n_obj * n * n_pat * 4);
+    out->off_warp = off;  off = align_up(off + (int64_t)n_obj * d * 2 * 4);
     out->bytes = off;
     return SCOOT_OK;
 }
@@ -248,6 +272,15 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
                               const float* h_y, const float* h_lengthscale,
                               const float* h_signal_var, const float* h_noise_var,
                               const scoot_gp_layout* L, void* h_blob, double* h_cond) {
+    return scoot_gp_prepare_warped(h_space, h_x_obs, ld_obs, h_y, h_lengthscale, h_signal_var, h_noise_var,
+                                   nullptr, L, h_blob, h_cond);
+}
+
+scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
+                                     const float* h_y, const float* h_lengthscale,
+                                     const float* h_signal_var, const float* h_noise_var,
+                                     const float* h_warp, const scoot_gp_layout* L, void* h_blob,
+                                     double* h_cond) {
     if (!h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var || !L || !h_blob)
         return SCOOT_EINVAL;
     scoot_gp_layout chk;
@@ -308,14 +341,21 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
     float* alpha_out = reinterpret_cast<float*>(blob + L->off_alpha);
     float* linv_out = reinterpret_cast<float*>(blob + L->off_linv);
     float* scal = reinterpret_cast<float*>(blob + L->off_scal);
+    float* warp_out = reinterpret_cast<float*>(blob + L->off_warp);
 
     std::vector<double> Li((size_t)n * n), e(n), col(n);
     HostGP g;
     for (int m = 0; m < M; ++m) {
         scoot_status s = scoot_host_gp(h_space, d, h_x_obs, ld_obs, n, h_y + (size_t)m * n,
                                        h_lengthscale + (size_t)m * d, h_signal_var[m], h_noise_var[m],
-                                       L->kernel, &g, h_cond ? &h_cond[m] : nullptr);
+                                       L->kernel, &g, h_cond ? &h_cond[m] : nullptr,
+                                       h_warp ? h_warp + (size_t)m * d * 2 : nullptr);
         if (s != SCOOT_OK) return s;
+        for (int f = 0; f < d; ++f) {
+            const int c = order[f];
+            warp_out[((size_t)m * d + f) * 2 + 0] = g.warp.empty() || g.cat[c] ? 1.0f : (float)g.warp[2 * c];
+            warp_out[((size_t)m * d + f) * 2 + 1] = g.warp.empty() || g.cat[c] ? 1.0f : (float)g.warp[2 * c + 1];
+        }
         for (int f = 0; f < d; ++f) {
             const int c = order[f];
             const double l = g.ell[c];
@@ -363,6 +403,7 @@ scoot_status scoot_gp_prepare(const scoot_param* h_space, const uint32_t* h_x_ob
         scal[m * 4 + 0] = h_signal_var[m];
         scal[m * 4 + 1] = h_noise_var[m];
         scal[m * 4 + 2] = ybest;
+        scal[m * 4 + 3] = h_warp ? 1.0f : 0.0f;
     }
     return SCOOT_OK;
 }

@@ -46,17 +46,21 @@ struct HostGP {
     std::vector<double> ell;      // [d] lengthscales
     std::vector<double> chol;     // [n][n], lower triangle
     std::vector<double> alpha;    // [n]
-    double cov(const double* ua, const double* ub) const;       // k(a, b)
-    void kstar(const double* ux, double* k) const;              // k(x, X_j), j < n
+    std::vector<double> warp;     // [d][2] Kumaraswamy (a, b) per parameter; empty: no warping
+    double cov(const double* ua, const double* ub) const;       // k(a, b) of (warped) features
+    void warp_features(double* u) const;                        // in place; no-op without warping
+    void kstar(const double* ux, double* k) const;              // k(x, X_j), j < n; ux unwarped
     void solve_lower(const double* b, double* x) const;         // C x = b
 };
 // Features of configuration j of a SoA word array (ld = leading dimension).
 bool scoot_host_features(const scoot_param* sp, int d, const uint32_t* words, int64_t ld, int64_t j, double* u);
 // Factor objective m; SCOOT_EINVAL on bad inputs or a matrix that is not
 // numerically positive definite.  cond (optional) receives (max/min pivot)^2.
+// warp: [d][2] Kumaraswamy (a, b) per parameter, or NULL; g->u holds the
+// warped features of the observations.
 scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, int64_t ld_obs, int n,
                            const float* y, const float* lengthscale, float signal_var, float noise_var,
-                           int kernel, HostGP* out, double* cond);
+                           int kernel, HostGP* out, double* cond, const float* warp = nullptr);
 
 // Consistency of a GP layout's offsets with its own sizes.
 bool scoot_gp_layout_valid(const scoot_gp_layout* L);

@@ -33,7 +33,7 @@ enum Epilogue { kWriteMoments = 0, kEI = 1, kEHVI = 2, kWriteWhitened = 3, kMACE
 
 struct ScoreArgs {
     const char* state;
-    int64_t off_fmap, off_xs, off_ils, off_alpha, off_linv, off_scal, off_cat;
+    int64_t off_fmap, off_xs, off_ils, off_alpha, off_linv, off_scal, off_cat, off_warp;
     int32_t n_obs, d, dp, n_obj, kernel, n_rb, n_tiles, n_ord, n_pat;
     const uint32_t* cand;
     int64_t n, ld;
@@ -292,8 +292,16 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             const float sf2 = gscal[m * 4 + 0];
             const float* catrow = gcat + (size_t)m * a.n_obs * a.n_pat + pid;
             float ut[DO];
+            const bool warped = gscal[m * 4 + 3] != 0.0f;  // the same in every thread
 #pragma unroll
-            for (int q = 0; q < DO; ++q) ut[q] = q < n_ord ? u[q] * gils[m * a.d + q] : 0.0f;
+            for (int q = 0; q < DO; ++q) {
+                float x = u[q];
+                if (warped && q < n_ord) {
+                    const float2 ab = __ldg(reinterpret_cast<const float2*>(a.state + a.off_warp) + m * a.d + q);
+                    x = kumaraswamy_cdf(x, ab.x, ab.y);
+                }
+                ut[q] = q < n_ord ? x * gils[m * a.d + q] : 0.0f;
+            }
             __syncthreads();
             // 1. covariance row (this half's j) and the partial mean.
             float acc = 0.0f;
@@ -585,6 +593,7 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
     a.off_linv = L->off_linv;
     a.off_scal = L->off_scal;
     a.off_cat = L->off_cat;
+    a.off_warp = L->off_warp;
     a.n_ord = L->n_ord;
     a.n_pat = L->n_pat;
     a.n_obs = L->n;

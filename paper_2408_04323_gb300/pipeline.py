@@ -42,6 +42,7 @@ class RoundInputs:
     fantasy: bool = False      # q sequential picks with kriging-believer fantasies
     kappa: float | None = None  # MACE: UCB coefficient (None: mace_beta(n_obs))
     seed: int = 0               # MACE: seed of the random draw from the front
+    warp: np.ndarray | None = None  # float32 [M][d][2]: Kumaraswamy input warping (None: no warping)
 
 
 def mace_beta(t: int) -> float:
@@ -60,8 +61,12 @@ class State:
         d = len(inp.space)
         M = inp.y_obs.shape[0]
         self.gp_layout = S.scoot_gp_layout_init(inp.space, inp.y_obs.shape[1], M, inp.kernel)
-        blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
-                                             inp.signal_var, inp.noise_var, self.gp_layout)
+        if inp.warp is None:
+            blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                                 inp.signal_var, inp.noise_var, self.gp_layout)
+        else:
+            blob, self.cond = S.scoot_gp_prepare_warped(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                                        inp.signal_var, inp.noise_var, inp.warp, self.gp_layout)
         self.forest_layout = S.scoot_forest_layout_init(inp.nodes, inp.tree_offset, d, inp.leaf_scale)
         fblob = S.scoot_forest_pack(self.forest_layout, inp.nodes, inp.tree_offset)
         self.h_blobs = (blob, fblob)

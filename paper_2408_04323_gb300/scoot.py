@@ -57,7 +57,7 @@ class scoot_gp_layout(C.Structure):
                 ("n_rb", C.c_int32), ("n_tiles", C.c_int32), ("n_ord", C.c_int32), ("n_pat", C.c_int32),
                 ("bytes", C.c_int64), ("off_fmap", C.c_int64), ("off_xs", C.c_int64), ("off_ils", C.c_int64),
                 ("off_alpha", C.c_int64), ("off_linv", C.c_int64), ("off_scal", C.c_int64),
-                ("off_cat", C.c_int64)]
+                ("off_cat", C.c_int64), ("off_warp", C.c_int64)]
 
 
 assert C.sizeof(scoot_param) == 16 and C.sizeof(scoot_clause) == 80 and C.sizeof(scoot_node) == 8
@@ -77,6 +77,7 @@ _PROTOS = {
                          _vp, _vp, _vp, _vp],
     "scoot_gp_layout_init": [_vp, _i32, _i32, _i32, _i32, C.POINTER(scoot_gp_layout)],
     "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
+    "scoot_gp_prepare_warped": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_posterior": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i64, _vp],
     "scoot_acq_ei": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp],
     "scoot_boxes_build": [_vp, _i32, _i32, _vp, _i32, _vp, _vp, C.POINTER(_i32), C.POINTER(_i32)],
@@ -240,6 +241,21 @@ def scoot_gp_prepare(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise
                                   _host(h_signal_var, dtype=np.float32, name="h_signal_var"),
                                   _host(h_noise_var, dtype=np.float32, name="h_noise_var"),
                                   C.byref(layout), _host(blob), _host(cond)), "scoot_gp_prepare")
+    return blob, cond
+
+
+def scoot_gp_prepare_warped(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, h_warp, layout):
+    """scoot_gp_prepare with Kumaraswamy input warping h_warp float32 [M][d][2]."""
+    blob = np.zeros(layout.bytes, np.uint8)
+    cond = np.zeros(layout.n_obj, np.float64)
+    _check(lib().scoot_gp_prepare_warped(_host(h_space, 16, name="h_space"), _host(h_x_obs, 4, name="h_x_obs"),
+                                         int(h_x_obs.shape[1]), _host(h_y, dtype=np.float32, name="h_y"),
+                                         _host(h_lengthscale, dtype=np.float32, name="h_lengthscale"),
+                                         _host(h_signal_var, dtype=np.float32, name="h_signal_var"),
+                                         _host(h_noise_var, dtype=np.float32, name="h_noise_var"),
+                                         _host(np.ascontiguousarray(h_warp, np.float32), dtype=np.float32,
+                                               name="h_warp"),
+                                         C.byref(layout), _host(blob), _host(cond)), "scoot_gp_prepare_warped")
     return blob, cond
 
 

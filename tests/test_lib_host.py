@@ -234,3 +234,35 @@ def test_boxes_index_reproduces_the_boxes(S, M, npts):
     with pytest.raises(S.ScootError) as e:
         S.scoot_boxes_index(lo, bad)
     assert e.value.status == -1
+
+
+def test_gp_prepare_warped_matches_oracle(S):
+    from workloads import warp_params
+    inst = make_instance("d10-ei", seeds("d10-ei")[0], n_cand=64)
+    M, n, d = inst.n_obj, inst.n_obs, inst.d
+    warp = warp_params("d10-ei", 7)
+    L = S.scoot_gp_layout_init(inst.space, n, M, 1)
+    blob, _ = S.scoot_gp_prepare_warped(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                        inst.noise_var, warp, L)
+    alpha, linv, scal, xs, ils, src = _unpack_gp(S, L, blob)
+    gp = O.GP(inst.space, inst.x_obs, inst.y_obs[0], inst.lengthscale[0], inst.signal_var[0], inst.noise_var[0],
+              1, warp=warp[0])
+    assert np.allclose(alpha[0], gp.alpha, rtol=1e-6, atol=1e-6 * np.abs(gp.alpha).max())
+    Li = np.linalg.inv(gp.chol)
+    assert np.allclose(linv[0], Li, rtol=1e-6, atol=1e-6 * np.abs(Li).max())
+    cat = gp.is_cat
+    w = gp.warped(gp.u_obs)
+    assert np.allclose(xs[0][:, ~cat], w[:, ~cat] / inst.lengthscale[0][~cat], rtol=1e-6)
+    assert scal[0, 3] == 1.0
+    wa = blob[L.off_warp:L.off_warp + 8 * d].view(np.float32).reshape(d, 2)
+    kinds = inst.space["kind"][src]
+    assert np.array_equal(wa[kinds != 2], warp[0][src][kinds != 2]) and np.all(wa[kinds == 2] == 1.0)
+    plain, _ = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                  inst.noise_var, L)
+    assert _unpack_gp(S, L, plain)[2][0, 3] == 0.0
+    bad = warp.copy()
+    bad[0, 0, 1] = 0.0
+    with pytest.raises(S.ScootError) as e:
+        S.scoot_gp_prepare_warped(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                  inst.noise_var, bad, L)
+    assert e.value.status == -1
