@@ -119,6 +119,45 @@ def test_prune_edge_cases(S, ctx):
     assert np_(mask).all()
 
 
+@pytest.mark.parametrize("big", [False, True])
+def test_prune_many_clauses_and_wide_sums(S, ctx, big):
+    """Sixteen random guarded clauses over most of the twelve parameters
+    (distinct-column slots), with 2^40-sized coefficients when big (the
+    int128 path) or small ones (the int64 path)."""
+    from workloads import CLAUSE_DTYPE
+    inst = make_instance("d12-fantasy", seeds("d12-fantasy")[2], n_cand=20011)
+    st = Stream(88 + big, "clauses")
+    ints = [c for c in range(inst.d) if int(inst.space[c]["kind"]) != 3]
+    cats = [c for c in ints if int(inst.space[c]["kind"]) == 2]
+    cl = np.zeros(16, CLAUSE_DTYPE)
+    vals = inst.cand.view(np.int32)
+    for k in range(16):
+        nt = 1 + k % 4
+        terms = [ints[int(x)] for x in st.integers(0, len(ints) - 1, nt)]
+        scale = (1 << 40) if big else 1000
+        coef = [int(x) for x in (st.integers(0, 2 * scale, nt) - scale)]
+        cl[k]["n_term"] = nt
+        for t in range(nt):
+            cl[k]["term_param"][t] = terms[t]
+            cl[k]["coef"][t] = coef[t]
+        # rhs at the 5% quantile of the sum over a sample: each clause fails
+        # for about 5% of the pool, all sixteen together for about half
+        smp = sum(c * vals[p, :2000].astype(object) for c, p in zip(coef, terms))
+        cl[k]["rhs"] = int(sorted(smp)[100])
+        if cats and k % 3 == 0:
+            g = cats[k % len(cats)]
+            cl[k]["n_guard"] = 1
+            cl[k]["guard_param"][0] = g
+            cl[k]["guard_value"][0] = int(vals[g, 0])
+    n = inst.n_cand
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int64, device="cuda")
+    S.scoot_prune(ctx, inst.space, cl, cand_dev(inst), n, mask, cnt)
+    want = O.prune_mask(inst.space, cl, inst.cand, n)
+    assert np.array_equal(np_(mask).astype(bool), want)
+    assert int(np_(cnt)[0]) == int(want.sum()) and 0 < want.sum() < n
+
+
 def test_prune_rejects_bad_arguments(S, ctx):
     inst = make_instance("tiny", 1001, n_cand=64)
     cand = cand_dev(inst)
