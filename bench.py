@@ -48,9 +48,9 @@ FP32_LANES_PER_SM = 128
 KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["score.cu", "device_common.cuh"],
                 "topq": ["topq.cu", "device_common.cuh"], "pareto": ["pareto.cu"]}
 TRAFFIC = {
-    ("prune", "d8-ehvi2"): {"bytes": 3152896, "sha": "8774c0f1248b1325"},
-    ("rf", "d8-ehvi2"): {"bytes": 8809984, "sha": "8774c0f1248b1325"},
-    ("score", "d8-ehvi2"): {"bytes": 8843520, "sha": "28fc276540321214"},
+    ("prune", "d8-ehvi2"): {"bytes": 3151360, "sha": "669855124f47da70"},
+    ("rf", "d8-ehvi2"): {"bytes": 8809728, "sha": "669855124f47da70"},
+    ("score", "d8-ehvi2"): {"bytes": 8846848, "sha": "6549339ec963bb51"},
 }
 
 

@@ -367,21 +367,22 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
         return scoot_fail(ctx, SCOOT_EINVAL, "work buffer of %lld bytes, %lld needed", (long long)work_bytes, (long long)w.bytes);
     if ((reinterpret_cast<uintptr_t>(work) & 255u) != 0) return scoot_fail(ctx, SCOOT_EINVAL, "work is not 256-byte aligned");
     if (n == 0) return SCOOT_OK;
-    {
-        // The per-pick downdates rebuild the covariance without warping.
-        std::vector<float> scal((size_t)M * 4);
-        SCOOT_CUDA(ctx, cudaMemcpy(scal.data(), static_cast<const char*>(state) + L->off_scal,
-                                   scal.size() * sizeof(float), cudaMemcpyDeviceToHost));
-        for (int m = 0; m < M; ++m)
-            if (scal[(size_t)m * 4 + 3] != 0.0f)
-                return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "fantasy picks on a warped GP state");
-    }
 
     std::vector<HostGP> gps(M);
     for (int m = 0; m < M; ++m) {
         s = scoot_host_gp(h_space, L->d, h_x_obs, ld_obs, L->n, h_y + (size_t)m * L->n, h_lengthscale + (size_t)m * L->d,
                           h_signal_var[m], h_noise_var[m], L->kernel, &gps[m], nullptr);
         if (s != SCOOT_OK) return scoot_fail(ctx, s, "GP of objective %d could not be factored", m);
+    }
+    {
+        // The per-pick downdates rebuild the covariance without warping.  Read
+        // after the host factorisation, which overlaps the caller's queued work.
+        std::vector<float> scal((size_t)M * 4);
+        SCOOT_CUDA(ctx, cudaMemcpy(scal.data(), static_cast<const char*>(state) + L->off_scal,
+                                   scal.size() * sizeof(float), cudaMemcpyDeviceToHost));
+        for (int m = 0; m < M; ++m)
+            if (scal[(size_t)m * 4 + 3] != 0.0f)
+                return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "fantasy picks on a warped GP state");
     }
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     char* wk = static_cast<char*>(work);

@@ -11,15 +11,9 @@ constexpr int kRfThreads = 256;
 constexpr int kRfCand = 32;                      // candidates per tile (one per lane)
 constexpr int kRfGroups = kRfThreads / kRfCand;  // warps = tree groups
 
-constexpr int kMaxCols = 16;  // distinct parameters a clause set may reference (<= SCOOT_MAX_DIM)
-
 struct PruneArgs {
     int32_t n_clauses;
-    int32_t n_cols;               // distinct referenced parameters
     int32_t exact64;              // 1: every clause sum fits in int64 (sum of |coef| < 2^32)
-    int32_t col[kMaxCols];        // their parameter indices
-    uint8_t gslot[SCOOT_MAX_CLAUSES][2];  // guard -> slot in col
-    uint8_t tslot[SCOOT_MAX_CLAUSES][4];  // term -> slot in col
     scoot_clause cl[SCOOT_MAX_CLAUSES];
 };
 
@@ -37,41 +31,38 @@ __device__ __forceinline__ void add_count(unsigned long long* count, uint32_t mi
     }
 }
 
-// One thread per candidate.  The referenced parameters of the candidate are
-// loaded first, all at once (so their latencies overlap), into the thread's
-// column of a shared-memory table; then every clause is evaluated from there
-// with exact integer sums: int64 when the host has shown that no clause sum
-// can overflow it (sum of |coef| < 2^32 with 32-bit values), else int128.
+// One thread per candidate: every clause is evaluated with exact integer
+// sums, int64 when the host has shown that no clause sum can overflow it
+// (sum of |coef| < 2^32 with 32-bit values), else int128; column reads are
+// coalesced 4-byte loads (repeated columns hit L1).  One candidate per thread
+// keeps enough warps in flight to cover the load latency even for pools of a
+// few hundred thousand candidates.
 template <bool kExact64>
 __global__ void __launch_bounds__(kPruneThreads)
 prune_kernel(const __grid_constant__ PruneArgs a, const uint32_t* __restrict__ cand, int64_t n,
              int64_t ld, uint8_t* __restrict__ mask, unsigned long long* count) {
-    __shared__ int32_t sv[kMaxCols][kPruneThreads];
-    const int tid = threadIdx.x;
     uint32_t feasible = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + tid; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-#pragma unroll
-        for (int s = 0; s < kMaxCols; ++s)
-            if (s < a.n_cols) sv[s][tid] = (int32_t)__ldg(cand + (int64_t)a.col[s] * ld + i);
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         bool ok = true;
         for (int c = 0; c < a.n_clauses; ++c) {
             const scoot_clause& C = a.cl[c];
             bool g = true;
 #pragma unroll
             for (int k = 0; k < 2; ++k)
-                if (k < C.n_guard) g &= sv[a.gslot[c][k]][tid] == C.guard_value[k];
+                if (k < C.n_guard) g &= (int32_t)__ldg(cand + (int64_t)C.guard_param[k] * ld + i) == C.guard_value[k];
+            if (!g) continue;
             if (kExact64) {
                 int64_t sum = 0;
 #pragma unroll
                 for (int t = 0; t < 4; ++t)
-                    if (t < C.n_term) sum += C.coef[t] * (int64_t)sv[a.tslot[c][t]][tid];
-                ok &= !g || sum >= C.rhs;
+                    if (t < C.n_term) sum += C.coef[t] * (int64_t)(int32_t)__ldg(cand + (int64_t)C.term_param[t] * ld + i);
+                ok &= sum >= C.rhs;
             } else {
                 __int128 sum = 0;
 #pragma unroll
                 for (int t = 0; t < 4; ++t)
-                    if (t < C.n_term) sum += (__int128)C.coef[t] * sv[a.tslot[c][t]][tid];
-                ok &= !g || sum >= (__int128)C.rhs;
+                    if (t < C.n_term) sum += (__int128)C.coef[t] * (int32_t)__ldg(cand + (int64_t)C.term_param[t] * ld + i);
+                ok &= sum >= (__int128)C.rhs;
             }
         }
         mask[i] = ok;
@@ -241,22 +232,12 @@ scoot_status scoot_prune(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
         }
         a.cl[c] = C;
     }
-    // Distinct referenced parameters and the slot of every guard and term.
-    auto slot_of = [&](int param) -> int {
-        for (int k = 0; k < a.n_cols; ++k)
-            if (a.col[k] == param) return k;
-        a.col[a.n_cols] = param;
-        return a.n_cols++;
-    };
     unsigned __int128 abs_sum_max = 0;
     for (int c = 0; c < n_clauses; ++c) {
         const scoot_clause& C = h_clauses[c];
-        for (int g = 0; g < C.n_guard; ++g) a.gslot[c][g] = (uint8_t)slot_of(C.guard_param[g]);
         unsigned __int128 abs_sum = 0;
-        for (int t = 0; t < C.n_term; ++t) {
-            a.tslot[c][t] = (uint8_t)slot_of(C.term_param[t]);
+        for (int t = 0; t < C.n_term; ++t)
             abs_sum += (unsigned __int128)(C.coef[t] < 0 ? -(__int128)C.coef[t] : (__int128)C.coef[t]);
-        }
         if (abs_sum > abs_sum_max) abs_sum_max = abs_sum;
     }
     a.exact64 = abs_sum_max < ((unsigned __int128)1 << 32);

@@ -80,23 +80,10 @@ topq_pass1(const float* __restrict__ acq, const uint8_t* __restrict__ mask, int6
     for (int p = 0; p < QT; ++p) lst[p] = 0ull;
     const int64_t b0 = (int64_t)blockIdx.x * slice;
     const int64_t b1 = b0 + slice < n ? b0 + slice : n;
-    // kBatch values per thread are loaded before any of them is inserted, so
-    // their loads are in flight together.
-    constexpr int kBatch = 8;
-    for (int64_t i0 = b0 + threadIdx.x; i0 < b1; i0 += (int64_t)kBatch * blockDim.x) {
-        float v[kBatch];
-        bool ok[kBatch];
-#pragma unroll
-        for (int u = 0; u < kBatch; ++u) {
-            const int64_t i = i0 + (int64_t)u * blockDim.x;
-            ok[u] = i < b1;
-            v[u] = ok[u] ? __ldg(acq + i) : -INFINITY;
-            if (ok[u] && mask) ok[u] = __ldg(mask + i) != 0;
-        }
-#pragma unroll
-        for (int u = 0; u < kBatch; ++u)
-            if (ok[u] && !(v[u] != v[u]) && v[u] != -INFINITY)
-                insert<QT>(lst, make_key(v[u], (uint32_t)(i0 + (int64_t)u * blockDim.x)));
+    for (int64_t i = b0 + threadIdx.x; i < b1; i += blockDim.x) {
+        const float v = acq[i];
+        if ((mask == nullptr || mask[i] != 0) && !(v != v) && v != -INFINITY)
+            insert<QT>(lst, make_key(v, (uint32_t)i));
     }
     block_extract<QT>(lst, q, partial + (int64_t)blockIdx.x * q);
 }
