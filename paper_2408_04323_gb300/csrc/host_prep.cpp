@@ -24,6 +24,21 @@ int64_t align_up(int64_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 bool is_finite(double x) { return std::isfinite(x); }
 
+// sum_k a[k] b[k] for k < len, with four independent partial sums (the fp64
+// accumulation chains of the factorisation would otherwise run at FMA latency).
+double dot(const double* a, const double* b, int len) {
+    double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    int k = 0;
+    for (; k + 4 <= len; k += 4) {
+        s0 += a[k] * b[k];
+        s1 += a[k + 1] * b[k + 1];
+        s2 += a[k + 2] * b[k + 2];
+        s3 += a[k + 3] * b[k + 3];
+    }
+    for (; k < len; ++k) s0 += a[k] * b[k];
+    return (s0 + s1) + (s2 + s3);
+}
+
 double stored_value(const scoot_param& p, uint32_t w) {
     if (p.kind == SCOOT_CONTINUOUS) {
         float f;
@@ -104,7 +119,7 @@ void HostGP::kstar(const double* ux, double* k) const {
 void HostGP::solve_lower(const double* b, double* x) const {
     for (int i = 0; i < n; ++i) {
         double t = b[i];
-        for (int k = 0; k < i; ++k) t -= chol[(size_t)i * n + k] * x[k];
+        t -= dot(&chol[(size_t)i * n], x, i);
         x[i] = t / chol[(size_t)i * n + i];
     }
 }
@@ -153,15 +168,33 @@ scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, 
         if (!scoot_host_features(sp, d, x_obs, ld_obs, j, &g->u[(size_t)j * d])) return SCOOT_EINVAL;
         g->warp_features(&g->u[(size_t)j * d]);
     }
+    // K + tau^2 I from features scaled once (ordinal u / l; categorical
+    // mismatches weigh 1 / l^2): the same k(a, b) as HostGP::cov without a
+    // division per pair.
+    std::vector<double> us((size_t)n * d), icat(d, 0.0);
+    for (int c = 0; c < d; ++c)
+        if (g->cat[c]) icat[c] = 1.0 / (g->ell[c] * g->ell[c]);
+    for (int j = 0; j < n; ++j)
+        for (int c = 0; c < d; ++c)
+            us[(size_t)j * d + c] = g->cat[c] ? g->u[(size_t)j * d + c] : g->u[(size_t)j * d + c] / g->ell[c];
     std::vector<double>& K = g->chol;
     K.assign((size_t)n * n, 0.0);
-    for (int i = 0; i < n; ++i)
-        for (int j = 0; j <= i; ++j)
-            K[(size_t)i * n + j] = g->cov(&g->u[(size_t)i * d], &g->u[(size_t)j * d]) + (i == j ? g->tau2 : 0.0);
+    for (int i = 0; i < n; ++i) {
+        const double* ui = &us[(size_t)i * d];
+        for (int j = 0; j <= i; ++j) {
+            const double* uj = &us[(size_t)j * d];
+            double r2 = 0.0;
+            for (int c = 0; c < d; ++c) {
+                const double t = ui[c] - uj[c];
+                r2 += g->cat[c] ? (t != 0.0 ? icat[c] : 0.0) : t * t;
+            }
+            K[(size_t)i * n + j] = g->sf2 * matern(std::sqrt(r2), g->kernel) + (i == j ? g->tau2 : 0.0);
+        }
+    }
     double pmin = std::numeric_limits<double>::infinity(), pmax = 0.0;
     for (int j = 0; j < n; ++j) {
         double s = K[(size_t)j * n + j];
-        for (int k = 0; k < j; ++k) s -= K[(size_t)j * n + k] * K[(size_t)j * n + k];
+        s -= dot(&K[(size_t)j * n], &K[(size_t)j * n], j);
         if (!(s > 0.0) || !is_finite(s)) return SCOOT_EINVAL;
         const double piv = std::sqrt(s);
         K[(size_t)j * n + j] = piv;
@@ -169,7 +202,7 @@ scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, 
         pmax = std::max(pmax, piv);
         for (int i = j + 1; i < n; ++i) {
             double t = K[(size_t)i * n + j];
-            for (int k = 0; k < j; ++k) t -= K[(size_t)i * n + k] * K[(size_t)j * n + k];
+            t -= dot(&K[(size_t)i * n], &K[(size_t)j * n], j);
             K[(size_t)i * n + j] = t / piv;
         }
         for (int i = 0; i < j; ++i) K[(size_t)i * n + j] = 0.0;  // keep the upper triangle zero
@@ -343,7 +376,7 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
     float* scal = reinterpret_cast<float*>(blob + L->off_scal);
     float* warp_out = reinterpret_cast<float*>(blob + L->off_warp);
 
-    std::vector<double> Li((size_t)n * n), e(n), col(n);
+    std::vector<double> Li((size_t)n * n);
     HostGP g;
     for (int m = 0; m < M; ++m) {
         scoot_status s = scoot_host_gp(h_space, d, h_x_obs, ld_obs, n, h_y + (size_t)m * n,
@@ -365,12 +398,18 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
                                                            : (float)(g.u[(size_t)j * d + c] / l);
         }
         for (int i = 0; i < n; ++i) alpha_out[(size_t)m * n + i] = (float)g.alpha[i];
-        // L^{-1}: column by column, C col = e_col.
+        // L^{-1}: column by column, C col = e_col; column c is zero above row
+        // c, so its forward substitution starts there (n^3 / 6 in all).
+        // Li holds the columns contiguously: Li[c * n + i] = L^{-1}[i][c].
+        const std::vector<double>& C = g.chol;
+        std::fill(Li.begin(), Li.end(), 0.0);
         for (int c = 0; c < n; ++c) {
-            std::fill(e.begin(), e.end(), 0.0);
-            e[c] = 1.0;
-            g.solve_lower(e.data(), col.data());
-            for (int i = 0; i < n; ++i) Li[(size_t)i * n + c] = i >= c ? col[i] : 0.0;
+            double* col = &Li[(size_t)c * n];
+            col[c] = 1.0 / C[(size_t)c * n + c];
+            for (int i = c + 1; i < n; ++i) {
+                const double* Ci = &C[(size_t)i * n];
+                col[i] = -dot(Ci + c, col + c, i - c) / Ci[i];
+            }
         }
         // Tiles: row block rb covers rows [64 rb, 64 rb + 64) and column
         // chunks cj = 0 .. 2 rb + 1 of 32 columns; tile[jj][ii] = Li[row][col].
@@ -382,7 +421,7 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
                     for (int ii = 0; ii < kRowBlock; ++ii) {
                         const int row = rb * kRowBlock + ii, c = cj * kColChunk + jj;
                         float v = 0.0f;
-                        if (row < n && c <= row) v = (float)Li[(size_t)row * n + c];
+                        if (row < n && c <= row) v = (float)Li[(size_t)c * n + row];
                         tiles[((size_t)t * kColChunk + jj) * kRowBlock + ii] = v;
                     }
         // Categorical part of r^2 for every (observation, category pattern).
