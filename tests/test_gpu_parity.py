@@ -355,6 +355,40 @@ def test_score_ehvi_parity(S, ctx, name, k):
         assert np.all(np.abs(g2[fin] - g[fin]) <= 1e-6 + 1e-5 * np.abs(g[fin]))
 
 
+@pytest.mark.parametrize("name", ["d8-ehvi2", "d10-ehvi3"])
+def test_score_ehvi_bounded_boxes(S, ctx, name):
+    """Boxes bounded on the last objective take the kernel's general path
+    (the saturated form needs boxes open there): every library box is cut at
+    a finite height on that axis into two boxes covering the same region, so
+    the EHVI is unchanged."""
+    inst = make_instance(name, seeds(name)[2], n_cand=8192 + 19)
+    n = inst.n_cand
+    L, state = gp_state(S, inst)
+    lo, hi, fs = S.scoot_boxes_build(inst.y_obs, inst.ref)
+    cut = lo[:, -1] + 0.37
+    lo2 = np.concatenate([lo, lo]).copy()
+    hi2 = np.concatenate([hi, hi]).copy()
+    hi2[:len(lo), -1] = cut
+    lo2[len(lo):, -1] = cut
+    cand = cand_dev(inst)
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
+    out = []
+    for a, b in ((lo, hi), (lo2, hi2)):
+        acq = torch.empty(n, device="cuda")
+        S.scoot_score_ehvi(ctx, L, state, cand, n, dev(a), dev(b), dev(inst.eps), acq, mask)
+        out.append(np_(acq))
+    fin = np.isfinite(out[0])
+    assert np.array_equal(fin, np.isfinite(out[1]))
+    assert np.all(np.abs(out[1][fin] - out[0][fin]) <= 1e-6 + 1e-5 * np.abs(out[0][fin]))
+    live = np.nonzero(fin)[0]
+    idx = live[np.linspace(0, len(live) - 1, 48 if inst.n_obj > 2 else 181).astype(int)]
+    mu, var, e_mu, e_var = posterior_tols(oracle_gps(inst), np.ascontiguousarray(inst.cand[:, idx]))
+    front = O.pareto_front(inst.y_obs.T, inst.ref)
+    want, tol = propagated_tol(lambda a, b: O.ehvi_mc(a, b, inst.eps, front, inst.ref), mu, var, e_mu, e_var)
+    assert report_tol(f"score_ehvi bounded boxes {name} (B={2 * len(lo)})", out[1][idx], want, tol).max() <= 1.0
+
+
 def test_score_ei_parity(S, ctx):
     name = "d10-ei"
     inst = make_instance(name, seeds(name)[0])
