@@ -54,10 +54,39 @@ def mace_beta(t: int) -> float:
     return 2.0 * math.log(t * t * math.pi ** 2 / (6.0 * delta))
 
 
-class State:
-    """Per-round state prepared on the host and copied to the device."""
+class _Staging:
+    """A reused pinned host buffer for uploading a round's state in one copy.
 
-    def __init__(self, inp: RoundInputs, device: torch.device):
+    A new round may refill it only once the previous upload has left it (an
+    event recorded after each copy is waited for before the next fill)."""
+
+    def __init__(self):
+        self.buf = None
+        self.done = None
+
+    def take(self, nbytes: int) -> torch.Tensor:
+        if self.done is not None:
+            self.done.synchronize()
+        if self.buf is None or self.buf.numel() < nbytes:
+            self.buf = torch.empty(max(nbytes, 1 << 20), dtype=torch.uint8, pin_memory=True)
+        return self.buf[:nbytes]
+
+    def sent(self, stream) -> None:
+        self.done = torch.cuda.Event()
+        self.done.record(stream)
+
+
+_staging = _Staging()
+
+
+class State:
+    """Per-round state prepared on the host (the library's host functions) and
+    uploaded to the device in one copy from pinned memory; gp_state, forest,
+    box_lo, box_hi, eps, grid and corner are views into one device buffer.
+    With ``into`` (a State of the same shapes) the upload reuses that State's
+    device buffer, so work captured against it (a CUDA graph) stays valid."""
+
+    def __init__(self, inp: RoundInputs, device: torch.device, stream=None, into=None):
         d = len(inp.space)
         M = inp.y_obs.shape[0]
         self.gp_layout = S.scoot_gp_layout_init(inp.space, inp.y_obs.shape[1], M, inp.kernel)
@@ -70,22 +99,44 @@ class State:
         self.forest_layout = S.scoot_forest_layout_init(inp.nodes, inp.tree_offset, d, inp.leaf_scale)
         fblob = S.scoot_forest_pack(self.forest_layout, inp.nodes, inp.tree_offset)
         self.h_blobs = (blob, fblob)
-        self.gp_state = torch.from_numpy(blob).to(device)
-        self.forest = torch.from_numpy(fblob).to(device)
+        parts = [("gp_state", blob), ("forest", fblob)]
         self.n_boxes = 0
         self.front_size = 0
         if inp.acq in ("ehvi", "ehvi-exact"):
             lo, hi, self.front_size = S.scoot_boxes_build(inp.y_obs, inp.ref)
             self.n_boxes = len(lo)
             self.h_boxes = (lo, hi)
-            self.box_lo = torch.from_numpy(lo).to(device)
-            self.box_hi = torch.from_numpy(hi).to(device)
-            self.eps = torch.from_numpy(np.ascontiguousarray(inp.eps, np.float32)).to(device)
+            parts += [("box_lo", lo), ("box_hi", hi), ("eps", np.ascontiguousarray(inp.eps, np.float32))]
         if inp.acq == "ehvi-exact":
             grid, self.n_grid, corner = S.scoot_boxes_index(lo, hi)
             self.h_boxes = (lo, hi, grid, corner)
-            self.grid = torch.from_numpy(grid).to(device)
-            self.corner = torch.from_numpy(corner.view(np.int32)).to(device)
+            parts += [("grid", grid), ("corner", corner.view(np.int32))]
+        # one upload: 256-byte aligned slots in a pinned staging buffer
+        offs, total = [], 0
+        for _, arr in parts:
+            offs.append(total)
+            total += (arr.nbytes + 255) // 256 * 256
+        stream = torch.cuda.current_stream(device) if stream is None else stream
+        stage = _staging.take(total)
+        host = stage.numpy()
+        for (_, arr), o in zip(parts, offs):
+            host[o:o + arr.nbytes] = np.ascontiguousarray(arr).reshape(-1).view(np.uint8)
+        if into is not None and into.buffer.numel() == total and into.offsets == offs:
+            dev = into.buffer
+        else:
+            dev = torch.empty(total, dtype=torch.uint8, device=device)
+            if stream != torch.cuda.current_stream(device):
+                dev.record_stream(stream)
+        with torch.cuda.stream(stream):
+            dev.copy_(stage, non_blocking=True)
+        _staging.sent(stream)
+        self.buffer = dev
+        self.offsets = offs
+        for (name, arr), o in zip(parts, offs):
+            view = dev[o:o + arr.nbytes]
+            if arr.dtype != np.uint8:
+                view = view.view(torch.float32 if arr.dtype == np.float32 else torch.int32).reshape(arr.shape)
+            setattr(self, name, view)
 
 
 class ScoringRound:
