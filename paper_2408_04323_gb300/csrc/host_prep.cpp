@@ -8,6 +8,7 @@
 #include <cmath>
 #include <cstring>
 #include <limits>
+#include <thread>
 #include <vector>
 
 #include "internal.h"
@@ -23,6 +24,14 @@ constexpr int kMaxPatterns = 4096;        // joint category patterns of the GP's
 int64_t align_up(int64_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 bool is_finite(double x) { return std::isfinite(x); }
+
+// GP states with at least kParallelRows observations are prepared with one
+// host thread per objective, and with at least kColumnRows with
+// kColumnThreads per objective for L^{-1} (below that, starting threads costs
+// more than it saves).
+constexpr int kParallelRows = 128;
+constexpr int kColumnRows = 192;
+constexpr int kColumnThreads = 4;
 
 // sum_k a[k] b[k] for k < len, with four independent partial sums (the fp64
 // accumulation chains of the factorisation would otherwise run at FMA latency).
@@ -376,9 +385,10 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
     float* scal = reinterpret_cast<float*>(blob + L->off_scal);
     float* warp_out = reinterpret_cast<float*>(blob + L->off_warp);
 
-    std::vector<double> Li((size_t)n * n);
-    HostGP g;
-    for (int m = 0; m < M; ++m) {
+    // One objective's part of the blob; objectives write disjoint parts.
+    auto prep = [&](int m) -> scoot_status {
+        std::vector<double> Li((size_t)n * n);
+        HostGP g;
         scoot_status s = scoot_host_gp(h_space, d, h_x_obs, ld_obs, n, h_y + (size_t)m * n,
                                        h_lengthscale + (size_t)m * d, h_signal_var[m], h_noise_var[m],
                                        L->kernel, &g, h_cond ? &h_cond[m] : nullptr,
@@ -403,13 +413,26 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
         // Li holds the columns contiguously: Li[c * n + i] = L^{-1}[i][c].
         const std::vector<double>& C = g.chol;
         std::fill(Li.begin(), Li.end(), 0.0);
-        for (int c = 0; c < n; ++c) {
-            double* col = &Li[(size_t)c * n];
-            col[c] = 1.0 / C[(size_t)c * n + c];
-            for (int i = c + 1; i < n; ++i) {
-                const double* Ci = &C[(size_t)i * n];
-                col[i] = -dot(Ci + c, col + c, i - c) / Ci[i];
+        auto columns = [&](int c0, int step) {
+            for (int c = c0; c < n; c += step) {
+                double* col = &Li[(size_t)c * n];
+                col[c] = 1.0 / C[(size_t)c * n + c];
+                for (int i = c + 1; i < n; ++i) {
+                    const double* Ci = &C[(size_t)i * n];
+                    col[i] = -dot(Ci + c, col + c, i - c) / Ci[i];
+                }
             }
+        };
+        // Columns are independent: large states split them over host threads
+        // (interleaved, since column c costs ~(n - c)^2 / 2).
+        if (n >= kColumnRows) {
+            const int t = kColumnThreads;
+            std::vector<std::thread> th;
+            for (int k = 1; k < t; ++k) th.emplace_back(columns, k, t);
+            columns(0, t);
+            for (auto& x : th) x.join();
+        } else {
+            columns(0, 1);
         }
         // Tiles: row block rb covers rows [64 rb, 64 rb + 64) and column
         // chunks cj = 0 .. 2 rb + 1 of 32 columns; tile[jj][ii] = Li[row][col].
@@ -443,7 +466,20 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
         scal[m * 4 + 1] = h_noise_var[m];
         scal[m * 4 + 2] = ybest;
         scal[m * 4 + 3] = h_warp ? 1.0f : 0.0f;
+        return SCOOT_OK;
+    };
+    // Large states: objectives in parallel host threads (the work is O(n^3)
+    // per objective; small ones stay on the calling thread).
+    std::vector<scoot_status> status(M, SCOOT_OK);
+    if (M > 1 && n >= kParallelRows) {
+        std::vector<std::thread> th;
+        for (int m = 0; m < M; ++m) th.emplace_back([&, m] { status[m] = prep(m); });
+        for (auto& t : th) t.join();
+    } else {
+        for (int m = 0; m < M; ++m) status[m] = prep(m);
     }
+    for (int m = 0; m < M; ++m)
+        if (status[m] != SCOOT_OK) return status[m];
     return SCOOT_OK;
 }
 
