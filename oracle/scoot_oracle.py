@@ -638,3 +638,135 @@ def mace_select(acq3, mask, k: int, seed: int):
     order = sorted(front.tolist(), key=lambda i: (splitmix64(seed, i), i))
     picks = np.array(order[:k], np.int64)
     return picks, np.sort(front).astype(np.int64), len(picks)
+
+
+# --------------------------------------------------------------------------
+# 8. the tuning loop's sampling and threshold control (Algorithm 1, Section 4.6)
+
+def primitive_polynomials(count: int):
+    """The first ``count`` primitive polynomials over GF(2) of degree >= 1,
+    by degree, then by their middle coefficients read as a binary number.
+
+    A polynomial x^s + a_1 x^(s-1) + ... + a_(s-1) x + 1 (bit mask with bits
+    s and 0 set) is primitive when x has multiplicative order exactly
+    2^s - 1 modulo it.  Returned as (s, a) with a = a_1 ... a_(s-1) as an
+    integer (a_1 the most significant bit)."""
+    def mulmod(p, q, poly, s):
+        r = 0
+        while q:
+            if q & 1:
+                r ^= p
+            q >>= 1
+            p <<= 1
+            if p >> s & 1:
+                p ^= poly
+        return r
+
+    def order_is_full(poly, s):
+        e = (1 << s) - 1
+        # x^k mod poly by repeated multiplication; the order divides 2^s - 1
+        x = 1
+        for k in range(1, e + 1):
+            x = mulmod(x, 2, poly, s)
+            if x == 1:
+                return k == e
+        return False
+
+    out = []
+    s = 1
+    while len(out) < count:
+        for a in range(1 << (s - 1)):
+            poly = (1 << s) | (a << 1) | 1
+            if order_is_full(poly, s):
+                out.append((s, a))
+                if len(out) == count:
+                    break
+        s += 1
+    return out
+
+
+def sobol_integers(d: int, n: int, skip: int = 0) -> np.ndarray:
+    """Points skip .. skip + n - 1 of the d-dimensional Sobol sequence as
+    32-bit integers X (the point is X / 2^32), uint64 array [n][d].
+
+    Dimension 0 is the van der Corput sequence (V_k = 2^(32-k)).  Dimension
+    j >= 1 uses the j-th primitive polynomial (degree s, coefficients a_i)
+    with unit initial direction integers m_1 = ... = m_s = 1 and the
+    recurrence m_k = 2 a_1 m_(k-1) xor 4 a_2 m_(k-2) xor ... xor
+    2^(s-1) a_(s-1) m_(k-s+1) xor 2^s m_(k-s) xor m_(k-s); V_k = m_k 2^(32-k).
+    Point i is the xor of V_k over the set bits k - 1 of i."""
+    polys = primitive_polynomials(max(d - 1, 0))
+    V = np.zeros((d, 33), dtype=object)
+    for k in range(1, 33):
+        V[0, k] = 1 << (32 - k)
+    for j in range(1, d):
+        s, a = polys[j - 1]
+        m = [0] * 33
+        for k in range(1, 33):
+            if k <= s:
+                m[k] = 1
+            else:
+                v = m[k - s] ^ (m[k - s] << s)
+                for i in range(1, s):
+                    if (a >> (s - 1 - i)) & 1:
+                        v ^= m[k - i] << i
+                m[k] = v
+            V[j, k] = m[k] << (32 - k)
+    out = np.zeros((n, d), dtype=np.uint64)
+    for r in range(n):
+        i = skip + r
+        for j in range(d):
+            x, k = 0, 1
+            while i >> (k - 1):
+                if (i >> (k - 1)) & 1:
+                    x ^= V[j, k]
+                k += 1
+            out[r, j] = x
+    return out
+
+
+def sobol_configs(space, n: int, skip: int = 0) -> np.ndarray:
+    """Sobol points mapped onto the search space as stored words [d][n]
+    (Section 4.6: shortfall fill; Algorithm 1: initial design).
+
+    Reading: with u = X / 2^32 in [0, 1) per dimension, in fp64:
+    integer log-uniform: round(exp(ln lo + u (ln hi - ln lo))) clamped to
+    [lo, hi] (half to even); integer uniform: lo + floor(u (hi - lo + 1));
+    categorical: floor(u n_choices); continuous: lo + u (hi - lo), stored as
+    float32."""
+    d = len(space)
+    X = sobol_integers(d, n, skip)
+    words = np.zeros((d, n), np.uint32)
+    for j in range(d):
+        u = X[:, j].astype(np.float64) / 4294967296.0
+        p = space[j]
+        kind, lo, hi = int(p["kind"]), float(p["lo"]), float(p["hi"])
+        if kind == INT_LOG:
+            v = np.clip(np.rint(np.exp(math.log(lo) + u * (math.log(hi) - math.log(lo)))), lo, hi)
+            words[j] = v.astype(np.int64).astype(np.int32).view(np.uint32)
+        elif kind == INT_UNIFORM:
+            v = np.minimum(lo + np.floor(u * (hi - lo + 1.0)), hi)
+            words[j] = v.astype(np.int64).astype(np.int32).view(np.uint32)
+        elif kind == CATEGORICAL:
+            v = np.floor(u * int(p["n_choices"]))
+            words[j] = v.astype(np.int64).astype(np.int32).view(np.uint32)
+        else:
+            words[j] = (lo + u * (hi - lo)).astype(np.float32).view(np.uint32)
+    return words
+
+
+def delta_update(delta: float, count: int, k: int, any_invalid: bool, step: float = 0.05):
+    """Algorithm 1's feasibility-threshold controller after a batch of k
+    suggestions: an invalid result raises Delta to min(0.75, max(0.5,
+    Delta + step)) and clears the count of feasible suggestions; otherwise
+    the count grows by k and, once it reaches 5, Delta drops to
+    max(0.25, Delta - step) and the count loses 5.  Reading: the printed
+    max(0.5, .) is applied literally (an invalid result lifts Delta to at
+    least 0.5)."""
+    if any_invalid:
+        return min(0.75, max(0.5, delta + step)), 0
+    count += k
+    if count >= 5:
+        delta = max(0.25, delta - step)
+        count -= 5
+    return delta, count

@@ -708,3 +708,95 @@ def test_warped_gp_is_the_plain_gp_on_warped_features():
     k = (1 + math.sqrt(5) * r + 5 * r * r / 3) * np.exp(-math.sqrt(5) * r)
     mu, var = g1.posterior_u(uc)
     assert np.allclose(mu, k * y[0] / 1.1, rtol=1e-12) and np.allclose(var, 1 - k * k / 1.1, rtol=1e-10, atol=1e-14)
+
+
+# ------------------------------------------------------------------ Sobol sampling and the Delta controller (Algorithm 1)
+
+def _totient(m):
+    r, p, x = m, 2, m
+    while p * p <= x:
+        if x % p == 0:
+            while x % p == 0:
+                x //= p
+            r -= r // p
+        p += 1
+    if x > 1:
+        r -= r // x
+    return r
+
+
+def test_primitive_polynomials_count_and_period():
+    """There are phi(2^s - 1) / s primitive polynomials of degree s; each
+    drives a shift register through all 2^s - 1 nonzero states."""
+    polys = O.primitive_polynomials(1 + 1 + 2 + 2 + 6 + 6 + 18)
+    by_degree = {}
+    for s, a in polys:
+        by_degree.setdefault(s, []).append(a)
+    for s in range(1, 8):
+        assert len(by_degree.get(s, [])) == _totient((1 << s) - 1) // s, s
+    for s, a in polys:
+        taps = [(a >> (s - 1 - i)) & 1 for i in range(1, s)]  # a_1 .. a_(s-1)
+        state = [0] * (s - 1) + [1]
+        seen = set()
+        for _ in range((1 << s) - 1):
+            seen.add(tuple(state))
+            # x^s = a_1 x^(s-1) + ... + a_(s-1) x + 1 over GF(2): the linear recurrence of the register
+            new = state[0]
+            for i, t in enumerate(taps):
+                new ^= t & state[s - 1 - i]
+            state = state[1:] + [new]
+        assert len(seen) == (1 << s) - 1, (s, a)
+
+
+def test_sobol_first_dimension_is_van_der_corput():
+    X = O.sobol_integers(1, 300, skip=17)
+    for r in range(300):
+        i = 17 + r
+        rev = int(format(i, "032b")[::-1], 2)
+        assert int(X[r, 0]) == rev
+
+
+@pytest.mark.parametrize("m", [1, 3, 6, 8])
+def test_sobol_net_properties(m):
+    """Each dimension alone is a (0, 1)-sequence, and the first two
+    dimensions a (0, 2)-sequence: the first 2^m points fill every
+    elementary box of volume 2^-m exactly once."""
+    n = 1 << m
+    X = O.sobol_integers(6, n).astype(object)
+    for j in range(6):
+        assert sorted(int(x) >> (32 - m) for x in X[:, j]) == list(range(n))
+    for a in range(m + 1):
+        b = m - a
+        cells = {(int(x0) >> (32 - a), int(x1) >> (32 - b)) for x0, x1 in X[:, :2]}
+        assert len(cells) == n, (m, a)
+
+
+def test_sobol_skip_and_configs():
+    full = O.sobol_integers(4, 96)
+    assert np.array_equal(O.sobol_integers(4, 40, skip=56), full[56:])
+    sp = _space((INT_LOG, 0, 1, 1024), (INT_UNIFORM, 0, 3, 9), (CATEGORICAL, 4, 0, 0), (CONTINUOUS, 0, 0.5, 0.95))
+    w = O.sobol_configs(sp, 64)
+    v = w.view(np.int32)
+    assert v[0].min() >= 1 and v[0].max() <= 1024
+    assert np.array_equal(np.bincount(v[1] - 3, minlength=7)[:7] > 0, np.ones(7, bool))
+    assert v[2, :4].tolist() == [0, 2, 1, 3]     # floor(4 u) of the third dimension: 0, .5, .25, .75
+    f = w[3].view(np.float32)
+    assert f.min() >= 0.5 and f.max() < 0.95
+
+
+def test_delta_controller_trajectory():
+    """Worked by hand from Algorithm 1 with k = 2 and step 0.05."""
+    d, c = 0.5, 0
+    steps = []
+    for invalid in (False, False, False, True, False, False, False, False, False):
+        d, c = O.delta_update(d, c, 2, invalid)
+        steps.append((round(d, 10), c))
+    assert steps == [(0.5, 2), (0.5, 4), (0.45, 1), (0.5, 0), (0.5, 2), (0.5, 4), (0.45, 1), (0.45, 3), (0.4, 0)]
+    # bounds: never above 0.75 after invalid results, never below 0.25
+    d, c = 0.72, 0
+    d, c = O.delta_update(d, c, 1, True)
+    assert d == 0.75
+    d = 0.26
+    for _ in range(10):
+        d, c = O.delta_update(d, c, 5, False)
+    assert d == 0.25
