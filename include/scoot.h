@@ -15,6 +15,7 @@
  *   scoot_select_topq    top-q for parallel suggestion (Section 4.7)
  *   scoot_score_mace     posterior + UCB, PI, EI for MACE (Section 4.5)
  *   scoot_select_pareto  random k-subset of the (UCB, PI, EI) front (Section 4.7)
+ *   scoot_sobol_configs  Sobol configurations (initial design, shortfall fill)
  *
  * plus host-side preparation of per-round state (Cholesky factor of the
  * observations' covariance, box decomposition of the non-dominated region,
@@ -346,6 +347,37 @@ scoot_status scoot_score_ehvi_exact(scoot_ctx* ctx, const scoot_gp_layout* layou
  * outputs; entries beyond count are set to -1 / -inf.  1 <= q <= SCOOT_MAX_Q. */
 scoot_status scoot_select_topq(scoot_ctx* ctx, const float* acq, const uint8_t* mask, int64_t n,
                                int32_t q, int64_t* idx, float* val, int32_t* count, void* stream);
+
+/* ------------------------------------------------------------------ the tuning loop's sampling (Algorithm 1, Section 4.6) */
+
+/* Points skip .. skip + n - 1 of a d-dimensional Sobol sequence mapped onto
+ * the search space h_space and written as pool words cand [d][ld] (device):
+ * the initial design of Algorithm 1 and the shortfall fill of Section 4.6
+ * (both sample with a Sobol sequence).  Dimension 0 is the van der Corput
+ * sequence; dimension j >= 1 uses the j-th primitive polynomial over GF(2)
+ * (by degree, then by its middle coefficients as a binary number, the
+ * highest-degree one most significant) with unit initial direction
+ * integers.  With u = point / 2^32 in [0, 1), in fp64 with one rounding per
+ * operation: integer log-uniform round(exp(ln lo + u (ln hi - ln lo)))
+ * (half to even) clamped to [lo, hi]; integer uniform
+ * min(lo + floor(u (hi - lo + 1)), hi); categorical floor(u n_choices);
+ * continuous lo + u (hi - lo) rounded to float32.  skip + n <= 2^32 - 1. */
+scoot_status scoot_sobol_configs(scoot_ctx* ctx, const scoot_param* h_space, int32_t d, int64_t skip, int64_t n,
+                                 uint32_t* cand, int64_t ld, void* stream);
+
+/* The first `need` positions p < n with mask[p] != 0, in increasing order
+ * (the shortfall fill takes the first Sobol points that pass the known
+ * constraints): idx (int64 [need], -1 beyond the count), count (int32 [1]).
+ * 1 <= need <= SCOOT_MAX_Q, n < 2^31. */
+scoot_status scoot_first_feasible(scoot_ctx* ctx, const uint8_t* mask, int64_t n, int32_t need, int64_t* idx,
+                                  int32_t* count, void* stream);
+
+/* Algorithm 1's feasibility-threshold controller after k suggestions were
+ * evaluated (host): if any result was invalid, Delta becomes
+ * min(0.75, max(0.5, Delta + 0.05)) and the count of feasible suggestions
+ * is cleared; otherwise the count grows by k and, once it reaches 5, Delta
+ * becomes max(0.25, Delta - 0.05) and the count loses 5. */
+scoot_status scoot_delta_update(double* h_delta, int32_t* h_count, int32_t k, int32_t any_invalid);
 
 /* ------------------------------------------------------------------ 6. sequential fantasised picks */
 

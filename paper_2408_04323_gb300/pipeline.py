@@ -163,6 +163,7 @@ class ScoringRound:
             nbytes = S.scoot_fantasy_work_bytes(self.state.gp_layout, self.capacity, q)
             self.work = torch.empty(nbytes, dtype=torch.uint8, device=dev)
         self.picks = None
+        self.sobol_skip = 0  # next point of the Sobol sequence for shortfall fills
         self.acq3 = self.front = None
         if inp.acq == "mace":
             if inp.y_obs.shape[0] != 1:
@@ -187,6 +188,31 @@ class ScoringRound:
         if not self.inp.fantasy:
             return 7
         return 3 + 2 + 4 * self.inp.q - 1
+
+    def fill_shortfall(self, batch: int = 4096, stream=None):
+        """Section 4.6: when a round yields fewer than q suggestions, the rest
+        are Sobol points.  Reading: the first q - count points of the sequence
+        (continuing from self.sobol_skip) that satisfy the known constraints.
+        Returns host words [d][m] (m <= q - count, fewer only if a batch of
+        points holds too few feasible ones) and advances the sequence past
+        the last point used.  Synchronises with the round's count."""
+        count = int(self.top_count[0].item())
+        need = self.inp.q - count
+        if need <= 0:
+            return np.zeros((len(self.inp.space), 0), np.uint32)
+        batch = (int(batch) + 3) // 4 * 4
+        dev = self.device
+        words = torch.empty((len(self.inp.space), batch), dtype=torch.int32, device=dev)
+        mask = torch.empty(batch, dtype=torch.uint8, device=dev)
+        idx = torch.empty(need, dtype=torch.int64, device=dev)
+        cnt = torch.empty(1, dtype=torch.int32, device=dev)
+        S.scoot_sobol_configs(self.ctx, self.inp.space, self.sobol_skip, batch, words, stream)
+        S.scoot_prune(self.ctx, self.inp.space, self.inp.clauses, words, batch, mask, None, stream)
+        S.scoot_first_feasible(self.ctx, mask, batch, need, idx, cnt, stream)
+        got = int(cnt.item())
+        pos = idx[:got].cpu().numpy()
+        self.sobol_skip += int(pos[-1]) + 1 if got == need else batch
+        return words.cpu().numpy().view(np.uint32)[:, pos]
 
     def run(self, cand: torch.Tensor, n: int, stream=None):
         """prune -> rf -> score -> top-q on a resident pool cand (int32 [d][ld]).

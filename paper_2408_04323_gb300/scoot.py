@@ -92,6 +92,9 @@ _PROTOS = {
     "scoot_select_topq": [_vp, _vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
     "scoot_acq_mace": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _f32, _vp, _i64, _vp],
     "scoot_score_mace": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _f32, _f32, _vp, _i64, _vp],
+    "scoot_sobol_configs": [_vp, _vp, _i32, _i64, _i64, _vp, _i64, _vp],
+    "scoot_first_feasible": [_vp, _vp, _i64, _i32, _vp, _vp, _vp],
+    "scoot_delta_update": [C.POINTER(C.c_double), C.POINTER(_i32), _i32, _i32],
     "scoot_select_pareto": [_vp, _vp, _i64, _vp, _i64, _i32, C.c_uint64, _vp, _vp, _vp, _i64, _vp],
     "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
     "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, C.POINTER(_i64)],
@@ -435,6 +438,28 @@ def scoot_select_topq_static(acq, n, q, idx, val, count, mask=None, stream=None)
                                           int(n), int(q), _dev(idx, torch.int64, "idx"),
                                           _dev(val, torch.float32, "val"), _dev(count, torch.int32, "count"),
                                           _stream(stream)), "scoot_select_topq_static")
+
+
+def scoot_sobol_configs(ctx, h_space, skip, n, cand, stream=None):
+    """cand: int32 [d][ld] device tensor receiving Sobol points skip .. skip + n - 1."""
+    import torch
+    _check(lib().scoot_sobol_configs(_h(ctx), _host(h_space, 16, name="h_space"), len(h_space), int(skip), int(n),
+                                     _dev(cand, torch.int32, "cand"), int(cand.shape[1]), _stream(stream)),
+           "scoot_sobol_configs", _h(ctx))
+
+
+def scoot_first_feasible(ctx, mask, n, need, idx, count, stream=None):
+    import torch
+    _check(lib().scoot_first_feasible(_h(ctx), _dev(mask, torch.uint8, "mask"), int(n), int(need),
+                                      _dev(idx, torch.int64, "idx"), _dev(count, torch.int32, "count"),
+                                      _stream(stream)), "scoot_first_feasible", _h(ctx))
+
+
+def scoot_delta_update(delta: float, count: int, k: int, any_invalid: bool):
+    """Returns the new (delta, count)."""
+    d, c = C.c_double(delta), _i32(count)
+    _check(lib().scoot_delta_update(C.byref(d), C.byref(c), int(k), int(bool(any_invalid))), "scoot_delta_update")
+    return float(d.value), int(c.value)
 
 
 def scoot_fantasy_work_bytes(layout, n: int, q: int) -> int:

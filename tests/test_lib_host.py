@@ -266,3 +266,20 @@ def test_gp_prepare_warped_matches_oracle(S):
         S.scoot_gp_prepare_warped(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
                                   inst.noise_var, bad, L)
     assert e.value.status == -1
+
+
+def test_delta_controller_matches_oracle(S):
+    """Algorithm 1's threshold controller in the library against the oracle's
+    reading, over a seeded stream of batches."""
+    st = Stream(77, "delta")
+    d1 = d2 = 0.5
+    c1 = c2 = 0
+    for step in range(400):
+        k = int(st.integers(1, 8, 1)[0])
+        bad = bool(st.uniform(1)[0] < 0.3)
+        d1, c1 = S.scoot_delta_update(d1, c1, k, bad)
+        d2, c2 = O.delta_update(d2, c2, k, bad)
+        assert (d1, c1) == (pytest.approx(d2, abs=1e-12), c2), step
+        assert 0.25 <= d1 <= 0.75
+    with pytest.raises(S.ScootError):
+        S.scoot_delta_update(0.5, 0, -1, False)
