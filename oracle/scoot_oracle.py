@@ -770,3 +770,74 @@ def delta_update(delta: float, count: int, k: int, any_invalid: bool, step: floa
         delta = max(0.25, delta - step)
         count -= 5
     return delta, count
+
+
+# --------------------------------------------------------------------------
+# 9. random-forest training (Algorithm 1's TRAIN; Section 4.6)
+
+def train_cart(feats: np.ndarray, labels: np.ndarray, boot: np.ndarray, max_depth: int, leaf_scale: int):
+    """One regression tree on the bootstrap sample ``boot`` (indices into the
+    observations), grown breadth first.
+
+    feats [n][d] float32 (the stored values as floats), labels 0/1.
+    Reading (CART with squared error, as the paper's sklearn forest): a node
+    with m samples and p positives has SSE p (m - p) / m; it becomes a leaf
+    at depth max_depth, when pure, or when no split separates its samples;
+    otherwise it takes the split "x_f <= v" (v a sample value of feature f,
+    not the node's largest) with the smallest SSE(left) + SSE(right),
+    compared exactly as fractions, ties to the lower f, then the lower v.
+    A leaf stores round(leaf_scale p / m) (halves up) votes.  Nodes are
+    numbered breadth first, so the children of a node are adjacent and
+    follow it.  Returns a list of (val, left, feat, is_leaf), left counted
+    from the tree's first node."""
+    feats = np.asarray(feats, np.float32)
+    labels = np.asarray(labels).astype(np.int64)
+    nodes = []
+    queue = [(list(int(i) for i in boot), 0)]
+    head = 0
+    while head < len(queue):
+        samp, depth = queue[head]
+        head += 1
+        m = len(samp)
+        p = int(sum(labels[i] for i in samp))
+        best = None
+        if depth < max_depth and 0 < p < m:
+            for f in range(feats.shape[1]):
+                vals = sorted({float(feats[i, f]) for i in samp})
+                for v in vals[:-1]:
+                    left = [i for i in samp if float(feats[i, f]) <= v]
+                    nl, pl = len(left), int(sum(labels[i] for i in left))
+                    nr, pr = m - nl, p - pl
+                    # SSE(left) + SSE(right) = num / (nl nr)
+                    num = pl * (nl - pl) * nr + pr * (nr - pr) * nl
+                    den = nl * nr
+                    key = (num, den)
+                    if best is None or num * best[1] < best[0] * den:
+                        best = (num, den, f, v)
+        if best is None:
+            votes = (2 * leaf_scale * p + m) // (2 * m)
+            nodes.append([float(votes), 0, 0, True])
+            continue
+        _, _, f, v = best
+        left = [i for i in samp if float(feats[i, f]) <= v]
+        right = [i for i in samp if float(feats[i, f]) > v]
+        child = len(queue)
+        queue.append((left, depth + 1))
+        queue.append((right, depth + 1))
+        nodes.append([v, child, f, False])
+    return [tuple(x) for x in nodes]
+
+
+def train_forest(feats, labels, boot: np.ndarray, max_depth: int, leaf_scale: int):
+    """Trees on the bootstrap samples boot [T][n] as (nodes structured array
+    with fields val, left, feat, flags, and tree offsets [T + 1])."""
+    trees = [train_cart(feats, labels, b, max_depth, leaf_scale) for b in boot]
+    offs = np.zeros(len(trees) + 1, np.int32)
+    offs[1:] = np.cumsum([len(t) for t in trees])
+    out = np.zeros(offs[-1], dtype=[("val", "<f4"), ("left", "<u2"), ("feat", "u1"), ("flags", "u1")])
+    k = 0
+    for t in trees:
+        for val, left, f, leaf in t:
+            out[k] = (val, left, f, 1 if leaf else 0)
+            k += 1
+    return out, offs

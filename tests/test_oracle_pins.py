@@ -800,3 +800,56 @@ def test_delta_controller_trajectory():
     for _ in range(10):
         d, c = O.delta_update(d, c, 5, False)
     assert d == 0.25
+
+
+# ------------------------------------------------------------------ forest training (Algorithm 1, Section 4.6)
+
+def test_cart_hand_worked(golden_dir):
+    lines = [l.split() for l in open(os.path.join(golden_dir, "cart_hand.txt")) if not l.startswith("#")]
+    s = [float(v) for v in lines[0][1:]]
+    X = np.array([s[i:i + 2] for i in range(0, len(s), 3)], np.float32)
+    y = np.array(s[2::3], np.int64)
+    want = [(float(a), int(b), int(c), bool(int(d))) for _, a, b, c, d in lines[1:]]
+    assert O.train_cart(X, y, np.arange(len(y)), 4, 255) == want
+
+
+def _split_sse_brute(X, y, samp, f, v):
+    left = [i for i in samp if X[i, f] <= v]
+    right = [i for i in samp if X[i, f] > v]
+    sse = lambda g: sum((y[i] - np.mean([y[j] for j in g])) ** 2 for i in g) if g else 0.0
+    return sse(left) + sse(right)
+
+
+def test_cart_splits_are_optimal_and_leaves_round():
+    """Every split minimises the summed squared error over all splits of its
+    node's samples (brute force with floating means); leaves hold
+    round(V p / m); the tree ignores the order of the bootstrap list; grown
+    to purity without bootstrap it reproduces its labels."""
+    st = Stream(91, "cart")
+    n, d = 60, 4
+    X = np.floor(st.uniform(n * d).reshape(n, d) * 7).astype(np.float32)
+    y = (st.uniform(n) < 0.4).astype(np.int64)
+    boot = st.integers(0, n - 1, n)
+    tree = O.train_cart(X, y, boot, 5, 255)
+    # walk the tree again, node by node, to recover each node's samples
+    node_samples = {0: list(boot)}
+    for k, (val, left, f, leaf) in enumerate(tree):
+        samp = node_samples[k]
+        if leaf:
+            p, m = sum(y[i] for i in samp), len(samp)
+            assert val == math.floor(255 * p / m + 0.5)
+            continue
+        got = _split_sse_brute(X, y, samp, f, val)
+        for g in range(d):
+            for v in sorted(set(X[samp, g]))[:-1]:
+                assert got <= _split_sse_brute(X, y, samp, g, v) + 1e-9
+        node_samples[left] = [i for i in samp if X[i, f] <= val]
+        node_samples[left + 1] = [i for i in samp if X[i, f] > val]
+    assert O.train_cart(X, y, boot[::-1], 5, 255) == tree
+    Xp = (X + np.arange(n, dtype=np.float32)[:, None] * np.float32(0.001)).astype(np.float32)
+    full = O.train_cart(Xp, y, np.arange(n), 64, 1)
+    for i in range(n):
+        k = 0
+        while not full[k][3]:
+            k = full[k][1] + (0 if Xp[i, full[k][2]] <= full[k][0] else 1)
+        assert full[k][0] == y[i]
