@@ -785,8 +785,8 @@ def train_cart(feats: np.ndarray, labels: np.ndarray, boot: np.ndarray, max_dept
     at depth max_depth, when pure, or when no split separates its samples;
     otherwise it takes the split "x_f <= v" (v a sample value of feature f,
     not the node's largest) with the smallest SSE(left) + SSE(right),
-    compared exactly as fractions, ties to the lower f, then the lower v.
-    A leaf stores round(leaf_scale p / m) (halves up) votes.  Nodes are
+    compared exactly as fractions, ties to the lower f, then the lower v
+    (-0 and +0 count as one value, stored as +0).  A leaf stores round(leaf_scale p / m) (halves up) votes.  Nodes are
     numbered breadth first, so the children of a node are adjacent and
     follow it.  Returns a list of (val, left, feat, is_leaf), left counted
     from the tree's first node."""
@@ -824,7 +824,9 @@ def train_cart(feats: np.ndarray, labels: np.ndarray, boot: np.ndarray, max_dept
         child = len(queue)
         queue.append((left, depth + 1))
         queue.append((right, depth + 1))
-        nodes.append([v, child, f, False])
+        # -0 and +0 are one value ("x <= v" cannot tell them apart); the
+        # threshold is stored as +0.
+        nodes.append([0.0 if v == 0.0 else v, child, f, False])
     return [tuple(x) for x in nodes]
 
 

@@ -853,3 +853,17 @@ def test_cart_splits_are_optimal_and_leaves_round():
         while not full[k][3]:
             k = full[k][1] + (0 if Xp[i, full[k][2]] <= full[k][0] else 1)
         assert full[k][0] == y[i]
+
+
+def test_cart_signed_zero_is_one_value():
+    """-0 and +0 are one feature value (x <= v cannot separate them): they
+    form one candidate and the threshold is stored as +0, whichever of the
+    two the samples carry; the split matches the one with +0 everywhere."""
+    X = np.array([[-1.0], [-0.0], [0.0], [-0.0], [2.0]], np.float32)
+    y = np.array([0, 0, 1, 1, 1])
+    tree = O.train_cart(X, y, np.arange(5), 4, 255)
+    Xp = X + np.float32(0.0)  # -0 + 0 = +0; the other values unchanged
+    assert np.signbit(X).sum() == 3 and np.signbit(Xp).sum() == 1
+    assert tree == O.train_cart(Xp, y, np.arange(5), 4, 255)
+    zeros = [t for t in tree if not t[3] and t[0] == 0.0]
+    assert zeros and all(math.copysign(1.0, t[0]) == 1.0 for t in zeros)
