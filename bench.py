@@ -71,6 +71,8 @@ def parse_args():
     p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--stage", choices=["round", "rf-train"], default="round",
+                   help="rf-train: time the training of the workload's feasibility forest instead of a round")
     return p.parse_args()
 
 
@@ -247,8 +249,214 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+RF_METRIC = "CART trees trained/sec (Algorithm 1's feasibility forest, exact split search)"
+RF_UNIT = "trees/s"
+
+
+def rf_train_inputs(name):
+    """Observations, crash labels and T bootstrap samples of n draws of a workload."""
+    import numpy as np
+    from workloads import Stream, make_instance, seeds
+    seed = seeds(name)[0]
+    inst = make_instance(name, seed, n_cand=4)
+    w = inst.workload
+    n = w.n_obs
+    labels = (inst.label_obs > 0.5).astype(np.uint8)
+    boot = Stream(seed, "bootstrap").integers(0, n - 1, w.n_trees * n).reshape(w.n_trees, n).astype(np.int32)
+    return inst, labels, boot
+
+
+def rf_train_config(w, extra=None):
+    cfg = {"workload": f"{w.name} forest: {w.n_trees} CART trees on bootstraps of n={w.n_obs} observations, "
+                       f"d={w.d}, depth<={w.max_depth}",
+           "trees": w.n_trees, "observations": w.n_obs, "max_depth": w.max_depth,
+           "l2": "flushed between steps (256 MiB write)", "inputs": "seeded synthetic observations, resident in HBM"}
+    cfg.update(extra or {})
+    return cfg
+
+
+def rf_oracle_seconds(name, trees):
+    """The oracle's CART on the first `trees` bootstraps, in a fresh one-thread process."""
+    code = ("import sys, time, json; sys.path.insert(0, %r)\n"
+            "import numpy as np, oracle, bench\n"
+            "inst, labels, boot = bench.rf_train_inputs(%r)\n"
+            "w = inst.workload\n"
+            "feats = oracle.decode(inst.space, inst.x_obs, w.n_obs).astype(np.float32)\n"
+            "t = time.perf_counter()\n"
+            "oracle.train_forest(feats, labels, boot[:%d], w.max_depth, w.leaf_scale)\n"
+            "print(json.dumps({'seconds': time.perf_counter() - t}))\n" % (ROOT, name, trees))
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    if p.returncode != 0:
+        raise RuntimeError(p.stderr[-2000:])
+    return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
+
+
+def rf_oracle_sample(name, budget_s, n_trees):
+    t1 = rf_oracle_seconds(name, 1)
+    k = int(min(n_trees, max(1, budget_s / max(t1, 1e-3))))
+    return k, (rf_oracle_seconds(name, k) if k > 1 else t1)
+
+
+def rf_list_entries(S, nodes, counts, feats, labels, boot, max_depth):
+    """List entries the presorted split search touches on the trained trees:
+    every node that searches (depth < max_depth, not pure) scans its m'
+    samples in each of the d sorted lists, and every split node moves them
+    into its children's lists."""
+    import numpy as np
+    recs = nodes.view(S.NODE_DTYPE)
+    d = feats.shape[1]
+    total = 0
+    for t in range(len(counts)):
+        tree = recs[t, :int(counts[t])]
+        node = np.zeros(boot.shape[1], np.int64)
+        depth = np.zeros(len(tree), np.int64)
+        for k in range(len(tree)):
+            sel = boot[t][node == k]
+            mk, pk = len(sel), int(labels[sel].sum())
+            if depth[k] < max_depth and 0 < pk < mk:
+                total += d * mk
+            if not (tree["flags"][k] & 1):
+                total += d * mk
+                left = int(tree["left"][k])
+                depth[left] = depth[left + 1] = depth[k] + 1
+                here = node == k
+                go = feats[boot[t], int(tree["feat"][k])] <= tree["val"][k]
+                node[here & go] = left
+                node[here & ~go] = left + 1
+    return total
+
+
+def run_rf_train(args):
+    import numpy as np
+    import torch
+    import paper_2408_04323_gb300 as pkg
+    pkg.build()
+    from paper_2408_04323_gb300 import scoot as S
+    from workloads import CONTINUOUS, WORKLOADS
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1:
+        raise SystemExit("--stage rf-train runs on one GPU")
+    w = WORKLOADS[args.workload]
+    inst, labels_np, boot_np = rf_train_inputs(w.name)
+    n, T, d = w.n_obs, w.n_trees, w.d
+    device = torch.device("cuda", 0)
+    ctx = S.Context(0)
+    h_obs = torch.from_numpy(np.ascontiguousarray(inst.x_obs[:, :n]).view(np.int32)).pin_memory()
+    h_lab = torch.from_numpy(labels_np).pin_memory()
+    h_boot = torch.from_numpy(boot_np).pin_memory()
+    obs, lab, boot = h_obs.to(device), h_lab.to(device), h_boot.to(device)
+    nodes = torch.zeros((T, 2 * n - 1), dtype=torch.int64, device=device)
+    counts = torch.zeros(T, dtype=torch.int32, device=device)
+    h_nodes = torch.empty(nodes.shape, dtype=torch.int64, pin_memory=True)
+    h_counts = torch.empty(counts.shape, dtype=torch.int32, pin_memory=True)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
+    stream = torch.cuda.current_stream(device)
+
+    def train(o=obs, la=lab, b=boot):
+        S.scoot_rf_train(ctx, inst.space, o, n, la, b, w.max_depth, w.leaf_scale, nodes, counts, stream)
+
+    sampler = ClockSampler()
+    sampler.start()
+    t_end = time.perf_counter() + args.warmup_seconds
+    k = 0
+    while k < max(3, args.warmup) or time.perf_counter() < t_end:
+        flush.fill_(k & 0xFF)
+        train()
+        k += 1
+    torch.cuda.synchronize(device)
+    ctx.check(stream)
+    tev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    for kk in range(args.steps):
+        flush.fill_(kk & 0xFF)
+        tev[kk][0].record(stream)
+        train()
+        tev[kk][1].record(stream)
+    torch.cuda.synchronize(device)
+    clocks = sampler.stop()
+    ctx.check(stream)
+    ms = statistics.mean(e[0].elapsed_time(e[1]) for e in tev)
+
+    # end to end: inputs from pinned host memory, trees read back
+    e2e = None
+    if not args.no_e2e:
+        d_obs, d_lab, d_boot = torch.empty_like(obs), torch.empty_like(lab), torch.empty_like(boot)
+        times = []
+        for kk in range(args.warmup + args.steps):
+            flush.fill_(kk & 0xFF)
+            torch.cuda.synchronize(device)
+            t0 = time.perf_counter()
+            d_obs.copy_(h_obs, non_blocking=True)
+            d_lab.copy_(h_lab, non_blocking=True)
+            d_boot.copy_(h_boot, non_blocking=True)
+            train(d_obs, d_lab, d_boot)
+            h_nodes.copy_(nodes, non_blocking=True)
+            h_counts.copy_(counts, non_blocking=True)
+            torch.cuda.synchronize(device)
+            if kk >= args.warmup:
+                times.append(time.perf_counter() - t0)
+        e2e_s = statistics.mean(times)
+        e2e = {"value": T / e2e_s, "unit": RF_UNIT,
+               "h2d_bytes_per_step": int(h_obs.numel() * 4 + h_lab.numel() + h_boot.numel() * 4),
+               "d2h_bytes_per_step": int(h_nodes.numel() * 8 + h_counts.numel() * 4), "ms_per_step": 1e3 * e2e_s}
+
+    # roofline: one list entry per FP32/INT32 lane per clock
+    peaks, peak_src = measured_peaks()
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    lane_peak = sms * FP32_LANES_PER_SM * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # Tops/s
+    h_nodes.copy_(nodes)
+    h_counts.copy_(counts)
+    feats = np.stack([inst.x_obs[j, :n].view(np.float32) if int(inst.space[j]["kind"]) == CONTINUOUS
+                      else inst.x_obs[j, :n].view(np.int32).astype(np.float32) for j in range(d)], axis=1)
+    entries = rf_list_entries(S, h_nodes.numpy(), h_counts.numpy(), feats, labels_np, boot_np, w.max_depth)
+    achieved = entries / (ms / 1e3) / 1e12
+    roof = {"bound": "alu", "achieved": achieved, "peak": lane_peak, "unit": "Tentries/s",
+            "frac": achieved / lane_peak, "traffic": None, "kernel": "rf_train",
+            "peak_source": f"{peak_src} SM clock; one sorted-list entry per lane per clock = SMs x 128 x max SM "
+                           "clock (the kernel is bound by the latency of its breadth-first node sequence)",
+            "work_per_unit": entries / T, "units_per_launch": T}
+    cpu = None
+    if not args.no_cpu_baseline:
+        k_, secs = rf_oracle_sample(w.name, args.cpu_seconds, T)
+        cpu = {"value": k_ / secs, "unit": RF_UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"the first {k_} of the {T} trees, pure-Python breadth-first CART, one thread"}
+    line = {"metric": RF_METRIC, "value": T / (ms / 1e3), "unit": RF_UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+            "config": rf_train_config(w, {"nodes": int(h_counts.sum()),
+                                          "launch": "feature ranks, then one block per tree"}),
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * args.steps, "clocks": clocks}
+    print(json.dumps(line), flush=True)
+    ctx.close()
+
+
+def run_rf_reference(args):
+    from workloads import WORKLOADS
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    w = WORKLOADS[args.workload]
+    per_step = max(0.5, 120.0 / max(1, args.steps + args.warmup))
+    k, _ = rf_oracle_sample(w.name, per_step, w.n_trees)
+    for _ in range(args.warmup):
+        rf_oracle_seconds(w.name, k)
+    times = [rf_oracle_seconds(w.name, k) for _ in range(args.steps)]
+    ms = 1e3 * statistics.mean(times)
+    value = k / (ms / 1e3)
+    line = {"impl": "reference", "metric": RF_METRIC, "value": value, "unit": RF_UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": rf_train_config(w, {"reference": "CPU oracle (the paper ships no code)",
+                                          "trees_per_step": k}),
+            "cpu_baseline": {"value": value, "unit": RF_UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"the first {k} of the {w.n_trees} trees per step"},
+            "e2e": {"value": value, "unit": RF_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
+    if args.stage == "rf-train":
+        (run_rf_reference if args.impl == "reference" else run_rf_train)(args)
+        return
     if args.impl == "reference":
         run_reference(args)
         return

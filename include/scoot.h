@@ -16,6 +16,7 @@
  *   scoot_score_mace     posterior + UCB, PI, EI for MACE (Section 4.5)
  *   scoot_select_pareto  random k-subset of the (UCB, PI, EI) front (Section 4.7)
  *   scoot_sobol_configs  Sobol configurations (initial design, shortfall fill)
+ *   scoot_rf_train       CART training of the feasibility forest (Algorithm 1)
  *
  * plus host-side preparation of per-round state (Cholesky factor of the
  * observations' covariance, box decomposition of the non-dominated region,
@@ -126,7 +127,8 @@ const char* scoot_status_string(scoot_status s);
 /* Wait for `stream`, then read and clear the context's device error word:
  * SCOOT_EDEVICE if a kernel flagged a bad index or value since the last
  * check, SCOOT_ETIMEOUT if a bounded wait gave up, SCOOT_EUNSUPPORTED if a
- * Pareto filter ran out of survivor capacity, else SCOOT_OK. */
+ * Pareto filter ran out of survivor capacity, SCOOT_EINVAL if a kernel met a
+ * non-finite input it had to validate, else SCOOT_OK. */
 scoot_status scoot_ctx_check(scoot_ctx* ctx, void* stream);
 /* Bytes of device workspace the context currently holds. */
 scoot_status scoot_ctx_workspace_bytes(const scoot_ctx* ctx, int64_t* bytes);
@@ -378,6 +380,41 @@ scoot_status scoot_first_feasible(scoot_ctx* ctx, const uint8_t* mask, int64_t n
  * is cleared; otherwise the count grows by k and, once it reaches 5, Delta
  * becomes max(0.25, Delta - 0.05) and the count loses 5. */
 scoot_status scoot_delta_update(double* h_delta, int32_t* h_count, int32_t k, int32_t any_invalid);
+
+#define SCOOT_RF_TRAIN_MAX_OBS 1024  /* observations and bootstrap size per tree */
+
+/* Train the feasibility forest of Algorithm 1 (random forest regression of
+ * the crash labels, Section 4.6): tree t is a CART regression tree on the
+ * bootstrap sample boot[t * m + k], k < m (indices into the n observations;
+ * int32, device).  obs holds the observations as pool words [d][ld]
+ * (device; the features are their stored values as floats, as scoot_node's
+ * x[feat]); labels (uint8 [n], device) are 1 for a feasible observation, 0
+ * for a crash.
+ * Growth is breadth first.  A node of m' samples with p positives becomes a
+ * leaf at depth max_depth (the root has depth 0), when p is 0 or m', or when
+ * all its samples share every feature value; a leaf stores
+ * floor((2 leaf_scale p + m') / (2 m')) votes (leaf_scale p / m' rounded half
+ * up).  Otherwise the node splits on "x[f] <= v", v one of its samples'
+ * values of feature f other than the largest, minimising the squared error
+ * of the two children p_l (m_l - p_l) / m_l + p_r (m_r - p_r) / m_r, compared
+ * exactly; ties go to the lower f, then the lower v (-0 and +0 are one
+ * value; a zero threshold is stored as +0).  The two children of a node are
+ * numbered next to each other in breadth-first order.  Uses the context's
+ * workspace (feature ranks of the observations, 2 d n bytes).
+ * Output: nodes (scoot_node [n_trees][node_cap], device), tree t in
+ * nodes[t * node_cap ...] with child indices counted from its first node,
+ * n_nodes (int32 [n_trees], device) its node count (<= 2 m - 1, so node_cap
+ * >= 2 m - 1 is required).  Pass the compacted nodes to
+ * scoot_forest_layout_init.  1 <= n, m <= SCOOT_RF_TRAIN_MAX_OBS, 1 <= d <=
+ * SCOOT_MAX_DIM, 0 <= max_depth <= 255, 1 <= leaf_scale <= 2^24.  A
+ * bootstrap index outside 0..n-1 (SCOOT_EDEVICE from scoot_ctx_check), or a
+ * drawn observation with a non-finite feature or a label other than 0/1
+ * (SCOOT_EINVAL from scoot_ctx_check), leaves that tree empty
+ * (n_nodes[t] = 0). */
+scoot_status scoot_rf_train(scoot_ctx* ctx, const scoot_param* h_space, int32_t d, const uint32_t* obs, int32_t n,
+                            int64_t ld, const uint8_t* labels, const int32_t* boot, int32_t n_trees, int32_t m,
+                            int32_t max_depth, int32_t leaf_scale, scoot_node* nodes, int32_t node_cap,
+                            int32_t* n_nodes, void* stream);
 
 /* ------------------------------------------------------------------ 6. sequential fantasised picks */
 

@@ -105,6 +105,8 @@ scoot_status scoot_ctx_check(scoot_ctx* ctx, void* stream) {
     if (word) SCOOT_CUDA(ctx, cudaMemsetAsync(ctx->d_err, 0, sizeof(uint32_t), st));
     if (word & SCOOT_DEVERR_TIMEOUT) return scoot_fail(ctx, SCOOT_ETIMEOUT, "a bounded device wait gave up");
     if (word & SCOOT_DEVERR_INDEX) return scoot_fail(ctx, SCOOT_EDEVICE, "a kernel met an index out of range");
+    if (word & SCOOT_DEVERR_VALUE)
+        return scoot_fail(ctx, SCOOT_EINVAL, "a kernel met a non-finite feature or a label other than 0/1");
     if (word & SCOOT_DEVERR_CAPACITY)
         return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "more than %d candidates survived the pivots of a Pareto filter",
                           SCOOT_PARETO_CAP);

@@ -17,6 +17,7 @@
 #define SCOOT_DEVERR_INDEX   1u   // a node, feature or box index out of range
 #define SCOOT_DEVERR_TIMEOUT 2u   // a bounded wait gave up
 #define SCOOT_DEVERR_CAPACITY 4u  // a Pareto filter had more survivors than it can hold
+#define SCOOT_DEVERR_VALUE   8u   // a non-finite feature or a label other than 0/1
 
 struct scoot_ctx {
     int32_t device = 0;

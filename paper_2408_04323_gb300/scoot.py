@@ -60,6 +60,9 @@ class scoot_gp_layout(C.Structure):
                 ("off_cat", C.c_int64), ("off_warp", C.c_int64)]
 
 
+# scoot_node as a numpy record (host copies of trained trees)
+NODE_DTYPE = np.dtype([("val", "<f4"), ("left", "<u2"), ("feat", "u1"), ("flags", "u1")])
+
 assert C.sizeof(scoot_param) == 16 and C.sizeof(scoot_clause) == 80 and C.sizeof(scoot_node) == 8
 
 _vp, _i32, _i64, _u32, _f32 = C.c_void_p, C.c_int32, C.c_int64, C.c_uint32, C.c_float
@@ -95,6 +98,7 @@ _PROTOS = {
     "scoot_sobol_configs": [_vp, _vp, _i32, _i64, _i64, _vp, _i64, _vp],
     "scoot_first_feasible": [_vp, _vp, _i64, _i32, _vp, _vp, _vp],
     "scoot_delta_update": [C.POINTER(C.c_double), C.POINTER(_i32), _i32, _i32],
+    "scoot_rf_train": [_vp, _vp, _i32, _vp, _i32, _i64, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _i32, _vp, _vp],
     "scoot_select_pareto": [_vp, _vp, _i64, _vp, _i64, _i32, C.c_uint64, _vp, _vp, _vp, _i64, _vp],
     "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
     "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, C.POINTER(_i64)],
@@ -460,6 +464,30 @@ def scoot_delta_update(delta: float, count: int, k: int, any_invalid: bool):
     d, c = C.c_double(delta), _i32(count)
     _check(lib().scoot_delta_update(C.byref(d), C.byref(c), int(k), int(bool(any_invalid))), "scoot_delta_update")
     return float(d.value), int(c.value)
+
+
+def scoot_rf_train(ctx, h_space, obs, n, labels, boot, max_depth, leaf_scale, nodes, n_nodes, stream=None):
+    """obs: int32 [d][ld] observation words; labels: uint8 [n]; boot: int32
+    [T][m]; nodes: int64 [T][node_cap] receiving scoot_node records (view the
+    host copy as the node dtype); n_nodes: int32 [T]."""
+    import torch
+    T, m = (int(boot.shape[0]), int(boot.shape[1])) if boot.dim() == 2 else (0, 1)
+    _check(lib().scoot_rf_train(_h(ctx), _host(h_space, 16, name="h_space"), len(h_space),
+                                _dev(obs, torch.int32, "obs"), int(n), int(obs.shape[1]),
+                                _dev(labels, torch.uint8, "labels"), _dev(boot, torch.int32, "boot"), T, m,
+                                int(max_depth), int(leaf_scale), _dev(nodes, torch.int64, "nodes"),
+                                int(nodes.shape[1]), _dev(n_nodes, torch.int32, "n_nodes"), _stream(stream)),
+           "scoot_rf_train", _h(ctx))
+
+
+def compact_forest(nodes: np.ndarray, n_nodes: np.ndarray):
+    """Host copy of scoot_rf_train's output (int64 [T][node_cap], int32 [T])
+    -> (scoot_node records of all trees back to back, tree offsets [T + 1])."""
+    recs = np.ascontiguousarray(nodes).view(NODE_DTYPE)
+    offs = np.zeros(len(n_nodes) + 1, np.int32)
+    offs[1:] = np.cumsum(n_nodes)
+    out = np.concatenate([recs[t, :int(c)] for t, c in enumerate(n_nodes)]) if len(n_nodes) else recs[:0, 0]
+    return out, offs
 
 
 def scoot_fantasy_work_bytes(layout, n: int, q: int) -> int:
