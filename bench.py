@@ -71,6 +71,8 @@ def parse_args():
     p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--gp-prep", choices=["host", "device"], default="host",
+                   help="where the end-to-end step builds the GP state (fp64 factorisation)")
     p.add_argument("--stage", choices=["round", "rf-train"], default="round",
                    help="rf-train: time the training of the workload's feasibility forest instead of a round")
     return p.parse_args()
@@ -352,8 +354,10 @@ def run_rf_train(args):
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
     stream = torch.cuda.current_stream(device)
 
+    work = torch.empty(S.scoot_rf_train_work_bytes(n, d), dtype=torch.uint8, device=device)
+
     def train(o=obs, la=lab, b=boot):
-        S.scoot_rf_train(ctx, inst.space, o, n, la, b, w.max_depth, w.leaf_scale, nodes, counts, stream)
+        S.scoot_rf_train(ctx, inst.space, o, n, la, b, w.max_depth, w.leaf_scale, nodes, counts, work, stream)
 
     sampler = ClockSampler()
     sampler.start()
@@ -503,7 +507,8 @@ def main():
     if args.warp and w.fantasy:
         raise SystemExit("--warp: fantasy picks take unwarped GP states")
     ctx = S.Context(device.index)
-    rnd = ScoringRound(ctx, inp, N, device)
+    gp_dev = args.gp_prep == "device" and not inp.fantasy
+    rnd = ScoringRound(ctx, inp, N, device, gp_on_device=gp_dev)
     cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
     stream = torch.cuda.current_stream(device)
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
@@ -675,7 +680,7 @@ def main():
                 (cand if graph is not None else cand_e2e).copy_(host_pool, non_blocking=True)
             # host preparation through the C ABI + one upload (into the captured
             # step's state buffer when the step is replayed as a graph)
-            state = State(inp, device, into=st if graph is not None else None)
+            state = State(inp, device, into=st if graph is not None else None, gp_on_device=gp_dev, ctx=ctx)
             stream.wait_stream(copy_stream)
             if graph is not None:
                 graph.replay()
@@ -721,9 +726,7 @@ def main():
             torch.cuda.synchronize(device)
             if kk >= args.warmup:
                 times.append(time.perf_counter() - t0)
-        state_bytes = sum(b.nbytes for b in state.h_blobs)
-        if inp.acq in ("ehvi", "ehvi-exact"):
-            state_bytes += sum(b.nbytes for b in state.h_boxes) + inp.eps.nbytes
+        state_bytes = sum(b.nbytes for b in state.h_blobs)  # everything uploaded (GP inputs or state, forest, boxes)
         e2e_s = statistics.mean(times)
         if dist:
             t = torch.tensor([e2e_s], device=device)
@@ -752,7 +755,9 @@ def main():
                                               "launch": "CUDA graph of the step" if graph is not None
                                               else "eager launches",
                                               "eager_ms_per_step": round(eager_ms, 5),
-                                              "kernel": args.kernel, "warp": bool(args.warp)}, acq=inp.acq),
+                                              "kernel": args.kernel, "warp": bool(args.warp),
+                                              "e2e_gp_state": "built on the device" if gp_dev else
+                                              "built on the host"}, acq=inp.acq),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps * rnd.kernels_per_round(),
                 "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},

@@ -7,6 +7,7 @@
  *   scoot_prune          known constraints, Eq. (2)
  *   scoot_rf_predict     random-forest probability of feasibility, Eq. (3)
  *   scoot_gp_posterior   GP posterior mean and variance (Section 4.3)
+ *   scoot_gp_prepare_device  the GP state (fp64 factorisation) on the device
  *   scoot_acq_ei         expected improvement, Eq. (6)
  *   scoot_acq_ehvi       Monte-Carlo expected hypervolume improvement, Eq. (7)
  *   scoot_score_ei       posterior + EI in one kernel
@@ -74,7 +75,9 @@ typedef int32_t scoot_status;
 #define SCOOT_MAX_DIM      16   /* parameters per configuration */
 #define SCOOT_MAX_CLAUSES  16   /* known-constraint clauses per call */
 #define SCOOT_MAX_OBJ       4   /* objectives */
-#define SCOOT_MAX_OBS    1024   /* observed configurations */
+#define SCOOT_MAX_OBS     640   /* observed configurations: the posterior kernels hold a
+                                      64-candidate tile's covariance rows (n x 64 fp32) and the
+                                      observations in shared memory (227 KB) */
 #define SCOOT_MAX_Q        64   /* picks per top-q call */
 
 /* One parameter: kind, number of categories (categorical only) and the
@@ -251,6 +254,29 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
                                      const float* h_warp, const scoot_gp_layout* layout, void* h_blob,
                                      double* h_cond);
 
+/* Bytes of device scratch scoot_gp_prepare_device needs for a layout:
+ * 8 M (n d + n (n + 1) / 2), and another 8 M n (n + 1) / 2 when n > 160. */
+scoot_status scoot_gp_device_work_bytes(const scoot_gp_layout* layout, int64_t* bytes);
+
+/* scoot_gp_prepare (h_warp NULL) or scoot_gp_prepare_warped on the device,
+ * into a device blob of the same layout, asynchronously on `stream`: the
+ * features, K + tau^2 I and its Cholesky factorisation in fp64, L^{-1} formed
+ * by applying the factorisation's elimination to the identity, alpha, and
+ * the same fp32 tables.  Device inputs: obs (words [d][ld_obs]), y [M][n],
+ * lengthscale [M][d], signal_var [M], noise_var [M], warp [M][d][2] or NULL
+ * (the conventions of scoot_gp_prepare_warped); blob (layout->bytes,
+ * 16-byte aligned); work: caller-owned scratch of at least
+ * scoot_gp_device_work_bytes bytes, 16-byte aligned, not used by other work
+ * in flight (the context's workspace is not touched, so CUDA graphs captured
+ * on the context stay valid).  A non-finite or out-of-range input, or a
+ * matrix that is not numerically positive definite, makes scoot_ctx_check
+ * return SCOOT_EINVAL and leaves the blob undefined.  The conditioning
+ * indicator of the host function is not computed. */
+scoot_status scoot_gp_prepare_device(scoot_ctx* ctx, const scoot_param* h_space, const scoot_gp_layout* layout,
+                                     const uint32_t* obs, int64_t ld_obs, const float* y, const float* lengthscale,
+                                     const float* signal_var, const float* noise_var, const float* warp,
+                                     void* blob, void* work, int64_t work_bytes, void* stream);
+
 /* mean[m * ldo + i], var[m * ldo + i] for every candidate i < n and
  * objective m:  mu = k(x, X)(K + tau^2 I)^{-1} Y and
  * sigma^2 = k(x, x) - k(x, X)(K + tau^2 I)^{-1} k(X, x) (latent f, clamped
@@ -399,8 +425,9 @@ scoot_status scoot_delta_update(double* h_delta, int32_t* h_count, int32_t k, in
  * of the two children p_l (m_l - p_l) / m_l + p_r (m_r - p_r) / m_r, compared
  * exactly; ties go to the lower f, then the lower v (-0 and +0 are one
  * value; a zero threshold is stored as +0).  The two children of a node are
- * numbered next to each other in breadth-first order.  Uses the context's
- * workspace (feature ranks of the observations, 2 d n bytes).
+ * numbered next to each other in breadth-first order.  work: caller-owned
+ * device scratch of scoot_rf_train_work_bytes(n, d) bytes (the feature ranks
+ * of the observations), 16-byte aligned.
  * Output: nodes (scoot_node [n_trees][node_cap], device), tree t in
  * nodes[t * node_cap ...] with child indices counted from its first node,
  * n_nodes (int32 [n_trees], device) its node count (<= 2 m - 1, so node_cap
@@ -414,7 +441,9 @@ scoot_status scoot_delta_update(double* h_delta, int32_t* h_count, int32_t k, in
 scoot_status scoot_rf_train(scoot_ctx* ctx, const scoot_param* h_space, int32_t d, const uint32_t* obs, int32_t n,
                             int64_t ld, const uint8_t* labels, const int32_t* boot, int32_t n_trees, int32_t m,
                             int32_t max_depth, int32_t leaf_scale, scoot_node* nodes, int32_t node_cap,
-                            int32_t* n_nodes, void* stream);
+                            int32_t* n_nodes, void* work, int64_t work_bytes, void* stream);
+/* Bytes of scratch scoot_rf_train needs for n observations of d features. */
+scoot_status scoot_rf_train_work_bytes(int32_t n, int32_t d, int64_t* bytes);
 
 /* ------------------------------------------------------------------ 6. sequential fantasised picks */
 

@@ -1,0 +1,422 @@
+// The per-round GP state (Section 4.3) built on the device: features of the
+// observations, K + tau^2 I in fp64, its Cholesky factor, L^{-1} and
+// alpha = (K + tau^2 I)^{-1} y, written into the same blob layout that the
+// host preparation produces and the posterior and scoring kernels read.
+//
+// L^{-1} comes out of the factorisation itself: the elimination that turns
+// K into L^T, applied to the identity, gives L^{-1}.  At step j, with pivot
+// p_j = sqrt(A_jj) and l_ij = A_ij / p_j, every row i > j takes
+//   A_ik -= l_ij l_kj   (j < k <= i)   and   W_ic -= l_ij W_jc / p_j   (c <= j),
+// and row i of L^{-1} is W_i / p_i once the steps before i are done.  The
+// rows of one step are independent, so a step is one barrier.  fp64 runs at
+// a small fraction of the fp32 rate on this GPU; the n^3/3 multiply-adds of
+// a factorisation are its cost.
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+#include "internal.h"
+
+namespace {
+
+constexpr int kFeatThreads = 128;
+constexpr int kKmatThreads = 128;
+constexpr int kCholThreads = 1024;
+constexpr int kRowBlockDev = 64;   // rows of L^{-1} per tile (the layout's)
+constexpr int kColChunkDev = 32;   // columns of L^{-1} per tile
+constexpr int kSmemCholMaxN = 160; // A and W (packed lower triangles, fp64) in shared memory up to this n
+
+struct GpPrepArgs {
+    int32_t n, d, M, kernel, n_ord, n_pat, n_rb, n_tiles;
+    int64_t tri;                        // n (n + 1) / 2
+    int32_t order[SCOOT_MAX_DIM];       // feature f -> source parameter
+    int32_t kind[SCOOT_MAX_DIM];        // per source parameter
+    int32_t n_choices[SCOOT_MAX_DIM];
+    double lo[SCOOT_MAX_DIM], span[SCOOT_MAX_DIM];  // ordinal: (v - lo) / span; log: (ln v - lo) / span
+    float fmap[SCOOT_MAX_DIM][4];       // the blob's feature map, computed on the host
+    const uint32_t* obs;
+    int64_t ld_obs;
+    const float* y;                     // [M][n]
+    const float* ls;                    // [M][d], source order
+    const float* sf2;                   // [M]
+    const float* tau2;                  // [M]
+    const float* warp;                  // [M][d][2] or nullptr
+    char* blob;
+    int64_t off_fmap, off_xs, off_ils, off_alpha, off_linv, off_scal, off_cat, off_warp;
+    double* U;                          // [M][n][d] scaled features, source order
+    double* K;                          // [M][tri] packed lower triangle of K + tau^2 I (factorised in place when n is large)
+    double* W;                          // [M][tri] elimination of the identity (n large)
+    uint32_t* err;
+};
+
+__device__ __forceinline__ int64_t tri_idx(int i, int k) { return (int64_t)i * (i + 1) / 2 + k; }
+
+// 1 / sqrt(v) for v > 0 by Newton-Raphson on f(y) = 1 / y^2 - v from an
+// fp32 estimate, y <- y + y (1 - v y^2) / 2: each step doubles the correct
+// bits (24 -> 48 -> beyond fp64), in fused multiply-adds only, which keeps
+// the pivot off the slow fp64 division and square root.  Outside the fp32
+// range of the estimate the library's division and square root are used.
+__device__ __forceinline__ double rsqrt_newton(double v) {
+    if (!(v > 1e-30 && v < 1e30)) return 1.0 / sqrt(v);
+    double y = (double)rsqrtf((float)v);
+    const double h = 0.5 * v;
+    for (int it = 0; it < 3; ++it) {
+        const double e = fma(-h * y, y, 0.5);  // (1 - v y^2) / 2
+        y = fma(y, e, y);
+    }
+    return y;
+}
+
+__device__ __forceinline__ double matern_dev(double r, int kernel) {
+    if (kernel == SCOOT_MATERN32) {
+        const double a = 1.7320508075688772 * r;  // sqrt(3) r
+        return (1.0 + a) * exp(-a);
+    }
+    const double a = 2.23606797749979 * r;  // sqrt(5) r
+    return (1.0 + a + a * a / 3.0) * exp(-a);
+}
+
+// One thread per (observation j, feature f) of objective m: the feature,
+// warped and scaled (fp64 logarithms and powers are slow here, so they are
+// spread over n d threads).
+__global__ void __launch_bounds__(kFeatThreads) gp_feat_kernel(const __grid_constant__ GpPrepArgs a) {
+    const int t = blockIdx.x * kFeatThreads + threadIdx.x, m = blockIdx.y;
+    const int d = a.d, j = t / d, f = t - j * d;
+    bool bad = false;
+    if (j < a.n) {
+        float* xs = reinterpret_cast<float*>(a.blob + a.off_xs) + ((int64_t)m * a.n + j) * d;
+        double* U = a.U + ((int64_t)m * a.n + j) * d;
+        const int c = a.order[f];
+        const uint32_t w = a.obs[(int64_t)c * a.ld_obs + j];
+        const double l = (double)a.ls[m * d + c];
+        bad |= !(l > 0.0) || !isfinite(l);
+        if (a.kind[c] == SCOOT_CATEGORICAL) {
+            const double u = (double)(int32_t)w;
+            U[c] = u;
+            xs[f] = (float)u;
+        } else {
+            const double v = a.kind[c] == SCOOT_CONTINUOUS ? (double)__uint_as_float(w) : (double)(int32_t)w;
+            bad |= !isfinite(v) || (a.kind[c] == SCOOT_INT_LOG && !(v > 0.0));
+            double u;
+            if (a.kind[c] == SCOOT_INT_LOG) u = (log(v) - a.lo[c]) / a.span[c];
+            else u = a.span[c] > 0.0 ? (v - a.lo[c]) / a.span[c] : 0.0;
+            if (a.warp) {
+                const double wa = (double)a.warp[((int64_t)m * d + c) * 2];
+                const double wb = (double)a.warp[((int64_t)m * d + c) * 2 + 1];
+                bad |= !(wa > 0.0) || !isfinite(wa) || !(wb > 0.0) || !isfinite(wb);
+                const double x = fmin(fmax(u, 0.0), 1.0);
+                u = 1.0 - pow(1.0 - pow(x, wa), wb);
+            }
+            U[c] = u / l;
+            xs[f] = (float)(u / l);
+        }
+        if (f == 0) bad |= !isfinite(a.y[(int64_t)m * a.n + j]);
+    }
+    if (t == 0) {  // per-objective scalars (thread 0 of the objective's first block)
+        const float sf2 = a.sf2[m], tau2 = a.tau2[m];
+        bad |= !(sf2 > 0.0f) || !isfinite(sf2) || !(tau2 >= 0.0f) || !isfinite(tau2);
+        float* ils = reinterpret_cast<float*>(a.blob + a.off_ils) + m * d;
+        float* wo = reinterpret_cast<float*>(a.blob + a.off_warp) + (int64_t)m * d * 2;
+        for (int g = 0; g < d; ++g) {
+            const int c = a.order[g];
+            const double l = (double)a.ls[m * d + c];
+            const bool cat = a.kind[c] == SCOOT_CATEGORICAL;
+            ils[g] = cat ? (float)(1.0 / (l * l)) : (float)(1.0 / l);
+            wo[2 * g] = (a.warp && !cat) ? a.warp[((int64_t)m * d + c) * 2] : 1.0f;
+            wo[2 * g + 1] = (a.warp && !cat) ? a.warp[((int64_t)m * d + c) * 2 + 1] : 1.0f;
+        }
+        float* scal = reinterpret_cast<float*>(a.blob + a.off_scal) + m * 4;
+        scal[0] = sf2;
+        scal[1] = tau2;
+        scal[3] = a.warp ? 1.0f : 0.0f;  // scal[2] (best observed y) is written by the factorisation
+        if (m == 0) {
+            float* fm = reinterpret_cast<float*>(a.blob + a.off_fmap);
+            for (int g = 0; g < d; ++g)
+                for (int q = 0; q < 4; ++q) fm[g * 4 + q] = a.fmap[g][q];
+        }
+    }
+    if (bad) atomicOr(a.err, SCOOT_DEVERR_VALUE);
+}
+
+// Categorical part of r^2 for every (observation, category pattern).
+__global__ void __launch_bounds__(kKmatThreads) gp_cat_kernel(const __grid_constant__ GpPrepArgs a) {
+    const int64_t t = (int64_t)blockIdx.x * kKmatThreads + threadIdx.x;
+    const int m = blockIdx.y;
+    if (t >= (int64_t)a.n * a.n_pat) return;
+    const int j = (int)(t / a.n_pat), pat = (int)(t - (int64_t)j * a.n_pat);
+    double r2 = 0.0;
+    int rest = pat;
+    for (int f = a.n_ord; f < a.d; ++f) {
+        const int c = a.order[f];
+        const int v = rest % a.n_choices[c];
+        rest /= a.n_choices[c];
+        const double l = (double)a.ls[m * a.d + c];
+        if (v != (int32_t)a.obs[(int64_t)c * a.ld_obs + j]) r2 += 1.0 / (l * l);
+    }
+    reinterpret_cast<float*>(a.blob + a.off_cat)[((int64_t)m * a.n + j) * a.n_pat + pat] = (float)r2;
+}
+
+// K + tau^2 I, one thread per entry of the lower triangle.
+__global__ void __launch_bounds__(kKmatThreads) gp_kmat_kernel(const __grid_constant__ GpPrepArgs a) {
+    const int64_t t = (int64_t)blockIdx.x * kKmatThreads + threadIdx.x;
+    const int m = blockIdx.y;
+    if (t >= a.tri) return;
+    int i = (int)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
+    while ((int64_t)i * (i + 1) / 2 > t) --i;
+    while ((int64_t)(i + 1) * (i + 2) / 2 <= t) ++i;
+    const int k = (int)(t - (int64_t)i * (i + 1) / 2);
+    const double* ui = a.U + ((int64_t)m * a.n + i) * a.d;
+    const double* uk = a.U + ((int64_t)m * a.n + k) * a.d;
+    double r2 = 0.0;
+    for (int c = 0; c < a.d; ++c) {
+        const double diff = ui[c] - uk[c];
+        if (a.kind[c] == SCOOT_CATEGORICAL) {
+            const double l = (double)a.ls[m * a.d + c];
+            r2 += diff != 0.0 ? 1.0 / (l * l) : 0.0;
+        } else {
+            r2 += diff * diff;
+        }
+    }
+    double v = (double)a.sf2[m] * matern_dev(sqrt(r2), a.kernel);
+    if (i == k) v += (double)a.tau2[m];
+    a.K[(int64_t)m * a.tri + t] = v;
+}
+
+// One block per objective: the factorisation with L^{-1} alongside, then
+// alpha, the best observed y and the fp32 tiles of L^{-1}.
+//
+// Step j in a single multiply-add per entry: with g_i = A_ij / A_jj,
+//   A_ik -= g_i A_kj (j < k <= i)   and   W_ic -= g_i W_jc (c <= j),
+// one loop over t = 0 .. i per row (t <= j: W, t > j: A) so that the lanes
+// of a warp stay busy.  Column j is read from a contiguous copy (col), which
+// the threads that finish its entries in step j - 1 write (two buffers by
+// step parity).
+__global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_constant__ GpPrepArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int n = a.n, m = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = kCholThreads / 32;
+    double* rinv = reinterpret_cast<double*>(smem_raw);  // [n] 1 / pivot
+    double* rinv2 = rinv + n;                            // [n] 1 / pivot^2
+    double* z = rinv2 + n;                               // [n] L^{-1} y
+    double* col = z + n;                                 // [2][n] column j of A
+    double* A;
+    double* W;
+    if (n <= kSmemCholMaxN) {
+        A = col + 2 * n;
+        W = A + a.tri;
+        for (int64_t t = tid; t < a.tri; t += kCholThreads) A[t] = a.K[(int64_t)m * a.tri + t];
+        __syncthreads();
+    } else {
+        A = a.K + (int64_t)m * a.tri;
+        W = a.W + (int64_t)m * a.tri;
+    }
+    for (int i = warp; i < n; i += nwarps)
+        for (int c = lane; c <= i; c += 32) W[tri_idx(i, c)] = c == i ? 1.0 : 0.0;
+    for (int i = tid; i < n; i += kCholThreads) col[i] = A[tri_idx(i, 0)];
+    // s_bad_at: the first step whose pivot is not positive (n if none).  It is
+    // written during step j - 1 with the value j, so a thread still reading it
+    // for step j - 1 does not stop early; every thread stops at step j.  The
+    // pivot's reciprocals are computed once, by the thread that finishes the
+    // diagonal entry (fp64 square roots and divisions are slow here), and
+    // read after the step's barrier.
+    __shared__ int s_bad_at;
+    if (tid == 0) {
+        const double s0 = A[0];
+        const bool bad = !(s0 > 0.0) || !isfinite(s0);
+        s_bad_at = bad ? 0 : n;
+        rinv[0] = bad ? 0.0 : rsqrt_newton(s0);
+        rinv2[0] = rinv[0] * rinv[0];
+    }
+    __syncthreads();
+    for (int j = 0; j < n; ++j) {
+        if (s_bad_at <= j) break;  // the same in every thread
+        const double r2 = rinv2[j];
+        const double* cj = col + (j & 1) * n;
+        double* cn = col + ((j + 1) & 1) * n;
+        const double* Wj = W + tri_idx(j, 0);
+        for (int i = j + 1 + warp; i < n; i += nwarps) {
+            double* Ai = A + tri_idx(i, 0);
+            double* Wi = W + tri_idx(i, 0);
+            const double g = cj[i] * r2;
+            for (int t = lane; t <= i; t += 32) {
+                double* dst = t <= j ? Wi + t : Ai + t;
+                const double src = t <= j ? Wj[t] : cj[t];
+                const double v = *dst - g * src;
+                *dst = v;
+                if (t == j + 1) {  // A[i][j+1] is final: column j + 1 of the next step
+                    cn[i] = v;
+                    if (i == j + 1) {
+                        if (!(v > 0.0) || !isfinite(v)) {
+                            s_bad_at = j + 1;
+                        } else {
+                            const double y = rsqrt_newton(v);
+                            rinv[j + 1] = y;
+                            rinv2[j + 1] = y * y;
+                        }
+                    }
+                }
+            }
+        }
+        __syncthreads();
+    }
+    if (s_bad_at < n) {  // read after the loop's last barrier: the same in every thread
+        if (tid == 0) atomicOr(a.err, SCOOT_DEVERR_VALUE);
+        return;
+    }
+    const float* y = a.y + (int64_t)m * n;
+    // z = L^{-1} y, a warp per row
+    for (int i = warp; i < n; i += nwarps) {
+        const double* Wi = W + tri_idx(i, 0);
+        double t = 0.0;
+        for (int c = lane; c <= i; c += 32) t += Wi[c] * (double)y[c];
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) z[i] = t * rinv[i];
+    }
+    __syncthreads();
+    // alpha = L^{-T} z, a thread per column
+    float* alpha = reinterpret_cast<float*>(a.blob + a.off_alpha) + (int64_t)m * n;
+    for (int c = tid; c < n; c += kCholThreads) {
+        double t = 0.0;
+        for (int i = c; i < n; ++i) t += W[tri_idx(i, c)] * rinv[i] * z[i];
+        alpha[c] = (float)t;
+    }
+    if (warp == 0) {
+        float best = -INFINITY;
+        for (int j = lane; j < n; j += 32) best = fmaxf(best, y[j]);
+        for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, o));
+        if (lane == 0) reinterpret_cast<float*>(a.blob + a.off_scal)[m * 4 + 2] = best;
+    }
+    // tiles: row block rb, column chunk cj; tile[jj][ii] = L^{-1}[64 rb + ii][32 cj + jj]
+    float* tiles = reinterpret_cast<float*>(a.blob + a.off_linv) + (int64_t)m * a.n_tiles * kColChunkDev * kRowBlockDev;
+    const int64_t total = (int64_t)a.n_tiles * kColChunkDev * kRowBlockDev;
+    for (int64_t e = tid; e < total; e += kCholThreads) {
+        const int t = (int)(e / (kColChunkDev * kRowBlockDev));
+        const int jj = (int)(e / kRowBlockDev % kColChunkDev), ii = (int)(e % kRowBlockDev);
+        int rb = 0;
+        while ((rb + 1) * (rb + 2) <= t) ++rb;  // tiles of row blocks before rb: rb (rb + 1)
+        const int cj = t - rb * (rb + 1);
+        const int row = rb * kRowBlockDev + ii, c = cj * kColChunkDev + jj;
+        float v = 0.0f;
+        if (row < n && c <= row) v = (float)(W[tri_idx(row, c)] * rinv[row]);
+        tiles[e] = v;
+    }
+}
+
+}  // namespace
+
+extern "C" {
+
+scoot_status scoot_gp_device_work_bytes(const scoot_gp_layout* L, int64_t* bytes) {
+    if (!L || !bytes || !scoot_gp_layout_valid(L)) return SCOOT_EINVAL;
+    const int64_t n = L->n, tri = n * (n + 1) / 2;
+    *bytes = 8 * (int64_t)L->n_obj * (n * L->d + tri * (n <= kSmemCholMaxN ? 1 : 2));
+    return SCOOT_OK;
+}
+
+scoot_status scoot_gp_prepare_device(scoot_ctx* ctx, const scoot_param* h_space, const scoot_gp_layout* L,
+                                     const uint32_t* obs, int64_t ld_obs, const float* y, const float* lengthscale,
+                                     const float* signal_var, const float* noise_var, const float* warp, void* blob,
+                                     void* work, int64_t work_bytes, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (!h_space || !L) return scoot_fail(ctx, SCOOT_EINVAL, "h_space or layout is NULL");
+    scoot_gp_layout chk;
+    if (scoot_gp_layout_init(h_space, L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK ||
+        std::memcmp(&chk, L, sizeof(chk)) != 0)
+        return scoot_fail(ctx, SCOOT_EINVAL, "layout does not match h_space");
+    if (!obs || !y || !lengthscale || !signal_var || !noise_var || !blob)
+        return scoot_fail(ctx, SCOOT_EINVAL, "obs, y, lengthscale, signal_var, noise_var or blob is NULL");
+    if (ld_obs < L->n) return scoot_fail(ctx, SCOOT_EINVAL, "ld_obs = %lld < n = %d", (long long)ld_obs, L->n);
+    if (!scoot_aligned16(blob)) return scoot_fail(ctx, SCOOT_EINVAL, "blob is not 16-byte aligned");
+    int64_t need = 0;
+    scoot_gp_device_work_bytes(L, &need);
+    if (!work || work_bytes < need || !scoot_aligned16(work))
+        return scoot_fail(ctx, SCOOT_EINVAL, "work needs %lld bytes, 16-byte aligned", (long long)need);
+    GpPrepArgs a;
+    std::memset(&a, 0, sizeof(a));
+    const int n = L->n, d = L->d, M = L->n_obj;
+    a.n = n;
+    a.d = d;
+    a.M = M;
+    a.kernel = L->kernel;
+    a.n_ord = L->n_ord;
+    a.n_pat = L->n_pat;
+    a.n_rb = L->n_rb;
+    a.n_tiles = L->n_tiles;
+    a.tri = (int64_t)n * (n + 1) / 2;
+    int f = 0;
+    for (int pass = 0; pass < 2; ++pass)  // ordinal parameters first, then categorical ones
+        for (int c = 0; c < d; ++c)
+            if ((h_space[c].kind == SCOOT_CATEGORICAL) == (pass == 1)) a.order[f++] = c;
+    int stride = 1;
+    for (int g = 0; g < d; ++g) {
+        const int c = a.order[g];
+        const scoot_param& p = h_space[c];
+        a.kind[c] = p.kind;
+        a.n_choices[c] = p.n_choices;
+        float fa = 0.f, fb = 0.f;
+        if (p.kind == SCOOT_INT_LOG) {
+            a.lo[c] = std::log((double)p.lo);
+            a.span[c] = std::log((double)p.hi) - std::log((double)p.lo);
+            fa = (float)a.lo[c];
+            fb = (float)(1.0 / a.span[c]);
+        } else if (p.kind != SCOOT_CATEGORICAL) {
+            a.lo[c] = p.lo;
+            a.span[c] = (double)p.hi - (double)p.lo;
+            fa = p.lo;
+            fb = p.hi > p.lo ? (float)(1.0 / ((double)p.hi - (double)p.lo)) : 0.0f;
+        } else {
+            fa = (float)p.n_choices;
+            fb = (float)stride;
+            stride *= p.n_choices;
+        }
+        a.fmap[g][0] = (float)p.kind;
+        a.fmap[g][1] = fa;
+        a.fmap[g][2] = fb;
+        a.fmap[g][3] = (float)c;
+    }
+    a.obs = obs;
+    a.ld_obs = ld_obs;
+    a.y = y;
+    a.ls = lengthscale;
+    a.sf2 = signal_var;
+    a.tau2 = noise_var;
+    a.warp = warp;
+    a.blob = static_cast<char*>(blob);
+    a.off_fmap = L->off_fmap;
+    a.off_xs = L->off_xs;
+    a.off_ils = L->off_ils;
+    a.off_alpha = L->off_alpha;
+    a.off_linv = L->off_linv;
+    a.off_scal = L->off_scal;
+    a.off_cat = L->off_cat;
+    a.off_warp = L->off_warp;
+    const bool in_smem = n <= kSmemCholMaxN;
+    const size_t u_bytes = (size_t)M * n * d * sizeof(double);
+    const size_t k_bytes = (size_t)M * a.tri * sizeof(double);
+    char* ws = static_cast<char*>(work);
+    a.U = reinterpret_cast<double*>(ws);
+    a.K = reinterpret_cast<double*>(ws + u_bytes);
+    a.W = in_smem ? nullptr : reinterpret_cast<double*>(ws + u_bytes + k_bytes);
+    a.err = ctx->d_err;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    gp_feat_kernel<<<dim3((n * d + kFeatThreads - 1) / kFeatThreads, M), kFeatThreads, 0, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    if (L->n_ord < d) {
+        const int64_t cells = (int64_t)n * L->n_pat;
+        gp_cat_kernel<<<dim3((unsigned)((cells + kKmatThreads - 1) / kKmatThreads), M), kKmatThreads, 0, st>>>(a);
+        SCOOT_LAUNCHED(ctx);
+    } else {
+        // no categorical parameter: one pattern, zero distance
+        SCOOT_CUDA(ctx, cudaMemsetAsync(static_cast<char*>(blob) + L->off_cat, 0, (size_t)M * n * sizeof(float), st));
+    }
+    gp_kmat_kernel<<<dim3((unsigned)((a.tri + kKmatThreads - 1) / kKmatThreads), M), kKmatThreads, 0, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    const size_t smem = (size_t)5 * n * sizeof(double) + (in_smem ? (size_t)2 * a.tri * sizeof(double) : 0);
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(gp_chol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    gp_chol_kernel<<<M, kCholThreads, smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+}  // extern "C"

@@ -282,10 +282,16 @@ rf_train_kernel(const uint32_t* __restrict__ obs, int64_t ld, uint32_t float_col
 
 extern "C" {
 
+scoot_status scoot_rf_train_work_bytes(int32_t n, int32_t d, int64_t* bytes) {
+    if (!bytes || n < 1 || d < 1) return SCOOT_EINVAL;
+    *bytes = (2 * (int64_t)d * n + 15) / 16 * 16;
+    return SCOOT_OK;
+}
+
 scoot_status scoot_rf_train(scoot_ctx* ctx, const scoot_param* h_space, int32_t d, const uint32_t* obs, int32_t n,
                             int64_t ld, const uint8_t* labels, const int32_t* boot, int32_t n_trees, int32_t m,
                             int32_t max_depth, int32_t leaf_scale, scoot_node* nodes, int32_t node_cap,
-                            int32_t* n_nodes, void* stream) {
+                            int32_t* n_nodes, void* work, int64_t work_bytes, void* stream) {
     scoot_status s = scoot_enter(ctx);
     if (s != SCOOT_OK) return s;
     if (n < 1 || n > SCOOT_RF_TRAIN_MAX_OBS)
@@ -310,8 +316,9 @@ scoot_status scoot_rf_train(scoot_ctx* ctx, const scoot_param* h_space, int32_t 
     const size_t smem = (size_t)d * n * sizeof(float) + (size_t)n * sizeof(unsigned int) +
                         (size_t)2 * d * m * sizeof(uint16_t) + (size_t)cap * (3 * sizeof(uint16_t) + 1) + (size_t)2 * n;
     static_assert(sizeof(scoot_node) == 8, "scoot_node is 8 bytes");
-    if ((s = scoot_workspace(ctx, (size_t)d * n * sizeof(uint16_t))) != SCOOT_OK) return s;
-    uint16_t* perm = static_cast<uint16_t*>(ctx->ws);
+    if (!work || work_bytes < (int64_t)d * n * (int64_t)sizeof(uint16_t) || !scoot_aligned16(work))
+        return scoot_fail(ctx, SCOOT_EINVAL, "work needs %lld bytes, 16-byte aligned", (long long)d * n * 2);
+    uint16_t* perm = static_cast<uint16_t*>(work);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(rf_train_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     rank_kernel<<<dim3((n + kTrainThreads - 1) / kTrainThreads, d), kTrainThreads, 0, st>>>(obs, ld, float_cols, n,

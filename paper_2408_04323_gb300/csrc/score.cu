@@ -619,6 +619,12 @@ template <int EPI, int M, int DO>
 scoot_status launch_score_dm(scoot_ctx* ctx, const ScoreArgs& a, cudaStream_t st) {
     const size_t smem = score_smem(a, EPI, DO);
     auto kern = score_kernel<EPI, M, DO>;
+    int optin = 0;
+    SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
+    if (smem > (size_t)optin)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED,
+                          "score kernel needs %zu bytes of shared memory (n = %d observations, %d boxes), the "
+                          "device allows %d", smem, a.n_obs, a.n_boxes, optin);
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;
     SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));

@@ -4,8 +4,9 @@ objective with MACE, posterior + (UCB, PI, EI) -> random k-subset of their
 Pareto front (Sections 4.5 and 4.7).
 
 Host-side state (GP factor, box decomposition, packed forest) is prepared by
-the library's own host functions; torch only holds device memory and
-streams.  Nothing here computes any step of the path itself.
+the library's own host functions (the GP state optionally by the library's
+device kernels); torch only holds device memory and streams.  Nothing here
+computes any step of the path itself.
 """
 from __future__ import annotations
 
@@ -80,26 +81,46 @@ _staging = _Staging()
 
 
 class State:
-    """Per-round state prepared on the host (the library's host functions) and
-    uploaded to the device in one copy from pinned memory; gp_state, forest,
-    box_lo, box_hi, eps, grid and corner are views into one device buffer.
+    """Per-round state prepared by the library's host functions and uploaded
+    to the device in one copy from pinned memory; gp_state, forest, box_lo,
+    box_hi, eps, grid and corner are views into one device buffer.
+    With ``gp_on_device`` the GP state is built by the device instead
+    (scoot_gp_prepare_device, asynchronously on ``stream`` after the upload
+    of its inputs), overlapping the host's preparation of the rest.
     With ``into`` (a State of the same shapes) the upload reuses that State's
     device buffer, so work captured against it (a CUDA graph) stays valid."""
 
-    def __init__(self, inp: RoundInputs, device: torch.device, stream=None, into=None):
+    def __init__(self, inp: RoundInputs, device: torch.device, stream=None, into=None, gp_on_device=False,
+                 ctx=None):
         d = len(inp.space)
-        M = inp.y_obs.shape[0]
-        self.gp_layout = S.scoot_gp_layout_init(inp.space, inp.y_obs.shape[1], M, inp.kernel)
-        if inp.warp is None:
-            blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
-                                                 inp.signal_var, inp.noise_var, self.gp_layout)
+        M, n = inp.y_obs.shape
+        self.gp_layout = S.scoot_gp_layout_init(inp.space, n, M, inp.kernel)
+        self.cond = None
+        stream = torch.cuda.current_stream(device) if stream is None else stream
+        parts = []
+        if gp_on_device:
+            if ctx is None:
+                raise ValueError("gp_on_device needs a context")
+            gp_in = [("gpin_obs", np.ascontiguousarray(inp.x_obs[:, :n]).view(np.int32)),
+                     ("gpin_y", np.ascontiguousarray(inp.y_obs, np.float32)),
+                     ("gpin_ls", np.ascontiguousarray(inp.lengthscale, np.float32)),
+                     ("gpin_sf2", np.ascontiguousarray(inp.signal_var, np.float32)),
+                     ("gpin_tau2", np.ascontiguousarray(inp.noise_var, np.float32))]
+            if inp.warp is not None:
+                gp_in.append(("gpin_warp", np.ascontiguousarray(inp.warp, np.float32)))
+            parts += gp_in
         else:
-            blob, self.cond = S.scoot_gp_prepare_warped(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
-                                                        inp.signal_var, inp.noise_var, inp.warp, self.gp_layout)
+            if inp.warp is None:
+                blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                                     inp.signal_var, inp.noise_var, self.gp_layout)
+            else:
+                blob, self.cond = S.scoot_gp_prepare_warped(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                                            inp.signal_var, inp.noise_var, inp.warp,
+                                                            self.gp_layout)
+            parts.append(("gp_state", blob))
         self.forest_layout = S.scoot_forest_layout_init(inp.nodes, inp.tree_offset, d, inp.leaf_scale)
         fblob = S.scoot_forest_pack(self.forest_layout, inp.nodes, inp.tree_offset)
-        self.h_blobs = (blob, fblob)
-        parts = [("gp_state", blob), ("forest", fblob)]
+        parts.append(("forest", fblob))
         self.n_boxes = 0
         self.front_size = 0
         if inp.acq in ("ehvi", "ehvi-exact"):
@@ -111,13 +132,21 @@ class State:
             grid, self.n_grid, corner = S.scoot_boxes_index(lo, hi)
             self.h_boxes = (lo, hi, grid, corner)
             parts += [("grid", grid), ("corner", corner.view(np.int32))]
-        # one upload: 256-byte aligned slots in a pinned staging buffer
+        self.h_blobs = tuple(arr for _, arr in parts)
+        # one upload: 256-byte aligned slots in a pinned staging buffer; a
+        # device-built GP state takes a slot after the uploaded ones
         offs, total = [], 0
         for _, arr in parts:
             offs.append(total)
             total += (arr.nbytes + 255) // 256 * 256
-        stream = torch.cuda.current_stream(device) if stream is None else stream
-        stage = _staging.take(total)
+        upload = total
+        if gp_on_device:
+            gp_off = total
+            total += (self.gp_layout.bytes + 255) // 256 * 256
+            work_off = total
+            work_bytes = S.scoot_gp_device_work_bytes(self.gp_layout)
+            total += (work_bytes + 255) // 256 * 256
+        stage = _staging.take(upload)
         host = stage.numpy()
         for (_, arr), o in zip(parts, offs):
             host[o:o + arr.nbytes] = np.ascontiguousarray(arr).reshape(-1).view(np.uint8)
@@ -128,25 +157,36 @@ class State:
             if stream != torch.cuda.current_stream(device):
                 dev.record_stream(stream)
         with torch.cuda.stream(stream):
-            dev.copy_(stage, non_blocking=True)
+            dev[:upload].copy_(stage, non_blocking=True)
         _staging.sent(stream)
         self.buffer = dev
         self.offsets = offs
+        self.upload_bytes = upload
+        views = {}
         for (name, arr), o in zip(parts, offs):
             view = dev[o:o + arr.nbytes]
             if arr.dtype != np.uint8:
                 view = view.view(torch.float32 if arr.dtype == np.float32 else torch.int32).reshape(arr.shape)
-            setattr(self, name, view)
+            views[name] = view
+            if not name.startswith("gpin_"):
+                setattr(self, name, view)
+        if gp_on_device:
+            self.gp_state = dev[gp_off:gp_off + self.gp_layout.bytes]
+            S.scoot_gp_prepare_device(ctx, inp.space, self.gp_layout, views["gpin_obs"], views["gpin_y"],
+                                      views["gpin_ls"], views["gpin_sf2"], views["gpin_tau2"], self.gp_state,
+                                      work=dev[work_off:work_off + work_bytes], warp=views.get("gpin_warp"),
+                                      stream=stream)
 
 
 class ScoringRound:
     """Device buffers for pools of up to `capacity` candidates and the calls of one round."""
 
-    def __init__(self, ctx: S.Context, inp: RoundInputs, capacity: int, device=None):
+    def __init__(self, ctx: S.Context, inp: RoundInputs, capacity: int, device=None, gp_on_device=False):
         self.ctx = ctx
         self.inp = inp
         self.device = torch.device("cuda", ctx.device) if device is None else torch.device(device)
-        self.state = State(inp, self.device)
+        self.gp_on_device = bool(gp_on_device)
+        self.state = State(inp, self.device, gp_on_device=self.gp_on_device, ctx=ctx)
         self.capacity = int(capacity)
         dev = self.device
         self.mask = torch.empty(self.capacity, dtype=torch.uint8, device=dev)

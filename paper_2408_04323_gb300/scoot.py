@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_PKG, "libscoot.so")
 
 INT_UNIFORM, INT_LOG, CATEGORICAL, CONTINUOUS = 0, 1, 2, 3
 MATERN52, MATERN32 = 0, 1
-MAX_DIM, MAX_CLAUSES, MAX_OBJ, MAX_OBS, MAX_Q = 16, 16, 4, 1024, 64
+MAX_DIM, MAX_CLAUSES, MAX_OBJ, MAX_OBS, MAX_Q = 16, 16, 4, 640, 64
 
 STATUS = {0: "SCOOT_OK", -1: "SCOOT_EINVAL", -2: "SCOOT_ENOMEM", -3: "SCOOT_ECUDA",
           -4: "SCOOT_EDEVICE", -5: "SCOOT_ETIMEOUT", -6: "SCOOT_EUNSUPPORTED"}
@@ -81,6 +81,9 @@ _PROTOS = {
     "scoot_gp_layout_init": [_vp, _i32, _i32, _i32, _i32, C.POINTER(scoot_gp_layout)],
     "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_prepare_warped": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
+    "scoot_gp_device_work_bytes": [C.POINTER(scoot_gp_layout), C.POINTER(_i64)],
+    "scoot_gp_prepare_device": [_vp, _vp, C.POINTER(scoot_gp_layout), _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                _i64, _vp],
     "scoot_gp_posterior": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i64, _vp],
     "scoot_acq_ei": [_vp, _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp],
     "scoot_boxes_build": [_vp, _i32, _i32, _vp, _i32, _vp, _vp, C.POINTER(_i32), C.POINTER(_i32)],
@@ -98,7 +101,9 @@ _PROTOS = {
     "scoot_sobol_configs": [_vp, _vp, _i32, _i64, _i64, _vp, _i64, _vp],
     "scoot_first_feasible": [_vp, _vp, _i64, _i32, _vp, _vp, _vp],
     "scoot_delta_update": [C.POINTER(C.c_double), C.POINTER(_i32), _i32, _i32],
-    "scoot_rf_train": [_vp, _vp, _i32, _vp, _i32, _i64, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _i32, _vp, _vp],
+    "scoot_rf_train": [_vp, _vp, _i32, _vp, _i32, _i64, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _i32, _vp, _vp,
+                       _i64, _vp],
+    "scoot_rf_train_work_bytes": [_i32, _i32, C.POINTER(_i64)],
     "scoot_select_pareto": [_vp, _vp, _i64, _vp, _i64, _i32, C.c_uint64, _vp, _vp, _vp, _i64, _vp],
     "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
     "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, C.POINTER(_i64)],
@@ -466,17 +471,53 @@ def scoot_delta_update(delta: float, count: int, k: int, any_invalid: bool):
     return float(d.value), int(c.value)
 
 
-def scoot_rf_train(ctx, h_space, obs, n, labels, boot, max_depth, leaf_scale, nodes, n_nodes, stream=None):
+def scoot_gp_device_work_bytes(layout) -> int:
+    v = _i64()
+    _check(lib().scoot_gp_device_work_bytes(C.byref(layout), C.byref(v)), "scoot_gp_device_work_bytes")
+    return int(v.value)
+
+
+def scoot_gp_prepare_device(ctx, h_space, layout, obs, y, lengthscale, signal_var, noise_var, blob, work=None,
+                            warp=None, stream=None):
+    """Device inputs: obs int32 [d][ld], y float32 [M][n], lengthscale float32
+    [M][d], signal_var / noise_var float32 [M], warp float32 [M][d][2] or None;
+    blob: uint8 device tensor of layout.bytes; work: uint8 device scratch of
+    scoot_gp_device_work_bytes(layout) bytes (allocated here when None)."""
+    import torch
+    if work is None:
+        work = torch.empty(scoot_gp_device_work_bytes(layout), dtype=torch.uint8, device=blob.device)
+    _check(lib().scoot_gp_prepare_device(_h(ctx), _host(h_space, 16, name="h_space"), C.byref(layout),
+                                         _dev(obs, torch.int32, "obs"), int(obs.shape[1]),
+                                         _dev(y, torch.float32, "y"), _dev(lengthscale, torch.float32, "lengthscale"),
+                                         _dev(signal_var, torch.float32, "signal_var"),
+                                         _dev(noise_var, torch.float32, "noise_var"), _dev(warp, torch.float32, "warp"),
+                                         _dev(blob, torch.uint8, "blob"), _dev(work, torch.uint8, "work"),
+                                         int(work.numel()), _stream(stream)),
+           "scoot_gp_prepare_device", _h(ctx))
+
+
+def scoot_rf_train_work_bytes(n: int, d: int) -> int:
+    v = _i64()
+    _check(lib().scoot_rf_train_work_bytes(int(n), int(d), C.byref(v)), "scoot_rf_train_work_bytes")
+    return int(v.value)
+
+
+def scoot_rf_train(ctx, h_space, obs, n, labels, boot, max_depth, leaf_scale, nodes, n_nodes, work=None,
+                   stream=None):
     """obs: int32 [d][ld] observation words; labels: uint8 [n]; boot: int32
     [T][m]; nodes: int64 [T][node_cap] receiving scoot_node records (view the
-    host copy as the node dtype); n_nodes: int32 [T]."""
+    host copy as the node dtype); n_nodes: int32 [T]; work: uint8 device
+    scratch of scoot_rf_train_work_bytes(n, d) bytes (allocated here when None)."""
     import torch
     T, m = (int(boot.shape[0]), int(boot.shape[1])) if boot.dim() == 2 else (0, 1)
+    if work is None:
+        work = torch.empty(scoot_rf_train_work_bytes(n, len(h_space)), dtype=torch.uint8, device=obs.device)
     _check(lib().scoot_rf_train(_h(ctx), _host(h_space, 16, name="h_space"), len(h_space),
                                 _dev(obs, torch.int32, "obs"), int(n), int(obs.shape[1]),
                                 _dev(labels, torch.uint8, "labels"), _dev(boot, torch.int32, "boot"), T, m,
                                 int(max_depth), int(leaf_scale), _dev(nodes, torch.int64, "nodes"),
-                                int(nodes.shape[1]), _dev(n_nodes, torch.int32, "n_nodes"), _stream(stream)),
+                                int(nodes.shape[1]), _dev(n_nodes, torch.int32, "n_nodes"),
+                                _dev(work, torch.uint8, "work"), int(work.numel()), _stream(stream)),
            "scoot_rf_train", _h(ctx))
 
 
