@@ -726,7 +726,7 @@ def main():
             torch.cuda.synchronize(device)
             if kk >= args.warmup:
                 times.append(time.perf_counter() - t0)
-        state_bytes = sum(b.nbytes for b in state.h_blobs)  # everything uploaded (GP inputs or state, forest, boxes)
+        state_bytes = state.upload_bytes  # the one upload: GP state (or its inputs), forest, boxes
         e2e_s = statistics.mean(times)
         if dist:
             t = torch.tensor([e2e_s], device=device)

@@ -366,6 +366,58 @@ scoot_status scoot_score_ehvi_exact(scoot_ctx* ctx, const scoot_gp_layout* layou
                                     const float* grid, int32_t grid_cap, const int32_t* h_n_grid,
                                     const uint32_t* corner, int32_t n_boxes, float* acq, void* stream);
 
+/* ------------------------------------------------------------------ a round's host state in one call */
+
+/* Inputs of scoot_round_state_build (host arrays, conventions of the calls
+ * it combines). */
+typedef struct {
+    const scoot_param* space;
+    int32_t d;
+    const uint32_t* x_obs;       /* observations, words [d][ld_obs] */
+    int64_t ld_obs;
+    int32_t n;                   /* observations */
+    int32_t n_obj;               /* M */
+    const float* y;              /* [M][n] */
+    const float* lengthscale;    /* [M][d] */
+    const float* signal_var;     /* [M] */
+    const float* noise_var;      /* [M] */
+    const float* warp;           /* [M][d][2] or NULL */
+    int32_t kernel;
+    int32_t gp_on_device;        /* 1: no GP state here (scoot_gp_prepare_device builds it) */
+    const scoot_node* nodes;
+    const int32_t* tree_offset;  /* [n_trees + 1] */
+    int32_t n_trees;
+    int32_t leaf_scale;
+    int32_t boxes;               /* 0: none (EI, MACE); 1: boxes and eps (MC EHVI); 2: boxes and their grid index (exact EHVI) */
+    const float* ref;            /* [M] (boxes != 0) */
+    const float* eps;            /* [S][M] (boxes == 1) */
+    int32_t n_mc;                /* S */
+    int32_t grid_cap;            /* boxes == 2: coordinates per axis (0: 256) */
+} scoot_round_inputs;
+
+/* Where scoot_round_state_build put each part in the buffer (256-byte
+ * aligned offsets; -1 for an absent part). */
+typedef struct {
+    int64_t bytes;               /* bytes used: the upload */
+    int64_t off_gp, off_forest, off_box_lo, off_box_hi, off_eps, off_grid, off_corner;
+    int32_t n_boxes, front_size;
+    int32_t grid_cap;
+    int32_t n_grid[SCOOT_MAX_OBJ];
+    double cond[SCOOT_MAX_OBJ];  /* the GP factorisations' conditioning indicator */
+    scoot_gp_layout gp;
+    scoot_forest_layout forest;
+} scoot_round_state;
+
+/* A round's host-side state in one buffer h_buf (cap bytes, host): the GP
+ * blob (scoot_gp_prepare_warped), the packed forest (scoot_forest_pack) and,
+ * as asked, the boxes (scoot_boxes_build) with eps or with their grid index
+ * (scoot_boxes_index).  Copy the first out->bytes bytes to the device as
+ * they are.  The GP factorisation runs on a library worker thread while the
+ * calling thread packs the forest and builds the boxes.  SCOOT_ENOMEM if
+ * cap is too small (out->bytes then holds the size needed); the errors of
+ * the calls it combines otherwise. */
+scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, int64_t cap, scoot_round_state* out);
+
 /* ------------------------------------------------------------------ 5. top-q (Section 4.7) */
 
 /* The min(q, eligible) candidates with the largest acq, eligible meaning

@@ -25,11 +25,12 @@ int64_t align_up(int64_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 bool is_finite(double x) { return std::isfinite(x); }
 
-// GP states with at least kParallelRows observations are prepared with one
-// host thread per objective, and with at least kColumnRows with
-// kColumnThreads per objective for L^{-1} (below that, starting threads costs
-// more than it saves).
-constexpr int kParallelRows = 128;
+// GP states with at least kParallelRows observations are prepared with the
+// objectives spread over the library's persistent host threads, and with at
+// least kColumnRows with L^{-1}'s columns split kColumnThreads ways per
+// objective (below that, handing work to another thread costs more than it
+// saves).
+constexpr int kParallelRows = 32;
 constexpr int kColumnRows = 192;
 constexpr int kColumnThreads = 4;
 
@@ -427,10 +428,7 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
         // (interleaved, since column c costs ~(n - c)^2 / 2).
         if (n >= kColumnRows) {
             const int t = kColumnThreads;
-            std::vector<std::thread> th;
-            for (int k = 1; k < t; ++k) th.emplace_back(columns, k, t);
-            columns(0, t);
-            for (auto& x : th) x.join();
+            scoot_host_parallel(t, [&](int k) { columns(k, t); });
         } else {
             columns(0, 1);
         }
@@ -472,9 +470,7 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
     // per objective; small ones stay on the calling thread).
     std::vector<scoot_status> status(M, SCOOT_OK);
     if (M > 1 && n >= kParallelRows) {
-        std::vector<std::thread> th;
-        for (int m = 0; m < M; ++m) th.emplace_back([&, m] { status[m] = prep(m); });
-        for (auto& t : th) t.join();
+        scoot_host_parallel(M, [&](int m) { status[m] = prep(m); });
     } else {
         for (int m = 0; m < M; ++m) status[m] = prep(m);
     }

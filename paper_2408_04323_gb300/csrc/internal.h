@@ -4,6 +4,7 @@
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
+#include <functional>
 #include <string>
 #include <vector>
 
@@ -28,6 +29,9 @@ struct scoot_ctx {
 };
 
 scoot_status scoot_fail(scoot_ctx* ctx, scoot_status s, const char* fmt, ...);
+// fn(0 .. count-1) on the library's persistent host threads and the calling
+// thread; returns when all are done.  Safe to nest.
+void scoot_host_parallel(int count, const std::function<void(int)>& fn);
 // Make ctx->device current; sets an error on failure.
 scoot_status scoot_enter(scoot_ctx* ctx);
 // Ensure at least `bytes` of workspace (synchronising the device if it grows).

@@ -65,12 +65,20 @@ class _Staging:
         self.buf = None
         self.done = None
 
-    def take(self, nbytes: int) -> torch.Tensor:
+    def capacity(self) -> int:
+        return 1 << 20 if self.buf is None else self.buf.numel()
+
+    def take(self, nbytes: int, keep: int = 0) -> torch.Tensor:
+        """The buffer, at least nbytes long; when it has to grow, its first
+        `keep` bytes are carried over."""
         if self.done is not None:
             self.done.synchronize()
         if self.buf is None or self.buf.numel() < nbytes:
+            old = self.buf
             self.buf = torch.empty(max(nbytes, 1 << 20), dtype=torch.uint8, pin_memory=True)
-        return self.buf[:nbytes]
+            if old is not None and keep:
+                self.buf[:keep].copy_(old[:keep])
+        return self.buf
 
     def sent(self, stream) -> None:
         self.done = torch.cuda.Event()
@@ -81,101 +89,110 @@ _staging = _Staging()
 
 
 class State:
-    """Per-round state prepared by the library's host functions and uploaded
-    to the device in one copy from pinned memory; gp_state, forest, box_lo,
-    box_hi, eps, grid and corner are views into one device buffer.
-    With ``gp_on_device`` the GP state is built by the device instead
-    (scoot_gp_prepare_device, asynchronously on ``stream`` after the upload
-    of its inputs), overlapping the host's preparation of the rest.
-    With ``into`` (a State of the same shapes) the upload reuses that State's
-    device buffer, so work captured against it (a CUDA graph) stays valid."""
+    """Per-round state built by the library's host call
+    scoot_round_state_build (GP state, packed forest, boxes with eps or with
+    their grid index) straight into a pinned staging buffer and uploaded in
+    one copy; gp_state, forest, box_lo, box_hi, eps, grid and corner are
+    views into one device buffer.  With ``gp_on_device`` the GP state is
+    built by the device instead (scoot_gp_prepare_device, asynchronously on
+    ``stream`` after the upload of its inputs).  With ``into`` (a State of
+    the same shapes) the upload reuses that State's device buffer and views,
+    so work captured against it (a CUDA graph) stays valid."""
 
     def __init__(self, inp: RoundInputs, device: torch.device, stream=None, into=None, gp_on_device=False,
                  ctx=None):
-        d = len(inp.space)
         M, n = inp.y_obs.shape
-        self.gp_layout = S.scoot_gp_layout_init(inp.space, n, M, inp.kernel)
-        self.cond = None
         stream = torch.cuda.current_stream(device) if stream is None else stream
-        parts = []
+        if gp_on_device and ctx is None:
+            raise ValueError("gp_on_device needs a context")
+        boxes = {"ehvi": 1, "ehvi-exact": 2}.get(inp.acq, 0)
+        stage = _staging.take(_staging.capacity())
+        while True:
+            built, out = S.scoot_round_state_build(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                                   inp.signal_var, inp.noise_var, inp.nodes, inp.tree_offset,
+                                                   inp.leaf_scale, stage.numpy(), kernel=inp.kernel, warp=inp.warp,
+                                                   boxes=boxes, h_ref=inp.ref, h_eps=inp.eps,
+                                                   gp_on_device=gp_on_device)
+            if built is not None:
+                break
+            stage = _staging.take(int(out.bytes))
+        self.gp_layout = out.gp
+        self.forest_layout = out.forest
+        self.cond = [out.cond[m] for m in range(M)] if not gp_on_device else None
+        self.n_boxes = int(out.n_boxes)
+        self.front_size = int(out.front_size)
+        if boxes == 2:
+            self.n_grid = np.array(out.n_grid[:M], np.int32)
+        upload = int(out.bytes)
+        total = upload
+        gp_in = None
         if gp_on_device:
-            if ctx is None:
-                raise ValueError("gp_on_device needs a context")
-            gp_in = [("gpin_obs", np.ascontiguousarray(inp.x_obs[:, :n]).view(np.int32)),
-                     ("gpin_y", np.ascontiguousarray(inp.y_obs, np.float32)),
-                     ("gpin_ls", np.ascontiguousarray(inp.lengthscale, np.float32)),
-                     ("gpin_sf2", np.ascontiguousarray(inp.signal_var, np.float32)),
-                     ("gpin_tau2", np.ascontiguousarray(inp.noise_var, np.float32))]
+            # the GP inputs, the device-built state and its scratch after the host-built parts
+            gp_in = [np.ascontiguousarray(inp.x_obs[:, :n]).view(np.int32), np.ascontiguousarray(inp.y_obs, np.float32),
+                     np.ascontiguousarray(inp.lengthscale, np.float32), np.ascontiguousarray(inp.signal_var, np.float32),
+                     np.ascontiguousarray(inp.noise_var, np.float32)]
             if inp.warp is not None:
-                gp_in.append(("gpin_warp", np.ascontiguousarray(inp.warp, np.float32)))
-            parts += gp_in
-        else:
-            if inp.warp is None:
-                blob, self.cond = S.scoot_gp_prepare(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
-                                                     inp.signal_var, inp.noise_var, self.gp_layout)
-            else:
-                blob, self.cond = S.scoot_gp_prepare_warped(inp.space, inp.x_obs, inp.y_obs, inp.lengthscale,
-                                                            inp.signal_var, inp.noise_var, inp.warp,
-                                                            self.gp_layout)
-            parts.append(("gp_state", blob))
-        self.forest_layout = S.scoot_forest_layout_init(inp.nodes, inp.tree_offset, d, inp.leaf_scale)
-        fblob = S.scoot_forest_pack(self.forest_layout, inp.nodes, inp.tree_offset)
-        parts.append(("forest", fblob))
-        self.n_boxes = 0
-        self.front_size = 0
-        if inp.acq in ("ehvi", "ehvi-exact"):
-            lo, hi, self.front_size = S.scoot_boxes_build(inp.y_obs, inp.ref)
-            self.n_boxes = len(lo)
-            self.h_boxes = (lo, hi)
-            parts += [("box_lo", lo), ("box_hi", hi), ("eps", np.ascontiguousarray(inp.eps, np.float32))]
-        if inp.acq == "ehvi-exact":
-            grid, self.n_grid, corner = S.scoot_boxes_index(lo, hi)
-            self.h_boxes = (lo, hi, grid, corner)
-            parts += [("grid", grid), ("corner", corner.view(np.int32))]
-        self.h_blobs = tuple(arr for _, arr in parts)
-        # one upload: 256-byte aligned slots in a pinned staging buffer; a
-        # device-built GP state takes a slot after the uploaded ones
-        offs, total = [], 0
-        for _, arr in parts:
-            offs.append(total)
-            total += (arr.nbytes + 255) // 256 * 256
-        upload = total
-        if gp_on_device:
+                gp_in.append(np.ascontiguousarray(inp.warp, np.float32))
+            in_offs = []
+            for arr in gp_in:
+                in_offs.append(total)
+                total += (arr.nbytes + 255) // 256 * 256
+            if total > stage.numel():
+                stage = _staging.take(total, keep=upload)
+            host = stage.numpy()
+            for arr, o in zip(gp_in, in_offs):
+                host[o:o + arr.nbytes] = arr.reshape(-1).view(np.uint8)
+            upload = total
             gp_off = total
             total += (self.gp_layout.bytes + 255) // 256 * 256
             work_off = total
             work_bytes = S.scoot_gp_device_work_bytes(self.gp_layout)
             total += (work_bytes + 255) // 256 * 256
-        stage = _staging.take(upload)
-        host = stage.numpy()
-        for (_, arr), o in zip(parts, offs):
-            host[o:o + arr.nbytes] = np.ascontiguousarray(arr).reshape(-1).view(np.uint8)
-        if into is not None and into.buffer.numel() == total and into.offsets == offs:
+        offsets = (int(out.off_gp), int(out.off_forest), int(out.off_box_lo), int(out.off_box_hi), int(out.off_eps),
+                   int(out.off_grid), int(out.off_corner), upload, total)
+        reuse = into is not None and into.buffer.numel() == total and into.offsets == offsets
+        if reuse:
             dev = into.buffer
         else:
             dev = torch.empty(total, dtype=torch.uint8, device=device)
             if stream != torch.cuda.current_stream(device):
                 dev.record_stream(stream)
         with torch.cuda.stream(stream):
-            dev[:upload].copy_(stage, non_blocking=True)
+            dev[:upload].copy_(stage[:upload], non_blocking=True)
         _staging.sent(stream)
         self.buffer = dev
-        self.offsets = offs
+        self.offsets = offsets
         self.upload_bytes = upload
-        views = {}
-        for (name, arr), o in zip(parts, offs):
-            view = dev[o:o + arr.nbytes]
-            if arr.dtype != np.uint8:
-                view = view.view(torch.float32 if arr.dtype == np.float32 else torch.int32).reshape(arr.shape)
-            views[name] = view
-            if not name.startswith("gpin_"):
-                setattr(self, name, view)
+        if reuse:  # same offsets: the views of `into` are views of this buffer
+            for name in ("gp_state", "forest", "box_lo", "box_hi", "eps", "grid", "corner"):
+                if hasattr(into, name):
+                    setattr(self, name, getattr(into, name))
+        else:
+            def view(off, nbytes, dtype=None, shape=None):
+                v = dev[off:off + nbytes]
+                return v if dtype is None else v.view(dtype).reshape(shape)
+            if not gp_on_device:
+                self.gp_state = view(out.off_gp, self.gp_layout.bytes)
+            self.forest = view(out.off_forest, self.forest_layout.bytes)
+            B = self.n_boxes
+            if boxes:
+                self.box_lo = view(out.off_box_lo, B * M * 4, torch.float32, (B, M))
+                self.box_hi = view(out.off_box_hi, B * M * 4, torch.float32, (B, M))
+            if boxes == 1:
+                self.eps = view(out.off_eps, inp.eps.shape[0] * M * 4, torch.float32, (inp.eps.shape[0], M))
+            if boxes == 2:
+                self.grid = view(out.off_grid, M * out.grid_cap * 4, torch.float32, (M, out.grid_cap))
+                self.corner = view(out.off_corner, B * M * 4, torch.int32, (B, M))
+            if gp_on_device:
+                self.gp_state = view(gp_off, self.gp_layout.bytes)
         if gp_on_device:
-            self.gp_state = dev[gp_off:gp_off + self.gp_layout.bytes]
-            S.scoot_gp_prepare_device(ctx, inp.space, self.gp_layout, views["gpin_obs"], views["gpin_y"],
-                                      views["gpin_ls"], views["gpin_sf2"], views["gpin_tau2"], self.gp_state,
-                                      work=dev[work_off:work_off + work_bytes], warp=views.get("gpin_warp"),
-                                      stream=stream)
+            names = ["obs", "y", "ls", "sf2", "tau2", "warp"]
+            dv = {}
+            for name, arr, o in zip(names, gp_in, in_offs):
+                dv[name] = dev[o:o + arr.nbytes].view(torch.int32 if name == "obs" else torch.float32).reshape(arr.shape)
+            S.scoot_gp_prepare_device(ctx, inp.space, self.gp_layout, dv["obs"], dv["y"], dv["ls"], dv["sf2"],
+                                      dv["tau2"], self.gp_state, work=dev[work_off:work_off + work_bytes],
+                                      warp=dv.get("warp"), stream=stream)
 
 
 class ScoringRound:

@@ -60,6 +60,23 @@ class scoot_gp_layout(C.Structure):
                 ("off_cat", C.c_int64), ("off_warp", C.c_int64)]
 
 
+class scoot_round_inputs(C.Structure):
+    _fields_ = [("space", C.c_void_p), ("d", C.c_int32), ("x_obs", C.c_void_p), ("ld_obs", C.c_int64),
+                ("n", C.c_int32), ("n_obj", C.c_int32), ("y", C.c_void_p), ("lengthscale", C.c_void_p),
+                ("signal_var", C.c_void_p), ("noise_var", C.c_void_p), ("warp", C.c_void_p), ("kernel", C.c_int32),
+                ("gp_on_device", C.c_int32), ("nodes", C.c_void_p), ("tree_offset", C.c_void_p),
+                ("n_trees", C.c_int32), ("leaf_scale", C.c_int32), ("boxes", C.c_int32), ("ref", C.c_void_p),
+                ("eps", C.c_void_p), ("n_mc", C.c_int32), ("grid_cap", C.c_int32)]
+
+
+class scoot_round_state(C.Structure):
+    _fields_ = [("bytes", C.c_int64), ("off_gp", C.c_int64), ("off_forest", C.c_int64),
+                ("off_box_lo", C.c_int64), ("off_box_hi", C.c_int64), ("off_eps", C.c_int64),
+                ("off_grid", C.c_int64), ("off_corner", C.c_int64), ("n_boxes", C.c_int32),
+                ("front_size", C.c_int32), ("grid_cap", C.c_int32), ("n_grid", C.c_int32 * 4),
+                ("cond", C.c_double * 4), ("gp", scoot_gp_layout), ("forest", scoot_forest_layout)]
+
+
 # scoot_node as a numpy record (host copies of trained trees)
 NODE_DTYPE = np.dtype([("val", "<f4"), ("left", "<u2"), ("feat", "u1"), ("flags", "u1")])
 
@@ -82,6 +99,7 @@ _PROTOS = {
     "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_prepare_warped": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_device_work_bytes": [C.POINTER(scoot_gp_layout), C.POINTER(_i64)],
+    "scoot_round_state_build": [C.POINTER(scoot_round_inputs), _vp, _i64, C.POINTER(scoot_round_state)],
     "scoot_gp_prepare_device": [_vp, _vp, C.POINTER(scoot_gp_layout), _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                 _i64, _vp],
     "scoot_gp_posterior": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i64, _i64, _vp, _vp, _vp, _i64, _vp],
@@ -310,6 +328,50 @@ def scoot_boxes_index(h_lo, h_hi, grid_cap: int = 256):
                                    _host(np.ascontiguousarray(h_hi), dtype=np.float32, name="h_hi"), int(B), int(M),
                                    int(grid_cap), _host(grid), _host(n_grid), _host(corner)), "scoot_boxes_index")
     return grid, n_grid, corner[:B].copy()
+
+
+def scoot_round_state_build(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, h_nodes,
+                            h_tree_offset, leaf_scale: int, buf, kernel: int = 0, warp=None, boxes: int = 0,
+                            h_ref=None, h_eps=None, grid_cap: int = 0, gp_on_device: bool = False):
+    """A round's host state packed into the host uint8 array buf (pinned
+    staging memory; see include/scoot.h).  Returns the scoot_round_state, or
+    None when buf is too small (the size needed is then in .bytes of the
+    second return value).  Every array is kept alive by the caller for the
+    duration of the call."""
+    M, n = h_y.shape
+    keep = [np.ascontiguousarray(h_y, np.float32), np.ascontiguousarray(h_lengthscale, np.float32),
+            np.ascontiguousarray(h_signal_var, np.float32), np.ascontiguousarray(h_noise_var, np.float32)]
+    inp = scoot_round_inputs()
+    inp.space = _host(h_space, 16, name="h_space")
+    inp.d = len(h_space)
+    inp.x_obs = _host(h_x_obs, 4, name="h_x_obs")
+    inp.ld_obs = int(h_x_obs.shape[1])
+    inp.n, inp.n_obj = int(n), int(M)
+    inp.y, inp.lengthscale, inp.signal_var, inp.noise_var = (_host(a) for a in keep)
+    if warp is not None:
+        keep.append(np.ascontiguousarray(warp, np.float32))
+        inp.warp = _host(keep[-1])
+    inp.kernel = int(kernel)
+    inp.gp_on_device = int(bool(gp_on_device))
+    inp.nodes = _host(h_nodes, 8, name="h_nodes")
+    inp.tree_offset = _host(h_tree_offset, dtype=np.int32, name="h_tree_offset")
+    inp.n_trees = int(len(h_tree_offset) - 1)
+    inp.leaf_scale = int(leaf_scale)
+    inp.boxes = int(boxes)
+    if boxes:
+        keep.append(np.ascontiguousarray(h_ref, np.float32))
+        inp.ref = _host(keep[-1])
+    if boxes == 1:
+        keep.append(np.ascontiguousarray(h_eps, np.float32))
+        inp.eps = _host(keep[-1])
+        inp.n_mc = int(keep[-1].shape[0])
+    inp.grid_cap = int(grid_cap)
+    out = scoot_round_state()
+    st = lib().scoot_round_state_build(C.byref(inp), _host(buf), int(buf.nbytes), C.byref(out))
+    if st == -2 and out.bytes > buf.nbytes:  # SCOOT_ENOMEM: the buffer is too small
+        return None, out
+    _check(st, "scoot_round_state_build")
+    return out, out
 
 
 # ------------------------------------------------------------------ device calls

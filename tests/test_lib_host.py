@@ -283,3 +283,58 @@ def test_delta_controller_matches_oracle(S):
         assert 0.25 <= d1 <= 0.75
     with pytest.raises(S.ScootError):
         S.scoot_delta_update(0.5, 0, -1, False)
+
+
+@pytest.mark.parametrize("name,boxes,warped", [("tiny", 1, False), ("d8-ehvi2", 1, True), ("d10-ei", 0, False),
+                                               ("d10-ehvi3", 2, False), ("d12-fantasy", 1, False)])
+def test_round_state_build_equals_separate_calls(S, name, boxes, warped):
+    """scoot_round_state_build (GP factorisation on the library's host
+    threads while the caller packs the forest and builds the boxes) writes
+    exactly the bytes of the separate calls, at 256-byte aligned offsets; a
+    buffer that is too small is reported with the size needed; without the
+    GP part (built on the device) the other parts are unchanged."""
+    from workloads import warp_params
+    inst = make_instance(name, seeds(name)[0], n_cand=64)
+    warp = warp_params(name, seeds(name)[0]) if warped else None
+    buf = np.zeros(1 << 22, np.uint8)
+    st, out = S.scoot_round_state_build(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                        inst.noise_var, inst.nodes, inst.tree_offset, inst.workload.leaf_scale, buf,
+                                        warp=warp, boxes=boxes, h_ref=inst.ref, h_eps=inst.eps)
+    L = S.scoot_gp_layout_init(inst.space, inst.n_obs, inst.n_obj, 0)
+    if warp is None:
+        blob, cond = S.scoot_gp_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                        inst.noise_var, L)
+    else:
+        blob, cond = S.scoot_gp_prepare_warped(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
+                                               inst.signal_var, inst.noise_var, warp, L)
+    FL = S.scoot_forest_layout_init(inst.nodes, inst.tree_offset, inst.d, inst.workload.leaf_scale)
+    fb = S.scoot_forest_pack(FL, inst.nodes, inst.tree_offset)
+    offs = [st.off_gp, st.off_forest] + ([st.off_box_lo, st.off_box_hi] if boxes else [])
+    assert all(o % 256 == 0 for o in offs)
+    assert bytes(buf[st.off_gp:st.off_gp + L.bytes]) == blob.tobytes()
+    assert [st.cond[m] for m in range(inst.n_obj)] == list(cond)
+    assert bytes(buf[st.off_forest:st.off_forest + FL.bytes]) == fb.tobytes()
+    if boxes:
+        lo, hi, fs = S.scoot_boxes_build(inst.y_obs, inst.ref)
+        assert st.n_boxes == len(lo) and st.front_size == fs
+        assert np.array_equal(buf[st.off_box_lo:st.off_box_lo + lo.nbytes].view(np.float32), lo.ravel())
+        assert np.array_equal(buf[st.off_box_hi:st.off_box_hi + hi.nbytes].view(np.float32), hi.ravel())
+        if boxes == 1:
+            assert np.array_equal(buf[st.off_eps:st.off_eps + inst.eps.nbytes].view(np.float32),
+                                  inst.eps.astype(np.float32).ravel())
+        else:
+            grid, n_grid, corner = S.scoot_boxes_index(lo, hi)
+            assert list(st.n_grid[:inst.n_obj]) == list(n_grid)
+            assert np.array_equal(buf[st.off_grid:st.off_grid + grid.nbytes].view(np.float32), grid.ravel())
+            assert np.array_equal(buf[st.off_corner:st.off_corner + corner.nbytes].view(np.uint32), corner.ravel())
+    small = np.zeros(512, np.uint8)
+    none, need = S.scoot_round_state_build(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                           inst.noise_var, inst.nodes, inst.tree_offset, inst.workload.leaf_scale,
+                                           small, warp=warp, boxes=boxes, h_ref=inst.ref, h_eps=inst.eps)
+    assert none is None and need.bytes == st.bytes
+    buf2 = np.zeros(1 << 22, np.uint8)
+    st2, _ = S.scoot_round_state_build(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                       inst.noise_var, inst.nodes, inst.tree_offset, inst.workload.leaf_scale, buf2,
+                                       warp=warp, boxes=boxes, h_ref=inst.ref, h_eps=inst.eps, gp_on_device=True)
+    assert st2.off_gp == -1 and st2.off_forest == 0
+    assert bytes(buf2[:FL.bytes]) == fb.tobytes()
