@@ -31,8 +31,10 @@ bool is_finite(double x) { return std::isfinite(x); }
 // objective (below that, handing work to another thread costs more than it
 // saves).
 constexpr int kParallelRows = 32;
-constexpr int kColumnRows = 192;
+constexpr int kColumnRows = 128;
 constexpr int kColumnThreads = 4;
+constexpr int kKmatRows = 128;  // K + tau^2 I in kKmatChunks row ranges from this n
+constexpr int kKmatChunks = 4;
 
 // sum_k a[k] b[k] for k < len, with four independent partial sums (the fp64
 // accumulation chains of the factorisation would otherwise run at FMA latency).
@@ -189,17 +191,27 @@ scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, 
             us[(size_t)j * d + c] = g->cat[c] ? g->u[(size_t)j * d + c] : g->u[(size_t)j * d + c] / g->ell[c];
     std::vector<double>& K = g->chol;
     K.assign((size_t)n * n, 0.0);
-    for (int i = 0; i < n; ++i) {
-        const double* ui = &us[(size_t)i * d];
-        for (int j = 0; j <= i; ++j) {
-            const double* uj = &us[(size_t)j * d];
-            double r2 = 0.0;
-            for (int c = 0; c < d; ++c) {
-                const double t = ui[c] - uj[c];
-                r2 += g->cat[c] ? (t != 0.0 ? icat[c] : 0.0) : t * t;
+    auto rows = [&](int i0, int i1) {
+        for (int i = i0; i < i1; ++i) {
+            const double* ui = &us[(size_t)i * d];
+            for (int j = 0; j <= i; ++j) {
+                const double* uj = &us[(size_t)j * d];
+                double r2 = 0.0;
+                for (int c = 0; c < d; ++c) {
+                    const double t = ui[c] - uj[c];
+                    r2 += g->cat[c] ? (t != 0.0 ? icat[c] : 0.0) : t * t;
+                }
+                K[(size_t)i * n + j] = g->sf2 * matern(std::sqrt(r2), g->kernel) + (i == j ? g->tau2 : 0.0);
             }
-            K[(size_t)i * n + j] = g->sf2 * matern(std::sqrt(r2), g->kernel) + (i == j ? g->tau2 : 0.0);
         }
+    };
+    if (n >= kKmatRows) {
+        // row ranges of equal triangle area: row i has i + 1 entries
+        int bounds[kKmatChunks + 1];
+        for (int k = 0; k <= kKmatChunks; ++k) bounds[k] = (int)std::lround(n * std::sqrt((double)k / kKmatChunks));
+        scoot_host_parallel(kKmatChunks, [&](int k) { rows(bounds[k], bounds[k + 1]); });
+    } else {
+        rows(0, n);
     }
     double pmin = std::numeric_limits<double>::infinity(), pmax = 0.0;
     for (int j = 0; j < n; ++j) {
@@ -414,13 +426,15 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
         // Li holds the columns contiguously: Li[c * n + i] = L^{-1}[i][c].
         const std::vector<double>& C = g.chol;
         std::fill(Li.begin(), Li.end(), 0.0);
+        std::vector<double> rdiag(n);
+        for (int i = 0; i < n; ++i) rdiag[i] = 1.0 / C[(size_t)i * n + i];
         auto columns = [&](int c0, int step) {
             for (int c = c0; c < n; c += step) {
                 double* col = &Li[(size_t)c * n];
-                col[c] = 1.0 / C[(size_t)c * n + c];
+                col[c] = rdiag[c];
                 for (int i = c + 1; i < n; ++i) {
                     const double* Ci = &C[(size_t)i * n];
-                    col[i] = -dot(Ci + c, col + c, i - c) / Ci[i];
+                    col[i] = -dot(Ci + c, col + c, i - c) * rdiag[i];
                 }
             }
         };

@@ -53,11 +53,14 @@ public:
 
     void submit(std::function<void()> job, Latch* latch) {
         latch->left.fetch_add(1);
+        bool wake;
         {
             std::lock_guard<std::mutex> lk(mu_);
             jobs_.push_back({std::move(job), latch});
+            pending_.fetch_add(1);
+            wake = sleepers_ > 0;
         }
-        cv_.notify_one();
+        if (wake) cv_.notify_one();
     }
 
     // Until latch reaches zero: run queued jobs, else sleep briefly.
@@ -91,6 +94,7 @@ private:
             if (jobs_.empty()) return false;
             job = std::move(jobs_.front());
             jobs_.pop_front();
+            pending_.fetch_sub(1);
         }
         job.fn();
         if (job.latch->left.fetch_sub(1) == 1) {
@@ -100,19 +104,30 @@ private:
         return true;
     }
 
+    // After each job a thread polls for the next one for kSpin before it
+    // sleeps: waking a sleeping thread takes tens of microseconds, as long as
+    // the jobs themselves.
     void loop() {
         for (;;) {
-            {
+            const auto until = std::chrono::steady_clock::now() + kSpin;
+            while (pending_.load() == 0 && std::chrono::steady_clock::now() < until) std::this_thread::yield();
+            if (pending_.load() == 0) {
                 std::unique_lock<std::mutex> lk(mu_);
+                ++sleepers_;
                 cv_.wait(lk, [&] { return !jobs_.empty(); });
+                --sleepers_;
             }
             run_one();
         }
     }
 
+    static constexpr std::chrono::microseconds kSpin{500};
+
     std::mutex mu_;
     std::condition_variable cv_, done_cv_;
     std::deque<Job> jobs_;
+    std::atomic<int> pending_{0};  // jobs queued, readable without the lock
+    int sleepers_ = 0;             // threads waiting on cv_ (under mu_)
     int n_threads_ = 1;
 };
 
