@@ -20,6 +20,9 @@ Steps, in the order of one suggestion round (Section 4, Algorithm 1):
    its posterior mean as value and the GP is conditioned again);
 7. MACE for single-objective suggestion (Sections 4.5 and 4.7): UCB, PI and
    EI on the same posterior, their Pareto front, and a random k-subset of it.
+8. the tuning loop's Sobol sampling and Algorithm 1's threshold controller;
+9. CART training of the feasibility forest (Algorithm 1, Section 4.6);
+10. GP hyperparameters by maximum likelihood (Section 4.3).
 
 Readings of points the paper leaves open are marked "Reading:".
 Every function is pinned by the not-gpu tests against closed forms,
@@ -843,3 +846,92 @@ def train_forest(feats, labels, boot: np.ndarray, max_depth: int, leaf_scale: in
             out[k] = (val, left, f, 1 if leaf else 0)
             k += 1
     return out, offs
+
+
+# --------------------------------------------------------------------------
+# 10. GP hyperparameters by maximum likelihood (Section 4.3)
+
+def _matern_and_slope(r, kernel):
+    """k(r) / s_f^2 and its derivative in r^2 (finite at r = 0):
+    5/2: (1 + a + a^2/3) e^-a and -(5/6)(1 + a) e^-a, a = sqrt5 r;
+    3/2: (1 + a) e^-a and -(3/2) e^-a, a = sqrt3 r."""
+    r = np.asarray(r, np.float64)
+    if kernel == MATERN52:
+        a = math.sqrt(5.0) * r
+        e = np.exp(-a)
+        return (1.0 + a + a * a / 3.0) * e, -(5.0 / 6.0) * (1.0 + a) * e
+    if kernel == MATERN32:
+        a = math.sqrt(3.0) * r
+        e = np.exp(-a)
+        return (1.0 + a) * e, -1.5 * e
+    raise ValueError(kernel)
+
+
+def log_marginal_likelihood(space, x_obs_words, y, theta, kernel: int = MATERN52):
+    """log p(y | X, theta) of the zero-mean GP of Section 4.3 and its
+    gradient in theta = (ln l_1 .. ln l_d, ln s_f^2, ln tau^2).
+
+    With K = s_f^2 k(r) + tau^2 I and alpha = K^{-1} y:
+      lml = -y^T alpha / 2 - log det K / 2 - n log(2 pi) / 2,
+      d lml / d theta_p = tr((alpha alpha^T - K^{-1}) dK/dtheta_p) / 2,
+    dK/d ln s_f^2 = s_f^2 k(r), dK/d ln tau^2 = tau^2 I and
+    dK/d ln l_c = -2 s_f^2 k'(r^2) D_c, where D_c is the term of feature c in
+    r^2 ((u_c - u'_c)^2 / l_c^2, or [u_c != u'_c] / l_c^2 for a category).
+    Returns (lml, grad[d + 2])."""
+    theta = np.asarray(theta, np.float64)
+    d = len(space)
+    ell = np.exp(theta[:d])
+    sf2, tau2 = math.exp(theta[d]), math.exp(theta[d + 1])
+    u, is_cat = gp_features(space, decode(space, x_obs_words))
+    y = np.asarray(y, np.float64)
+    n = len(y)
+    D = np.zeros((d, n, n))
+    for c in range(d):
+        if is_cat[c]:
+            D[c] = (u[:, c][:, None] != u[:, c][None, :]).astype(np.float64) / (ell[c] * ell[c])
+        else:
+            diff = (u[:, c][:, None] - u[:, c][None, :]) / ell[c]
+            D[c] = diff * diff
+    r = np.sqrt(D.sum(axis=0))
+    k, dk = _matern_and_slope(r, kernel)
+    K = sf2 * k + tau2 * np.eye(n)
+    L = np.linalg.cholesky(K)
+    alpha = sla.cho_solve((L, True), y)
+    Kinv = sla.cho_solve((L, True), np.eye(n))
+    lml = -0.5 * y @ alpha - np.sum(np.log(np.diag(L))) - 0.5 * n * math.log(2.0 * math.pi)
+    Wm = np.outer(alpha, alpha) - Kinv
+    grad = np.zeros(d + 2)
+    for c in range(d):
+        grad[c] = 0.5 * np.sum(Wm * (-2.0 * sf2 * dk * D[c]))
+    grad[d] = 0.5 * np.sum(Wm * (sf2 * k))
+    grad[d + 1] = 0.5 * tau2 * np.trace(Wm)
+    return float(lml), grad
+
+
+def fit_hyperparameters(space, x_obs_words, y, theta0, lo, hi, free, steps: int, lr: float,
+                        kernel: int = MATERN52):
+    """Maximum-likelihood hyperparameters from the start theta0 by projected
+    Adam ascent (Kingma and Ba's Adam: beta1 = 0.9, beta2 = 0.999,
+    eps = 1e-8), `steps` steps with the step size decaying linearly,
+    lr (1 - t / steps) at step t = 0 .. steps-1; after each step theta is
+    clipped to [lo, hi]; parameters with free[p] == 0 stay at theta0.
+    Reading: the paper learns tau^2 by maximum likelihood (Section 4.3);
+    which parameters are free is the caller's choice (tau^2 alone is the
+    paper's statement).  Returns (theta, lml) at the last step."""
+    theta = np.array(theta0, np.float64)
+    lo, hi = np.asarray(lo, np.float64), np.asarray(hi, np.float64)
+    mask = np.asarray(free, bool).astype(np.float64)
+    m1 = np.zeros_like(theta)
+    m2 = np.zeros_like(theta)
+    b1, b2, eps = 0.9, 0.999, 1e-8
+    for t in range(steps):
+        _, g = log_marginal_likelihood(space, x_obs_words, y, theta, kernel)
+        g = g * mask
+        m1 = b1 * m1 + (1.0 - b1) * g
+        m2 = b2 * m2 + (1.0 - b2) * g * g
+        mh = m1 / (1.0 - b1 ** (t + 1))
+        vh = m2 / (1.0 - b2 ** (t + 1))
+        step = lr * (1.0 - t / steps)
+        theta = np.clip(theta + step * mh / (np.sqrt(vh) + eps), lo, hi)
+    lml, _ = log_marginal_likelihood(space, x_obs_words, y, theta, kernel)
+    return theta, lml

@@ -867,3 +867,93 @@ def test_cart_signed_zero_is_one_value():
     assert tree == O.train_cart(Xp, y, np.arange(5), 4, 255)
     zeros = [t for t in tree if not t[3] and t[0] == 0.0]
     assert zeros and all(math.copysign(1.0, t[0]) == 1.0 for t in zeros)
+
+
+# ------------------------------------------------------------------ GP hyperparameters by MLE (Section 4.3)
+
+def _mle_case(name="d8-ehvi2", n=24, m=0):
+    inst = make_instance(name, seeds(name)[0], n_cand=16)
+    x = np.ascontiguousarray(inst.x_obs[:, :n])
+    y = np.asarray(inst.y_obs[m, :n], np.float64)
+    theta = np.concatenate([np.log(inst.lengthscale[m].astype(np.float64)),
+                            [math.log(float(inst.signal_var[m])), math.log(max(float(inst.noise_var[m]), 1e-3))]])
+    return inst, x, y, theta
+
+
+@pytest.mark.parametrize("kernel", [0, 1])
+def test_lml_equals_gaussian_log_density(kernel):
+    """The log marginal likelihood is the log density of y under
+    N(0, K + tau^2 I): scipy's multivariate normal, with K from the
+    (separately pinned) GP covariance."""
+    from scipy.stats import multivariate_normal
+    inst, x, y, theta = _mle_case()
+    d = inst.d
+    lml, _ = O.log_marginal_likelihood(inst.space, x, y, theta, kernel)
+    gp = O.GP(inst.space, x, y, np.exp(theta[:d]), math.exp(theta[d]), math.exp(theta[d + 1]), kernel)
+    K = gp.cov(gp.u_obs, gp.u_obs) + math.exp(theta[d + 1]) * np.eye(len(y))
+    want = multivariate_normal(mean=np.zeros(len(y)), cov=K).logpdf(y)
+    assert lml == pytest.approx(want, rel=1e-10, abs=1e-9)
+
+
+@pytest.mark.parametrize("kernel,name", [(0, "d8-ehvi2"), (1, "d8-ehvi2"), (0, "d10-ei")])
+def test_lml_gradient_matches_finite_differences(kernel, name):
+    """Every component of the analytic gradient (ordinal and categorical
+    lengthscales, signal and noise variance) equals a central difference of
+    the log marginal likelihood."""
+    inst, x, y, theta = _mle_case(name, n=20)
+    _, g = O.log_marginal_likelihood(inst.space, x, y, theta, kernel)
+    h = 1e-5
+    for p in range(len(theta)):
+        tp, tm = theta.copy(), theta.copy()
+        tp[p] += h
+        tm[p] -= h
+        fd = (O.log_marginal_likelihood(inst.space, x, y, tp, kernel)[0] -
+              O.log_marginal_likelihood(inst.space, x, y, tm, kernel)[0]) / (2 * h)
+        assert g[p] == pytest.approx(fd, rel=1e-5, abs=1e-6), p
+
+
+def test_lml_one_observation_closed_form_and_noise_mle():
+    """n = 1: lml = -y^2 / (2 v) - log(v) / 2 - log(2 pi) / 2 with
+    v = s_f^2 + tau^2, d lml / d ln tau^2 = tau^2 (y^2 / v^2 - 1 / v) / 2;
+    fitting tau^2 alone reaches v = y^2, the closed-form maximiser."""
+    space = np.zeros(2, PARAM_DTYPE)
+    space["kind"] = CONTINUOUS
+    space["hi"] = 1.0
+    x = np.array([[np.float32(0.3).view(np.uint32)], [np.float32(0.7).view(np.uint32)]], np.uint32)
+    y = np.array([2.5])
+    sf2, tau2 = 1.0, 0.5
+    theta = np.array([0.0, 0.0, math.log(sf2), math.log(tau2)])
+    lml, g = O.log_marginal_likelihood(space, x, y, theta)
+    v = sf2 + tau2
+    assert lml == pytest.approx(-y[0] ** 2 / (2 * v) - 0.5 * math.log(v) - 0.5 * math.log(2 * math.pi), rel=1e-14)
+    assert g[3] == pytest.approx(0.5 * tau2 * (y[0] ** 2 / v ** 2 - 1 / v), rel=1e-12)
+    assert g[2] == pytest.approx(0.5 * sf2 * (y[0] ** 2 / v ** 2 - 1 / v), rel=1e-12)
+    assert g[0] == 0.0 and g[1] == 0.0
+    free = np.array([0, 0, 0, 1])
+    th, best = O.fit_hyperparameters(space, x, y, theta, [-9] * 4, [9] * 4, free, 400, 0.1)
+    assert math.exp(th[3]) == pytest.approx(y[0] ** 2 - sf2, rel=1e-4)
+    assert np.array_equal(th[:3], theta[:3])
+
+
+def test_fit_increases_lml_and_respects_bounds():
+    """The fit ends with a larger likelihood than its start, inside the
+    bounds, with frozen parameters untouched and the free ones at a
+    stationary point or a bound."""
+    inst, x, y, theta = _mle_case(n=30)
+    P = len(theta)
+    lo = np.full(P, -4.0)
+    hi = np.full(P, 3.0)
+    lo[-1] = math.log(1e-4)
+    free = np.ones(P, int)
+    free[0] = 0
+    start = np.clip(theta + 0.5, lo, hi)
+    l0, _ = O.log_marginal_likelihood(inst.space, x, y, start)
+    th, l1 = O.fit_hyperparameters(inst.space, x, y, start, lo, hi, free, 1000, 0.05)
+    assert l1 > l0 + 10.0
+    assert np.all(th >= lo) and np.all(th <= hi) and th[0] == start[0]
+    _, g = O.log_marginal_likelihood(inst.space, x, y, th)
+    inside = (th > lo + 1e-9) & (th < hi - 1e-9) & (free == 1)
+    at_bound = (free == 1) & ~inside
+    assert inside.sum() >= 7 and np.all(np.abs(g[inside]) < 1e-6)
+    # at a bound the gradient points outwards (the bound holds the maximiser back)
+    assert np.all(np.where(th[at_bound] <= lo[at_bound] + 1e-9, g[at_bound] <= 0, g[at_bound] >= 0))
