@@ -24,6 +24,7 @@ Under torchrun (--gpus N > 1) each rank scores its own pool of N candidates
 from __future__ import annotations
 
 import argparse
+import math
 import hashlib
 import json
 import os
@@ -73,8 +74,9 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--gp-prep", choices=["host", "device"], default="host",
                    help="where the end-to-end step builds the GP state (fp64 factorisation)")
-    p.add_argument("--stage", choices=["round", "rf-train"], default="round",
-                   help="rf-train: time the training of the workload's feasibility forest instead of a round")
+    p.add_argument("--stage", choices=["round", "rf-train", "gp-mle"], default="round",
+                   help="rf-train: the training of the workload's feasibility forest; gp-mle: its GP "
+                        "hyperparameter fit (32 starts x 100 Adam steps); instead of a round")
     return p.parse_args()
 
 
@@ -456,10 +458,180 @@ def run_rf_reference(args):
     print(json.dumps(line), flush=True)
 
 
+MLE_METRIC = "GP log-marginal-likelihood evaluations with gradient/sec (hyperparameter MLE, projected Adam)"
+MLE_UNIT = "evaluations/s"
+MLE_STARTS, MLE_STEPS, MLE_LR = 32, 100, 0.05
+FP64_NOMINAL_TFLOPS = 1.25  # GB300 FP64, nominal
+
+
+def mle_inputs(name):
+    """Observations of a workload and MLE_STARTS starts around its hyperparameters."""
+    import numpy as np
+    from workloads import Stream, make_instance, seeds
+    inst = make_instance(name, seeds(name)[0], n_cand=4)
+    M, P = inst.n_obj, inst.d + 2
+    base = np.stack([np.concatenate([np.log(inst.lengthscale[m].astype(np.float64)),
+                                     [0.0, math.log(max(float(inst.noise_var[m]), 1e-4))]]) for m in range(M)])
+    lo, hi = np.full(P, -4.0), np.full(P, 3.0)
+    lo[-1] = math.log(1e-4)
+    theta0 = np.clip(base[None] + Stream(1, "mle-starts").normal(MLE_STARTS * M * P).reshape(MLE_STARTS, M, P) * 0.5,
+                     lo, hi)
+    return inst, theta0, lo, hi
+
+
+def mle_flops(n, d):
+    """fp64 flops of one evaluation: the elimination with L^-1 (n^3/3 multiply-adds), K^-1 (n^3/6), the
+    two triangular products (n^2), and per pair of observations K's entry and the gradient's (6 d flops
+    and two exponentials, counted as 30 flops each)."""
+    return 2 * (n ** 3 / 3 + n ** 3 / 6 + n * n) + n * (n + 1) / 2 * (6 * d + 60)
+
+
+def mle_oracle_seconds(name, evals):
+    code = ("import sys, time, json; sys.path.insert(0, %r)\n"
+            "import numpy as np, oracle, bench\n"
+            "inst, theta0, lo, hi = bench.mle_inputs(%r)\n"
+            "n = inst.n_obs\n"
+            "t = time.perf_counter()\n"
+            "for k in range(%d):\n"
+            "    s, m = divmod(k, inst.n_obj)\n"
+            "    oracle.log_marginal_likelihood(inst.space, inst.x_obs[:, :n], inst.y_obs[m], theta0[s %% len(theta0), m])\n"
+            "print(json.dumps({'seconds': time.perf_counter() - t}))\n" % (ROOT, name, evals))
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    if p.returncode != 0:
+        raise RuntimeError(p.stderr[-2000:])
+    return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
+
+
+def mle_config(inst, extra=None):
+    w = inst.workload
+    cfg = {"workload": f"{w.name} GP fit: n={w.n_obs} observations, d={w.d}, M={w.n_obj} objectives, "
+                       f"{MLE_STARTS} starts x {MLE_STEPS} projected Adam steps (all parameters free)",
+           "observations": w.n_obs, "objectives": w.n_obj, "starts": MLE_STARTS, "steps": MLE_STEPS,
+           "inputs": "seeded synthetic observations, resident in HBM"}
+    cfg.update(extra or {})
+    return cfg
+
+
+def run_gp_mle(args):
+    import numpy as np
+    import torch
+    import paper_2408_04323_gb300 as pkg
+    pkg.build()
+    from paper_2408_04323_gb300 import scoot as S
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1:
+        raise SystemExit("--stage gp-mle runs on one GPU")
+    inst, theta0, lo, hi = mle_inputs(args.workload)
+    n, d, M, P = inst.n_obs, inst.d, inst.n_obj, inst.d + 2
+    device = torch.device("cuda", 0)
+    ctx = S.Context(0)
+    h_obs = torch.from_numpy(np.ascontiguousarray(inst.x_obs[:, :n]).view(np.int32)).pin_memory()
+    h_y = torch.from_numpy(np.ascontiguousarray(inst.y_obs, np.float32)).pin_memory()
+    h_t0 = torch.from_numpy(theta0).pin_memory()
+    obs, y, t0 = h_obs.to(device), h_y.to(device), h_t0.to(device)
+    th = torch.zeros_like(t0)
+    lml = torch.zeros((MLE_STARTS, M), dtype=torch.float64, device=device)
+    h_th = torch.empty(th.shape, dtype=torch.float64, pin_memory=True)
+    h_lml = torch.empty(lml.shape, dtype=torch.float64, pin_memory=True)
+    work = torch.empty(S.scoot_gp_mle_work_bytes(n, d, M, MLE_STARTS), dtype=torch.uint8, device=device)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
+    stream = torch.cuda.current_stream(device)
+    free = (1 << P) - 1
+
+    def fit(o=obs, yy=y, t=t0):
+        S.scoot_gp_mle(ctx, inst.space, o, n, yy, t, lo, hi, free, MLE_STEPS, MLE_LR, th, lml, work=work,
+                       stream=stream)
+
+    sampler = ClockSampler()
+    sampler.start()
+    for k in range(max(3, args.warmup)):
+        flush.fill_(k & 0xFF)
+        fit()
+    torch.cuda.synchronize(device)
+    ctx.check(stream)
+    steps = max(1, min(args.steps, 20))
+    tev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+    for kk in range(steps):
+        flush.fill_(kk & 0xFF)
+        tev[kk][0].record(stream)
+        fit()
+        tev[kk][1].record(stream)
+    torch.cuda.synchronize(device)
+    clocks = sampler.stop()
+    ctx.check(stream)
+    ms = statistics.mean(e[0].elapsed_time(e[1]) for e in tev)
+    evals = MLE_STARTS * M * (MLE_STEPS + 1)
+    e2e = None
+    if not args.no_e2e:
+        d_obs, d_y, d_t0 = torch.empty_like(obs), torch.empty_like(y), torch.empty_like(t0)
+        times = []
+        for kk in range(steps + 2):
+            torch.cuda.synchronize(device)
+            t_0 = time.perf_counter()
+            d_obs.copy_(h_obs, non_blocking=True)
+            d_y.copy_(h_y, non_blocking=True)
+            d_t0.copy_(h_t0, non_blocking=True)
+            fit(d_obs, d_y, d_t0)
+            h_th.copy_(th, non_blocking=True)
+            h_lml.copy_(lml, non_blocking=True)
+            torch.cuda.synchronize(device)
+            if kk >= 2:
+                times.append(time.perf_counter() - t_0)
+        e2e_s = statistics.mean(times)
+        e2e = {"value": evals / e2e_s, "unit": MLE_UNIT,
+               "h2d_bytes_per_step": int(h_obs.numel() * 4 + h_y.numel() * 4 + h_t0.numel() * 8),
+               "d2h_bytes_per_step": int(h_th.numel() * 8 + h_lml.numel() * 8), "ms_per_step": 1e3 * e2e_s}
+    achieved = mle_flops(n, d) * evals / (ms / 1e3) / 1e12
+    roof = {"bound": "alu", "achieved": achieved, "peak": FP64_NOMINAL_TFLOPS, "unit": "TFLOP/s (fp64)",
+            "frac": achieved / FP64_NOMINAL_TFLOPS, "traffic": None, "kernel": "gp_mle",
+            "peak_source": "nominal GB300 FP64 rate (no measured fp64 peak on this pool)",
+            "work_per_unit": mle_flops(n, d), "units_per_launch": evals}
+    cpu = None
+    if not args.no_cpu_baseline:
+        one = mle_oracle_seconds(args.workload, 2) / 2
+        k = max(2, int(args.cpu_seconds / max(one, 1e-4)))
+        secs = mle_oracle_seconds(args.workload, k)
+        cpu = {"value": k / secs, "unit": MLE_UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"{k} evaluations (likelihood and gradient) at the starts, numpy fp64, one thread"}
+    line = {"metric": MLE_METRIC, "value": evals / (ms / 1e3), "unit": MLE_UNIT, "n_gpus": 1, "steps": steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": mle_config(inst, {"launch": "features, then one block per (start, objective) for the whole fit",
+                                        "l2": "flushed between steps (256 MiB write)"}),
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * steps, "clocks": clocks}
+    print(json.dumps(line), flush=True)
+    ctx.close()
+
+
+def run_mle_reference(args):
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    inst, theta0, lo, hi = mle_inputs(args.workload)
+    one = mle_oracle_seconds(args.workload, 2) / 2
+    per_step = max(0.5, 120.0 / max(1, args.steps + args.warmup))
+    k = max(2, int(per_step / max(one, 1e-4)))
+    for _ in range(args.warmup):
+        mle_oracle_seconds(args.workload, k)
+    times = [mle_oracle_seconds(args.workload, k) for _ in range(args.steps)]
+    ms = 1e3 * statistics.mean(times)
+    value = k / (ms / 1e3)
+    line = {"impl": "reference", "metric": MLE_METRIC, "value": value, "unit": MLE_UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": mle_config(inst, {"reference": "CPU oracle (the paper ships no code)", "evaluations_per_step": k}),
+            "cpu_baseline": {"value": value, "unit": MLE_UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{k} evaluations per step"},
+            "e2e": {"value": value, "unit": MLE_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     if args.stage == "rf-train":
         (run_rf_reference if args.impl == "reference" else run_rf_train)(args)
+        return
+    if args.stage == "gp-mle":
+        (run_mle_reference if args.impl == "reference" else run_gp_mle)(args)
         return
     if args.impl == "reference":
         run_reference(args)

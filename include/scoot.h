@@ -8,6 +8,7 @@
  *   scoot_rf_predict     random-forest probability of feasibility, Eq. (3)
  *   scoot_gp_posterior   GP posterior mean and variance (Section 4.3)
  *   scoot_gp_prepare_device  the GP state (fp64 factorisation) on the device
+ *   scoot_gp_mle         GP hyperparameters by maximum likelihood (Section 4.3)
  *   scoot_acq_ei         expected improvement, Eq. (6)
  *   scoot_acq_ehvi       Monte-Carlo expected hypervolume improvement, Eq. (7)
  *   scoot_score_ei       posterior + EI in one kernel
@@ -276,6 +277,30 @@ scoot_status scoot_gp_prepare_device(scoot_ctx* ctx, const scoot_param* h_space,
                                      const uint32_t* obs, int64_t ld_obs, const float* y, const float* lengthscale,
                                      const float* signal_var, const float* noise_var, const float* warp,
                                      void* blob, void* work, int64_t work_bytes, void* stream);
+
+/* GP hyperparameters by maximum likelihood (Section 4.3 learns tau^2 this
+ * way), for every objective m and start s at once on the device.  theta =
+ * (ln l_1 .. ln l_d, ln s_f^2, ln tau^2), P = d + 2 values; the log marginal
+ * likelihood of the zero-mean GP with covariance s_f^2 k(r) + tau^2 I over
+ * the n observations (features as in scoot_gp_prepare, no warping) is
+ *   lml = -y^T K^{-1} y / 2 - log det K / 2 - n log(2 pi) / 2
+ * with gradient d lml / d theta_p = tr((alpha alpha^T - K^{-1}) dK/dtheta_p) / 2.
+ * From theta0 [S][M][P] (device, fp64) each (s, m) takes `steps` projected
+ * Adam ascent steps (beta1 0.9, beta2 0.999, eps 1e-8; step size
+ * lr (1 - t / steps) at step t; theta clipped to [h_lo, h_hi] (host [P])
+ * after each step; parameter p moves only if bit p of free_mask is set).
+ * Outputs (device, fp64): theta [S][M][P] after the last step, lml [S][M]
+ * there (-inf if K + tau^2 I stopped being positive definite, theta then
+ * being the last good one) and, if grad is not NULL, the gradient there
+ * [S][M][P].  obs: words [d][ld_obs]; y: [M][n] float32.  work: scratch of
+ * scoot_gp_mle_work_bytes bytes, 16-byte aligned.  S * M <= 65535.  A
+ * non-finite feature or y makes scoot_ctx_check return SCOOT_EINVAL. */
+scoot_status scoot_gp_mle(scoot_ctx* ctx, const scoot_param* h_space, int32_t d, const uint32_t* obs, int64_t ld_obs,
+                          int32_t n, const float* y, int32_t n_obj, int32_t kernel, const double* theta0,
+                          int32_t n_starts, const double* h_lo, const double* h_hi, uint32_t free_mask, int32_t steps,
+                          double lr, double* theta, double* lml, double* grad, void* work, int64_t work_bytes,
+                          void* stream);
+scoot_status scoot_gp_mle_work_bytes(int32_t n, int32_t d, int32_t n_obj, int32_t n_starts, int64_t* bytes);
 
 /* mean[m * ldo + i], var[m * ldo + i] for every candidate i < n and
  * objective m:  mu = k(x, X)(K + tau^2 I)^{-1} Y and

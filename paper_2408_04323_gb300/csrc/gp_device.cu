@@ -182,8 +182,11 @@ __global__ void __launch_bounds__(kKmatThreads) gp_kmat_kernel(const __grid_cons
     a.K[(int64_t)m * a.tri + t] = v;
 }
 
-// One block per objective: the factorisation with L^{-1} alongside, then
-// alpha, the best observed y and the fp32 tiles of L^{-1}.
+// The factorisation of the packed lower triangle A (n x n, K + tau^2 I on
+// entry) with the elimination applied to the identity in W, by the whole
+// block.  On return, row i of L^{-1} is W_i * rinv[i];
+// rinv2[i] = rinv[i]^2; A holds the eliminated values.  col: [2][n] scratch.
+// Returns false (in every thread) if a pivot is not positive and finite.
 //
 // Step j in a single multiply-add per entry: with g_i = A_ij / A_jj,
 //   A_ik -= g_i A_kj (j < k <= i)   and   W_ic -= g_i W_jc (c <= j),
@@ -191,28 +194,8 @@ __global__ void __launch_bounds__(kKmatThreads) gp_kmat_kernel(const __grid_cons
 // of a warp stay busy.  Column j is read from a contiguous copy (col), which
 // the threads that finish its entries in step j - 1 write (two buffers by
 // step parity).
-__global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_constant__ GpPrepArgs a) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    const int n = a.n, m = blockIdx.x;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = kCholThreads / 32;
-    double* rinv = reinterpret_cast<double*>(smem_raw);  // [n] 1 / pivot
-    double* rinv2 = rinv + n;                            // [n] 1 / pivot^2
-    double* z = rinv2 + n;                               // [n] L^{-1} y
-    double* col = z + n;                                 // [2][n] column j of A
-    double* A;
-    double* W;
-    if (n <= kSmemCholMaxN) {
-        A = col + 2 * n;
-        W = A + a.tri;
-        for (int64_t t = tid; t < a.tri; t += kCholThreads) A[t] = a.K[(int64_t)m * a.tri + t];
-        __syncthreads();
-    } else {
-        A = a.K + (int64_t)m * a.tri;
-        W = a.W + (int64_t)m * a.tri;
-    }
-    for (int i = warp; i < n; i += nwarps)
-        for (int c = lane; c <= i; c += 32) W[tri_idx(i, c)] = c == i ? 1.0 : 0.0;
-    for (int i = tid; i < n; i += kCholThreads) col[i] = A[tri_idx(i, 0)];
+__device__ bool eliminate(double* A, double* W, double* col, double* rinv, double* rinv2, int n) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = blockDim.x >> 5;
     // s_bad_at: the first step whose pivot is not positive (n if none).  It is
     // written during step j - 1 with the value j, so a thread still reading it
     // for step j - 1 does not stop early; every thread stops at step j.  The
@@ -220,6 +203,10 @@ __global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_cons
     // diagonal entry (fp64 square roots and divisions are slow here), and
     // read after the step's barrier.
     __shared__ int s_bad_at;
+    __syncthreads();  // A is complete; s_bad_at of an earlier call is read by no one
+    for (int i = warp; i < n; i += nwarps)
+        for (int c = lane; c <= i; c += 32) W[tri_idx(i, c)] = c == i ? 1.0 : 0.0;
+    for (int i = tid; i < n; i += (int)blockDim.x) col[i] = A[tri_idx(i, 0)];
     if (tid == 0) {
         const double s0 = A[0];
         const bool bad = !(s0 > 0.0) || !isfinite(s0);
@@ -259,7 +246,32 @@ __global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_cons
         }
         __syncthreads();
     }
-    if (s_bad_at < n) {  // read after the loop's last barrier: the same in every thread
+    const bool ok = s_bad_at >= n;  // read after the loop's last barrier: the same in every thread
+    __syncthreads();                // before a later call rewrites s_bad_at
+    return ok;
+}
+
+// One block per objective: the factorisation with L^{-1} alongside, then
+// alpha, the best observed y and the fp32 tiles of L^{-1}.
+__global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_constant__ GpPrepArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int n = a.n, m = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = kCholThreads / 32;
+    double* rinv = reinterpret_cast<double*>(smem_raw);  // [n] 1 / pivot
+    double* rinv2 = rinv + n;                            // [n] 1 / pivot^2
+    double* z = rinv2 + n;                               // [n] L^{-1} y
+    double* col = z + n;                                 // [2][n] column j of A
+    double* A;
+    double* W;
+    if (n <= kSmemCholMaxN) {
+        A = col + 2 * n;
+        W = A + a.tri;
+        for (int64_t t = tid; t < a.tri; t += kCholThreads) A[t] = a.K[(int64_t)m * a.tri + t];
+    } else {
+        A = a.K + (int64_t)m * a.tri;
+        W = a.W + (int64_t)m * a.tri;
+    }
+    if (!eliminate(A, W, col, rinv, rinv2, n)) {
         if (tid == 0) atomicOr(a.err, SCOOT_DEVERR_VALUE);
         return;
     }
@@ -300,6 +312,224 @@ __global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_cons
         if (row < n && c <= row) v = (float)(W[tri_idx(row, c)] * rinv[row]);
         tiles[e] = v;
     }
+}
+
+constexpr int kMleMaxP = SCOOT_MAX_DIM + 2;  // ln l_1 .. ln l_d, ln s_f^2, ln tau^2
+constexpr int kSmemMleMaxN = 128;             // A and W in shared memory up to this n
+constexpr int kMleThreads = 512;
+
+struct MleArgs {
+    int32_t n, d, M, P, kernel, S, steps;
+    int64_t tri;
+    uint32_t free_mask;                      // bit p: parameter p is fitted
+    uint32_t cat_mask;                       // bit c: parameter c is categorical
+    double lr;
+    double lo[kMleMaxP], hi[kMleMaxP];
+    const double* U;                         // [n][d] features (unscaled, unwarped)
+    const float* y;                          // [M][n]
+    const double* theta0;                    // [S][M][P]
+    double* theta;                           // [S][M][P]
+    double* lml;                             // [S][M]
+    double* grad;                            // [S][M][P] or nullptr
+    double* scratch;                         // [S M][2][tri] when n > kSmemMleMaxN
+};
+
+// Features of the observations, once per call: one thread per (j, c).
+__global__ void __launch_bounds__(kFeatThreads) mle_feat_kernel(const __grid_constant__ GpPrepArgs a) {
+    const int t = blockIdx.x * kFeatThreads + threadIdx.x;
+    const int j = t / a.d, c = t - j * a.d;
+    if (j >= a.n) return;
+    const uint32_t w = a.obs[(int64_t)c * a.ld_obs + j];
+    double u;
+    bool bad = false;
+    if (a.kind[c] == SCOOT_CATEGORICAL) {
+        u = (double)(int32_t)w;
+    } else {
+        const double v = a.kind[c] == SCOOT_CONTINUOUS ? (double)__uint_as_float(w) : (double)(int32_t)w;
+        bad = !isfinite(v) || (a.kind[c] == SCOOT_INT_LOG && !(v > 0.0));
+        if (a.kind[c] == SCOOT_INT_LOG) u = (log(v) - a.lo[c]) / a.span[c];
+        else u = a.span[c] > 0.0 ? (v - a.lo[c]) / a.span[c] : 0.0;
+    }
+    a.U[(int64_t)j * a.d + c] = u;
+    if (c == 0)
+        for (int m = 0; m < a.M; ++m) bad |= !isfinite(a.y[(int64_t)m * a.n + j]);
+    if (bad) atomicOr(a.err, SCOOT_DEVERR_VALUE);
+}
+
+// k(r) / s_f^2 and its derivative in r^2 for r^2 = r2.
+__device__ __forceinline__ void matern_slope(double r2, int kernel, double* k, double* dk) {
+    const double r = sqrt(r2);
+    if (kernel == SCOOT_MATERN32) {
+        const double a = 1.7320508075688772 * r, e = exp(-a);
+        *k = (1.0 + a) * e;
+        *dk = -1.5 * e;
+    } else {
+        const double a = 2.23606797749979 * r, e = exp(-a);
+        *k = (1.0 + a + a * a / 3.0) * e;
+        *dk = -(5.0 / 6.0) * (1.0 + a) * e;
+    }
+}
+
+// One block per (start s, objective m): `steps` projected Adam steps on the
+// log marginal likelihood (beta1 0.9, beta2 0.999, eps 1e-8, step size
+// lr (1 - t / steps)), then the likelihood and gradient at the result.  Each
+// evaluation: K + tau^2 I from the features, the factorisation with L^{-1},
+// alpha = K^{-1} y, K^{-1} = L^{-T} L^{-1} (into A), and
+// d lml / d theta_p = sum_{i >= j} w_ij (alpha_i alpha_j - K^{-1}_ij) dK_ij / dtheta_p
+// with w = 1 off the diagonal and 1/2 on it.
+__global__ void __launch_bounds__(kMleThreads) gp_mle_kernel(const __grid_constant__ MleArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int n = a.n, d = a.d, P = a.P;
+    const int sm = blockIdx.x, m = sm % a.M;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = kMleThreads / 32;
+    double* rinv = reinterpret_cast<double*>(smem_raw);  // [n]
+    double* rinv2 = rinv + n;                            // [n]
+    double* yv = rinv2 + n;                              // [n]
+    double* z = yv + n;                                  // [n] L^{-1} y
+    double* al = z + n;                                  // [n] alpha
+    double* col = al + n;                                // [2][n]
+    double* U = col + 2 * n;                             // [n][d]
+    double* A;
+    double* W;
+    if (n <= kSmemMleMaxN) {
+        A = U + (size_t)n * d;
+        W = A + a.tri;
+    } else {
+        A = a.scratch + (size_t)sm * 2 * a.tri;
+        W = A + a.tri;
+    }
+    __shared__ double th[kMleMaxP], m1[kMleMaxP], m2[kMleMaxP], g[kMleMaxP];
+    __shared__ double il2[SCOOT_MAX_DIM];  // 1 / l_c^2
+    __shared__ double s_sf2, s_tau2;
+    __shared__ double red[kMleThreads / 32][kMleMaxP + 1];
+    __shared__ double s_total;  // y^T alpha + log det K
+    __shared__ int s_fail;
+    for (int i = tid; i < n; i += kMleThreads) yv[i] = (double)a.y[(int64_t)m * n + i];
+    for (int t = tid; t < n * d; t += kMleThreads) U[t] = a.U[t];
+    if (tid < P) {
+        th[tid] = a.theta0[(int64_t)sm * P + tid];
+        m1[tid] = 0.0;
+        m2[tid] = 0.0;
+    }
+    if (tid == 0) s_fail = 0;
+    double lml = 0.0;
+    for (int it = 0; it <= a.steps; ++it) {
+        __syncthreads();
+        if (tid < d) il2[tid] = exp(-2.0 * th[tid]);
+        if (tid == 0) {
+            s_sf2 = exp(th[d]);
+            s_tau2 = exp(th[d + 1]);
+        }
+        __syncthreads();
+        const double sf2 = s_sf2, tau2 = s_tau2;
+        // K + tau^2 I
+        for (int64_t t = tid; t < a.tri; t += kMleThreads) {
+            int i = (int)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
+            while ((int64_t)i * (i + 1) / 2 > t) --i;
+            while ((int64_t)(i + 1) * (i + 2) / 2 <= t) ++i;
+            const int k = (int)(t - (int64_t)i * (i + 1) / 2);
+            double r2 = 0.0;
+            for (int c = 0; c < d; ++c) {
+                const double df = U[i * d + c] - U[k * d + c];
+                r2 += ((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c];
+            }
+            double kv, dk;
+            matern_slope(r2, a.kernel, &kv, &dk);
+            A[t] = sf2 * kv + (i == k ? tau2 : 0.0);
+        }
+        if (!eliminate(A, W, col, rinv, rinv2, n)) {
+            if (tid == 0) s_fail = 1;
+            __syncthreads();
+            break;
+        }
+        // z = L^{-1} y (a warp per row), then alpha = L^{-T} z (a thread per column)
+        for (int i = warp; i < n; i += nwarps) {
+            const double* Wi = W + tri_idx(i, 0);
+            double t = 0.0;
+            for (int c = lane; c <= i; c += 32) t += Wi[c] * yv[c];
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            if (lane == 0) z[i] = t * rinv[i];
+        }
+        __syncthreads();
+        for (int c = tid; c < n; c += kMleThreads) {
+            double t = 0.0;
+            for (int i = c; i < n; ++i) t += W[tri_idx(i, c)] * rinv[i] * z[i];
+            al[c] = t;
+        }
+        // K^{-1} into A: (i, j <= i) = sum_{k >= i} L^{-1}_ki L^{-1}_kj
+        for (int64_t t = tid; t < a.tri; t += kMleThreads) {
+            int i = (int)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
+            while ((int64_t)i * (i + 1) / 2 > t) --i;
+            while ((int64_t)(i + 1) * (i + 2) / 2 <= t) ++i;
+            const int j = (int)(t - (int64_t)i * (i + 1) / 2);
+            double v = 0.0;
+            for (int k = i; k < n; ++k) v += W[tri_idx(k, i)] * W[tri_idx(k, j)] * rinv2[k];
+            A[t] = v;
+        }
+        __syncthreads();
+        // gradient terms and the likelihood's two sums, per thread
+        double acc[kMleMaxP + 1];
+        for (int p = 0; p <= P; ++p) acc[p] = 0.0;
+        for (int64_t t = tid; t < a.tri; t += kMleThreads) {
+            int i = (int)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
+            while ((int64_t)i * (i + 1) / 2 > t) --i;
+            while ((int64_t)(i + 1) * (i + 2) / 2 <= t) ++i;
+            const int k = (int)(t - (int64_t)i * (i + 1) / 2);
+            const double w = (al[i] * al[k] - A[t]) * (i == k ? 0.5 : 1.0);
+            if (i == k) {
+                acc[d + 1] += w * tau2;
+                acc[d] += w * sf2;  // k(0) = 1
+                continue;
+            }
+            double r2 = 0.0;
+            for (int c = 0; c < d; ++c) {
+                const double df = U[i * d + c] - U[k * d + c];
+                r2 += ((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c];
+            }
+            double kv, dk;
+            matern_slope(r2, a.kernel, &kv, &dk);
+            const double f = -2.0 * sf2 * dk * w;
+            for (int c = 0; c < d; ++c) {  // the feature's term of r^2 again
+                const double df = U[i * d + c] - U[k * d + c];
+                acc[c] += f * (((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c]);
+            }
+            acc[d] += w * sf2 * kv;
+        }
+        for (int i = tid; i < n; i += kMleThreads) acc[P] += yv[i] * al[i] - 2.0 * log(rinv[i]);
+        // y^T alpha + log det K in acc[P]; block reduction of P + 1 sums
+        for (int p = 0; p <= P; ++p) {
+            double v = acc[p];
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            if (lane == 0) red[warp][p] = v;
+        }
+        __syncthreads();
+        if (tid <= P) {
+            double v = 0.0;
+            for (int w2 = 0; w2 < nwarps; ++w2) v += red[w2][tid];
+            if (tid < P) g[tid] = v;
+            else s_total = v;
+        }
+        __syncthreads();
+        lml = -0.5 * s_total - 0.5 * n * 1.8378770664093453;  // log(2 pi)
+        if (it == a.steps) break;
+        if (tid == 0) {  // projected Adam step on the free parameters
+            const double step = a.lr * (1.0 - (double)it / a.steps);
+            const double c1 = 1.0 - pow(0.9, it + 1), c2 = 1.0 - pow(0.999, it + 1);
+            for (int p = 0; p < P; ++p) {
+                if (!((a.free_mask >> p) & 1u)) continue;
+                const double gp = g[p];
+                m1[p] = 0.9 * m1[p] + 0.1 * gp;
+                m2[p] = 0.999 * m2[p] + 0.001 * gp * gp;
+                const double upd = step * (m1[p] / c1) / (sqrt(m2[p] / c2) + 1e-8);
+                th[p] = fmin(fmax(th[p] + upd, a.lo[p]), a.hi[p]);
+            }
+        }
+    }
+    if (tid < P) {
+        a.theta[(int64_t)sm * P + tid] = th[tid];
+        if (a.grad) a.grad[(int64_t)sm * P + tid] = s_fail ? 0.0 : g[tid];
+    }
+    if (tid == 0) a.lml[sm] = s_fail ? -INFINITY : lml;
 }
 
 }  // namespace
@@ -415,6 +645,101 @@ scoot_status scoot_gp_prepare_device(scoot_ctx* ctx, const scoot_param* h_space,
     const size_t smem = (size_t)5 * n * sizeof(double) + (in_smem ? (size_t)2 * a.tri * sizeof(double) : 0);
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(gp_chol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     gp_chol_kernel<<<M, kCholThreads, smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+scoot_status scoot_gp_mle_work_bytes(int32_t n, int32_t d, int32_t n_obj, int32_t n_starts, int64_t* bytes) {
+    if (!bytes || n < 1 || d < 1 || n_obj < 1 || n_starts < 1) return SCOOT_EINVAL;
+    const int64_t tri = (int64_t)n * (n + 1) / 2;
+    int64_t b = ((int64_t)n * d * 8 + 255) / 256 * 256;
+    if (n > kSmemMleMaxN) b += (int64_t)n_starts * n_obj * 2 * tri * 8;
+    *bytes = b;
+    return SCOOT_OK;
+}
+
+scoot_status scoot_gp_mle(scoot_ctx* ctx, const scoot_param* h_space, int32_t d, const uint32_t* obs, int64_t ld_obs,
+                          int32_t n, const float* y, int32_t n_obj, int32_t kernel, const double* theta0,
+                          int32_t n_starts, const double* h_lo, const double* h_hi, uint32_t free_mask, int32_t steps,
+                          double lr, double* theta, double* lml, double* grad, void* work, int64_t work_bytes,
+                          void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    if (!h_space || !h_lo || !h_hi) return scoot_fail(ctx, SCOOT_EINVAL, "h_space, h_lo or h_hi is NULL");
+    if (d < 1 || d > SCOOT_MAX_DIM) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "d = %d outside 1..%d", d, SCOOT_MAX_DIM);
+    if (n < 1 || n > SCOOT_MAX_OBS) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n = %d outside 1..%d", n, SCOOT_MAX_OBS);
+    if (n_obj < 1 || n_obj > SCOOT_MAX_OBJ) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n_obj = %d", n_obj);
+    if (kernel != SCOOT_MATERN52 && kernel != SCOOT_MATERN32) return scoot_fail(ctx, SCOOT_EINVAL, "kernel %d", kernel);
+    if (n_starts < 1 || (int64_t)n_starts * n_obj > 65535)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n_starts = %d", n_starts);
+    if (steps < 0 || !(lr >= 0.0) || !std::isfinite(lr)) return scoot_fail(ctx, SCOOT_EINVAL, "steps or lr");
+    if (ld_obs < n) return scoot_fail(ctx, SCOOT_EINVAL, "ld_obs = %lld < n", (long long)ld_obs);
+    if (!obs || !y || !theta0 || !theta || !lml) return scoot_fail(ctx, SCOOT_EINVAL, "a device array is NULL");
+    const int P = d + 2;
+    MleArgs a;
+    std::memset(&a, 0, sizeof(a));
+    for (int p = 0; p < P; ++p) {
+        if (!std::isfinite(h_lo[p]) || !std::isfinite(h_hi[p]) || h_lo[p] > h_hi[p])
+            return scoot_fail(ctx, SCOOT_EINVAL, "bounds of parameter %d", p);
+        a.lo[p] = h_lo[p];
+        a.hi[p] = h_hi[p];
+    }
+    GpPrepArgs f;
+    std::memset(&f, 0, sizeof(f));
+    for (int c = 0; c < d; ++c) {
+        const scoot_param& p = h_space[c];
+        f.kind[c] = p.kind;
+        if (p.kind == SCOOT_CATEGORICAL) {
+            if (p.n_choices < 1) return scoot_fail(ctx, SCOOT_EINVAL, "parameter %d: n_choices", c);
+            a.cat_mask |= 1u << c;
+        } else if (p.kind == SCOOT_INT_LOG) {
+            if (!(p.lo > 0.0f) || !(p.hi > p.lo)) return scoot_fail(ctx, SCOOT_EINVAL, "parameter %d: log range", c);
+            f.lo[c] = std::log((double)p.lo);
+            f.span[c] = std::log((double)p.hi) - std::log((double)p.lo);
+        } else if (p.kind == SCOOT_INT_UNIFORM || p.kind == SCOOT_CONTINUOUS) {
+            f.lo[c] = p.lo;
+            f.span[c] = (double)p.hi - (double)p.lo;
+        } else {
+            return scoot_fail(ctx, SCOOT_EINVAL, "parameter %d: kind %d", c, p.kind);
+        }
+    }
+    int64_t need = 0;
+    scoot_gp_mle_work_bytes(n, d, n_obj, n_starts, &need);
+    if (!work || work_bytes < need || !scoot_aligned16(work))
+        return scoot_fail(ctx, SCOOT_EINVAL, "work needs %lld bytes, 16-byte aligned", (long long)need);
+    char* ws = static_cast<char*>(work);
+    f.n = n;
+    f.d = d;
+    f.obs = obs;
+    f.ld_obs = ld_obs;
+    f.U = reinterpret_cast<double*>(ws);
+    f.M = n_obj;
+    f.y = y;
+    f.err = ctx->d_err;
+    a.n = n;
+    a.d = d;
+    a.M = n_obj;
+    a.P = P;
+    a.kernel = kernel;
+    a.S = n_starts;
+    a.steps = steps;
+    a.tri = (int64_t)n * (n + 1) / 2;
+    a.free_mask = free_mask & ((1u << P) - 1u);
+    a.lr = lr;
+    a.U = f.U;
+    a.y = y;
+    a.theta0 = theta0;
+    a.theta = theta;
+    a.lml = lml;
+    a.grad = grad;
+    a.scratch = n > kSmemMleMaxN ? reinterpret_cast<double*>(ws + ((int64_t)n * d * 8 + 255) / 256 * 256) : nullptr;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    mle_feat_kernel<<<(n * d + kFeatThreads - 1) / kFeatThreads, kFeatThreads, 0, st>>>(f);
+    SCOOT_LAUNCHED(ctx);
+    const size_t smem = (size_t)(7 * n + (size_t)n * d) * sizeof(double) +
+                        (n <= kSmemMleMaxN ? (size_t)2 * a.tri * sizeof(double) : 0);
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(gp_mle_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    gp_mle_kernel<<<n_starts * n_obj, kMleThreads, smem, st>>>(a);
     SCOOT_LAUNCHED(ctx);
     return SCOOT_OK;
 }

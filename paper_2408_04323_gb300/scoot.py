@@ -99,6 +99,9 @@ _PROTOS = {
     "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_prepare_warped": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_device_work_bytes": [C.POINTER(scoot_gp_layout), C.POINTER(_i64)],
+    "scoot_gp_mle": [_vp, _vp, _i32, _vp, _i64, _i32, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _u32, _i32,
+                     C.c_double, _vp, _vp, _vp, _vp, _i64, _vp],
+    "scoot_gp_mle_work_bytes": [_i32, _i32, _i32, _i32, C.POINTER(_i64)],
     "scoot_round_state_build": [C.POINTER(scoot_round_inputs), _vp, _i64, C.POINTER(scoot_round_state)],
     "scoot_gp_prepare_device": [_vp, _vp, C.POINTER(scoot_gp_layout), _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                 _i64, _vp],
@@ -556,6 +559,34 @@ def scoot_gp_prepare_device(ctx, h_space, layout, obs, y, lengthscale, signal_va
                                          _dev(blob, torch.uint8, "blob"), _dev(work, torch.uint8, "work"),
                                          int(work.numel()), _stream(stream)),
            "scoot_gp_prepare_device", _h(ctx))
+
+
+def scoot_gp_mle_work_bytes(n: int, d: int, n_obj: int, n_starts: int) -> int:
+    v = _i64()
+    _check(lib().scoot_gp_mle_work_bytes(int(n), int(d), int(n_obj), int(n_starts), C.byref(v)),
+           "scoot_gp_mle_work_bytes")
+    return int(v.value)
+
+
+def scoot_gp_mle(ctx, h_space, obs, n, y, theta0, h_lo, h_hi, free_mask, steps, lr, theta, lml, grad=None,
+                 kernel=0, work=None, stream=None):
+    """obs int32 [d][ld]; y float32 [M][n]; theta0 / theta float64 [S][M][d+2];
+    lml float64 [S][M]; grad float64 [S][M][d+2] or None (all device);
+    h_lo / h_hi host float64 [d+2]."""
+    import torch
+    S_, M = int(theta0.shape[0]), int(y.shape[0])
+    d = len(h_space)
+    if work is None:
+        work = torch.empty(scoot_gp_mle_work_bytes(n, d, M, S_), dtype=torch.uint8, device=obs.device)
+    lo = np.ascontiguousarray(h_lo, np.float64)
+    hi = np.ascontiguousarray(h_hi, np.float64)
+    _check(lib().scoot_gp_mle(_h(ctx), _host(h_space, 16, name="h_space"), d, _dev(obs, torch.int32, "obs"),
+                              int(obs.shape[1]), int(n), _dev(y, torch.float32, "y"), M, int(kernel),
+                              _dev(theta0, torch.float64, "theta0"), S_, _host(lo), _host(hi),
+                              int(free_mask) & 0xFFFFFFFF, int(steps), float(lr), _dev(theta, torch.float64, "theta"),
+                              _dev(lml, torch.float64, "lml"), _dev(grad, torch.float64, "grad"),
+                              _dev(work, torch.uint8, "work"), int(work.numel()), _stream(stream)),
+           "scoot_gp_mle", _h(ctx))
 
 
 def scoot_rf_train_work_bytes(n: int, d: int) -> int:
