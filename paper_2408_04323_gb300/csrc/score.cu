@@ -208,6 +208,9 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 template <int EPI, int M, int DO>
 __global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 5 : 1)
 score_kernel(const __grid_constant__ ScoreArgs a) {
+    // Five blocks per SM for the 2-objective EHVI of <= 8 parameters caps
+    // registers at 96.
+    constexpr bool kRegCapped = EPI == kEHVI && M == 2 && DO == 8;
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
     // Ks, and after the posterior the exact-EHVI psi table [psi_rows][kTC]
@@ -333,11 +336,14 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             const float4* Ks4 = reinterpret_cast<const float4*>(Ks);
             int t = 0;
             for (int rb = 0; rb < a.n_rb; ++rb) {
-                float accm[8][4];
+                // accumulators in column pairs: acc2[r][cp] = (V[r][2 cp], V[r][2 cp + 1]),
+                // updated by packed fp32 FMAs (two per instruction, each lane
+                // rounded as fmaf): the k loads give the candidate pairs, the
+                // row's L^{-1} value is broadcast to both lanes, one row at a
+                // time (so that only one broadcast pair is live).
+                float2 acc2[8][2];
 #pragma unroll
-                for (int r = 0; r < 8; ++r)
-#pragma unroll
-                    for (int c = 0; c < 4; ++c) accm[r][c] = 0.0f;
+                for (int r = 0; r < 8; ++r) acc2[r][0] = acc2[r][1] = make_float2(0.0f, 0.0f);
                 for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t) {
                     // Tile t has landed in buffer t&1 and every thread is done
                     // with tile t-1, so tile t+1 may overwrite buffer (t+1)&1
@@ -359,13 +365,30 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                         const float4 k4 = Ks4[(j0 + jj) * (kTC / 4) + cg];
                         const float4 l0 = Lt4[jj * (kRB / 4) + rg * 2];
                         const float4 l1 = Lt4[jj * (kRB / 4) + rg * 2 + 1];
-                        const float kv[4] = {k4.x, k4.y, k4.z, k4.w};
+                        const float2 k01 = make_float2(k4.x, k4.y), k23 = make_float2(k4.z, k4.w);
                         const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
 #pragma unroll
-                        for (int r = 0; r < 8; ++r)
-#pragma unroll
-                            for (int c = 0; c < 4; ++c) accm[r][c] = fmaf(lv[r], kv[c], accm[r][c]);
+                        for (int r = 0; r < 8; ++r) {
+                            if (kRegCapped) {  // scalar FMAs: the broadcast pairs would spill at 96 registers
+                                acc2[r][0].x = fmaf(lv[r], k4.x, acc2[r][0].x);
+                                acc2[r][0].y = fmaf(lv[r], k4.y, acc2[r][0].y);
+                                acc2[r][1].x = fmaf(lv[r], k4.z, acc2[r][1].x);
+                                acc2[r][1].y = fmaf(lv[r], k4.w, acc2[r][1].y);
+                            } else {
+                                const float2 lb = make_float2(lv[r], lv[r]);
+                                acc2[r][0] = __ffma2_rn(lb, k01, acc2[r][0]);
+                                acc2[r][1] = __ffma2_rn(lb, k23, acc2[r][1]);
+                            }
+                        }
                     }
+                }
+                float accm[8][4];
+#pragma unroll
+                for (int r = 0; r < 8; ++r) {
+                    accm[r][0] = acc2[r][0].x;
+                    accm[r][1] = acc2[r][0].y;
+                    accm[r][2] = acc2[r][1].x;
+                    accm[r][3] = acc2[r][1].y;
                 }
 #pragma unroll
                 for (int r = 0; r < 8; ++r)
