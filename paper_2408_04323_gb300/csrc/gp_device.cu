@@ -388,7 +388,7 @@ __global__ void __launch_bounds__(kMleThreads) gp_mle_kernel(const __grid_consta
     double* z = yv + n;                                  // [n] L^{-1} y
     double* al = z + n;                                  // [n] alpha
     double* col = al + n;                                // [2][n]
-    double* U = col + 2 * n;                             // [n][d]
+    double* U = col + 2 * n;                             // [d][n]: feature c of observation j at c n + j
     double* A;
     double* W;
     if (n <= kSmemMleMaxN) {
@@ -405,7 +405,10 @@ __global__ void __launch_bounds__(kMleThreads) gp_mle_kernel(const __grid_consta
     __shared__ double s_total;  // y^T alpha + log det K
     __shared__ int s_fail;
     for (int i = tid; i < n; i += kMleThreads) yv[i] = (double)a.y[(int64_t)m * n + i];
-    for (int t = tid; t < n * d; t += kMleThreads) U[t] = a.U[t];
+    for (int t = tid; t < n * d; t += kMleThreads) {  // transposed, so that lanes on consecutive
+        const int j = t / d, c = t - j * d;           // observations read consecutive words
+        U[c * n + j] = a.U[t];
+    }
     if (tid < P) {
         th[tid] = a.theta0[(int64_t)sm * P + tid];
         m1[tid] = 0.0;
@@ -430,7 +433,7 @@ __global__ void __launch_bounds__(kMleThreads) gp_mle_kernel(const __grid_consta
             const int k = (int)(t - (int64_t)i * (i + 1) / 2);
             double r2 = 0.0;
             for (int c = 0; c < d; ++c) {
-                const double df = U[i * d + c] - U[k * d + c];
+                const double df = U[c * n + i] - U[c * n + k];
                 r2 += ((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c];
             }
             double kv, dk;
@@ -469,7 +472,8 @@ __global__ void __launch_bounds__(kMleThreads) gp_mle_kernel(const __grid_consta
         __syncthreads();
         // gradient terms and the likelihood's two sums, per thread
         double acc[kMleMaxP + 1];
-        for (int p = 0; p <= P; ++p) acc[p] = 0.0;
+#pragma unroll
+        for (int p = 0; p <= kMleMaxP; ++p) acc[p] = 0.0;
         for (int64_t t = tid; t < a.tri; t += kMleThreads) {
             int i = (int)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
             while ((int64_t)i * (i + 1) / 2 > t) --i;
@@ -477,37 +481,44 @@ __global__ void __launch_bounds__(kMleThreads) gp_mle_kernel(const __grid_consta
             const int k = (int)(t - (int64_t)i * (i + 1) / 2);
             const double w = (al[i] * al[k] - A[t]) * (i == k ? 0.5 : 1.0);
             if (i == k) {
-                acc[d + 1] += w * tau2;
-                acc[d] += w * sf2;  // k(0) = 1
+                acc[kMleMaxP - 1] += w * tau2;
+                acc[kMleMaxP - 2] += w * sf2;  // k(0) = 1
                 continue;
             }
             double r2 = 0.0;
             for (int c = 0; c < d; ++c) {
-                const double df = U[i * d + c] - U[k * d + c];
+                const double df = U[c * n + i] - U[c * n + k];
                 r2 += ((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c];
             }
             double kv, dk;
             matern_slope(r2, a.kernel, &kv, &dk);
             const double f = -2.0 * sf2 * dk * w;
-            for (int c = 0; c < d; ++c) {  // the feature's term of r^2 again
-                const double df = U[i * d + c] - U[k * d + c];
-                acc[c] += f * (((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c]);
+#pragma unroll
+            for (int c = 0; c < SCOOT_MAX_DIM; ++c) {  // the feature's term of r^2 again (unrolled:
+                if (c < d) {                           // acc stays in registers)
+                    const double df = U[c * n + i] - U[c * n + k];
+                    acc[c] += f * (((a.cat_mask >> c) & 1u) ? (df != 0.0 ? il2[c] : 0.0) : df * df * il2[c]);
+                }
             }
-            acc[d] += w * sf2 * kv;
+            acc[kMleMaxP - 2] += w * sf2 * kv;
         }
-        for (int i = tid; i < n; i += kMleThreads) acc[P] += yv[i] * al[i] - 2.0 * log(rinv[i]);
-        // y^T alpha + log det K in acc[P]; block reduction of P + 1 sums
-        for (int p = 0; p <= P; ++p) {
+        for (int i = tid; i < n; i += kMleThreads) acc[kMleMaxP] += yv[i] * al[i] - 2.0 * log(rinv[i]);
+        // acc: lengthscales in 0 .. d-1, s_f^2 and tau^2 at kMleMaxP - 2 and - 1, and
+        // y^T alpha + log det K at kMleMaxP; block reduction of the sums
+#pragma unroll
+        for (int p = 0; p <= kMleMaxP; ++p) {
             double v = acc[p];
             for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
             if (lane == 0) red[warp][p] = v;
         }
         __syncthreads();
-        if (tid <= P) {
+        if (tid <= kMleMaxP) {
             double v = 0.0;
             for (int w2 = 0; w2 < nwarps; ++w2) v += red[w2][tid];
-            if (tid < P) g[tid] = v;
-            else s_total = v;
+            if (tid < d) g[tid] = v;
+            else if (tid == kMleMaxP - 2) g[d] = v;
+            else if (tid == kMleMaxP - 1) g[d + 1] = v;
+            else if (tid == kMleMaxP) s_total = v;
         }
         __syncthreads();
         lml = -0.5 * s_total - 0.5 * n * 1.8378770664093453;  // log(2 pi)
