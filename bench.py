@@ -72,8 +72,9 @@ def parse_args():
     p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
-    p.add_argument("--gp-prep", choices=["host", "device"], default="host",
-                   help="where the end-to-end step builds the GP state (fp64 factorisation)")
+    p.add_argument("--gp-prep", choices=["auto", "host", "device"], default="auto",
+                   help="where the end-to-end step builds the GP state (fp64 factorisation); auto: the "
+                        "device from 100 observations (measured faster there), the host below")
     p.add_argument("--stage", choices=["round", "rf-train", "gp-mle"], default="round",
                    help="rf-train: the training of the workload's feasibility forest; gp-mle: its GP "
                         "hyperparameter fit (32 starts x 100 Adam steps); instead of a round")
@@ -679,7 +680,7 @@ def main():
     if args.warp and w.fantasy:
         raise SystemExit("--warp: fantasy picks take unwarped GP states")
     ctx = S.Context(device.index)
-    gp_dev = args.gp_prep == "device" and not inp.fantasy
+    gp_dev = (args.gp_prep == "device" or (args.gp_prep == "auto" and w.n_obs >= 100)) and not inp.fantasy
     rnd = ScoringRound(ctx, inp, N, device, gp_on_device=gp_dev)
     cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
     stream = torch.cuda.current_stream(device)

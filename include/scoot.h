@@ -302,6 +302,23 @@ scoot_status scoot_gp_mle(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
                           void* stream);
 scoot_status scoot_gp_mle_work_bytes(int32_t n, int32_t d, int32_t n_obj, int32_t n_starts, int64_t* bytes);
 
+/* One device buffer for scoot_gp_prepare_device_from_host: the uploaded
+ * inputs (upload_bytes), the blob at blob_off, the scratch at work_off;
+ * total_bytes in all (256-byte aligned parts). */
+scoot_status scoot_gp_device_buffer_layout(const scoot_gp_layout* layout, int32_t warped, int64_t* upload_bytes,
+                                           int64_t* blob_off, int64_t* work_off, int64_t* total_bytes);
+/* scoot_gp_prepare_device from host inputs (the arguments of
+ * scoot_gp_prepare_warped; h_warp may be NULL): packs them into h_stage
+ * (pinned host memory of at least upload_bytes, free to reuse once `stream`
+ * has passed this call), copies them to the start of buf (device,
+ * total_bytes of scoot_gp_device_buffer_layout) and launches the device
+ * build into buf + blob_off, all asynchronously on `stream`. */
+scoot_status scoot_gp_prepare_device_from_host(scoot_ctx* ctx, const scoot_param* h_space, const scoot_gp_layout* layout,
+                                               const uint32_t* h_x_obs, int64_t ld_obs, const float* h_y,
+                                               const float* h_lengthscale, const float* h_signal_var,
+                                               const float* h_noise_var, const float* h_warp, void* h_stage,
+                                               void* buf, int64_t buf_bytes, void* stream);
+
 /* mean[m * ldo + i], var[m * ldo + i] for every candidate i < n and
  * objective m:  mu = k(x, X)(K + tau^2 I)^{-1} Y and
  * sigma^2 = k(x, x) - k(x, X)(K + tau^2 I)^{-1} k(X, x) (latent f, clamped

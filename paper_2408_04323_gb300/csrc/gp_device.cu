@@ -15,6 +15,8 @@
 #include <cstring>
 #include <vector>
 
+#include <cooperative_groups.h>
+
 #include "internal.h"
 
 namespace {
@@ -312,6 +314,171 @@ __global__ void __launch_bounds__(kCholThreads) gp_chol_kernel(const __grid_cons
         if (row < n && c <= row) v = (float)(W[tri_idx(row, c)] * rinv[row]);
         tiles[e] = v;
     }
+}
+
+constexpr int kClusterCTAs = 8;          // CTAs sharing one factorisation (portable cluster size)
+constexpr int kClusterThreads = 256;
+constexpr int kClusterMaxN = 384;        // rows of A and W split over the cluster's shared memory
+
+// Offset of local row li (global row rank + C li) in a CTA's packed rows:
+// row i holds i + 1 entries.
+__device__ __forceinline__ int64_t local_row_off(int li, int rank) {
+    return (int64_t)li * (rank + 1) + (int64_t)kClusterCTAs * li * (li - 1) / 2;
+}
+
+// The factorisation of gp_chol_kernel spread over a cluster of kClusterCTAs
+// CTAs (one cluster per objective): CTA r owns rows i = r (mod C) of A and
+// W in its shared memory.  What a step needs from other rows travels through
+// distributed shared memory before the step's cluster barrier: the thread
+// that finishes A_i,j+1 stores it into every CTA's copy of the next pivot
+// column, the row j+1 of W is stored the same way as its entries become
+// final, and the thread that finishes the next diagonal entry stores its
+// reciprocals (or the failure) everywhere.  Then z = L^{-1} y per owned row
+// (broadcast), per-CTA partial sums of alpha = L^{-T} z over owned rows
+// (added in rank order by CTA 0), and each CTA writes its rows' tiles.
+__global__ void __cluster_dims__(kClusterCTAs, 1, 1) __launch_bounds__(kClusterThreads)
+gp_chol_cluster_kernel(const __grid_constant__ GpPrepArgs a) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int n = a.n, C = kClusterCTAs;
+    const int rank = (int)cluster.block_rank(), m = blockIdx.x / C;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = kClusterThreads / 32;
+    double* rinv = reinterpret_cast<double*>(smem_raw);  // [n]
+    double* rinv2 = rinv + n;                            // [n]
+    double* col = rinv2 + n;                             // [2][n] pivot column
+    double* wrow = col + 2 * n;                          // [2][n] row j of W
+    double* z = wrow + 2 * n;                            // [n]
+    double* part = z + n;                                // [n] this CTA's share of alpha
+    const int nl = (n - rank + C - 1) / C;               // rows owned
+    double* A = part + n;                                // owned rows, packed
+    double* W = A + local_row_off(nl, rank);
+    __shared__ int s_bad_at;
+    const double* K = a.K + (int64_t)m * a.tri;
+    // load owned rows; W = I
+    for (int li = warp; li < nl; li += nwarps) {
+        const int i = rank + C * li;
+        const int64_t o = local_row_off(li, rank);
+        for (int t = lane; t <= i; t += 32) {
+            A[o + t] = K[tri_idx(i, t)];
+            W[o + t] = t == i ? 1.0 : 0.0;
+        }
+    }
+    // the first pivot column, row 0 of W and the first pivot, everywhere
+    for (int li = tid; li < nl; li += kClusterThreads) {
+        const int i = rank + C * li;
+        const double v = K[tri_idx(i, 0)];
+        for (int r = 0; r < C; ++r) cluster.map_shared_rank(col, r)[i] = v;
+    }
+    if (tid == 0) {
+        const double s0 = K[0];
+        const bool bad = !(s0 > 0.0) || !isfinite(s0);
+        s_bad_at = bad ? 0 : n;
+        rinv[0] = bad ? 0.0 : rsqrt_newton(s0);
+        rinv2[0] = rinv[0] * rinv[0];
+        wrow[0] = 1.0;
+    }
+    cluster.sync();
+    for (int j = 0; j < n; ++j) {
+        if (s_bad_at <= j) break;  // the same in every thread of the cluster
+        const double r2 = rinv2[j];
+        const double* cj = col + (j & 1) * n;
+        const double* wj = wrow + (j & 1) * n;
+        const int nb = (j + 1) & 1;
+        // owned rows i > j
+        int li0 = (j + 1 - rank + C - 1) / C;
+        if (li0 < 0) li0 = 0;
+        for (int li = li0 + warp; li < nl; li += nwarps) {
+            const int i = rank + C * li;
+            const int64_t o = local_row_off(li, rank);
+            const double g = cj[i] * r2;
+            for (int t = lane; t <= i; t += 32) {
+                double* dst = t <= j ? W + o + t : A + o + t;
+                const double src = t <= j ? wj[t] : cj[t];
+                const double v = *dst - g * src;
+                *dst = v;
+                if (t == j + 1) {  // A_i,j+1 is final: the next pivot column, everywhere
+                    for (int r = 0; r < C; ++r) cluster.map_shared_rank(col + nb * n, r)[i] = v;
+                    if (i == j + 1) {
+                        if (!(v > 0.0) || !isfinite(v)) {
+                            for (int r = 0; r < C; ++r) *cluster.map_shared_rank(&s_bad_at, r) = j + 1;
+                        } else {
+                            const double y = rsqrt_newton(v);
+                            for (int r = 0; r < C; ++r) {
+                                cluster.map_shared_rank(rinv, r)[j + 1] = y;
+                                cluster.map_shared_rank(rinv2, r)[j + 1] = y * y;
+                            }
+                        }
+                    }
+                }
+                if (i == j + 1 && t <= j)  // W_j+1,t is final: row j + 1 of W, everywhere
+                    for (int r = 0; r < C; ++r) cluster.map_shared_rank(wrow + nb * n, r)[t] = v;
+            }
+            if (i == j + 1 && lane == 0)
+                for (int r = 0; r < C; ++r) cluster.map_shared_rank(wrow + nb * n, r)[j + 1] = 1.0;
+        }
+        cluster.sync();
+    }
+    if (s_bad_at < n) {  // the same everywhere; no shared memory of another CTA is touched after this
+        if (tid == 0 && rank == 0) atomicOr(a.err, SCOOT_DEVERR_VALUE);
+        return;
+    }
+    const float* y = a.y + (int64_t)m * n;
+    // z_i for owned rows, everywhere
+    for (int li = warp; li < nl; li += nwarps) {
+        const int i = rank + C * li;
+        const int64_t o = local_row_off(li, rank);
+        double t = 0.0;
+        for (int c = lane; c <= i; c += 32) t += W[o + c] * (double)y[c];
+        for (int sh = 16; sh > 0; sh >>= 1) t += __shfl_xor_sync(0xffffffffu, t, sh);
+        if (lane == 0) {
+            const double zi = t * rinv[i];
+            for (int r = 0; r < C; ++r) cluster.map_shared_rank(z, r)[i] = zi;
+        }
+    }
+    cluster.sync();
+    // this CTA's share of alpha_c = sum over owned rows i >= c of L^{-1}_ic z_i
+    for (int c = tid; c < n; c += kClusterThreads) {
+        double t = 0.0;
+        int li = (c - rank + C - 1) / C;
+        if (li < 0) li = 0;
+        for (; li < nl; ++li) {
+            const int i = rank + C * li;
+            t += W[local_row_off(li, rank) + c] * rinv[i] * z[i];
+        }
+        part[c] = t;
+    }
+    cluster.sync();
+    if (rank == 0) {
+        float* alpha = reinterpret_cast<float*>(a.blob + a.off_alpha) + (int64_t)m * n;
+        for (int c = tid; c < n; c += kClusterThreads) {
+            double t = 0.0;
+            for (int r = 0; r < C; ++r) t += cluster.map_shared_rank(part, r)[c];
+            alpha[c] = (float)t;
+        }
+        if (warp == 0) {
+            float best = -INFINITY;
+            for (int j = lane; j < n; j += 32) best = fmaxf(best, y[j]);
+            for (int sh = 16; sh > 0; sh >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, sh));
+            if (lane == 0) reinterpret_cast<float*>(a.blob + a.off_scal)[m * 4 + 2] = best;
+        }
+    }
+    // tiles: the owner of a row writes its entries (CTA 0 the padding rows)
+    float* tiles = reinterpret_cast<float*>(a.blob + a.off_linv) + (int64_t)m * a.n_tiles * kColChunkDev * kRowBlockDev;
+    const int64_t total = (int64_t)a.n_tiles * kColChunkDev * kRowBlockDev;
+    for (int64_t e = tid; e < total; e += kClusterThreads) {
+        const int t = (int)(e / (kColChunkDev * kRowBlockDev));
+        const int jj = (int)(e / kRowBlockDev % kColChunkDev), ii = (int)(e % kRowBlockDev);
+        int rb = 0;
+        while ((rb + 1) * (rb + 2) <= t) ++rb;
+        const int cj = t - rb * (rb + 1);
+        const int row = rb * kRowBlockDev + ii, c = cj * kColChunkDev + jj;
+        if (row < n ? row % C != rank : rank != 0) continue;
+        float v = 0.0f;
+        if (row < n && c <= row) v = (float)(W[local_row_off(row / C, rank) + c] * rinv[row]);
+        tiles[e] = v;
+    }
+    cluster.sync();  // CTA 0 has read every CTA's part before any CTA exits
 }
 
 constexpr int kMleMaxP = SCOOT_MAX_DIM + 2;  // ln l_1 .. ln l_d, ln s_f^2, ln tau^2
@@ -653,6 +820,21 @@ scoot_status scoot_gp_prepare_device(scoot_ctx* ctx, const scoot_param* h_space,
     }
     gp_kmat_kernel<<<dim3((unsigned)((a.tri + kKmatThreads - 1) / kKmatThreads), M), kKmatThreads, 0, st>>>(a);
     SCOOT_LAUNCHED(ctx);
+    if (n <= kClusterMaxN) {
+        // rows split over a cluster; shared memory for the CTA with the most entries
+        int64_t own = 0;
+        for (int r = 0; r < kClusterCTAs; ++r) {
+            const int64_t nl = (n - r + kClusterCTAs - 1) / kClusterCTAs;
+            const int64_t e = nl * (r + 1) + (int64_t)kClusterCTAs * nl * (nl - 1) / 2;  // local_row_off(nl, r)
+            if (e > own) own = e;
+        }
+        const size_t csmem = (size_t)8 * n * sizeof(double) + (size_t)2 * own * sizeof(double);
+        SCOOT_CUDA(ctx, cudaFuncSetAttribute(gp_chol_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)csmem));
+        gp_chol_cluster_kernel<<<M * kClusterCTAs, kClusterThreads, csmem, st>>>(a);
+        SCOOT_LAUNCHED(ctx);
+        return SCOOT_OK;
+    }
     const size_t smem = (size_t)5 * n * sizeof(double) + (in_smem ? (size_t)2 * a.tri * sizeof(double) : 0);
     SCOOT_CUDA(ctx, cudaFuncSetAttribute(gp_chol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     gp_chol_kernel<<<M, kCholThreads, smem, st>>>(a);
@@ -753,6 +935,72 @@ scoot_status scoot_gp_mle(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
     gp_mle_kernel<<<n_starts * n_obj, kMleThreads, smem, st>>>(a);
     SCOOT_LAUNCHED(ctx);
     return SCOOT_OK;
+}
+
+static int64_t slot256(int64_t b) { return (b + 255) / 256 * 256; }
+
+scoot_status scoot_gp_device_buffer_layout(const scoot_gp_layout* L, int32_t warped, int64_t* upload_bytes,
+                                           int64_t* blob_off, int64_t* work_off, int64_t* total_bytes) {
+    if (!L || !upload_bytes || !blob_off || !work_off || !total_bytes || !scoot_gp_layout_valid(L)) return SCOOT_EINVAL;
+    const int64_t n = L->n, d = L->d, M = L->n_obj;
+    int64_t off = slot256(4 * d * n) + slot256(4 * M * n) + slot256(4 * M * d) + 2 * slot256(4 * M);
+    if (warped) off += slot256(8 * M * d);
+    *upload_bytes = off;
+    *blob_off = off;
+    off += slot256(L->bytes);
+    *work_off = off;
+    int64_t wb = 0;
+    scoot_gp_device_work_bytes(L, &wb);
+    *total_bytes = off + slot256(wb);
+    return SCOOT_OK;
+}
+
+scoot_status scoot_gp_prepare_device_from_host(scoot_ctx* ctx, const scoot_param* h_space, const scoot_gp_layout* L,
+                                               const uint32_t* h_x_obs, int64_t ld_obs, const float* h_y,
+                                               const float* h_lengthscale, const float* h_signal_var,
+                                               const float* h_noise_var, const float* h_warp, void* h_stage,
+                                               void* buf, int64_t buf_bytes, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    int64_t up = 0, blob_off = 0, work_off = 0, total = 0;
+    if (scoot_gp_device_buffer_layout(L, h_warp != nullptr, &up, &blob_off, &work_off, &total) != SCOOT_OK)
+        return scoot_fail(ctx, SCOOT_EINVAL, "invalid layout");
+    if (!h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var || !h_stage || !buf)
+        return scoot_fail(ctx, SCOOT_EINVAL, "a pointer is NULL");
+    if (buf_bytes < total || !scoot_aligned16(buf))
+        return scoot_fail(ctx, SCOOT_EINVAL, "buf needs %lld bytes, 16-byte aligned", (long long)total);
+    if (ld_obs < L->n) return scoot_fail(ctx, SCOOT_EINVAL, "ld_obs < n");
+    const int64_t n = L->n, d = L->d, M = L->n_obj;
+    char* hs = static_cast<char*>(h_stage);
+    int64_t off = 0, o_obs, o_y, o_ls, o_sf, o_tau, o_warp = -1;
+    o_obs = off;
+    for (int64_t c = 0; c < d; ++c) std::memcpy(hs + off + 4 * c * n, h_x_obs + c * ld_obs, 4 * n);
+    off += slot256(4 * d * n);
+    o_y = off;
+    std::memcpy(hs + off, h_y, 4 * M * n);
+    off += slot256(4 * M * n);
+    o_ls = off;
+    std::memcpy(hs + off, h_lengthscale, 4 * M * d);
+    off += slot256(4 * M * d);
+    o_sf = off;
+    std::memcpy(hs + off, h_signal_var, 4 * M);
+    off += slot256(4 * M);
+    o_tau = off;
+    std::memcpy(hs + off, h_noise_var, 4 * M);
+    off += slot256(4 * M);
+    if (h_warp) {
+        o_warp = off;
+        std::memcpy(hs + off, h_warp, 8 * M * d);
+        off += slot256(8 * M * d);
+    }
+    char* db = static_cast<char*>(buf);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    SCOOT_CUDA(ctx, cudaMemcpyAsync(db, hs, (size_t)up, cudaMemcpyHostToDevice, st));
+    return scoot_gp_prepare_device(ctx, h_space, L, reinterpret_cast<const uint32_t*>(db + o_obs), n,
+                                   reinterpret_cast<const float*>(db + o_y), reinterpret_cast<const float*>(db + o_ls),
+                                   reinterpret_cast<const float*>(db + o_sf), reinterpret_cast<const float*>(db + o_tau),
+                                   o_warp >= 0 ? reinterpret_cast<const float*>(db + o_warp) : nullptr, db + blob_off,
+                                   db + work_off, total - work_off, stream);
 }
 
 }  // extern "C"

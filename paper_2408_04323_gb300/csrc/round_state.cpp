@@ -2,9 +2,9 @@
 // (Section 4.3), the packed forest (Eq. 3) and, for EHVI, the box
 // decomposition of the region the front does not dominate (Section 4.4)
 // with the base samples, or the boxes' grid index for the exact EHVI.  The
-// fp64 GP factorisation runs on the library's host threads (objectives in
-// parallel) while the calling thread packs the forest and decomposes the
-// boxes, so the round's host time is the longer of the two rather than their
+// fp64 GP factorisation (objectives in parallel) and the forest's packing run
+// on the library's host threads while the calling thread decomposes the
+// boxes, so the round's host time is the longest of them rather than their
 // sum.
 #include <algorithm>
 #include <atomic>
@@ -186,10 +186,27 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
     };
     out->off_forest = off;
     off += slot(out->forest.bytes);
+    // The forest's packing on another thread while this one builds the boxes.
+    scoot_status forest_status = SCOOT_OK;
+    Pool::Latch forest_latch;
+    const bool forest_job = out->off_forest + out->forest.bytes <= cap;
+    if (forest_job) {
+        const scoot_round_inputs* pin = in;
+        const scoot_forest_layout* fl = &out->forest;
+        char* dst = buf + out->off_forest;
+        Pool::get().submit([pin, fl, dst, &forest_status] {
+            forest_status = scoot_forest_pack(fl, pin->nodes, pin->tree_offset, dst);
+        }, &forest_latch);
+    }
+    auto finish_all = [&](scoot_status st) {
+        if (forest_job) Pool::get().wait(&forest_latch);
+        if (st == SCOOT_OK && forest_status != SCOOT_OK) st = forest_status;
+        return finish(st);
+    };
     std::vector<float> lo, hi, grid;
     std::vector<uint32_t> corner;
     if (in->boxes) {
-        if (M < 2 || !in->ref) return finish(SCOOT_EINVAL);
+        if (M < 2 || !in->ref) return finish_all(SCOOT_EINVAL);
         int32_t nb = 0, fs = 0, bcap = 1024;
         for (;;) {
             lo.assign((size_t)bcap * M, 0.0f);
@@ -199,7 +216,7 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
                 bcap = nb;
                 continue;
             }
-            if (s != SCOOT_OK) return finish(s);
+            if (s != SCOOT_OK) return finish_all(s);
             break;
         }
         out->n_boxes = nb;
@@ -209,7 +226,7 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
         out->off_box_hi = off;
         off += slot((int64_t)nb * M * 4);
         if (in->boxes == 1) {
-            if (!in->eps || in->n_mc < 1) return finish(SCOOT_EINVAL);
+            if (!in->eps || in->n_mc < 1) return finish_all(SCOOT_EINVAL);
             out->off_eps = off;
             off += slot((int64_t)in->n_mc * M * 4);
         } else {
@@ -217,7 +234,7 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
             grid.assign((size_t)M * gc, 0.0f);
             corner.assign((size_t)(nb > 0 ? nb : 1) * M, 0u);
             s = scoot_boxes_index(lo.data(), hi.data(), nb, M, gc, grid.data(), out->n_grid, corner.data());
-            if (s != SCOOT_OK) return finish(s);
+            if (s != SCOOT_OK) return finish_all(s);
             out->grid_cap = gc;
             out->off_grid = off;
             off += slot((int64_t)M * gc * 4);
@@ -226,9 +243,8 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
         }
     }
     out->bytes = off;
-    if (off > cap) return finish(SCOOT_ENOMEM);  // out->bytes holds the size needed
-    s = scoot_forest_pack(&out->forest, in->nodes, in->tree_offset, buf + out->off_forest);
-    if (s == SCOOT_OK && in->boxes) {
+    if (off > cap) return finish_all(SCOOT_ENOMEM);  // out->bytes holds the size needed
+    if (in->boxes) {
         std::memcpy(buf + out->off_box_lo, lo.data(), (size_t)out->n_boxes * M * 4);
         std::memcpy(buf + out->off_box_hi, hi.data(), (size_t)out->n_boxes * M * 4);
         if (in->boxes == 1) {
@@ -238,7 +254,7 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
             std::memcpy(buf + out->off_corner, corner.data(), (size_t)out->n_boxes * M * 4);
         }
     }
-    return finish(s);
+    return finish_all(s);
 }
 
 }  // extern "C"

@@ -86,6 +86,7 @@ class _Staging:
 
 
 _staging = _Staging()
+_staging_gp = _Staging()  # the GP inputs, uploaded before the rest when the device builds the GP state
 
 
 class State:
@@ -93,11 +94,12 @@ class State:
     scoot_round_state_build (GP state, packed forest, boxes with eps or with
     their grid index) straight into a pinned staging buffer and uploaded in
     one copy; gp_state, forest, box_lo, box_hi, eps, grid and corner are
-    views into one device buffer.  With ``gp_on_device`` the GP state is
-    built by the device instead (scoot_gp_prepare_device, asynchronously on
-    ``stream`` after the upload of its inputs).  With ``into`` (a State of
-    the same shapes) the upload reuses that State's device buffer and views,
-    so work captured against it (a CUDA graph) stays valid."""
+    views into device buffers.  With ``gp_on_device`` the GP state is built
+    by the device (scoot_gp_prepare_device): its inputs are uploaded and its
+    kernels launched on ``stream`` first, so that the device factorises
+    while the host packs the forest and builds the boxes.  With ``into`` (a
+    State of the same shapes) the uploads reuse that State's device buffers
+    and views, so work captured against them (a CUDA graph) stays valid."""
 
     def __init__(self, inp: RoundInputs, device: torch.device, stream=None, into=None, gp_on_device=False,
                  ctx=None):
@@ -105,6 +107,9 @@ class State:
         stream = torch.cuda.current_stream(device) if stream is None else stream
         if gp_on_device and ctx is None:
             raise ValueError("gp_on_device needs a context")
+        self.gp_buffer = None
+        if gp_on_device:
+            self._gp_on_device(inp, device, stream, into, ctx)
         boxes = {"ehvi": 1, "ehvi-exact": 2}.get(inp.acq, 0)
         stage = _staging.take(_staging.capacity())
         while True:
@@ -123,33 +128,9 @@ class State:
         self.front_size = int(out.front_size)
         if boxes == 2:
             self.n_grid = np.array(out.n_grid[:M], np.int32)
-        upload = int(out.bytes)
-        total = upload
-        gp_in = None
-        if gp_on_device:
-            # the GP inputs, the device-built state and its scratch after the host-built parts
-            gp_in = [np.ascontiguousarray(inp.x_obs[:, :n]).view(np.int32), np.ascontiguousarray(inp.y_obs, np.float32),
-                     np.ascontiguousarray(inp.lengthscale, np.float32), np.ascontiguousarray(inp.signal_var, np.float32),
-                     np.ascontiguousarray(inp.noise_var, np.float32)]
-            if inp.warp is not None:
-                gp_in.append(np.ascontiguousarray(inp.warp, np.float32))
-            in_offs = []
-            for arr in gp_in:
-                in_offs.append(total)
-                total += (arr.nbytes + 255) // 256 * 256
-            if total > stage.numel():
-                stage = _staging.take(total, keep=upload)
-            host = stage.numpy()
-            for arr, o in zip(gp_in, in_offs):
-                host[o:o + arr.nbytes] = arr.reshape(-1).view(np.uint8)
-            upload = total
-            gp_off = total
-            total += (self.gp_layout.bytes + 255) // 256 * 256
-            work_off = total
-            work_bytes = S.scoot_gp_device_work_bytes(self.gp_layout)
-            total += (work_bytes + 255) // 256 * 256
+        total = int(out.bytes)
         offsets = (int(out.off_gp), int(out.off_forest), int(out.off_box_lo), int(out.off_box_hi), int(out.off_eps),
-                   int(out.off_grid), int(out.off_corner), upload, total)
+                   int(out.off_grid), int(out.off_corner), total)
         reuse = into is not None and into.buffer.numel() == total and into.offsets == offsets
         if reuse:
             dev = into.buffer
@@ -158,41 +139,53 @@ class State:
             if stream != torch.cuda.current_stream(device):
                 dev.record_stream(stream)
         with torch.cuda.stream(stream):
-            dev[:upload].copy_(stage[:upload], non_blocking=True)
+            dev.copy_(stage[:total], non_blocking=True)
         _staging.sent(stream)
         self.buffer = dev
         self.offsets = offsets
-        self.upload_bytes = upload
+        self.upload_bytes = total + (self.gp_upload_bytes if gp_on_device else 0)
         if reuse:  # same offsets: the views of `into` are views of this buffer
-            for name in ("gp_state", "forest", "box_lo", "box_hi", "eps", "grid", "corner"):
+            for name in ("forest", "box_lo", "box_hi", "eps", "grid", "corner") + (() if gp_on_device else ("gp_state",)):
                 if hasattr(into, name):
                     setattr(self, name, getattr(into, name))
+            return
+
+        def view(off, nbytes, dtype=None, shape=None):
+            v = dev[off:off + nbytes]
+            return v if dtype is None else v.view(dtype).reshape(shape)
+        if not gp_on_device:
+            self.gp_state = view(out.off_gp, self.gp_layout.bytes)
+        self.forest = view(out.off_forest, self.forest_layout.bytes)
+        B = self.n_boxes
+        if boxes:
+            self.box_lo = view(out.off_box_lo, B * M * 4, torch.float32, (B, M))
+            self.box_hi = view(out.off_box_hi, B * M * 4, torch.float32, (B, M))
+        if boxes == 1:
+            self.eps = view(out.off_eps, inp.eps.shape[0] * M * 4, torch.float32, (inp.eps.shape[0], M))
+        if boxes == 2:
+            self.grid = view(out.off_grid, M * out.grid_cap * 4, torch.float32, (M, out.grid_cap))
+            self.corner = view(out.off_corner, B * M * 4, torch.int32, (B, M))
+
+    def _gp_on_device(self, inp, device, stream, into, ctx):
+        """Upload the GP inputs and launch the device build of the GP state
+        (one library call)."""
+        M, n = inp.y_obs.shape
+        layout = S.scoot_gp_layout_init(inp.space, n, M, inp.kernel)
+        up, blob_off, _, total = S.scoot_gp_device_buffer_layout(layout, inp.warp is not None)
+        if into is not None and into.gp_buffer is not None and into.gp_buffer.numel() == total:
+            dev = into.gp_buffer
+            self.gp_state = into.gp_state
         else:
-            def view(off, nbytes, dtype=None, shape=None):
-                v = dev[off:off + nbytes]
-                return v if dtype is None else v.view(dtype).reshape(shape)
-            if not gp_on_device:
-                self.gp_state = view(out.off_gp, self.gp_layout.bytes)
-            self.forest = view(out.off_forest, self.forest_layout.bytes)
-            B = self.n_boxes
-            if boxes:
-                self.box_lo = view(out.off_box_lo, B * M * 4, torch.float32, (B, M))
-                self.box_hi = view(out.off_box_hi, B * M * 4, torch.float32, (B, M))
-            if boxes == 1:
-                self.eps = view(out.off_eps, inp.eps.shape[0] * M * 4, torch.float32, (inp.eps.shape[0], M))
-            if boxes == 2:
-                self.grid = view(out.off_grid, M * out.grid_cap * 4, torch.float32, (M, out.grid_cap))
-                self.corner = view(out.off_corner, B * M * 4, torch.int32, (B, M))
-            if gp_on_device:
-                self.gp_state = view(gp_off, self.gp_layout.bytes)
-        if gp_on_device:
-            names = ["obs", "y", "ls", "sf2", "tau2", "warp"]
-            dv = {}
-            for name, arr, o in zip(names, gp_in, in_offs):
-                dv[name] = dev[o:o + arr.nbytes].view(torch.int32 if name == "obs" else torch.float32).reshape(arr.shape)
-            S.scoot_gp_prepare_device(ctx, inp.space, self.gp_layout, dv["obs"], dv["y"], dv["ls"], dv["sf2"],
-                                      dv["tau2"], self.gp_state, work=dev[work_off:work_off + work_bytes],
-                                      warp=dv.get("warp"), stream=stream)
+            dev = torch.empty(total, dtype=torch.uint8, device=device)
+            if stream != torch.cuda.current_stream(device):
+                dev.record_stream(stream)
+            self.gp_state = dev[blob_off:blob_off + layout.bytes]
+        stage = _staging_gp.take(up)
+        S.scoot_gp_prepare_device_from_host(ctx, inp.space, layout, inp.x_obs, inp.y_obs, inp.lengthscale,
+                                            inp.signal_var, inp.noise_var, stage, dev, warp=inp.warp, stream=stream)
+        _staging_gp.sent(stream)
+        self.gp_buffer = dev
+        self.gp_upload_bytes = up
 
 
 class ScoringRound:

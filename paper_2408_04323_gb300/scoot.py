@@ -99,6 +99,10 @@ _PROTOS = {
     "scoot_gp_prepare": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_prepare_warped": [_vp, _vp, _i64, _vp, _vp, _vp, _vp, _vp, C.POINTER(scoot_gp_layout), _vp, _vp],
     "scoot_gp_device_work_bytes": [C.POINTER(scoot_gp_layout), C.POINTER(_i64)],
+    "scoot_gp_device_buffer_layout": [C.POINTER(scoot_gp_layout), _i32, C.POINTER(_i64), C.POINTER(_i64),
+                                      C.POINTER(_i64), C.POINTER(_i64)],
+    "scoot_gp_prepare_device_from_host": [_vp, _vp, C.POINTER(scoot_gp_layout), _vp, _i64, _vp, _vp, _vp, _vp, _vp,
+                                          _vp, _vp, _i64, _vp],
     "scoot_gp_mle": [_vp, _vp, _i32, _vp, _i64, _i32, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _u32, _i32,
                      C.c_double, _vp, _vp, _vp, _vp, _i64, _vp],
     "scoot_gp_mle_work_bytes": [_i32, _i32, _i32, _i32, C.POINTER(_i64)],
@@ -587,6 +591,29 @@ def scoot_gp_mle(ctx, h_space, obs, n, y, theta0, h_lo, h_hi, free_mask, steps, 
                               _dev(lml, torch.float64, "lml"), _dev(grad, torch.float64, "grad"),
                               _dev(work, torch.uint8, "work"), int(work.numel()), _stream(stream)),
            "scoot_gp_mle", _h(ctx))
+
+
+def scoot_gp_device_buffer_layout(layout, warped: bool):
+    """(upload_bytes, blob_off, work_off, total_bytes)."""
+    v = [_i64() for _ in range(4)]
+    _check(lib().scoot_gp_device_buffer_layout(C.byref(layout), int(bool(warped)), *[C.byref(x) for x in v]),
+           "scoot_gp_device_buffer_layout")
+    return tuple(int(x.value) for x in v)
+
+
+def scoot_gp_prepare_device_from_host(ctx, h_space, layout, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var,
+                                      h_stage, buf, warp=None, stream=None):
+    """h_stage: pinned uint8 host tensor; buf: uint8 device tensor (scoot_gp_device_buffer_layout)."""
+    import torch
+    _check(lib().scoot_gp_prepare_device_from_host(
+        _h(ctx), _host(h_space, 16, name="h_space"), C.byref(layout), _host(h_x_obs, 4, name="h_x_obs"),
+        int(h_x_obs.shape[1]), _host(h_y, dtype=np.float32, name="h_y"),
+        _host(h_lengthscale, dtype=np.float32, name="h_lengthscale"),
+        _host(h_signal_var, dtype=np.float32, name="h_signal_var"),
+        _host(h_noise_var, dtype=np.float32, name="h_noise_var"),
+        _host(warp, dtype=np.float32, name="warp") if warp is not None else None,
+        _vp(h_stage.data_ptr()), _dev(buf, torch.uint8, "buf"), int(buf.numel()), _stream(stream)),
+        "scoot_gp_prepare_device_from_host", _h(ctx))
 
 
 def scoot_rf_train_work_bytes(n: int, d: int) -> int:

@@ -130,10 +130,11 @@ def test_device_state_matches(S, ctx, name, kernel, warped):
     posterior_check(S, ctx, inst, L, db, f"{name} k{kernel}{' warped' if warped else ''}", kernel, warp)
 
 
-@pytest.mark.parametrize("n_obs", [1, 2, 63, 64, 65, 160, 161, 640])
+@pytest.mark.parametrize("n_obs", [1, 2, 7, 63, 64, 65, 160, 161, 384, 385, 640])
 def test_device_state_sizes(S, ctx, n_obs):
     """Observation counts across tile edges, the shared-memory limit of the
-    factorisation (160 / 161) and the maximum; the d8 space, two objectives."""
+    factorisation (160 / 161), the cluster path's limit (384 / 385) and the maximum; the d8
+    space, two objectives."""
     base = make_instance("d8-ehvi2", seeds("d8-ehvi2")[0], n_cand=4096)
     from workloads.generate import draw_configs
     w = base.workload
