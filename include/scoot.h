@@ -22,7 +22,7 @@
  *
  * plus host-side preparation of per-round state (Cholesky factor of the
  * observations' covariance, box decomposition of the non-dominated region,
- * forest packing).
+ * forest packing), all three in one call by scoot_round_state_build.
  *
  * Conventions
  *  - Every call returns a scoot_status: SCOOT_OK (0) or a negative error.
