@@ -57,6 +57,8 @@ struct ScoreArgs {
     int32_t psi_rows;             // kEHVIX: sum_j (n_grid[j] + 1), rows of the psi table
     const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
     const unsigned int* n_list;
+    int32_t cat_smem;             // floats of the categorical table staged in shared memory (0: read from L1)
+    int32_t cat_off;              // where, in floats from the start of shared memory
     float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad][ldv] by list position
     int64_t ldv;
     uint32_t* err;                // device error word
@@ -240,6 +242,10 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
     const float* gcat = reinterpret_cast<const float*>(a.state + a.off_cat);
 
+    // The categorical part of r^2 for every objective, observation and
+    // pattern, when small: one shared-memory load per pair instead of L1.
+    float* cat_s = sm + a.cat_off;
+    for (int e = tid; e < a.cat_smem; e += kThreads) cat_s[e] = __ldg(gcat + e);
     if (EPI == kEHVI) stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
     if (EPI == kEHVIX) stage_box_grid(a.grid, a.grid_cap, a.n_grid, a.corner, a.n_boxes, M, grid_s, corner_s, a.err);
     if (tid < kMaxD) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
@@ -293,7 +299,9 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             }
             for (int j = tid; j < n_pad; j += kThreads) al[j] = j < a.n_obs ? galpha[(size_t)m * a.n_obs + j] : 0.0f;
             const float sf2 = gscal[m * 4 + 0];
-            const float* catrow = gcat + (size_t)m * a.n_obs * a.n_pat + pid;
+            // this candidate's column of the categorical table: shared memory when
+            // staged, else global (one generic pointer either way)
+            const float* catrow = (a.cat_smem ? cat_s : gcat) + (size_t)m * a.n_obs * a.n_pat + pid;
             float ut[DO];
             const bool warped = gscal[m * 4 + 3] != 0.0f;  // the same in every thread
 #pragma unroll
@@ -311,7 +319,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
 #pragma unroll 2
             for (int j = half; j < a.n_obs; j += 2) {
                 const float4* xj4 = reinterpret_cast<const float4*>(xs + j * DO);
-                float r2 = __ldg(catrow + (size_t)j * a.n_pat);  // categorical part
+                float r2 = catrow[(size_t)j * a.n_pat];  // categorical part
 #pragma unroll
                 for (int q4 = 0; q4 < DO / 4; ++q4) {
                     const float4 v = xj4[q4];
@@ -629,6 +637,8 @@ scoot_status fill_state_args(scoot_ctx* ctx, const scoot_gp_layout* L, const voi
     return SCOOT_OK;
 }
 
+constexpr int kCatSmemMax = 1024;  // floats of categorical table worth staging per block
+
 size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
     const size_t ks_rows = epi == kEHVIX && (size_t)a.psi_rows > n_pad ? (size_t)a.psi_rows : n_pad;
@@ -639,8 +649,13 @@ size_t score_smem(const ScoreArgs& a, int epi, int DO) {
 }
 
 template <int EPI, int M, int DO>
-scoot_status launch_score_dm(scoot_ctx* ctx, const ScoreArgs& a, cudaStream_t st) {
-    const size_t smem = score_smem(a, EPI, DO);
+scoot_status launch_score_dm(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
+    // the categorical table of the objectives this epilogue reads, staged when small
+    const int nobj = (EPI == kEHVI || EPI == kEHVIX) ? M : ((EPI == kEI || EPI == kMACE) ? 1 : a.n_obj);
+    const int64_t cat = (int64_t)nobj * a.n_obs * a.n_pat;
+    a.cat_off = (int32_t)(score_smem(a, EPI, DO) / 4);
+    a.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
+    const size_t smem = score_smem(a, EPI, DO) + (size_t)((a.cat_smem + 3) & ~3) * 4;
     auto kern = score_kernel<EPI, M, DO>;
     int optin = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
