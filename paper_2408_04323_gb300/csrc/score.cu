@@ -59,6 +59,7 @@ struct ScoreArgs {
     const unsigned int* n_list;
     int32_t cat_smem;             // floats of the categorical table staged in shared memory (0: read from L1)
     int32_t cat_off;              // where, in floats from the start of shared memory
+    int32_t wbuf_off;             // the next tile's pool words [d][kTC], in floats from the start
     float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad][ldv] by list position
     int64_t ldv;
     uint32_t* err;                // device error word
@@ -188,6 +189,24 @@ __device__ __forceinline__ void stage_tile_async(float* dst, const float4* src, 
     asm volatile("cp.async.commit_group;\n" ::: "memory");
 }
 
+// Gathers the d words of the candidates of a tile into wbuf[q][slot] (feature
+// order) with 4-byte cp.async, two threads per candidate, one group.
+__device__ __forceinline__ void prefetch_words(uint32_t* wbuf, const uint32_t* cand, int64_t ld, const int32_t* list,
+                                               const float4* fm, int d, int64_t tile, int64_t n_tiles,
+                                               int64_t n_work, int tid) {
+    const int s = tid & (kTC - 1);
+    const int64_t p = tile * kTC + s;
+    if (tile < n_tiles && p < n_work) {
+        const int64_t i = list ? (int64_t)list[p] : p;
+        for (int q = tid >> 6; q < d; q += 2) {
+            const unsigned dst = (unsigned)__cvta_generic_to_shared(wbuf + q * kTC + s);
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst),
+                         "l"(cand + (int64_t)fm[q].w * ld + i) : "memory");
+        }
+    }
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+
 // Waits until every cp.async group this thread committed has landed.
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
@@ -261,17 +280,22 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
 
     const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
     const int64_t n_tiles = (n_work + kTC - 1) / kTC;
+    // The next tile's pool words stream into wbuf while this tile is scored.
+    uint32_t* wbuf = reinterpret_cast<uint32_t*>(sm + a.wbuf_off);  // [d][kTC]
+    prefetch_words(wbuf, a.cand, a.ld, a.list, fm, a.d, blockIdx.x, n_tiles, n_work, tid);
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
         const int64_t pos = tile * kTC + slot;
         const bool live = pos < n_work;
         const int64_t i = live ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
+        cp_async_wait_all();
+        __syncthreads();  // this tile's words are in wbuf
         float u[DO];
 #pragma unroll
         for (int q = 0; q < DO; ++q) {
             u[q] = 0.0f;
             if (q < n_ord && live) {
                 const float4 f = fm[q];
-                u[q] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + i), (int)f.x, f.y, f.z);
+                u[q] = feature_of(wbuf[q * kTC + slot], (int)f.x, f.y, f.z);
             }
         }
         // Joint category pattern (mixed radix); out-of-range categories are
@@ -280,13 +304,15 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
         for (int q = n_ord; q < a.d && live; ++q) {
             const float4 f = fm[q];
             const int nc = (int)f.y;
-            int v = (int)__ldg(a.cand + (int64_t)f.w * a.ld + i);
+            int v = (int)wbuf[q * kTC + slot];
             if (v < 0 || v >= nc) {
                 atomicOr(a.err, SCOOT_DEVERR_INDEX);
                 v = v < 0 ? 0 : nc - 1;
             }
             pid += v * (int)f.z;
         }
+        __syncthreads();  // every thread has read its words
+        prefetch_words(wbuf, a.cand, a.ld, a.list, fm, a.d, tile + gridDim.x, n_tiles, n_work, tid);
         float mu[kMaxM], vr[kMaxM];
         for (int m = 0; m < nobj; ++m) {
             __syncthreads();  // previous users of xs / al / part / Lt are done
@@ -655,7 +681,8 @@ scoot_status launch_score_dm(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
     const int64_t cat = (int64_t)nobj * a.n_obs * a.n_pat;
     a.cat_off = (int32_t)(score_smem(a, EPI, DO) / 4);
     a.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
-    const size_t smem = score_smem(a, EPI, DO) + (size_t)((a.cat_smem + 3) & ~3) * 4;
+    a.wbuf_off = a.cat_off + ((a.cat_smem + 3) & ~3);
+    const size_t smem = (size_t)(a.wbuf_off + a.d * kTC) * 4;
     auto kern = score_kernel<EPI, M, DO>;
     int optin = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
