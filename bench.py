@@ -655,7 +655,7 @@ def main():
     pkg.build()
     from paper_2408_04323_gb300 import scoot as S
     from paper_2408_04323_gb300.pipeline import RoundInputs, ScoringRound, State
-    from paper_2408_04323_gb300.shard import gather_topq
+    from paper_2408_04323_gb300.shard import gather_mace_front, gather_topq
     from workloads import WORKLOADS, Stream, draw_configs, make_instance, seeds, warp_params
 
     w = WORKLOADS[args.workload]
@@ -664,8 +664,6 @@ def main():
         raise SystemExit("--acq mace needs a one-objective workload")
     if acq_kind == "ehvi-exact" and (w.n_obj < 2 or w.fantasy):
         raise SystemExit("--acq ehvi-exact needs a multi-objective workload without fantasies")
-    if acq_kind == "mace" and world > 1:
-        raise SystemExit("--acq mace runs on one GPU: its front is not merged across ranks")
     seed = seeds(w.name)[0]
     inst = make_instance(w.name, seed)
     cand_np = inst.cand
@@ -684,6 +682,16 @@ def main():
     rnd = ScoringRound(ctx, inp, N, device, gp_on_device=gp_dev)
     cand = torch.from_numpy(cand_np.view(np.int32)).to(device)
     stream = torch.cuda.current_stream(device)
+
+    def exchange():
+        """The ranks' only exchange: their top-q lists, or for MACE their fronts."""
+        if inp.acq == "mace":
+            f = int(rnd.top_count[1].item())
+            if f > rnd.front_cap:
+                raise SystemExit(f"a front of {f} candidates exceeds the exchange's {rnd.front_cap}")
+            gather_mace_front(rnd.acq3, rnd.front, f, rank * N, w.q, rnd.seed)
+        else:
+            gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
     st = rnd.state
 
@@ -789,7 +797,7 @@ def main():
             step()
         tev[kk][1].record(stream)
         if dist:
-            gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
+            exchange()
     torch.cuda.synchronize(device)
     if dist:
         dist.barrier()
@@ -861,7 +869,7 @@ def main():
                     dst.copy_(src, non_blocking=True)
                 picks = pinned_picks
                 if dist:
-                    gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
+                    exchange()
                 torch.cuda.synchronize(device)
                 if kk >= args.warmup:
                     times.append(time.perf_counter() - t0)
@@ -895,7 +903,7 @@ def main():
                 dst.copy_(src, non_blocking=True)
             picks = pinned_picks
             if dist:
-                gather_topq(rnd.top_idx, rnd.top_val, rnd.top_count, w.q)
+                exchange()
             torch.cuda.synchronize(device)
             if kk >= args.warmup:
                 times.append(time.perf_counter() - t0)
