@@ -215,3 +215,30 @@ def test_round_with_device_state(S, ctx, name):
     (ih, vh), (id_, vd) = out
     assert len(ih) == w.q and np.array_equal(ih, id_)
     assert np.allclose(vd, vh, rtol=1e-5, atol=1e-7)
+
+
+@pytest.mark.parametrize("name,warped", [("d8-ehvi2", False), ("d8-ehvi2", True), ("d12-fantasy", False)])
+def test_device_state_from_host_inputs(S, ctx, name, warped):
+    """The one-call path (host inputs packed into pinned memory, copied and
+    built on the device) writes the same blob as scoot_gp_prepare_device fed
+    the same inputs from device memory."""
+    inst = make_instance(name, seeds(name)[0], n_cand=16)
+    L = S.scoot_gp_layout_init(inst.space, inst.n_obs, inst.n_obj, 0)
+    warp = warp_params(name, seeds(name)[0]) if warped else None
+    want = device_blob(S, ctx, inst, L, warp).cpu().numpy()
+    up, blob_off, work_off, total = S.scoot_gp_device_buffer_layout(L, warped)
+    assert blob_off >= up and work_off >= blob_off + L.bytes and total >= work_off
+    buf = torch.full((total,), 0xCD, dtype=torch.uint8, device="cuda")
+    stage = torch.empty(up, dtype=torch.uint8, pin_memory=True)
+    S.scoot_gp_prepare_device_from_host(ctx, inst.space, L, np.ascontiguousarray(inst.x_obs),
+                                        inst.y_obs.astype(np.float32), inst.lengthscale.astype(np.float32),
+                                        inst.signal_var.astype(np.float32), inst.noise_var.astype(np.float32),
+                                        stage, buf, warp=None if warp is None else warp.astype(np.float32))
+    torch.cuda.synchronize()
+    ctx.check()
+    got = buf[blob_off:blob_off + L.bytes].cpu().numpy()
+    # the regions the posterior reads (padding between regions is not written)
+    for off, cnt in [(L.off_fmap, L.d * 4), (L.off_xs, L.n_obj * L.n * L.d), (L.off_ils, L.n_obj * L.d),
+                     (L.off_alpha, L.n_obj * L.n), (L.off_linv, L.n_obj * L.n_tiles * 32 * 64),
+                     (L.off_scal, L.n_obj * 4), (L.off_cat, L.n_obj * L.n * L.n_pat), (L.off_warp, L.n_obj * L.d * 2)]:
+        assert np.array_equal(got[off:off + 4 * cnt], want[off:off + 4 * cnt]), off
