@@ -227,11 +227,15 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 // branch.  The categorical part of r^2 depends only on the candidate's joint
 // category pattern and is read from the host-built table (one load).
 template <int EPI, int M, int DO>
-__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 5 : 1)
+__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 5 : ((EPI == kEI || EPI == kMACE) ? 4 : 1))
 score_kernel(const __grid_constant__ ScoreArgs a) {
     // Five blocks per SM for the 2-objective EHVI of <= 8 parameters caps
-    // registers at 96.
+    // registers at 96.  The one-objective epilogues run four blocks per SM
+    // (128 registers) with a single L^{-1} tile buffer, which the fourth
+    // block's shared memory needs: their tile loads are hidden by the other
+    // blocks rather than by double buffering.
     constexpr bool kRegCapped = EPI == kEHVI && M == 2 && DO == 8;
+    constexpr bool kSingleL = EPI == kEI || EPI == kMACE;
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
     // Ks, and after the posterior the exact-EHVI psi table [psi_rows][kTC]
@@ -240,7 +244,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     float* xs = Ks + (size_t)ks_rows * kTC;                           // [n_obs][DO] ordinal features
     float* al = xs + (size_t)a.n_obs * DO;                            // [n_pad]
     float* Lt = al + n_pad;                                           // [2][kCJ][kRB] double buffer
-    float* part = Lt + 2 * kCJ * kRB;                                 // [8][kTC]
+    float* part = Lt + (kSingleL ? 1 : 2) * kCJ * kRB;                // [8][kTC]
     float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [kMaxD] feature map
     float4* blo = fm + kMaxD;                          // [B] (general boxes) or [2B] (saturated form)
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
@@ -384,16 +388,16 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                     // while tile t is multiplied.
                     cp_async_wait_all();
                     __syncthreads();
-                    if (t + 1 < a.n_tiles)
+                    if (!kSingleL && t + 1 < a.n_tiles)
                         stage_tile_async(Lt + ((t + 1) & 1) * (kCJ * kRB), tiles + (size_t)(t + 1) * (kCJ * kRB / 4), tid);
-                    const float4* Lt4 = reinterpret_cast<const float4*>(Lt + (t & 1) * (kCJ * kRB));
+                    const float4* Lt4 = reinterpret_cast<const float4*>(Lt + (kSingleL ? 0 : (t & 1)) * (kCJ * kRB));
                     // rows of this warp: rb*64 + 16*warp .. +15; columns cj*32 .. +31;
                     // L^{-1} is zero right of the diagonal, so a warp stops at its
                     // last row (in steps of 16 columns).
                     const int j0 = cj * kCJ;
                     const int last_row = rb * kRB + 16 * warp + 15;
-                    if (j0 > last_row) continue;
-                    const int jj_end = last_row - j0 + 1 >= kCJ ? kCJ : 16;
+                    if (!kSingleL && j0 > last_row) continue;  // (single buffer: every thread reaches the staging below)
+                    const int jj_end = j0 > last_row ? 0 : (last_row - j0 + 1 >= kCJ ? kCJ : 16);
 #pragma unroll 4
                     for (int jj = 0; jj < jj_end; ++jj) {
                         const float4 k4 = Ks4[(j0 + jj) * (kTC / 4) + cg];
@@ -414,6 +418,10 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                                 acc2[r][1] = __ffma2_rn(lb, k23, acc2[r][1]);
                             }
                         }
+                    }
+                    if (kSingleL && t + 1 < a.n_tiles) {  // every thread is done with tile t
+                        __syncthreads();
+                        stage_tile_async(Lt, tiles + (size_t)(t + 1) * (kCJ * kRB / 4), tid);
                     }
                 }
                 float accm[8][4];
@@ -668,7 +676,8 @@ constexpr int kCatSmemMax = 1024;  // floats of categorical table worth staging 
 size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
     const size_t ks_rows = epi == kEHVIX && (size_t)a.psi_rows > n_pad ? (size_t)a.psi_rows : n_pad;
-    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + 2 * kCJ * kRB + 8 * kTC + 4 * kMaxD;
+    const size_t l_bufs = (epi == kEI || epi == kMACE) ? 1 : 2;
+    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + l_bufs * kCJ * kRB + 8 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
     if (epi == kEHVIX) f += (size_t)((a.psi_rows + 3) & ~3) + (size_t)a.n_boxes * kMaxM;
     return f * 4;
