@@ -51,7 +51,7 @@ KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["scor
 TRAFFIC = {
     ("prune", "d8-ehvi2"): {"bytes": 3151360, "sha": "669855124f47da70"},
     ("rf", "d8-ehvi2"): {"bytes": 8809728, "sha": "669855124f47da70"},
-    ("score", "d8-ehvi2"): {"bytes": 8851712, "sha": "76e1bd62a9d25955"},
+    ("score", "d8-ehvi2"): {"bytes": 8858112, "sha": "3ee4c80f5161c740"},
 }
 
 
