@@ -61,7 +61,7 @@ typedef int32_t scoot_status;
 #define SCOOT_ECUDA        -3   /* a CUDA runtime call failed */
 #define SCOOT_EDEVICE      -4   /* a kernel flagged a bad index or value at run time */
 #define SCOOT_ETIMEOUT     -5   /* a bounded device-side wait gave up */
-#define SCOOT_EUNSUPPORTED -6   /* size or option beyond what this build handles */
+#define SCOOT_EUNSUPPORTED -6   /* size or option beyond what the library handles */
 
 /* Parameter kinds of the mixed search space (Section 3, Table 1). */
 #define SCOOT_INT_UNIFORM 0

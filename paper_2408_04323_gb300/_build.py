@@ -1,7 +1,7 @@
 """Compile libscoot.so (the C-ABI library) for sm_103a with nvcc, in-tree.
 
 Each translation unit is compiled in parallel, then linked with the CUDA
-runtime linked statically, so the library depends on nothing but the driver.
+runtime linked statically, so the library depends on nothing but the CUDA driver.
 """
 from __future__ import annotations
 
