@@ -338,3 +338,39 @@ def test_round_state_build_equals_separate_calls(S, name, boxes, warped):
                                        warp=warp, boxes=boxes, h_ref=inst.ref, h_eps=inst.eps, gp_on_device=True)
     assert st2.off_gp == -1 and st2.off_forest == 0
     assert bytes(buf2[:FL.bytes]) == fb.tobytes()
+
+
+def test_round_state_build_concurrent_callers(S):
+    """Several host threads building round states at once share the
+    library's thread pool (the GP objectives and the forest's packing run on
+    it, nested): every result equals the single-threaded one."""
+    import threading
+    names = ["d8-ehvi2", "d10-ei", "tiny", "d10-ehvi3"]
+    insts = [make_instance(nm, seeds(nm)[0], n_cand=16) for nm in names]
+    boxes = [1, 0, 1, 2]
+
+    def build(inst, bx):
+        buf = np.zeros(1 << 21, np.uint8)
+        st, _ = S.scoot_round_state_build(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                          inst.noise_var, inst.nodes, inst.tree_offset, inst.workload.leaf_scale,
+                                          buf, boxes=bx, h_ref=inst.ref, h_eps=inst.eps)
+        return bytes(buf[:st.bytes])
+
+    want = [build(i, b) for i, b in zip(insts, boxes)]
+    errors = []
+
+    def worker(k):
+        try:
+            for r in range(12):
+                j = (k + r) % len(insts)
+                if build(insts[j], boxes[j]) != want[j]:
+                    errors.append((k, r, j))
+        except Exception as e:  # reported below
+            errors.append(repr(e))
+
+    threads = [threading.Thread(target=worker, args=(k,)) for k in range(6)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors[:5]
