@@ -374,3 +374,31 @@ def test_round_state_build_concurrent_callers(S):
     for t in threads:
         t.join()
     assert not errors, errors[:5]
+
+
+def test_scratch_sizes_and_buffer_layout(S):
+    """Host-only sizing calls of the device builders: their documented
+    formulas, 16-byte (256-byte) alignment, and rejection of bad input."""
+    inst = make_instance("d8-ehvi2", seeds("d8-ehvi2")[0], n_cand=16)
+    for n in (1, 64, 160, 161, 640):
+        L = S.scoot_gp_layout_init(inst.space, n, 2, 0)
+        tri = n * (n + 1) // 2
+        want = 8 * 2 * (n * inst.d + tri * (1 if n <= 160 else 2))
+        assert S.scoot_gp_device_work_bytes(L) == want
+        for warped in (False, True):
+            up, blob, work, total = S.scoot_gp_device_buffer_layout(L, warped)
+            assert up % 256 == 0 and blob % 256 == 0 and work % 256 == 0 and total % 256 == 0
+            assert up <= blob and blob + L.bytes <= work and work + want <= total
+            need = 4 * inst.d * n + 4 * 2 * n + 4 * 2 * inst.d + 8 + (8 * 2 * inst.d if warped else 0)
+            assert up >= need
+    assert S.scoot_rf_train_work_bytes(256, 12) == 2 * 256 * 12
+    assert S.scoot_rf_train_work_bytes(7, 3) == 48  # 42 rounded up to 16
+    tri = 200 * 201 // 2
+    base = (200 * 10 * 8 + 255) // 256 * 256
+    assert S.scoot_gp_mle_work_bytes(200, 10, 3, 32) == base + 32 * 3 * 2 * tri * 8
+    assert S.scoot_gp_mle_work_bytes(128, 10, 1, 64) == (128 * 10 * 8 + 255) // 256 * 256
+    for bad in [(0, 10, 1, 1), (10, 0, 1, 1), (10, 10, 0, 1), (10, 10, 1, 0)]:
+        with pytest.raises(S.ScootError):
+            S.scoot_gp_mle_work_bytes(*bad)
+    with pytest.raises(S.ScootError):
+        S.scoot_rf_train_work_bytes(0, 3)
