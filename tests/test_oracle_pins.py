@@ -541,6 +541,150 @@ def test_fantasy_refit_properties():
     assert np.allclose(var1, np.maximum(var0 - c * c, 0), rtol=1e-8, atol=1e-11)
 
 
+def _hv2(points, ref):
+    """2-D hypervolume by the textbook sweep: points strictly above r, taken
+    in decreasing first objective, each adding the strip of its second
+    objective above the best one seen so far."""
+    P = sorted((p for p in np.asarray(points, np.float64) if p[0] > ref[0] and p[1] > ref[1]),
+               key=lambda p: (-p[0], -p[1]))
+    hv, top = 0.0, float(ref[1])
+    for p0, p1 in P:
+        if p1 > top:
+            hv += (p0 - ref[0]) * (p1 - top)
+            top = p1
+    return hv
+
+
+def _fantasy_from_scratch(inst, q, feasible):
+    """Sequential kriging-believer picks recomputed step by step from the
+    definitions, sharing nothing with the oracle's loop but GP and the
+    decoding: at step j a NEW GP per objective on the observations plus the
+    previous picks' words (fantasised values, noise tau^2), the fantasised
+    value of a pick taken as that step's own posterior mean at it, the front
+    as the points (observed and fantasised) no other point dominates, EHVI as
+    the mean over the base samples of HV(front + y_s) - HV(front) by the 2-D
+    sweep, picked candidates excluded, argmax with the lowest index."""
+    M = inst.n_obj
+    words = inst.cand[:, :inst.n_cand]
+    eligible = np.asarray(feasible, bool).copy()
+    picks, acqs, vars_, fvals, fronts = [], [], [], [], []
+    repick_needed = False
+    for j in range(q):
+        xw = np.concatenate([inst.x_obs, words[:, picks]], axis=1) if picks else inst.x_obs
+        gps = [O.GP(inst.space, xw, np.concatenate([inst.y_obs[m].astype(np.float64), [f[m] for f in fvals]]),
+                    inst.lengthscale[m], inst.signal_var[m], inst.noise_var[m]) for m in range(M)]
+        mv = [gp.posterior(words) for gp in gps]
+        mu = np.stack([a for a, _ in mv], 1)
+        var = np.stack([b for _, b in mv], 1)
+        pts = np.concatenate([inst.y_obs.T.astype(np.float64), np.array(fvals).reshape(-1, M)])
+        front = [p for p in pts if p[0] > inst.ref[0] and p[1] > inst.ref[1]
+                 and not any(np.all(z >= p) and np.any(z > p) for z in pts)]
+        base = _hv2(front, inst.ref)
+        sd = np.sqrt(var)
+        a = np.full(len(mu), -np.inf)
+        for i in range(len(mu)):
+            if feasible[i]:
+                ys = mu[i] + sd[i] * inst.eps
+                a[i] = np.mean([_hv2(front + [y], inst.ref) - base for y in ys])
+        val = np.where(eligible, a, -np.inf)
+        if not np.any(np.isfinite(val)):
+            break
+        p = int(np.flatnonzero(val == val.max())[0])
+        repick_needed |= bool(picks) and int(np.flatnonzero(a == a[feasible].max())[0]) in picks
+        picks.append(p)
+        acqs.append(a)
+        vars_.append(var)
+        fronts.append(np.array(front).reshape(-1, M))
+        fvals.append(np.array([gp.posterior(words[:, [p]])[0][0] for gp in gps]))
+        eligible[p] = False
+    return picks, acqs, vars_, fronts, repick_needed
+
+
+@pytest.mark.parametrize("noise", [None, 0.3])
+def test_fantasy_picks_equal_a_from_scratch_recomputation(noise):
+    """Pins the oracle's sequential-pick loop (refit GP, fantasised front,
+    exclusion, argmax) against a recomputation from scratch at every step.
+    With a large noise variance a picked candidate keeps a high EHVI after
+    its own fantasy, so the exclusion of picked candidates decides a pick."""
+    import dataclasses
+    inst = make_instance("tiny", seeds("tiny")[2], n_cand=160)
+    if noise is not None:
+        inst = dataclasses.replace(inst, noise_var=np.full(inst.n_obj, noise, np.float32))
+    feas = Stream(77, "feas").uniform(inst.n_cand) < 0.8
+    q = 5
+    ref = O.fantasy_picks(inst, q, feas)
+    picks, acqs, vars_, fronts, repick = _fantasy_from_scratch(inst, q, feas)
+    assert ref["picks"] == picks
+    for j in range(q):
+        ok = np.isfinite(acqs[j])
+        assert np.array_equal(ok, feas)
+        want = np.where(np.isin(np.arange(inst.n_cand), picks[:j]), -np.inf, acqs[j])
+        got = ref["acq"][j]
+        both = np.isfinite(got) & np.isfinite(want)
+        assert np.array_equal(np.isfinite(got), np.isfinite(want))
+        assert np.allclose(got[both], want[both], rtol=1e-9, atol=1e-12)
+        assert np.allclose(ref["var"][j], vars_[j], rtol=1e-8, atol=1e-12)
+        f_ref = np.array(sorted(map(tuple, ref["fronts"][j])))
+        f_new = np.array(sorted(map(tuple, fronts[j])))
+        assert f_ref.shape == f_new.shape and np.allclose(f_ref, f_new, rtol=1e-10, atol=1e-12)
+    if noise is not None:
+        assert repick, "the case must exercise the exclusion of picked candidates"
+
+
+def _hand_instance(targets, q_noise=1e-8):
+    """One observation x = 0 with y = (1, -1), one continuous parameter in
+    [0, 1], both objectives with lengthscale 0.25, s_f^2 = 1, tau^2 = 1e-8;
+    candidate i sits where the Matern-5/2 covariance with the observation is
+    targets[i], so its posterior mean is (k_i, -k_i) / (1 + tau^2)."""
+    from types import SimpleNamespace
+    from scipy.optimize import brentq
+    from workloads.generate import PARAM_DTYPE
+    space = np.zeros(1, PARAM_DTYPE)
+    space[0] = (3, 0, 0.0, 1.0)
+    ell = 0.25
+    xs = [brentq(lambda x: float(O.matern(x / ell, 1.0)) - t, 0.0, 1.0, xtol=1e-15) for t in targets]
+    n = len(xs)
+    cand = np.zeros((1, (n + 3) // 4 * 4), np.uint32)
+    cand[0, :n] = np.array(xs, np.float32).view(np.uint32)
+    k = np.array([float(O.matern(np.float32(x) / ell, 1.0)) for x in xs])
+    inst = SimpleNamespace(n_cand=n, cand=cand, space=space, x_obs=np.zeros((1, 1), np.uint32),
+                           y_obs=np.array([[1.0], [-1.0]], np.float32), lengthscale=np.full((2, 1), ell, np.float32),
+                           signal_var=np.ones(2, np.float32), noise_var=np.full(2, q_noise, np.float32), n_obj=2,
+                           eps=np.zeros((1, 2), np.float32), ref=np.array([-1.0, -1.5], np.float32))
+    return inst, k
+
+
+def test_fantasy_picks_hand_worked_one_observation():
+    """n = 1, M = 2, a single base sample eps = 0 (EHVI = HVI at the mean),
+    r = (-1, -1.5), candidates with k = 0.5, 0.2, 0.8, 0.25 (means (k, -k)).
+    Worked by hand from the rectangles of Section 4.4:
+      step 1: HVI = (k + 1)(1 - k) = 0.75, 0.96, 0.36, 0.9375 -> index 1;
+      step 2 (front + (0.2, -0.2)): k = 0.5 keeps (0.5 - 0.2) x (1 - 0.5)
+              = 0.15, k = 0.8 keeps 0.6 x 0.2 = 0.12, k = 0.25 keeps
+              0.05 x 0.75 = 0.0375 -> index 0 (a loop that kept the front
+              unchanged would take k = 0.25, index 3, the second-best value
+              of step 1);
+      step 3 (front + (0.5, -0.5)): k = 0.8 keeps 0.3 x 0.2 = 0.06, k = 0.25
+              keeps 0.05 x 0.25 = 0.0125 -> index 2;
+      step 4: index 3 with 0.0125;
+    and with q = 5 the loop stops after 4 picks (the candidates run out)."""
+    inst, k = _hand_instance([0.5, 0.2, 0.8, 0.25])
+    feas = np.ones(4, bool)
+    r2 = O.fantasy_picks(inst, 2, feas)
+    assert r2["picks"] == [1, 0]
+    assert np.allclose(r2["acq"][0], [0.75, 0.96, 0.36, 0.9375], atol=2e-6)
+    assert np.allclose(r2["acq"][1][[0, 2, 3]], [0.15, 0.12, 0.0375], atol=2e-6)
+    assert r2["acq"][1][1] == -np.inf
+    r5 = O.fantasy_picks(inst, 5, feas)
+    assert r5["picks"] == [1, 0, 2, 3]
+    assert r5["acq"][2][2] == pytest.approx(0.06, abs=2e-6)
+    assert r5["acq"][2][3] == pytest.approx(0.0125, abs=2e-6)
+    assert r5["acq"][3][3] == pytest.approx(0.0125, abs=2e-6)
+    # the fronts: the observation, then each fantasised mean (k, -k)
+    assert len(r5["fronts"][3]) == 4
+    assert np.allclose(sorted(r5["fronts"][3][:, 0]), sorted([1.0, k[1], k[0], k[2]]), atol=1e-7)
+
+
 # ------------------------------------------------------------------ MACE (Sections 4.5 and 4.7)
 
 def test_pi_closed_form_matches_quadrature():
