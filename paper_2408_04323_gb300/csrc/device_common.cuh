@@ -156,9 +156,12 @@ __device__ __forceinline__ float feature_of(uint32_t w, int kind, float a, float
 // Selection key of a candidate (Section 4.7 order): the high word is the
 // value mapped to an order-preserving unsigned integer, the low word is
 // 0xFFFFFFFF - index, so a larger key is a larger value or, on equal
-// values, a lower index.  0 is never a key of an eligible candidate.
+// values, a lower index.  -0 and +0 are one value (the comparison of the
+// selection rule is numeric), so -0 is mapped to +0 first.  0 is never a key
+// of an eligible candidate.
 __device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
     uint32_t b = __float_as_uint(v);
+    if (b == 0x80000000u) b = 0u;
     b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
     return ((uint64_t)b << 32) | (uint64_t)(0xFFFFFFFFu - idx);
 }
