@@ -634,7 +634,10 @@ scoot_status scoot_select_pareto(scoot_ctx* ctx, const float* acq, int64_t lda, 
  * library keeps until the process exits; a call uses at most blocks * q <=
  * 32768 keys, so no pool size overflows it.  The first call on a device
  * looks up the array's device address (make that first call before any
- * stream capture).  All calls share the array: calls that overlap on the GPU
+ * stream capture); a lookup that fails returns SCOOT_ECUDA and is tried
+ * again by the next call.  An error left pending by the caller's earlier
+ * CUDA work is cleared before the launches, so the status reports only this
+ * call's own.  All calls share the array: calls that overlap on the GPU
  * (different streams, or different host threads) race and must not be
  * issued; calls ordered on one stream are safe.  Nothing needs clearing
  * between calls: every entry read is written by the same call.  Errors:

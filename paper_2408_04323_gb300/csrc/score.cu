@@ -167,12 +167,21 @@ __device__ __forceinline__ float ehvi_partial_sat(const float* mu, const float* 
     return total;
 }
 
-// True (in every thread) when every staged box is open on the last objective.
-__device__ __forceinline__ bool boxes_fast(const float4* bhi, int n_boxes, int M) {
-    int ok = 1;
-    for (int b = threadIdx.x; b < n_boxes; b += blockDim.x) {
-        const float4 h = bhi[b];
+// True (in every thread) when the saturated form is exact for the staged
+// boxes: every box is open on the last objective, M <= 3, and every lower
+// corner lies within 2^30 of zero.  The form folds one open width 2^40 per
+// open leading axis into W, so W <= 2^80 and |C| <= 2^110 for M <= 3 (finite
+// in fp32 for samples within 2^40 of the corner); with M = 4 the last box
+// would carry W = 2^120, whose products with y_last and l_last overflow (and
+// whose reciprocal factors underflow) at ordinary objective scales, so M = 4
+// always takes the general form.
+__device__ __forceinline__ bool boxes_fast(const float4* blo, const float4* bhi, int n_boxes, int M) {
+    int ok = M <= 3;
+    constexpr float kCornerMax = 1073741824.0f;  // 2^30
+    for (int b = threadIdx.x; b < n_boxes && ok; b += blockDim.x) {
+        const float4 h = bhi[b], l = blo[b];
         ok &= (M == 2 ? h.y : (M == 3 ? h.z : h.w)) == INFINITY;
+        ok &= fabsf(l.x) < kCornerMax && fabsf(l.y) < kCornerMax && (M < 3 || fabsf(l.z) < kCornerMax);
     }
     return __syncthreads_and(ok) != 0;
 }
@@ -275,7 +284,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     __syncthreads();
     // Boxes open on the last objective (as scoot_boxes_build makes them) are
     // restaged in saturated form over the same storage (2 float4 per box).
-    const bool fast = EPI == kEHVI ? boxes_fast(bhi, a.n_boxes, M) : false;
+    const bool fast = EPI == kEHVI ? boxes_fast(blo, bhi, a.n_boxes, M) : false;
     if (EPI == kEHVI && fast) {
         stage_boxes_sat(a.box_lo, a.box_hi, a.n_boxes, M, blo);
         __syncthreads();

@@ -179,9 +179,25 @@ constexpr int kStaticKeys = 32768;  // 256 KiB of 64-bit keys
 static __device__ __align__(256) uint64_t g_topq_scratch[kStaticKeys];
 
 constexpr int kMaxDevices = 64;
-std::once_flag g_scratch_once[kMaxDevices];
-uint64_t* g_scratch_ptr[kMaxDevices];
-cudaError_t g_scratch_err[kMaxDevices];
+std::mutex g_scratch_mutex;
+uint64_t* g_scratch_ptr[kMaxDevices];  // guarded by g_scratch_mutex; NULL until a lookup succeeds
+
+// Device address of the scratch array on `device` (current), looked up on
+// the first call that needs it.  A failed lookup is not remembered: the next
+// call tries again, so one call made at a bad moment (inside a stream
+// capture, say) does not disable the entry point for the process.
+uint64_t* scratch_on(int device) {
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    if (!g_scratch_ptr[device]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_topq_scratch) != cudaSuccess) {
+            cudaGetLastError();  // this call reports the failure; leave no error pending
+            return nullptr;
+        }
+        g_scratch_ptr[device] = static_cast<uint64_t*>(p);
+    }
+    return g_scratch_ptr[device];
+}
 
 }  // namespace
 
@@ -196,17 +212,15 @@ extern "C" scoot_status scoot_select_topq_static(const float* acq, const uint8_t
         cudaGetLastError();
         return SCOOT_ECUDA;
     }
-    // First call on a device: look up the device address of the scratch
-    // array with that device current (host code cannot use the symbol's
-    // name as a device pointer).
-    std::call_once(g_scratch_once[device], [device] {
-        void* p = nullptr;
-        g_scratch_err[device] = cudaGetSymbolAddress(&p, g_topq_scratch);
-        g_scratch_ptr[device] = static_cast<uint64_t*>(p);
-    });
-    if (g_scratch_err[device] != cudaSuccess || !g_scratch_ptr[device]) return SCOOT_ECUDA;
+    // Host code cannot use the array's name as a device pointer: its address
+    // on this device is looked up with the device current.
+    uint64_t* partial = scratch_on(device);
+    if (!partial) return SCOOT_ECUDA;
     int sms = 0;
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) return SCOOT_ECUDA;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {
+        cudaGetLastError();
+        return SCOOT_ECUDA;
+    }
     // Blocks are capped so that blocks * q keys fit the array; every key pass
     // 2 reads is written by pass 1 of the same call, so nothing needs clearing.
     int64_t blocks = (n + kTopqThreads * 8 - 1) / (kTopqThreads * 8);
@@ -215,8 +229,10 @@ extern "C" scoot_status scoot_select_topq_static(const float* acq, const uint8_t
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
     const int64_t slice = (n + blocks - 1) / blocks;
-    uint64_t* partial = g_scratch_ptr[device];
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // An error left pending by the caller's earlier work is not this call's:
+    // clear it so that the status below reports only these two launches.
+    cudaGetLastError();
     auto go = [&](auto p1, auto p2) {
         p1<<<(unsigned)blocks, kTopqThreads, 0, st>>>(acq, mask, n, slice, q, partial);
         p2<<<1, kMergeThreads, 0, st>>>(partial, blocks * q, q, idx, val, count);

@@ -389,6 +389,46 @@ def test_score_ehvi_bounded_boxes(S, ctx, name):
     assert report_tol(f"score_ehvi bounded boxes {name} (B={2 * len(lo)})", out[1][idx], want, tol).max() <= 1.0
 
 
+def test_score_ehvi_four_objectives_at_large_scale(S, ctx):
+    """The fused 4-objective EHVI on objectives of magnitude ~1e3 (the
+    library's last box is open on all three leading axes): the kernel must
+    not fold the open widths into one product that overflows fp32, and must
+    match the oracle's Monte-Carlo EHVI (Eq. 7) within the propagated bar."""
+    inst = make_instance("tiny", seeds("tiny")[1], n_cand=4096 + 37)
+    n = inst.n_cand
+    y = inst.y_obs.astype(np.float64)
+    Y = (np.stack([y[0], y[1], -0.5 * y[0] + 0.2 * y[1], 0.3 * y[0] - 0.6 * y[1]]) * 1000.0 + 500.0)
+    Y = Y.astype(np.float32)
+    M = 4
+    ell = np.ascontiguousarray(inst.lengthscale[[0, 1, 0, 1]])
+    sv = np.full(M, 1e6, np.float32)
+    nv = np.full(M, 1e6 * float(inst.noise_var[0]), np.float32)
+    ref = Y.min(axis=1)
+    eps = Stream(4242, "eps4").normal(64 * M).reshape(64, M).astype(np.float32)
+    L = S.scoot_gp_layout_init(inst.space, inst.n_obs, M)
+    blob, _ = S.scoot_gp_prepare(inst.space, inst.x_obs, Y, ell, sv, nv, L)
+    lo, hi, fs = S.scoot_boxes_build(Y, ref)
+    assert np.all(np.isinf(hi[:, -1])) and np.any(np.all(np.isinf(hi[:, :-1]), axis=1))
+    cand = cand_dev(inst)
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
+    acq = torch.empty(n, device="cuda")
+    S.scoot_score_ehvi(ctx, L, dev(blob), cand, n, dev(lo), dev(hi), dev(eps), acq, mask)
+    g = np_(acq)
+    known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
+    assert np.array_equal(np.isfinite(g), known)
+    assert not np.any(np.isnan(g))
+    idx = sample_idx(n, 512, 11)
+    idx = idx[known[idx]]
+    gps = [O.GP(inst.space, inst.x_obs, Y[m], ell[m], sv[m], nv[m]) for m in range(M)]
+    mu, var, e_mu, e_var = posterior_tols(gps, np.ascontiguousarray(inst.cand[:, idx]))
+    front = O.pareto_front(Y.T.astype(np.float64), ref.astype(np.float64))
+    f = lambda a, b: O.ehvi_mc(a, b, eps, front, ref.astype(np.float64))
+    want, tol = propagated_tol(f, mu, var, e_mu, e_var)
+    assert np.any(want > 1e6)  # volumes at the scale of the objectives
+    assert report_tol(f"score_ehvi M=4 at scale 1e3 (P={fs}, B={len(lo)})", g[idx], want, tol).max() <= 1.0
+
+
 def test_score_ei_parity(S, ctx):
     name = "d10-ei"
     inst = make_instance(name, seeds(name)[0])
@@ -432,6 +472,32 @@ def test_topq_bit_exact_on_generated_arrays(S, ctx, n, q):
         assert gi[:c].tolist() == want.tolist()
         assert np.array_equal(gv[:c], acq[want])
         assert np.all(gi[c:] == -1) and np.all(gv[c:] == -np.inf)
+
+
+def test_topq_signed_zeros_are_one_value(S, ctx):
+    """-0 and +0 compare equal in the selection rule (Section 4.7 order), so
+    among interleaved -0/+0 values the lowest indices win, whatever the sign
+    bit; the static entry point agrees."""
+    n, q = 4099, 16
+    cases = []
+    for neg in (0, 1):  # -0 at the even indices, then at the odd ones
+        a = np.zeros(n, np.float32)
+        a[neg::2] = -0.0
+        a[5] = -1.0
+        a[n - 1] = -np.inf
+        cases.append(a)
+    assert np.signbit(cases[0][0]) and not np.signbit(cases[1][0])
+    for a in cases:
+        idx = torch.empty(q, dtype=torch.int64, device="cuda")
+        val = torch.empty(q, device="cuda")
+        cnt = torch.empty(1, dtype=torch.int32, device="cuda")
+        S.scoot_select_topq(ctx, dev(a), n, q, idx, val, cnt)
+        want, _, c = O.select_topq(a.astype(np.float64), None, q)
+        assert int(np_(cnt)[0]) == c == q
+        assert np_(idx).tolist() == want.tolist() == [0, 1, 2, 3, 4] + list(range(6, 17))
+        assert np.all(np_(val) == 0.0)
+        S.scoot_select_topq_static(dev(a), n, q, idx, val, cnt)
+        assert np_(idx).tolist() == want.tolist()
 
 
 def test_topq_degenerate(S, ctx):

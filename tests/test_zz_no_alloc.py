@@ -4,11 +4,12 @@ It serves callers that cannot allocate device memory when they select, so
 it keeps its partial results in a fixed device array instead of a context
 workspace.  Its picks must equal scoot_select_topq's exactly, on calls made
 one after the other on the same stream (the second call sees the array as
-the first left it).  This file is collected last so that a failure here does
+the first left it), and the oracle's selection.  This file is collected last so that a failure here does
 not hide any other test."""
 import numpy as np
 import pytest
 
+import oracle as O
 from workloads import Stream
 
 torch = pytest.importorskip("torch")
@@ -56,6 +57,12 @@ def test_static_topq_matches_workspace_topq_on_consecutive_calls(S):
             for w, g in zip(want, got):
                 assert torch.equal(w.cpu(), g.cpu()), (seed, n, q)
             assert int(got[2].item()) > 0
+            # and the oracle's selection (Section 4.7 order) on the same values
+            a_h = acq.cpu().numpy().astype(np.float64)
+            oi, ov, oc = O.select_topq(a_h, None if m is None else mask.cpu().numpy(), q)
+            assert int(got[2].item()) == oc
+            assert got[0].cpu().numpy()[:oc].tolist() == oi.tolist()
+            assert np.array_equal(got[1].cpu().numpy()[:oc].astype(np.float64), ov)
     finally:
         ctx.close()
 
