@@ -707,9 +707,9 @@ def main():
         if evs:
             evs[2].record(stream)
         if inp.fantasy:
-            S.scoot_suggest_fantasy(ctx, st.gp_layout, st.gp_state, inp.space, inp.x_obs, inp.y_obs,
-                                    inp.lengthscale, inp.signal_var, inp.noise_var, cand, N, inp.ref, st.eps,
-                                    inp.q, rnd.work, mask=rnd.mask, stream=stream)
+            S.scoot_suggest_fantasy(ctx, st.gp_layout, st.gp_state, st.fant_state, st.fant_box_cap, cand, N, st.eps,
+                                    inp.q, rnd.work, rnd.top_idx, rnd.top_val, rnd.top_count, mask=rnd.mask,
+                                    stream=stream)
             if evs:
                 evs[3].record(stream)
                 evs[4].record(stream)
@@ -765,23 +765,22 @@ def main():
     eager_ms = statistics.mean(e[0].elapsed_time(e[4]) for e in evs)
 
     # The step as one CUDA graph (its launches and memsets replayed without
-    # host gaps); the fantasy round synchronises with the host and stays eager.
+    # host gaps).
     graph = None
-    if not inp.fantasy:
-        try:
-            cap = torch.cuda.Stream(device)
-            cap.wait_stream(stream)
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph, stream=cap, capture_error_mode="thread_local"):
-                step(stream=cap)
-            torch.cuda.synchronize(device)
-            for _ in range(3):
-                graph.replay()
-            torch.cuda.synchronize(device)
-        except Exception as e:  # capture refused: time eager launches instead
-            graph = None
-            print(f"# CUDA graph capture unavailable ({e}); timing eager launches", file=sys.stderr)
-            torch.cuda.synchronize(device)
+    try:
+        cap = torch.cuda.Stream(device)
+        cap.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=cap, capture_error_mode="thread_local"):
+            step(stream=cap)
+        torch.cuda.synchronize(device)
+        for _ in range(3):
+            graph.replay()
+        torch.cuda.synchronize(device)
+    except Exception as e:  # capture refused: time eager launches instead
+        graph = None
+        print(f"# CUDA graph capture unavailable ({e}); timing eager launches", file=sys.stderr)
+        torch.cuda.synchronize(device)
 
     # The timed K steps.
     if dist:
@@ -878,11 +877,9 @@ def main():
             S.scoot_rf_predict(ctx, state.forest_layout, state.forest, inp.space, cand_e2e, N, inp.delta_num,
                                inp.delta_den, rnd.votes, rnd.mask, None, stream)
             if inp.fantasy:
-                idx_h, val_h = S.scoot_suggest_fantasy(ctx, state.gp_layout, state.gp_state, inp.space, inp.x_obs,
-                                                       inp.y_obs, inp.lengthscale, inp.signal_var, inp.noise_var,
-                                                       cand_e2e, N, inp.ref, state.eps, inp.q, rnd.work,
-                                                       mask=rnd.mask, stream=stream)
-                rnd.top_idx[:len(idx_h)].copy_(torch.from_numpy(idx_h))
+                S.scoot_suggest_fantasy(ctx, state.gp_layout, state.gp_state, state.fant_state, state.fant_box_cap,
+                                        cand_e2e, N, state.eps, inp.q, rnd.work, rnd.top_idx, rnd.top_val,
+                                        rnd.top_count, mask=rnd.mask, stream=stream)
             elif inp.acq == "ei":
                 S.scoot_score_ei(ctx, state.gp_layout, state.gp_state, cand_e2e, N, inp.xi, rnd.acq, rnd.mask, stream)
             elif inp.acq == "mace":

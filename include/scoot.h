@@ -435,6 +435,8 @@ typedef struct {
     const float* eps;            /* [S][M] (boxes == 1) */
     int32_t n_mc;                /* S */
     int32_t grid_cap;            /* boxes == 2: coordinates per axis (0: 256) */
+    int32_t fantasy_q;           /* > 0: also the fantasy state for this many picks (needs ref; no warp,
+                                    gp_on_device 0) */
 } scoot_round_inputs;
 
 /* Where scoot_round_state_build put each part in the buffer (256-byte
@@ -442,6 +444,8 @@ typedef struct {
 typedef struct {
     int64_t bytes;               /* bytes used: the upload */
     int64_t off_gp, off_forest, off_box_lo, off_box_hi, off_eps, off_grid, off_corner;
+    int64_t off_fant;            /* fantasy state (fantasy_q > 0) */
+    int32_t fant_box_cap;        /* its box_cap */
     int32_t n_boxes, front_size;
     int32_t grid_cap;
     int32_t n_grid[SCOOT_MAX_OBJ];
@@ -453,7 +457,9 @@ typedef struct {
 /* A round's host-side state in one buffer h_buf (cap bytes, host): the GP
  * blob (scoot_gp_prepare_warped), the packed forest (scoot_forest_pack) and,
  * as asked, the boxes (scoot_boxes_build) with eps or with their grid index
- * (scoot_boxes_index).  Copy the first out->bytes bytes to the device as
+ * (scoot_boxes_index), and the fantasy state (scoot_fantasy_prepare, from
+ * the GP blob's own factorisation).  Copy the first out->bytes bytes to the
+ * device as
  * they are.  The GP factorisation runs on a library worker thread while the
  * calling thread packs the forest and builds the boxes.  SCOOT_ENOMEM if
  * cap is too small (out->bytes then holds the size needed); the errors of
@@ -541,11 +547,35 @@ scoot_status scoot_rf_train_work_bytes(int32_t n, int32_t d, int64_t* bytes);
 
 /* ------------------------------------------------------------------ 6. sequential fantasised picks */
 
+/* Bytes of the fantasy state of a GP layout and q picks (host buffer of
+ * scoot_fantasy_prepare; about 8 M n^2 bytes). */
+scoot_status scoot_fantasy_state_bytes(const scoot_gp_layout* layout, int32_t q, int64_t* bytes);
+
+/* The fp64 state of q sequential fantasised picks, on the host, into h_out
+ * (cap bytes, 256-byte aligned when copied to the device): the covariance
+ * inputs of the observations (their features, lengthscales, s_f^2, tau^2),
+ * alpha = (K + tau^2 I)^{-1} y and L^{-1} (K + tau^2 I = L L^T) in fp64 per
+ * objective (Section 4.3), the reference point and the Pareto front of the
+ * observations (Section 4.4).  The inputs are those scoot_gp_prepare takes
+ * (unwarped states only) plus h_ref [M] and q.  *box_cap (may be NULL)
+ * receives the number of boxes the picks may need: the box_cap argument of
+ * scoot_fantasy_work_bytes and scoot_suggest_fantasy.  Errors: SCOOT_ENOMEM
+ * if cap < scoot_fantasy_state_bytes; SCOOT_EINVAL on bad inputs or a matrix
+ * that is not positive definite; SCOOT_EUNSUPPORTED for M outside 2..4 or q
+ * outside 1..SCOOT_MAX_Q.  (scoot_round_state_build can write the same state
+ * beside the GP blob from one factorisation.) */
+scoot_status scoot_fantasy_prepare(const scoot_param* h_space, const scoot_gp_layout* layout,
+                                   const uint32_t* h_x_obs, int64_t ld_obs, const float* h_y,
+                                   const float* h_lengthscale, const float* h_signal_var,
+                                   const float* h_noise_var, const float* h_ref, int32_t q, void* h_out,
+                                   int64_t cap, int32_t* box_cap);
+
 /* Bytes of the caller-owned device work buffer scoot_suggest_fantasy needs
- * for a pool of n candidates and q picks (about 4 n (M (2 + 64 n_rb + q) + 1)
- * bytes: moments, whitened covariance rows and downdate factors of every
- * candidate). */
-scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* layout, int64_t n, int32_t q, int64_t* bytes);
+ * for a pool of n candidates, q picks and box_cap boxes (about
+ * 4 n M (2 + 64 n_rb + q) bytes: moments, whitened covariance rows and
+ * downdate factors of every candidate). */
+scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* layout, int64_t n, int32_t q, int32_t box_cap,
+                                      int64_t* bytes);
 
 /* q sequential EHVI picks with kriging-believer fantasies (a variant of the
  * parallel suggestion of Section 4.7, whose picks are plain top-k): pick 1 is
@@ -553,24 +583,28 @@ scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* layout, int64_t n, 
  * NULL); after each pick p every objective's value at x_p is fantasised as
  * its posterior mean, the GP is conditioned on it with noise tau^2 (means
  * unchanged, variances lowered by a rank-1 term), the fantasised point joins
- * the Pareto front above h_ref (boxes rebuilt on the host), and the next
- * pick is the EHVI argmax among the candidates not yet picked.  Ties go to
- * the lowest index.  The GP host inputs (h_x_obs [d][ld_obs], h_y [M][n],
- * h_lengthscale, h_signal_var, h_noise_var) must be those the state blob was
- * prepared from; the per-pick rank-1 terms are computed from them in fp64.
- * eps: device base samples [S][M].  work: device buffer of at least
- * scoot_fantasy_work_bytes bytes, 256-byte aligned.  Outputs: h_idx, h_val
- * (host, [q]) and *h_count (fewer than q when the candidates run out); if
- * var_out is not NULL (device [M][n]) it receives the variances after the
- * last downdate for candidates with mask[i] == 1.  Synchronous: returns after
- * the picks are on the host.  2 <= M <= 4, 1 <= q <= SCOOT_MAX_Q. */
+ * the Pareto front above the reference point (boxes rebuilt on the device),
+ * and the next pick is the EHVI argmax among the candidates not yet picked.
+ * Ties go to the lowest index.  state: the GP blob; fant_state: the device
+ * copy (256-byte aligned) of scoot_fantasy_prepare's output for the same
+ * inputs, with q no larger than the q it was prepared for; box_cap as it
+ * returned (or larger).  eps: device base samples [S][M].  work: device
+ * buffer of at least scoot_fantasy_work_bytes bytes, 256-byte aligned.
+ * Outputs (device): idx int64 [q] and val float [q] (the picks and their
+ * EHVI values; -1 and -inf beyond the count), count int32 [1] (fewer than q
+ * when the candidates run out); if var_out is not NULL (device [M][n]) it
+ * receives the variances after the last downdate for candidates with
+ * mask[i] == 1.  Asynchronous on `stream`, with no host synchronisation:
+ * the rank-1 terms of every pick are computed on the device in fp64 from
+ * fant_state.  Errors found on the device (a fantasy state that does not
+ * match the GP layout or a warped GP state: SCOOT_EINVAL; more boxes than
+ * box_cap: SCOOT_EUNSUPPORTED) stop the picks and are reported by
+ * scoot_ctx_check.  2 <= M <= 4, 1 <= q <= SCOOT_MAX_Q, n < 2^31. */
 scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
-                                   const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
-                                   const float* h_y, const float* h_lengthscale, const float* h_signal_var,
-                                   const float* h_noise_var, const uint32_t* cand, int64_t n, int64_t ld,
-                                   const uint8_t* mask, const float* h_ref, const float* eps, int32_t n_mc,
-                                   int32_t q, void* work, int64_t work_bytes, int64_t* h_idx, float* h_val,
-                                   int32_t* h_count, float* var_out, void* stream);
+                                   const void* fant_state, int32_t box_cap, const uint32_t* cand, int64_t n,
+                                   int64_t ld, const uint8_t* mask, const float* eps, int32_t n_mc, int32_t q,
+                                   void* work, int64_t work_bytes, int64_t* idx, float* val, int32_t* count,
+                                   float* var_out, void* stream);
 
 /* ------------------------------------------------------------------ 7. MACE (Sections 4.5 and 4.7) */
 

@@ -508,7 +508,7 @@ def score_round(inst, acq_kind: str, xi: float = 1e-4, kernel: int = MATERN52,
 # 6. sequential picks with fantasies
 
 def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
-                  forced: list | None = None):
+                  forced: list | None = None, subset=None):
     """q sequential EHVI picks with kriging-believer fantasies (refit form).
 
     After each pick p the GP of every objective is conditioned again on the
@@ -516,17 +516,28 @@ def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
     with mu(x_p) added, and EHVI is recomputed over the pool with the picked
     candidates excluded.  ``forced`` replays a given pick sequence (to follow
     another implementation's choices step by step) instead of taking argmax.
-    Returns the picks and the acquisition array of each step.
+    ``subset`` (pool indices; with ``forced`` only) evaluates the steps at
+    those candidates and the forced picks alone, for pools too large to
+    evaluate whole.  Returns the picks, the evaluated indices and the
+    acquisition, variance, mean and front of each step (arrays over the
+    evaluated indices).
     """
     n = inst.n_cand
     words = inst.cand[:, :n]
+    if subset is None:
+        sel = np.arange(n)
+    else:
+        if forced is None:
+            raise ValueError("subset needs forced picks")
+        sel = np.unique(np.concatenate([np.asarray(subset, np.int64), np.asarray(forced[:q], np.int64)]))
+    where = {int(i): k for k, i in enumerate(sel)}
     gps = [GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m],
               inst.signal_var[m], inst.noise_var[m], kernel) for m in range(inst.n_obj)]
-    u_pool, _ = gp_features(inst.space, decode(inst.space, words, n))
+    u_pool, _ = gp_features(inst.space, decode(inst.space, np.ascontiguousarray(words[:, sel]), len(sel)))
     mu0 = np.stack([gp.posterior_u(u_pool)[0] for gp in gps], axis=1)
     Yf = inst.y_obs.T.astype(np.float64)
     picks, acqs, mus, vars_, fronts = [], [], [], [], []
-    eligible = np.asarray(feasible, bool).copy()
+    eligible = np.asarray(feasible, bool)[sel].copy()
     for j in range(q):
         var = np.stack([gp.posterior_u(u_pool)[1] for gp in gps], axis=1)
         front = pareto_front(Yf, inst.ref)
@@ -534,21 +545,24 @@ def fantasy_picks(inst, q: int, feasible: np.ndarray, kernel: int = MATERN52,
         a = ehvi_mc(mu0, var, inst.eps, front, inst.ref)
         a = np.where(eligible, a, -np.inf)
         if forced is not None:
+            if j >= len(forced):
+                break
             p = int(forced[j])
         else:
             idx, _, cnt = select_topq(a, None, 1)
             if cnt == 0:
                 break
-            p = int(idx[0])
+            p = int(sel[idx[0]])
+        k = where[p]
         picks.append(p)
         acqs.append(a)
         vars_.append(var)
         mus.append(mu0)
-        eligible[p] = False
+        eligible[k] = False
         for m, gp in enumerate(gps):
-            gp.add_observations(u_pool[p:p + 1], [mu0[p, m]])
-        Yf = np.concatenate([Yf, mu0[p:p + 1]], axis=0)
-    return dict(picks=picks, acq=acqs, var=vars_, mu=mus, fronts=fronts)
+            gp.add_observations(u_pool[k:k + 1], [mu0[k, m]])
+        Yf = np.concatenate([Yf, mu0[k:k + 1]], axis=0)
+    return dict(picks=picks, index=sel, acq=acqs, var=vars_, mu=mus, fronts=fronts)
 
 
 # --------------------------------------------------------------------------

@@ -14,14 +14,21 @@
 // is recomputed over the pool with the picks excluded, and the next pick is
 // its argmax (lowest index on ties).
 //
-// Device: one posterior pass storing mean, variance and V for the live
-// candidates (list-position order); per pick an EHVI pass, an argmax and a
-// downdate pass that reads V once.  Host, fp64, per pick: the picked point's
-// features, k(X, x_p), v_p, mu(x_p), the c_l(x_p) and s_j.
+// Everything runs on the device, in stream order, with no host round trip
+// (so a whole call can be captured in a CUDA graph):
+//   once     compaction of the live candidates; one posterior pass storing
+//            mean, variance and V for them by list position (score.cu);
+//            fant_init (one block): the observations' front and its boxes;
+//   pick j   fant_pass (every live candidate): the downdate of pick j-1, which
+//            reads the candidate's rows of V once, then its EHVI over the
+//            boxes staged in shared memory, and a per-block argmax;
+//            fant_pick (one block per objective): the argmax, then the pick's
+//            rank-1 terms in fp64 from the fantasy state (k(X, x_p),
+//            v_p = L^{-1} k, mu(x_p), c_l(x_p), s_j); the last block to finish
+//            adds the fantasised point to the front and rebuilds the boxes.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
-#include <vector>
 
 #include "device_common.cuh"
 #include "internal.h"
@@ -30,152 +37,599 @@ namespace {
 
 using namespace scoot_dev;
 
-constexpr int kFThreads = 128;
-constexpr int kBoxCap = 4096;
-constexpr int kArgBlocks = 1024;
+constexpr int kPassThreads = 256;
+constexpr int kPickThreads = 256;
+constexpr int kPartMax = 2048;   // per-block argmax partials of one pass
+
+// Control words of one call, in the work buffer.
+struct Ctrl {
+    uint32_t done;      // 1 once the loop has stopped (no eligible candidate left, or an error)
+    uint32_t arrived;   // fant_pick blocks that finished their objective (the last resets it)
+    int32_t n_boxes;
+    int32_t n_front;
+    int64_t pick_idx;   // candidate index of the latest pick
+    int64_t pick_pos;   // its list position
+};
 
 struct FantArgs {
     const int32_t* list;          // list position -> candidate index (NULL: identity)
-    int64_t n_live, ldc;
+    const unsigned int* n_list;   // live candidates (device; NULL: n)
+    int64_t n, ldc;
     const float* mean;            // [M][ldc]
     float* var;                   // [M][ldc]
     const float* V;               // [M][n_pad][ldc]
-    float* C;                     // [q][M][ldc]
-    const float* vp;              // [M][n_pad]
-    const float* cxp;             // [M][q]
-    const float* inv_s;           // [M]
-    const int64_t* picked;
-    int32_t n_picked, n_pad, q, j;
-    float* acq;                   // [ldc]
-    const char* state;
+    float* C;                     // [q][M][ldc] downdate factors c_l of every candidate
+    int32_t n_obs, n_pad, d, kernel, q, n_mc, box_cap, front_cap;
+    const char* gp;               // GP state blob (fp32; feature order)
     int64_t off_fmap, off_ils, off_scal;
-    int32_t n_obs, d, kernel;
+    const char* fant;             // fantasy state (fp64; parameter order)
     const uint32_t* cand;
-    int64_t ld, p;
-    const float* box_lo;
-    const float* box_hi;
-    int32_t n_boxes;
-    const float* eps;
-    int32_t n_mc;
-    uint64_t* partial;
-    uint64_t* best;
+    int64_t ld;
+    const float* eps;             // [S][M]
+    float* box_lo;                // [box_cap][M]
+    float* box_hi;
+    double* cell;                 // [box_cap] floor of each grid cell (box builder scratch)
+    double* front;                // [front_cap][M]
+    Ctrl* ctrl;
+    int64_t* picked_pos;          // [q]
+    float* vp;                    // [M][n_pad] v_p of the latest pick (fp32, zero-padded)
+    float* cxp;                   // [M][q] c_l(x_p) of the latest pick
+    float* inv_s;                 // [M] 1 / s of the latest pick
+    double* upick;                // [q][d] features of the picks
+    double* vpick;                // [q][M][n] v_p of the picks
+    double* cpick;                // [q][M][q] c_l(x_p) of the picks
+    double* spick;                // [q][M]
+    double* mupick;               // [q][M] fantasised values
+    uint64_t* part_key;           // [kPartMax]
+    int32_t* part_pos;
+    int64_t* out_idx;             // [q]
+    float* out_val;               // [q]
+    int32_t* out_count;
+    uint32_t* err;
 };
 
-template <int M>
-__global__ void __launch_bounds__(kFThreads) fant_ehvi(const __grid_constant__ FantArgs a) {
-    extern __shared__ __align__(16) float sm[];
-    float4* blo = reinterpret_cast<float4*>(sm);
-    float4* bhi = blo + a.n_boxes;
-    float4* epsv = bhi + a.n_boxes;
-    stage_boxes(a.box_lo, a.box_hi, a.n_boxes, a.eps, a.n_mc, M, blo, bhi, epsv);
-    __syncthreads();
-    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < a.n_live;
-         pos += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
-        bool taken = false;
-        for (int k = 0; k < a.n_picked; ++k) taken |= a.picked[k] == i;
-        float v = -INFINITY;
-        if (!taken) {
-            float mu[M], sd[M];
-#pragma unroll
-            for (int m = 0; m < M; ++m) {
-                mu[m] = a.mean[(int64_t)m * a.ldc + pos];
-                sd[m] = sqrtf(fmaxf(a.var[(int64_t)m * a.ldc + pos], 0.0f));
-            }
-            v = ehvi_value<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc);
-        }
-        a.acq[pos] = v;
+__device__ __forceinline__ void keymax(uint64_t& k, int32_t& p, uint64_t k2, int32_t p2) {
+    if (k2 > k) {
+        k = k2;
+        p = p2;
     }
 }
 
-__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-    for (int o = 16; o > 0; o >>= 1) {
-        const uint64_t w = __shfl_xor_sync(0xffffffffu, v, o);
-        v = w > v ? w : v;
-    }
-    return v;
-}
-
-__device__ __forceinline__ uint64_t block_max_u64(uint64_t v) {
-    __shared__ uint64_t wm[32];
+// Block-wide maximum of (key, position); valid in thread 0.
+__device__ __forceinline__ void block_keymax(uint64_t& k, int32_t& p) {
+    __shared__ uint64_t wk[32];
+    __shared__ int32_t wp[32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    v = warp_max_u64(v);
-    if (lane == 0) wm[warp] = v;
+    for (int o = 16; o > 0; o >>= 1) keymax(k, p, __shfl_xor_sync(0xffffffffu, k, o), __shfl_xor_sync(0xffffffffu, p, o));
+    if (lane == 0) {
+        wk[warp] = k;
+        wp[warp] = p;
+    }
     __syncthreads();
-    v = threadIdx.x < (blockDim.x >> 5) ? wm[threadIdx.x] : 0ull;
-    if (warp == 0) v = warp_max_u64(v);
-    return v;  // valid in thread 0
+    if (warp == 0) {
+        k = lane < (int)(blockDim.x >> 5) ? wk[lane] : 0ull;
+        p = lane < (int)(blockDim.x >> 5) ? wp[lane] : -1;
+        for (int o = 16; o > 0; o >>= 1)
+            keymax(k, p, __shfl_xor_sync(0xffffffffu, k, o), __shfl_xor_sync(0xffffffffu, p, o));
+    }
+    __syncthreads();
 }
 
-// Argmax over list positions with the selection key of the candidate index.
-__global__ void __launch_bounds__(kFThreads) fant_argmax1(const __grid_constant__ FantArgs a) {
-    uint64_t best = 0ull;
-    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < a.n_live;
-         pos += (int64_t)gridDim.x * blockDim.x) {
-        const float v = a.acq[pos];
-        if (!(v != v) && v != -INFINITY) {
-            const uint64_t k = make_key(v, (uint32_t)(a.list ? a.list[pos] : pos));
-            best = k > best ? k : best;
+__device__ __forceinline__ double block_sum(double v, double* scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) scratch[warp] = v;
+    __syncthreads();
+    double t = 0.0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += scratch[w];  // same order in every thread
+    return t;
+}
+
+__device__ __forceinline__ double matern64(double r, int kernel) {
+    if (kernel == SCOOT_MATERN32) {
+        const double a = sqrt(3.0) * r;
+        return (1.0 + a) * exp(-a);
+    }
+    const double a = sqrt(5.0) * r;
+    return (1.0 + a + a * a / 3.0) * exp(-a);
+}
+
+// k(a, b) of one objective in fp64: ordinal coordinates scaled by 1/l,
+// categorical mismatches weigh 1/l^2 (the covariance of Section 4.3).
+__device__ __forceinline__ double cov64(const double* ua, const double* ub, const double* sp, const double* ell,
+                                        int d, double sf2, int kernel) {
+    double r2 = 0.0;
+    for (int c = 0; c < d; ++c) {
+        if ((int)sp[c * 4] == SCOOT_CATEGORICAL) {
+            if (ua[c] != ub[c]) r2 += 1.0 / (ell[c] * ell[c]);
+        } else {
+            const double t = (ua[c] - ub[c]) / ell[c];
+            r2 += t * t;
         }
     }
-    best = block_max_u64(best);
-    if (threadIdx.x == 0) a.partial[blockIdx.x] = best;
+    return sf2 * matern64(sqrt(r2), kernel);
 }
 
-__global__ void __launch_bounds__(kFThreads) fant_argmax2(const __grid_constant__ FantArgs a, int n_partial) {
-    uint64_t best = 0ull;
-    for (int k = threadIdx.x; k < n_partial; k += blockDim.x) best = a.partial[k] > best ? a.partial[k] : best;
-    best = block_max_u64(best);
-    if (threadIdx.x == 0) *a.best = best;
+// Feature coordinate (fp64) of a stored word of parameter c: log scale for
+// integer log-uniform, linear for integer uniform and continuous, the index
+// for categoricals.  Returns false for a word that has no feature.
+__device__ __forceinline__ bool feature64(const double* sp, int c, uint32_t w, double* u) {
+    const int kind = (int)sp[c * 4];
+    const double lo = sp[c * 4 + 1], hi = sp[c * 4 + 2];
+    const double v = kind == SCOOT_CONTINUOUS ? (double)__uint_as_float(w) : (double)(int32_t)w;
+    if (kind == SCOOT_INT_LOG) {
+        if (!(v > 0.0)) return false;
+        *u = (log(v) - log(lo)) / (log(hi) - log(lo));
+    } else if (kind == SCOOT_INT_UNIFORM || kind == SCOOT_CONTINUOUS) {
+        *u = hi > lo ? (v - lo) / (hi - lo) : 0.0;
+    } else {
+        *u = v;
+    }
+    return isfinite(*u);
 }
 
-// Variance downdate of every live candidate for pick j (see the file comment).
+// ---------------------------------------------------------------- front and boxes
+
+// Shared-memory need of front_update_and_boxes (bytes).
+__host__ __device__ inline size_t boxes_smem(int front_cap, int M, int box_cap) {
+    return (size_t)front_cap * M * 8 + (size_t)(M - 1) * (front_cap + 1) * 8 + (size_t)(front_cap + 1) * 4 +
+           (size_t)(box_cap + 1) * 4 + 64;
+}
+
+// One block: optionally adds point z (fp64 of the fp32 fantasised value) to
+// the front (if it lies above the reference point and no front point weakly
+// dominates it; front points it dominates leave), then decomposes the region
+// the front does not dominate into boxes exactly as scoot_boxes_build does:
+// columns over the grid of the first M - 1 axes (the reference coordinate and
+// the front's, sorted, unique), each open upwards on the last objective from
+// max(r_last, the highest last value among front points dominating the
+// cell's upper corner), cells merged along the last grid axis while that
+// floor repeats.  Boxes in the builder's order.  On a box count beyond
+// box_cap the loop stops with a capacity error.
 template <int M>
-__global__ void __launch_bounds__(kFThreads) fant_update(const __grid_constant__ FantArgs a) {
-    const float* fmap = reinterpret_cast<const float*>(a.state + a.off_fmap);
-    const float* gils = reinterpret_cast<const float*>(a.state + a.off_ils);
-    const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
-    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < a.n_live;
+__device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, bool add, const double* z,
+                                       char* smem) {
+    constexpr int G = M - 1;
+    const int fcap = a.front_cap;
+    double* F = reinterpret_cast<double*>(smem);                  // [fcap][M]
+    double* axis = F + (size_t)fcap * M;                           // [G][fcap + 1]
+    int32_t* first = reinterpret_cast<int32_t*>(axis + (size_t)G * (fcap + 1));  // [fcap + 1]
+    int32_t* rowcnt = first + fcap + 1;                                            // [rows + 1]
+    __shared__ int32_t s_nf, s_A[4], s_total, s_ok;
+    const int tid = threadIdx.x;
+    if (tid == 0) s_nf = a.ctrl->n_front;
+    __syncthreads();
+    for (int e = tid; e < s_nf * M; e += blockDim.x) F[e] = a.front[e];
+    __syncthreads();
+    if (add && tid == 0) {
+        bool above = true, covered = false;
+        for (int m = 0; m < M; ++m) above &= z[m] > h.ref[m];
+        for (int k = 0; k < s_nf && !covered; ++k) {
+            bool ge = true;
+            for (int m = 0; m < M; ++m) ge &= F[k * M + m] >= z[m];
+            covered = ge;
+        }
+        if (above && !covered) {
+            int w = 0;
+            for (int k = 0; k < s_nf; ++k) {
+                bool ge = true, gt = false;
+                for (int m = 0; m < M; ++m) {
+                    ge &= z[m] >= F[k * M + m];
+                    gt |= z[m] > F[k * M + m];
+                }
+                if (ge && gt) continue;  // dominated by the fantasy
+                for (int m = 0; m < M; ++m) F[w * M + m] = F[k * M + m];
+                ++w;
+            }
+            if (w < fcap) {
+                for (int m = 0; m < M; ++m) F[w * M + m] = z[m];
+                ++w;
+            } else {
+                atomicOr(a.err, SCOOT_DEVERR_CAPACITY);
+            }
+            s_nf = w;
+        }
+    }
+    __syncthreads();
+    const int nf = s_nf;
+    for (int e = tid; e < nf * M; e += blockDim.x) a.front[e] = F[e];
+    // Axes: {r_j} and the front's coordinates, sorted and unique.  Value t
+    // (t = 0 the reference, t = k + 1 front point k) is kept if no earlier t
+    // holds the same value; its place is the number of kept values below it.
+    for (int j = 0; j < G; ++j) {
+        for (int t = tid; t <= nf; t += blockDim.x) {
+            const double v = t == 0 ? h.ref[j] : F[(t - 1) * M + j];
+            int f = 1;
+            for (int u = 0; u < t && f; ++u) f = (u == 0 ? h.ref[j] : F[(u - 1) * M + j]) != v;
+            first[t] = f;
+        }
+        __syncthreads();
+        for (int t = tid; t <= nf; t += blockDim.x) {
+            if (!first[t]) continue;
+            const double v = t == 0 ? h.ref[j] : F[(t - 1) * M + j];
+            int below = 0;
+            for (int u = 0; u <= nf; ++u) below += first[u] && (u == 0 ? h.ref[j] : F[(u - 1) * M + j]) < v;
+            axis[j * (fcap + 1) + below] = v;
+        }
+        if (tid == 0) {
+            int cnt = 0;
+            for (int t = 0; t <= nf; ++t) cnt += first[t];
+            s_A[j] = cnt;
+        }
+        __syncthreads();
+    }
+    int cells = 1;
+    for (int j = 0; j < G; ++j) cells *= s_A[j];
+    const int A_last = s_A[G - 1];
+    const int rows = cells / A_last;
+    if (cells > a.box_cap) {
+        if (tid == 0) {
+            atomicOr(a.err, SCOOT_DEVERR_CAPACITY);
+            a.ctrl->done = 1u;
+            a.ctrl->n_boxes = 0;
+        }
+        return;
+    }
+    // Floor of every cell (row-major over the grid, the last axis fastest).
+    const double inf = __longlong_as_double(0x7ff0000000000000ll);
+    for (int c = tid; c < cells; c += blockDim.x) {
+        double up[G];
+        int rest = c;
+        for (int j = G - 1; j >= 0; --j) {
+            const int kj = rest % s_A[j];
+            rest /= s_A[j];
+            up[j] = kj + 1 < s_A[j] ? axis[j * (fcap + 1) + kj + 1] : inf;
+        }
+        double hh = -inf;
+        for (int k = 0; k < nf; ++k) {
+            bool dom = true;
+            for (int j = 0; j < G; ++j) dom &= F[k * M + j] >= up[j];
+            if (dom) hh = fmax(hh, F[k * M + M - 1]);
+        }
+        a.cell[c] = fmax(h.ref[M - 1], hh);
+    }
+    __syncthreads();
+    // Boxes per row (cells merged while the floor repeats), then their offsets.
+    for (int r = tid; r < rows; r += blockDim.x) {
+        int cnt = 1;
+        for (int kk = 1; kk < A_last; ++kk) cnt += a.cell[r * A_last + kk] != a.cell[r * A_last + kk - 1];
+        rowcnt[r + 1] = cnt;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        rowcnt[0] = 0;
+        for (int r = 0; r < rows; ++r) rowcnt[r + 1] += rowcnt[r];
+        s_total = rowcnt[rows];
+        s_ok = s_total <= a.box_cap;
+    }
+    __syncthreads();
+    for (int r = tid; r < rows && s_ok; r += blockDim.x) {
+        double lo_pre[G > 1 ? G - 1 : 1], up_pre[G > 1 ? G - 1 : 1];
+        int rest = r;
+        for (int j = G - 2; j >= 0; --j) {
+            const int kj = rest % s_A[j];
+            rest /= s_A[j];
+            lo_pre[j] = axis[j * (fcap + 1) + kj];
+            up_pre[j] = kj + 1 < s_A[j] ? axis[j * (fcap + 1) + kj + 1] : inf;
+        }
+        int b = rowcnt[r] - 1;
+        const double* al = axis + (G - 1) * (fcap + 1);
+        for (int kk = 0; kk < A_last; ++kk) {
+            const double fl = a.cell[r * A_last + kk];
+            const double upl = kk + 1 < A_last ? al[kk + 1] : inf;
+            if (kk == 0 || fl != a.cell[r * A_last + kk - 1]) {
+                ++b;
+                for (int j = 0; j < G - 1; ++j) {
+                    a.box_lo[b * M + j] = (float)lo_pre[j];
+                    a.box_hi[b * M + j] = (float)up_pre[j];
+                }
+                a.box_lo[b * M + G - 1] = (float)al[kk];
+                a.box_lo[b * M + M - 1] = (float)fl;
+                a.box_hi[b * M + M - 1] = __int_as_float(0x7f800000);
+            }
+            a.box_hi[b * M + G - 1] = (float)upl;
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        a.ctrl->n_front = nf;
+        if (s_ok) {
+            a.ctrl->n_boxes = s_total;
+        } else {
+            atomicOr(a.err, SCOOT_DEVERR_CAPACITY);
+            a.ctrl->done = 1u;
+            a.ctrl->n_boxes = 0;
+        }
+    }
+}
+
+// ---------------------------------------------------------------- kernels
+
+// One block: checks the fantasy state against the call, resets the control
+// words and outputs, and decomposes the observations' front into boxes.
+template <int M>
+__global__ void __launch_bounds__(kPickThreads) fant_init(const __grid_constant__ FantArgs a) {
+    extern __shared__ __align__(16) char smem[];
+    const FantHeader& h = *reinterpret_cast<const FantHeader*>(a.fant);
+    const float* gscal = reinterpret_cast<const float*>(a.gp + a.off_scal);
+    __shared__ int ok;
+    if (threadIdx.x == 0) {
+        ok = h.magic == kFantMagic && h.n == a.n_obs && h.d == a.d && h.M == M && h.q >= a.q &&
+             h.kernel == a.kernel && h.front0 >= 0 && h.front0 <= a.n_obs;
+        for (int m = 0; m < M; ++m) ok &= gscal[m * 4 + 3] == 0.0f;  // an unwarped GP state
+        a.ctrl->done = ok ? 0u : 1u;
+        a.ctrl->arrived = 0u;
+        a.ctrl->n_boxes = 0;
+        a.ctrl->n_front = ok ? h.front0 : 0;
+        *a.out_count = 0;
+        if (!ok) atomicOr(a.err, SCOOT_DEVERR_VALUE);
+    }
+    for (int j = threadIdx.x; j < a.q; j += blockDim.x) {
+        a.out_idx[j] = -1;
+        a.out_val[j] = -INFINITY;
+    }
+    __syncthreads();
+    if (!ok) return;
+    const double* f0 = reinterpret_cast<const double*>(a.fant + h.off_front);
+    for (int e = threadIdx.x; e < h.front0 * M; e += blockDim.x) a.front[e] = f0[e];
+    __syncthreads();
+    front_update_and_boxes<M>(a, h, false, nullptr, smem);
+}
+
+// Pick j's pass over the live candidates: for j > 0 the downdate of pick
+// j - 1, then EHVI over the current boxes with the picks excluded, and each
+// block's best (key, list position).
+template <int M>
+__global__ void __launch_bounds__(kPassThreads) fant_pass(const __grid_constant__ FantArgs a, int j) {
+    if (*(volatile const uint32_t*)&a.ctrl->done) {
+        if (threadIdx.x == 0) a.part_key[blockIdx.x] = 0ull;
+        return;
+    }
+    extern __shared__ __align__(16) float sm[];
+    const int nb = a.ctrl->n_boxes;
+    float4* blo = reinterpret_cast<float4*>(sm);
+    float4* bhi = blo + nb;
+    float4* epsv = bhi + nb;
+    int64_t* pk = reinterpret_cast<int64_t*>(epsv + a.n_mc);  // [q] list positions of the picks
+    float* vps = reinterpret_cast<float*>(pk + a.q);          // [M][n_pad]
+    float* cxs = vps + M * a.n_pad;                           // [M][q]
+    float* ins = cxs + M * a.q;                               // [M]
+    float* ups = ins + M;                                     // [d] features of the latest pick (feature order)
+    const float4* fm = reinterpret_cast<const float4*>(a.gp + a.off_fmap);
+    const float* gils = reinterpret_cast<const float*>(a.gp + a.off_ils);
+    const float* gscal = reinterpret_cast<const float*>(a.gp + a.off_scal);
+    stage_boxes(a.box_lo, a.box_hi, nb, a.eps, a.n_mc, M, blo, bhi, epsv);
+    const int l = j - 1;  // the downdate of this pass
+    int64_t p = 0;
+    if (l >= 0) {
+        p = a.ctrl->pick_idx;
+        for (int e = threadIdx.x; e < M * a.n_pad; e += blockDim.x) vps[e] = a.vp[e];
+        for (int e = threadIdx.x; e < M * a.q; e += blockDim.x) cxs[e] = a.cxp[e];
+        if (threadIdx.x < M) ins[threadIdx.x] = a.inv_s[threadIdx.x];
+        for (int c = threadIdx.x; c < a.d; c += blockDim.x) {
+            const float4 f = fm[c];
+            ups[c] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + p), (int)f.x, f.y, f.z);
+        }
+    }
+    for (int e = threadIdx.x; e < j; e += blockDim.x) pk[e] = a.picked_pos[e];
+    __syncthreads();
+    const bool fast = boxes_fast(blo, bhi, nb, M);
+    if (fast) {
+        stage_boxes_sat(a.box_lo, a.box_hi, nb, M, blo);
+        __syncthreads();
+    }
+    const int64_t n_live = a.n_list ? (int64_t)*a.n_list : a.n;
+    uint64_t best = 0ull;
+    int32_t best_pos = -1;
+    const float inv_mc = 1.0f / (float)a.n_mc;
+    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < n_live;
          pos += (int64_t)gridDim.x * blockDim.x) {
         const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
-        float r2[M];
+        float vr[M];
+        if (l >= 0) {
+            float r2[M];
 #pragma unroll
-        for (int m = 0; m < M; ++m) r2[m] = 0.0f;
-        for (int c = 0; c < a.d; ++c) {
-            const int kind = (int)fmap[c * 4];
-            const int64_t col = (int64_t)fmap[c * 4 + 3];  // features are in feature order
-            const float ux = feature_of(__ldg(a.cand + col * a.ld + i), kind, fmap[c * 4 + 1], fmap[c * 4 + 2]);
-            const float up = feature_of(__ldg(a.cand + col * a.ld + a.p), kind, fmap[c * 4 + 1], fmap[c * 4 + 2]);
+            for (int m = 0; m < M; ++m) r2[m] = 0.0f;
+            for (int c = 0; c < a.d; ++c) {
+                const float4 f = fm[c];
+                const int kind = (int)f.x;
+                const float ux = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + i), kind, f.y, f.z);
+                const float up = ups[c];
 #pragma unroll
-            for (int m = 0; m < M; ++m) {
-                const float s = gils[m * a.d + c];
-                if (kind == SCOOT_CATEGORICAL) {
-                    r2[m] += ux != up ? s : 0.0f;
-                } else {
-                    const float t = (ux - up) * s;
-                    r2[m] = fmaf(t, t, r2[m]);
+                for (int m = 0; m < M; ++m) {
+                    const float s = gils[m * a.d + c];
+                    if (kind == SCOOT_CATEGORICAL) {
+                        r2[m] += ux != up ? s : 0.0f;
+                    } else {
+                        const float t = (ux - up) * s;
+                        r2[m] = fmaf(t, t, r2[m]);
+                    }
                 }
             }
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                const float k = gscal[m * 4] * matern(sqrtf(r2[m]), a.kernel);
+                const float* vrow = a.V + (int64_t)m * a.n_pad * a.ldc + pos;
+                const float* vpm = vps + m * a.n_pad;
+                float d0 = 0.0f, d1 = 0.0f;
+                int row = 0;
+#pragma unroll 8
+                for (; row + 1 < a.n_obs; row += 2) {
+                    d0 = fmaf(vrow[(int64_t)row * a.ldc], vpm[row], d0);
+                    d1 = fmaf(vrow[(int64_t)(row + 1) * a.ldc], vpm[row + 1], d1);
+                }
+                if (row < a.n_obs) d0 = fmaf(vrow[(int64_t)row * a.ldc], vpm[row], d0);
+                float cc = 0.0f;
+                for (int t = 0; t < l; ++t) cc = fmaf(a.C[((int64_t)t * M + m) * a.ldc + pos], cxs[m * a.q + t], cc);
+                const float c = (k - (d0 + d1) - cc) * ins[m];
+                if (l < a.q - 2) a.C[((int64_t)l * M + m) * a.ldc + pos] = c;  // read by later downdates
+                float* vv = a.var + (int64_t)m * a.ldc + pos;
+                vr[m] = fmaxf(*vv - c * c, 0.0f);
+                *vv = vr[m];
+            }
+        } else {
+#pragma unroll
+            for (int m = 0; m < M; ++m) vr[m] = a.var[(int64_t)m * a.ldc + pos];
         }
+        bool taken = false;
+        for (int t = 0; t < j; ++t) taken |= pk[t] == pos;
+        if (taken) continue;
+        float mu[M], sd[M];
 #pragma unroll
         for (int m = 0; m < M; ++m) {
-            const float k = gscal[m * 4] * matern(sqrtf(r2[m]), a.kernel);
-            const float* vrow = a.V + (int64_t)m * a.n_pad * a.ldc + pos;
-            const float* vp = a.vp + m * a.n_pad;
-            float dot = 0.0f;
-            for (int row = 0; row < a.n_obs; ++row) dot = fmaf(vrow[(int64_t)row * a.ldc], vp[row], dot);
-            float cc = 0.0f;
-            for (int l = 0; l < a.j; ++l) cc = fmaf(a.C[((int64_t)l * M + m) * a.ldc + pos], a.cxp[m * a.q + l], cc);
-            const float c = (k - dot - cc) * a.inv_s[m];
-            a.C[((int64_t)a.j * M + m) * a.ldc + pos] = c;
-            float* vv = a.var + (int64_t)m * a.ldc + pos;
-            *vv = fmaxf(*vv - c * c, 0.0f);
+            mu[m] = a.mean[(int64_t)m * a.ldc + pos];
+            sd[m] = sqrtf(fmaxf(vr[m], 0.0f));
         }
+        const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, nb, epsv, a.n_mc, 0, 1) * inv_mc
+                             : ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
+        if (!(v != v) && v != -INFINITY) keymax(best, best_pos, make_key(v, (uint32_t)i), (int32_t)pos);
+    }
+    block_keymax(best, best_pos);
+    if (threadIdx.x == 0) {
+        a.part_key[blockIdx.x] = best;
+        a.part_pos[blockIdx.x] = best_pos;
     }
 }
 
-__global__ void __launch_bounds__(kFThreads)
-scatter_var(const int32_t* list, int64_t n_live, int64_t ldc, int M, const float* var, float* out, int64_t ldo) {
+// Pick j: the argmax of the pass's partials (every block); block 0 records
+// the pick; block m then computes objective m's rank-1 terms of the pick in
+// fp64; the last block to finish adds the fantasised point to the front and
+// rebuilds the boxes for the next pass.
+template <int M>
+__global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant__ FantArgs a, int j, int n_part) {
+    extern __shared__ __align__(16) char smem[];
+    if (*(volatile const uint32_t*)&a.ctrl->done) return;
+    const FantHeader& h = *reinterpret_cast<const FantHeader*>(a.fant);
+    const int tid = threadIdx.x, m = blockIdx.x;
+    uint64_t best = 0ull;
+    int32_t bpos = -1;
+    for (int k = tid; k < n_part; k += blockDim.x) keymax(best, bpos, a.part_key[k], a.part_pos[k]);
+    block_keymax(best, bpos);
+    __shared__ uint64_t s_best;
+    __shared__ int32_t s_pos;
+    if (tid == 0) {
+        s_best = best;
+        s_pos = bpos;
+    }
+    __syncthreads();
+    best = s_best;
+    bpos = s_pos;
+    if (best == 0ull) {  // no eligible candidate left: the picks end here
+        if (m == 0 && tid == 0) a.ctrl->done = 1u;
+        return;
+    }
+    const int64_t p = key_index(best);
+    if (m == 0 && tid == 0) {
+        a.out_idx[j] = p;
+        a.out_val[j] = key_value(best);
+        *a.out_count = j + 1;
+        a.picked_pos[j] = bpos;
+        a.ctrl->pick_idx = p;
+        a.ctrl->pick_pos = bpos;
+    }
+    if (j + 1 >= a.q) return;  // no later pick needs this one's fantasy
+    const int n = a.n_obs, d = a.d, q = a.q;
+    const double* sp = reinterpret_cast<const double*>(a.fant + h.off_space);
+    const double* uo = reinterpret_cast<const double*>(a.fant + h.off_u);
+    const double* ell = reinterpret_cast<const double*>(a.fant + h.off_ell) + (size_t)m * d;
+    const double* alpha = reinterpret_cast<const double*>(a.fant + h.off_alpha) + (size_t)m * n;
+    const double* Li = reinterpret_cast<const double*>(a.fant + h.off_linv) + (size_t)m * n * n;
+    const double sf2 = h.sf2[m], tau2 = h.tau2[m];
+    double* u = reinterpret_cast<double*>(smem);     // [16] features of the pick
+    double* ks = u + 16;                              // [n] k(X, x_p)
+    double* vv = ks + n;                              // [n] v_p
+    double* D = vv + n;                               // [q] v_p . v_{p_t}
+    double* red = D + q;                              // [32] reduction scratch
+    __shared__ int s_bad;
+    if (tid == 0) s_bad = 0;
+    __syncthreads();
+    if (tid < d) {
+        double x = 0.0;
+        if (!feature64(sp, tid, __ldg(a.cand + (int64_t)tid * a.ld + p), &x)) s_bad = 1;
+        u[tid] = x;
+        if (m == 0) a.upick[(size_t)j * d + tid] = x;
+    }
+    __syncthreads();
+    if (s_bad) {
+        if (tid == 0) {
+            atomicOr(a.err, SCOOT_DEVERR_VALUE);
+            a.ctrl->done = 1u;
+        }
+        return;
+    }
+    double mu_part = 0.0;
+    for (int i = tid; i < n; i += blockDim.x) {
+        ks[i] = cov64(u, uo + (size_t)i * d, sp, ell, d, sf2, a.kernel);
+        mu_part += ks[i] * alpha[i];
+    }
+    __syncthreads();
+    // v_p = L^{-1} k*: row i reads column-major L^{-1} (coalesced across rows).
+    double vv_part = 0.0;
+    for (int i = tid; i < n; i += blockDim.x) {
+        double s0 = 0.0, s1 = 0.0;
+        int c = 0;
+        for (; c + 1 <= i; c += 2) {
+            s0 = fma(Li[(size_t)c * n + i], ks[c], s0);
+            s1 = fma(Li[(size_t)(c + 1) * n + i], ks[c + 1], s1);
+        }
+        if (c <= i) s0 = fma(Li[(size_t)c * n + i], ks[c], s0);
+        const double v = s0 + s1;
+        vv[i] = v;
+        a.vpick[((size_t)j * M + m) * n + i] = v;
+        vv_part += v * v;
+    }
+    const double mu = block_sum(mu_part, red);
+    const double vnorm = block_sum(vv_part, red);   // (its barriers also publish vv)
+    // Dots with the earlier picks' rows: warp w takes picks w, w + 8, ...
+    {
+        const int lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+        for (int t = warp; t < j; t += nw) {
+            const double* vt = a.vpick + ((size_t)t * M + m) * n;
+            double s = 0.0;
+            for (int i = lane; i < n; i += 32) s = fma(vv[i], vt[i], s);
+            for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+            if (lane == 0) D[t] = s;
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        double var = sf2 - vnorm;
+        double* cj = a.cpick + ((size_t)j * M + m) * q;
+        for (int t = 0; t < j; ++t) {
+            const double* ct = a.cpick + ((size_t)t * M + m) * q;
+            double num = cov64(u, a.upick + (size_t)t * d, sp, ell, d, sf2, a.kernel) - D[t];
+            for (int r = 0; r < t; ++r) num -= cj[r] * ct[r];
+            const double st = a.spick[(size_t)t * M + m];
+            cj[t] = st > 0.0 ? num / st : 0.0;
+            var -= cj[t] * cj[t];
+        }
+        const double s = sqrt(fmax(var, 0.0) + tau2);
+        a.spick[(size_t)j * M + m] = s;
+        a.mupick[(size_t)j * M + m] = mu;
+        a.inv_s[m] = s > 0.0 ? (float)(1.0 / s) : 0.0f;
+        for (int t = 0; t < q; ++t) a.cxp[m * q + t] = t < j ? (float)cj[t] : 0.0f;
+    }
+    for (int i = tid; i < a.n_pad; i += blockDim.x) a.vp[m * a.n_pad + i] = i < n ? (float)vv[i] : 0.0f;
+    // The last block to get here adds the fantasised point and rebuilds the boxes.
+    __threadfence();
+    __syncthreads();
+    __shared__ int s_last;
+    if (tid == 0) s_last = atomicAdd(&a.ctrl->arrived, 1u) == (unsigned)(M - 1);
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    if (tid == 0) a.ctrl->arrived = 0u;
+    double z[M];
+#pragma unroll
+    for (int k = 0; k < M; ++k) z[k] = (double)(float)(*(volatile const double*)&a.mupick[(size_t)j * M + k]);
+    front_update_and_boxes<M>(a, h, true, z, smem);
+}
+
+__global__ void __launch_bounds__(kPassThreads)
+scatter_var(const int32_t* list, const unsigned int* n_list, int64_t n, int64_t ldc, int M, const float* var,
+            float* out, int64_t ldo) {
+    const int64_t n_live = n_list ? (int64_t)*n_list : n;
     for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < n_live;
          pos += (int64_t)gridDim.x * blockDim.x) {
         const int64_t i = list ? (int64_t)list[pos] : pos;
@@ -183,29 +637,40 @@ scatter_var(const int32_t* list, int64_t n_live, int64_t ldc, int M, const float
     }
 }
 
+// ---------------------------------------------------------------- work buffer
+
 struct WorkLayout {
-    int64_t mean, var, V, C, acq, picked, vp, cxp, inv_s, box_lo, box_hi, partial, best, bytes;
+    int64_t mean, var, V, C, ctrl, picked, vp, cxp, inv_s, upick, vpick, cpick, spick, mupick, front, box_lo,
+        box_hi, cell, part_key, part_pos, bytes;
 };
 
 int64_t up256(int64_t x) { return (x + 255) / 256 * 256; }
 
-WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q) {
-    const int64_t M = L->n_obj, n_pad = (int64_t)L->n_rb * 64;
+WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q, int box_cap) {
+    const int64_t M = L->n_obj, n_pad = (int64_t)L->n_rb * 64, no = L->n, d = L->d;
+    const int64_t fcap = no + q;
     WorkLayout w;
     int64_t o = 0;
-    w.mean = o;    o = up256(o + M * n * 4);
-    w.var = o;     o = up256(o + M * n * 4);
-    w.V = o;       o = up256(o + M * n_pad * n * 4);
-    w.C = o;       o = up256(o + (int64_t)q * M * n * 4);
-    w.acq = o;     o = up256(o + n * 4);
-    w.picked = o;  o = up256(o + (int64_t)q * 8);
-    w.vp = o;      o = up256(o + M * n_pad * 4);
-    w.cxp = o;     o = up256(o + M * q * 4);
-    w.inv_s = o;   o = up256(o + M * 4);
-    w.box_lo = o;  o = up256(o + (int64_t)kBoxCap * M * 4);
-    w.box_hi = o;  o = up256(o + (int64_t)kBoxCap * M * 4);
-    w.partial = o; o = up256(o + kArgBlocks * 8);
-    w.best = o;    o = up256(o + 8);
+    w.mean = o;     o = up256(o + M * n * 4);
+    w.var = o;      o = up256(o + M * n * 4);
+    w.V = o;        o = up256(o + M * n_pad * n * 4);
+    w.C = o;        o = up256(o + (int64_t)std::max(q - 2, 1) * M * n * 4);
+    w.ctrl = o;     o = up256(o + (int64_t)sizeof(Ctrl));
+    w.picked = o;   o = up256(o + (int64_t)q * 8);
+    w.vp = o;       o = up256(o + M * n_pad * 4);
+    w.cxp = o;      o = up256(o + M * q * 4);
+    w.inv_s = o;    o = up256(o + M * 4);
+    w.upick = o;    o = up256(o + (int64_t)q * d * 8);
+    w.vpick = o;    o = up256(o + (int64_t)q * M * no * 8);
+    w.cpick = o;    o = up256(o + (int64_t)q * M * q * 8);
+    w.spick = o;    o = up256(o + (int64_t)q * M * 8);
+    w.mupick = o;   o = up256(o + (int64_t)q * M * 8);
+    w.front = o;    o = up256(o + fcap * M * 8);
+    w.box_lo = o;   o = up256(o + (int64_t)box_cap * M * 4);
+    w.box_hi = o;   o = up256(o + (int64_t)box_cap * M * 4);
+    w.cell = o;     o = up256(o + (int64_t)box_cap * 8);
+    w.part_key = o; o = up256(o + kPartMax * 8);
+    w.part_pos = o; o = up256(o + kPartMax * 4);
     w.bytes = o;
     return w;
 }
@@ -216,115 +681,31 @@ int sm_count(int device) {
     return v > 0 ? v : 1;
 }
 
-struct Pick {
-    std::vector<double> u;                  // features
-    std::vector<std::vector<double>> v;     // [M][n] whitened covariance row
-    std::vector<std::vector<double>> c;     // [M][l < j] c_l(x_p)
-    std::vector<double> s;                  // [M] s_j
-};
-
 template <int M>
-scoot_status run_picks(scoot_ctx* ctx, const scoot_gp_layout* L, FantArgs a, const std::vector<HostGP>& gps,
-                       const scoot_param* h_space, const uint32_t* cand, int64_t ld, const float* h_y,
-                       const float* h_ref, int32_t q, char* work, const WorkLayout& w, int64_t* h_idx,
-                       float* h_val, int32_t* h_count, cudaStream_t st) {
-    const int n = L->n, d = L->d, n_pad = L->n_rb * 64;
-    std::vector<float> Y((size_t)M * n);
-    std::memcpy(Y.data(), h_y, Y.size() * sizeof(float));
-    int n_pts = n;
-    std::vector<float> lo((size_t)kBoxCap * M), hi((size_t)kBoxCap * M);
-    std::vector<float> vp_h((size_t)M * n_pad), cxp_h((size_t)M * q), inv_s_h(M);
-    std::vector<Pick> picks;
-    std::vector<uint32_t> words(d);
-    const int sms = sm_count(ctx->device);
-    int64_t blocks = (a.n_live + kFThreads - 1) / kFThreads;
-    if (blocks > (int64_t)sms * 16) blocks = (int64_t)sms * 16;
+scoot_status run_picks(scoot_ctx* ctx, FantArgs a, int64_t n, cudaStream_t st) {
+    const size_t pass_smem = (size_t)(2 * a.box_cap + a.n_mc) * 16 + (size_t)a.q * 8 + (size_t)M * a.n_pad * 4 +
+                             (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4;
+    const size_t pick_smem = std::max((size_t)(16 + 2 * a.n_obs + a.q + 32) * 8,
+                                      boxes_smem(a.front_cap, M, a.box_cap));
+    int max_smem = 0;
+    SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
+    if (pass_smem > (size_t)max_smem || pick_smem > (size_t)max_smem)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "%d boxes and %d samples exceed the shared memory of a block",
+                          a.box_cap, a.n_mc);
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_pass<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pass_smem));
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_pick<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pick_smem));
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_init<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pick_smem));
+    fant_init<M><<<1, kPickThreads, pick_smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    // Enough blocks for many loads in flight per SM; the live count is read on the device.
+    int64_t blocks = (n + kPassThreads - 1) / kPassThreads;
+    const int64_t cap = std::min<int64_t>((int64_t)sm_count(ctx->device) * 8, kPartMax);
+    if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    int arg_blocks = (int)std::min<int64_t>(blocks, kArgBlocks);
-    *h_count = 0;
-    for (int j = 0; j < q; ++j) {
-        // Boxes of the front with the fantasised points added.
-        int32_t nb = 0, fs = 0;
-        scoot_status s = scoot_boxes_build(Y.data(), n_pts, M, h_ref, kBoxCap, lo.data(), hi.data(), &nb, &fs);
-        if (s != SCOOT_OK) return scoot_fail(ctx, s, "box decomposition of the fantasised front failed (%d boxes)", nb);
-        if ((size_t)(2 * nb + a.n_mc) * 16 > 160 * 1024)
-            return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "%d boxes and %d samples exceed the shared-memory budget", nb, a.n_mc);
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(work + w.box_lo, lo.data(), (size_t)nb * M * 4, cudaMemcpyHostToDevice, st));
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(work + w.box_hi, hi.data(), (size_t)nb * M * 4, cudaMemcpyHostToDevice, st));
-        a.n_boxes = nb;
-        a.n_picked = j;
-        a.j = j;
-        const size_t smem = (size_t)(2 * nb + a.n_mc) * 16;
-        SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_ehvi<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        fant_ehvi<M><<<(unsigned)blocks, kFThreads, smem, st>>>(a);
+    for (int j = 0; j < a.q; ++j) {
+        fant_pass<M><<<(unsigned)blocks, kPassThreads, pass_smem, st>>>(a, j);
         SCOOT_LAUNCHED(ctx);
-        fant_argmax1<<<arg_blocks, kFThreads, 0, st>>>(a);
-        SCOOT_LAUNCHED(ctx);
-        fant_argmax2<<<1, kFThreads, 0, st>>>(a, arg_blocks);
-        SCOOT_LAUNCHED(ctx);
-        uint64_t key = 0;
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(&key, work + w.best, 8, cudaMemcpyDeviceToHost, st));
-        SCOOT_CUDA(ctx, cudaStreamSynchronize(st));
-        if (key == 0) break;
-        const int64_t p = (int64_t)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFu));
-        uint32_t vb = (uint32_t)(key >> 32);
-        vb = (vb & 0x80000000u) ? (vb & 0x7FFFFFFFu) : ~vb;
-        float val;
-        std::memcpy(&val, &vb, 4);
-        h_idx[j] = p;
-        h_val[j] = val;
-        *h_count = j + 1;
-        if (j + 1 == q) break;  // no later pick needs this one's fantasy
-        // The picked configuration, on the host.
-        SCOOT_CUDA(ctx, cudaMemcpy2DAsync(words.data(), 4, cand + p, (size_t)ld * 4, 4, d, cudaMemcpyDeviceToHost, st));
-        SCOOT_CUDA(ctx, cudaStreamSynchronize(st));
-        Pick pk;
-        pk.u.resize(d);
-        if (!scoot_host_features(h_space, d, words.data(), 1, 0, pk.u.data()))
-            return scoot_fail(ctx, SCOOT_EINVAL, "picked configuration %lld has an invalid value", (long long)p);
-        pk.v.assign(M, std::vector<double>(n));
-        pk.c.assign(M, std::vector<double>(j));
-        pk.s.assign(M, 0.0);
-        std::vector<double> kx(n), mus(M);
-        for (int m = 0; m < M; ++m) {
-            const HostGP& g = gps[m];
-            g.kstar(pk.u.data(), kx.data());
-            g.solve_lower(kx.data(), pk.v[m].data());
-            double mu = 0.0, vv = 0.0;
-            for (int t = 0; t < n; ++t) {
-                mu += kx[t] * g.alpha[t];
-                vv += pk.v[m][t] * pk.v[m][t];
-            }
-            mus[m] = mu;  // kriging believer: the fantasised value is the posterior mean
-            double var = g.sf2 - vv;
-            for (int l = 0; l < j; ++l) {
-                const Pick& pl = picks[l];
-                double num = g.cov(pk.u.data(), pl.u.data());
-                for (int t = 0; t < n; ++t) num -= pk.v[m][t] * pl.v[m][t];
-                for (int t = 0; t < l; ++t) num -= pk.c[m][t] * pl.c[m][t];
-                pk.c[m][l] = pl.s[m] > 0.0 ? num / pl.s[m] : 0.0;
-                var -= pk.c[m][l] * pk.c[m][l];
-            }
-            pk.s[m] = std::sqrt(std::max(var, 0.0) + g.tau2);
-            for (int t = 0; t < n_pad; ++t) vp_h[(size_t)m * n_pad + t] = t < n ? (float)pk.v[m][t] : 0.0f;
-            for (int l = 0; l < q; ++l) cxp_h[(size_t)m * q + l] = l < j ? (float)pk.c[m][l] : 0.0f;
-            inv_s_h[m] = pk.s[m] > 0.0 ? (float)(1.0 / pk.s[m]) : 0.0f;
-        }
-        // The fantasised observation joins the front.
-        std::vector<float> Yn((size_t)M * (n_pts + 1));
-        for (int m = 0; m < M; ++m) {
-            std::memcpy(&Yn[(size_t)m * (n_pts + 1)], &Y[(size_t)m * n_pts], (size_t)n_pts * sizeof(float));
-            Yn[(size_t)m * (n_pts + 1) + n_pts] = (float)mus[m];
-        }
-        Y.swap(Yn);
-        n_pts += 1;
-        picks.push_back(pk);
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(work + w.vp, vp_h.data(), vp_h.size() * 4, cudaMemcpyHostToDevice, st));
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(work + w.cxp, cxp_h.data(), cxp_h.size() * 4, cudaMemcpyHostToDevice, st));
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(work + w.inv_s, inv_s_h.data(), inv_s_h.size() * 4, cudaMemcpyHostToDevice, st));
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(work + w.picked + 8 * (size_t)j, &h_idx[j], 8, cudaMemcpyHostToDevice, st));
-        a.p = p;
-        fant_update<M><<<(unsigned)blocks, kFThreads, 0, st>>>(a);
+        fant_pick<M><<<M, kPickThreads, pick_smem, st>>>(a, j, (int)blocks);
         SCOOT_LAUNCHED(ctx);
     }
     return SCOOT_OK;
@@ -334,118 +715,108 @@ scoot_status run_picks(scoot_ctx* ctx, const scoot_gp_layout* L, FantArgs a, con
 
 extern "C" {
 
-scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* L, int64_t n, int32_t q, int64_t* bytes) {
-    if (!L || !bytes || n < 0 || q < 1 || q > SCOOT_MAX_Q) return SCOOT_EINVAL;
-    *bytes = work_layout(L, n, q).bytes;
+scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* L, int64_t n, int32_t q, int32_t box_cap,
+                                      int64_t* bytes) {
+    if (!L || !bytes || n < 0 || box_cap < 1 || box_cap > kFantBoxMax) return SCOOT_EINVAL;
+    if (q < 1 || q > SCOOT_MAX_Q) return SCOOT_EUNSUPPORTED;
+    *bytes = work_layout(L, n, q, box_cap).bytes;
     return SCOOT_OK;
 }
 
 scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
-                                   const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs,
-                                   const float* h_y, const float* h_lengthscale, const float* h_signal_var,
-                                   const float* h_noise_var, const uint32_t* cand, int64_t n, int64_t ld,
-                                   const uint8_t* mask, const float* h_ref, const float* eps, int32_t n_mc,
-                                   int32_t q, void* work, int64_t work_bytes, int64_t* h_idx, float* h_val,
-                                   int32_t* h_count, float* var_out, void* stream) {
+                                   const void* fant_state, int32_t box_cap, const uint32_t* cand, int64_t n,
+                                   int64_t ld, const uint8_t* mask, const float* eps, int32_t n_mc, int32_t q,
+                                   void* work, int64_t work_bytes, int64_t* idx, float* val, int32_t* count,
+                                   float* var_out, void* stream) {
     scoot_status s = scoot_enter(ctx);
     if (s != SCOOT_OK) return s;
-    if (!L || !state || !h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var ||
-        !h_ref || !eps || !h_idx || !h_val || !h_count || !work)
+    if (!L || !state || !fant_state || !eps || !idx || !val || !count || !work)
         return scoot_fail(ctx, SCOOT_EINVAL, "a required pointer is NULL");
-    *h_count = 0;
     if (!scoot_gp_layout_valid(L))
         return scoot_fail(ctx, SCOOT_EINVAL, "GP layout is not one made by scoot_gp_layout_init");
     const int M = L->n_obj;
     if (M < 2 || M > 4) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "fantasy picks need 2 <= M <= 4, got %d", M);
     if (q < 1 || q > SCOOT_MAX_Q) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "q = %d outside 1..%d", q, SCOOT_MAX_Q);
     if (n_mc < 1) return scoot_fail(ctx, SCOOT_EINVAL, "n_mc < 1");
+    if (box_cap < 1 || box_cap > kFantBoxMax)
+        return scoot_fail(ctx, SCOOT_EINVAL, "box_cap = %d outside 1..%d", box_cap, kFantBoxMax);
     if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
     if (n > 0x7FFFFFFFll) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n >= 2^31");
-    if (ld_obs < L->n) return scoot_fail(ctx, SCOOT_EINVAL, "ld_obs < n_obs");
-    const WorkLayout w = work_layout(L, n, q);
+    const WorkLayout w = work_layout(L, n, q, box_cap);
     if (work_bytes < w.bytes)
         return scoot_fail(ctx, SCOOT_EINVAL, "work buffer of %lld bytes, %lld needed", (long long)work_bytes, (long long)w.bytes);
     if ((reinterpret_cast<uintptr_t>(work) & 255u) != 0) return scoot_fail(ctx, SCOOT_EINVAL, "work is not 256-byte aligned");
-    if (n == 0) return SCOOT_OK;
-
-    std::vector<HostGP> gps(M);
-    for (int m = 0; m < M; ++m) {
-        s = scoot_host_gp(h_space, L->d, h_x_obs, ld_obs, L->n, h_y + (size_t)m * L->n, h_lengthscale + (size_t)m * L->d,
-                          h_signal_var[m], h_noise_var[m], L->kernel, &gps[m], nullptr);
-        if (s != SCOOT_OK) return scoot_fail(ctx, s, "GP of objective %d could not be factored", m);
-    }
-    {
-        // The per-pick downdates rebuild the covariance without warping.  Read
-        // after the host factorisation, which overlaps the caller's queued work.
-        std::vector<float> scal((size_t)M * 4);
-        SCOOT_CUDA(ctx, cudaMemcpy(scal.data(), static_cast<const char*>(state) + L->off_scal,
-                                   scal.size() * sizeof(float), cudaMemcpyDeviceToHost));
-        for (int m = 0; m < M; ++m)
-            if (scal[(size_t)m * 4 + 3] != 0.0f)
-                return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "fantasy picks on a warped GP state");
-    }
+    if ((reinterpret_cast<uintptr_t>(fant_state) & 255u) != 0)
+        return scoot_fail(ctx, SCOOT_EINVAL, "fant_state is not 256-byte aligned");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     char* wk = static_cast<char*>(work);
     FantArgs a;
     std::memset(&a, 0, sizeof(a));
-    const unsigned int* n_list = nullptr;
-    int64_t n_live = n;
-    if (mask) {
+    a.n = n;
+    a.ldc = n > 0 ? n : 1;
+    if (mask && n > 0) {
         ScootList lst;
         if ((s = scoot_compact(ctx, mask, n, nullptr, 0u, st, &lst)) != SCOOT_OK) return s;
         a.list = lst.list;
-        n_list = lst.count;
-        unsigned int cnt = 0;
-        SCOOT_CUDA(ctx, cudaMemcpyAsync(&cnt, lst.count, 4, cudaMemcpyDeviceToHost, st));
-        SCOOT_CUDA(ctx, cudaStreamSynchronize(st));
-        n_live = cnt;
+        a.n_list = lst.count;
     }
-    a.n_live = n_live;
-    a.ldc = n;
     a.mean = reinterpret_cast<float*>(wk + w.mean);
     a.var = reinterpret_cast<float*>(wk + w.var);
     a.V = reinterpret_cast<float*>(wk + w.V);
     a.C = reinterpret_cast<float*>(wk + w.C);
-    a.vp = reinterpret_cast<float*>(wk + w.vp);
-    a.cxp = reinterpret_cast<float*>(wk + w.cxp);
-    a.inv_s = reinterpret_cast<float*>(wk + w.inv_s);
-    a.picked = reinterpret_cast<int64_t*>(wk + w.picked);
+    a.n_obs = L->n;
     a.n_pad = L->n_rb * 64;
+    a.d = L->d;
+    a.kernel = L->kernel;
     a.q = q;
-    a.acq = reinterpret_cast<float*>(wk + w.acq);
-    a.state = static_cast<const char*>(state);
+    a.n_mc = n_mc;
+    a.box_cap = box_cap;
+    a.front_cap = L->n + q;
+    a.gp = static_cast<const char*>(state);
     a.off_fmap = L->off_fmap;
     a.off_ils = L->off_ils;
     a.off_scal = L->off_scal;
-    a.n_obs = L->n;
-    a.d = L->d;
-    a.kernel = L->kernel;
+    a.fant = static_cast<const char*>(fant_state);
     a.cand = cand;
     a.ld = ld;
+    a.eps = eps;
     a.box_lo = reinterpret_cast<float*>(wk + w.box_lo);
     a.box_hi = reinterpret_cast<float*>(wk + w.box_hi);
-    a.eps = eps;
-    a.n_mc = n_mc;
-    a.partial = reinterpret_cast<uint64_t*>(wk + w.partial);
-    a.best = reinterpret_cast<uint64_t*>(wk + w.best);
-    if (n_live > 0) {
-        s = scoot_posterior_whitened(ctx, L, state, cand, n, ld, a.list, n_list, reinterpret_cast<float*>(wk + w.mean),
-                                     reinterpret_cast<float*>(wk + w.var), reinterpret_cast<float*>(wk + w.V), n, st);
-        if (s != SCOOT_OK) return s;
-        switch (M) {
-        case 2: s = run_picks<2>(ctx, L, a, gps, h_space, cand, ld, h_y, h_ref, q, wk, w, h_idx, h_val, h_count, st); break;
-        case 3: s = run_picks<3>(ctx, L, a, gps, h_space, cand, ld, h_y, h_ref, q, wk, w, h_idx, h_val, h_count, st); break;
-        default: s = run_picks<4>(ctx, L, a, gps, h_space, cand, ld, h_y, h_ref, q, wk, w, h_idx, h_val, h_count, st); break;
-        }
+    a.cell = reinterpret_cast<double*>(wk + w.cell);
+    a.front = reinterpret_cast<double*>(wk + w.front);
+    a.ctrl = reinterpret_cast<Ctrl*>(wk + w.ctrl);
+    a.picked_pos = reinterpret_cast<int64_t*>(wk + w.picked);
+    a.vp = reinterpret_cast<float*>(wk + w.vp);
+    a.cxp = reinterpret_cast<float*>(wk + w.cxp);
+    a.inv_s = reinterpret_cast<float*>(wk + w.inv_s);
+    a.upick = reinterpret_cast<double*>(wk + w.upick);
+    a.vpick = reinterpret_cast<double*>(wk + w.vpick);
+    a.cpick = reinterpret_cast<double*>(wk + w.cpick);
+    a.spick = reinterpret_cast<double*>(wk + w.spick);
+    a.mupick = reinterpret_cast<double*>(wk + w.mupick);
+    a.part_key = reinterpret_cast<uint64_t*>(wk + w.part_key);
+    a.part_pos = reinterpret_cast<int32_t*>(wk + w.part_pos);
+    a.out_idx = idx;
+    a.out_val = val;
+    a.out_count = count;
+    a.err = ctx->d_err;
+    if (n > 0) {
+        s = scoot_posterior_whitened(ctx, L, state, cand, n, ld, a.list, a.n_list, reinterpret_cast<float*>(wk + w.mean),
+                                     a.var, reinterpret_cast<float*>(wk + w.V), a.ldc, st);
         if (s != SCOOT_OK) return s;
     }
-    if (var_out && n_live > 0) {
-        int64_t blocks = (n_live + kFThreads - 1) / kFThreads;
-        if (blocks > (int64_t)sm_count(ctx->device) * 16) blocks = (int64_t)sm_count(ctx->device) * 16;
-        scatter_var<<<(unsigned)blocks, kFThreads, 0, st>>>(a.list, n_live, n, M, a.var, var_out, n);
+    switch (M) {
+    case 2: s = run_picks<2>(ctx, a, n, st); break;
+    case 3: s = run_picks<3>(ctx, a, n, st); break;
+    default: s = run_picks<4>(ctx, a, n, st); break;
+    }
+    if (s != SCOOT_OK) return s;
+    if (var_out && n > 0) {
+        int64_t blocks = (n + kPassThreads - 1) / kPassThreads;
+        if (blocks > (int64_t)sm_count(ctx->device) * 8) blocks = (int64_t)sm_count(ctx->device) * 8;
+        scatter_var<<<(unsigned)blocks, kPassThreads, 0, st>>>(a.list, a.n_list, n, a.ldc, M, a.var, var_out, n);
         SCOOT_LAUNCHED(ctx);
     }
-    SCOOT_CUDA(ctx, cudaStreamSynchronize(st));
     return SCOOT_OK;
 }
 

@@ -336,8 +336,20 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
                                      const float* h_signal_var, const float* h_noise_var,
                                      const float* h_warp, const scoot_gp_layout* L, void* h_blob,
                                      double* h_cond) {
-    if (!h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var || !L || !h_blob)
+    if (!h_blob) return SCOOT_EINVAL;
+    return scoot_gp_build(h_space, h_x_obs, ld_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, h_warp, L, h_blob,
+                          h_cond, nullptr);
+}
+
+}  // extern "C"
+
+scoot_status scoot_gp_build(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs, const float* h_y,
+                            const float* h_lengthscale, const float* h_signal_var, const float* h_noise_var,
+                            const float* h_warp, const scoot_gp_layout* L, void* h_blob, double* h_cond,
+                            void* h_fant) {
+    if (!h_space || !h_x_obs || !h_y || !h_lengthscale || !h_signal_var || !h_noise_var || !L || (!h_blob && !h_fant))
         return SCOOT_EINVAL;
+    if (h_fant && h_warp) return SCOOT_EUNSUPPORTED;
     scoot_gp_layout chk;
     if (scoot_gp_layout_init(h_space, L->n, L->d, L->n_obj, L->kernel, &chk) != SCOOT_OK ||
         std::memcmp(&chk, L, sizeof(chk)) != 0)
@@ -353,8 +365,14 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
             if (!is_finite(h_y[m * n + j])) return SCOOT_EINVAL;
     }
 
-    char* blob = static_cast<char*>(h_blob);
+    // Without a blob (the fantasy state alone) the fp32 parts are written to
+    // a scratch copy that is dropped.
+    std::vector<char> scratch;
+    if (!h_blob) scratch.resize((size_t)L->bytes);
+    char* blob = h_blob ? static_cast<char*>(h_blob) : scratch.data();
     std::memset(blob, 0, (size_t)L->bytes);
+    FantHeader* fh = static_cast<FantHeader*>(h_fant);
+    char* fbase = static_cast<char*>(h_fant);
     // Feature order: ordinal parameters first, then categorical ones, so the
     // kernels' distance loops need no per-dimension branch on the kind.
     std::vector<int> order;
@@ -421,6 +439,14 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
                                                            : (float)(g.u[(size_t)j * d + c] / l);
         }
         for (int i = 0; i < n; ++i) alpha_out[(size_t)m * n + i] = (float)g.alpha[i];
+        if (fh) {  // the fp64 inputs of the fantasy picks' rank-1 terms (original parameter order)
+            double* fu = reinterpret_cast<double*>(fbase + fh->off_u);
+            double* fell = reinterpret_cast<double*>(fbase + fh->off_ell) + (size_t)m * d;
+            double* falpha = reinterpret_cast<double*>(fbase + fh->off_alpha) + (size_t)m * n;
+            if (m == 0) std::memcpy(fu, g.u.data(), (size_t)n * d * sizeof(double));
+            std::memcpy(fell, g.ell.data(), (size_t)d * sizeof(double));
+            std::memcpy(falpha, g.alpha.data(), (size_t)n * sizeof(double));
+        }
         // L^{-1}: column by column, C col = e_col; column c is zero above row
         // c, so its forward substitution starts there (n^3 / 6 in all).
         // Li holds the columns contiguously: Li[c * n + i] = L^{-1}[i][c].
@@ -445,6 +471,10 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
             scoot_host_parallel(t, [&](int k) { columns(k, t); });
         } else {
             columns(0, 1);
+        }
+        if (fh) {
+            double* flinv = reinterpret_cast<double*>(fbase + fh->off_linv) + (size_t)m * n * n;
+            std::memcpy(flinv, Li.data(), (size_t)n * n * sizeof(double));
         }
         // Tiles: row block rb covers rows [64 rb, 64 rb + 64) and column
         // chunks cj = 0 .. 2 rb + 1 of 32 columns; tile[jj][ii] = Li[row][col].
@@ -493,30 +523,29 @@ scoot_status scoot_gp_prepare_warped(const scoot_param* h_space, const uint32_t*
     return SCOOT_OK;
 }
 
+extern "C" {
+
 // ---------------------------------------------------------------- boxes
 
-scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, const float* h_ref,
-                               int32_t cap, float* h_lo, float* h_hi, int32_t* n_boxes,
-                               int32_t* front_size) {
-    if (!h_ref || !n_boxes || cap < 0 || n_pts < 0 || (n_pts > 0 && !h_y)) return SCOOT_EINVAL;
-    if (n_obj < 2 || n_obj > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
-    const int M = n_obj;
+// The points of y ([M][n_pts]) strictly above the reference point that no
+// other such point dominates (duplicates kept once: the first).  False on a
+// non-finite value.
+static bool pareto_front(const float* h_y, int32_t n_pts, int M, const float* h_ref,
+                         std::vector<std::vector<double>>* front) {
     for (int j = 0; j < M; ++j)
-        if (!is_finite(h_ref[j])) return SCOOT_EINVAL;
-    // Points strictly above the reference point.
+        if (!is_finite(h_ref[j])) return false;
     std::vector<std::vector<double>> pts;
     for (int i = 0; i < n_pts; ++i) {
         std::vector<double> p(M);
         bool above = true;
         for (int j = 0; j < M; ++j) {
             p[j] = h_y[(size_t)j * n_pts + i];
-            if (!is_finite(p[j])) return SCOOT_EINVAL;
+            if (!is_finite(p[j])) return false;
             above &= p[j] > (double)h_ref[j];
         }
         if (above) pts.push_back(p);
     }
-    // Non-dominated subset (duplicates kept once).
-    std::vector<std::vector<double>> front;
+    front->clear();
     for (size_t i = 0; i < pts.size(); ++i) {
         bool dom = false;
         for (size_t k = 0; k < pts.size() && !dom; ++k) {
@@ -528,8 +557,19 @@ scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, c
             }
             dom = ge && (gt || k < i);
         }
-        if (!dom) front.push_back(pts[i]);
+        if (!dom) front->push_back(pts[i]);
     }
+    return true;
+}
+
+scoot_status scoot_boxes_build(const float* h_y, int32_t n_pts, int32_t n_obj, const float* h_ref,
+                               int32_t cap, float* h_lo, float* h_hi, int32_t* n_boxes,
+                               int32_t* front_size) {
+    if (!h_ref || !n_boxes || cap < 0 || n_pts < 0 || (n_pts > 0 && !h_y)) return SCOOT_EINVAL;
+    if (n_obj < 2 || n_obj > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
+    const int M = n_obj;
+    std::vector<std::vector<double>> front;
+    if (!pareto_front(h_y, n_pts, M, h_ref, &front)) return SCOOT_EINVAL;
     if (front_size) *front_size = (int32_t)front.size();
     // Grid on axes 0 .. M-2: the reference coordinate and the front's.
     const int G = M - 1;
@@ -726,6 +766,92 @@ scoot_status scoot_forest_pack(const scoot_forest_layout* L, const scoot_node* h
                     out[i].left = (uint16_t)(h_tree_offset[t] - node0 + h_nodes[i].left);
             }
     }
+    return SCOOT_OK;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------- fantasy state
+
+void scoot_fant_layout(int32_t n, int32_t d, int32_t M, int32_t q, FantHeader* h) {
+    std::memset(h, 0, sizeof(*h));
+    h->magic = kFantMagic;
+    h->n = n;
+    h->d = d;
+    h->M = M;
+    h->q = q;
+    int64_t off = align_up((int64_t)sizeof(FantHeader));
+    h->off_space = off; off = align_up(off + (int64_t)d * 4 * 8);
+    h->off_u = off;     off = align_up(off + (int64_t)n * d * 8);
+    h->off_ell = off;   off = align_up(off + (int64_t)M * d * 8);
+    h->off_alpha = off; off = align_up(off + (int64_t)M * n * 8);
+    h->off_linv = off;  off = align_up(off + (int64_t)M * n * n * 8);
+    h->off_front = off; off = align_up(off + (int64_t)n * M * 8);
+    h->bytes = off;
+}
+
+scoot_status scoot_fant_header(const scoot_param* h_space, const scoot_gp_layout* L, const float* h_y,
+                               const float* h_signal_var, const float* h_noise_var, const float* h_ref, int32_t q,
+                               void* h_fant, int64_t cap) {
+    if (!h_space || !L || !h_y || !h_signal_var || !h_noise_var || !h_ref || !h_fant) return SCOOT_EINVAL;
+    const int n = L->n, d = L->d, M = L->n_obj;
+    if (M < 2 || M > SCOOT_MAX_OBJ) return SCOOT_EUNSUPPORTED;
+    if (q < 1 || q > SCOOT_MAX_Q) return SCOOT_EUNSUPPORTED;
+    FantHeader h;
+    scoot_fant_layout(n, d, M, q, &h);
+    if (cap < h.bytes) return SCOOT_ENOMEM;
+    std::vector<std::vector<double>> front;
+    if (!pareto_front(h_y, n, M, h_ref, &front)) return SCOOT_EINVAL;
+    h.kernel = L->kernel;
+    h.front0 = (int32_t)front.size();
+    h.front_cap = h.front0 + q;
+    // Cells of the box decomposition of a front of front_cap points: at most
+    // front_cap + 1 grid coordinates on each of the first M - 1 axes.
+    double cells = 1.0;
+    for (int j = 0; j < M - 1; ++j) cells *= (double)(h.front_cap + 1);
+    h.box_cap = cells > (double)kFantBoxMax ? kFantBoxMax : (int32_t)cells;
+    for (int m = 0; m < M; ++m) {
+        h.ref[m] = h_ref[m];
+        h.sf2[m] = h_signal_var[m];
+        h.tau2[m] = h_noise_var[m];
+    }
+    char* base = static_cast<char*>(h_fant);
+    std::memcpy(base, &h, sizeof(h));
+    double* sp = reinterpret_cast<double*>(base + h.off_space);
+    for (int c = 0; c < d; ++c) {
+        sp[c * 4 + 0] = h_space[c].kind;
+        sp[c * 4 + 1] = h_space[c].lo;
+        sp[c * 4 + 2] = h_space[c].hi;
+        sp[c * 4 + 3] = h_space[c].n_choices;
+    }
+    double* fr = reinterpret_cast<double*>(base + h.off_front);
+    for (size_t i = 0; i < front.size(); ++i)
+        for (int m = 0; m < M; ++m) fr[i * M + m] = front[i][m];
+    return SCOOT_OK;
+}
+
+extern "C" {
+
+scoot_status scoot_fantasy_state_bytes(const scoot_gp_layout* L, int32_t q, int64_t* bytes) {
+    if (!L || !bytes || !scoot_gp_layout_valid(L)) return SCOOT_EINVAL;
+    if (q < 1 || q > SCOOT_MAX_Q) return SCOOT_EUNSUPPORTED;
+    FantHeader h;
+    scoot_fant_layout(L->n, L->d, L->n_obj, q, &h);
+    *bytes = h.bytes;
+    return SCOOT_OK;
+}
+
+scoot_status scoot_fantasy_prepare(const scoot_param* h_space, const scoot_gp_layout* L, const uint32_t* h_x_obs,
+                                   int64_t ld_obs, const float* h_y, const float* h_lengthscale,
+                                   const float* h_signal_var, const float* h_noise_var, const float* h_ref,
+                                   int32_t q, void* h_out, int64_t cap, int32_t* box_cap) {
+    if (!L || !scoot_gp_layout_valid(L)) return SCOOT_EINVAL;
+    scoot_status s = scoot_fant_header(h_space, L, h_y, h_signal_var, h_noise_var, h_ref, q, h_out, cap);
+    if (s != SCOOT_OK) return s;
+    s = scoot_gp_build(h_space, h_x_obs, ld_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, nullptr, L,
+                       nullptr, nullptr, h_out);
+    if (s != SCOOT_OK) return s;
+    if (box_cap) *box_cap = static_cast<const FantHeader*>(h_out)->box_cap;
     return SCOOT_OK;
 }
 

@@ -67,6 +67,47 @@ scoot_status scoot_host_gp(const scoot_param* sp, int d, const uint32_t* x_obs, 
                            const float* y, const float* lengthscale, float signal_var, float noise_var,
                            int kernel, HostGP* out, double* cond, const float* warp = nullptr);
 
+// Layout of the fp64 state of the sequential fantasised picks: built on the
+// host (scoot_fantasy_prepare, or scoot_round_state_build with fantasy_q >
+// 0) and read by the fantasy kernels.  Offsets count from the start of the
+// state and are 256-byte aligned; parameters are in their original order.
+struct FantHeader {
+    int32_t magic;                 // kFantMagic
+    int32_t n, d, M, kernel, q;    // observations, parameters, objectives, covariance, picks
+    int32_t front0;                // size of the observations' Pareto front
+    int32_t front_cap;             // front0 + q: the front can only grow by one point per pick
+    int32_t box_cap;               // cells of the box decomposition the picks may need
+    int32_t pad[7];
+    double ref[4], sf2[4], tau2[4];
+    int64_t off_space;             // double [d][4]: kind, lo, hi, n_choices
+    int64_t off_u;                 // double [n][d]: features of the observations
+    int64_t off_ell;               // double [M][d]: lengthscales
+    int64_t off_alpha;             // double [M][n]: (K + tau^2 I)^{-1} y
+    int64_t off_linv;              // double [M][n][n]: L^{-1}, column-major (entry (i, c) at c n + i)
+    int64_t off_front;             // double [n][M]: the observations' front (first front0 rows)
+    int64_t bytes;
+};
+constexpr int32_t kFantMagic = 0x544e4146;
+// Largest box count the fantasy kernels stage (2 float4 per box in shared memory).
+constexpr int32_t kFantBoxMax = 6144;
+// Offsets and size of a fantasy state for n observations, d parameters, M
+// objectives and q picks (front0, front_cap, box_cap and the values are left 0).
+void scoot_fant_layout(int32_t n, int32_t d, int32_t M, int32_t q, FantHeader* h);
+
+// The GP blob (h_blob, may be NULL) and/or the fp64 arrays of a fantasy state
+// whose header is already laid out (h_fant, may be NULL) from one
+// factorisation per objective; scoot_gp_prepare_warped is this call with
+// h_fant = NULL.  Fantasy states take no warping (SCOOT_EUNSUPPORTED).
+scoot_status scoot_gp_build(const scoot_param* h_space, const uint32_t* h_x_obs, int64_t ld_obs, const float* h_y,
+                            const float* h_lengthscale, const float* h_signal_var, const float* h_noise_var,
+                            const float* h_warp, const scoot_gp_layout* L, void* h_blob, double* h_cond,
+                            void* h_fant);
+// The header, space, front and scalars of a fantasy state (everything but the
+// factorisation's arrays, which scoot_gp_build writes).
+scoot_status scoot_fant_header(const scoot_param* h_space, const scoot_gp_layout* L, const float* h_y,
+                               const float* h_signal_var, const float* h_noise_var, const float* h_ref, int32_t q,
+                               void* h_fant, int64_t cap);
+
 // Consistency of a GP layout's offsets with its own sizes.
 bool scoot_gp_layout_valid(const scoot_gp_layout* L);
 

@@ -152,7 +152,7 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
     if (!in || !out || (cap > 0 && !h_buf) || cap < 0) return SCOOT_EINVAL;
     std::memset(out, 0, sizeof(*out));
     out->off_gp = out->off_forest = out->off_box_lo = out->off_box_hi = out->off_eps = -1;
-    out->off_grid = out->off_corner = -1;
+    out->off_grid = out->off_corner = out->off_fant = -1;
     if (!in->space || !in->x_obs || !in->y || !in->nodes || !in->tree_offset) return SCOOT_EINVAL;
     if (in->boxes < 0 || in->boxes > 2) return SCOOT_EINVAL;
     const int M = in->n_obj, n = in->n;
@@ -166,6 +166,23 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
         off += slot(out->gp.bytes);
     }
     char* buf = static_cast<char*>(h_buf);
+    // The fantasy state: its header and front now, its fp64 arrays from the
+    // GP job's own factorisation.
+    void* fant = nullptr;
+    if (in->fantasy_q > 0) {
+        if (in->gp_on_device || in->warp || !in->ref) return SCOOT_EINVAL;
+        FantHeader fl;
+        scoot_fant_layout(n, in->d, M, in->fantasy_q, &fl);
+        out->off_fant = off;
+        off += slot(fl.bytes);
+        if (out->off_fant + fl.bytes <= cap) {
+            s = scoot_fant_header(in->space, &out->gp, in->y, in->signal_var, in->noise_var, in->ref, in->fantasy_q,
+                                  buf + out->off_fant, fl.bytes);
+            if (s != SCOOT_OK) return s;
+            fant = buf + out->off_fant;
+            out->fant_box_cap = static_cast<const FantHeader*>(fant)->box_cap;
+        }
+    }
     // The GP factorisation first, on the worker, if its slot fits.
     scoot_status gp_status = SCOOT_OK;
     Pool::Latch latch;
@@ -174,9 +191,9 @@ scoot_status scoot_round_state_build(const scoot_round_inputs* in, void* h_buf, 
         double* cond = out->cond;
         const scoot_round_inputs* pin = in;
         const scoot_gp_layout* gl = &out->gp;
-        Pool::get().submit([pin, gl, buf, cond, &gp_status] {
-            gp_status = scoot_gp_prepare_warped(pin->space, pin->x_obs, pin->ld_obs, pin->y, pin->lengthscale,
-                                                pin->signal_var, pin->noise_var, pin->warp, gl, buf, cond);
+        Pool::get().submit([pin, gl, buf, cond, fant, &gp_status] {
+            gp_status = scoot_gp_build(pin->space, pin->x_obs, pin->ld_obs, pin->y, pin->lengthscale,
+                                       pin->signal_var, pin->noise_var, pin->warp, gl, buf, cond, fant);
         }, &latch);
     }
     auto finish = [&](scoot_status st) {

@@ -102,90 +102,6 @@ __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, 
     return total;
 }
 
-// Width that stands in for an unbounded side of a box on the first M-1
-// objectives: a power of two, so scaling by it and by its inverse is exact;
-// valid while every sample lies within 2^40 of the box's lower corner.
-constexpr float kOpenWidth = 1099511627776.0f;  // 2^40
-
-// Boxes open on the last objective in "saturated" form: for the first M-1
-// objectives a_j = 1/w_j and b_j = -l_j/w_j (w_j the box width), and for the
-// last one W = prod_j w_j and C = -l_last * W, so that a box's HVI term is
-//   prod_{j<M-1} sat(y_j a_j + b_j) * max(y_last W + C, 0)
-// (sat clamps to [0, 1]): one saturated FMA per bounded objective.
-// Row b holds (a_0, b_0, a_1, b_1) and (a_2, b_2, W, C) as two float4.
-__device__ __forceinline__ void stage_boxes_sat(const float* box_lo, const float* box_hi, int n_boxes, int M,
-                                                float4* bs) {
-    for (int b = threadIdx.x; b < n_boxes; b += blockDim.x) {
-        float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        float W = 1.0f;
-        for (int j = 0; j < M - 1; ++j) {
-            const float l = box_lo[b * M + j], h = box_hi[b * M + j];
-            const float w = h == INFINITY ? kOpenWidth : h - l;
-            v[2 * j] = 1.0f / w;
-            v[2 * j + 1] = -l / w;
-            W *= w;
-        }
-        v[6] = W;
-        v[7] = -box_lo[b * M + M - 1] * W;
-        bs[2 * b] = make_float4(v[0], v[1], v[2], v[3]);
-        bs[2 * b + 1] = make_float4(v[4], v[5], v[6], v[7]);
-    }
-}
-
-template <int M>
-__device__ __forceinline__ float ehvi_partial_sat(const float* mu, const float* sd, const float4* bs, int n_boxes,
-                                                 const float4* eps, int n_mc, int first, int stride) {
-    constexpr int kCh = 8;
-    float total = 0.0f;
-    for (int s0 = first * kCh; s0 < n_mc; s0 += stride * kCh) {
-        float y[kCh][M], acc[kCh];
-#pragma unroll
-        for (int k = 0; k < kCh; ++k) {
-            acc[k] = 0.0f;
-            const bool in = s0 + k < n_mc;
-            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float ev[4] = {e.x, e.y, e.z, e.w};
-#pragma unroll
-            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
-        }
-        for (int b = 0; b < n_boxes; ++b) {
-            const float4 q0 = bs[2 * b];
-            const float4 q1 = (M > 2) ? bs[2 * b + 1] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float W = M > 2 ? q1.z : bs[2 * b + 1].z;
-            const float Cc = M > 2 ? q1.w : bs[2 * b + 1].w;
-#pragma unroll
-            for (int k = 0; k < kCh; ++k) {
-                float p = __saturatef(fmaf(y[k][0], q0.x, q0.y));
-                if (M > 2) p *= __saturatef(fmaf(y[k][1], q0.z, q0.w));
-                if (M > 3) p *= __saturatef(fmaf(y[k][2], q1.x, q1.y));
-                acc[k] = fmaf(p, fmaxf(fmaf(y[k][M - 1], W, Cc), 0.0f), acc[k]);
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < kCh; ++k) total += acc[k];
-    }
-    return total;
-}
-
-// True (in every thread) when the saturated form is exact for the staged
-// boxes: every box is open on the last objective, M <= 3, and every lower
-// corner lies within 2^30 of zero.  The form folds one open width 2^40 per
-// open leading axis into W, so W <= 2^80 and |C| <= 2^110 for M <= 3 (finite
-// in fp32 for samples within 2^40 of the corner); with M = 4 the last box
-// would carry W = 2^120, whose products with y_last and l_last overflow (and
-// whose reciprocal factors underflow) at ordinary objective scales, so M = 4
-// always takes the general form.
-__device__ __forceinline__ bool boxes_fast(const float4* blo, const float4* bhi, int n_boxes, int M) {
-    int ok = M <= 3;
-    constexpr float kCornerMax = 1073741824.0f;  // 2^30
-    for (int b = threadIdx.x; b < n_boxes && ok; b += blockDim.x) {
-        const float4 h = bhi[b], l = blo[b];
-        ok &= (M == 2 ? h.y : (M == 3 ? h.z : h.w)) == INFINITY;
-        ok &= fabsf(l.x) < kCornerMax && fabsf(l.y) < kCornerMax && (M < 3 || fabsf(l.z) < kCornerMax);
-    }
-    return __syncthreads_and(ok) != 0;
-}
-
 // Asynchronous copy of one 32 x 64 tile of L^{-1} (8 KiB, 16-byte aligned at
 // both ends) into shared memory: each of the 128 threads moves four 16-byte
 // pieces with cp.async and commits them as one group.

@@ -117,7 +117,8 @@ class State:
                                                    inp.signal_var, inp.noise_var, inp.nodes, inp.tree_offset,
                                                    inp.leaf_scale, stage.numpy(), kernel=inp.kernel, warp=inp.warp,
                                                    boxes=boxes, h_ref=inp.ref, h_eps=inp.eps,
-                                                   gp_on_device=gp_on_device)
+                                                   gp_on_device=gp_on_device,
+                                                   fantasy_q=inp.q if inp.fantasy else 0)
             if built is not None:
                 break
             stage = _staging.take(int(out.bytes))
@@ -130,7 +131,8 @@ class State:
             self.n_grid = np.array(out.n_grid[:M], np.int32)
         total = int(out.bytes)
         offsets = (int(out.off_gp), int(out.off_forest), int(out.off_box_lo), int(out.off_box_hi), int(out.off_eps),
-                   int(out.off_grid), int(out.off_corner), total)
+                   int(out.off_grid), int(out.off_corner), int(out.off_fant), total)
+        self.fant_box_cap = int(out.fant_box_cap)
         reuse = into is not None and into.buffer.numel() == total and into.offsets == offsets
         if reuse:
             dev = into.buffer
@@ -145,7 +147,8 @@ class State:
         self.offsets = offsets
         self.upload_bytes = total + (self.gp_upload_bytes if gp_on_device else 0)
         if reuse:  # same offsets: the views of `into` are views of this buffer
-            for name in ("forest", "box_lo", "box_hi", "eps", "grid", "corner") + (() if gp_on_device else ("gp_state",)):
+            for name in ("forest", "box_lo", "box_hi", "eps", "grid", "corner", "fant_state") + \
+                    (() if gp_on_device else ("gp_state",)):
                 if hasattr(into, name):
                     setattr(self, name, getattr(into, name))
             return
@@ -156,6 +159,8 @@ class State:
         if not gp_on_device:
             self.gp_state = view(out.off_gp, self.gp_layout.bytes)
         self.forest = view(out.off_forest, self.forest_layout.bytes)
+        if inp.fantasy:
+            self.fant_state = view(out.off_fant, S.scoot_fantasy_state_bytes(self.gp_layout, inp.q))
         B = self.n_boxes
         if boxes:
             self.box_lo = view(out.off_box_lo, B * M * 4, torch.float32, (B, M))
@@ -210,7 +215,7 @@ class ScoringRound:
         self.top_count = torch.empty(1, dtype=torch.int32, device=dev)
         self.work = None
         if inp.fantasy:
-            nbytes = S.scoot_fantasy_work_bytes(self.state.gp_layout, self.capacity, q)
+            nbytes = S.scoot_fantasy_work_bytes(self.state.gp_layout, self.capacity, q, self.state.fant_box_cap)
             self.work = torch.empty(nbytes, dtype=torch.uint8, device=dev)
         self.picks = None
         self.sobol_skip = 0  # next point of the Sobol sequence for shortfall fills
@@ -231,13 +236,13 @@ class ScoringRound:
     def kernels_per_round(self):
         """Library kernel launches of one run(): prune, compaction, forest walk, then
         either compaction + fused score + two top-q passes, or (fantasies)
-        compaction + posterior + per pick EHVI, two argmax passes and a downdate
-        (the last pick skips the downdate)."""
+        compaction + posterior + the front's boxes + per pick a pass (downdate,
+        EHVI, block argmax) and the pick's terms."""
         if self.inp.acq == "mace":
             return 10  # prune, compaction, forest, compaction, score, five Pareto kernels
         if not self.inp.fantasy:
             return 7
-        return 3 + 2 + 4 * self.inp.q - 1
+        return 3 + 3 + 2 * self.inp.q
 
     def fill_shortfall(self, batch: int = 4096, stream=None):
         """Section 4.6: when a round yields fewer than q suggestions, the rest
@@ -277,14 +282,9 @@ class ScoringRound:
         S.scoot_rf_predict(self.ctx, st.forest_layout, st.forest, inp.space, cand, n, inp.delta_num,
                            inp.delta_den, self.votes, self.mask, self.n_feasible, stream)
         if inp.fantasy:
-            idx, val = S.scoot_suggest_fantasy(self.ctx, st.gp_layout, st.gp_state, inp.space, inp.x_obs, inp.y_obs,
-                                               inp.lengthscale, inp.signal_var, inp.noise_var, cand, n, inp.ref,
-                                               st.eps, inp.q, self.work, mask=self.mask, stream=stream)
-            self.picks = (idx, val)
-            k = len(idx)
-            self.top_idx[:k].copy_(torch.from_numpy(idx))
-            self.top_val[:k].copy_(torch.from_numpy(val))
-            self.top_count.fill_(k)
+            S.scoot_suggest_fantasy(self.ctx, st.gp_layout, st.gp_state, st.fant_state, st.fant_box_cap, cand, n,
+                                    st.eps, inp.q, self.work, self.top_idx, self.top_val, self.top_count,
+                                    mask=self.mask, stream=stream)
             return self.top_idx, self.top_val, self.top_count
         if inp.acq == "mace":
             S.scoot_score_mace(self.ctx, st.gp_layout, st.gp_state, cand, n, inp.xi, self.kappa, self.acq3,

@@ -66,13 +66,14 @@ class scoot_round_inputs(C.Structure):
                 ("signal_var", C.c_void_p), ("noise_var", C.c_void_p), ("warp", C.c_void_p), ("kernel", C.c_int32),
                 ("gp_on_device", C.c_int32), ("nodes", C.c_void_p), ("tree_offset", C.c_void_p),
                 ("n_trees", C.c_int32), ("leaf_scale", C.c_int32), ("boxes", C.c_int32), ("ref", C.c_void_p),
-                ("eps", C.c_void_p), ("n_mc", C.c_int32), ("grid_cap", C.c_int32)]
+                ("eps", C.c_void_p), ("n_mc", C.c_int32), ("grid_cap", C.c_int32), ("fantasy_q", C.c_int32)]
 
 
 class scoot_round_state(C.Structure):
     _fields_ = [("bytes", C.c_int64), ("off_gp", C.c_int64), ("off_forest", C.c_int64),
                 ("off_box_lo", C.c_int64), ("off_box_hi", C.c_int64), ("off_eps", C.c_int64),
-                ("off_grid", C.c_int64), ("off_corner", C.c_int64), ("n_boxes", C.c_int32),
+                ("off_grid", C.c_int64), ("off_corner", C.c_int64), ("off_fant", C.c_int64),
+                ("fant_box_cap", C.c_int32), ("n_boxes", C.c_int32),
                 ("front_size", C.c_int32), ("grid_cap", C.c_int32), ("n_grid", C.c_int32 * 4),
                 ("cond", C.c_double * 4), ("gp", scoot_gp_layout), ("forest", scoot_forest_layout)]
 
@@ -131,9 +132,12 @@ _PROTOS = {
     "scoot_rf_train_work_bytes": [_i32, _i32, C.POINTER(_i64)],
     "scoot_select_pareto": [_vp, _vp, _i64, _vp, _i64, _i32, C.c_uint64, _vp, _vp, _vp, _i64, _vp],
     "scoot_select_topq_static": [_vp, _vp, _i64, _i32, _vp, _vp, _vp, _vp],
-    "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, C.POINTER(_i64)],
-    "scoot_suggest_fantasy": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _vp, _i64, _vp, _vp, _vp, _vp,
-                              _vp, _i64, _i64, _vp, _vp, _vp, _i32, _i32, _vp, _i64, _vp, _vp, _vp, _vp, _vp],
+    "scoot_fantasy_state_bytes": [C.POINTER(scoot_gp_layout), _i32, C.POINTER(_i64)],
+    "scoot_fantasy_prepare": [_vp, C.POINTER(scoot_gp_layout), _vp, _i64, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _i64,
+                              C.POINTER(_i32)],
+    "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, _i32, C.POINTER(_i64)],
+    "scoot_suggest_fantasy": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i32, _vp, _i64, _i64, _vp, _vp, _i32,
+                              _i32, _vp, _i64, _vp, _vp, _vp, _vp, _vp],
 }
 _STRING_FUNCS = {"scoot_last_error", "scoot_status_string"}
 EXPORTS = tuple(_PROTOS)
@@ -339,7 +343,8 @@ def scoot_boxes_index(h_lo, h_hi, grid_cap: int = 256):
 
 def scoot_round_state_build(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, h_nodes,
                             h_tree_offset, leaf_scale: int, buf, kernel: int = 0, warp=None, boxes: int = 0,
-                            h_ref=None, h_eps=None, grid_cap: int = 0, gp_on_device: bool = False):
+                            h_ref=None, h_eps=None, grid_cap: int = 0, gp_on_device: bool = False,
+                            fantasy_q: int = 0):
     """A round's host state packed into the host uint8 array buf (pinned
     staging memory; see include/scoot.h).  Returns the scoot_round_state, or
     None when buf is too small (the size needed is then in .bytes of the
@@ -373,6 +378,11 @@ def scoot_round_state_build(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, 
         inp.eps = _host(keep[-1])
         inp.n_mc = int(keep[-1].shape[0])
     inp.grid_cap = int(grid_cap)
+    if fantasy_q:
+        if not boxes:
+            keep.append(np.ascontiguousarray(h_ref, np.float32))
+            inp.ref = _host(keep[-1])
+        inp.fantasy_q = int(fantasy_q)
     out = scoot_round_state()
     st = lib().scoot_round_state_build(C.byref(inp), _host(buf), int(buf.nbytes), C.byref(out))
     if st == -2 and out.bytes > buf.nbytes:  # SCOOT_ENOMEM: the buffer is too small
@@ -651,27 +661,41 @@ def compact_forest(nodes: np.ndarray, n_nodes: np.ndarray):
     return out, offs
 
 
-def scoot_fantasy_work_bytes(layout, n: int, q: int) -> int:
+def scoot_fantasy_state_bytes(layout, q: int) -> int:
     v = _i64()
-    _check(lib().scoot_fantasy_work_bytes(C.byref(layout), int(n), int(q), C.byref(v)), "scoot_fantasy_work_bytes")
+    _check(lib().scoot_fantasy_state_bytes(C.byref(layout), int(q), C.byref(v)), "scoot_fantasy_state_bytes")
     return int(v.value)
 
 
-def scoot_suggest_fantasy(ctx, layout, state, h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var,
-                          cand, n, h_ref, eps, q, work, mask=None, var_out=None, stream=None):
-    """Returns (idx int64[count], val float32[count]) of q sequential fantasised picks."""
-    import torch
-    idx = np.full(q, -1, np.int64)
-    val = np.full(q, -np.inf, np.float32)
-    cnt = _i32()
-    _check(lib().scoot_suggest_fantasy(
-        _h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"), _host(h_space, 16, name="h_space"),
-        _host(h_x_obs, 4, name="h_x_obs"), int(h_x_obs.shape[1]), _host(h_y, dtype=np.float32, name="h_y"),
-        _host(h_lengthscale, dtype=np.float32, name="h_lengthscale"),
+def scoot_fantasy_prepare(h_space, h_x_obs, h_y, h_lengthscale, h_signal_var, h_noise_var, h_ref, q, layout):
+    """The fp64 fantasy state (host uint8 array) and its box_cap."""
+    out = np.zeros(scoot_fantasy_state_bytes(layout, q), np.uint8)
+    box_cap = _i32()
+    _check(lib().scoot_fantasy_prepare(
+        _host(h_space, 16, name="h_space"), C.byref(layout), _host(h_x_obs, 4, name="h_x_obs"), int(h_x_obs.shape[1]),
+        _host(h_y, dtype=np.float32, name="h_y"), _host(h_lengthscale, dtype=np.float32, name="h_lengthscale"),
         _host(h_signal_var, dtype=np.float32, name="h_signal_var"),
-        _host(h_noise_var, dtype=np.float32, name="h_noise_var"), _dev(cand, torch.int32, "cand"), int(n),
-        int(cand.shape[1]), _dev(mask, torch.uint8, "mask"), _host(h_ref, dtype=np.float32, name="h_ref"),
+        _host(h_noise_var, dtype=np.float32, name="h_noise_var"), _host(h_ref, dtype=np.float32, name="h_ref"),
+        int(q), _host(out), int(out.nbytes), C.byref(box_cap)), "scoot_fantasy_prepare")
+    return out, int(box_cap.value)
+
+
+def scoot_fantasy_work_bytes(layout, n: int, q: int, box_cap: int) -> int:
+    v = _i64()
+    _check(lib().scoot_fantasy_work_bytes(C.byref(layout), int(n), int(q), int(box_cap), C.byref(v)),
+           "scoot_fantasy_work_bytes")
+    return int(v.value)
+
+
+def scoot_suggest_fantasy(ctx, layout, state, fant_state, box_cap, cand, n, eps, q, work, idx, val, count,
+                          mask=None, var_out=None, stream=None):
+    """q sequential fantasised picks into the device arrays idx (int64 [q]),
+    val (float32 [q]) and count (int32 [1]); asynchronous on stream."""
+    import torch
+    _check(lib().scoot_suggest_fantasy(
+        _h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"), _dev(fant_state, torch.uint8, "fant_state"),
+        int(box_cap), _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]), _dev(mask, torch.uint8, "mask"),
         _dev(eps, torch.float32, "eps"), int(eps.shape[0]), int(q), _vp(work.data_ptr()), int(work.numel()),
-        _host(idx), _host(val), C.byref(cnt), _dev(var_out, torch.float32, "var_out"), _stream(stream)),
+        _dev(idx, torch.int64, "idx"), _dev(val, torch.float32, "val"), _dev(count, torch.int32, "count"),
+        _dev(var_out, torch.float32, "var_out"), _stream(stream)),
         "scoot_suggest_fantasy", _h(ctx))
-    return idx[:cnt.value], val[:cnt.value]

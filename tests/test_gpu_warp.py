@@ -124,12 +124,20 @@ def test_identity_warp_equals_no_warp(S, ctx):
 
 
 def test_fantasy_refuses_a_warped_state(S, ctx):
+    """The fantasy downdates rebuild the covariance without warping: a warped
+    GP state stops the picks on the device, reported as SCOOT_EINVAL."""
     name = "d12-fantasy"
     inst = make_instance(name, seeds(name)[0], n_cand=4096)
     L, state = warped_state(S, inst, warp_params(name, 1), 0)
-    work = torch.empty(S.scoot_fantasy_work_bytes(L, inst.n_cand, 2), dtype=torch.uint8, device="cuda")
+    fant, box_cap = S.scoot_fantasy_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                            inst.noise_var, inst.ref, 2, L)
+    work = torch.empty(S.scoot_fantasy_work_bytes(L, inst.n_cand, 2, box_cap), dtype=torch.uint8, device="cuda")
+    idx = torch.empty(2, dtype=torch.int64, device="cuda")
+    val = torch.empty(2, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int32, device="cuda")
+    S.scoot_suggest_fantasy(ctx, L, state, dev(fant), box_cap, dev(inst.cand.view(np.int32)), inst.n_cand,
+                            dev(inst.eps), 2, work, idx, val, cnt)
     with pytest.raises(S.ScootError) as e:
-        S.scoot_suggest_fantasy(ctx, L, state, inst.space, inst.x_obs, inst.y_obs, inst.lengthscale,
-                                inst.signal_var, inst.noise_var, dev(inst.cand.view(np.int32)), inst.n_cand,
-                                inst.ref, dev(inst.eps), 2, work)
-    assert e.value.status == -6
+        ctx.check()
+    assert e.value.status == -1
+    assert int(cnt.item()) == 0

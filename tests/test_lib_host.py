@@ -402,3 +402,46 @@ def test_scratch_sizes_and_buffer_layout(S):
             S.scoot_gp_mle_work_bytes(*bad)
     with pytest.raises(S.ScootError):
         S.scoot_rf_train_work_bytes(0, 3)
+
+
+@pytest.mark.parametrize("name,q", [("d12-fantasy", 16), ("d8-ehvi2", 4), ("d10-ehvi3", 3)])
+def test_fantasy_state_holds_the_fp64_factorisation(S, name, q):
+    """The fantasy state: header, space, features, lengthscales, alpha and
+    L^{-1} in fp64 (L L^T = K + tau^2 I of the oracle's GP), the front of the
+    observations above r (the oracle's pareto_front) and the box bound
+    (front + q + 1)^(M - 1); the round-state builder writes the same bytes."""
+    inst = make_instance(name, seeds(name)[0], n_cand=8)
+    M, n, d = inst.n_obj, inst.n_obs, inst.d
+    G = S.scoot_gp_layout_init(inst.space, n, M)
+    st, box_cap = S.scoot_fantasy_prepare(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                          inst.noise_var, inst.ref, q, G)
+    hdr = st[:64].view(np.int32)
+    magic, hn, hd, hM, kern, hq, front0, front_cap, hbox = hdr[:9]
+    assert magic == 0x544e4146 and (hn, hd, hM, kern, hq) == (n, d, M, 0, q)
+    front = O.pareto_front(inst.y_obs.T.astype(np.float64), inst.ref.astype(np.float64))
+    assert front0 == len(front) and front_cap == len(front) + q
+    assert hbox == box_cap == min((len(front) + q + 1) ** (M - 1), 6144)
+    offs = st[160:216].view(np.int64)
+    off_space, off_u, off_ell, off_alpha, off_linv, off_front, nbytes = offs
+    assert nbytes == S.scoot_fantasy_state_bytes(G, q) == len(st)
+    dbl = lambda off, cnt: st[off:off + 8 * cnt].view(np.float64)
+    sp = dbl(off_space, 4 * d).reshape(d, 4)
+    assert np.array_equal(sp[:, 0], inst.space["kind"]) and np.array_equal(sp[:, 1], inst.space["lo"].astype(np.float64))
+    fr = dbl(off_front, front0 * M).reshape(front0, M)
+    assert np.array_equal(np.array(sorted(map(tuple, fr))), np.array(sorted(map(tuple, front))))
+    for m in range(M):
+        gp = O.GP(inst.space, inst.x_obs, inst.y_obs[m], inst.lengthscale[m], inst.signal_var[m], inst.noise_var[m])
+        assert np.allclose(dbl(off_u, n * d).reshape(n, d), gp.u_obs, rtol=1e-14, atol=1e-14)
+        assert np.array_equal(dbl(off_ell + 8 * m * d, d), inst.lengthscale[m].astype(np.float64))
+        alpha = dbl(off_alpha + 8 * m * n, n)
+        assert np.allclose(alpha, gp.alpha, rtol=1e-9, atol=1e-10 * np.abs(gp.alpha).max())
+        Li = dbl(off_linv + 8 * m * n * n, n * n).reshape(n, n).T  # column-major
+        assert np.allclose(np.tril(Li), Li)
+        assert np.allclose(Li @ gp.chol, np.eye(n), atol=1e-8)
+    # the round-state builder writes the same fantasy state from its own factorisation
+    buf = np.zeros(64 << 20, np.uint8)
+    out, _ = S.scoot_round_state_build(inst.space, inst.x_obs, inst.y_obs, inst.lengthscale, inst.signal_var,
+                                       inst.noise_var, inst.nodes, inst.tree_offset, inst.workload.leaf_scale, buf,
+                                       boxes=1, h_ref=inst.ref, h_eps=inst.eps, fantasy_q=q)
+    assert out.off_fant >= 0 and out.off_fant % 256 == 0 and out.fant_box_cap == box_cap
+    assert np.array_equal(buf[out.off_fant:out.off_fant + len(st)], st)

@@ -631,6 +631,22 @@ def test_fantasy_picks_equal_a_from_scratch_recomputation(noise):
         assert repick, "the case must exercise the exclusion of picked candidates"
 
 
+def test_fantasy_picks_on_a_subset_equal_the_whole_pool():
+    """Forced replay evaluated at a subset of the pool gives, at those
+    candidates, the values of the whole-pool run (the refits and fronts do
+    not depend on which candidates are evaluated)."""
+    inst = make_instance("tiny", seeds("tiny")[0], n_cand=200)
+    feas = Stream(5, "feas").uniform(inst.n_cand) < 0.9
+    full = O.fantasy_picks(inst, 4, feas)
+    sub = np.sort(Stream(6, "sub").u64(40) % np.uint64(inst.n_cand)).astype(np.int64)
+    part = O.fantasy_picks(inst, 4, feas, forced=full["picks"], subset=sub)
+    assert part["picks"] == full["picks"]
+    assert set(full["picks"]) <= set(part["index"].tolist())
+    for j in range(4):
+        assert np.allclose(part["acq"][j], full["acq"][j][part["index"]], rtol=1e-12, atol=1e-15)
+        assert np.allclose(part["var"][j], full["var"][j][part["index"]], rtol=1e-12, atol=1e-15)
+
+
 def _hand_instance(targets, q_noise=1e-8):
     """One observation x = 0 with y = (1, -1), one continuous parameter in
     [0, 1], both objectives with lengthscale 0.25, s_f^2 = 1, tau^2 = 1e-8;
