@@ -38,15 +38,16 @@ sys.path.insert(0, ROOT)
 
 METRIC = "candidate configs scored/sec (prune+RF+GP+acq+top-q) and % FP32/HBM roofline"
 UNIT = "candidates/s"
-DEFAULT_WORKLOAD = "d8-ehvi2"
+DEFAULT_WORKLOAD = "d12-fantasy"   # the largest workload (N = 2^22, q = 16 sequential picks)
+SUBRUN_WORKLOADS = ("d10-ei", "d10-ehvi3")  # the N = 2^20 workloads, measured beside the headline
 FLUSH_BYTES = 256 << 20   # > 129 MB of L2
 FP32_LANES_PER_SM = 128
 
 # DRAM bytes per launch from ncu (dram__bytes_read.sum + dram__bytes_write.sum),
-# keyed by (stage, workload), valid only while the stage kernel's sources are
-# unchanged (sha256 prefix of their contents when the counters were taken);
-# the captures are summarised in profiles/kernels_full_<workload>.md.
+# keyed by (kernel, workload), valid only while the kernel's sources are
+# unchanged (sha256 prefix of their contents when the counters were taken).
 KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["score.cu", "device_common.cuh"],
+                "posterior": ["score.cu", "device_common.cuh"], "fant_pass": ["fantasy.cu", "device_common.cuh"],
                 "topq": ["topq.cu", "device_common.cuh"], "pareto": ["pareto.cu"]}
 TRAFFIC = {
     ("prune", "d8-ehvi2"): {"bytes": 3151360, "sha": "669855124f47da70"},
@@ -62,6 +63,8 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--pool", type=int, default=None,
+                   help="pool size instead of the workload's own (smaller cases for profiling)")
     p.add_argument("--kernel", choices=["matern52", "matern32"], default="matern52",
                    help="covariance (matern32 with --warp is the paper's own kernel)")
     p.add_argument("--warp", action="store_true", help="Kumaraswamy input warping of ordinal features")
@@ -72,6 +75,8 @@ def parse_args():
     p.add_argument("--warmup-seconds", type=float, default=1.0, help="minimum warm-up time under load")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-extra", action="store_true",
+                   help="skip the probes and the N = 2^20 workloads measured beside the headline")
     p.add_argument("--gp-prep", choices=["auto", "host", "device"], default="auto",
                    help="where the end-to-end step builds the GP state (fp64 factorisation); auto: the "
                         "device from 100 observations (measured faster there), the host below")
@@ -81,12 +86,13 @@ def parse_args():
     return p.parse_args()
 
 
-def workload_config(w, extra=None, acq=None):
+def workload_config(w, extra=None, acq=None, pool=None):
     acq = acq or w.acq
-    desc = (f"{w.name}: d={w.d}, n={w.n_obs}, N={w.n_cand}, M={w.n_obj} {acq.upper()}"
+    pool = w.n_cand if pool is None else int(pool)
+    desc = (f"{w.name}: d={w.d}, n={w.n_obs}, N={pool}, M={w.n_obj} {acq.upper()}"
             + (f" S={w.n_mc}" if w.acq == "ehvi" else "")
             + f", RF {w.n_trees} trees depth<={w.max_depth}, q={w.q}")
-    cfg = {"workload": desc, "pool": w.n_cand, "observations": w.n_obs, "objectives": w.n_obj,
+    cfg = {"workload": desc, "pool": pool, "observations": w.n_obs, "objectives": w.n_obj,
            "acquisition": acq, "trees": w.n_trees, "q": w.q,
            "l2": "flushed between steps (256 MiB write)", "inputs": "seeded synthetic pool, resident in HBM"}
     if extra:
@@ -131,6 +137,108 @@ def work_model(inst, n_boxes, acq_kind=None, n_grid=None):
         "topq": ("hbm", 4 + 1),
         "pareto": ("hbm", 12 + 1),
     }
+
+
+def fantasy_pass_bytes(inst, q, n_live):
+    """Algorithmic DRAM bytes of each of the q passes of a fantasy round over
+    n_live candidates: pass 0 reads the moments; pass j >= 1 also applies the
+    downdate of pick j-1, reading the candidate's n rows of V per objective,
+    its d configuration words and the j-1 earlier downdate factors, and
+    writing the variance and (if a later downdate needs it) the new factor."""
+    M, n, d = inst.n_obj, inst.n_obs, inst.d
+    out = []
+    for j in range(q):
+        b = M * 8
+        if j > 0:
+            b += M * 4 * n + 4 * d + M * 4 * (j - 1) + M * 4 + (M * 4 if j - 1 < q - 2 else 0)
+        out.append(b * n_live)
+    return out
+
+
+def posterior_flops(inst, n_obj=None):
+    """Flops per candidate of the GP posterior (covariance row, mean,
+    triangular product, variance), all objectives."""
+    d, n = inst.d, inst.n_obs
+    m = inst.n_obj if n_obj is None else n_obj
+    return m * (n * (3 * d + 12) + 2 * n + n * (n + 1) + 2 * n)
+
+
+def forest_visits(inst, idx):
+    """Mean node visits (root to leaf, leaf included, summed over the trees)
+    of the forest walk for the pool candidates idx, by a vectorised walk of
+    the host copy of the trees: the work of one candidate in the forest kernel."""
+    import numpy as np
+    nodes, offs = inst.nodes, inst.tree_offset
+    words = inst.cand[:, idx]
+    x = np.empty(words.shape, np.float32)
+    for c in range(inst.d):
+        if int(inst.space[c]["kind"]) == 3:
+            x[c] = words[c].view(np.float32)
+        else:
+            x[c] = words[c].view(np.int32).astype(np.float32)
+    cols = np.arange(len(idx))
+    total = 0
+    for t in range(len(offs) - 1):
+        base = int(offs[t])
+        node = np.zeros(len(idx), np.int64)
+        active = np.ones(len(idx), bool)
+        while active.any():
+            total += int(active.sum())
+            rec = nodes[base + node]
+            leaf = (rec["flags"] & 1).astype(bool)
+            active &= ~leaf
+            go = x[rec["feat"].astype(np.int64), cols] <= rec["val"]
+            node = np.where(active, rec["left"].astype(np.int64) + np.where(go, 0, 1), node)
+    return total / max(1, len(idx))
+
+
+def measure_probes(S, ctx, device, stream, sms):
+    """Measured peaks: FFMA and FFMA2 chains (TFLOP/s) and dependent node
+    gathers from shared memory (visits/s), best of five timed launches."""
+    import torch
+    blocks = sms * 8
+    sink = torch.zeros(blocks, device=device)
+
+    def timed(fn):
+        for _ in range(2):
+            fn()
+        best = float("inf")
+        for _ in range(5):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            e1.synchronize()
+            best = min(best, e0.elapsed_time(e1) / 1e3)
+        return best
+    iters, steps, n_nodes = 8192, 4096, 4095
+    out = {}
+    for packed, key in ((0, "ffma_tflops"), (1, "ffma2_tflops")):
+        t = timed(lambda: S.scoot_probe_fma(ctx, packed, blocks, iters, sink, stream))
+        out[key] = 2 * 16 * 256 * blocks * iters / t / 1e12
+    t = timed(lambda: S.scoot_probe_gather(ctx, n_nodes, blocks, steps, sink, stream))
+    out["smem_gather_visits_per_s"] = 256 * blocks * steps / t
+    out["how"] = (f"{blocks} blocks x 256 threads; 16 independent FMA chains x {iters} steps per thread "
+                  f"(scalar / packed pairs); {steps} dependent 8-byte node loads per thread from a "
+                  f"{n_nodes}-node tree in shared memory; best of 5 launches, CUDA events")
+    return out
+
+
+def sub_run(name, steps=20, warmup=5):
+    """The round of another workload, measured by this script in a child
+    process (no CPU baseline, no end-to-end leg): its value, stage times and
+    stage roofline fractions."""
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--workload", name, "--steps", str(steps),
+           "--warmup", str(warmup), "--no-cpu-baseline", "--no-e2e", "--no-extra"]
+    p = subprocess.run(cmd, capture_output=True, text=True, timeout=900)
+    if p.returncode != 0:
+        return {"error": p.stderr.strip().splitlines()[-1] if p.stderr.strip() else f"exit {p.returncode}"}
+    line = json.loads(p.stdout.strip().splitlines()[-1])
+    return {"workload": line["config"]["workload"], "value": line["value"], "unit": line["unit"],
+            "ms_per_step": line["ms_per_step"], "stages_ms": line["stages_ms"],
+            "stage_roofline_frac": line["stage_roofline_frac"], "clocks": line["clocks"],
+            "stage_bounds": {"prune": "hbm", "rf": "hbm (effective bytes)", "score": "alu (FP32 peak)",
+                             "topq": "hbm"}}
 
 
 def sources_sha(stage):
@@ -182,14 +290,21 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(loaded)}
 
 
-def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None, kernel=0, warp=False):
-    """Time the oracle on n_sample candidates of the workload in a fresh process
-    (with mace_kappa set: the MACE round, UCB coefficient mace_kappa; acq
-    overrides the workload's acquisition)."""
-    env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
-               MKL_NUM_THREADS=str(threads))
+def _oracle_code(name, seed, n_sample, mace_kappa=None, acq=None, kernel=0, warp=False, start_at=None):
+    """Python source that times the oracle's round on n_sample candidates of
+    the workload (same round state) and prints {"seconds": t}: prune, forest,
+    posterior, acquisition and top-q; for the fantasy workload the q
+    sequential picks with refits; with mace_kappa the MACE round."""
+    from workloads import WORKLOADS
+    w = WORKLOADS[name]
     gp_opts = "kernel=%d, warp=%s" % (kernel, "warp_params(%r, %d)" % (name, seed) if warp else "None")
-    if mace_kappa is None:
+    if w.fantasy:
+        select = ("feas = oracle.prune_mask(inst.space, inst.clauses, inst.cand, inst.n_cand)\n"
+                  "v = oracle.rf_votes(inst.nodes, inst.tree_offset, inst.space, inst.cand, inst.n_cand)\n"
+                  "w = inst.workload\n"
+                  "feas &= oracle.pof_feasible(v, inst.n_trees, w.leaf_scale, w.delta_num, w.delta_den)\n"
+                  "oracle.fantasy_picks(inst, w.q, feas, kernel=%d)\n" % kernel)
+    elif mace_kappa is None:
         select = ("r = oracle.score_round(inst, %s, %s)\n" % (repr(acq) if acq else "inst.workload.acq", gp_opts) +
                   "oracle.select_topq(r['acq'], r['feasible'], inst.workload.q)\n")
     else:
@@ -198,29 +313,89 @@ def cpu_oracle_sample(name, seed, n_sample, threads=1, mace_kappa=None, acq=None
                   "1e-4, %r)\n"
                   "A[:, ~r['feasible']] = -np.inf\n"
                   "oracle.mace_select(A, r['feasible'], inst.workload.q, 0)\n" % float(mace_kappa))
-    code = (
-        "import sys, time, json; sys.path.insert(0, %r)\n"
-        "import numpy as np, oracle\n"
-        "from workloads import make_instance, warp_params\n"
-        "inst = make_instance(%r, %d, n_cand=%d)\n"
-        "t = time.perf_counter()\n" % (ROOT, name, seed, n_sample)
-        + select
-        + "print(json.dumps({'seconds': time.perf_counter() - t}))\n")
-    p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=900)
+    return ("import sys, time, json; sys.path.insert(0, %r)\n"
+            "import numpy as np, oracle\n"
+            "from workloads import make_instance, warp_params\n"
+            "inst = make_instance(%r, %d, n_cand=%d)\n"
+            "time.sleep(max(0.0, %r - time.time()))\n"
+            "t = time.perf_counter()\n" % (ROOT, name, seed, n_sample, float(start_at or 0.0))
+            + select
+            + "print(json.dumps({'seconds': time.perf_counter() - t}))\n")
+
+
+def _one_thread_env():
+    return dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+
+
+def cpu_oracle_sample(name, seed, n_sample, mace_kappa=None, acq=None, kernel=0, warp=False, wall=False):
+    """Seconds of the oracle's round on n_sample candidates, one thread, in a
+    fresh process (with wall: also the process's whole wall time)."""
+    code = _oracle_code(name, seed, n_sample, mace_kappa, acq, kernel, warp)
+    t0 = time.perf_counter()
+    p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=_one_thread_env(),
+                       timeout=900)
     if p.returncode != 0:
         raise RuntimeError(p.stderr[-2000:])
-    return json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
+    secs = json.loads(p.stdout.strip().splitlines()[-1])["seconds"]
+    return (secs, time.perf_counter() - t0) if wall else secs
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_oracle_all_cores(name, seed, n_sample, procs, startup_s, **opts):
+    """The oracle's round on n_sample candidates in each of `procs`
+    one-thread processes at once (every core busy): the processes start
+    their timers together, after their set-up; returns the slowest one's
+    seconds (the throughput is procs * n_sample / seconds)."""
+    code = _oracle_code(name, seed, n_sample, start_at=time.time() + 2.0 * startup_s + 2.0, **opts)
+    ps = [subprocess.Popen([sys.executable, "-c", code], stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True,
+                           env=_one_thread_env()) for _ in range(procs)]
+    secs = []
+    for p in ps:
+        out, err = p.communicate(timeout=1800)
+        if p.returncode != 0:
+            raise RuntimeError(err[-2000:])
+        secs.append(json.loads(out.strip().splitlines()[-1])["seconds"])
+    return max(secs)
 
 
 def calibrate_sample(name, seed, budget_s, mace_kappa=None, acq=None, kernel=0, warp=False):
-    """Largest sample whose oracle round fits the budget (scaled from a probe)."""
-    probe = 64
-    t = cpu_oracle_sample(name, seed, probe, mace_kappa=mace_kappa, acq=acq, kernel=kernel, warp=warp)
-    per = max(t / probe, 1e-6)
-    return max(16, int(budget_s / per))
+    """Largest sample whose oracle round fits the budget (scaled from two
+    probes), and the set-up seconds of one oracle process."""
+    opts = dict(mace_kappa=mace_kappa, acq=acq, kernel=kernel, warp=warp)
+    t1, w1 = cpu_oracle_sample(name, seed, 32, wall=True, **opts)
+    t2 = cpu_oracle_sample(name, seed, 96, **opts)
+    per = max((t2 - t1) / 64, 1e-6)
+    fixed = max(t1 - 32 * per, 0.0)
+    return max(16, int((budget_s - fixed) / per)), max(w1 - t1, 0.0)
+
+
+def cpu_baseline_line(name, seed, budget_s, unit, **opts):
+    """cpu_baseline: the oracle on a bounded sample of the workload, on one
+    core and on every core of the host (one process per core)."""
+    sample, startup = calibrate_sample(name, seed, budget_s, **opts)
+    t1 = cpu_oracle_sample(name, seed, sample, **opts)
+    procs = host_cores()
+    tn = cpu_oracle_all_cores(name, seed, sample, procs, startup, **opts)
+    from workloads import WORKLOADS
+    what = ("prune, forest, then the q sequential EHVI picks with a GP refit per pick"
+            if WORKLOADS[name].fantasy else "all five steps")
+    return {"value": procs * sample / tn, "unit": unit, "cores": procs, "kind": "oracle",
+            "value_one_core": sample / t1,
+            "sample": f"{sample} candidates of the {name} pool (same round state) per process, {what}; "
+                      f"fp64 numpy, one thread per process, {procs} processes at once (one core: "
+                      f"{sample / t1:.4g} {unit})"}
 
 
 def run_reference(args):
+    """The reference arm: the oracle itself (the paper ships no code), each
+    step a bounded sample of the workload on every host core (one one-thread
+    process per core, timers started together)."""
     from workloads import WORKLOADS, seeds
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -234,22 +409,26 @@ def run_reference(args):
     acq = "ehvi-exact" if args.acq == "ehvi-exact" else None
     kern = 1 if args.kernel == "matern32" else 0
     opts = dict(mace_kappa=kappa, acq=acq, kernel=kern, warp=args.warp)
-    per_step = max(0.05, 120.0 / max(1, args.steps + args.warmup))
-    sample = calibrate_sample(w.name, seed, per_step, kappa, acq, kern, args.warp)
+    procs = host_cores()
+    per_step = max(0.05, 100.0 / max(1, args.steps + args.warmup))
+    sample, startup = calibrate_sample(w.name, seed, per_step, **opts)
     for _ in range(args.warmup):
-        cpu_oracle_sample(w.name, seed, sample, **opts)
-    times = [cpu_oracle_sample(w.name, seed, sample, **opts) for _ in range(args.steps)]
+        cpu_oracle_all_cores(w.name, seed, sample, procs, startup, **opts)
+    times = [cpu_oracle_all_cores(w.name, seed, sample, procs, startup, **opts) for _ in range(args.steps)]
     ms = 1e3 * statistics.mean(times)
-    value = sample / (ms / 1e3)
+    value = procs * sample / (ms / 1e3)
+    what = ("prune, forest, then the q sequential EHVI picks with a GP refit per pick" if w.fantasy
+            else "all five steps")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(w, {"reference": "fp64 CPU oracle (the paper ships no code)",
-                                          "sample_per_step": sample, "kernel": args.kernel,
+                                          "sample_per_step": procs * sample, "kernel": args.kernel,
                                           "warp": bool(args.warp)},
                                       acq=None if args.acq == "default" else args.acq),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"{sample} candidates of the {w.name} pool per step, all five steps"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": procs, "kind": "oracle",
+                             "sample": f"{sample} candidates of the {w.name} pool per process and step, {what}; "
+                                       f"{procs} one-thread processes at once"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -665,7 +844,7 @@ def main():
     if acq_kind == "ehvi-exact" and (w.n_obj < 2 or w.fantasy):
         raise SystemExit("--acq ehvi-exact needs a multi-objective workload without fantasies")
     seed = seeds(w.name)[0]
-    inst = make_instance(w.name, seed)
+    inst = make_instance(w.name, seed, n_cand=args.pool)
     cand_np = inst.cand
     if rank > 0:  # each rank scores a pool of its own; the round state is shared
         cand_np = draw_configs(w, Stream(seed, f"pool-rank{rank}"), inst.n_cand, inst.ld)
@@ -756,9 +935,16 @@ def main():
     # Per-stage times from eagerly launched steps (diagnostic; they feed the roofline).
     n_diag = min(args.steps, 50)
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n_diag)]
+    phases = []  # the fantasy call's launches, timed by the library with events on the stream
+    if inp.fantasy:
+        S.scoot_ctx_set_timing(ctx, True)
     for kk in range(n_diag):
         flush.fill_(kk & 0xFF)
         step(evs[kk])
+        if inp.fantasy:
+            phases.append(S.scoot_ctx_phase_times(ctx))
+    if inp.fantasy:
+        S.scoot_ctx_set_timing(ctx, False)
     torch.cuda.synchronize(device)
     stage_names = ["prune", "rf", "score", "pareto" if inp.acq == "mace" else "topq"]
     stage_ms = {s: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, s in enumerate(stage_names)}
@@ -809,35 +995,74 @@ def main():
         step_ms = float(t.item())
     value = world * N / (step_ms / 1e3)
 
-    # roofline of the dominant stage
+    # roofline of the dominant kernel
     peaks, peak_src = measured_peaks()
     sms = torch.cuda.get_device_properties(device).multi_processor_count
     fp32_peak = sms * FP32_LANES_PER_SM * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # TFLOP/s
+    hbm = peaks["hbm_gbs"]
     work = work_model(inst, st.n_boxes, inp.acq, getattr(st, "n_grid", None))
-    dom = max(stage_names, key=lambda s: stage_ms[s])
-    kind, per_cand = work[dom]
-    units = n_feasible if dom == "score" else N
-    launch_s = stage_ms[dom] / 1e3
-    tr = TRAFFIC.get((dom, w.name if inp.acq == w.acq else f"{w.name}/{inp.acq}"))
-    traffic = tr["bytes"] if tr and tr["sha"] == sources_sha(dom) else None
-    if kind == "hbm":
-        achieved = per_cand * units / launch_s / 1e9
-        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / peaks["hbm_gbs"], "traffic": traffic}
+    n_known = int(rnd.n_known.item())
+
+    def hbm_roof(bytes_per_launch, launch_ms, name):
+        a = bytes_per_launch / (launch_ms / 1e3) / 1e9
+        return {"bound": "hbm", "achieved": a, "peak": hbm, "unit": "GB/s", "frac": a / hbm, "kernel": name,
+                "work_per_launch": bytes_per_launch, "launch_ms": launch_ms}
+
+    def alu_roof(flops_per_launch, launch_ms, name):
+        a = flops_per_launch / (launch_ms / 1e3) / 1e12
+        return {"bound": "alu", "achieved": a, "peak": fp32_peak, "unit": "TFLOP/s", "frac": a / fp32_peak,
+                "kernel": name, "work_per_launch": flops_per_launch, "launch_ms": launch_ms}
+    kernels = {}
+    for s_ in ("prune", "rf"):
+        k_, pc = work[s_]
+        kernels[s_] = hbm_roof(pc * N, stage_ms[s_], s_)
+    if inp.fantasy:
+        def mean_of(kind):
+            v = [sum(ms for k, ms in ph if k == kind) for ph in phases]
+            c = [sum(1 for k, _ in ph if k == kind) for ph in phases]
+            return statistics.mean(v), max(1, c[0])
+        post_ms, _ = mean_of("posterior")
+        pass_ms, n_pass = mean_of("fant_pass")
+        pick_ms, n_pick = mean_of("fant_pick")
+        init_ms, _ = mean_of("fant_init")
+        kernels["posterior"] = alu_roof(posterior_flops(inst) * n_feasible, post_ms, "posterior (whitened rows)")
+        pb = fantasy_pass_bytes(inst, inp.q, n_feasible)[:n_pass]
+        kernels["fant_pass"] = hbm_roof(statistics.mean(pb), pass_ms / n_pass, "fant_pass")
+        kernels["fant_pass"]["launches_per_step"] = n_pass
+        kernel_ms = {"prune": stage_ms["prune"], "rf": stage_ms["rf"], "posterior": post_ms,
+                     "fant_pass": pass_ms, "fant_pick": pick_ms + init_ms}
     else:
-        achieved = per_cand * units / launch_s / 1e12
-        roof = {"bound": "alu", "achieved": achieved, "peak": fp32_peak, "unit": "TFLOP/s",
-                "frac": achieved / fp32_peak, "traffic": traffic}
-    roof.update({"kernel": dom, "peak_source": f"{peak_src}; FP32 = SMs x 128 lanes x 2 x max SM clock",
-                 "work_per_unit": per_cand, "units_per_launch": units})
-    stage_roofs = {}
-    for s in stage_names:
-        k_, pc = work[s]
-        u = n_feasible if s == "score" else N
-        if k_ == "hbm":
-            stage_roofs[s] = round(pc * u / (stage_ms[s] / 1e3) / 1e9 / peaks["hbm_gbs"], 4)
-        else:
-            stage_roofs[s] = round(pc * u / (stage_ms[s] / 1e3) / 1e12 / fp32_peak, 4)
+        k_, pc = work["score"]
+        kernels["score"] = alu_roof(pc * n_feasible, stage_ms["score"], "score")
+        last = "pareto" if inp.acq == "mace" else "topq"
+        kernels[last] = hbm_roof(work[last][1] * N, stage_ms[last], last)
+        kernel_ms = {k: stage_ms[k] for k in stage_names}
+    dom = max((k for k in kernels), key=lambda k: kernel_ms[k] if k in kernel_ms else 0.0)
+    roof = dict(kernels[dom])
+    tr = TRAFFIC.get((dom, w.name if inp.acq == w.acq else f"{w.name}/{inp.acq}"))
+    roof["traffic"] = tr["bytes"] if tr and tr["sha"] == sources_sha(tr.get("stage", dom)) else None
+    roof["peak_source"] = (f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if roof["bound"] == "hbm" else
+                           "FP32 = SMs x 128 lanes x 2 x max SM clock (nominal; measured FFMA peaks in probes)")
+    stage_roofs = {k: round(v["frac"], 4) for k, v in kernels.items()}
+    probes = None
+    if not args.no_extra and rank == 0:
+        probes = measure_probes(S, ctx, device, stream, sms)
+        for k, v in kernels.items():
+            if v["bound"] == "alu":
+                v["frac_of_measured_ffma2"] = v["achieved"] / max(probes["ffma_tflops"], probes["ffma2_tflops"])
+        # the forest's true bound: node visits against the shared-memory gather peak
+        st_ = Stream(seed, "visit-sample")
+        mask_k = torch.empty(N, dtype=torch.uint8, device=device)
+        S.scoot_prune(ctx, inp.space, inp.clauses, cand, N, mask_k, None, stream)
+        known = np.nonzero(mask_k.cpu().numpy())[0]
+        samp = known[(st_.u64(4096) % np.uint64(max(1, len(known)))).astype(np.int64)] if len(known) else known
+        visits = forest_visits(inst, samp) * n_known
+        rate = visits / (stage_ms["rf"] / 1e3)
+        kernels["rf"].update({"node_visits_per_launch": visits, "node_visits_per_s": rate,
+                              "frac_of_smem_gather_peak": rate / probes["smem_gather_visits_per_s"]})
+        if inp.fantasy:
+            kernels["fant_pass"]["ehvi_flops_per_launch"] = n_feasible * inp.eps.shape[0] * st.n_boxes * 4 * inst.n_obj
+        roof = dict(kernels[dom], traffic=roof["traffic"], peak_source=roof["peak_source"])
 
     # end to end through the C ABI from pinned host buffers
     e2e = None
@@ -918,11 +1143,11 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         kappa = rnd.kappa if inp.acq == "mace" else None
         acq = "ehvi-exact" if inp.acq == "ehvi-exact" else None
-        sample = calibrate_sample(w.name, seed, args.cpu_seconds, kappa, acq, inp.kernel, args.warp)
-        secs = cpu_oracle_sample(w.name, seed, sample, mace_kappa=kappa, acq=acq, kernel=inp.kernel, warp=args.warp)
-        cpu = {"value": sample / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"{sample} candidates of the {w.name} pool (same round state), all five steps, "
-                         f"fp64 numpy, one thread"}
+        cpu = cpu_baseline_line(w.name, seed, args.cpu_seconds, UNIT, mace_kappa=kappa, acq=acq, kernel=inp.kernel,
+                                warp=args.warp)
+    extra = None
+    if rank == 0 and world == 1 and not args.no_extra:
+        extra = {name: sub_run(name) for name in SUBRUN_WORKLOADS if name != w.name}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -935,11 +1160,13 @@ def main():
                                               "eager_ms_per_step": round(eager_ms, 5),
                                               "kernel": args.kernel, "warp": bool(args.warp),
                                               "e2e_gp_state": "built on the device" if gp_dev else
-                                              "built on the host"}, acq=inp.acq),
+                                              "built on the host"}, acq=inp.acq, pool=N),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps * rnd.kernels_per_round(),
                 "clocks": clocks, "stages_ms": {k: round(v, 5) for k, v in stage_ms.items()},
-                "stage_roofline_frac": stage_roofs}
+                "kernels_ms": {k: round(v, 5) for k, v in kernel_ms.items()},
+                "stage_roofline_frac": stage_roofs, "kernels": kernels, "peaks_measured_here": probes,
+                "at_2_20": extra}
         print(json.dumps(line), flush=True)
     ctx.close()
     if dist:

@@ -137,6 +137,24 @@ scoot_status scoot_ctx_check(scoot_ctx* ctx, void* stream);
 /* Bytes of device workspace the context currently holds. */
 scoot_status scoot_ctx_workspace_bytes(const scoot_ctx* ctx, int64_t* bytes);
 
+/* Phase timing, a measurement aid (off by default).  With enable != 0 the
+ * calls that launch several kinds of kernel (scoot_suggest_fantasy) record a
+ * CUDA event on their stream before their first launch and after each
+ * launch, up to SCOOT_MAX_MARKS launches per call; scoot_ctx_phase_times
+ * waits for the last timed call's events and returns, per launch in order,
+ * its kind (SCOOT_PHASE_*) in h_kind and its milliseconds in h_ms (at most
+ * cap entries; *count = the number of timed launches).  Leave it off for
+ * calls captured in a CUDA graph. */
+#define SCOOT_MAX_MARKS          256
+#define SCOOT_PHASE_COMPACT        0   /* compaction of the live candidates */
+#define SCOOT_PHASE_POSTERIOR      1   /* posterior with the whitened rows V */
+#define SCOOT_PHASE_FANT_INIT      2   /* the observations' front and boxes */
+#define SCOOT_PHASE_FANT_PASS      3   /* a pick's pass: downdate, EHVI, block argmax */
+#define SCOOT_PHASE_FANT_PICK      4   /* a pick's fp64 terms, front and boxes */
+#define SCOOT_PHASE_SCATTER        5   /* variances scattered to var_out */
+scoot_status scoot_ctx_set_timing(scoot_ctx* ctx, int32_t enable);
+scoot_status scoot_ctx_phase_times(scoot_ctx* ctx, int32_t cap, int32_t* h_kind, float* h_ms, int32_t* count);
+
 /* ------------------------------------------------------------------ 1. prune, Eq. (2) */
 
 /* mask[i] = 1 when candidate i satisfies every clause of h_clauses, else 0
@@ -500,6 +518,23 @@ scoot_status scoot_sobol_configs(scoot_ctx* ctx, const scoot_param* h_space, int
 scoot_status scoot_first_feasible(scoot_ctx* ctx, const uint8_t* mask, int64_t n, int32_t need, int64_t* idx,
                                   int32_t* count, void* stream);
 
+/* beta_t, the UCB coefficient of tuning iteration t >= 1 (Section 4.5):
+ * beta_t = 2 log(t^2 pi^2 / (6 delta)) with delta = 1 / t^2, taken as the
+ * factor of sigma in UCB = mu + beta sigma, as printed (the kappa argument
+ * of scoot_acq_mace / scoot_score_mace).  Host, synchronous. */
+scoot_status scoot_ucb_beta(int32_t t, double* beta);
+
+/* The observed objectives as the GP models them: per objective m,
+ * h_y_std[m][i] = (h_y[m][i] - mean_m) / sd_m over the n observations
+ * (population standard deviation, floored at 1e-12), computed in fp64
+ * (Section 4.3 fits zero-mean GPs; the loop standardises before each fit).
+ * If h_ref is not NULL, h_ref[m] = min_i h_y_std[m][i] - ref_margin: a
+ * reference point below every observation (the loop's reading of the
+ * default configuration's objectives, Section 4.5).  h_y, h_y_std [n_obj][n]
+ * host; SCOOT_EINVAL on a non-finite value.  Host, synchronous. */
+scoot_status scoot_standardize(const float* h_y, int32_t n_obj, int32_t n, float* h_y_std, float* h_ref,
+                               float ref_margin);
+
 /* Algorithm 1's feasibility-threshold controller after k suggestions were
  * evaluated (host): if any result was invalid, Delta becomes
  * min(0.75, max(0.5, Delta + 0.05)) and the count of feasible suggestions
@@ -606,6 +641,49 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* layout
                                    void* work, int64_t work_bytes, int64_t* idx, float* val, int32_t* count,
                                    float* var_out, void* stream);
 
+/* The same picks over a pool sharded across ranks (one process per GPU,
+ * each holding a contiguous share of the candidates and the same GP and
+ * fantasy states), as phase calls with one exchange per pick:
+ *   scoot_fantasy_begin       compaction of the shard's live candidates, their
+ *                             posterior and whitened rows, the observations'
+ *                             front and boxes; opens the context's session
+ *                             (global index of the shard's candidate 0:
+ *                             index_offset; index_offset + n < 2^32);
+ *   for j = 0 .. q-1:
+ *     scoot_fantasy_local_best   pass j over the shard (the downdate of pick
+ *                             j-1, EHVI, the argmax) into rec (device uint64
+ *                             [SCOOT_FANT_REC], may be NULL): rec[0] the
+ *                             selection key of the shard's best candidate
+ *                             (order-preserving bits of its fp32 EHVI value
+ *                             << 32 | 0xFFFFFFFF - global index; 0 when the
+ *                             shard has no eligible candidate), rec[1 ..] its
+ *                             d configuration words, two per element (word
+ *                             2k in the low half);
+ *     (the caller gathers every rank's record into one device array)
+ *     scoot_fantasy_commit    recs: n_rec gathered records (device
+ *                             [n_rec][SCOOT_FANT_REC]); the one with the
+ *                             largest key is pick j (value descending, global
+ *                             index ascending); every rank records it in idx,
+ *                             val and count, computes its rank-1 terms from
+ *                             the configuration in the record (so no rank
+ *                             needs another rank's pool) and rebuilds the
+ *                             boxes; the rank holding it excludes it;
+ *   scoot_fantasy_end         variances to var_out (may be NULL; the shard's
+ *                             [M][n]) and closes the session.
+ * Every rank's picks are identical to those of one rank holding the whole
+ * pool.  scoot_suggest_fantasy is this sequence on one rank (n_rec = 1).  A
+ * context holds one session; no other call on it may come between begin and
+ * end (they share its workspace).  All calls are asynchronous on `stream`. */
+#define SCOOT_FANT_REC 9
+scoot_status scoot_fantasy_begin(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
+                                 const void* fant_state, int32_t box_cap, const uint32_t* cand, int64_t n,
+                                 int64_t ld, const uint8_t* mask, int64_t index_offset, const float* eps,
+                                 int32_t n_mc, int32_t q, void* work, int64_t work_bytes, int64_t* idx, float* val,
+                                 int32_t* count, void* stream);
+scoot_status scoot_fantasy_local_best(scoot_ctx* ctx, int32_t j, uint64_t* rec, void* stream);
+scoot_status scoot_fantasy_commit(scoot_ctx* ctx, int32_t j, const uint64_t* recs, int32_t n_rec, void* stream);
+scoot_status scoot_fantasy_end(scoot_ctx* ctx, float* var_out, void* stream);
+
 /* ------------------------------------------------------------------ 7. MACE (Sections 4.5 and 4.7) */
 
 /* Candidates that may survive the pivot stage of scoot_select_pareto (see
@@ -680,6 +758,23 @@ scoot_status scoot_select_pareto(scoot_ctx* ctx, const float* acq, int64_t lda, 
  * (there is no context, so no message). */
 scoot_status scoot_select_topq_static(const float* acq, const uint8_t* mask, int64_t n, int32_t q,
                                       int64_t* idx, float* val, int32_t* count, void* stream);
+
+/* ------------------------------------------------------------------ measurement probes */
+
+/* Peaks the library's kernels are reported against where no vendor figure
+ * applies (the paper has no counterpart; these are measurement aids).
+ * scoot_probe_fma: `blocks` blocks of 256 threads, each thread running 16
+ * independent fp32 FMA chains for `iters` steps, as scalar FFMAs (packed = 0)
+ * or as packed pairs (packed = 1): 2 * 16 * 256 * blocks * iters flops.
+ * scoot_probe_gather: `blocks` blocks of 256 threads, each thread taking
+ * `steps` dependent steps through a binary tree of n_nodes 8-byte nodes
+ * (scoot_node) in shared memory, as a forest walk does (1 <= n_nodes <=
+ * 12288): 256 * blocks * steps node visits.  sink: device float [blocks]
+ * (receives nothing in practice; it keeps the work live).  Asynchronous. */
+scoot_status scoot_probe_fma(scoot_ctx* ctx, int32_t packed, int32_t blocks, int32_t iters, float* sink,
+                             void* stream);
+scoot_status scoot_probe_gather(scoot_ctx* ctx, int32_t n_nodes, int32_t blocks, int32_t steps, float* sink,
+                                void* stream);
 
 #ifdef __cplusplus
 }

@@ -40,15 +40,18 @@ using namespace scoot_dev;
 constexpr int kPassThreads = 256;
 constexpr int kPickThreads = 256;
 constexpr int kPartMax = 2048;   // per-block argmax partials of one pass
+constexpr int kPickRows = 8;     // row blocks per objective of the pick's L^{-1} k product
 
 // Control words of one call, in the work buffer.
 struct Ctrl {
     uint32_t done;      // 1 once the loop has stopped (no eligible candidate left, or an error)
-    uint32_t arrived;   // fant_pick blocks that finished their objective (the last resets it)
+    uint32_t arrived;   // objectives whose pick terms are final (the last one resets it)
+    uint32_t arrived_m[SCOOT_MAX_OBJ];  // row blocks of objective m done (its last one resets it)
+    uint32_t passed;    // blocks of the current pass done (the last one resets it)
     int32_t n_boxes;
     int32_t n_front;
-    int64_t pick_idx;   // candidate index of the latest pick
-    int64_t pick_pos;   // its list position
+    int32_t local_pos;  // list position of this shard's best candidate of the current pass (-1: none)
+    uint64_t local_key; // its selection key (global index)
 };
 
 struct FantArgs {
@@ -60,6 +63,7 @@ struct FantArgs {
     const float* V;               // [M][n_pad][ldc]
     float* C;                     // [q][M][ldc] downdate factors c_l of every candidate
     int32_t n_obs, n_pad, d, kernel, q, n_mc, box_cap, front_cap;
+    int64_t index_offset;         // global index of this shard's candidate 0 (selection keys, picks)
     const char* gp;               // GP state blob (fp32; feature order)
     int64_t off_fmap, off_ils, off_scal;
     const char* fant;             // fantasy state (fp64; parameter order)
@@ -68,7 +72,6 @@ struct FantArgs {
     const float* eps;             // [S][M]
     float* box_lo;                // [box_cap][M]
     float* box_hi;
-    double* cell;                 // [box_cap] floor of each grid cell (box builder scratch)
     double* front;                // [front_cap][M]
     Ctrl* ctrl;
     int64_t* picked_pos;          // [q]
@@ -82,6 +85,9 @@ struct FantArgs {
     double* mupick;               // [q][M] fantasised values
     uint64_t* part_key;           // [kPartMax]
     int32_t* part_pos;
+    int32_t n_part;               // blocks of a pass
+    uint64_t* rec;                // [SCOOT_FANT_REC] this shard's record of the current pass
+    uint32_t* pick_words;         // [16] configuration of the latest pick (from the winning record)
     int64_t* out_idx;             // [q]
     float* out_val;               // [q]
     int32_t* out_count;
@@ -135,22 +141,6 @@ __device__ __forceinline__ double matern64(double r, int kernel) {
     return (1.0 + a + a * a / 3.0) * exp(-a);
 }
 
-// k(a, b) of one objective in fp64: ordinal coordinates scaled by 1/l,
-// categorical mismatches weigh 1/l^2 (the covariance of Section 4.3).
-__device__ __forceinline__ double cov64(const double* ua, const double* ub, const double* sp, const double* ell,
-                                        int d, double sf2, int kernel) {
-    double r2 = 0.0;
-    for (int c = 0; c < d; ++c) {
-        if ((int)sp[c * 4] == SCOOT_CATEGORICAL) {
-            if (ua[c] != ub[c]) r2 += 1.0 / (ell[c] * ell[c]);
-        } else {
-            const double t = (ua[c] - ub[c]) / ell[c];
-            r2 += t * t;
-        }
-    }
-    return sf2 * matern64(sqrt(r2), kernel);
-}
-
 // Feature coordinate (fp64) of a stored word of parameter c: log scale for
 // integer log-uniform, linear for integer uniform and continuous, the index
 // for categoricals.  Returns false for a word that has no feature.
@@ -173,8 +163,8 @@ __device__ __forceinline__ bool feature64(const double* sp, int c, uint32_t w, d
 
 // Shared-memory need of front_update_and_boxes (bytes).
 __host__ __device__ inline size_t boxes_smem(int front_cap, int M, int box_cap) {
-    return (size_t)front_cap * M * 8 + (size_t)(M - 1) * (front_cap + 1) * 8 + (size_t)(front_cap + 1) * 4 +
-           (size_t)(box_cap + 1) * 4 + 64;
+    return (size_t)box_cap * 8 + (size_t)front_cap * M * 8 + (size_t)(M - 1) * (front_cap + 1) * 8 +
+           (size_t)(front_cap + 1) * 4 + (size_t)(box_cap + 1) * 4 + 64;
 }
 
 // One block: optionally adds point z (fp64 of the fp32 fantasised value) to
@@ -192,7 +182,8 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
                                        char* smem) {
     constexpr int G = M - 1;
     const int fcap = a.front_cap;
-    double* F = reinterpret_cast<double*>(smem);                  // [fcap][M]
+    double* cell = reinterpret_cast<double*>(smem);               // [box_cap] floor of each grid cell
+    double* F = cell + a.box_cap;                                  // [fcap][M]
     double* axis = F + (size_t)fcap * M;                           // [G][fcap + 1]
     int32_t* first = reinterpret_cast<int32_t*>(axis + (size_t)G * (fcap + 1));  // [fcap + 1]
     int32_t* rowcnt = first + fcap + 1;                                            // [rows + 1]
@@ -287,13 +278,13 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
             for (int j = 0; j < G; ++j) dom &= F[k * M + j] >= up[j];
             if (dom) hh = fmax(hh, F[k * M + M - 1]);
         }
-        a.cell[c] = fmax(h.ref[M - 1], hh);
+        cell[c] = fmax(h.ref[M - 1], hh);
     }
     __syncthreads();
     // Boxes per row (cells merged while the floor repeats), then their offsets.
     for (int r = tid; r < rows; r += blockDim.x) {
         int cnt = 1;
-        for (int kk = 1; kk < A_last; ++kk) cnt += a.cell[r * A_last + kk] != a.cell[r * A_last + kk - 1];
+        for (int kk = 1; kk < A_last; ++kk) cnt += cell[r * A_last + kk] != cell[r * A_last + kk - 1];
         rowcnt[r + 1] = cnt;
     }
     __syncthreads();
@@ -316,9 +307,9 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
         int b = rowcnt[r] - 1;
         const double* al = axis + (G - 1) * (fcap + 1);
         for (int kk = 0; kk < A_last; ++kk) {
-            const double fl = a.cell[r * A_last + kk];
+            const double fl = cell[r * A_last + kk];
             const double upl = kk + 1 < A_last ? al[kk + 1] : inf;
-            if (kk == 0 || fl != a.cell[r * A_last + kk - 1]) {
+            if (kk == 0 || fl != cell[r * A_last + kk - 1]) {
                 ++b;
                 for (int j = 0; j < G - 1; ++j) {
                     a.box_lo[b * M + j] = (float)lo_pre[j];
@@ -344,6 +335,44 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
     }
 }
 
+// ---------------------------------------------------------------- records
+
+// The last block of a pass to finish reduces the per-block partials to this
+// shard's record: the selection key of its best candidate (global index)
+// and that candidate's d configuration words, two per 64-bit word (word 2k
+// in the low half); key 0 when the shard has no eligible candidate left.
+__device__ void pass_record(const FantArgs& a) {
+    __shared__ int s_last;
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(&a.ctrl->passed, 1u) == gridDim.x - 1;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    uint64_t best = 0ull;
+    int32_t pos = -1;
+    for (int k = threadIdx.x; k < (int)gridDim.x; k += blockDim.x)
+        keymax(best, pos, __ldcg(a.part_key + k), __ldcg(a.part_pos + k));
+    block_keymax(best, pos);
+    if (threadIdx.x == 0) {
+        a.ctrl->passed = 0u;
+        a.ctrl->local_key = best;
+        a.ctrl->local_pos = best != 0ull ? pos : -1;
+        a.rec[0] = best;
+    }
+    if (threadIdx.x < (SCOOT_FANT_REC - 1)) {
+        uint64_t w = 0ull;
+        if (best != 0ull) {
+            const int64_t i = a.list ? (int64_t)a.list[pos] : (int64_t)pos;
+            const int c0 = 2 * threadIdx.x, c1 = c0 + 1;
+            const uint32_t lo = c0 < a.d ? __ldg(a.cand + (int64_t)c0 * a.ld + i) : 0u;
+            const uint32_t hi = c1 < a.d ? __ldg(a.cand + (int64_t)c1 * a.ld + i) : 0u;
+            w = (uint64_t)lo | ((uint64_t)hi << 32);
+        }
+        a.rec[1 + threadIdx.x] = w;
+    }
+}
+
 // ---------------------------------------------------------------- kernels
 
 // One block: checks the fantasy state against the call, resets the control
@@ -360,6 +389,10 @@ __global__ void __launch_bounds__(kPickThreads) fant_init(const __grid_constant_
         for (int m = 0; m < M; ++m) ok &= gscal[m * 4 + 3] == 0.0f;  // an unwarped GP state
         a.ctrl->done = ok ? 0u : 1u;
         a.ctrl->arrived = 0u;
+        for (int m = 0; m < SCOOT_MAX_OBJ; ++m) a.ctrl->arrived_m[m] = 0u;
+        a.ctrl->passed = 0u;
+        a.ctrl->local_key = 0ull;
+        a.ctrl->local_pos = -1;
         a.ctrl->n_boxes = 0;
         a.ctrl->n_front = ok ? h.front0 : 0;
         *a.out_count = 0;
@@ -381,7 +414,9 @@ __global__ void __launch_bounds__(kPickThreads) fant_init(const __grid_constant_
 // j - 1, then EHVI over the current boxes with the picks excluded, and each
 // block's best (key, list position).
 template <int M>
-__global__ void __launch_bounds__(kPassThreads) fant_pass(const __grid_constant__ FantArgs a, int j) {
+__global__ void __launch_bounds__(kPassThreads, M == 2 ? 4 : 1) fant_pass(const __grid_constant__ FantArgs a, int j) {
+    // Two objectives fit 64 registers without spills: four blocks (32 warps)
+    // per SM keep more rows of V in flight.
     if (*(volatile const uint32_t*)&a.ctrl->done) {
         if (threadIdx.x == 0) a.part_key[blockIdx.x] = 0ull;
         return;
@@ -392,7 +427,7 @@ __global__ void __launch_bounds__(kPassThreads) fant_pass(const __grid_constant_
     float4* bhi = blo + nb;
     float4* epsv = bhi + nb;
     int64_t* pk = reinterpret_cast<int64_t*>(epsv + a.n_mc);  // [q] list positions of the picks
-    float* vps = reinterpret_cast<float*>(pk + a.q);          // [M][n_pad]
+    float* vps = reinterpret_cast<float*>(pk + ((a.q + 1) & ~1));  // [M][n_pad] (16-byte aligned)
     float* cxs = vps + M * a.n_pad;                           // [M][q]
     float* ins = cxs + M * a.q;                               // [M]
     float* ups = ins + M;                                     // [d] features of the latest pick (feature order)
@@ -401,15 +436,13 @@ __global__ void __launch_bounds__(kPassThreads) fant_pass(const __grid_constant_
     const float* gscal = reinterpret_cast<const float*>(a.gp + a.off_scal);
     stage_boxes(a.box_lo, a.box_hi, nb, a.eps, a.n_mc, M, blo, bhi, epsv);
     const int l = j - 1;  // the downdate of this pass
-    int64_t p = 0;
     if (l >= 0) {
-        p = a.ctrl->pick_idx;
         for (int e = threadIdx.x; e < M * a.n_pad; e += blockDim.x) vps[e] = a.vp[e];
         for (int e = threadIdx.x; e < M * a.q; e += blockDim.x) cxs[e] = a.cxp[e];
         if (threadIdx.x < M) ins[threadIdx.x] = a.inv_s[threadIdx.x];
         for (int c = threadIdx.x; c < a.d; c += blockDim.x) {
             const float4 f = fm[c];
-            ups[c] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + p), (int)f.x, f.y, f.z);
+            ups[c] = feature_of(a.pick_words[(int)f.w], (int)f.x, f.y, f.z);
         }
     }
     for (int e = threadIdx.x; e < j; e += blockDim.x) pk[e] = a.picked_pos[e];
@@ -450,19 +483,24 @@ __global__ void __launch_bounds__(kPassThreads) fant_pass(const __grid_constant_
 #pragma unroll
             for (int m = 0; m < M; ++m) {
                 const float k = gscal[m * 4] * matern(sqrtf(r2[m]), a.kernel);
-                const float* vrow = a.V + (int64_t)m * a.n_pad * a.ldc + pos;
-                const float* vpm = vps + m * a.n_pad;
-                float d0 = 0.0f, d1 = 0.0f;
-                int row = 0;
+                // v(x) . v_p over float4 groups of four rows (16-byte loads;
+                // rows past n_obs are zero on both sides).
+                const float4* vrow = reinterpret_cast<const float4*>(a.V) + (int64_t)m * (a.n_pad / 4) * a.ldc + pos;
+                const float4* vpm = reinterpret_cast<const float4*>(vps + m * a.n_pad);
+                const int groups = (a.n_obs + 3) / 4;
+                float d0 = 0.0f, d1 = 0.0f, d2 = 0.0f, d3 = 0.0f;
 #pragma unroll 8
-                for (; row + 1 < a.n_obs; row += 2) {
-                    d0 = fmaf(vrow[(int64_t)row * a.ldc], vpm[row], d0);
-                    d1 = fmaf(vrow[(int64_t)(row + 1) * a.ldc], vpm[row + 1], d1);
+                for (int g = 0; g < groups; ++g) {
+                    const float4 v = __ldcs(vrow + (int64_t)g * a.ldc);
+                    const float4 w = vpm[g];
+                    d0 = fmaf(v.x, w.x, d0);
+                    d1 = fmaf(v.y, w.y, d1);
+                    d2 = fmaf(v.z, w.z, d2);
+                    d3 = fmaf(v.w, w.w, d3);
                 }
-                if (row < a.n_obs) d0 = fmaf(vrow[(int64_t)row * a.ldc], vpm[row], d0);
                 float cc = 0.0f;
                 for (int t = 0; t < l; ++t) cc = fmaf(a.C[((int64_t)t * M + m) * a.ldc + pos], cxs[m * a.q + t], cc);
-                const float c = (k - (d0 + d1) - cc) * ins[m];
+                const float c = (k - ((d0 + d1) + (d2 + d3)) - cc) * ins[m];
                 if (l < a.q - 2) a.C[((int64_t)l * M + m) * a.ldc + pos] = c;  // read by later downdates
                 float* vv = a.var + (int64_t)m * a.ldc + pos;
                 vr[m] = fmaxf(*vv - c * c, 0.0f);
@@ -483,51 +521,77 @@ __global__ void __launch_bounds__(kPassThreads) fant_pass(const __grid_constant_
         }
         const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, nb, epsv, a.n_mc, 0, 1) * inv_mc
                              : ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
-        if (!(v != v) && v != -INFINITY) keymax(best, best_pos, make_key(v, (uint32_t)i), (int32_t)pos);
+        if (!(v != v) && v != -INFINITY)
+            keymax(best, best_pos, make_key(v, (uint32_t)(a.index_offset + i)), (int32_t)pos);
     }
     block_keymax(best, best_pos);
     if (threadIdx.x == 0) {
         a.part_key[blockIdx.x] = best;
         a.part_pos[blockIdx.x] = best_pos;
     }
+    pass_record(a);
 }
 
-// Pick j: the argmax of the pass's partials (every block); block 0 records
-// the pick; block m then computes objective m's rank-1 terms of the pick in
-// fp64; the last block to finish adds the fantasised point to the front and
-// rebuilds the boxes for the next pass.
+// First row of slice r of R slices of the rows of a lower triangle of order
+// n with equal areas (row i holds i + 1 entries).
+__device__ __forceinline__ int tri_row(int r, int R, int n) {
+    if (r <= 0) return 0;
+    if (r >= R) return n;
+    return min(n, (int)ceil(sqrt((double)r / R) * n));
+}
+
+// Pick j, on a grid of kPickRows x M blocks.  Every block reduces the pass's
+// partials to the argmax; block (0, 0) records the pick.  Block (r, m) then
+// computes slice r of v_p = L^{-1} k(X, x_p) of objective m in fp64 (and,
+// for r = 0, mu(x_p)).  The last slice of objective m to finish completes
+// that objective's terms (|v_p|^2, v_p . v_{p_t}, the c_t(x_p) recurrence,
+// s_j) and the fp32 copies the next pass reads; the last objective to finish
+// adds the fantasised point to the front and rebuilds the boxes.
 template <int M>
-__global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant__ FantArgs a, int j, int n_part) {
+__global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant__ FantArgs a, int j,
+                                                          const uint64_t* recs, int n_rec) {
     extern __shared__ __align__(16) char smem[];
     if (*(volatile const uint32_t*)&a.ctrl->done) return;
     const FantHeader& h = *reinterpret_cast<const FantHeader*>(a.fant);
-    const int tid = threadIdx.x, m = blockIdx.x;
-    uint64_t best = 0ull;
-    int32_t bpos = -1;
-    for (int k = tid; k < n_part; k += blockDim.x) keymax(best, bpos, a.part_key[k], a.part_pos[k]);
-    block_keymax(best, bpos);
+    const int tid = threadIdx.x, r = blockIdx.x, m = blockIdx.y, R = gridDim.x;
+    // The winning record: the largest selection key over the shards.
     __shared__ uint64_t s_best;
-    __shared__ int32_t s_pos;
+    __shared__ int32_t s_win;
+    __shared__ uint32_t s_words[16];
     if (tid == 0) {
+        uint64_t best = 0ull;
+        int win = -1;
+        for (int k = 0; k < n_rec; ++k) {
+            const uint64_t key = __ldcg(recs + (size_t)k * SCOOT_FANT_REC);
+            if (key > best) {
+                best = key;
+                win = k;
+            }
+        }
         s_best = best;
-        s_pos = bpos;
+        s_win = win;
     }
     __syncthreads();
-    best = s_best;
-    bpos = s_pos;
-    if (best == 0ull) {  // no eligible candidate left: the picks end here
-        if (m == 0 && tid == 0) a.ctrl->done = 1u;
+    const uint64_t best = s_best;
+    const bool lead = r == 0 && m == 0;
+    if (best == 0ull) {  // no eligible candidate left on any shard: the picks end here
+        if (lead && tid == 0) a.ctrl->done = 1u;
         return;
     }
+    if (tid < 16) {
+        const uint64_t w = __ldcg(recs + (size_t)s_win * SCOOT_FANT_REC + 1 + tid / 2);
+        s_words[tid] = (tid & 1) ? (uint32_t)(w >> 32) : (uint32_t)w;
+    }
+    __syncthreads();
     const int64_t p = key_index(best);
-    if (m == 0 && tid == 0) {
+    if (lead && tid == 0) {
+        const bool owner = a.ctrl->local_key == best;  // this shard holds the pick
         a.out_idx[j] = p;
         a.out_val[j] = key_value(best);
         *a.out_count = j + 1;
-        a.picked_pos[j] = bpos;
-        a.ctrl->pick_idx = p;
-        a.ctrl->pick_pos = bpos;
+        a.picked_pos[j] = owner ? a.ctrl->local_pos : -1;
     }
+    if (lead && tid < a.d) a.pick_words[tid] = s_words[tid];
     if (j + 1 >= a.q) return;  // no later pick needs this one's fantasy
     const int n = a.n_obs, d = a.d, q = a.q;
     const double* sp = reinterpret_cast<const double*>(a.fant + h.off_space);
@@ -537,18 +601,18 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
     const double* Li = reinterpret_cast<const double*>(a.fant + h.off_linv) + (size_t)m * n * n;
     const double sf2 = h.sf2[m], tau2 = h.tau2[m];
     double* u = reinterpret_cast<double*>(smem);     // [16] features of the pick
-    double* ks = u + 16;                              // [n] k(X, x_p)
-    double* vv = ks + n;                              // [n] v_p
-    double* D = vv + n;                               // [q] v_p . v_{p_t}
-    double* red = D + q;                              // [32] reduction scratch
-    __shared__ int s_bad;
+    double* il = u + 16;                              // [16] 1/l (ordinal) or 1/l^2 (categorical)
+    double* ks = il + 16;                             // [n] k(X, x_p)
+    double* red = ks + n;                             // [32] reduction scratch
+    __shared__ int s_bad, s_last;
     if (tid == 0) s_bad = 0;
     __syncthreads();
     if (tid < d) {
         double x = 0.0;
-        if (!feature64(sp, tid, __ldg(a.cand + (int64_t)tid * a.ld + p), &x)) s_bad = 1;
+        if (!feature64(sp, tid, s_words[tid], &x)) s_bad = 1;
         u[tid] = x;
-        if (m == 0) a.upick[(size_t)j * d + tid] = x;
+        il[tid] = (int)sp[tid * 4] == SCOOT_CATEGORICAL ? 1.0 / (ell[tid] * ell[tid]) : 1.0 / ell[tid];
+        if (lead) a.upick[(size_t)j * d + tid] = x;
     }
     __syncthreads();
     if (s_bad) {
@@ -558,15 +622,28 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         }
         return;
     }
+    // k(x_p, X_i), fp64: ordinal coordinates times 1/l, categorical mismatches 1/l^2.
+    auto cov = [&](const double* ub) {
+        double r2 = 0.0;
+        for (int c = 0; c < d; ++c) {
+            if ((int)sp[c * 4] == SCOOT_CATEGORICAL) {
+                r2 += u[c] != ub[c] ? il[c] : 0.0;
+            } else {
+                const double t = (u[c] - ub[c]) * il[c];
+                r2 = fma(t, t, r2);
+            }
+        }
+        return sf2 * matern64(sqrt(r2), a.kernel);
+    };
+    const int i0 = tri_row(r, R, n), i1 = tri_row(r + 1, R, n);
     double mu_part = 0.0;
-    for (int i = tid; i < n; i += blockDim.x) {
-        ks[i] = cov64(u, uo + (size_t)i * d, sp, ell, d, sf2, a.kernel);
-        mu_part += ks[i] * alpha[i];
+    for (int i = tid; i < (r == 0 ? n : i1); i += blockDim.x) {
+        ks[i] = cov(uo + (size_t)i * d);
+        if (r == 0) mu_part = fma(ks[i], alpha[i], mu_part);
     }
-    __syncthreads();
-    // v_p = L^{-1} k*: row i reads column-major L^{-1} (coalesced across rows).
-    double vv_part = 0.0;
-    for (int i = tid; i < n; i += blockDim.x) {
+    const double mu = block_sum(mu_part, red);  // (its barriers also publish ks)
+    double* vrow = a.vpick + ((size_t)j * M + m) * n;
+    for (int i = i0 + tid; i < i1; i += blockDim.x) {
         double s0 = 0.0, s1 = 0.0;
         int c = 0;
         for (; c + 1 <= i; c += 2) {
@@ -574,14 +651,39 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
             s1 = fma(Li[(size_t)(c + 1) * n + i], ks[c + 1], s1);
         }
         if (c <= i) s0 = fma(Li[(size_t)c * n + i], ks[c], s0);
-        const double v = s0 + s1;
-        vv[i] = v;
-        a.vpick[((size_t)j * M + m) * n + i] = v;
-        vv_part += v * v;
+        vrow[i] = s0 + s1;
     }
-    const double mu = block_sum(mu_part, red);
-    const double vnorm = block_sum(vv_part, red);   // (its barriers also publish vv)
-    // Dots with the earlier picks' rows: warp w takes picks w, w + 8, ...
+    if (r == 0 && tid == 0) a.mupick[(size_t)j * M + m] = mu;
+    // The last slice of objective m completes its terms.
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) s_last = atomicAdd(&a.ctrl->arrived_m[m], 1u) == (unsigned)(R - 1);
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    if (tid == 0) a.ctrl->arrived_m[m] = 0u;
+    double* vv = ks;            // [n] v_p, read back from the slices
+    double* D = ks + n;         // [q] v_p . v_{p_t}
+    double* kpt = D + q;        // [q] k(x_p, x_{p_t})
+    double* red2 = kpt + q;     // [32]
+    double* Ct = red2 + 32;     // [q][q] c_k(x_{p_t}) of the earlier picks
+    double* st = Ct + q * q;    // [q] their s
+    double* cj = st + q;        // [q] this pick's c_t(x_p)
+    for (int e = tid; e < j * j; e += blockDim.x) {
+        const int t = e / j, k = e - t * j;
+        Ct[e] = k < t ? a.cpick[((size_t)t * M + m) * q + k] : 0.0;
+    }
+    for (int t = tid; t < j; t += blockDim.x) st[t] = a.spick[(size_t)t * M + m];
+    double vv_part = 0.0;
+    for (int i = tid; i < n; i += blockDim.x) {
+        const double v = __ldcg(vrow + i);
+        vv[i] = v;
+        vv_part = fma(v, v, vv_part);
+        a.vp[m * a.n_pad + i] = (float)v;
+    }
+    for (int i = n + tid; i < a.n_pad; i += blockDim.x) a.vp[m * a.n_pad + i] = 0.0f;
+    for (int t = tid; t < j; t += blockDim.x) kpt[t] = cov(a.upick + (size_t)t * d);
+    const double vnorm = block_sum(vv_part, red2);  // (its barriers also publish vv and kpt)
     {
         const int lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
         for (int t = warp; t < j; t += nw) {
@@ -593,28 +695,26 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         }
     }
     __syncthreads();
-    if (tid == 0) {
+    if (tid == 0) {  // the recurrence over the earlier picks, in shared memory
         double var = sf2 - vnorm;
-        double* cj = a.cpick + ((size_t)j * M + m) * q;
         for (int t = 0; t < j; ++t) {
-            const double* ct = a.cpick + ((size_t)t * M + m) * q;
-            double num = cov64(u, a.upick + (size_t)t * d, sp, ell, d, sf2, a.kernel) - D[t];
-            for (int r = 0; r < t; ++r) num -= cj[r] * ct[r];
-            const double st = a.spick[(size_t)t * M + m];
-            cj[t] = st > 0.0 ? num / st : 0.0;
+            double num = kpt[t] - D[t];
+            for (int k = 0; k < t; ++k) num -= cj[k] * Ct[t * j + k];
+            cj[t] = st[t] > 0.0 ? num / st[t] : 0.0;
             var -= cj[t] * cj[t];
         }
         const double s = sqrt(fmax(var, 0.0) + tau2);
         a.spick[(size_t)j * M + m] = s;
-        a.mupick[(size_t)j * M + m] = mu;
         a.inv_s[m] = s > 0.0 ? (float)(1.0 / s) : 0.0f;
-        for (int t = 0; t < q; ++t) a.cxp[m * q + t] = t < j ? (float)cj[t] : 0.0f;
     }
-    for (int i = tid; i < a.n_pad; i += blockDim.x) a.vp[m * a.n_pad + i] = i < n ? (float)vv[i] : 0.0f;
-    // The last block to get here adds the fantasised point and rebuilds the boxes.
+    __syncthreads();
+    for (int t = tid; t < q; t += blockDim.x) {
+        if (t < j) a.cpick[((size_t)j * M + m) * q + t] = cj[t];
+        a.cxp[m * q + t] = t < j ? (float)cj[t] : 0.0f;
+    }
+    // The last objective adds the fantasised point and rebuilds the boxes.
     __threadfence();
     __syncthreads();
-    __shared__ int s_last;
     if (tid == 0) s_last = atomicAdd(&a.ctrl->arrived, 1u) == (unsigned)(M - 1);
     __syncthreads();
     if (!s_last) return;
@@ -622,7 +722,7 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
     if (tid == 0) a.ctrl->arrived = 0u;
     double z[M];
 #pragma unroll
-    for (int k = 0; k < M; ++k) z[k] = (double)(float)(*(volatile const double*)&a.mupick[(size_t)j * M + k]);
+    for (int k = 0; k < M; ++k) z[k] = (double)(float)__ldcg(a.mupick + (size_t)j * M + k);
     front_update_and_boxes<M>(a, h, true, z, smem);
 }
 
@@ -641,7 +741,7 @@ scatter_var(const int32_t* list, const unsigned int* n_list, int64_t n, int64_t 
 
 struct WorkLayout {
     int64_t mean, var, V, C, ctrl, picked, vp, cxp, inv_s, upick, vpick, cpick, spick, mupick, front, box_lo,
-        box_hi, cell, part_key, part_pos, bytes;
+        box_hi, part_key, part_pos, rec, words, bytes;
 };
 
 int64_t up256(int64_t x) { return (x + 255) / 256 * 256; }
@@ -668,9 +768,10 @@ WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q, int box_cap) 
     w.front = o;    o = up256(o + fcap * M * 8);
     w.box_lo = o;   o = up256(o + (int64_t)box_cap * M * 4);
     w.box_hi = o;   o = up256(o + (int64_t)box_cap * M * 4);
-    w.cell = o;     o = up256(o + (int64_t)box_cap * 8);
     w.part_key = o; o = up256(o + kPartMax * 8);
     w.part_pos = o; o = up256(o + kPartMax * 4);
+    w.rec = o;      o = up256(o + SCOOT_FANT_REC * 8);
+    w.words = o;    o = up256(o + 16 * 4);
     w.bytes = o;
     return w;
 }
@@ -681,34 +782,36 @@ int sm_count(int device) {
     return v > 0 ? v : 1;
 }
 
+// An open session of sequential picks: the kernels' arguments and launch shapes.
+struct Session {
+    FantArgs a;
+    int M;
+    int64_t n;
+    unsigned blocks;
+    size_t pass_smem, pick_smem;
+};
+
 template <int M>
-scoot_status run_picks(scoot_ctx* ctx, FantArgs a, int64_t n, cudaStream_t st) {
-    const size_t pass_smem = (size_t)(2 * a.box_cap + a.n_mc) * 16 + (size_t)a.q * 8 + (size_t)M * a.n_pad * 4 +
-                             (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4;
-    const size_t pick_smem = std::max((size_t)(16 + 2 * a.n_obs + a.q + 32) * 8,
-                                      boxes_smem(a.front_cap, M, a.box_cap));
+scoot_status set_attributes(scoot_ctx* ctx, Session& ss) {
+    const FantArgs& a = ss.a;
+    ss.pass_smem = (size_t)(2 * a.box_cap + a.n_mc) * 16 + (size_t)((a.q + 1) & ~1) * 8 + (size_t)M * a.n_pad * 4 +
+                   (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4;
+    ss.pick_smem = std::max((size_t)(32 + a.n_obs + a.q * a.q + 4 * a.q + 64) * 8,
+                            boxes_smem(a.front_cap, M, a.box_cap));
     int max_smem = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
-    if (pass_smem > (size_t)max_smem || pick_smem > (size_t)max_smem)
+    if (ss.pass_smem > (size_t)max_smem || ss.pick_smem > (size_t)max_smem)
         return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "%d boxes and %d samples exceed the shared memory of a block",
                           a.box_cap, a.n_mc);
-    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_pass<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pass_smem));
-    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_pick<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pick_smem));
-    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_init<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pick_smem));
-    fant_init<M><<<1, kPickThreads, pick_smem, st>>>(a);
-    SCOOT_LAUNCHED(ctx);
-    // Enough blocks for many loads in flight per SM; the live count is read on the device.
-    int64_t blocks = (n + kPassThreads - 1) / kPassThreads;
-    const int64_t cap = std::min<int64_t>((int64_t)sm_count(ctx->device) * 8, kPartMax);
-    if (blocks > cap) blocks = cap;
-    if (blocks < 1) blocks = 1;
-    for (int j = 0; j < a.q; ++j) {
-        fant_pass<M><<<(unsigned)blocks, kPassThreads, pass_smem, st>>>(a, j);
-        SCOOT_LAUNCHED(ctx);
-        fant_pick<M><<<M, kPickThreads, pick_smem, st>>>(a, j, (int)blocks);
-        SCOOT_LAUNCHED(ctx);
-    }
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_pass<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ss.pass_smem));
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_pick<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ss.pick_smem));
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(fant_init<M>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ss.pick_smem));
     return SCOOT_OK;
+}
+
+Session* session_of(scoot_ctx* ctx) {
+    return ctx->fant_session.size() == sizeof(Session) ? reinterpret_cast<Session*>(ctx->fant_session.data())
+                                                        : nullptr;
 }
 
 }  // namespace
@@ -723,13 +826,13 @@ scoot_status scoot_fantasy_work_bytes(const scoot_gp_layout* L, int64_t n, int32
     return SCOOT_OK;
 }
 
-scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
-                                   const void* fant_state, int32_t box_cap, const uint32_t* cand, int64_t n,
-                                   int64_t ld, const uint8_t* mask, const float* eps, int32_t n_mc, int32_t q,
-                                   void* work, int64_t work_bytes, int64_t* idx, float* val, int32_t* count,
-                                   float* var_out, void* stream) {
+scoot_status scoot_fantasy_begin(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state, const void* fant_state,
+                                 int32_t box_cap, const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
+                                 int64_t index_offset, const float* eps, int32_t n_mc, int32_t q, void* work,
+                                 int64_t work_bytes, int64_t* idx, float* val, int32_t* count, void* stream) {
     scoot_status s = scoot_enter(ctx);
     if (s != SCOOT_OK) return s;
+    ctx->fant_session.clear();
     if (!L || !state || !fant_state || !eps || !idx || !val || !count || !work)
         return scoot_fail(ctx, SCOOT_EINVAL, "a required pointer is NULL");
     if (!scoot_gp_layout_valid(L))
@@ -742,6 +845,8 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
         return scoot_fail(ctx, SCOOT_EINVAL, "box_cap = %d outside 1..%d", box_cap, kFantBoxMax);
     if ((s = scoot_check_pool(ctx, cand, n, ld, L->d)) != SCOOT_OK) return s;
     if (n > 0x7FFFFFFFll) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "n >= 2^31");
+    if (index_offset < 0 || index_offset + n > 0xFFFFFFFFll)
+        return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "global indices must lie below 2^32");
     const WorkLayout w = work_layout(L, n, q, box_cap);
     if (work_bytes < w.bytes)
         return scoot_fail(ctx, SCOOT_EINVAL, "work buffer of %lld bytes, %lld needed", (long long)work_bytes, (long long)w.bytes);
@@ -750,15 +855,19 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
         return scoot_fail(ctx, SCOOT_EINVAL, "fant_state is not 256-byte aligned");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     char* wk = static_cast<char*>(work);
-    FantArgs a;
-    std::memset(&a, 0, sizeof(a));
+    Session ss;
+    std::memset(&ss, 0, sizeof(ss));
+    FantArgs& a = ss.a;
     a.n = n;
     a.ldc = n > 0 ? n : 1;
+    a.index_offset = index_offset;
+    if ((s = scoot_marks_begin(ctx, st)) != SCOOT_OK) return s;
     if (mask && n > 0) {
         ScootList lst;
         if ((s = scoot_compact(ctx, mask, n, nullptr, 0u, st, &lst)) != SCOOT_OK) return s;
         a.list = lst.list;
         a.n_list = lst.count;
+        if ((s = scoot_mark(ctx, st, SCOOT_PHASE_COMPACT)) != SCOOT_OK) return s;
     }
     a.mean = reinterpret_cast<float*>(wk + w.mean);
     a.var = reinterpret_cast<float*>(wk + w.var);
@@ -782,7 +891,6 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
     a.eps = eps;
     a.box_lo = reinterpret_cast<float*>(wk + w.box_lo);
     a.box_hi = reinterpret_cast<float*>(wk + w.box_hi);
-    a.cell = reinterpret_cast<double*>(wk + w.cell);
     a.front = reinterpret_cast<double*>(wk + w.front);
     a.ctrl = reinterpret_cast<Ctrl*>(wk + w.ctrl);
     a.picked_pos = reinterpret_cast<int64_t*>(wk + w.picked);
@@ -796,6 +904,8 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
     a.mupick = reinterpret_cast<double*>(wk + w.mupick);
     a.part_key = reinterpret_cast<uint64_t*>(wk + w.part_key);
     a.part_pos = reinterpret_cast<int32_t*>(wk + w.part_pos);
+    a.rec = reinterpret_cast<uint64_t*>(wk + w.rec);
+    a.pick_words = reinterpret_cast<uint32_t*>(wk + w.words);
     a.out_idx = idx;
     a.out_val = val;
     a.out_count = count;
@@ -804,20 +914,101 @@ scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, con
         s = scoot_posterior_whitened(ctx, L, state, cand, n, ld, a.list, a.n_list, reinterpret_cast<float*>(wk + w.mean),
                                      a.var, reinterpret_cast<float*>(wk + w.V), a.ldc, st);
         if (s != SCOOT_OK) return s;
+        if ((s = scoot_mark(ctx, st, SCOOT_PHASE_POSTERIOR)) != SCOOT_OK) return s;
     }
+    ss.M = M;
+    ss.n = n;
+    // Enough blocks for many loads in flight per SM; the live count is read on the device.
+    int64_t blocks = (n + kPassThreads - 1) / kPassThreads;
+    const int64_t cap = std::min<int64_t>((int64_t)sm_count(ctx->device) * 8, kPartMax);
+    ss.blocks = (unsigned)std::max<int64_t>(1, std::min(blocks, cap));
     switch (M) {
-    case 2: s = run_picks<2>(ctx, a, n, st); break;
-    case 3: s = run_picks<3>(ctx, a, n, st); break;
-    default: s = run_picks<4>(ctx, a, n, st); break;
+    case 2: s = set_attributes<2>(ctx, ss); break;
+    case 3: s = set_attributes<3>(ctx, ss); break;
+    default: s = set_attributes<4>(ctx, ss); break;
     }
     if (s != SCOOT_OK) return s;
-    if (var_out && n > 0) {
-        int64_t blocks = (n + kPassThreads - 1) / kPassThreads;
-        if (blocks > (int64_t)sm_count(ctx->device) * 8) blocks = (int64_t)sm_count(ctx->device) * 8;
-        scatter_var<<<(unsigned)blocks, kPassThreads, 0, st>>>(a.list, a.n_list, n, a.ldc, M, a.var, var_out, n);
-        SCOOT_LAUNCHED(ctx);
+    switch (M) {
+    case 2: fant_init<2><<<1, kPickThreads, ss.pick_smem, st>>>(a); break;
+    case 3: fant_init<3><<<1, kPickThreads, ss.pick_smem, st>>>(a); break;
+    default: fant_init<4><<<1, kPickThreads, ss.pick_smem, st>>>(a); break;
     }
+    SCOOT_LAUNCHED(ctx);
+    if ((s = scoot_mark(ctx, st, SCOOT_PHASE_FANT_INIT)) != SCOOT_OK) return s;
+    ctx->fant_session.resize(sizeof(Session));
+    std::memcpy(ctx->fant_session.data(), &ss, sizeof(Session));
     return SCOOT_OK;
+}
+
+scoot_status scoot_fantasy_local_best(scoot_ctx* ctx, int32_t j, uint64_t* rec, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    Session* ss = session_of(ctx);
+    if (!ss) return scoot_fail(ctx, SCOOT_EINVAL, "no open fantasy session (scoot_fantasy_begin)");
+    if (j < 0 || j >= ss->a.q) return scoot_fail(ctx, SCOOT_EINVAL, "pick %d outside 0..%d", j, ss->a.q - 1);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    switch (ss->M) {
+    case 2: fant_pass<2><<<ss->blocks, kPassThreads, ss->pass_smem, st>>>(ss->a, j); break;
+    case 3: fant_pass<3><<<ss->blocks, kPassThreads, ss->pass_smem, st>>>(ss->a, j); break;
+    default: fant_pass<4><<<ss->blocks, kPassThreads, ss->pass_smem, st>>>(ss->a, j); break;
+    }
+    SCOOT_LAUNCHED(ctx);
+    if ((s = scoot_mark(ctx, st, SCOOT_PHASE_FANT_PASS)) != SCOOT_OK) return s;
+    if (rec)
+        SCOOT_CUDA(ctx, cudaMemcpyAsync(rec, ss->a.rec, SCOOT_FANT_REC * sizeof(uint64_t), cudaMemcpyDeviceToDevice, st));
+    return SCOOT_OK;
+}
+
+scoot_status scoot_fantasy_commit(scoot_ctx* ctx, int32_t j, const uint64_t* recs, int32_t n_rec, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    Session* ss = session_of(ctx);
+    if (!ss) return scoot_fail(ctx, SCOOT_EINVAL, "no open fantasy session (scoot_fantasy_begin)");
+    if (j < 0 || j >= ss->a.q) return scoot_fail(ctx, SCOOT_EINVAL, "pick %d outside 0..%d", j, ss->a.q - 1);
+    if (!recs || n_rec < 1) return scoot_fail(ctx, SCOOT_EINVAL, "no records");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const dim3 grid(kPickRows, ss->M);
+    switch (ss->M) {
+    case 2: fant_pick<2><<<grid, kPickThreads, ss->pick_smem, st>>>(ss->a, j, recs, n_rec); break;
+    case 3: fant_pick<3><<<grid, kPickThreads, ss->pick_smem, st>>>(ss->a, j, recs, n_rec); break;
+    default: fant_pick<4><<<grid, kPickThreads, ss->pick_smem, st>>>(ss->a, j, recs, n_rec); break;
+    }
+    SCOOT_LAUNCHED(ctx);
+    return scoot_mark(ctx, st, SCOOT_PHASE_FANT_PICK);
+}
+
+scoot_status scoot_fantasy_end(scoot_ctx* ctx, float* var_out, void* stream) {
+    scoot_status s = scoot_enter(ctx);
+    if (s != SCOOT_OK) return s;
+    Session* ss = session_of(ctx);
+    if (!ss) return scoot_fail(ctx, SCOOT_EINVAL, "no open fantasy session (scoot_fantasy_begin)");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (var_out && ss->n > 0) {
+        int64_t blocks = (ss->n + kPassThreads - 1) / kPassThreads;
+        if (blocks > (int64_t)sm_count(ctx->device) * 8) blocks = (int64_t)sm_count(ctx->device) * 8;
+        scatter_var<<<(unsigned)blocks, kPassThreads, 0, st>>>(ss->a.list, ss->a.n_list, ss->n, ss->a.ldc, ss->M,
+                                                               ss->a.var, var_out, ss->n);
+        SCOOT_LAUNCHED(ctx);
+        if ((s = scoot_mark(ctx, st, SCOOT_PHASE_SCATTER)) != SCOOT_OK) return s;
+    }
+    ctx->fant_session.clear();
+    return SCOOT_OK;
+}
+
+scoot_status scoot_suggest_fantasy(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
+                                   const void* fant_state, int32_t box_cap, const uint32_t* cand, int64_t n,
+                                   int64_t ld, const uint8_t* mask, const float* eps, int32_t n_mc, int32_t q,
+                                   void* work, int64_t work_bytes, int64_t* idx, float* val, int32_t* count,
+                                   float* var_out, void* stream) {
+    scoot_status s = scoot_fantasy_begin(ctx, L, state, fant_state, box_cap, cand, n, ld, mask, 0, eps, n_mc, q, work,
+                                         work_bytes, idx, val, count, stream);
+    if (s != SCOOT_OK) return s;
+    const uint64_t* rec = session_of(ctx)->a.rec;
+    for (int j = 0; j < q; ++j) {
+        if ((s = scoot_fantasy_local_best(ctx, j, nullptr, stream)) != SCOOT_OK) return s;
+        if ((s = scoot_fantasy_commit(ctx, j, rec, 1, stream)) != SCOOT_OK) return s;
+    }
+    return scoot_fantasy_end(ctx, var_out, stream);
 }
 
 }  // extern "C"

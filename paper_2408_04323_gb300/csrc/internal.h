@@ -26,6 +26,14 @@ struct scoot_ctx {
     void* ws = nullptr;          // device workspace (grown on demand)
     size_t ws_bytes = 0;
     uint32_t* d_err = nullptr;   // device error word
+    // Phase timing (scoot_ctx_set_timing): events recorded between the
+    // launches of the last timed call, and the kind of each launch.
+    int32_t timing = 0;
+    std::vector<void*> events;   // cudaEvent_t, created on first use
+    std::vector<int32_t> mark_kind;
+    // The open session of sequential fantasised picks (scoot_fantasy_begin
+    // .. scoot_fantasy_end), opaque to everything but fantasy.cu.
+    std::vector<char> fant_session;
 };
 
 scoot_status scoot_fail(scoot_ctx* ctx, scoot_status s, const char* fmt, ...);
@@ -111,6 +119,12 @@ scoot_status scoot_fant_header(const scoot_param* h_space, const scoot_gp_layout
 // Consistency of a GP layout's offsets with its own sizes.
 bool scoot_gp_layout_valid(const scoot_gp_layout* L);
 
+// Phase timing: scoot_marks_begin records the first event of a call on
+// stream st, scoot_mark one event after each launch of kind `kind` (no-ops
+// unless timing is enabled).  Kinds are listed in include/scoot.h.
+scoot_status scoot_marks_begin(scoot_ctx* ctx, void* st);
+scoot_status scoot_mark(scoot_ctx* ctx, void* st, int32_t kind);
+
 // Checks shared by the device entry points.
 scoot_status scoot_check_pool(scoot_ctx* ctx, const uint32_t* cand, int64_t n, int64_t ld, int32_t d);
 
@@ -127,8 +141,10 @@ scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint3
                            cudaStream_t st, ScootList* out, int fill_rows = 1, int64_t fill_ld = 0);
 
 // Posterior of the listed candidates into list-position order: mean and var
-// [M][ldc], and the whitened rows V = L^{-1} k(X, x) [M][n_rb * 64][ldc]
-// (rows >= n left unwritten).  ldc >= the list length.
+// [M][ldc], and the whitened rows V = L^{-1} k(X, x) in float4 groups of four
+// rows, [M][n_rb * 16][ldc][4] (16-byte aligned; groups wholly past row n
+// left unwritten, rows past n inside a written group zero).  ldc >= the list
+// length.
 scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
                                       const uint32_t* cand, int64_t n, int64_t ld, const int32_t* list,
                                       const unsigned int* n_list, float* mean, float* var, float* V, int64_t ldc,

@@ -31,42 +31,85 @@ __device__ __forceinline__ void add_count(unsigned long long* count, uint32_t mi
     }
 }
 
-// One thread per candidate: every clause is evaluated with exact integer
-// sums, int64 when the host has shown that no clause sum can overflow it
-// (sum of |coef| < 2^32 with 32-bit values), else int128; column reads are
-// coalesced 4-byte loads (repeated columns hit L1).  One candidate per thread
-// keeps enough warps in flight to cover the load latency even for pools of a
-// few hundred thousand candidates.
+// Four consecutive candidates per thread: each clause column is read as one
+// 16-byte vector (columns are 16-byte aligned and ld % 4 == 0, so the vector
+// at i0 = 4k stays inside the column even for the last, ragged group), every
+// guard and term of every clause is loaded without a branch on the guards
+// (repeated columns hit L1) so all loads of a group are in flight together,
+// the clause sums are exact (int64 when the host has shown that no clause sum
+// can overflow it, i.e. sum of |coef| < 2^32 with 32-bit values, else int128),
+// and the four mask bytes are stored as one 32-bit word (bytes of a ragged
+// tail, or of a mask that is not 4-byte aligned, one by one).
+template <bool kExact64>
+__device__ __forceinline__ void clause_sums(const scoot_clause& C, const uint32_t* __restrict__ cand, int64_t ld,
+                                            int64_t i0, bool (&ok)[4]) {
+    bool g[4] = {true, true, true, true};
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        if (k < C.n_guard) {
+            const uint4 v = __ldg(reinterpret_cast<const uint4*>(cand + (int64_t)C.guard_param[k] * ld + i0));
+            const int32_t want = C.guard_value[k];
+            g[0] &= (int32_t)v.x == want;
+            g[1] &= (int32_t)v.y == want;
+            g[2] &= (int32_t)v.z == want;
+            g[3] &= (int32_t)v.w == want;
+        }
+    }
+    if (kExact64) {
+        int64_t sum[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            if (t < C.n_term) {
+                const uint4 v = __ldg(reinterpret_cast<const uint4*>(cand + (int64_t)C.term_param[t] * ld + i0));
+                const int64_t a = C.coef[t];
+                sum[0] += a * (int64_t)(int32_t)v.x;
+                sum[1] += a * (int64_t)(int32_t)v.y;
+                sum[2] += a * (int64_t)(int32_t)v.z;
+                sum[3] += a * (int64_t)(int32_t)v.w;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) ok[e] &= !g[e] || sum[e] >= C.rhs;
+    } else {
+        __int128 sum[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            if (t < C.n_term) {
+                const uint4 v = __ldg(reinterpret_cast<const uint4*>(cand + (int64_t)C.term_param[t] * ld + i0));
+                const __int128 a = C.coef[t];
+                sum[0] += a * (int32_t)v.x;
+                sum[1] += a * (int32_t)v.y;
+                sum[2] += a * (int32_t)v.z;
+                sum[3] += a * (int32_t)v.w;
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) ok[e] &= !g[e] || sum[e] >= (__int128)C.rhs;
+    }
+}
+
 template <bool kExact64>
 __global__ void __launch_bounds__(kPruneThreads)
 prune_kernel(const __grid_constant__ PruneArgs a, const uint32_t* __restrict__ cand, int64_t n,
-             int64_t ld, uint8_t* __restrict__ mask, unsigned long long* count) {
+             int64_t ld, uint8_t* __restrict__ mask, unsigned long long* count, int mask_aligned) {
     uint32_t feasible = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        bool ok = true;
-        for (int c = 0; c < a.n_clauses; ++c) {
-            const scoot_clause& C = a.cl[c];
-            bool g = true;
-#pragma unroll
-            for (int k = 0; k < 2; ++k)
-                if (k < C.n_guard) g &= (int32_t)__ldg(cand + (int64_t)C.guard_param[k] * ld + i) == C.guard_value[k];
-            if (!g) continue;
-            if (kExact64) {
-                int64_t sum = 0;
-#pragma unroll
-                for (int t = 0; t < 4; ++t)
-                    if (t < C.n_term) sum += C.coef[t] * (int64_t)(int32_t)__ldg(cand + (int64_t)C.term_param[t] * ld + i);
-                ok &= sum >= C.rhs;
-            } else {
-                __int128 sum = 0;
-#pragma unroll
-                for (int t = 0; t < 4; ++t)
-                    if (t < C.n_term) sum += (__int128)C.coef[t] * (int32_t)__ldg(cand + (int64_t)C.term_param[t] * ld + i);
-                ok &= sum >= (__int128)C.rhs;
+    const int64_t groups = (n + 3) / 4;
+    for (int64_t gi = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < groups;
+         gi += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i0 = 4 * gi;
+        bool ok[4] = {true, true, true, true};
+        for (int c = 0; c < a.n_clauses; ++c) clause_sums<kExact64>(a.cl[c], cand, ld, i0, ok);
+        if (i0 + 4 <= n && mask_aligned) {
+            const uint32_t word = (uint32_t)ok[0] | ((uint32_t)ok[1] << 8) | ((uint32_t)ok[2] << 16) |
+                                  ((uint32_t)ok[3] << 24);
+            *reinterpret_cast<uint32_t*>(mask + i0) = word;
+            feasible += (uint32_t)ok[0] + ok[1] + ok[2] + ok[3];
+        } else {
+            for (int e = 0; e < 4 && i0 + e < n; ++e) {
+                mask[i0 + e] = ok[e];
+                feasible += ok[e];
             }
         }
-        mask[i] = ok;
-        feasible += ok;
     }
     if (count) add_count(count, feasible);
 }
@@ -91,9 +134,9 @@ struct RfArgs {
 
 // Persistent blocks of 256 threads score tiles of 32 candidates: lane l of
 // warp g serves candidate slot l and walks trees g, g + 8, g + 16, ... of the
-// forest, so the 32 lanes of a warp walk the same tree for 32 candidates
-// (the upper levels are broadcast loads) and each candidate has eight
-// independent walks in flight.  The forest (or one chunk of whole trees at a
+// forest one after the other without waiting for the other lanes (the lanes
+// of a warp start on the same tree, so its upper levels are broadcast loads),
+// and each candidate has eight independent walks in flight.  The forest (or one chunk of whole trees at a
 // time) sits in shared memory with chunk-relative child indices; the tile's
 // feature values sit in shared memory as feat[slot][f] with an odd row
 // stride (conflict-free when a warp reads one feature).  The eight partial
@@ -157,21 +200,33 @@ rf_kernel(const __grid_constant__ RfArgs a) {
             __syncthreads();
             const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
             if (!live) continue;
-            for (int t = t0 + grp; t < t0 + nt; t += kRfGroups) {
-                int node = sroot[t];
-                bool done = false;
-#pragma unroll 2
-                for (int step = 0; step <= a.max_depth; ++step) {
-                    const uint2 nd = snodes[node];
-                    if ((int)nd.y < 0) {
-                        vote += (uint32_t)__uint_as_float(nd.x);
-                        done = true;
-                        break;
+            // This lane's trees t0 + grp, t0 + grp + 8, ... as one queue: on
+            // reaching a leaf it adds the votes and starts its next tree at
+            // once, so a lane never idles while another lane of the warp is
+            // still deep in a tree of the same round.
+            int t = t0 + grp;
+            if (t >= t0 + nt) continue;
+            int node = sroot[t], depth = 0;
+            for (;;) {
+                const uint2 nd = snodes[node];
+                if ((int)nd.y < 0) {
+                    vote += (uint32_t)__uint_as_float(nd.x);
+                    t += kRfGroups;
+                    if (t >= t0 + nt) break;
+                    node = sroot[t];
+                    depth = 0;
+                } else {
+                    if (++depth > a.max_depth) {  // deeper than the validated depth: flag, drop the tree
+                        atomicOr(a.err, SCOOT_DEVERR_INDEX);
+                        t += kRfGroups;
+                        if (t >= t0 + nt) break;
+                        node = sroot[t];
+                        depth = 0;
+                        continue;
                     }
                     const float x = *reinterpret_cast<const float*>(my + (nd.y >> 16));
                     node = (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
                 }
-                if (!done) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
             }
         }
         svote[grp * kRfCand + slot] = vote;
@@ -244,12 +299,14 @@ scoot_status scoot_prune(scoot_ctx* ctx, const scoot_param* h_space, int32_t d,
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (n_feasible) SCOOT_CUDA(ctx, cudaMemsetAsync(n_feasible, 0, sizeof(int64_t), st));
     if (n == 0) return SCOOT_OK;
-    int64_t blocks = (n + kPruneThreads - 1) / kPruneThreads;
-    const int64_t cap = (int64_t)sm_count(ctx->device) * 16;
+    const int mask_aligned = (reinterpret_cast<uintptr_t>(mask) & 3u) == 0;
+    const int64_t groups = (n + 3) / 4;
+    int64_t blocks = (groups + kPruneThreads - 1) / kPruneThreads;
+    const int64_t cap = (int64_t)sm_count(ctx->device) * 8;
     if (blocks > cap) blocks = cap;
     auto kern = a.exact64 ? prune_kernel<true> : prune_kernel<false>;
     kern<<<(unsigned)blocks, kPruneThreads, 0, st>>>(a, cand, n, ld, mask,
-                                                     reinterpret_cast<unsigned long long*>(n_feasible));
+                                                     reinterpret_cast<unsigned long long*>(n_feasible), mask_aligned);
     SCOOT_LAUNCHED(ctx);
     return SCOOT_OK;
 }

@@ -60,7 +60,7 @@ struct ScoreArgs {
     int32_t cat_smem;             // floats of the categorical table staged in shared memory (0: read from L1)
     int32_t cat_off;              // where, in floats from the start of shared memory
     int32_t wbuf_off;             // the next tile's pool words [d][kTC], in floats from the start
-    float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad][ldv] by list position
+    float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad / 4][ldv][4] by list position
     int64_t ldv;
     uint32_t* err;                // device error word
 };
@@ -362,16 +362,21 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
 #pragma unroll
                     for (int c = 0; c < 4; ++c) sq[c] = fmaf(accm[r][c], accm[r][c], sq[c]);
                 if (EPI == kWriteWhitened) {
-                    // Rows of V for the fantasy downdates, indexed by list position.
+                    // Rows of V for the fantasy downdates, indexed by list
+                    // position, in float4 groups of four rows: group g of
+                    // candidate p at (m n_pad / 4 + g) * ldv + p.  Rows past
+                    // n_obs hold zeros (L^{-1} is zero-filled there).
+                    float4* dst4 = reinterpret_cast<float4*>(a.vout);
 #pragma unroll
-                    for (int r = 0; r < 8; ++r) {
-                        const int row = rb * kRB + rg * 8 + r;
-                        if (row >= a.n_obs) continue;
-                        float* dst = a.vout + ((int64_t)m * n_pad64 + row) * a.ldv;
+                    for (int h = 0; h < 2; ++h) {
+                        const int g = (rb * kRB + rg * 8) / 4 + h;
+                        if (4 * g >= a.n_obs) continue;
 #pragma unroll
                         for (int c = 0; c < 4; ++c) {
                             const int64_t p = tile * kTC + cg * 4 + c;
-                            if (p < n_work) dst[p] = accm[r][c];
+                            if (p < n_work)
+                                dst4[((int64_t)m * (n_pad64 / 4) + g) * a.ldv + p] =
+                                    make_float4(accm[4 * h][c], accm[4 * h + 1][c], accm[4 * h + 2][c], accm[4 * h + 3][c]);
                         }
                     }
                 }

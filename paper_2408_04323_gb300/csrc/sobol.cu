@@ -213,6 +213,38 @@ scoot_status scoot_first_feasible(scoot_ctx* ctx, const uint8_t* mask, int64_t n
     return SCOOT_OK;
 }
 
+scoot_status scoot_ucb_beta(int32_t t, double* beta) {
+    if (!beta || t < 1) return SCOOT_EINVAL;
+    const double tt = (double)t * (double)t;
+    const double delta = 1.0 / tt;
+    *beta = 2.0 * std::log(tt * M_PI * M_PI / (6.0 * delta));
+    return SCOOT_OK;
+}
+
+scoot_status scoot_standardize(const float* h_y, int32_t n_obj, int32_t n, float* h_y_std, float* h_ref,
+                               float ref_margin) {
+    if (!h_y || !h_y_std || n_obj < 1 || n < 1) return SCOOT_EINVAL;
+    for (int m = 0; m < n_obj; ++m) {
+        const float* y = h_y + (size_t)m * n;
+        double mean = 0.0;
+        for (int i = 0; i < n; ++i) {
+            if (!std::isfinite(y[i])) return SCOOT_EINVAL;
+            mean += y[i];
+        }
+        mean /= n;
+        double var = 0.0;
+        for (int i = 0; i < n; ++i) var += ((double)y[i] - mean) * ((double)y[i] - mean);
+        const double sd = std::fmax(std::sqrt(var / n), 1e-12);
+        float lo = INFINITY;
+        for (int i = 0; i < n; ++i) {
+            h_y_std[(size_t)m * n + i] = (float)(((double)y[i] - mean) / sd);
+            lo = std::fmin(lo, h_y_std[(size_t)m * n + i]);
+        }
+        if (h_ref) h_ref[m] = lo - ref_margin;
+    }
+    return SCOOT_OK;
+}
+
 scoot_status scoot_delta_update(double* delta, int32_t* count, int32_t k, int32_t any_invalid) {
     if (!delta || !count || k < 0) return SCOOT_EINVAL;
     constexpr double kStep = 0.05;

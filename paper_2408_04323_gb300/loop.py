@@ -125,12 +125,9 @@ class TuningLoop:
         if good.sum() < 2:
             return self.initial_design(self.q)
         words = np.ascontiguousarray(self.x[:, good])
-        yv = self.y[:, good]
-        y_std = np.ascontiguousarray((yv - yv.mean(axis=1, keepdims=True)) /
-                                     np.maximum(yv.std(axis=1, keepdims=True), 1e-12))
+        y_std, ref = S.scoot_standardize(self.y[:, good], ref_margin=1e-3)
         nodes, offs = self._forest()
         ls, sf2, tau2 = self._gp(words, y_std)
-        ref = y_std.min(axis=1).astype(np.float32) - np.float32(1e-3)
         inp = RoundInputs(self.space, self.clauses, nodes, offs, self.leaf_scale, int(round(self.delta * 20)), 20,
                           words, np.ascontiguousarray(y_std, np.float32), ls, sf2, tau2, ref, self.eps, self.acq,
                           self.q)

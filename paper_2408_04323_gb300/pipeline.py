@@ -10,7 +10,6 @@ computes any step of the path itself.
 """
 from __future__ import annotations
 
-import math
 from dataclasses import dataclass
 
 import numpy as np
@@ -47,12 +46,9 @@ class RoundInputs:
 
 
 def mace_beta(t: int) -> float:
-    """UCB coefficient for tuning iteration t (Section 4.5):
-    beta_t = 2 log(t^2 pi^2 / (6 delta)) with delta = 1 / t^2, taken as the
-    factor of sigma in UCB = mu + beta sigma as printed."""
-    t = max(int(t), 1)
-    delta = 1.0 / (t * t)
-    return 2.0 * math.log(t * t * math.pi ** 2 / (6.0 * delta))
+    """UCB coefficient for tuning iteration t (Section 4.5), from the library
+    (scoot_ucb_beta); t < 1 counts as 1."""
+    return S.scoot_ucb_beta(max(int(t), 1))
 
 
 class _Staging:

@@ -91,6 +91,10 @@ _PROTOS = {
     "scoot_status_string": [_i32],
     "scoot_ctx_check": [_vp, _vp],
     "scoot_ctx_workspace_bytes": [_vp, C.POINTER(_i64)],
+    "scoot_ctx_set_timing": [_vp, _i32],
+    "scoot_probe_fma": [_vp, _i32, _i32, _i32, _vp, _vp],
+    "scoot_probe_gather": [_vp, _i32, _i32, _i32, _vp, _vp],
+    "scoot_ctx_phase_times": [_vp, _i32, _vp, _vp, C.POINTER(_i32)],
     "scoot_prune": [_vp, _vp, _i32, _vp, _i32, _vp, _i64, _i64, _vp, _vp, _vp],
     "scoot_forest_layout_init": [_vp, _vp, _i32, _i32, _i32, C.POINTER(scoot_forest_layout)],
     "scoot_forest_pack": [C.POINTER(scoot_forest_layout), _vp, _vp, _vp],
@@ -127,6 +131,8 @@ _PROTOS = {
     "scoot_sobol_configs": [_vp, _vp, _i32, _i64, _i64, _vp, _i64, _vp],
     "scoot_first_feasible": [_vp, _vp, _i64, _i32, _vp, _vp, _vp],
     "scoot_delta_update": [C.POINTER(C.c_double), C.POINTER(_i32), _i32, _i32],
+    "scoot_ucb_beta": [_i32, C.POINTER(C.c_double)],
+    "scoot_standardize": [_vp, _i32, _i32, _vp, _vp, _f32],
     "scoot_rf_train": [_vp, _vp, _i32, _vp, _i32, _i64, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _i32, _vp, _vp,
                        _i64, _vp],
     "scoot_rf_train_work_bytes": [_i32, _i32, C.POINTER(_i64)],
@@ -136,6 +142,11 @@ _PROTOS = {
     "scoot_fantasy_prepare": [_vp, C.POINTER(scoot_gp_layout), _vp, _i64, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _i64,
                               C.POINTER(_i32)],
     "scoot_fantasy_work_bytes": [C.POINTER(scoot_gp_layout), _i64, _i32, _i32, C.POINTER(_i64)],
+    "scoot_fantasy_begin": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i32, _vp, _i64, _i64, _vp, _i64, _vp, _i32,
+                            _i32, _vp, _i64, _vp, _vp, _vp, _vp],
+    "scoot_fantasy_local_best": [_vp, _i32, _vp, _vp],
+    "scoot_fantasy_commit": [_vp, _i32, _vp, _i32, _vp],
+    "scoot_fantasy_end": [_vp, _vp, _vp],
     "scoot_suggest_fantasy": [_vp, C.POINTER(scoot_gp_layout), _vp, _vp, _i32, _vp, _i64, _i64, _vp, _vp, _i32,
                               _i32, _vp, _i64, _vp, _vp, _vp, _vp, _vp],
 }
@@ -225,6 +236,36 @@ def scoot_ctx_workspace_bytes(ctx) -> int:
     v = _i64()
     _check(lib().scoot_ctx_workspace_bytes(ctx, C.byref(v)), "scoot_ctx_workspace_bytes")
     return int(v.value)
+
+
+PHASES = {0: "compact", 1: "posterior", 2: "fant_init", 3: "fant_pass", 4: "fant_pick", 5: "scatter"}
+
+
+def scoot_ctx_set_timing(ctx, enable: bool) -> None:
+    _check(lib().scoot_ctx_set_timing(_h(ctx), int(bool(enable))), "scoot_ctx_set_timing", _h(ctx))
+
+
+def scoot_ctx_phase_times(ctx, cap: int = 256):
+    """[(phase name, milliseconds)] of the last timed call's launches, in order."""
+    kind = np.zeros(cap, np.int32)
+    ms = np.zeros(cap, np.float32)
+    cnt = _i32()
+    _check(lib().scoot_ctx_phase_times(_h(ctx), int(cap), _host(kind), _host(ms), C.byref(cnt)),
+           "scoot_ctx_phase_times", _h(ctx))
+    k = min(cnt.value, cap)
+    return [(PHASES.get(int(kind[i]), str(int(kind[i]))), float(ms[i])) for i in range(k)]
+
+
+def scoot_probe_fma(ctx, packed: bool, blocks: int, iters: int, sink, stream=None) -> None:
+    import torch
+    _check(lib().scoot_probe_fma(_h(ctx), int(bool(packed)), int(blocks), int(iters),
+                                 _dev(sink, torch.float32, "sink"), _stream(stream)), "scoot_probe_fma", _h(ctx))
+
+
+def scoot_probe_gather(ctx, n_nodes: int, blocks: int, steps: int, sink, stream=None) -> None:
+    import torch
+    _check(lib().scoot_probe_gather(_h(ctx), int(n_nodes), int(blocks), int(steps),
+                                    _dev(sink, torch.float32, "sink"), _stream(stream)), "scoot_probe_gather", _h(ctx))
 
 
 def scoot_status_string(status: int) -> str:
@@ -543,6 +584,22 @@ def scoot_first_feasible(ctx, mask, n, need, idx, count, stream=None):
                                       _stream(stream)), "scoot_first_feasible", _h(ctx))
 
 
+def scoot_ucb_beta(t: int) -> float:
+    v = C.c_double()
+    _check(lib().scoot_ucb_beta(int(t), C.byref(v)), "scoot_ucb_beta")
+    return float(v.value)
+
+
+def scoot_standardize(h_y, ref_margin: float = 1e-3):
+    """(standardised objectives float32 [M][n], reference point float32 [M])."""
+    y = np.ascontiguousarray(h_y, np.float32)
+    out = np.empty_like(y)
+    ref = np.empty(y.shape[0], np.float32)
+    _check(lib().scoot_standardize(_host(y), int(y.shape[0]), int(y.shape[1]), _host(out), _host(ref),
+                                   float(ref_margin)), "scoot_standardize")
+    return out, ref
+
+
 def scoot_delta_update(delta: float, count: int, k: int, any_invalid: bool):
     """Returns the new (delta, count)."""
     d, c = C.c_double(delta), _i32(count)
@@ -699,3 +756,37 @@ def scoot_suggest_fantasy(ctx, layout, state, fant_state, box_cap, cand, n, eps,
         _dev(idx, torch.int64, "idx"), _dev(val, torch.float32, "val"), _dev(count, torch.int32, "count"),
         _dev(var_out, torch.float32, "var_out"), _stream(stream)),
         "scoot_suggest_fantasy", _h(ctx))
+
+
+FANT_REC = 9  # SCOOT_FANT_REC: 64-bit words of a shard's record
+
+
+def scoot_fantasy_begin(ctx, layout, state, fant_state, box_cap, cand, n, eps, q, work, idx, val, count, mask=None,
+                        index_offset=0, stream=None):
+    import torch
+    _check(lib().scoot_fantasy_begin(
+        _h(ctx), C.byref(layout), _dev(state, torch.uint8, "state"), _dev(fant_state, torch.uint8, "fant_state"),
+        int(box_cap), _dev(cand, torch.int32, "cand"), int(n), int(cand.shape[1]), _dev(mask, torch.uint8, "mask"),
+        int(index_offset), _dev(eps, torch.float32, "eps"), int(eps.shape[0]), int(q), _vp(work.data_ptr()),
+        int(work.numel()), _dev(idx, torch.int64, "idx"), _dev(val, torch.float32, "val"),
+        _dev(count, torch.int32, "count"), _stream(stream)), "scoot_fantasy_begin", _h(ctx))
+
+
+def scoot_fantasy_local_best(ctx, j, rec=None, stream=None):
+    """rec: device int64 [FANT_REC] (the uint64 record's bits) or None."""
+    import torch
+    _check(lib().scoot_fantasy_local_best(_h(ctx), int(j), _dev(rec, torch.int64, "rec"), _stream(stream)),
+           "scoot_fantasy_local_best", _h(ctx))
+
+
+def scoot_fantasy_commit(ctx, j, recs, stream=None):
+    """recs: device int64 [n_rec][FANT_REC], the gathered records."""
+    import torch
+    _check(lib().scoot_fantasy_commit(_h(ctx), int(j), _dev(recs, torch.int64, "recs"), int(recs.shape[0]),
+                                      _stream(stream)), "scoot_fantasy_commit", _h(ctx))
+
+
+def scoot_fantasy_end(ctx, var_out=None, stream=None):
+    import torch
+    _check(lib().scoot_fantasy_end(_h(ctx), _dev(var_out, torch.float32, "var_out"), _stream(stream)),
+           "scoot_fantasy_end", _h(ctx))

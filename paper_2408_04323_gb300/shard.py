@@ -10,6 +10,12 @@ a candidate is on the pool's front iff it is on its rank's front and no
 other rank's front member dominates it, and the random k-subset is drawn
 with the same keys (SplitMix64 of the global index) as on one GPU, so the
 picks equal the single-pool picks.
+
+The sequential fantasised picks exchange once per pick: every rank's best
+candidate of the pass (its record: selection key with the global index and
+the candidate's configuration words) is all-gathered, and every rank commits
+the record with the largest key, computing the pick's rank-1 terms from the
+configuration it carries; no rank needs another rank's pool.
 """
 from __future__ import annotations
 
@@ -121,3 +127,80 @@ def gather_mace_front(acq3, front_idx, front_count: int, base: int, k: int, seed
     dist.all_gather(tris, tri, group=group)
     dist.all_gather(gids, gid, group=group)
     return merge_mace_fronts(torch.stack(tris).cpu().numpy(), torch.stack(gids).cpu().numpy(), C, k, seed)
+
+
+# ------------------------------------------------------------------ sequential fantasised picks
+
+FANT_REC = 9  # 64-bit words of a record (include/scoot.h, SCOOT_FANT_REC)
+
+
+def selection_key(value: float, global_index: int) -> int:
+    """The 64-bit selection key of Section 4.7's order (the device's make_key):
+    order-preserving bits of the fp32 value (-0 as +0) in the high word,
+    0xFFFFFFFF - index in the low word; 0 for NaN and -inf (never selected)."""
+    v = np.float32(value)
+    if np.isnan(v) or v == -np.inf:
+        return 0
+    b = int(np.array([v], np.float32).view(np.uint32)[0])
+    if b == 0x80000000:
+        b = 0
+    b = (~b & 0xFFFFFFFF) if b & 0x80000000 else (b | 0x80000000)
+    return (b << 32) | (0xFFFFFFFF - int(global_index))
+
+
+def encode_fantasy_record(value: float, global_index: int, words) -> np.ndarray:
+    """A shard's record as the device writes it (int64 view of the uint64
+    words): the key, then the configuration words two per element."""
+    rec = np.zeros(FANT_REC, np.uint64)
+    key = selection_key(value, global_index)
+    rec[0] = np.uint64(key)
+    if key:
+        w = np.zeros(2 * (FANT_REC - 1), np.uint32)
+        w[:len(words)] = np.asarray(words, np.uint32)
+        rec[1:] = w.view(np.uint64)
+    return rec.view(np.int64)
+
+
+def decode_fantasy_record(rec, d: int):
+    """(value, global index, words) of a record, or None for key 0."""
+    r = np.asarray(rec).view(np.uint64)
+    key = int(r[0])
+    if key == 0:
+        return None
+    b = key >> 32
+    b = (b & 0x7FFFFFFF) if b & 0x80000000 else (~b & 0xFFFFFFFF)
+    value = float(np.array([b], np.uint32).view(np.float32)[0])
+    return value, 0xFFFFFFFF - (key & 0xFFFFFFFF), r[1:].view(np.uint32)[:d].copy()
+
+
+def best_record(recs) -> int:
+    """Row of the record with the largest (unsigned) key, -1 if every key is 0."""
+    keys = np.asarray(recs).view(np.uint64)[:, 0]
+    k = int(np.argmax(keys))
+    return k if keys[k] != 0 else -1
+
+
+def gather_fantasy_records(rec, group=None):
+    """All ranks' records ([world][FANT_REC], same device as rec)."""
+    import torch
+    import torch.distributed as dist
+    world = dist.get_world_size(group)
+    parts = [torch.empty_like(rec.reshape(-1)) for _ in range(world)]
+    dist.all_gather(parts, rec.reshape(-1).contiguous(), group=group)
+    return torch.stack(parts)
+
+
+def sharded_fantasy_picks(S, ctx, layout, state, fant_state, box_cap, cand, n, eps, q, work, idx, val, count,
+                          index_offset, mask=None, var_out=None, group=None, stream=None):
+    """q sequential fantasised picks over a pool sharded across the ranks of
+    `group`: this rank holds candidates index_offset .. index_offset + n - 1.
+    One all-gather of the ranks' records per pick; idx, val, count (device)
+    end up identical on every rank and equal to the single-pool picks."""
+    import torch
+    S.scoot_fantasy_begin(ctx, layout, state, fant_state, box_cap, cand, n, eps, q, work, idx, val, count, mask=mask,
+                          index_offset=index_offset, stream=stream)
+    rec = torch.zeros(FANT_REC, dtype=torch.int64, device=idx.device)
+    for j in range(q):
+        S.scoot_fantasy_local_best(ctx, j, rec, stream)
+        S.scoot_fantasy_commit(ctx, j, gather_fantasy_records(rec, group), stream)
+    S.scoot_fantasy_end(ctx, var_out, stream)

@@ -282,3 +282,58 @@ def test_fantasy_errors_found_on_the_device(S):
         assert int(cnt.item()) == 4
     finally:
         ctx.close()
+
+
+def test_sharded_picks_equal_the_single_pool_call(S):
+    """The phase calls over three shards of one pool (the multi-GPU
+    protocol, run one shard after another on one GPU: no kernel waits on
+    another shard's): after each pass the shards' records are stacked and
+    every shard commits them; every shard's picks, values and count equal
+    the single-pool call bit for bit, and so do its variances.  Each record
+    decodes (on the host) to the shard's candidate's value, global index and
+    configuration words."""
+    from paper_2408_04323_gb300.shard import FANT_REC, decode_fantasy_record, selection_key, shard_range
+    name, n, q = "d12-fantasy", 30011, 8
+    inst = make_instance(name, seeds(name)[2], n_cand=n)
+    ctx0 = S.Context(0)
+    ctxs = [S.Context(0) for _ in range(3)]
+    try:
+        r = _round_inputs(S, inst, q)
+        var0 = torch.full((inst.n_obj, n), -1.0, device="cuda")
+        mask, _, idx0, val0, cnt0 = _gpu_round(S, ctx0, inst, q, n, r, var_out=var0)
+        ctx0.check()
+        shards = []
+        for s in range(3):
+            b, e = shard_range(n, s, 3)
+            ld = (e - b + 3) // 4 * 4
+            cand_s = torch.zeros((inst.d, ld), dtype=torch.int32, device="cuda")
+            cand_s[:, :e - b] = r["cand"][:, b:e]
+            mask_s = mask[b:e].contiguous()
+            work = torch.empty(S.scoot_fantasy_work_bytes(r["G"], e - b, q, r["box_cap"]), dtype=torch.uint8,
+                               device="cuda")
+            out = _outputs(q)
+            S.scoot_fantasy_begin(ctxs[s], r["G"], r["state"], r["fant"], r["box_cap"], cand_s, e - b, r["eps"], q,
+                                  work, *out, mask=mask_s, index_offset=b)
+            shards.append((b, e, cand_s, mask_s, work, out))
+        recs = torch.zeros((3, FANT_REC), dtype=torch.int64, device="cuda")
+        for j in range(q):
+            for s in range(3):
+                S.scoot_fantasy_local_best(ctxs[s], j, recs[s])
+            if j == 0:
+                for s, (b, e, cand_s, *_rest) in enumerate(shards):
+                    dec = decode_fantasy_record(recs[s].cpu().numpy(), inst.d)
+                    assert dec is not None and b <= dec[1] < e
+                    assert np.array_equal(dec[2], inst.cand[:, dec[1]])
+                    assert int(recs[s].cpu().numpy().view(np.uint64)[0]) == selection_key(dec[0], dec[1])
+            for s in range(3):
+                S.scoot_fantasy_commit(ctxs[s], j, recs)
+        for s, (b, e, _, _, _, out) in enumerate(shards):
+            var_s = torch.full((inst.n_obj, e - b), -1.0, device="cuda")
+            S.scoot_fantasy_end(ctxs[s], var_s)
+            ctxs[s].check()
+            assert torch.equal(out[0], idx0) and torch.equal(out[1], val0) and torch.equal(out[2], cnt0), s
+            assert torch.equal(var_s, var0[:, b:e]), s
+    finally:
+        for c in ctxs + [ctx0]:
+            c.close()
+    assert int(cnt0.item()) == q

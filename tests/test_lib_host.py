@@ -445,3 +445,34 @@ def test_fantasy_state_holds_the_fp64_factorisation(S, name, q):
                                        boxes=1, h_ref=inst.ref, h_eps=inst.eps, fantasy_q=q)
     assert out.off_fant >= 0 and out.off_fant % 256 == 0 and out.fant_box_cap == box_cap
     assert np.array_equal(buf[out.off_fant:out.off_fant + len(st)], st)
+
+
+def test_ucb_beta_is_the_printed_schedule(S):
+    """beta_t = 2 log(t^2 pi^2 / (6 delta)) with delta = 1/t^2 (Section 4.5)
+    = 2 log(pi^2 t^4 / 6): 0.994... at t = 1, growing like 8 log t."""
+    import math
+    for t in (1, 2, 16, 128, 1000):
+        assert S.scoot_ucb_beta(t) == pytest.approx(2.0 * math.log(math.pi ** 2 * t ** 4 / 6.0), rel=1e-14)
+    assert S.scoot_ucb_beta(1) == pytest.approx(2.0 * math.log(math.pi ** 2 / 6.0), rel=1e-14)
+    assert S.scoot_ucb_beta(20) - S.scoot_ucb_beta(10) == pytest.approx(8.0 * math.log(2.0), rel=1e-12)
+    with pytest.raises(S.ScootError):
+        S.scoot_ucb_beta(0)
+
+
+def test_standardize_gives_zero_mean_unit_sd_and_a_reference_below(S):
+    y = (Stream(41, "std").normal(3 * 50).reshape(3, 50) * [[3.0], [0.01], [100.0]] + [[5.0], [-2.0], [1e3]])
+    y = y.astype(np.float32)
+    z, ref = S.scoot_standardize(y, ref_margin=1e-3)
+    assert np.allclose(z.astype(np.float64).mean(axis=1), 0.0, atol=1e-6)
+    assert np.allclose(z.astype(np.float64).std(axis=1), 1.0, atol=1e-6)
+    assert np.all(ref < z.min(axis=1)) and np.allclose(ref, z.min(axis=1) - 1e-3, atol=1e-7)
+    # invariant to an affine change of units
+    z2, _ = S.scoot_standardize((y.astype(np.float64) * 7.0 - 3.0).astype(np.float32))
+    assert np.allclose(z, z2, atol=1e-4)  # up to the fp32 rounding of the rescaled inputs
+    # a constant objective stays finite (the floor of the standard deviation)
+    z3, _ = S.scoot_standardize(np.ones((1, 5), np.float32))
+    assert np.all(z3 == 0.0)
+    bad = y.copy()
+    bad[1, 3] = np.nan
+    with pytest.raises(S.ScootError):
+        S.scoot_standardize(bad)
