@@ -134,9 +134,9 @@ struct RfArgs {
 
 // Persistent blocks of 256 threads score tiles of 32 candidates: lane l of
 // warp g serves candidate slot l and walks trees g, g + 8, g + 16, ... of the
-// forest one after the other without waiting for the other lanes (the lanes
-// of a warp start on the same tree, so its upper levels are broadcast loads),
-// and each candidate has eight independent walks in flight.  The forest (or one chunk of whole trees at a
+// forest, so the 32 lanes of a warp walk the same tree for 32 candidates
+// (the upper levels are broadcast loads) and each candidate has eight
+// independent walks in flight.  The forest (or one chunk of whole trees at a
 // time) sits in shared memory with chunk-relative child indices; the tile's
 // feature values sit in shared memory as feat[slot][f] with an odd row
 // stride (conflict-free when a warp reads one feature).  The eight partial
@@ -200,33 +200,26 @@ rf_kernel(const __grid_constant__ RfArgs a) {
             __syncthreads();
             const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
             if (!live) continue;
-            // This lane's trees t0 + grp, t0 + grp + 8, ... as one queue: on
-            // reaching a leaf it adds the votes and starts its next tree at
-            // once, so a lane never idles while another lane of the warp is
-            // still deep in a tree of the same round.
-            int t = t0 + grp;
-            if (t >= t0 + nt) continue;
-            int node = sroot[t], depth = 0;
-            for (;;) {
-                const uint2 nd = snodes[node];
-                if ((int)nd.y < 0) {
-                    vote += (uint32_t)__uint_as_float(nd.x);
-                    t += kRfGroups;
-                    if (t >= t0 + nt) break;
-                    node = sroot[t];
-                    depth = 0;
-                } else {
-                    if (++depth > a.max_depth) {  // deeper than the validated depth: flag, drop the tree
-                        atomicOr(a.err, SCOOT_DEVERR_INDEX);
-                        t += kRfGroups;
-                        if (t >= t0 + nt) break;
-                        node = sroot[t];
-                        depth = 0;
-                        continue;
+            // The lanes of a warp walk the same tree (for 32 candidates) in
+            // lockstep, so the upper levels of the tree are broadcast loads;
+            // letting each lane run on to its next tree as soon as it reaches
+            // a leaf was measured twice as slow: the lanes drift onto
+            // different trees and the node loads stop being broadcasts.
+            for (int t = t0 + grp; t < t0 + nt; t += kRfGroups) {
+                int node = sroot[t];
+                bool done = false;
+#pragma unroll 2
+                for (int step = 0; step <= a.max_depth; ++step) {
+                    const uint2 nd = snodes[node];
+                    if ((int)nd.y < 0) {
+                        vote += (uint32_t)__uint_as_float(nd.x);
+                        done = true;
+                        break;
                     }
                     const float x = *reinterpret_cast<const float*>(my + (nd.y >> 16));
                     node = (int)(nd.y & 0xffffu) + (x <= __uint_as_float(nd.x) ? 0 : 1);
                 }
+                if (!done) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
             }
         }
         svote[grp * kRfCand + slot] = vote;
