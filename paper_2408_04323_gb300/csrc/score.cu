@@ -1,13 +1,14 @@
 // GP posterior (Section 4.3) and acquisition values: EI (Eq. 6) and
 // Monte-Carlo EHVI over a box decomposition (Eq. 7), fused or separate.
 //
-// A block of 128 threads (two per candidate) owns a tile of 64 candidates.
+// A block of 128 threads (four per candidate: warp w is quarter w of every
+// candidate, lane l serves candidate slot l) owns a tile of 32 candidates.
 // Per objective:
-//  1. the two threads of a candidate evaluate its covariance row k(x, X)
+//  1. the four threads of a candidate evaluate its covariance row k(x, X)
 //     against the n observations (staged in shared memory) into Ks[j][c],
-//     splitting j by parity, and accumulate mu = k . alpha;
+//     splitting j by j mod 4, and accumulate mu = k . alpha;
 //  2. the block computes V = L^{-1} Ks as a register-tiled SIMT product
-//     (4 candidates x 8 rows per thread) over 32 x 64 tiles of L^{-1} that the
+//     (4 candidates x 4 rows per thread) over 32 x 64 tiles of L^{-1} that the
 //     host laid out transposed and zero-filled; the tiles are double-buffered
 //     in shared memory by cp.async, so the next tile streams in while the
 //     current one is multiplied; sigma^2 = s_f^2 - sum_i V_ic^2, clamped at 0.
@@ -21,8 +22,9 @@ namespace {
 
 using namespace scoot_dev;
 
-constexpr int kTC = 64;     // candidates per tile
-constexpr int kThreads = 128;  // two threads per candidate
+constexpr int kTC = 32;     // candidates per tile
+constexpr int kThreads = 128;  // four threads per candidate
+constexpr int kQ = kThreads / kTC;  // threads per candidate (= warps: warp w is quarter w)
 constexpr int kRB = 64;     // rows of L^{-1} per tile
 constexpr int kCJ = 32;     // columns of L^{-1} per tile
 constexpr int kMaxD = SCOOT_MAX_DIM;
@@ -60,6 +62,7 @@ struct ScoreArgs {
     int32_t cat_smem;             // floats of the categorical table staged in shared memory (0: read from L1)
     int32_t cat_off;              // where, in floats from the start of shared memory
     int32_t wbuf_off;             // the next tile's pool words [d][kTC], in floats from the start
+    int32_t single_l;             // 1: one L^{-1} tile buffer (more blocks per SM), 0: double buffering
     float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad / 4][ldv][4] by list position
     int64_t ldv;
     uint32_t* err;                // device error word
@@ -115,7 +118,7 @@ __device__ __forceinline__ void stage_tile_async(float* dst, const float4* src, 
 }
 
 // Gathers the d words of the candidates of a tile into wbuf[q][slot] (feature
-// order) with 4-byte cp.async, two threads per candidate, one group.
+// order) with 4-byte cp.async, four threads per candidate, one group.
 __device__ __forceinline__ void prefetch_words(uint32_t* wbuf, const uint32_t* cand, int64_t ld, const int32_t* list,
                                                const float4* fm, int d, int64_t tile, int64_t n_tiles,
                                                int64_t n_work, int tid) {
@@ -123,7 +126,7 @@ __device__ __forceinline__ void prefetch_words(uint32_t* wbuf, const uint32_t* c
     const int64_t p = tile * kTC + s;
     if (tile < n_tiles && p < n_work) {
         const int64_t i = list ? (int64_t)list[p] : p;
-        for (int q = tid >> 6; q < d; q += 2) {
+        for (int q = tid / kTC; q < d; q += kQ) {
             const unsigned dst = (unsigned)__cvta_generic_to_shared(wbuf + q * kTC + s);
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst),
                          "l"(cand + (int64_t)fm[q].w * ld + i) : "memory");
@@ -135,32 +138,33 @@ __device__ __forceinline__ void prefetch_words(uint32_t* wbuf, const uint32_t* c
 // Waits until every cp.async group this thread committed has landed.
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-// One block of 128 threads scores a tile of 64 candidates; thread t works on
-// candidate slot t % 64 with its partner t +- 64 ("half" t / 64):
-//  1. both halves compute the candidate's features; for each objective the
-//     halves split the covariance row k(x, X_j) (j even / odd) into Ks[j][slot]
-//     and the partial sums of mu = k . alpha;
+// One block of 128 threads scores a tile of 32 candidates; thread t works on
+// candidate slot t % 32 as quarter t / 32 (its warp) of that candidate:
+//  1. the quarters compute the candidate's features; for each objective they
+//     split the covariance row k(x, X_j) (j mod 4) into Ks[j][slot] and the
+//     partial sums of mu = k . alpha;
 //  2. all 128 threads compute V = L^{-1} Ks over 32 x 64 tiles of L^{-1} with a
-//     4-candidate x 8-row register tile each; a warp whose 16 rows lie wholly
+//     4-candidate x 4-row register tile each; a warp whose 16 rows lie wholly
 //     above a tile's columns (upper triangle, all zero) skips that tile;
 //     sigma^2 = s_f^2 - sum_i V_i^2;
-//  3. the epilogue (EI on one half, EHVI with the halves splitting the
-//     sample chunks, or the moments / whitened rows) writes the tile.
+//  3. the epilogue (EI on one quarter, EHVI or exact EHVI with the quarters
+//     splitting the sample chunks or boxes, or the moments / whitened rows)
+//     writes the tile.
 // Features come in feature order (ordinal parameters first).  DO >= n_ord
 // bounds the ordinal register arrays; padded ordinal dimensions are zero on
 // both sides and add nothing, so the distance loop has no per-dimension
 // branch.  The categorical part of r^2 depends only on the candidate's joint
 // category pattern and is read from the host-built table (one load).
 template <int EPI, int M, int DO>
-__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 5 : ((EPI == kEI || EPI == kMACE) ? 4 : 1))
+__global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 6 : 4)
 score_kernel(const __grid_constant__ ScoreArgs a) {
-    // Five blocks per SM for the 2-objective EHVI of <= 8 parameters caps
-    // registers at 96.  The one-objective epilogues run four blocks per SM
-    // (128 registers) with a single L^{-1} tile buffer, which the fourth
-    // block's shared memory needs: their tile loads are hidden by the other
-    // blocks rather than by double buffering.
+    // At least four blocks (16 warps) per SM: registers capped at 128 (80 for
+    // the 2-objective EHVI of <= 8 parameters, six blocks).  When the L^{-1}
+    // double buffer would cost a block per SM of shared memory, the launch
+    // asks for a single buffer (a.single_l): the tile loads are then hidden
+    // by the other blocks rather than by double buffering.
     constexpr bool kRegCapped = EPI == kEHVI && M == 2 && DO == 8;
-    constexpr bool kSingleL = EPI == kEI || EPI == kMACE;
+    const bool kSingleL = a.single_l != 0;  // the same in every thread
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
     // Ks, and after the posterior the exact-EHVI psi table [psi_rows][kTC]
@@ -169,8 +173,8 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     float* xs = Ks + (size_t)ks_rows * kTC;                           // [n_obs][DO] ordinal features
     float* al = xs + (size_t)a.n_obs * DO;                            // [n_pad]
     float* Lt = al + n_pad;                                           // [2][kCJ][kRB] double buffer
-    float* part = Lt + (kSingleL ? 1 : 2) * kCJ * kRB;                // [8][kTC]
-    float4* fm = reinterpret_cast<float4*>(part + 8 * kTC);           // [kMaxD] feature map
+    float* part = Lt + (kSingleL ? 1 : 2) * kCJ * kRB;                // [16][kTC]
+    float4* fm = reinterpret_cast<float4*>(part + 16 * kTC);          // [kMaxD] feature map
     float4* blo = fm + kMaxD;                          // [B] (general boxes) or [2B] (saturated form)
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
     float4* epsv = bhi + (EPI == kEHVI ? a.n_boxes : 0);
@@ -178,7 +182,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     uint32_t* corner_s = reinterpret_cast<uint32_t*>(grid_s + ((a.psi_rows + 3) & ~3));  // [B][M]
 
     const int tid = threadIdx.x;
-    const int slot = tid & (kTC - 1), half = tid >> 6;
+    const int slot = tid & (kTC - 1), qtr = tid / kTC;
     const int warp = tid >> 5;
     const int nobj = (EPI == kEHVI || EPI == kEHVIX) ? M : ((EPI == kEI || EPI == kMACE) ? 1 : a.n_obj);
     const int64_t n_pad64 = n_pad;
@@ -269,10 +273,10 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 ut[q] = q < n_ord ? x * gils[m * a.d + q] : 0.0f;
             }
             __syncthreads();
-            // 1. covariance row (this half's j) and the partial mean.
+            // 1. covariance row (this quarter's j) and the partial mean.
             float acc = 0.0f;
 #pragma unroll 2
-            for (int j = half; j < a.n_obs; j += 2) {
+            for (int j = qtr; j < a.n_obs; j += kQ) {
                 const float4* xj4 = reinterpret_cast<const float4*>(xs + j * DO);
                 float r2 = catrow[(size_t)j * a.n_pat];  // categorical part
 #pragma unroll
@@ -289,12 +293,14 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 Ks[j * kTC + slot] = k;
                 acc = fmaf(k, al[j], acc);
             }
-            for (int j = a.n_obs + half; j < n_pad; j += 2) Ks[j * kTC + slot] = 0.0f;
-            part[half * kTC + slot] = acc;
+            for (int j = a.n_obs + qtr; j < n_pad; j += kQ) Ks[j * kTC + slot] = 0.0f;
+            part[qtr * kTC + slot] = acc;
             __syncthreads();
-            mu[m] = part[slot] + part[kTC + slot];
-            // 2. V = L^{-1} Ks and the sum of squares per candidate.
-            const int cg = tid & 15, rg = tid >> 4;
+            mu[m] = (part[slot] + part[kTC + slot]) + (part[2 * kTC + slot] + part[3 * kTC + slot]);
+            // 2. V = L^{-1} Ks and the sum of squares per candidate: thread
+            // (cg, rg) holds candidates 4 cg .. 4 cg + 3 and rows 4 rg .. 4 rg + 3
+            // of each 64-row block; a warp's rows are 16 consecutive ones.
+            const int cg = tid & 7, rg = tid >> 3;
             float sq[4] = {0.f, 0.f, 0.f, 0.f};
             const float4* Ks4 = reinterpret_cast<const float4*>(Ks);
             int t = 0;
@@ -302,11 +308,10 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 // accumulators in column pairs: acc2[r][cp] = (V[r][2 cp], V[r][2 cp + 1]),
                 // updated by packed fp32 FMAs (two per instruction, each lane
                 // rounded as fmaf): the k loads give the candidate pairs, the
-                // row's L^{-1} value is broadcast to both lanes, one row at a
-                // time (so that only one broadcast pair is live).
-                float2 acc2[8][2];
+                // row's L^{-1} value is broadcast to both lanes.
+                float2 acc2[4][2];
 #pragma unroll
-                for (int r = 0; r < 8; ++r) acc2[r][0] = acc2[r][1] = make_float2(0.0f, 0.0f);
+                for (int r = 0; r < 4; ++r) acc2[r][0] = acc2[r][1] = make_float2(0.0f, 0.0f);
                 for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t) {
                     // Tile t has landed in buffer t&1 and every thread is done
                     // with tile t-1, so tile t+1 may overwrite buffer (t+1)&1
@@ -323,16 +328,15 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                     const int last_row = rb * kRB + 16 * warp + 15;
                     if (!kSingleL && j0 > last_row) continue;  // (single buffer: every thread reaches the staging below)
                     const int jj_end = j0 > last_row ? 0 : (last_row - j0 + 1 >= kCJ ? kCJ : 16);
-#pragma unroll 4
+#pragma unroll 8
                     for (int jj = 0; jj < jj_end; ++jj) {
                         const float4 k4 = Ks4[(j0 + jj) * (kTC / 4) + cg];
-                        const float4 l0 = Lt4[jj * (kRB / 4) + rg * 2];
-                        const float4 l1 = Lt4[jj * (kRB / 4) + rg * 2 + 1];
+                        const float4 l4 = Lt4[jj * (kRB / 4) + rg];
                         const float2 k01 = make_float2(k4.x, k4.y), k23 = make_float2(k4.z, k4.w);
-                        const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
+                        const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
 #pragma unroll
-                        for (int r = 0; r < 8; ++r) {
-                            if (kRegCapped) {  // scalar FMAs: the broadcast pairs would spill at 96 registers
+                        for (int r = 0; r < 4; ++r) {
+                            if (kRegCapped) {  // scalar FMAs in the register-capped variant
                                 acc2[r][0].x = fmaf(lv[r], k4.x, acc2[r][0].x);
                                 acc2[r][0].y = fmaf(lv[r], k4.y, acc2[r][0].y);
                                 acc2[r][1].x = fmaf(lv[r], k4.z, acc2[r][1].x);
@@ -349,62 +353,61 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                         stage_tile_async(Lt, tiles + (size_t)(t + 1) * (kCJ * kRB / 4), tid);
                     }
                 }
-                float accm[8][4];
+                float accm[4][4];
 #pragma unroll
-                for (int r = 0; r < 8; ++r) {
+                for (int r = 0; r < 4; ++r) {
                     accm[r][0] = acc2[r][0].x;
                     accm[r][1] = acc2[r][0].y;
                     accm[r][2] = acc2[r][1].x;
                     accm[r][3] = acc2[r][1].y;
                 }
 #pragma unroll
-                for (int r = 0; r < 8; ++r)
+                for (int r = 0; r < 4; ++r)
 #pragma unroll
                     for (int c = 0; c < 4; ++c) sq[c] = fmaf(accm[r][c], accm[r][c], sq[c]);
                 if (EPI == kWriteWhitened) {
                     // Rows of V for the fantasy downdates, indexed by list
-                    // position, in float4 groups of four rows: group g of
-                    // candidate p at (m n_pad / 4 + g) * ldv + p.  Rows past
-                    // n_obs hold zeros (L^{-1} is zero-filled there).
+                    // position, in float4 groups of four rows (this thread's
+                    // rows are one group): group g of candidate p at
+                    // (m n_pad / 4 + g) * ldv + p.  Rows past n_obs hold zeros
+                    // (L^{-1} is zero-filled there).
                     float4* dst4 = reinterpret_cast<float4*>(a.vout);
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int g = (rb * kRB + rg * 8) / 4 + h;
-                        if (4 * g >= a.n_obs) continue;
+                    const int g = rb * (kRB / 4) + rg;
+                    if (4 * g < a.n_obs) {
 #pragma unroll
                         for (int c = 0; c < 4; ++c) {
                             const int64_t p = tile * kTC + cg * 4 + c;
                             if (p < n_work)
                                 dst4[((int64_t)m * (n_pad64 / 4) + g) * a.ldv + p] =
-                                    make_float4(accm[4 * h][c], accm[4 * h + 1][c], accm[4 * h + 2][c], accm[4 * h + 3][c]);
+                                    make_float4(accm[0][c], accm[1][c], accm[2][c], accm[3][c]);
                         }
                     }
                 }
             }
-            __syncthreads();  // every thread has read its mean halves from part
+            __syncthreads();  // every thread has read its mean quarters from part
 #pragma unroll
             for (int c = 0; c < 4; ++c) part[rg * kTC + cg * 4 + c] = sq[c];
             __syncthreads();
             float ss = 0.0f;
 #pragma unroll
-            for (int g = 0; g < 8; ++g) ss += part[g * kTC + slot];
+            for (int g = 0; g < kRB / 4; ++g) ss += part[g * kTC + slot];
             vr[m] = fmaxf(sf2 - ss, 0.0f);
         }
         // 3. epilogue.
         if (EPI == kWriteMoments) {
-            if (live && half == 0)
+            if (live && qtr == 0)
                 for (int m = 0; m < nobj; ++m) {
                     a.mean[(int64_t)m * a.ldo + i] = mu[m];
                     a.var[(int64_t)m * a.ldo + i] = vr[m];
                 }
         } else if (EPI == kWriteWhitened) {
-            if (live && half == 0)
+            if (live && qtr == 0)
                 for (int m = 0; m < nobj; ++m) {
                     a.mean[(int64_t)m * a.ldo + pos] = mu[m];
                     a.var[(int64_t)m * a.ldo + pos] = vr[m];
                 }
         } else if (EPI == kEI) {
-            if (live && half == 0) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
+            if (live && qtr == 0) a.acq[i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
         } else if (EPI == kEHVIX) {
             // psi table: row poff_j + g holds psi_j(grid_j[g]) (the row past
             // the last grid coordinate, +inf, holds 0).  Every thread read its
@@ -415,15 +418,15 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             int goff = 0, poff = 0;
 #pragma unroll
             for (int m = 0; m < M; ++m) {
-                for (int g = half; g < a.n_grid[m]; g += 2)
+                for (int g = qtr; g < a.n_grid[m]; g += kQ)
                     Ks[(poff + g) * kTC + slot] = expected_excess(mu[m], sd[m], grid_s[goff + g]);
-                if (half == 0) Ks[(poff + a.n_grid[m]) * kTC + slot] = 0.0f;
+                if (qtr == 0) Ks[(poff + a.n_grid[m]) * kTC + slot] = 0.0f;
                 goff += a.n_grid[m];
                 poff += a.n_grid[m] + 1;
             }
             __syncthreads();
             float v = 0.0f;
-            for (int b = half; b < a.n_boxes; b += 2) {
+            for (int b = qtr; b < a.n_boxes; b += kQ) {
                 float p = 1.0f;
                 int po = 0;
 #pragma unroll
@@ -435,11 +438,11 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 v += p;
             }
             __syncthreads();  // part is free again; the psi table is read
-            part[half * kTC + slot] = v;
+            part[qtr * kTC + slot] = v;
             __syncthreads();
-            if (live && half == 0) a.acq[i] = part[slot] + part[kTC + slot];
+            if (live && qtr == 0) a.acq[i] = (part[slot] + part[kTC + slot]) + (part[2 * kTC + slot] + part[3 * kTC + slot]);
         } else if (EPI == kMACE) {
-            if (live && half == 0) {
+            if (live && qtr == 0) {
                 a.acq[i] = ucb_value(mu[0], vr[0], a.kappa);
                 a.acq[a.lda + i] = pi_value(mu[0], vr[0], gscal[2], a.xi);
                 a.acq[2 * a.lda + i] = ei_value(mu[0], vr[0], gscal[2], a.xi);
@@ -448,12 +451,14 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             float sd[kMaxM];
 #pragma unroll
             for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
-            const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, a.n_boxes, epsv, a.n_mc, half, 2)
-                                 : ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, half, 2);
+            const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, a.n_boxes, epsv, a.n_mc, qtr, kQ)
+                                 : ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, qtr, kQ);
             __syncthreads();  // part is free again
-            part[half * kTC + slot] = v;
+            part[qtr * kTC + slot] = v;
             __syncthreads();
-            if (live && half == 0) a.acq[i] = (part[slot] + part[kTC + slot]) * (1.0f / (float)a.n_mc);
+            if (live && qtr == 0)
+                a.acq[i] = ((part[slot] + part[kTC + slot]) + (part[2 * kTC + slot] + part[3 * kTC + slot])) *
+                           (1.0f / (float)a.n_mc);
         }
     }
 }
@@ -606,8 +611,8 @@ constexpr int kCatSmemMax = 1024;  // floats of categorical table worth staging 
 size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
     const size_t ks_rows = epi == kEHVIX && (size_t)a.psi_rows > n_pad ? (size_t)a.psi_rows : n_pad;
-    const size_t l_bufs = (epi == kEI || epi == kMACE) ? 1 : 2;
-    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + l_bufs * kCJ * kRB + 8 * kTC + 4 * kMaxD;
+    const size_t l_bufs = a.single_l ? 1 : 2;
+    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + l_bufs * kCJ * kRB + 16 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
     if (epi == kEHVIX) f += (size_t)((a.psi_rows + 3) & ~3) + (size_t)a.n_boxes * kMaxM;
     return f * 4;
@@ -618,20 +623,33 @@ scoot_status launch_score_dm(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
     // the categorical table of the objectives this epilogue reads, staged when small
     const int nobj = (EPI == kEHVI || EPI == kEHVIX) ? M : ((EPI == kEI || EPI == kMACE) ? 1 : a.n_obj);
     const int64_t cat = (int64_t)nobj * a.n_obs * a.n_pat;
-    a.cat_off = (int32_t)(score_smem(a, EPI, DO) / 4);
-    a.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
-    a.wbuf_off = a.cat_off + ((a.cat_smem + 3) & ~3);
-    const size_t smem = (size_t)(a.wbuf_off + a.d * kTC) * 4;
     auto kern = score_kernel<EPI, M, DO>;
     int optin = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
-    if (smem > (size_t)optin)
+    // Shared memory of the launch with one or two L^{-1} tile buffers; the
+    // double buffer unless it costs a resident block per SM.
+    auto smem_for = [&](int single) {
+        a.single_l = single;
+        a.cat_off = (int32_t)(score_smem(a, EPI, DO) / 4);
+        a.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
+        a.wbuf_off = a.cat_off + ((a.cat_smem + 3) & ~3);
+        return (size_t)(a.wbuf_off + a.d * kTC) * 4;
+    };
+    int per_sm_single = 0, per_sm = 0;
+    const size_t smem_single = smem_for(1);
+    if (smem_single > (size_t)optin)
         return scoot_fail(ctx, SCOOT_EUNSUPPORTED,
                           "score kernel needs %zu bytes of shared memory (n = %d observations, %d boxes), the "
-                          "device allows %d", smem, a.n_obs, a.n_boxes, optin);
-    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    int per_sm = 0;
-    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));
+                          "device allows %d", smem_single, a.n_obs, a.n_boxes, optin);
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin));
+    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_single, kern, kThreads, smem_single));
+    size_t smem = smem_for(0);
+    if (smem <= (size_t)optin)
+        SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));
+    if (per_sm < per_sm_single) {
+        smem = smem_for(1);
+        per_sm = per_sm_single;
+    }
     if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "score kernel needs %zu bytes of shared memory", smem);
     const int64_t tiles = (a.n + kTC - 1) / kTC;
     int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
