@@ -834,7 +834,7 @@ def main():
     pkg.build()
     from paper_2408_04323_gb300 import scoot as S
     from paper_2408_04323_gb300.pipeline import RoundInputs, ScoringRound, State
-    from paper_2408_04323_gb300.shard import gather_mace_front, gather_topq
+    from paper_2408_04323_gb300.shard import gather_mace_front, gather_topq, sharded_fantasy_picks
     from workloads import WORKLOADS, Stream, draw_configs, make_instance, seeds, warp_params
 
     w = WORKLOADS[args.workload]
@@ -863,7 +863,11 @@ def main():
     stream = torch.cuda.current_stream(device)
 
     def exchange():
-        """The ranks' only exchange: their top-q lists, or for MACE their fronts."""
+        """The ranks' only exchange after a step: their top-q lists, or for
+        MACE their fronts (the fantasy round exchanges once per pick inside
+        the step instead)."""
+        if inp.fantasy:
+            return
         if inp.acq == "mace":
             f = int(rnd.top_count[1].item())
             if f > rnd.front_cap:
@@ -886,9 +890,14 @@ def main():
         if evs:
             evs[2].record(stream)
         if inp.fantasy:
-            S.scoot_suggest_fantasy(ctx, st.gp_layout, st.gp_state, st.fant_state, st.fant_box_cap, cand, N, st.eps,
-                                    inp.q, rnd.work, rnd.top_idx, rnd.top_val, rnd.top_count, mask=rnd.mask,
-                                    stream=stream)
+            if dist:  # the ranks' pools are shards of one pool of world x N candidates
+                sharded_fantasy_picks(S, ctx, st.gp_layout, st.gp_state, st.fant_state, st.fant_box_cap, cand, N,
+                                      st.eps, inp.q, rnd.work, rnd.top_idx, rnd.top_val, rnd.top_count,
+                                      index_offset=rank * N, mask=rnd.mask, stream=stream)
+            else:
+                S.scoot_suggest_fantasy(ctx, st.gp_layout, st.gp_state, st.fant_state, st.fant_box_cap, cand, N,
+                                        st.eps, inp.q, rnd.work, rnd.top_idx, rnd.top_val, rnd.top_count,
+                                        mask=rnd.mask, stream=stream)
             if evs:
                 evs[3].record(stream)
                 evs[4].record(stream)
@@ -954,6 +963,8 @@ def main():
     # host gaps).
     graph = None
     try:
+        if dist and inp.fantasy:
+            raise RuntimeError("the sharded fantasy round exchanges records between its launches")
         cap = torch.cuda.Stream(device)
         cap.wait_stream(stream)
         graph = torch.cuda.CUDAGraph()
@@ -1101,7 +1112,11 @@ def main():
             S.scoot_prune(ctx, inp.space, inp.clauses, cand_e2e, N, rnd.mask, None, stream)
             S.scoot_rf_predict(ctx, state.forest_layout, state.forest, inp.space, cand_e2e, N, inp.delta_num,
                                inp.delta_den, rnd.votes, rnd.mask, None, stream)
-            if inp.fantasy:
+            if inp.fantasy and dist:
+                sharded_fantasy_picks(S, ctx, state.gp_layout, state.gp_state, state.fant_state, state.fant_box_cap,
+                                      cand_e2e, N, state.eps, inp.q, rnd.work, rnd.top_idx, rnd.top_val,
+                                      rnd.top_count, index_offset=rank * N, mask=rnd.mask, stream=stream)
+            elif inp.fantasy:
                 S.scoot_suggest_fantasy(ctx, state.gp_layout, state.gp_state, state.fant_state, state.fant_box_cap,
                                         cand_e2e, N, state.eps, inp.q, rnd.work, rnd.top_idx, rnd.top_val,
                                         rnd.top_count, mask=rnd.mask, stream=stream)
