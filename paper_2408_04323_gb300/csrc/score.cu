@@ -26,7 +26,8 @@ constexpr int kTC = 32;     // candidates per tile
 constexpr int kThreads = 128;  // four threads per candidate
 constexpr int kQ = kThreads / kTC;  // threads per candidate (= warps: warp w is quarter w)
 constexpr int kRB = 64;     // rows of L^{-1} per tile
-constexpr int kCJ = 32;     // columns of L^{-1} per tile
+constexpr int kCJ = 32;     // columns of L^{-1} per host tile
+constexpr int kCH = 16;     // columns of L^{-1} per staged half tile (4 KiB)
 constexpr int kMaxD = SCOOT_MAX_DIM;
 constexpr int kMaxM = SCOOT_MAX_OBJ;
 constexpr int kAcqThreads = 128;
@@ -62,7 +63,6 @@ struct ScoreArgs {
     int32_t cat_smem;             // floats of the categorical table staged in shared memory (0: read from L1)
     int32_t cat_off;              // where, in floats from the start of shared memory
     int32_t wbuf_off;             // the next tile's pool words [d][kTC], in floats from the start
-    int32_t single_l;             // 1: one L^{-1} tile buffer (more blocks per SM), 0: double buffering
     float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad / 4][ldv][4] by list position
     int64_t ldv;
     uint32_t* err;                // device error word
@@ -105,12 +105,13 @@ __device__ __forceinline__ float ehvi_partial(const float* mu, const float* sd, 
     return total;
 }
 
-// Asynchronous copy of one 32 x 64 tile of L^{-1} (8 KiB, 16-byte aligned at
-// both ends) into shared memory: each of the 128 threads moves four 16-byte
-// pieces with cp.async and commits them as one group.
+// Asynchronous copy of one half of a 32 x 64 tile of L^{-1} (16 columns x 64
+// rows, 4 KiB, contiguous in the host's transposed tile layout and 16-byte
+// aligned at both ends) into shared memory: each of the 128 threads moves two
+// 16-byte pieces with cp.async and commits them as one group.
 __device__ __forceinline__ void stage_tile_async(float* dst, const float4* src, int tid) {
 #pragma unroll
-    for (int k = 0; k < kCJ * kRB / 4 / kThreads; ++k) {
+    for (int k = 0; k < kCH * kRB / 4 / kThreads; ++k) {
         const unsigned s = (unsigned)__cvta_generic_to_shared(dst + 4 * (tid + k * kThreads));
         asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(src + tid + k * kThreads) : "memory");
     }
@@ -159,12 +160,9 @@ template <int EPI, int M, int DO>
 __global__ void __launch_bounds__(kThreads, (EPI == kEHVI && M == 2 && DO == 8) ? 6 : 4)
 score_kernel(const __grid_constant__ ScoreArgs a) {
     // At least four blocks (16 warps) per SM: registers capped at 128 (80 for
-    // the 2-objective EHVI of <= 8 parameters, six blocks).  When the L^{-1}
-    // double buffer would cost a block per SM of shared memory, the launch
-    // asks for a single buffer (a.single_l): the tile loads are then hidden
-    // by the other blocks rather than by double buffering.
+    // the 2-objective EHVI of <= 8 parameters, six blocks).  L^{-1} is staged
+    // in half tiles of 16 columns, double-buffered: 8 KiB in all.
     constexpr bool kRegCapped = EPI == kEHVI && M == 2 && DO == 8;
-    const bool kSingleL = a.single_l != 0;  // the same in every thread
     extern __shared__ __align__(16) float sm[];
     const int n_pad = a.n_rb * kRB;
     // Ks, and after the posterior the exact-EHVI psi table [psi_rows][kTC]
@@ -172,8 +170,8 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
     float* Ks = sm;                                                   // [n_pad][kTC]
     float* xs = Ks + (size_t)ks_rows * kTC;                           // [n_obs][DO] ordinal features
     float* al = xs + (size_t)a.n_obs * DO;                            // [n_pad]
-    float* Lt = al + n_pad;                                           // [2][kCJ][kRB] double buffer
-    float* part = Lt + (kSingleL ? 1 : 2) * kCJ * kRB;                // [16][kTC]
+    float* Lt = al + n_pad;                                           // [2][kCH][kRB] double buffer
+    float* part = Lt + 2 * kCH * kRB;                                 // [16][kTC]
     float4* fm = reinterpret_cast<float4*>(part + 16 * kTC);          // [kMaxD] feature map
     float4* blo = fm + kMaxD;                          // [B] (general boxes) or [2B] (saturated form)
     float4* bhi = blo + (EPI == kEHVI ? a.n_boxes : 0);
@@ -250,7 +248,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
         for (int m = 0; m < nobj; ++m) {
             __syncthreads();  // previous users of xs / al / part / Lt are done
             const float4* tiles = glinv + (size_t)m * a.n_tiles * (kCJ * kRB / 4);
-            stage_tile_async(Lt, tiles, tid);  // tile 0 lands while the covariance row is computed
+            stage_tile_async(Lt, tiles, tid);  // half tile 0 lands while the covariance row is computed
             const float* sx = gxs + (size_t)m * a.n_obs * a.d;
             for (int e = tid; e < a.n_obs * DO; e += kThreads) {
                 const int j = e / DO, q = e - j * DO;
@@ -312,24 +310,24 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 float2 acc2[4][2];
 #pragma unroll
                 for (int r = 0; r < 4; ++r) acc2[r][0] = acc2[r][1] = make_float2(0.0f, 0.0f);
-                for (int cj = 0; cj < 2 * (rb + 1); ++cj, ++t) {
-                    // Tile t has landed in buffer t&1 and every thread is done
-                    // with tile t-1, so tile t+1 may overwrite buffer (t+1)&1
-                    // while tile t is multiplied.
+                for (int ch = 0; ch < 4 * (rb + 1); ++ch, ++t) {
+                    // Half tile t (columns 16 ch .. 16 ch + 15 of this row
+                    // block's tiles) has landed in buffer t&1 and every thread
+                    // is done with half tile t-1, so half tile t+1 may
+                    // overwrite buffer (t+1)&1 while t is multiplied.
                     cp_async_wait_all();
                     __syncthreads();
-                    if (!kSingleL && t + 1 < a.n_tiles)
-                        stage_tile_async(Lt + ((t + 1) & 1) * (kCJ * kRB), tiles + (size_t)(t + 1) * (kCJ * kRB / 4), tid);
-                    const float4* Lt4 = reinterpret_cast<const float4*>(Lt + (kSingleL ? 0 : (t & 1)) * (kCJ * kRB));
-                    // rows of this warp: rb*64 + 16*warp .. +15; columns cj*32 .. +31;
+                    if (t + 1 < 2 * a.n_tiles)
+                        stage_tile_async(Lt + ((t + 1) & 1) * (kCH * kRB), tiles + (size_t)(t + 1) * (kCH * kRB / 4), tid);
+                    const float4* Lt4 = reinterpret_cast<const float4*>(Lt + (t & 1) * (kCH * kRB));
+                    // rows of this warp: rb*64 + 16*warp .. +15; columns ch*16 .. +15;
                     // L^{-1} is zero right of the diagonal, so a warp stops at its
-                    // last row (in steps of 16 columns).
-                    const int j0 = cj * kCJ;
+                    // last row.
+                    const int j0 = ch * kCH;
                     const int last_row = rb * kRB + 16 * warp + 15;
-                    if (!kSingleL && j0 > last_row) continue;  // (single buffer: every thread reaches the staging below)
-                    const int jj_end = j0 > last_row ? 0 : (last_row - j0 + 1 >= kCJ ? kCJ : 16);
+                    if (j0 > last_row) continue;
 #pragma unroll 8
-                    for (int jj = 0; jj < jj_end; ++jj) {
+                    for (int jj = 0; jj < kCH; ++jj) {
                         const float4 k4 = Ks4[(j0 + jj) * (kTC / 4) + cg];
                         const float4 l4 = Lt4[jj * (kRB / 4) + rg];
                         const float2 k01 = make_float2(k4.x, k4.y), k23 = make_float2(k4.z, k4.w);
@@ -347,10 +345,6 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                                 acc2[r][1] = __ffma2_rn(lb, k23, acc2[r][1]);
                             }
                         }
-                    }
-                    if (kSingleL && t + 1 < a.n_tiles) {  // every thread is done with tile t
-                        __syncthreads();
-                        stage_tile_async(Lt, tiles + (size_t)(t + 1) * (kCJ * kRB / 4), tid);
                     }
                 }
                 float accm[4][4];
@@ -611,8 +605,7 @@ constexpr int kCatSmemMax = 1024;  // floats of categorical table worth staging 
 size_t score_smem(const ScoreArgs& a, int epi, int DO) {
     const size_t n_pad = (size_t)a.n_rb * kRB;
     const size_t ks_rows = epi == kEHVIX && (size_t)a.psi_rows > n_pad ? (size_t)a.psi_rows : n_pad;
-    const size_t l_bufs = a.single_l ? 1 : 2;
-    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + l_bufs * kCJ * kRB + 16 * kTC + 4 * kMaxD;
+    size_t f = ks_rows * kTC + (size_t)a.n_obs * DO + n_pad + 2 * kCH * kRB + 16 * kTC + 4 * kMaxD;
     if (epi == kEHVI) f += (size_t)(2 * a.n_boxes + a.n_mc) * 4;
     if (epi == kEHVIX) f += (size_t)((a.psi_rows + 3) & ~3) + (size_t)a.n_boxes * kMaxM;
     return f * 4;
@@ -626,30 +619,17 @@ scoot_status launch_score_dm(scoot_ctx* ctx, ScoreArgs a, cudaStream_t st) {
     auto kern = score_kernel<EPI, M, DO>;
     int optin = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
-    // Shared memory of the launch with one or two L^{-1} tile buffers; the
-    // double buffer unless it costs a resident block per SM.
-    auto smem_for = [&](int single) {
-        a.single_l = single;
-        a.cat_off = (int32_t)(score_smem(a, EPI, DO) / 4);
-        a.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
-        a.wbuf_off = a.cat_off + ((a.cat_smem + 3) & ~3);
-        return (size_t)(a.wbuf_off + a.d * kTC) * 4;
-    };
-    int per_sm_single = 0, per_sm = 0;
-    const size_t smem_single = smem_for(1);
-    if (smem_single > (size_t)optin)
+    a.cat_off = (int32_t)(score_smem(a, EPI, DO) / 4);
+    a.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
+    a.wbuf_off = a.cat_off + ((a.cat_smem + 3) & ~3);
+    const size_t smem = (size_t)(a.wbuf_off + a.d * kTC) * 4;
+    if (smem > (size_t)optin)
         return scoot_fail(ctx, SCOOT_EUNSUPPORTED,
                           "score kernel needs %zu bytes of shared memory (n = %d observations, %d boxes), the "
-                          "device allows %d", smem_single, a.n_obs, a.n_boxes, optin);
-    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin));
-    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_single, kern, kThreads, smem_single));
-    size_t smem = smem_for(0);
-    if (smem <= (size_t)optin)
-        SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));
-    if (per_sm < per_sm_single) {
-        smem = smem_for(1);
-        per_sm = per_sm_single;
-    }
+                          "device allows %d", smem, a.n_obs, a.n_boxes, optin);
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    int per_sm = 0;
+    SCOOT_CUDA(ctx, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem));
     if (per_sm < 1) return scoot_fail(ctx, SCOOT_EUNSUPPORTED, "score kernel needs %zu bytes of shared memory", smem);
     const int64_t tiles = (a.n + kTC - 1) / kTC;
     int64_t blocks = (int64_t)sm_count(ctx->device) * per_sm;
