@@ -50,9 +50,13 @@ KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["scor
                 "posterior": ["score.cu", "device_common.cuh"], "fant_pass": ["fantasy.cu", "device_common.cuh"],
                 "topq": ["topq.cu", "device_common.cuh"], "pareto": ["pareto.cu"]}
 TRAFFIC = {
-    ("prune", "d8-ehvi2"): {"bytes": 3151360, "sha": "669855124f47da70"},
-    ("rf", "d8-ehvi2"): {"bytes": 8809728, "sha": "669855124f47da70"},
-    ("score", "d8-ehvi2"): {"bytes": 8858112, "sha": "3ee4c80f5161c740"},
+    # d12-fantasy: captured on a 2^20 pool of the same workload, scaled to the 2^22 launch by its
+    # live candidates (x 4.0025; fant_pass and the posterior) or its pool size (x 4; prune, forest)
+    ("fant_pass", "d12-fantasy"): {"bytes": 3562300000, "sha": "aa97db9cc922aeb9"},
+    ("posterior", "d12-fantasy"): {"bytes": 3485600000, "sha": "6b2aeb7ebc645ff4"},
+    ("rf", "d12-fantasy"): {"bytes": 210480000, "sha": "f14ca23df538ac20"},
+    ("prune", "d12-fantasy"): {"bytes": 100680000, "sha": "f14ca23df538ac20"},
+    ("score", "d10-ehvi3"): {"bytes": 44739000, "sha": "6b2aeb7ebc645ff4"},
 }
 
 
@@ -1049,9 +1053,11 @@ def main():
         kernels[last] = hbm_roof(work[last][1] * N, stage_ms[last], last)
         kernel_ms = {k: stage_ms[k] for k in stage_names}
     dom = max((k for k in kernels), key=lambda k: kernel_ms[k] if k in kernel_ms else 0.0)
+    tag = w.name if inp.acq == w.acq and args.pool in (None, w.n_cand) else None
+    for k, v in kernels.items():  # DRAM bytes per launch from ncu, while the kernel's sources are unchanged
+        tr = TRAFFIC.get((k, tag))
+        v["traffic"] = tr["bytes"] if tr and tr["sha"] == sources_sha(k) else None
     roof = dict(kernels[dom])
-    tr = TRAFFIC.get((dom, w.name if inp.acq == w.acq else f"{w.name}/{inp.acq}"))
-    roof["traffic"] = tr["bytes"] if tr and tr["sha"] == sources_sha(tr.get("stage", dom)) else None
     roof["peak_source"] = (f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if roof["bound"] == "hbm" else
                            "FP32 = SMs x 128 lanes x 2 x max SM clock (nominal; measured FFMA peaks in probes)")
     stage_roofs = {k: round(v["frac"], 4) for k, v in kernels.items()}
@@ -1073,7 +1079,7 @@ def main():
                               "frac_of_smem_gather_peak": rate / probes["smem_gather_visits_per_s"]})
         if inp.fantasy:
             kernels["fant_pass"]["ehvi_flops_per_launch"] = n_feasible * inp.eps.shape[0] * st.n_boxes * 4 * inst.n_obj
-        roof = dict(kernels[dom], traffic=roof["traffic"], peak_source=roof["peak_source"])
+        roof = dict(kernels[dom], peak_source=roof["peak_source"])
 
     # end to end through the C ABI from pinned host buffers
     e2e = None
