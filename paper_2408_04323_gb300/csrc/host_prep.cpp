@@ -18,7 +18,7 @@ namespace {
 constexpr int64_t kAlign = 256;
 constexpr int kRowBlock = 64;   // rows of L^{-1} per tile
 constexpr int kColChunk = 32;   // columns of L^{-1} per tile
-constexpr int kForestChunkNodes = 12288;  // 96 KiB of nodes staged at a time
+constexpr int kForestChunkNodes = 6144;   // 48 KiB of nodes staged at a time: four forest blocks per SM
 constexpr int kMaxPatterns = 4096;        // joint category patterns of the GP's categorical table
 
 int64_t align_up(int64_t x) { return (x + kAlign - 1) / kAlign * kAlign; }

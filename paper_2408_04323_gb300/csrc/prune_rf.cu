@@ -126,7 +126,6 @@ struct RfArgs {
     uint8_t* mask;
     unsigned long long* count;
     uint32_t* err;
-    int32_t single_chunk;
     const int32_t* list;          // live candidates (NULL: all of 0 .. n-1)
     const unsigned int* n_list;
     int32_t max_chunk_nodes;
@@ -172,40 +171,41 @@ rf_kernel(const __grid_constant__ RfArgs a) {
         }
         for (int k = tid; k < nt; k += kRfThreads) sroot[t0 + k] = roots[t0 + k] - first_node;
     };
-    if (a.single_chunk) stage_chunk(0);  // visible after the first barrier below
-
-    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-        const int64_t base = tile * kRfCand;
-        __syncthreads();  // the previous tile's features and votes are no longer read
-        for (int k = tid; k < kRfCand * a.d; k += kRfThreads) {
-            const int f = k / kRfCand, c = k - f * kRfCand;
-            const int64_t pos = base + c;
-            float x = 0.0f;
-            if (pos < n_work) {
-                const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
-                const uint32_t w = __ldg(a.cand + (int64_t)f * a.ld + i);
-                x = ((a.float_cols >> f) & 1u) ? __uint_as_float(w) : (float)(int32_t)w;
-            }
-            sfeat[c * fs + f] = x;
-        }
-        const int64_t pos = base + slot;
-        const bool live = pos < n_work;
-        const char* my = reinterpret_cast<const char*>(sfeat + slot * fs);
-        uint32_t vote = 0;
-        for (int ch = 0; ch < a.n_chunks; ++ch) {
-            if (!a.single_chunk) {
-                __syncthreads();
-                stage_chunk(ch);
+    // Chunk-major: the block walks all of its tiles with chunk 0 of the
+    // forest, then all of them with chunk 1, ..., carrying each candidate's
+    // partial vote count in votes[] between chunks (the tiles of a block are
+    // the same in every chunk), so that a chunk of <= 48 KiB lets four
+    // blocks share an SM.
+    for (int ch = 0; ch < a.n_chunks; ++ch) {
+        const bool first = ch == 0, last = ch + 1 == a.n_chunks;
+        __syncthreads();  // the previous chunk's nodes are no longer read
+        stage_chunk(ch);  // visible after the first barrier below
+        const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
+        for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+            const int64_t base = tile * kRfCand;
+            __syncthreads();  // the previous tile's features and votes are no longer read
+            for (int k = tid; k < kRfCand * a.d; k += kRfThreads) {
+                const int f = k / kRfCand, c = k - f * kRfCand;
+                const int64_t pos = base + c;
+                float x = 0.0f;
+                if (pos < n_work) {
+                    const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+                    const uint32_t w = __ldg(a.cand + (int64_t)f * a.ld + i);
+                    x = ((a.float_cols >> f) & 1u) ? __uint_as_float(w) : (float)(int32_t)w;
+                }
+                sfeat[c * fs + f] = x;
             }
             __syncthreads();
-            const int t0 = chunks[ch * 4 + 0], nt = chunks[ch * 4 + 1];
-            if (!live) continue;
+            const int64_t pos = base + slot;
+            const bool live = pos < n_work;
+            const char* my = reinterpret_cast<const char*>(sfeat + slot * fs);
+            uint32_t vote = 0;
             // The lanes of a warp walk the same tree (for 32 candidates) in
             // lockstep, so the upper levels of the tree are broadcast loads;
             // letting each lane run on to its next tree as soon as it reaches
             // a leaf was measured twice as slow: the lanes drift onto
             // different trees and the node loads stop being broadcasts.
-            for (int t = t0 + grp; t < t0 + nt; t += kRfGroups) {
+            for (int t = t0 + grp; t < t0 + nt && live; t += kRfGroups) {
                 int node = sroot[t];
                 bool done = false;
 #pragma unroll 2
@@ -221,19 +221,22 @@ rf_kernel(const __grid_constant__ RfArgs a) {
                 }
                 if (!done) atomicOr(a.err, SCOOT_DEVERR_INDEX);  // deeper than the validated depth
             }
-        }
-        svote[grp * kRfCand + slot] = vote;
-        __syncthreads();
-        if (grp == 0 && live) {
-            uint32_t v = 0;
+            svote[grp * kRfCand + slot] = vote;
+            __syncthreads();
+            if (grp == 0 && live) {
+                uint32_t v = 0;
 #pragma unroll
-            for (int g = 0; g < kRfGroups; ++g) v += svote[g * kRfCand + slot];
-            const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
-            const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
-            a.votes[i] = v;
-            const bool ok = (unsigned __int128)a.delta_den * v >= need;
-            if (a.mask) a.mask[i] = ok;
-            feasible += ok;
+                for (int g = 0; g < kRfGroups; ++g) v += svote[g * kRfCand + slot];
+                const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+                if (!first) v += a.votes[i];  // the earlier chunks' count (written by this thread)
+                a.votes[i] = v;
+                if (last) {
+                    const unsigned __int128 need = (unsigned __int128)a.delta_num * a.leaf_scale * (uint32_t)a.n_trees;
+                    const bool ok = (unsigned __int128)a.delta_den * v >= need;
+                    if (a.mask) a.mask[i] = ok;
+                    feasible += ok;
+                }
+            }
         }
     }
     if (a.count) add_count(a.count, feasible);
@@ -346,7 +349,6 @@ scoot_status scoot_rf_predict(scoot_ctx* ctx, const scoot_forest_layout* L, cons
     a.mask = mask;
     a.count = reinterpret_cast<unsigned long long*>(n_feasible);
     a.err = ctx->d_err;
-    a.single_chunk = L->n_chunks == 1;
     if (mask) {
         // Walk only the candidates still in play; the others get 0 votes.
         ScootList lst;
