@@ -22,11 +22,18 @@
 //   pick j   fant_pass (every live candidate): the downdate of pick j-1, which
 //            reads the candidate's rows of V once, then its EHVI over the
 //            boxes staged in shared memory, and a per-block argmax;
-//            fant_pick (one block per objective): the argmax, then the pick's
-//            rank-1 terms in fp64 from the fantasy state (k(X, x_p),
-//            v_p = L^{-1} k, mu(x_p), c_l(x_p), s_j); the last block to finish
-//            adds the fantasised point to the front and rebuilds the boxes.
+//            fant_pick (column slabs x objectives): the argmax, then the pick's
+//            rank-1 terms in fp64 from the fantasy state: each block takes a
+//            slab of columns of L^{-1} and forms its part of v_p = L^{-1} k and
+//            of mu(x_p); the last slab of an objective sums the parts and
+//            solves for c_l(x_p) and s_j; the last objective adds the
+//            fantasised point to the front and rebuilds the boxes.
+// GB300 runs fp64 on a narrow pipe (a dependent fp64 operation costs on the
+// order of a hundred cycles), so the pick spreads its fp64 work over many
+// blocks, keeps dependent chains short (the fantasy factor is kept inverted,
+// so its solve is a product), and compares front values as integer keys.
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstring>
 
@@ -40,7 +47,10 @@ using namespace scoot_dev;
 constexpr int kPassThreads = 256;
 constexpr int kPickThreads = 256;
 constexpr int kPartMax = 2048;   // per-block argmax partials of one pass
-constexpr int kPickRows = 8;     // row blocks per objective of the pick's L^{-1} k product
+constexpr int kPickSlabMax = 32;  // column slabs per objective of the pick's L^{-1} k product
+
+// Column slabs of the pick's product for n observations: about eight columns each.
+inline int pick_slabs(int n) { return std::min(kPickSlabMax, std::max(1, (n + 7) / 8)); }
 
 // Control words of one call, in the work buffer.
 struct Ctrl {
@@ -80,8 +90,11 @@ struct FantArgs {
     float* inv_s;                 // [M] 1 / s of the latest pick
     double* upick;                // [q][d] features of the picks
     double* vpick;                // [q][M][n] v_p of the picks
-    double* cpick;                // [q][M][q] c_l(x_p) of the picks
-    double* spick;                // [q][M]
+    double* wf;                   // [M][q][q] inverse of each objective's fantasy factor (row-major, lower)
+    double* part;                 // [M][n_slab][n] each slab's part of v_p
+    double* mupart;               // [M][n_slab] each slab's part of mu(x_p)
+    double* kpt;                  // [M][q] k(x_p, x_{p_t}) of the earlier picks
+    int32_t n_slab, slab_w;       // column slabs of the pick's product and their width
     double* mupick;               // [q][M] fantasised values
     uint64_t* part_key;           // [kPartMax]
     int32_t* part_pos;
@@ -121,16 +134,35 @@ __device__ __forceinline__ void block_keymax(uint64_t& k, int32_t& p) {
     __syncthreads();
 }
 
+// Sum over a block of kPickThreads threads: the same value, summed in the
+// same order, in every thread.
 __device__ __forceinline__ double block_sum(double v, double* scratch) {
+    static_assert(kPickThreads == 256, "the tree below sums eight warps");
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     __syncthreads();
     if (lane == 0) scratch[warp] = v;
     __syncthreads();
-    double t = 0.0;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += scratch[w];  // same order in every thread
-    return t;
+    const double* w = scratch;
+    return ((w[0] + w[1]) + (w[2] + w[3])) + ((w[4] + w[5]) + (w[6] + w[7]));
 }
+
+// Sum over warp 0's lanes of v (fixed order), in every lane of warp 0.
+__device__ __forceinline__ double warp_sum(double v) {
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Order-preserving integer key of a double: x < y exactly when key(x) <
+// key(y), for values that are not NaN; -0 and +0 share the key of +0.  The
+// front and box logic compares these keys on the integer pipes.
+__device__ __forceinline__ long long okey(double x) {
+    long long b = __double_as_longlong(x);
+    if (b == LLONG_MIN) b = 0;  // -0
+    return b >= 0 ? b : b ^ LLONG_MAX;
+}
+
+__device__ __forceinline__ double okey_value(long long k) { return __longlong_as_double(k >= 0 ? k : k ^ LLONG_MAX); }
 
 __device__ __forceinline__ double matern64(double r, int kernel) {
     if (kernel == SCOOT_MATERN32) {
@@ -182,23 +214,30 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
                                        char* smem) {
     constexpr int G = M - 1;
     const int fcap = a.front_cap;
-    double* cell = reinterpret_cast<double*>(smem);               // [box_cap] floor of each grid cell
-    double* F = cell + a.box_cap;                                  // [fcap][M]
-    double* axis = F + (size_t)fcap * M;                           // [G][fcap + 1]
+    // Every value below is an order-preserving key (okey).
+    long long* cell = reinterpret_cast<long long*>(smem);           // [box_cap] floor of each grid cell
+    long long* F = cell + a.box_cap;                                 // [fcap][M]
+    long long* axis = F + (size_t)fcap * M;                          // [G][fcap + 1]
     int32_t* first = reinterpret_cast<int32_t*>(axis + (size_t)G * (fcap + 1));  // [fcap + 1]
     int32_t* rowcnt = first + fcap + 1;                                            // [rows + 1]
     __shared__ int32_t s_nf, s_A[4], s_total, s_ok;
+    __shared__ long long s_ref[M];
     const int tid = threadIdx.x;
     if (tid == 0) s_nf = a.ctrl->n_front;
+    if (tid < M) s_ref[tid] = okey(h.ref[tid]);
     __syncthreads();
-    for (int e = tid; e < s_nf * M; e += blockDim.x) F[e] = a.front[e];
+    for (int e = tid; e < s_nf * M; e += blockDim.x) F[e] = okey(a.front[e]);
     __syncthreads();
     if (add && tid == 0) {
+        long long zk[M];
         bool above = true, covered = false;
-        for (int m = 0; m < M; ++m) above &= z[m] > h.ref[m];
+        for (int m = 0; m < M; ++m) {
+            zk[m] = okey(z[m]);
+            above &= zk[m] > s_ref[m];
+        }
         for (int k = 0; k < s_nf && !covered; ++k) {
             bool ge = true;
-            for (int m = 0; m < M; ++m) ge &= F[k * M + m] >= z[m];
+            for (int m = 0; m < M; ++m) ge &= F[k * M + m] >= zk[m];
             covered = ge;
         }
         if (above && !covered) {
@@ -206,15 +245,15 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
             for (int k = 0; k < s_nf; ++k) {
                 bool ge = true, gt = false;
                 for (int m = 0; m < M; ++m) {
-                    ge &= z[m] >= F[k * M + m];
-                    gt |= z[m] > F[k * M + m];
+                    ge &= zk[m] >= F[k * M + m];
+                    gt |= zk[m] > F[k * M + m];
                 }
                 if (ge && gt) continue;  // dominated by the fantasy
                 for (int m = 0; m < M; ++m) F[w * M + m] = F[k * M + m];
                 ++w;
             }
             if (w < fcap) {
-                for (int m = 0; m < M; ++m) F[w * M + m] = z[m];
+                for (int m = 0; m < M; ++m) F[w * M + m] = zk[m];
                 ++w;
             } else {
                 atomicOr(a.err, SCOOT_DEVERR_CAPACITY);
@@ -224,23 +263,23 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
     }
     __syncthreads();
     const int nf = s_nf;
-    for (int e = tid; e < nf * M; e += blockDim.x) a.front[e] = F[e];
+    for (int e = tid; e < nf * M; e += blockDim.x) a.front[e] = okey_value(F[e]);
     // Axes: {r_j} and the front's coordinates, sorted and unique.  Value t
     // (t = 0 the reference, t = k + 1 front point k) is kept if no earlier t
     // holds the same value; its place is the number of kept values below it.
     for (int j = 0; j < G; ++j) {
         for (int t = tid; t <= nf; t += blockDim.x) {
-            const double v = t == 0 ? h.ref[j] : F[(t - 1) * M + j];
+            const long long v = t == 0 ? s_ref[j] : F[(t - 1) * M + j];
             int f = 1;
-            for (int u = 0; u < t && f; ++u) f = (u == 0 ? h.ref[j] : F[(u - 1) * M + j]) != v;
+            for (int u = 0; u < t && f; ++u) f = (u == 0 ? s_ref[j] : F[(u - 1) * M + j]) != v;
             first[t] = f;
         }
         __syncthreads();
         for (int t = tid; t <= nf; t += blockDim.x) {
             if (!first[t]) continue;
-            const double v = t == 0 ? h.ref[j] : F[(t - 1) * M + j];
+            const long long v = t == 0 ? s_ref[j] : F[(t - 1) * M + j];
             int below = 0;
-            for (int u = 0; u <= nf; ++u) below += first[u] && (u == 0 ? h.ref[j] : F[(u - 1) * M + j]) < v;
+            for (int u = 0; u <= nf; ++u) below += first[u] && (u == 0 ? s_ref[j] : F[(u - 1) * M + j]) < v;
             axis[j * (fcap + 1) + below] = v;
         }
         if (tid == 0) {
@@ -263,22 +302,22 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
         return;
     }
     // Floor of every cell (row-major over the grid, the last axis fastest).
-    const double inf = __longlong_as_double(0x7ff0000000000000ll);
+    const long long inf = okey(__longlong_as_double(0x7ff0000000000000ll));
     for (int c = tid; c < cells; c += blockDim.x) {
-        double up[G];
+        long long up[G];
         int rest = c;
         for (int j = G - 1; j >= 0; --j) {
             const int kj = rest % s_A[j];
             rest /= s_A[j];
             up[j] = kj + 1 < s_A[j] ? axis[j * (fcap + 1) + kj + 1] : inf;
         }
-        double hh = -inf;
+        long long hh = s_ref[M - 1];
         for (int k = 0; k < nf; ++k) {
             bool dom = true;
             for (int j = 0; j < G; ++j) dom &= F[k * M + j] >= up[j];
-            if (dom) hh = fmax(hh, F[k * M + M - 1]);
+            if (dom) hh = max(hh, F[k * M + M - 1]);
         }
-        cell[c] = fmax(h.ref[M - 1], hh);
+        cell[c] = hh;
     }
     __syncthreads();
     // Boxes per row (cells merged while the floor repeats), then their offsets.
@@ -296,30 +335,29 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
     }
     __syncthreads();
     for (int r = tid; r < rows && s_ok; r += blockDim.x) {
-        double lo_pre[G > 1 ? G - 1 : 1], up_pre[G > 1 ? G - 1 : 1];
+        float lo_pre[G > 1 ? G - 1 : 1], up_pre[G > 1 ? G - 1 : 1];
         int rest = r;
         for (int j = G - 2; j >= 0; --j) {
             const int kj = rest % s_A[j];
             rest /= s_A[j];
-            lo_pre[j] = axis[j * (fcap + 1) + kj];
-            up_pre[j] = kj + 1 < s_A[j] ? axis[j * (fcap + 1) + kj + 1] : inf;
+            lo_pre[j] = (float)okey_value(axis[j * (fcap + 1) + kj]);
+            up_pre[j] = kj + 1 < s_A[j] ? (float)okey_value(axis[j * (fcap + 1) + kj + 1]) : __int_as_float(0x7f800000);
         }
         int b = rowcnt[r] - 1;
-        const double* al = axis + (G - 1) * (fcap + 1);
+        const long long* al = axis + (G - 1) * (fcap + 1);
         for (int kk = 0; kk < A_last; ++kk) {
-            const double fl = cell[r * A_last + kk];
-            const double upl = kk + 1 < A_last ? al[kk + 1] : inf;
+            const long long fl = cell[r * A_last + kk];
             if (kk == 0 || fl != cell[r * A_last + kk - 1]) {
                 ++b;
                 for (int j = 0; j < G - 1; ++j) {
-                    a.box_lo[b * M + j] = (float)lo_pre[j];
-                    a.box_hi[b * M + j] = (float)up_pre[j];
+                    a.box_lo[b * M + j] = lo_pre[j];
+                    a.box_hi[b * M + j] = up_pre[j];
                 }
-                a.box_lo[b * M + G - 1] = (float)al[kk];
-                a.box_lo[b * M + M - 1] = (float)fl;
+                a.box_lo[b * M + G - 1] = (float)okey_value(al[kk]);
+                a.box_lo[b * M + M - 1] = (float)okey_value(fl);
                 a.box_hi[b * M + M - 1] = __int_as_float(0x7f800000);
             }
-            a.box_hi[b * M + G - 1] = (float)upl;
+            a.box_hi[b * M + G - 1] = kk + 1 < A_last ? (float)okey_value(al[kk + 1]) : __int_as_float(0x7f800000);
         }
     }
     __syncthreads();
@@ -532,28 +570,25 @@ __global__ void __launch_bounds__(kPassThreads, M == 2 ? 4 : 1) fant_pass(const 
     pass_record(a);
 }
 
-// First row of slice r of R slices of the rows of a lower triangle of order
-// n with equal areas (row i holds i + 1 entries).
-__device__ __forceinline__ int tri_row(int r, int R, int n) {
-    if (r <= 0) return 0;
-    if (r >= R) return n;
-    return min(n, (int)ceil(sqrt((double)r / R) * n));
-}
-
-// Pick j, on a grid of kPickRows x M blocks.  Every block reduces the pass's
-// partials to the argmax; block (0, 0) records the pick.  Block (r, m) then
-// computes slice r of v_p = L^{-1} k(X, x_p) of objective m in fp64 (and,
-// for r = 0, mu(x_p)).  The last slice of objective m to finish completes
-// that objective's terms (|v_p|^2, v_p . v_{p_t}, the c_t(x_p) recurrence,
-// s_j) and the fp32 copies the next pass reads; the last objective to finish
-// adds the fantasised point to the front and rebuilds the boxes.
+// Pick j, on a grid of n_slab x M blocks.  Every block reduces the shards'
+// records to the winner; block (0, 0) records the pick.  Block (b, m) then
+// evaluates k(X_c, x_p) of objective m for the columns c of slab b, and
+// forms that slab's part of v_p = L^{-1} k (sum over its columns, every row
+// below them) and of mu(x_p) = alpha . k, plus k(x_p, x_{p_t}) for the
+// earlier picks t = b, b + n_slab, ...  The last slab of objective m to
+// finish sums the parts (in slab order) and completes that objective's
+// terms: |v_p|^2, v_p . v_{p_t}, c(x_p) = W (k(x_p, x_{p_t}) - v_p . v_{p_t})
+// with W the inverse of the fantasy factor (row t: c_l(x_{p_t}) for l < t,
+// s_t on the diagonal), s_j, the new row of W, and the fp32 copies the next
+// pass reads.  The last objective to finish adds the fantasised point to
+// the front and rebuilds the boxes.
 template <int M>
 __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant__ FantArgs a, int j,
                                                           const uint64_t* recs, int n_rec) {
     extern __shared__ __align__(16) char smem[];
     if (*(volatile const uint32_t*)&a.ctrl->done) return;
     const FantHeader& h = *reinterpret_cast<const FantHeader*>(a.fant);
-    const int tid = threadIdx.x, r = blockIdx.x, m = blockIdx.y, R = gridDim.x;
+    const int tid = threadIdx.x, b = blockIdx.x, m = blockIdx.y, B = gridDim.x;
     // The winning record: the largest selection key over the shards.
     __shared__ uint64_t s_best;
     __shared__ int32_t s_win;
@@ -573,7 +608,7 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
     }
     __syncthreads();
     const uint64_t best = s_best;
-    const bool lead = r == 0 && m == 0;
+    const bool lead = b == 0 && m == 0;
     if (best == 0ull) {  // no eligible candidate left on any shard: the picks end here
         if (lead && tid == 0) a.ctrl->done = 1u;
         return;
@@ -602,17 +637,20 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
     const double sf2 = h.sf2[m], tau2 = h.tau2[m];
     double* u = reinterpret_cast<double*>(smem);     // [16] features of the pick
     double* il = u + 16;                              // [16] 1/l (ordinal) or 1/l^2 (categorical)
-    double* ks = il + 16;                             // [n] k(X, x_p)
-    double* red = ks + n;                             // [32] reduction scratch
-    __shared__ int s_bad, s_last;
+    double* ks = il + 16;                             // [slab_w] k(X_c, x_p) of this slab's columns
+    __shared__ int s_bad, s_last, s_cat[16];
     if (tid == 0) s_bad = 0;
     __syncthreads();
-    if (tid < d) {
+    if (tid < d) {  // the pick's features (one thread each) ...
         double x = 0.0;
         if (!feature64(sp, tid, s_words[tid], &x)) s_bad = 1;
         u[tid] = x;
-        il[tid] = (int)sp[tid * 4] == SCOOT_CATEGORICAL ? 1.0 / (ell[tid] * ell[tid]) : 1.0 / ell[tid];
         if (lead) a.upick[(size_t)j * d + tid] = x;
+    } else if (tid >= 32 && tid < 32 + d) {  // ... and, in another warp, the length scales
+        const int c = tid - 32;
+        const bool cat = (int)sp[c * 4] == SCOOT_CATEGORICAL;
+        s_cat[c] = cat;
+        il[c] = cat ? 1.0 / (ell[c] * ell[c]) : 1.0 / ell[c];
     }
     __syncthreads();
     if (s_bad) {
@@ -622,11 +660,11 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         }
         return;
     }
-    // k(x_p, X_i), fp64: ordinal coordinates times 1/l, categorical mismatches 1/l^2.
+    // k(x_p, x), fp64: ordinal coordinates times 1/l, categorical mismatches 1/l^2.
     auto cov = [&](const double* ub) {
         double r2 = 0.0;
         for (int c = 0; c < d; ++c) {
-            if ((int)sp[c * 4] == SCOOT_CATEGORICAL) {
+            if (s_cat[c]) {
                 r2 += u[c] != ub[c] ? il[c] : 0.0;
             } else {
                 const double t = (u[c] - ub[c]) * il[c];
@@ -635,83 +673,137 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         }
         return sf2 * matern64(sqrt(r2), a.kernel);
     };
-    const int i0 = tri_row(r, R, n), i1 = tri_row(r + 1, R, n);
-    double mu_part = 0.0;
-    for (int i = tid; i < (r == 0 ? n : i1); i += blockDim.x) {
-        ks[i] = cov(uo + (size_t)i * d);
-        if (r == 0) mu_part = fma(ks[i], alpha[i], mu_part);
+    const int w = a.slab_w, c0 = b * w, c1 = min(n, c0 + w);
+    for (int c = c0 + tid; c < c1; c += blockDim.x) ks[c - c0] = cov(uo + (size_t)c * d);
+    for (int t = b + B * (int)(blockDim.x - 1 - tid); t < j; t += B * (int)blockDim.x)  // top threads
+        a.kpt[(size_t)m * q + t] = cov(a.upick + (size_t)t * d);
+    __syncthreads();
+    if (tid < 32) {
+        double s = 0.0;
+        for (int c = c0 + tid; c < c1; c += 32) s = fma(alpha[c], ks[c - c0], s);
+        s = warp_sum(s);
+        if (tid == 0) a.mupart[(size_t)m * B + b] = s;
     }
-    const double mu = block_sum(mu_part, red);  // (its barriers also publish ks)
-    double* vrow = a.vpick + ((size_t)j * M + m) * n;
-    for (int i = i0 + tid; i < i1; i += blockDim.x) {
+    // Rows i >= c0 of this slab's part: sum over its columns c <= i of L^{-1}[i][c] k_c
+    // (L^{-1} column-major: the threads of a warp read consecutive rows of a column).
+    double* part = a.part + ((size_t)m * B + b) * n;
+    for (int i = c0 + tid; i < n; i += blockDim.x) {
+        const int ce = min(c1, i + 1);
         double s0 = 0.0, s1 = 0.0;
-        int c = 0;
-        for (; c + 1 <= i; c += 2) {
-            s0 = fma(Li[(size_t)c * n + i], ks[c], s0);
-            s1 = fma(Li[(size_t)(c + 1) * n + i], ks[c + 1], s1);
+        int c = c0;
+        for (; c + 1 < ce; c += 2) {
+            s0 = fma(Li[(size_t)c * n + i], ks[c - c0], s0);
+            s1 = fma(Li[(size_t)(c + 1) * n + i], ks[c + 1 - c0], s1);
         }
-        if (c <= i) s0 = fma(Li[(size_t)c * n + i], ks[c], s0);
-        vrow[i] = s0 + s1;
+        if (c < ce) s0 = fma(Li[(size_t)c * n + i], ks[c - c0], s0);
+        part[i] = s0 + s1;
     }
-    if (r == 0 && tid == 0) a.mupick[(size_t)j * M + m] = mu;
-    // The last slice of objective m completes its terms.
+    // The last slab of objective m completes its terms.
     __threadfence();
     __syncthreads();
-    if (tid == 0) s_last = atomicAdd(&a.ctrl->arrived_m[m], 1u) == (unsigned)(R - 1);
+    if (tid == 0) s_last = atomicAdd(&a.ctrl->arrived_m[m], 1u) == (unsigned)(B - 1);
     __syncthreads();
     if (!s_last) return;
     __threadfence();
     if (tid == 0) a.ctrl->arrived_m[m] = 0u;
-    double* vv = ks;            // [n] v_p, read back from the slices
-    double* D = ks + n;         // [q] v_p . v_{p_t}
-    double* kpt = D + q;        // [q] k(x_p, x_{p_t})
-    double* red2 = kpt + q;     // [32]
-    double* Ct = red2 + 32;     // [q][q] c_k(x_{p_t}) of the earlier picks
-    double* st = Ct + q * q;    // [q] their s
-    double* cj = st + q;        // [q] this pick's c_t(x_p)
-    for (int e = tid; e < j * j; e += blockDim.x) {
-        const int t = e / j, k = e - t * j;
-        Ct[e] = k < t ? a.cpick[((size_t)t * M + m) * q + k] : 0.0;
-    }
-    for (int t = tid; t < j; t += blockDim.x) st[t] = a.spick[(size_t)t * M + m];
+    double* vv = reinterpret_cast<double*>(smem);  // [n] v_p
+    double* D = vv + n;                            // [q] v_p . v_{p_t}
+    double* bq = D + q;                            // [q] k(x_p, x_{p_t}) - v_p . v_{p_t}
+    double* cq = bq + q;                           // [q] c_t(x_p)
+    double* red = cq + q;                          // [32]
+    double* red2 = red + 32;                       // [32]
+    const double* pm = a.part + (size_t)m * B * n;
+    double* vrow = a.vpick + ((size_t)j * M + m) * n;
     double vv_part = 0.0;
     for (int i = tid; i < n; i += blockDim.x) {
-        const double v = __ldcg(vrow + i);
+        const int nb = min(B, i / w + 1);  // the slabs with c0 <= i, summed in slab order by fours
+        double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+        int k = 0;
+        for (; k + 3 < nb; k += 4) {
+            s0 += __ldcg(pm + (size_t)k * n + i);
+            s1 += __ldcg(pm + (size_t)(k + 1) * n + i);
+            s2 += __ldcg(pm + (size_t)(k + 2) * n + i);
+            s3 += __ldcg(pm + (size_t)(k + 3) * n + i);
+        }
+        for (; k < nb; ++k) s0 += __ldcg(pm + (size_t)k * n + i);
+        const double v = (s0 + s1) + (s2 + s3);
         vv[i] = v;
-        vv_part = fma(v, v, vv_part);
+        vrow[i] = v;
         a.vp[m * a.n_pad + i] = (float)v;
+        vv_part = fma(v, v, vv_part);
     }
     for (int i = n + tid; i < a.n_pad; i += blockDim.x) a.vp[m * a.n_pad + i] = 0.0f;
-    for (int t = tid; t < j; t += blockDim.x) kpt[t] = cov(a.upick + (size_t)t * d);
-    const double vnorm = block_sum(vv_part, red2);  // (its barriers also publish vv and kpt)
-    {
+    if (tid < 32) {
+        double s = 0.0;
+        for (int k = tid; k < B; k += 32) s += __ldcg(a.mupart + (size_t)m * B + k);
+        s = warp_sum(s);
+        if (tid == 0) a.mupick[(size_t)j * M + m] = s;
+    }
+    const double vnorm = block_sum(vv_part, red);  // (its barriers also publish vv)
+    {  // v_p . v_{p_t}: a warp per two earlier picks
         const int lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
-        for (int t = warp; t < j; t += nw) {
-            const double* vt = a.vpick + ((size_t)t * M + m) * n;
-            double s = 0.0;
-            for (int i = lane; i < n; i += 32) s = fma(vv[i], vt[i], s);
-            for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-            if (lane == 0) D[t] = s;
+        for (int t = warp; t < j; t += 2 * nw) {
+            const int t2 = t + nw < j ? t + nw : t;
+            const double* va = a.vpick + ((size_t)t * M + m) * n;
+            const double* vb = a.vpick + ((size_t)t2 * M + m) * n;
+            double sa = 0.0, sb = 0.0;
+            for (int i = lane; i < n; i += 32) {
+                sa = fma(vv[i], va[i], sa);
+                sb = fma(vv[i], vb[i], sb);
+            }
+            for (int o = 16; o > 0; o >>= 1) {
+                sa += __shfl_xor_sync(0xffffffffu, sa, o);
+                sb += __shfl_xor_sync(0xffffffffu, sb, o);
+            }
+            if (lane == 0) {
+                D[t] = sa;
+                D[t2] = sb;
+            }
         }
     }
     __syncthreads();
-    if (tid == 0) {  // the recurrence over the earlier picks, in shared memory
-        double var = sf2 - vnorm;
-        for (int t = 0; t < j; ++t) {
-            double num = kpt[t] - D[t];
-            for (int k = 0; k < t; ++k) num -= cj[k] * Ct[t * j + k];
-            cj[t] = st[t] > 0.0 ? num / st[t] : 0.0;
-            var -= cj[t] * cj[t];
-        }
-        const double s = sqrt(fmax(var, 0.0) + tau2);
-        a.spick[(size_t)j * M + m] = s;
-        a.inv_s[m] = s > 0.0 ? (float)(1.0 / s) : 0.0f;
-    }
+    for (int t = tid; t < j; t += blockDim.x) bq[t] = __ldcg(a.kpt + (size_t)m * q + t) - D[t];
     __syncthreads();
-    for (int t = tid; t < q; t += blockDim.x) {
-        if (t < j) a.cpick[((size_t)j * M + m) * q + t] = cj[t];
-        a.cxp[m * q + t] = t < j ? (float)cj[t] : 0.0f;
+    // c(x_p) = W b: row t of W holds t + 1 entries.
+    const double* W = a.wf + (size_t)m * q * q;
+    double csq = 0.0;
+    for (int t = tid; t < j; t += blockDim.x) {
+        const double* wt = W + (size_t)t * q;
+        double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+        int k = 0;
+        for (; k + 3 <= t; k += 4) {
+            s0 = fma(wt[k], bq[k], s0);
+            s1 = fma(wt[k + 1], bq[k + 1], s1);
+            s2 = fma(wt[k + 2], bq[k + 2], s2);
+            s3 = fma(wt[k + 3], bq[k + 3], s3);
+        }
+        for (; k <= t; ++k) s0 = fma(wt[k], bq[k], s0);
+        const double c = (s0 + s1) + (s2 + s3);
+        cq[t] = c;
+        csq = fma(c, c, csq);
     }
+    const double csum = block_sum(csq, red2);  // (its barriers also publish cq)
+    // s_j^2 = sigma^2(x_p) - sum_t c_t(x_p)^2 + tau^2; 1/s_j from one reciprocal square root.
+    const double x = fmax(sf2 - vnorm - csum, 0.0) + tau2;
+    const double inv = x > 0.0 ? rsqrt(x) : 0.0;
+    if (tid == 0) a.inv_s[m] = (float)inv;
+    // Row j of W: -(1/s_j) sum_{k=t}^{j-1} c_k W[k][t] for t < j, 1/s_j on the diagonal.
+    double* wj = a.wf + ((size_t)m * q + j) * q;
+    for (int t = tid; t <= j; t += blockDim.x) {
+        if (t == j) {
+            wj[t] = inv;
+            continue;
+        }
+        double s0 = 0.0, s1 = 0.0;
+        int k = t;
+        for (; k + 1 < j; k += 2) {
+            s0 = fma(cq[k], W[(size_t)k * q + t], s0);
+            s1 = fma(cq[k + 1], W[(size_t)(k + 1) * q + t], s1);
+        }
+        if (k < j) s0 = fma(cq[k], W[(size_t)k * q + t], s0);
+        wj[t] = -inv * (s0 + s1);
+    }
+    for (int t = tid; t < q; t += blockDim.x) a.cxp[m * q + t] = t < j ? (float)cq[t] : 0.0f;
     // The last objective adds the fantasised point and rebuilds the boxes.
     __threadfence();
     __syncthreads();
@@ -740,8 +832,8 @@ scatter_var(const int32_t* list, const unsigned int* n_list, int64_t n, int64_t 
 // ---------------------------------------------------------------- work buffer
 
 struct WorkLayout {
-    int64_t mean, var, V, C, ctrl, picked, vp, cxp, inv_s, upick, vpick, cpick, spick, mupick, front, box_lo,
-        box_hi, part_key, part_pos, rec, words, bytes;
+    int64_t mean, var, V, C, ctrl, picked, vp, cxp, inv_s, upick, vpick, wf, part, mupart, kpt, mupick, front,
+        box_lo, box_hi, part_key, part_pos, rec, words, bytes;
 };
 
 int64_t up256(int64_t x) { return (x + 255) / 256 * 256; }
@@ -762,8 +854,10 @@ WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q, int box_cap) 
     w.inv_s = o;    o = up256(o + M * 4);
     w.upick = o;    o = up256(o + (int64_t)q * d * 8);
     w.vpick = o;    o = up256(o + (int64_t)q * M * no * 8);
-    w.cpick = o;    o = up256(o + (int64_t)q * M * q * 8);
-    w.spick = o;    o = up256(o + (int64_t)q * M * 8);
+    w.wf = o;       o = up256(o + M * q * q * 8);
+    w.part = o;     o = up256(o + M * pick_slabs((int)no) * no * 8);
+    w.mupart = o;   o = up256(o + M * pick_slabs((int)no) * 8);
+    w.kpt = o;      o = up256(o + M * q * 8);
     w.mupick = o;   o = up256(o + (int64_t)q * M * 8);
     w.front = o;    o = up256(o + fcap * M * 8);
     w.box_lo = o;   o = up256(o + (int64_t)box_cap * M * 4);
@@ -796,7 +890,7 @@ scoot_status set_attributes(scoot_ctx* ctx, Session& ss) {
     const FantArgs& a = ss.a;
     ss.pass_smem = (size_t)(2 * a.box_cap + a.n_mc) * 16 + (size_t)((a.q + 1) & ~1) * 8 + (size_t)M * a.n_pad * 4 +
                    (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4;
-    ss.pick_smem = std::max((size_t)(32 + a.n_obs + a.q * a.q + 4 * a.q + 64) * 8,
+    ss.pick_smem = std::max((size_t)std::max(32 + a.slab_w, a.n_obs + 3 * a.q + 64) * 8,
                             boxes_smem(a.front_cap, M, a.box_cap));
     int max_smem = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
@@ -899,8 +993,12 @@ scoot_status scoot_fantasy_begin(scoot_ctx* ctx, const scoot_gp_layout* L, const
     a.inv_s = reinterpret_cast<float*>(wk + w.inv_s);
     a.upick = reinterpret_cast<double*>(wk + w.upick);
     a.vpick = reinterpret_cast<double*>(wk + w.vpick);
-    a.cpick = reinterpret_cast<double*>(wk + w.cpick);
-    a.spick = reinterpret_cast<double*>(wk + w.spick);
+    a.wf = reinterpret_cast<double*>(wk + w.wf);
+    a.part = reinterpret_cast<double*>(wk + w.part);
+    a.mupart = reinterpret_cast<double*>(wk + w.mupart);
+    a.kpt = reinterpret_cast<double*>(wk + w.kpt);
+    a.n_slab = pick_slabs(L->n);
+    a.slab_w = (L->n + a.n_slab - 1) / a.n_slab;
     a.mupick = reinterpret_cast<double*>(wk + w.mupick);
     a.part_key = reinterpret_cast<uint64_t*>(wk + w.part_key);
     a.part_pos = reinterpret_cast<int32_t*>(wk + w.part_pos);
@@ -967,7 +1065,7 @@ scoot_status scoot_fantasy_commit(scoot_ctx* ctx, int32_t j, const uint64_t* rec
     if (j < 0 || j >= ss->a.q) return scoot_fail(ctx, SCOOT_EINVAL, "pick %d outside 0..%d", j, ss->a.q - 1);
     if (!recs || n_rec < 1) return scoot_fail(ctx, SCOOT_EINVAL, "no records");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const dim3 grid(kPickRows, ss->M);
+    const dim3 grid(ss->a.n_slab, ss->M);
     switch (ss->M) {
     case 2: fant_pick<2><<<grid, kPickThreads, ss->pick_smem, st>>>(ss->a, j, recs, n_rec); break;
     case 3: fant_pick<3><<<grid, kPickThreads, ss->pick_smem, st>>>(ss->a, j, recs, n_rec); break;
