@@ -153,6 +153,16 @@ scoot_status scoot_ctx_workspace_bytes(const scoot_ctx* ctx, int64_t* bytes);
 #define SCOOT_PHASE_FANT_PICK      4   /* a pick's fp64 terms, front and boxes */
 #define SCOOT_PHASE_SCATTER        5   /* variances scattered to var_out */
 scoot_status scoot_ctx_set_timing(scoot_ctx* ctx, int32_t enable);
+
+/* Tensor cores for the whitened posterior (on by default).  With enable != 0
+ * the posterior of scoot_suggest_fantasy / scoot_fantasy_begin computes
+ * V = L^{-1} k(X, x) on the tcgen05 tensor cores when the padded observation
+ * count is at most 256 and the state fits a block's shared memory: each fp32
+ * operand split into three bf16 parts, six part products accumulated in fp32
+ * (the m l, l m, l l products, of order 2^-24, dropped); with enable == 0,
+ * or outside those limits, the fp32 SIMT product.  The paper has no
+ * counterpart (Section 4.3 states the posterior, not how it is computed). */
+scoot_status scoot_ctx_set_tensor_cores(scoot_ctx* ctx, int32_t enable);
 scoot_status scoot_ctx_phase_times(scoot_ctx* ctx, int32_t cap, int32_t* h_kind, float* h_ms, int32_t* count);
 
 /* ------------------------------------------------------------------ 1. prune, Eq. (2) */

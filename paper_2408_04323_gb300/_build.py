@@ -17,7 +17,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libscoot.so")
 SOURCES = ["context.cu", "host_prep.cpp", "compact.cu", "prune_rf.cu", "score.cu", "topq.cu", "fantasy.cu", "pareto.cu",
            "sobol.cu", "rf_train.cu",
-           "gp_device.cu", "round_state.cpp", "probes.cu"]
+           "gp_device.cu", "round_state.cpp", "probes.cu", "posterior_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall"]
 

@@ -151,6 +151,12 @@ scoot_status scoot_ctx_set_timing(scoot_ctx* ctx, int32_t enable) {
     return SCOOT_OK;
 }
 
+scoot_status scoot_ctx_set_tensor_cores(scoot_ctx* ctx, int32_t enable) {
+    if (!ctx) return SCOOT_EINVAL;
+    ctx->tensor_cores = enable != 0;
+    return SCOOT_OK;
+}
+
 scoot_status scoot_ctx_phase_times(scoot_ctx* ctx, int32_t cap, int32_t* h_kind, float* h_ms, int32_t* count) {
     scoot_status s = scoot_enter(ctx);
     if (s != SCOOT_OK) return s;

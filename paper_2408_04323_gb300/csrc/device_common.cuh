@@ -131,7 +131,8 @@ constexpr float kOpenWidth = 1099511627776.0f;  // 2^40
 // last one W = prod_j w_j and C = -l_last * W, so that a box's HVI term is
 //   prod_{j<M-1} sat(y_j a_j + b_j) * max(y_last W + C, 0)
 // (sat clamps to [0, 1]): one saturated FMA per bounded objective.
-// Row b holds (a_0, b_0, a_1, b_1) and (a_2, b_2, W, C) as two float4.
+// Row b holds (a_0, b_0, a_1, b_1) and (W, W, C, C) as two float4 (M <= 3:
+// the second row is two packed pairs for the f32x2 instructions).
 __device__ __forceinline__ void stage_boxes_sat(const float* box_lo, const float* box_hi, int n_boxes, int M,
                                                 float4* bs) {
     for (int b = threadIdx.x; b < n_boxes; b += blockDim.x) {
@@ -144,44 +145,57 @@ __device__ __forceinline__ void stage_boxes_sat(const float* box_lo, const float
             v[2 * j + 1] = -l / w;
             W *= w;
         }
-        v[6] = W;
-        v[7] = -box_lo[b * M + M - 1] * W;
+        const float C = -box_lo[b * M + M - 1] * W;
         bs[2 * b] = make_float4(v[0], v[1], v[2], v[3]);
-        bs[2 * b + 1] = make_float4(v[4], v[5], v[6], v[7]);
+        bs[2 * b + 1] = make_float4(W, W, C, C);
     }
 }
 
+// Sum over samples first, first + stride, ... (chunks of eight) of the HVI of
+// y_s = mu + sd * eps_s against boxes staged by stage_boxes_sat (M <= 3).
+// Samples go in pairs through the packed f32x2 FMA and multiply (the same
+// roundings as the scalar operations); the saturated FMAs and the maximum
+// stay scalar.
 template <int M>
 __device__ __forceinline__ float ehvi_partial_sat(const float* mu, const float* sd, const float4* bs, int n_boxes,
                                                  const float4* eps, int n_mc, int first, int stride) {
-    constexpr int kCh = 8;
+    static_assert(M == 2 || M == 3, "the saturated form takes two or three objectives");
+    constexpr int kCh = 8, kP = kCh / 2;
     float total = 0.0f;
     for (int s0 = first * kCh; s0 < n_mc; s0 += stride * kCh) {
-        float y[kCh][M], acc[kCh];
+        float ya[kCh], yb[kCh];  // the first M - 1 objectives (yb unused for M = 2)
+        float2 yl[kP], acc[kP];  // the last objective and the sums, in pairs of samples
 #pragma unroll
-        for (int k = 0; k < kCh; ++k) {
-            acc[k] = 0.0f;
-            const bool in = s0 + k < n_mc;
-            const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float ev[4] = {e.x, e.y, e.z, e.w};
+        for (int h = 0; h < kP; ++h) {
+            float last[2];
 #pragma unroll
-            for (int j = 0; j < M; ++j) y[k][j] = in ? fmaf(sd[j], ev[j], mu[j]) : -INFINITY;
+            for (int u = 0; u < 2; ++u) {
+                const int k = 2 * h + u;
+                const bool in = s0 + k < n_mc;
+                const float4 e = in ? eps[s0 + k] : make_float4(0.f, 0.f, 0.f, 0.f);
+                ya[k] = in ? fmaf(sd[0], e.x, mu[0]) : -INFINITY;
+                yb[k] = M > 2 ? (in ? fmaf(sd[1], e.y, mu[1]) : -INFINITY) : 0.0f;
+                last[u] = in ? fmaf(sd[M - 1], M > 2 ? e.z : e.y, mu[M - 1]) : -INFINITY;
+            }
+            yl[h] = make_float2(last[0], last[1]);
+            acc[h] = make_float2(0.0f, 0.0f);
         }
         for (int b = 0; b < n_boxes; ++b) {
-            const float4 q0 = bs[2 * b];
-            const float4 q1 = (M > 2) ? bs[2 * b + 1] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float W = M > 2 ? q1.z : bs[2 * b + 1].z;
-            const float Cc = M > 2 ? q1.w : bs[2 * b + 1].w;
+            const float4 q0 = bs[2 * b], q1 = bs[2 * b + 1];
+            const float2 Wp = make_float2(q1.x, q1.y), Cp = make_float2(q1.z, q1.w);
 #pragma unroll
-            for (int k = 0; k < kCh; ++k) {
-                float p = __saturatef(fmaf(y[k][0], q0.x, q0.y));
-                if (M > 2) p *= __saturatef(fmaf(y[k][1], q0.z, q0.w));
-                if (M > 3) p *= __saturatef(fmaf(y[k][2], q1.x, q1.y));
-                acc[k] = fmaf(p, fmaxf(fmaf(y[k][M - 1], W, Cc), 0.0f), acc[k]);
+            for (int h = 0; h < kP; ++h) {
+                float2 p = make_float2(__saturatef(fmaf(ya[2 * h], q0.x, q0.y)),
+                                       __saturatef(fmaf(ya[2 * h + 1], q0.x, q0.y)));
+                if (M > 2)
+                    p = __fmul2_rn(p, make_float2(__saturatef(fmaf(yb[2 * h], q0.z, q0.w)),
+                                                  __saturatef(fmaf(yb[2 * h + 1], q0.z, q0.w))));
+                const float2 t = __ffma2_rn(yl[h], Wp, Cp);
+                acc[h] = __ffma2_rn(p, make_float2(fmaxf(t.x, 0.0f), fmaxf(t.y, 0.0f)), acc[h]);
             }
         }
 #pragma unroll
-        for (int k = 0; k < kCh; ++k) total += acc[k];
+        for (int h = 0; h < kP; ++h) total += acc[h].x + acc[h].y;
     }
     return total;
 }

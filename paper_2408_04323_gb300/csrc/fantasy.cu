@@ -557,8 +557,12 @@ __global__ void __launch_bounds__(kPassThreads, M == 2 ? 4 : 1) fant_pass(const 
             mu[m] = a.mean[(int64_t)m * a.ldc + pos];
             sd[m] = sqrtf(fmaxf(vr[m], 0.0f));
         }
-        const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, nb, epsv, a.n_mc, 0, 1) * inv_mc
-                             : ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
+        float v;
+        if constexpr (M <= 3)  // (the saturated form takes two or three objectives)
+            v = fast ? ehvi_partial_sat<M>(mu, sd, blo, nb, epsv, a.n_mc, 0, 1) * inv_mc
+                     : ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
+        else
+            v = ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
         if (!(v != v) && v != -INFINITY)
             keymax(best, best_pos, make_key(v, (uint32_t)(a.index_offset + i)), (int32_t)pos);
     }
@@ -833,7 +837,7 @@ scatter_var(const int32_t* list, const unsigned int* n_list, int64_t n, int64_t 
 
 struct WorkLayout {
     int64_t mean, var, V, C, ctrl, picked, vp, cxp, inv_s, upick, vpick, wf, part, mupart, kpt, mupick, front,
-        box_lo, box_hi, part_key, part_pos, rec, words, bytes;
+        box_lo, box_hi, part_key, part_pos, rec, words, tcb, tcb_bytes, bytes;
 };
 
 int64_t up256(int64_t x) { return (x + 255) / 256 * 256; }
@@ -866,6 +870,9 @@ WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q, int box_cap) 
     w.part_pos = o; o = up256(o + kPartMax * 4);
     w.rec = o;      o = up256(o + SCOOT_FANT_REC * 8);
     w.words = o;    o = up256(o + 16 * 4);
+    // the split copy of L^{-1} for the tensor-core posterior (when n_pad allows it)
+    w.tcb_bytes = n_pad <= kMaxNpadTc ? scoot_tc_bsplit_bytes((int)n_pad, (int)M) : 0;
+    w.tcb = o;      o = up256(o + w.tcb_bytes);
     w.bytes = o;
     return w;
 }
@@ -1010,7 +1017,8 @@ scoot_status scoot_fantasy_begin(scoot_ctx* ctx, const scoot_gp_layout* L, const
     a.err = ctx->d_err;
     if (n > 0) {
         s = scoot_posterior_whitened(ctx, L, state, cand, n, ld, a.list, a.n_list, reinterpret_cast<float*>(wk + w.mean),
-                                     a.var, reinterpret_cast<float*>(wk + w.V), a.ldc, st);
+                                     a.var, reinterpret_cast<float*>(wk + w.V), a.ldc,
+                                     w.tcb_bytes > 0 ? static_cast<void*>(wk + w.tcb) : nullptr, st);
         if (s != SCOOT_OK) return s;
         if ((s = scoot_mark(ctx, st, SCOOT_PHASE_POSTERIOR)) != SCOOT_OK) return s;
     }

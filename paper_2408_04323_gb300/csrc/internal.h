@@ -34,6 +34,9 @@ struct scoot_ctx {
     // The open session of sequential fantasised picks (scoot_fantasy_begin
     // .. scoot_fantasy_end), opaque to everything but fantasy.cu.
     std::vector<char> fant_session;
+    // scoot_ctx_set_tensor_cores: the whitened posterior may run its L^{-1} k
+    // product on the tensor cores (posterior_tc.cu) where the state fits.
+    int32_t tensor_cores = 1;
 };
 
 scoot_status scoot_fail(scoot_ctx* ctx, scoot_status s, const char* fmt, ...);
@@ -145,10 +148,37 @@ scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint3
 // rows, [M][n_rb * 16][ldc][4] (16-byte aligned; groups wholly past row n
 // left unwritten, rows past n inside a written group zero).  ldc >= the list
 // length.
+// tc_work (may be NULL: the SIMT product) is device scratch of at least
+// scoot_tc_bsplit_bytes(n_pad, M) bytes, 16-byte aligned, for the split copy
+// of L^{-1} that the tensor-core product reads.
 scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
                                       const uint32_t* cand, int64_t n, int64_t ld, const int32_t* list,
                                       const unsigned int* n_list, float* mean, float* var, float* V, int64_t ldc,
-                                      cudaStream_t st);
+                                      void* tc_work, cudaStream_t st);
+
+// The tensor-core whitened posterior (posterior_tc.cu): the arguments of the
+// SIMT kernel's whitened epilogue plus the split copy of L^{-1}.
+constexpr int kMaxNpadTc = 256;  // output rows held in tensor memory (fp32 columns)
+struct ScootTcArgs {
+    const char* state;
+    int64_t off_fmap, off_xs, off_ils, off_alpha, off_scal, off_cat, off_warp, off_linv;
+    int32_t n_obs, d, n_obj, kernel, n_pad, n_ord, n_pat, n_tiles, cat_smem;
+    const uint32_t* cand;
+    int64_t n, ld;
+    const int32_t* list;
+    const unsigned int* n_list;
+    float* mean;
+    float* var;
+    int64_t ldo;
+    float* vout;      // NULL: moments only
+    int64_t ldv;
+    int32_t by_index; // mean / var at the candidate's index (else at its list position)
+    uint8_t* bsplit;  // [M][n_pad / 32][3][n_pad * 64 bytes]
+    uint32_t* err;
+};
+int64_t scoot_tc_bsplit_bytes(int n_pad, int M);
+bool scoot_tc_supported(scoot_ctx* ctx, const ScootTcArgs& a, int DO);
+scoot_status scoot_posterior_tc(scoot_ctx* ctx, const ScootTcArgs& a, int DO, cudaStream_t st);
 
 #define SCOOT_CUDA(ctx, call)                                                          \
     do {                                                                               \

@@ -1,0 +1,507 @@
+// GP posterior (Section 4.3) with the whitened rows V = L^{-1} k(X, x) on
+// the fifth-generation tensor cores (tcgen05), for n_pad <= 256 rows.
+//
+// V^T = K*^T L^{-T} is a dense contraction: for a tile of 128 candidates,
+// A = K*^T [128 x n] (the candidates' covariance rows) and B = L^{-1} [n x n]
+// (row i of B is row i of L^{-1}, so D[x][i] = sum_c K*[c][x] L^{-1}[i][c]).
+// Both operands are fp32 values split into three bf16 parts,
+//   x = x_h + x_m + x_l  (x_h = bf16(x), x_m = bf16(x - x_h), x_l = bf16(x - x_h - x_m)),
+// which hold all 24 bits of an fp32 significand (each part to within 2^-8
+// of the remainder it takes).  The product keeps the six part products down
+// to order 2^-16 and drops m l, l m and l l (order 2^-24, one fp32
+// rounding).  The tensor core's fp32 accumulation truncates once per MMA
+// relative to the accumulator's magnitude, so the full-size products h h go
+// to a main accumulator (one truncation per 16 columns of L^{-1}) and the
+// five smaller ones (h m, m h, h l, l h, m m) to a correction accumulator,
+// where their truncations weigh 2^-8 less; V = main + corr.
+//
+// One CTA per SM, 256 threads: thread t serves candidate row t mod 128 (the
+// TMEM lane its warp can read) and column half t / 128.  Per objective the
+// rows of L^{-1} go in k-blocks of 32 columns; k-block kb only reaches output
+// rows i >= 32 kb (L^{-1} is lower triangular), so its products are MMAs of
+// N = n_pad - 32 kb columns starting at column 32 kb of each accumulator
+// (main at TMEM columns [0, n_pad), corrections at [n_pad, 2 n_pad)).  Pipeline per
+// k-block g (counted over the CTA's whole sequence):
+//   - wait until the MMAs of g - 2 are done (mbarrier), freeing A slot g mod 2
+//     and B slot (g + 1) mod 3;
+//   - cp.async the three B parts of k-block g + 1 (from the split copy of
+//     L^{-1} prepared once per call by bsplit_kernel) into B slot (g + 1) mod 3;
+//   - every thread evaluates its 16 covariances of k-block g, splits them and
+//     stores the parts into A slot g mod 2 (the MMAs of g - 1 run meanwhile);
+//   - one thread issues the 12 MMAs of k-block g (2 K-steps x 6 part products)
+//     and commits them to mbarrier g mod 2.
+// After the last k-block the threads read D back (tcgen05.ld), write V in the
+// float4-group layout of the fantasy pass, and finish mu and sigma^2.
+//
+// Operand layout in shared memory: the canonical no-swizzle K-major form of
+// a 32-wide k-block: 8-row x 16-byte core matrices, 128 bytes apart along K
+// (leading byte offset) and 512 bytes apart along the rows (stride byte
+// offset).
+#include <cuda_bf16.h>
+
+#include "device_common.cuh"
+#include "internal.h"
+
+namespace {
+
+using namespace scoot_dev;
+
+constexpr int kTM = 128;          // candidates per tile: the MMA's M and the TMEM lanes
+constexpr int kKB = 32;           // columns of L^{-1} per k-block
+constexpr int kThr = 256;         // two threads per candidate row
+constexpr int kParts = 3;         // bf16 parts of an fp32 operand
+constexpr uint32_t kLBO = 128;    // bytes between core matrices along K
+constexpr uint32_t kSBO = 512;    // bytes between 8-row groups of a k-block
+constexpr uint32_t kAPart = kTM * kKB * 2;  // bytes of one part of an A k-block (8 KiB)
+constexpr int kMaxD = SCOOT_MAX_DIM;
+constexpr unsigned long long kWaitNs = 2000000000ull;  // bounded waits give up after 2 s
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// Byte offset of element (row, kk) of a k-block in the canonical layout.
+__host__ __device__ __forceinline__ uint32_t canon_off(int row, int kk) {
+    return (uint32_t)((row & 7) * 16 + (row >> 3) * (int)kSBO + (kk >> 3) * (int)kLBO + (kk & 7) * 2);
+}
+
+// Shared-memory matrix descriptor (tcgen05): start address, leading and
+// stride byte offsets (each >> 4), descriptor version 1, no swizzle.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+    return (uint64_t)((addr >> 4) & 0x3FFFu) | ((uint64_t)((kLBO >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((kSBO >> 4) & 0x3FFFu) << 32) | (1ull << 46);
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, M = 128, N columns.
+__device__ __forceinline__ uint32_t instr_desc(uint32_t N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((N >> 3) << 17) | ((uint32_t)(kTM >> 4) << 24);
+}
+
+// The three bf16 parts of x.
+__device__ __forceinline__ void split3(float x, __nv_bfloat16& h, __nv_bfloat16& m, __nv_bfloat16& l) {
+    h = __float2bfloat16_rn(x);
+    const float r1 = x - __bfloat162float(h);  // exact
+    m = __float2bfloat16_rn(r1);
+    const float r2 = r1 - __bfloat162float(m);  // exact
+    l = __float2bfloat16_rn(r2);
+}
+
+__device__ __forceinline__ uint32_t pack2(__nv_bfloat16 lo, __nv_bfloat16 hi) {
+    return (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Waits (bounded) until the phase of the given parity of an mbarrier has
+// completed; false if it gave up.
+__device__ __forceinline__ bool mbar_wait(uint32_t addr, uint32_t parity) {
+    const unsigned long long t0 = global_ns();
+    while (true) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if (global_ns() - t0 > kWaitNs) return false;
+    }
+}
+
+// B = L^{-1} of every objective, split into bf16 parts, per k-block of 32
+// columns in the canonical layout: [M][n_pad / 32][3][n_pad rows x 64 bytes].
+// One thread per (objective, k-block, row, group of 8 columns).
+__device__ __forceinline__ float linv_at(const float* tiles, int n, int row, int c) {
+    // tiles: row block rb, column chunk cj; tile[jj][ii] = L^{-1}[64 rb + ii][32 cj + jj]
+    const int rb = row >> 6, ii = row & 63, cj = c >> 5, jj = c & 31;
+    return (row < n && c <= row) ? tiles[((size_t)(rb * (rb + 1) + cj) * 32 + jj) * 64 + ii] : 0.0f;
+}
+
+__global__ void __launch_bounds__(256) bsplit_kernel(const float* tiles_all, int n_tiles, int n, int n_pad, int M,
+                                                     uint8_t* out) {
+    const int KB = n_pad / kKB;
+    const size_t chunk = (size_t)n_pad * 64;
+    const int64_t total = (int64_t)M * KB * n_pad * (kKB / 8);
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+        const int kg = (int)(e % (kKB / 8));
+        int64_t rest = e / (kKB / 8);
+        const int row = (int)(rest % n_pad);
+        rest /= n_pad;
+        const int kb = (int)(rest % KB), m = (int)(rest / KB);
+        const float* tiles = tiles_all + (size_t)m * n_tiles * 32 * 64;
+        uint32_t w[kParts][4];
+#pragma unroll
+        for (int u = 0; u < 8; u += 2) {
+            const int c = kb * kKB + kg * 8 + u;
+            __nv_bfloat16 h0, m0, l0, h1, m1, l1;
+            split3(linv_at(tiles, n, row, c), h0, m0, l0);
+            split3(linv_at(tiles, n, row, c + 1), h1, m1, l1);
+            w[0][u / 2] = pack2(h0, h1);
+            w[1][u / 2] = pack2(m0, m1);
+            w[2][u / 2] = pack2(l0, l1);
+        }
+        uint8_t* base = out + ((size_t)(m * KB + kb) * kParts) * chunk + canon_off(row, kg * 8);
+#pragma unroll
+        for (int p = 0; p < kParts; ++p)
+            *reinterpret_cast<uint4*>(base + p * chunk) = make_uint4(w[p][0], w[p][1], w[p][2], w[p][3]);
+    }
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(b)) : "memory");
+}
+
+// Waits (bounded) for use u of a barrier that completes one phase per use.
+__device__ __forceinline__ bool mbar_wait_use(uint64_t* b, int64_t u) { return mbar_wait(smem_u32(b), (uint32_t)(u & 1)); }
+
+// Barrier slots in shared memory.
+enum { kAFull = 0, kMmaDone = 2, kBFull = 4, kDFree = 7, kRed = 8, kBars = 9 };
+
+template <int DO>
+__global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid_constant__ ScootTcArgs a) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    const int KB = a.n_pad / kKB;
+    const uint32_t bchunk = (uint32_t)a.n_pad * 64;
+    uint8_t* sA = smem;                                              // [2][3][8 KiB]
+    uint8_t* sB = sA + 2 * kParts * kAPart;                          // [3][3][bchunk]
+    float* xs = reinterpret_cast<float*>(sB + 3 * kParts * bchunk);  // [M][n_obs][DO] scaled observations
+    float* al = xs + (size_t)a.n_obj * a.n_obs * DO;                 // [M][n_pad] alpha
+    float* red = al + (size_t)a.n_obj * a.n_pad;                     // [4][kTM]: |V|^2 and mu halves
+    float* cat_s = red + 4 * kTM;                                    // staged categorical table
+    __shared__ float4 fm[kMaxD];
+    __shared__ __align__(8) uint64_t bars[kBars];
+    __shared__ uint32_t tslot;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const float4* gfmap = reinterpret_cast<const float4*>(a.state + a.off_fmap);
+    const float* gxs = reinterpret_cast<const float*>(a.state + a.off_xs);
+    const float* gils = reinterpret_cast<const float*>(a.state + a.off_ils);
+    const float* galpha = reinterpret_cast<const float*>(a.state + a.off_alpha);
+    const float* gscal = reinterpret_cast<const float*>(a.state + a.off_scal);
+    const float* gcat = reinterpret_cast<const float*>(a.state + a.off_cat);
+    if (tid < kMaxD) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
+    for (int e = tid; e < a.cat_smem; e += blockDim.x) cat_s[e] = __ldg(gcat + e);
+    // The observations' scaled ordinal coordinates and alpha, every objective, once.
+    for (int e = tid; e < a.n_obj * a.n_obs * DO; e += blockDim.x) {
+        const int mj = e / DO, q = e - mj * DO;
+        xs[e] = q < a.n_ord ? gxs[(size_t)mj * a.d + q] : 0.0f;
+    }
+    for (int e = tid; e < a.n_obj * a.n_pad; e += blockDim.x) {
+        const int m = e / a.n_pad, j = e - m * a.n_pad;
+        al[e] = j < a.n_obs ? galpha[(size_t)m * a.n_obs + j] : 0.0f;
+    }
+    if (tid == 0) {
+        mbar_init(&bars[kAFull], kThr);
+        mbar_init(&bars[kAFull + 1], kThr);
+        mbar_init(&bars[kMmaDone], 1);
+        mbar_init(&bars[kMmaDone + 1], 1);
+        for (int s = 0; s < 3; ++s) mbar_init(&bars[kBFull + s], 1);
+        mbar_init(&bars[kDFree], kThr);
+        mbar_init(&bars[kRed], kThr);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tslot)),
+                     "r"((uint32_t)(2 * kMaxNpadTc)));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tslot;
+    const int M = a.n_obj, n_ord = a.n_ord;
+    const int64_t n_work = a.list ? (int64_t)*a.n_list : a.n;
+    const int64_t n_tiles = (n_work + kTM - 1) / kTM;
+    const int64_t my_tiles = n_tiles > (int64_t)blockIdx.x ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+    const int64_t total_g = my_tiles * M * KB;
+
+    if (warp == kThr / 32) {
+        // ---- control warp (one thread): B copies and the MMAs.
+        if ((tid & 31) == 0) {
+            // B of k-block g (objective (g / KB) mod M, k-block g mod KB) into slot g mod 3:
+            // rows >= 32 kb only, one contiguous tail of each part.
+            auto issue_b = [&](int64_t g) {
+                const int kb = (int)(g % KB), m = (int)((g / KB) % M);
+                const uint32_t skip = (uint32_t)(kKB * kb) * 64u, bytes = bchunk - skip;
+                uint64_t* bar = &bars[kBFull + (int)(g % 3)];
+                asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                             "r"(kParts * bytes)
+                             : "memory");
+                const uint8_t* src = a.bsplit + ((size_t)(m * KB + kb) * kParts) * bchunk + skip;
+                const uint32_t dst = smem_u32(sB) + (uint32_t)(g % 3) * kParts * bchunk + skip;
+                for (int p = 0; p < kParts; ++p)
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                            dst + (uint32_t)p * bchunk),
+                        "l"(src + (size_t)p * bchunk), "r"(bytes), "r"(smem_u32(bar))
+                        : "memory");
+            };
+            bool ok = true;
+            if (total_g > 0) issue_b(0);
+            for (int64_t g = 0; g < total_g && ok; ++g) {
+                const int kb = (int)(g % KB);
+                if (g + 1 < total_g) {
+                    // slot (g + 1) mod 3 was last read by the MMAs of g - 2
+                    if (g >= 2) ok &= mbar_wait_use(&bars[kMmaDone + (int)(g & 1)], (g - 2) >> 1);
+                    if (ok) issue_b(g + 1);
+                }
+                ok = ok && mbar_wait_use(&bars[kBFull + (int)(g % 3)], g / 3);  // B of g has landed
+                ok = ok && mbar_wait_use(&bars[kAFull + (int)(g & 1)], g >> 1);  // A of g is written
+                if (kb == 0 && g > 0) ok = ok && mbar_wait_use(&bars[kDFree], g / KB - 1);  // D was read back
+                if (!ok) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t r0 = (uint32_t)(kKB * kb);
+                const uint32_t a_base = smem_u32(sA) + (uint32_t)(g & 1) * kParts * kAPart;
+                const uint32_t b_base = smem_u32(sB) + (uint32_t)(g % 3) * kParts * bchunk + r0 * 64u;
+                const uint32_t idesc = instr_desc((uint32_t)a.n_pad - r0);
+                // part products (A part, B part): h h into the main accumulator;
+                // h m, m h, h l, l h, m m into the corrections
+                const uint32_t pa = 0x120100u, pb = 0x102010u;  // nibble q = part of product q
+#pragma unroll
+                for (int s2 = 0; s2 < kKB / 16; ++s2)
+#pragma unroll
+                    for (int q = 0; q < 6; ++q) {
+                        const uint64_t da = smem_desc(a_base + ((pa >> (4 * q)) & 0xFu) * kAPart + s2 * 256u);
+                        const uint64_t db = smem_desc(b_base + ((pb >> (4 * q)) & 0xFu) * bchunk + s2 * 256u);
+                        const uint32_t acc = (kb > 0 || s2 > 0 || q > 1) ? 1u : 0u;
+                        const uint32_t dcol = tmem + (q == 0 ? 0u : (uint32_t)a.n_pad) + r0;
+                        asm volatile(
+                            "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                            "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(dcol),
+                            "l"(da), "l"(db), "r"(idesc), "r"(acc));
+                    }
+                asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                                 smem_u32(&bars[kMmaDone + (int)(g & 1)]))
+                             : "memory");
+            }
+            if (!ok) atomicOr(a.err, SCOOT_DEVERR_TIMEOUT);
+        }
+    } else {
+        // ---- SIMT warps: thread t serves candidate row t mod 128 and column half t / 128.
+        const int r = tid & (kTM - 1), half = tid >> 7;
+        int64_t g = 0, t_obj = 0;  // k-blocks and tile-objectives done
+        bool ok = true;
+        for (int64_t it = 0; it < my_tiles && ok; ++it) {
+            const int64_t tile = blockIdx.x + it * gridDim.x;
+            const int64_t pos = tile * kTM + r;
+            const bool live = pos < n_work;
+            const int64_t i = live ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
+            float u[DO];
+#pragma unroll
+            for (int q = 0; q < DO; ++q) {
+                u[q] = 0.0f;
+                if (q < n_ord && live) {
+                    const float4 f = fm[q];
+                    u[q] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + i), (int)f.x, f.y, f.z);
+                }
+            }
+            int pid = 0;  // joint category pattern (mixed radix), out-of-range categories clamped and flagged
+            for (int q = n_ord; q < a.d && live; ++q) {
+                const float4 f = fm[q];
+                const int nc = (int)f.y;
+                int v = (int)__ldg(a.cand + (int64_t)f.w * a.ld + i);
+                if (v < 0 || v >= nc) {
+                    if (half == 0) atomicOr(a.err, SCOOT_DEVERR_INDEX);
+                    v = v < 0 ? 0 : nc - 1;
+                }
+                pid += v * (int)f.z;
+            }
+            for (int m = 0; m < M && ok; ++m) {
+                const float* xsm = xs + (size_t)m * a.n_obs * DO;
+                const float* alm = al + (size_t)m * a.n_pad;
+                const float sf2 = gscal[m * 4 + 0];
+                const bool warped = gscal[m * 4 + 3] != 0.0f;
+                const float* catrow = (a.cat_smem ? cat_s : gcat) + (size_t)m * a.n_obs * a.n_pat + pid;
+                float ut[DO];
+#pragma unroll
+                for (int q = 0; q < DO; ++q) {
+                    float x = u[q];
+                    if (warped && q < n_ord) {
+                        const float2 ab = __ldg(reinterpret_cast<const float2*>(a.state + a.off_warp) + m * a.d + q);
+                        x = kumaraswamy_cdf(x, ab.x, ab.y);
+                    }
+                    ut[q] = q < n_ord ? x * gils[m * a.d + q] : 0.0f;
+                }
+                float mu_part = 0.0f;
+                // The categorical part of r^2 for this thread's 16 columns of the
+                // k-block, loaded one k-block ahead (rows past n_obs clamped).
+                float catv[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) catv[e] = catrow[(size_t)min(16 * half + e, a.n_obs - 1) * a.n_pat];
+                for (int kb = 0; kb < KB; ++kb, ++g) {
+                    // This thread's 16 covariances: columns 32 kb + 16 half + [0, 16).
+                    const int c0 = kKB * kb + 16 * half;
+                    float kv[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const int c = c0 + e;
+                        const float4* xj4 = reinterpret_cast<const float4*>(xsm + (size_t)min(c, a.n_obs - 1) * DO);
+                        float r2 = catv[e];
+#pragma unroll
+                        for (int q4 = 0; q4 < DO / 4; ++q4) {
+                            const float4 xv = xj4[q4];
+                            const float t0 = ut[q4 * 4] - xv.x, t1 = ut[q4 * 4 + 1] - xv.y;
+                            const float t2 = ut[q4 * 4 + 2] - xv.z, t3 = ut[q4 * 4 + 3] - xv.w;
+                            r2 = fmaf(t0, t0, r2);
+                            r2 = fmaf(t1, t1, r2);
+                            r2 = fmaf(t2, t2, r2);
+                            r2 = fmaf(t3, t3, r2);
+                        }
+                        const float k = (live && c < a.n_obs) ? sf2 * matern(sqrtf(r2), a.kernel) : 0.0f;
+                        mu_part = fmaf(k, alm[c], mu_part);
+                        kv[e] = k;
+                    }
+                    if (kb + 1 < KB) {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) catv[e] = catrow[(size_t)min(c0 + kKB + e, a.n_obs - 1) * a.n_pat];
+                    }
+                    // A slot g & 1 was last read by the MMAs of g - 2.
+                    if (g >= 2 && !mbar_wait_use(&bars[kMmaDone + (int)(g & 1)], (g - 2) >> 1)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* adst = sA + (size_t)(g & 1) * kParts * kAPart;
+#pragma unroll
+                    for (int grp = 0; grp < 2; ++grp) {
+                        uint32_t w[kParts][4];
+#pragma unroll
+                        for (int u2 = 0; u2 < 8; u2 += 2) {
+                            __nv_bfloat16 h0, m0, l0, h1, m1, l1;
+                            split3(kv[grp * 8 + u2], h0, m0, l0);
+                            split3(kv[grp * 8 + u2 + 1], h1, m1, l1);
+                            w[0][u2 / 2] = pack2(h0, h1);
+                            w[1][u2 / 2] = pack2(m0, m1);
+                            w[2][u2 / 2] = pack2(l0, l1);
+                        }
+                        const uint32_t off = canon_off(r, 16 * half + 8 * grp);
+#pragma unroll
+                        for (int p = 0; p < kParts; ++p)
+                            *reinterpret_cast<uint4*>(adst + p * kAPart + off) =
+                                make_uint4(w[p][0], w[p][1], w[p][2], w[p][3]);
+                    }
+                    // visible to the tensor core (async proxy), then announced
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    mbar_arrive(&bars[kAFull + (int)(g & 1)]);
+                }
+                if (!ok) break;
+                // Epilogue: the MMAs of the last k-block (g - 1) are done.
+                if (!mbar_wait_use(&bars[kMmaDone + (int)((g - 1) & 1)], (g - 1) >> 1)) {
+                    ok = false;
+                    break;
+                }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                float sq = 0.0f;
+                float4* dst4 = reinterpret_cast<float4*>(a.vout);
+                const int hw = a.n_pad / 2;
+                for (int cc = half * hw; cc < (half + 1) * hw; cc += 16) {
+                    uint32_t v[16], w[16];
+                    const uint32_t taddr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)cc;
+                    asm volatile(
+                        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+                        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+                          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]),
+                          "=r"(v[15])
+                        : "r"(taddr));
+                    asm volatile(
+                        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+                        : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7]),
+                          "=r"(w[8]), "=r"(w[9]), "=r"(w[10]), "=r"(w[11]), "=r"(w[12]), "=r"(w[13]), "=r"(w[14]),
+                          "=r"(w[15])
+                        : "r"(taddr + (uint32_t)a.n_pad));
+                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                    float vf[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        vf[e] = __uint_as_float(v[e]) + __uint_as_float(w[e]);
+                        sq = fmaf(vf[e], vf[e], sq);
+                    }
+                    if (live && a.vout) {
+#pragma unroll
+                        for (int g4 = 0; g4 < 4; ++g4) {
+                            const int gi = (cc >> 2) + g4;  // float4 group of rows 4 gi .. 4 gi + 3
+                            if (4 * gi < a.n_obs)
+                                dst4[((int64_t)m * (a.n_pad / 4) + gi) * a.ldv + pos] =
+                                    make_float4(vf[4 * g4], vf[4 * g4 + 1], vf[4 * g4 + 2], vf[4 * g4 + 3]);
+                        }
+                    }
+                }
+                // D may be overwritten by the next tile-objective's MMAs.
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                mbar_arrive(&bars[kDFree]);
+                red[half * kTM + r] = sq;
+                red[(2 + half) * kTM + r] = mu_part;
+                // Both halves' sums are in red (a bounded wait, not a hardware barrier, so
+                // that a thread that gave up elsewhere cannot hold the others).
+                mbar_arrive(&bars[kRed]);
+                if (!mbar_wait_use(&bars[kRed], t_obj++)) {
+                    ok = false;
+                    break;
+                }
+                if (half == 0 && live) {
+                    const int64_t o = (int64_t)m * a.ldo + (a.by_index ? i : pos);
+                    a.mean[o] = red[2 * kTM + r] + red[3 * kTM + r];
+                    a.var[o] = fmaxf(sf2 - (red[r] + red[kTM + r]), 0.0f);
+                }
+            }
+        }
+        if (!ok) atomicOr(a.err, SCOOT_DEVERR_TIMEOUT);
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)(2 * kMaxNpadTc)));
+}
+
+size_t tc_smem(const ScootTcArgs& a, int DO) {
+    return (size_t)2 * kParts * kAPart + (size_t)3 * kParts * a.n_pad * 64 + (size_t)a.n_obj * a.n_obs * DO * 4 +
+           (size_t)a.n_obj * a.n_pad * 4 + (size_t)4 * kTM * 4 + (size_t)a.cat_smem * 4;
+}
+
+template <int DO>
+scoot_status launch_tc(scoot_ctx* ctx, const ScootTcArgs& a, cudaStream_t st) {
+    const size_t smem = tc_smem(a, DO);
+    SCOOT_CUDA(ctx, cudaFuncSetAttribute(posterior_tc_kernel<DO>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    int sms = 0;
+    SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, ctx->device));
+    const int64_t tiles = (a.n + kTM - 1) / kTM;
+    const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>(tiles, sms));
+    posterior_tc_kernel<DO><<<(unsigned)blocks, kThr + 32, smem, st>>>(a);
+    SCOOT_LAUNCHED(ctx);
+    return SCOOT_OK;
+}
+
+}  // namespace
+
+int64_t scoot_tc_bsplit_bytes(int n_pad, int M) { return (int64_t)M * n_pad * n_pad * 2 * kParts; }
+
+bool scoot_tc_supported(scoot_ctx* ctx, const ScootTcArgs& a, int DO) {
+    if (a.n_pad < 64 || a.n_pad > kMaxNpadTc || a.n_pad % 64 != 0) return false;
+    int optin = 0;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device) != cudaSuccess) return false;
+    return tc_smem(a, DO) <= (size_t)optin;
+}
+
+scoot_status scoot_posterior_tc(scoot_ctx* ctx, const ScootTcArgs& a, int DO, cudaStream_t st) {
+    if (a.n == 0) return SCOOT_OK;
+    {
+        const int KB = a.n_pad / kKB;
+        const int64_t total = (int64_t)a.n_obj * KB * a.n_pad * (kKB / 8);
+        int64_t blocks = (total + 255) / 256;
+        if (blocks > 4096) blocks = 4096;
+        bsplit_kernel<<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<const float*>(a.state + a.off_linv), a.n_tiles,
+                                                       a.n_obs, a.n_pad, a.n_obj, a.bsplit);
+        SCOOT_LAUNCHED(ctx);
+    }
+    switch (DO) {
+    case 4: return launch_tc<4>(ctx, a, st);
+    case 8: return launch_tc<8>(ctx, a, st);
+    case 12: return launch_tc<12>(ctx, a, st);
+    default: return launch_tc<16>(ctx, a, st);
+    }
+}

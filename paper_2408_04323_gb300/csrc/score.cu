@@ -445,8 +445,12 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
             float sd[kMaxM];
 #pragma unroll
             for (int m = 0; m < M; ++m) sd[m] = sqrtf(vr[m]);
-            const float v = fast ? ehvi_partial_sat<M>(mu, sd, blo, a.n_boxes, epsv, a.n_mc, qtr, kQ)
-                                 : ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, qtr, kQ);
+            float v;
+            if constexpr (M >= 2 && M <= 3)  // (the saturated form takes two or three objectives)
+                v = fast ? ehvi_partial_sat<M>(mu, sd, blo, a.n_boxes, epsv, a.n_mc, qtr, kQ)
+                         : ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, qtr, kQ);
+            else
+                v = ehvi_partial<M>(mu, sd, blo, bhi, a.n_boxes, epsv, a.n_mc, qtr, kQ);
             __syncthreads();  // part is free again
             part[qtr * kTC + slot] = v;
             __syncthreads();
@@ -677,15 +681,62 @@ scoot_status dispatch_m(scoot_ctx* ctx, const ScoreArgs& a, int M, cudaStream_t 
     }
 }
 
+// The state part of the tensor-core posterior's arguments.
+ScootTcArgs tc_args(scoot_ctx* ctx, const ScoreArgs& a) {
+    ScootTcArgs t;
+    std::memset(&t, 0, sizeof(t));
+    t.state = a.state;
+    t.off_fmap = a.off_fmap;
+    t.off_xs = a.off_xs;
+    t.off_ils = a.off_ils;
+    t.off_alpha = a.off_alpha;
+    t.off_scal = a.off_scal;
+    t.off_cat = a.off_cat;
+    t.off_warp = a.off_warp;
+    t.off_linv = a.off_linv;
+    t.n_obs = a.n_obs;
+    t.d = a.d;
+    t.n_obj = a.n_obj;
+    t.kernel = a.kernel;
+    t.n_pad = a.n_rb * kRB;
+    t.n_ord = a.n_ord;
+    t.n_pat = a.n_pat;
+    t.n_tiles = a.n_tiles;
+    const int64_t cat = (int64_t)a.n_obj * a.n_obs * a.n_pat;
+    t.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
+    t.err = ctx->d_err;
+    return t;
+}
+
+// Padded ordinal feature count of the kernels (DO).
+int tc_do(const ScoreArgs& a) { return a.n_ord <= 4 ? 4 : a.n_ord <= 8 ? 8 : a.n_ord <= 12 ? 12 : 16; }
+
 }  // namespace
 
 scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
                                       const uint32_t* cand, int64_t n, int64_t ld, const int32_t* list,
                                       const unsigned int* n_list, float* mean, float* var, float* V, int64_t ldc,
-                                      cudaStream_t st) {
+                                      void* tc_work, cudaStream_t st) {
     ScoreArgs a;
     scoot_status s = fill_state_args(ctx, L, state, a);
     if (s != SCOOT_OK) return s;
+    if (tc_work && ctx->tensor_cores) {
+        ScootTcArgs t = tc_args(ctx, a);
+        t.cand = cand;
+        t.n = n;
+        t.ld = ld;
+        t.list = list;
+        t.n_list = n_list;
+        t.mean = mean;
+        t.var = var;
+        t.ldo = ldc;
+        t.vout = V;
+        t.ldv = ldc;
+        t.by_index = 0;
+        t.bsplit = static_cast<uint8_t*>(tc_work);
+        const int DO = tc_do(a);
+        if (scoot_tc_supported(ctx, t, DO)) return scoot_posterior_tc(ctx, t, DO, st);
+    }
     a.cand = cand;
     a.n = n;
     a.ld = ld;
@@ -718,7 +769,35 @@ scoot_status scoot_gp_posterior(scoot_ctx* ctx, const scoot_gp_layout* L, const 
     a.mean = mean;
     a.var = var;
     a.ldo = ldo;
-    return launch_score<kWriteMoments, 1>(ctx, a, static_cast<cudaStream_t>(stream));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (ctx->tensor_cores && a.n_rb * kRB <= kMaxNpadTc) {
+        // Workspace: the compacted list (when masked), then the split copy of
+        // L^{-1}; reserved whole before the compaction writes the list.
+        ScootTcArgs t = tc_args(ctx, a);
+        const int DO = tc_do(a);
+        if (scoot_tc_supported(ctx, t, DO)) {
+            const size_t list_bytes = mask ? ((256 + (size_t)n * 4 + 255) & ~(size_t)255) : 0;
+            if ((s = scoot_workspace(ctx, list_bytes + (size_t)scoot_tc_bsplit_bytes(t.n_pad, t.n_obj))) != SCOOT_OK)
+                return s;
+            if (mask) {
+                ScootList lst;
+                if ((s = scoot_compact(ctx, mask, n, nullptr, 0u, st, &lst)) != SCOOT_OK) return s;
+                t.list = lst.list;
+                t.n_list = lst.count;
+            }
+            t.cand = cand;
+            t.n = n;
+            t.ld = ld;
+            t.mean = mean;
+            t.var = var;
+            t.ldo = ldo;
+            t.vout = nullptr;
+            t.by_index = 1;
+            t.bsplit = static_cast<uint8_t*>(ctx->ws) + list_bytes;
+            return scoot_posterior_tc(ctx, t, DO, st);
+        }
+    }
+    return launch_score<kWriteMoments, 1>(ctx, a, st);
 }
 
 scoot_status scoot_acq_ei(scoot_ctx* ctx, const float* mean, const float* var, const uint8_t* mask,

@@ -92,6 +92,7 @@ _PROTOS = {
     "scoot_ctx_check": [_vp, _vp],
     "scoot_ctx_workspace_bytes": [_vp, C.POINTER(_i64)],
     "scoot_ctx_set_timing": [_vp, _i32],
+    "scoot_ctx_set_tensor_cores": [_vp, _i32],
     "scoot_probe_fma": [_vp, _i32, _i32, _i32, _vp, _vp],
     "scoot_probe_gather": [_vp, _i32, _i32, _i32, _vp, _vp],
     "scoot_ctx_phase_times": [_vp, _i32, _vp, _vp, C.POINTER(_i32)],
@@ -243,6 +244,10 @@ PHASES = {0: "compact", 1: "posterior", 2: "fant_init", 3: "fant_pass", 4: "fant
 
 def scoot_ctx_set_timing(ctx, enable: bool) -> None:
     _check(lib().scoot_ctx_set_timing(_h(ctx), int(bool(enable))), "scoot_ctx_set_timing", _h(ctx))
+
+
+def scoot_ctx_set_tensor_cores(ctx, enable: bool) -> None:
+    _check(lib().scoot_ctx_set_tensor_cores(_h(ctx), int(bool(enable))), "scoot_ctx_set_tensor_cores", _h(ctx))
 
 
 def scoot_ctx_phase_times(ctx, cap: int = 256):

@@ -237,18 +237,26 @@ def oracle_gps(inst, kernel=0):
                  inst.noise_var[m], kernel) for m in range(inst.n_obj)]
 
 
+@pytest.mark.parametrize("tc", [1, 0], ids=["tensor", "simt"])
 @pytest.mark.parametrize("name,kernel", [("tiny", 0), ("d8-ehvi2", 0), ("d10-ei", 0), ("d10-ehvi3", 0),
                                          ("d12-fantasy", 0), ("d8-ehvi2", 1)])
-def test_posterior_parity(S, ctx, name, kernel):
-    n = 4096 + 37  # several tiles and a ragged tail
+def test_posterior_parity(S, ctx, name, kernel, tc):
+    """Both products of L^{-1} k: the tensor-core one (three bf16 parts, six
+    part products) and the fp32 SIMT one."""
+    n = 4096 + 37  # several tiles (32 and 128 candidates) and a ragged tail
     inst = make_instance(name, seeds(name)[1], n_cand=n)
     L, state = gp_state(S, inst, kernel)
     M = inst.n_obj
     ldo = n + 3
     mean = torch.full((M, ldo), 77.0, device="cuda")
     var = torch.full((M, ldo), 77.0, device="cuda")
-    S.scoot_gp_posterior(ctx, L, state, cand_dev(inst), n, mean, var)
-    gm, gv = np_(mean), np_(var)
+    S.scoot_ctx_set_tensor_cores(ctx, tc)
+    try:
+        S.scoot_gp_posterior(ctx, L, state, cand_dev(inst), n, mean, var)
+        gm, gv = np_(mean), np_(var)
+    finally:
+        S.scoot_ctx_set_tensor_cores(ctx, 1)
+    name = f"{name} {'tensor' if tc else 'simt'}"
     assert np.all(gm[:, n:] == 77.0) and np.all(gv[:, n:] == 77.0)
     for m, gp in enumerate(oracle_gps(inst, kernel)):
         mu, v = gp.posterior(inst.cand, n)
