@@ -15,8 +15,9 @@
 // five smaller ones (h m, m h, h l, l h, m m) to a correction accumulator,
 // where their truncations weigh 2^-8 less; V = main + corr.
 //
-// One CTA per SM, 256 threads: thread t serves candidate row t mod 128 (the
-// TMEM lane its warp can read) and column half t / 128.  Per objective the
+// One CTA per SM, 16 SIMT warps and a control warp: SIMT thread t serves
+// candidate row t mod 128 (the TMEM lane its warp can read) and column
+// quarter t / 128.  Per objective the
 // rows of L^{-1} go in k-blocks of 32 columns; k-block kb only reaches output
 // rows i >= 32 kb (L^{-1} is lower triangular), so its products are MMAs of
 // N = n_pad - 32 kb columns starting at column 32 kb of each accumulator
@@ -26,10 +27,11 @@
 //     and B slot (g + 1) mod 3;
 //   - cp.async the three B parts of k-block g + 1 (from the split copy of
 //     L^{-1} prepared once per call by bsplit_kernel) into B slot (g + 1) mod 3;
-//   - every thread evaluates its 16 covariances of k-block g, splits them and
-//     stores the parts into A slot g mod 2 (the MMAs of g - 1 run meanwhile);
-//   - one thread issues the 12 MMAs of k-block g (2 K-steps x 6 part products)
-//     and commits them to mbarrier g mod 2.
+//   - every SIMT thread evaluates its 8 covariances of k-block g, splits them,
+//     stores the parts into A slot g mod 2 and arrives on its full barrier
+//     (the MMAs of g - 1 run meanwhile);
+//   - the control thread waits for A and B of g, issues the 12 MMAs of k-block
+//     g (2 K-steps x 6 part products) and commits them to mbarrier g mod 2.
 // After the last k-block the threads read D back (tcgen05.ld), write V in the
 // float4-group layout of the fantasy pass, and finish mu and sigma^2.
 //
@@ -48,7 +50,8 @@ using namespace scoot_dev;
 
 constexpr int kTM = 128;          // candidates per tile: the MMA's M and the TMEM lanes
 constexpr int kKB = 32;           // columns of L^{-1} per k-block
-constexpr int kThr = 256;         // two threads per candidate row
+constexpr int kQt = 4;            // threads per candidate row (column quarters of a k-block)
+constexpr int kThr = kTM * kQt;   // SIMT threads (16 warps); one more warp issues copies and MMAs
 constexpr int kParts = 3;         // bf16 parts of an fp32 operand
 constexpr uint32_t kLBO = 128;    // bytes between core matrices along K
 constexpr uint32_t kSBO = 512;    // bytes between 8-row groups of a k-block
@@ -173,8 +176,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
     uint8_t* sB = sA + 2 * kParts * kAPart;                          // [3][3][bchunk]
     float* xs = reinterpret_cast<float*>(sB + 3 * kParts * bchunk);  // [M][n_obs][DO] scaled observations
     float* al = xs + (size_t)a.n_obj * a.n_obs * DO;                 // [M][n_pad] alpha
-    float* red = al + (size_t)a.n_obj * a.n_pad;                     // [4][kTM]: |V|^2 and mu halves
-    float* cat_s = red + 4 * kTM;                                    // staged categorical table
+    float* red = al + (size_t)a.n_obj * a.n_pad;                     // [2][kQt][kTM]: |V|^2 and mu quarters
+    float* cat_s = red + 2 * kQt * kTM;                              // staged categorical table
     __shared__ float4 fm[kMaxD];
     __shared__ __align__(8) uint64_t bars[kBars];
     __shared__ uint32_t tslot;
@@ -283,8 +286,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
             if (!ok) atomicOr(a.err, SCOOT_DEVERR_TIMEOUT);
         }
     } else {
-        // ---- SIMT warps: thread t serves candidate row t mod 128 and column half t / 128.
-        const int r = tid & (kTM - 1), half = tid >> 7;
+        // ---- SIMT warps: thread t serves candidate row t mod 128 and column quarter t / 128.
+        const int r = tid & (kTM - 1), qd = tid >> 7;
         int64_t g = 0, t_obj = 0;  // k-blocks and tile-objectives done
         bool ok = true;
         for (int64_t it = 0; it < my_tiles && ok; ++it) {
@@ -307,7 +310,7 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 const int nc = (int)f.y;
                 int v = (int)__ldg(a.cand + (int64_t)f.w * a.ld + i);
                 if (v < 0 || v >= nc) {
-                    if (half == 0) atomicOr(a.err, SCOOT_DEVERR_INDEX);
+                    if (qd == 0) atomicOr(a.err, SCOOT_DEVERR_INDEX);
                     v = v < 0 ? 0 : nc - 1;
                 }
                 pid += v * (int)f.z;
@@ -329,37 +332,37 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                     ut[q] = q < n_ord ? x * gils[m * a.d + q] : 0.0f;
                 }
                 float mu_part = 0.0f;
-                // The categorical part of r^2 for this thread's 16 columns of the
+                // The categorical part of r^2 for this thread's 8 columns of the
                 // k-block, loaded one k-block ahead (rows past n_obs clamped).
-                float catv[16];
+                float catv[8];
 #pragma unroll
-                for (int e = 0; e < 16; ++e) catv[e] = catrow[(size_t)min(16 * half + e, a.n_obs - 1) * a.n_pat];
+                for (int e = 0; e < 8; ++e) catv[e] = catrow[(size_t)min(8 * qd + e, a.n_obs - 1) * a.n_pat];
                 for (int kb = 0; kb < KB; ++kb, ++g) {
-                    // This thread's 16 covariances: columns 32 kb + 16 half + [0, 16).
-                    const int c0 = kKB * kb + 16 * half;
-                    float kv[16];
+                    // This thread's 8 covariances: columns 32 kb + 8 qd + [0, 8).
+                    const int c0 = kKB * kb + 8 * qd;
+                    float kv[8];
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) {
+                    for (int e = 0; e < 8; ++e) {
                         const int c = c0 + e;
                         const float4* xj4 = reinterpret_cast<const float4*>(xsm + (size_t)min(c, a.n_obs - 1) * DO);
-                        float r2 = catv[e];
+                        float rp[DO / 4];  // one partial sum per float4 of coordinates
 #pragma unroll
                         for (int q4 = 0; q4 < DO / 4; ++q4) {
                             const float4 xv = xj4[q4];
                             const float t0 = ut[q4 * 4] - xv.x, t1 = ut[q4 * 4 + 1] - xv.y;
                             const float t2 = ut[q4 * 4 + 2] - xv.z, t3 = ut[q4 * 4 + 3] - xv.w;
-                            r2 = fmaf(t0, t0, r2);
-                            r2 = fmaf(t1, t1, r2);
-                            r2 = fmaf(t2, t2, r2);
-                            r2 = fmaf(t3, t3, r2);
+                            rp[q4] = fmaf(t3, t3, fmaf(t2, t2, fmaf(t1, t1, t0 * t0)));
                         }
+                        float r2 = catv[e];
+#pragma unroll
+                        for (int q4 = 0; q4 < DO / 4; ++q4) r2 += rp[q4];
                         const float k = (live && c < a.n_obs) ? sf2 * matern(sqrtf(r2), a.kernel) : 0.0f;
                         mu_part = fmaf(k, alm[c], mu_part);
                         kv[e] = k;
                     }
                     if (kb + 1 < KB) {
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) catv[e] = catrow[(size_t)min(c0 + kKB + e, a.n_obs - 1) * a.n_pat];
+                        for (int e = 0; e < 8; ++e) catv[e] = catrow[(size_t)min(c0 + kKB + e, a.n_obs - 1) * a.n_pat];
                     }
                     // A slot g & 1 was last read by the MMAs of g - 2.
                     if (g >= 2 && !mbar_wait_use(&bars[kMmaDone + (int)(g & 1)], (g - 2) >> 1)) {
@@ -367,23 +370,21 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                         break;
                     }
                     uint8_t* adst = sA + (size_t)(g & 1) * kParts * kAPart;
-#pragma unroll
-                    for (int grp = 0; grp < 2; ++grp) {
+                    {
                         uint32_t w[kParts][4];
 #pragma unroll
                         for (int u2 = 0; u2 < 8; u2 += 2) {
                             __nv_bfloat16 h0, m0, l0, h1, m1, l1;
-                            split3(kv[grp * 8 + u2], h0, m0, l0);
-                            split3(kv[grp * 8 + u2 + 1], h1, m1, l1);
+                            split3(kv[u2], h0, m0, l0);
+                            split3(kv[u2 + 1], h1, m1, l1);
                             w[0][u2 / 2] = pack2(h0, h1);
                             w[1][u2 / 2] = pack2(m0, m1);
                             w[2][u2 / 2] = pack2(l0, l1);
                         }
-                        const uint32_t off = canon_off(r, 16 * half + 8 * grp);
+                        const uint32_t off = canon_off(r, 8 * qd);
 #pragma unroll
                         for (int p = 0; p < kParts; ++p)
-                            *reinterpret_cast<uint4*>(adst + p * kAPart + off) =
-                                make_uint4(w[p][0], w[p][1], w[p][2], w[p][3]);
+                            *reinterpret_cast<uint4*>(adst + p * kAPart + off) = make_uint4(w[p][0], w[p][1], w[p][2], w[p][3]);
                     }
                     // visible to the tensor core (async proxy), then announced
                     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -398,8 +399,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 float sq = 0.0f;
                 float4* dst4 = reinterpret_cast<float4*>(a.vout);
-                const int hw = a.n_pad / 2;
-                for (int cc = half * hw; cc < (half + 1) * hw; cc += 16) {
+                const int qw = a.n_pad / kQt;  // columns of this thread's quarter (a multiple of 16)
+                for (int cc = qd * qw; cc < (qd + 1) * qw; cc += 16) {
                     uint32_t v[16], w[16];
                     const uint32_t taddr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)cc;
                     asm volatile(
@@ -434,8 +435,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 // D may be overwritten by the next tile-objective's MMAs.
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 mbar_arrive(&bars[kDFree]);
-                red[half * kTM + r] = sq;
-                red[(2 + half) * kTM + r] = mu_part;
+                red[qd * kTM + r] = sq;
+                red[(kQt + qd) * kTM + r] = mu_part;
                 // Both halves' sums are in red (a bounded wait, not a hardware barrier, so
                 // that a thread that gave up elsewhere cannot hold the others).
                 mbar_arrive(&bars[kRed]);
@@ -443,10 +444,11 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                     ok = false;
                     break;
                 }
-                if (half == 0 && live) {
+                if (qd == 0 && live) {
+                    const float* rs = red + r;
                     const int64_t o = (int64_t)m * a.ldo + (a.by_index ? i : pos);
-                    a.mean[o] = red[2 * kTM + r] + red[3 * kTM + r];
-                    a.var[o] = fmaxf(sf2 - (red[r] + red[kTM + r]), 0.0f);
+                    a.mean[o] = (rs[4 * kTM] + rs[5 * kTM]) + (rs[6 * kTM] + rs[7 * kTM]);
+                    a.var[o] = fmaxf(sf2 - ((rs[0] + rs[kTM]) + (rs[2 * kTM] + rs[3 * kTM])), 0.0f);
                 }
             }
         }
@@ -460,7 +462,7 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
 
 size_t tc_smem(const ScootTcArgs& a, int DO) {
     return (size_t)2 * kParts * kAPart + (size_t)3 * kParts * a.n_pad * 64 + (size_t)a.n_obj * a.n_obs * DO * 4 +
-           (size_t)a.n_obj * a.n_pad * 4 + (size_t)4 * kTM * 4 + (size_t)a.cat_smem * 4;
+           (size_t)a.n_obj * a.n_pad * 4 + (size_t)2 * kQt * kTM * 4 + (size_t)a.cat_smem * 4;
 }
 
 template <int DO>
