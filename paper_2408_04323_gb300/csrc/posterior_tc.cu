@@ -290,31 +290,48 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
         const int r = tid & (kTM - 1), qd = tid >> 7;
         int64_t g = 0, t_obj = 0;  // k-blocks and tile-objectives done
         bool ok = true;
+        // The list entries are read one tile ahead and the next tile's pool
+        // words prefetched into L2, so a tile starts on an L2 read, not on two
+        // dependent HBM reads.
+        auto index_at = [&](int64_t it2) -> int64_t {
+            const int64_t p2 = (blockIdx.x + it2 * gridDim.x) * kTM + r;
+            return (it2 < my_tiles && p2 < n_work) ? (a.list ? (int64_t)a.list[p2] : p2) : 0;
+        };
+        int64_t i_cur = index_at(0), i_nxt = index_at(1);
         for (int64_t it = 0; it < my_tiles && ok; ++it) {
             const int64_t tile = blockIdx.x + it * gridDim.x;
             const int64_t pos = tile * kTM + r;
             const bool live = pos < n_work;
-            const int64_t i = live ? (a.list ? (int64_t)a.list[pos] : pos) : 0;
+            const int64_t i = i_cur;
+            uint32_t wcur[kMaxD];
+#pragma unroll
+            for (int q = 0; q < kMaxD; ++q) wcur[q] = q < a.d ? __ldg(a.cand + (int64_t)fm[q].w * a.ld + i) : 0u;
             float u[DO];
 #pragma unroll
             for (int q = 0; q < DO; ++q) {
                 u[q] = 0.0f;
                 if (q < n_ord && live) {
                     const float4 f = fm[q];
-                    u[q] = feature_of(__ldg(a.cand + (int64_t)f.w * a.ld + i), (int)f.x, f.y, f.z);
+                    u[q] = feature_of(wcur[q], (int)f.x, f.y, f.z);
                 }
             }
             int pid = 0;  // joint category pattern (mixed radix), out-of-range categories clamped and flagged
-            for (int q = n_ord; q < a.d && live; ++q) {
+#pragma unroll
+            for (int q = 0; q < kMaxD; ++q) {
+                if (q < n_ord || q >= a.d || !live) continue;
                 const float4 f = fm[q];
                 const int nc = (int)f.y;
-                int v = (int)__ldg(a.cand + (int64_t)f.w * a.ld + i);
+                int v = (int)wcur[q];
                 if (v < 0 || v >= nc) {
                     if (qd == 0) atomicOr(a.err, SCOOT_DEVERR_INDEX);
                     v = v < 0 ? 0 : nc - 1;
                 }
                 pid += v * (int)f.z;
             }
+            const int64_t i_nn = index_at(it + 2);
+            if (qd == 0)
+                for (int q = 0; q < a.d; ++q)
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(a.cand + (int64_t)fm[q].w * a.ld + i_nxt));
             for (int m = 0; m < M && ok; ++m) {
                 const float* xsm = xs + (size_t)m * a.n_obs * DO;
                 const float* alm = al + (size_t)m * a.n_pad;
@@ -427,8 +444,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                         for (int g4 = 0; g4 < 4; ++g4) {
                             const int gi = (cc >> 2) + g4;  // float4 group of rows 4 gi .. 4 gi + 3
                             if (4 * gi < a.n_obs)
-                                dst4[((int64_t)m * (a.n_pad / 4) + gi) * a.ldv + pos] =
-                                    make_float4(vf[4 * g4], vf[4 * g4 + 1], vf[4 * g4 + 2], vf[4 * g4 + 3]);
+                                __stcs(dst4 + ((int64_t)m * (a.n_pad / 4) + gi) * a.ldv + pos,
+                                       make_float4(vf[4 * g4], vf[4 * g4 + 1], vf[4 * g4 + 2], vf[4 * g4 + 3]));
                         }
                     }
                 }
@@ -451,6 +468,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                     a.var[o] = fmaxf(sf2 - ((rs[0] + rs[kTM]) + (rs[2 * kTM] + rs[3 * kTM])), 0.0f);
                 }
             }
+            i_cur = i_nxt;
+            i_nxt = i_nn;
         }
         if (!ok) atomicOr(a.err, SCOOT_DEVERR_TIMEOUT);
     }
