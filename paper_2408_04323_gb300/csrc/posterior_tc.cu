@@ -92,6 +92,21 @@ __device__ __forceinline__ uint32_t pack2(__nv_bfloat16 lo, __nv_bfloat16 hi) {
     return (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
 }
 
+// split3 of a pair (x0 in the low halves), with paired conversions: the parts
+// as packed bf16 pairs h, m, l.
+__device__ __forceinline__ void split3x2(float x0, float x1, uint32_t& h, uint32_t& m, uint32_t& l) {
+    const __nv_bfloat162 hb = __floats2bfloat162_rn(x0, x1);
+    const float2 hf = __bfloat1622float2(hb);
+    const float2 r1 = __fadd2_rn(make_float2(x0, x1), make_float2(-hf.x, -hf.y));  // exact
+    const __nv_bfloat162 mb = __floats2bfloat162_rn(r1.x, r1.y);
+    const float2 mf = __bfloat1622float2(mb);
+    const float2 r2 = __fadd2_rn(r1, make_float2(-mf.x, -mf.y));                    // exact
+    const __nv_bfloat162 lb = __floats2bfloat162_rn(r2.x, r2.y);
+    h = *reinterpret_cast<const uint32_t*>(&hb);
+    m = *reinterpret_cast<const uint32_t*>(&mb);
+    l = *reinterpret_cast<const uint32_t*>(&lb);
+}
+
 __device__ __forceinline__ unsigned long long global_ns() {
     unsigned long long t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -174,8 +189,9 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
     const uint32_t bchunk = (uint32_t)a.n_pad * 64;
     uint8_t* sA = smem;                                              // [2][3][8 KiB]
     uint8_t* sB = sA + 2 * kParts * kAPart;                          // [3][3][bchunk]
-    float* xs = reinterpret_cast<float*>(sB + 3 * kParts * bchunk);  // [M][n_obs][DO] scaled observations
-    float* al = xs + (size_t)a.n_obj * a.n_obs * DO;                 // [M][n_pad] alpha
+    const int npair = (a.n_obs + 1) / 2;
+    float* xs = reinterpret_cast<float*>(sB + 3 * kParts * bchunk);  // [M][npair][DO][2] scaled observations
+    float* al = xs + (size_t)a.n_obj * npair * DO * 2;               // [M][n_pad] alpha
     float* red = al + (size_t)a.n_obj * a.n_pad;                     // [2][kQt][kTM]: |V|^2 and mu quarters
     float* cat_s = red + 2 * kQt * kTM;                              // staged categorical table
     __shared__ float4 fm[kMaxD];
@@ -190,10 +206,14 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
     const float* gcat = reinterpret_cast<const float*>(a.state + a.off_cat);
     if (tid < kMaxD) fm[tid] = tid < a.d ? gfmap[tid] : make_float4((float)SCOOT_CATEGORICAL, 0.f, 0.f, 0.f);
     for (int e = tid; e < a.cat_smem; e += blockDim.x) cat_s[e] = __ldg(gcat + e);
-    // The observations' scaled ordinal coordinates and alpha, every objective, once.
-    for (int e = tid; e < a.n_obj * a.n_obs * DO; e += blockDim.x) {
-        const int mj = e / DO, q = e - mj * DO;
-        xs[e] = q < a.n_ord ? gxs[(size_t)mj * a.d + q] : 0.0f;
+    // The observations' scaled ordinal coordinates and alpha, every objective,
+    // once; coordinates interleaved by pairs of observations (2p, 2p + 1), so
+    // one 16-byte load gives two coordinates of both (the last pair of an odd
+    // count repeats its observation).
+    for (int e = tid; e < a.n_obj * npair * DO * 2; e += blockDim.x) {
+        const int s = e & 1, q = (e >> 1) % DO, mp = (e >> 1) / DO;
+        const int m = mp / npair, j = min(2 * (mp - m * npair) + s, a.n_obs - 1);
+        xs[e] = q < a.n_ord ? gxs[((size_t)m * a.n_obs + j) * a.d + q] : 0.0f;
     }
     for (int e = tid; e < a.n_obj * a.n_pad; e += blockDim.x) {
         const int m = e / a.n_pad, j = e - m * a.n_pad;
@@ -333,7 +353,7 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 for (int q = 0; q < a.d; ++q)
                     asm volatile("prefetch.global.L2 [%0];" ::"l"(a.cand + (int64_t)fm[q].w * a.ld + i_nxt));
             for (int m = 0; m < M && ok; ++m) {
-                const float* xsm = xs + (size_t)m * a.n_obs * DO;
+                const float* xsm = xs + (size_t)m * npair * DO * 2;
                 const float* alm = al + (size_t)m * a.n_pad;
                 const float sf2 = gscal[m * 4 + 0];
                 const bool warped = gscal[m * 4 + 3] != 0.0f;
@@ -357,25 +377,36 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 for (int kb = 0; kb < KB; ++kb, ++g) {
                     // This thread's 8 covariances: columns 32 kb + 8 qd + [0, 8).
                     const int c0 = kKB * kb + 8 * qd;
+                    // Distances two columns at a time (packed fp32 pairs): d = u - x
+                    // exactly (an FMA with -1), r^2 accumulated per float4 of coordinates.
                     float kv[8];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const int c = c0 + e;
-                        const float4* xj4 = reinterpret_cast<const float4*>(xsm + (size_t)min(c, a.n_obs - 1) * DO);
-                        float rp[DO / 4];  // one partial sum per float4 of coordinates
+                    for (int e = 0; e < 8; e += 2) {
+                        const int c = c0 + e;  // even
+                        const float4* xp = reinterpret_cast<const float4*>(xsm + (size_t)min(c >> 1, npair - 1) * DO * 2);
+                        float2 rp[DO / 4];
 #pragma unroll
                         for (int q4 = 0; q4 < DO / 4; ++q4) {
-                            const float4 xv = xj4[q4];
-                            const float t0 = ut[q4 * 4] - xv.x, t1 = ut[q4 * 4 + 1] - xv.y;
-                            const float t2 = ut[q4 * 4 + 2] - xv.z, t3 = ut[q4 * 4 + 3] - xv.w;
-                            rp[q4] = fmaf(t3, t3, fmaf(t2, t2, fmaf(t1, t1, t0 * t0)));
+                            const float4 v01 = xp[2 * q4], v23 = xp[2 * q4 + 1];  // coordinates 4 q4 .. 4 q4 + 3
+                            const float2 d0 = __ffma2_rn(make_float2(v01.x, v01.y), make_float2(-1.f, -1.f),
+                                                         make_float2(ut[4 * q4], ut[4 * q4]));
+                            const float2 d1 = __ffma2_rn(make_float2(v01.z, v01.w), make_float2(-1.f, -1.f),
+                                                         make_float2(ut[4 * q4 + 1], ut[4 * q4 + 1]));
+                            const float2 d2 = __ffma2_rn(make_float2(v23.x, v23.y), make_float2(-1.f, -1.f),
+                                                         make_float2(ut[4 * q4 + 2], ut[4 * q4 + 2]));
+                            const float2 d3 = __ffma2_rn(make_float2(v23.z, v23.w), make_float2(-1.f, -1.f),
+                                                         make_float2(ut[4 * q4 + 3], ut[4 * q4 + 3]));
+                            rp[q4] = __ffma2_rn(d3, d3, __ffma2_rn(d2, d2, __ffma2_rn(d1, d1, __fmul2_rn(d0, d0))));
                         }
-                        float r2 = catv[e];
 #pragma unroll
-                        for (int q4 = 0; q4 < DO / 4; ++q4) r2 += rp[q4];
-                        const float k = (live && c < a.n_obs) ? sf2 * matern(sqrtf(r2), a.kernel) : 0.0f;
-                        mu_part = fmaf(k, alm[c], mu_part);
-                        kv[e] = k;
+                        for (int h = 0; h < 2; ++h) {
+                            float r2 = catv[e + h];
+#pragma unroll
+                            for (int q4 = 0; q4 < DO / 4; ++q4) r2 += h ? rp[q4].y : rp[q4].x;
+                            const float k = (live && c + h < a.n_obs) ? sf2 * matern(sqrtf(r2), a.kernel) : 0.0f;
+                            mu_part = fmaf(k, alm[c + h], mu_part);
+                            kv[e + h] = k;
+                        }
                     }
                     if (kb + 1 < KB) {
 #pragma unroll
@@ -390,14 +421,7 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                     {
                         uint32_t w[kParts][4];
 #pragma unroll
-                        for (int u2 = 0; u2 < 8; u2 += 2) {
-                            __nv_bfloat16 h0, m0, l0, h1, m1, l1;
-                            split3(kv[u2], h0, m0, l0);
-                            split3(kv[u2 + 1], h1, m1, l1);
-                            w[0][u2 / 2] = pack2(h0, h1);
-                            w[1][u2 / 2] = pack2(m0, m1);
-                            w[2][u2 / 2] = pack2(l0, l1);
-                        }
+                        for (int u2 = 0; u2 < 8; u2 += 2) split3x2(kv[u2], kv[u2 + 1], w[0][u2 / 2], w[1][u2 / 2], w[2][u2 / 2]);
                         const uint32_t off = canon_off(r, 8 * qd);
 #pragma unroll
                         for (int p = 0; p < kParts; ++p)
@@ -480,7 +504,7 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
 }
 
 size_t tc_smem(const ScootTcArgs& a, int DO) {
-    return (size_t)2 * kParts * kAPart + (size_t)3 * kParts * a.n_pad * 64 + (size_t)a.n_obj * a.n_obs * DO * 4 +
+    return (size_t)2 * kParts * kAPart + (size_t)3 * kParts * a.n_pad * 64 + (size_t)a.n_obj * ((a.n_obs + 1) / 2) * DO * 8 +
            (size_t)a.n_obj * a.n_pad * 4 + (size_t)2 * kQt * kTM * 4 + (size_t)a.cat_smem * 4;
 }
 
