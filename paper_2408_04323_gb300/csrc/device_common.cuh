@@ -6,6 +6,15 @@
 
 namespace scoot_dev {
 
+// The whitened rows V of the fantasy path, tiled by 32 list positions: the
+// float4 group g (rows 4 g .. 4 g + 3) of objective m of list position p is
+// float4 number ((p / 32) M + m) (n_pad / 4) 32 + 32 g + p mod 32.  The 32
+// candidates of a warp then read or write 512 contiguous bytes per group,
+// and each tile of 32 candidates is one contiguous block of HBM.
+__host__ __device__ __forceinline__ int64_t vtile_index(int64_t p, int m, int g, int M, int n4) {
+    return (((p >> 5) * M + m) * (int64_t)n4 + g) * 32 + (p & 31);
+}
+
 __device__ __forceinline__ float matern(float r, int kernel) {
     if (kernel == SCOOT_MATERN32) {
         const float a = 1.7320508075688772f * r;

@@ -523,13 +523,13 @@ __global__ void __launch_bounds__(kPassThreads, M == 2 ? 4 : 1) fant_pass(const 
                 const float k = gscal[m * 4] * matern(sqrtf(r2[m]), a.kernel);
                 // v(x) . v_p over float4 groups of four rows (16-byte loads;
                 // rows past n_obs are zero on both sides).
-                const float4* vrow = reinterpret_cast<const float4*>(a.V) + (int64_t)m * (a.n_pad / 4) * a.ldc + pos;
+                const float4* vrow = reinterpret_cast<const float4*>(a.V) + vtile_index(pos, m, 0, M, a.n_pad / 4);
                 const float4* vpm = reinterpret_cast<const float4*>(vps + m * a.n_pad);
                 const int groups = (a.n_obs + 3) / 4;
                 float d0 = 0.0f, d1 = 0.0f, d2 = 0.0f, d3 = 0.0f;
 #pragma unroll 8
                 for (int g = 0; g < groups; ++g) {
-                    const float4 v = __ldcs(vrow + (int64_t)g * a.ldc);
+                    const float4 v = __ldcs(vrow + 32 * g);
                     const float4 w = vpm[g];
                     d0 = fmaf(v.x, w.x, d0);
                     d1 = fmaf(v.y, w.y, d1);
@@ -849,7 +849,7 @@ WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q, int box_cap) 
     int64_t o = 0;
     w.mean = o;     o = up256(o + M * n * 4);
     w.var = o;      o = up256(o + M * n * 4);
-    w.V = o;        o = up256(o + M * n_pad * n * 4);
+    w.V = o;        o = up256(o + M * n_pad * ((n + 31) / 32 * 32) * 4);  // tiled by 32 candidates
     w.C = o;        o = up256(o + (int64_t)std::max(q - 2, 1) * M * n * 4);
     w.ctrl = o;     o = up256(o + (int64_t)sizeof(Ctrl));
     w.picked = o;   o = up256(o + (int64_t)q * 8);

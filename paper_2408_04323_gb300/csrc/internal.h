@@ -145,9 +145,10 @@ scoot_status scoot_compact(scoot_ctx* ctx, const uint8_t* mask, int64_t n, uint3
 
 // Posterior of the listed candidates into list-position order: mean and var
 // [M][ldc], and the whitened rows V = L^{-1} k(X, x) in float4 groups of four
-// rows, [M][n_rb * 16][ldc][4] (16-byte aligned; groups wholly past row n
-// left unwritten, rows past n inside a written group zero).  ldc >= the list
-// length.
+// rows, tiled by 32 list positions (scoot_dev::vtile_index), ceil(list
+// length / 32) tiles of M * n_rb * 16 * 32 float4 (16-byte aligned; groups
+// wholly past row n left unwritten, rows past n inside a written group zero).
+// ldc >= the list length.
 // tc_work (may be NULL: the SIMT product) is device scratch of at least
 // scoot_tc_bsplit_bytes(n_pad, M) bytes, 16-byte aligned, for the split copy
 // of L^{-1} that the tensor-core product reads.
@@ -171,7 +172,6 @@ struct ScootTcArgs {
     float* var;
     int64_t ldo;
     float* vout;      // NULL: moments only
-    int64_t ldv;
     int32_t by_index; // mean / var at the candidate's index (else at its list position)
     uint8_t* bsplit;  // [M][n_pad / 32][3][n_pad * 64 bytes]
     uint32_t* err;

@@ -33,7 +33,8 @@
 //   - the control thread waits for A and B of g, issues the 12 MMAs of k-block
 //     g (2 K-steps x 6 part products) and commits them to mbarrier g mod 2.
 // After the last k-block the threads read D back (tcgen05.ld), write V in the
-// float4-group layout of the fantasy pass, and finish mu and sigma^2.
+// tiled float4-group layout of the fantasy pass (vtile_index), and finish mu
+// and sigma^2.
 //
 // Operand layout in shared memory: the canonical no-swizzle K-major form of
 // a 32-wide k-block: 8-row x 16-byte core matrices, 128 bytes apart along K
@@ -468,7 +469,7 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                         for (int g4 = 0; g4 < 4; ++g4) {
                             const int gi = (cc >> 2) + g4;  // float4 group of rows 4 gi .. 4 gi + 3
                             if (4 * gi < a.n_obs)
-                                __stcs(dst4 + ((int64_t)m * (a.n_pad / 4) + gi) * a.ldv + pos,
+                                __stcs(dst4 + vtile_index(pos, m, gi, M, a.n_pad / 4),
                                        make_float4(vf[4 * g4], vf[4 * g4 + 1], vf[4 * g4 + 2], vf[4 * g4 + 3]));
                         }
                     }

@@ -63,8 +63,7 @@ struct ScoreArgs {
     int32_t cat_smem;             // floats of the categorical table staged in shared memory (0: read from L1)
     int32_t cat_off;              // where, in floats from the start of shared memory
     int32_t wbuf_off;             // the next tile's pool words [d][kTC], in floats from the start
-    float* vout;                  // kWriteWhitened: V = L^{-1} k*, [M][n_pad / 4][ldv][4] by list position
-    int64_t ldv;
+    float* vout;                  // kWriteWhitened: V = L^{-1} k* by list position, tiled (vtile_index)
     uint32_t* err;                // device error word
 };
 
@@ -362,9 +361,9 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                 if (EPI == kWriteWhitened) {
                     // Rows of V for the fantasy downdates, indexed by list
                     // position, in float4 groups of four rows (this thread's
-                    // rows are one group): group g of candidate p at
-                    // (m n_pad / 4 + g) * ldv + p.  Rows past n_obs hold zeros
-                    // (L^{-1} is zero-filled there).
+                    // rows are one group), tiled by 32 candidates
+                    // (vtile_index).  Rows past n_obs hold zeros (L^{-1} is
+                    // zero-filled there).
                     float4* dst4 = reinterpret_cast<float4*>(a.vout);
                     const int g = rb * (kRB / 4) + rg;
                     if (4 * g < a.n_obs) {
@@ -372,7 +371,7 @@ score_kernel(const __grid_constant__ ScoreArgs a) {
                         for (int c = 0; c < 4; ++c) {
                             const int64_t p = tile * kTC + cg * 4 + c;
                             if (p < n_work)
-                                dst4[((int64_t)m * (n_pad64 / 4) + g) * a.ldv + p] =
+                                dst4[vtile_index(p, m, g, a.n_obj, (int)(n_pad64 / 4))] =
                                     make_float4(accm[0][c], accm[1][c], accm[2][c], accm[3][c]);
                         }
                     }
@@ -731,7 +730,6 @@ scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, 
         t.var = var;
         t.ldo = ldc;
         t.vout = V;
-        t.ldv = ldc;
         t.by_index = 0;
         t.bsplit = static_cast<uint8_t*>(tc_work);
         const int DO = tc_do(a);
@@ -746,7 +744,6 @@ scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, 
     a.var = var;
     a.ldo = ldc;
     a.vout = V;
-    a.ldv = ldc;
     return launch_score<kWriteWhitened, 1>(ctx, a, st);
 }
 

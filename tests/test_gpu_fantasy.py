@@ -85,11 +85,15 @@ def _tol_at(inst, ref, gps, j, ks):
     return propagated_tol(f, mu, var, e_mu, ATOL + RTOL * var)
 
 
-@pytest.mark.parametrize("seed_i,n,q", [(0, 2048, 16), (1, 1500, 6)])
-def test_fantasy_picks_follow_the_refit_oracle(S, seed_i, n, q):
+@pytest.mark.parametrize("seed_i,n,q,tc", [(0, 2048, 16, 1), (1, 1500, 6, 1), (0, 2048, 16, 0)],
+                         ids=["2048-q16-tensor", "1500-q6-tensor", "2048-q16-simt"])
+def test_fantasy_picks_follow_the_refit_oracle(S, seed_i, n, q, tc):
+    """tc: the whitened posterior's L^{-1} k product on the tensor cores or in
+    fp32 SIMT (both write the tiled rows of V the passes read)."""
     name = "d12-fantasy"
     inst = make_instance(name, seeds(name)[seed_i], n_cand=n)
     ctx = S.Context(0)
+    S.scoot_ctx_set_tensor_cores(ctx, tc)
     try:
         r = _round_inputs(S, inst, q)
         var_out = torch.full((inst.n_obj, n), -1.0, device="cuda")
