@@ -380,7 +380,10 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                     const int c0 = kKB * kb + 8 * qd;
                     // Distances two columns at a time (packed fp32 pairs): d = u - x
                     // exactly (an FMA with -1), r^2 accumulated per float4 of coordinates.
-                    float kv[8];
+                    // In stages over the 8 columns (distances, then square roots,
+                    // then the kernel), so that their independent sqrt / exp
+                    // chains overlap.
+                    float r2v[8];
 #pragma unroll
                     for (int e = 0; e < 8; e += 2) {
                         const int c = c0 + e;  // even
@@ -404,11 +407,16 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                             float r2 = catv[e + h];
 #pragma unroll
                             for (int q4 = 0; q4 < DO / 4; ++q4) r2 += h ? rp[q4].y : rp[q4].x;
-                            const float k = (live && c + h < a.n_obs) ? sf2 * matern(sqrtf(r2), a.kernel) : 0.0f;
-                            mu_part = fmaf(k, alm[c + h], mu_part);
-                            kv[e + h] = k;
+                            r2v[e + h] = r2;
                         }
                     }
+                    float kv[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) kv[e] = sqrtf(r2v[e]);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) kv[e] = (live && c0 + e < a.n_obs) ? sf2 * matern(kv[e], a.kernel) : 0.0f;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) mu_part = fmaf(kv[e], alm[c0 + e], mu_part);
                     if (kb + 1 < KB) {
 #pragma unroll
                         for (int e = 0; e < 8; ++e) catv[e] = catrow[(size_t)min(c0 + kKB + e, a.n_obs - 1) * a.n_pat];
