@@ -47,15 +47,15 @@ FP32_LANES_PER_SM = 128
 # keyed by (kernel, workload), valid only while the kernel's sources are
 # unchanged (sha256 prefix of their contents when the counters were taken).
 KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["score.cu", "device_common.cuh"],
-                "posterior": ["score.cu", "device_common.cuh"], "fant_pass": ["fantasy.cu", "device_common.cuh"],
+                "posterior": ["posterior_tc.cu", "device_common.cuh"], "fant_pass": ["fantasy.cu", "device_common.cuh"],
                 "topq": ["topq.cu", "device_common.cuh"], "pareto": ["pareto.cu"]}
 TRAFFIC = {
     # d12-fantasy: captured on a 2^20 pool of the same workload, scaled to the 2^22 launch by its
     # live candidates (x 4.0025; fant_pass and the posterior) or its pool size (x 4; prune, forest)
-    ("fant_pass", "d12-fantasy"): {"bytes": 3562300000, "sha": "aa97db9cc922aeb9"},
-    ("posterior", "d12-fantasy"): {"bytes": 3485600000, "sha": "6b2aeb7ebc645ff4"},
-    ("rf", "d12-fantasy"): {"bytes": 210480000, "sha": "f14ca23df538ac20"},
-    ("prune", "d12-fantasy"): {"bytes": 100680000, "sha": "f14ca23df538ac20"},
+    ("fant_pass", "d12-fantasy"): {"bytes": 3566500000, "sha": "391d07d63f4e8047"},
+    ("posterior", "d12-fantasy"): {"bytes": 3442600000, "sha": "fef1b84575f65e56"},
+    ("rf", "d12-fantasy"): {"bytes": 227260000, "sha": "df8284c4f1f3b084"},
+    ("prune", "d12-fantasy"): {"bytes": 100700000, "sha": "df8284c4f1f3b084"},
     ("score", "d10-ehvi3"): {"bytes": 44739000, "sha": "6b2aeb7ebc645ff4"},
 }
 
@@ -165,6 +165,15 @@ def posterior_flops(inst, n_obj=None):
     d, n = inst.d, inst.n_obs
     m = inst.n_obj if n_obj is None else n_obj
     return m * (n * (3 * d + 12) + 2 * n + n * (n + 1) + 2 * n)
+
+
+def posterior_tensor_flops(inst, n_obj=None):
+    """bf16 flops per candidate that the tensor-core posterior issues: per
+    objective, k-block kb of 32 columns of L^{-1} reaches rows 32 kb .. n_pad - 1,
+    and each of its 32 columns takes six part products (2 flops each)."""
+    n_pad = 64 * ((inst.n_obs + 63) // 64)
+    m = inst.n_obj if n_obj is None else n_obj
+    return m * 6 * 2 * 32 * sum(n_pad - 32 * kb for kb in range(n_pad // 32))
 
 
 def forest_visits(inst, idx):
@@ -1041,6 +1050,15 @@ def main():
         pick_ms, n_pick = mean_of("fant_pick")
         init_ms, _ = mean_of("fant_init")
         kernels["posterior"] = alu_roof(posterior_flops(inst) * n_feasible, post_ms, "posterior (whitened rows)")
+        if 64 * ((inst.n_obs + 63) // 64) <= 256:  # the L^{-1} k product runs on the tensor cores
+            tf = posterior_tensor_flops(inst) * n_feasible
+            bf16 = peaks.get("bf16_tflops") if peaks else None
+            kernels["posterior"]["tensor"] = {
+                "bf16_flops_per_launch": tf, "achieved_tflops": tf / (post_ms / 1e3) / 1e12,
+                "peak_tflops": bf16, "frac": (tf / (post_ms / 1e3) / 1e12) / bf16 if bf16 else None,
+                "peak_source": "measured (MEASURED_PEAKS.json bf16_tflops, burst)" if bf16 else None,
+                "note": "the work above counts the fp32-equivalent product once; the tensor cores run six bf16 "
+                        "part products of it"}
         pb = fantasy_pass_bytes(inst, inp.q, n_feasible)[:n_pass]
         kernels["fant_pass"] = hbm_roof(statistics.mean(pb), pass_ms / n_pass, "fant_pass")
         kernels["fant_pass"]["launches_per_step"] = n_pass
