@@ -101,6 +101,7 @@ struct FantArgs {
     int32_t n_part;               // blocks of a pass
     uint64_t* rec;                // [SCOOT_FANT_REC] this shard's record of the current pass
     uint32_t* pick_words;         // [16] configuration of the latest pick (from the winning record)
+    double* fmap64;               // [16][2] offset and scale of each parameter's feature map (feature_map64)
     int64_t* out_idx;             // [q]
     float* out_val;               // [q]
     int32_t* out_count;
@@ -153,6 +154,24 @@ __device__ __forceinline__ double warp_sum(double v) {
     return v;
 }
 
+// Exclusive prefix over the block (kPickThreads threads) of one flag per
+// thread, and the flags' total; every thread calls it.
+__device__ __forceinline__ int block_flag_prefix(bool flag, int* warp_tot, int* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const unsigned b = __ballot_sync(0xffffffffu, flag);
+    if (lane == 0) warp_tot[warp] = __popc(b);
+    __syncthreads();
+    int off = 0, tot = 0;
+    for (int k = 0; k < nw; ++k) {
+        const int c = warp_tot[k];
+        off += k < warp ? c : 0;
+        tot += c;
+    }
+    __syncthreads();  // warp_tot may be reused
+    *total = tot;
+    return off + __popc(b & ((1u << lane) - 1u));
+}
+
 // Order-preserving integer key of a double: x < y exactly when key(x) <
 // key(y), for values that are not NaN; -0 and +0 share the key of +0.  The
 // front and box logic compares these keys on the integer pipes.
@@ -173,18 +192,35 @@ __device__ __forceinline__ double matern64(double r, int kernel) {
     return (1.0 + a + a * a / 3.0) * exp(-a);
 }
 
-// Feature coordinate (fp64) of a stored word of parameter c: log scale for
-// integer log-uniform, linear for integer uniform and continuous, the index
-// for categoricals.  Returns false for a word that has no feature.
-__device__ __forceinline__ bool feature64(const double* sp, int c, uint32_t w, double* u) {
+// Offset and scale of parameter c's feature map (fp64): log(lo) and
+// 1 / (log(hi) - log(lo)) for integer log-uniform, lo and 1 / (hi - lo) (0
+// when hi <= lo) for integer uniform and continuous; computed once per call
+// (fant_init), so that a pick's features cost one log at most.
+__device__ __forceinline__ void feature_map64(const double* sp, int c, double* fm2) {
     const int kind = (int)sp[c * 4];
     const double lo = sp[c * 4 + 1], hi = sp[c * 4 + 2];
+    if (kind == SCOOT_INT_LOG) {
+        const double l0 = log(lo);
+        fm2[0] = l0;
+        fm2[1] = 1.0 / (log(hi) - l0);
+    } else {
+        fm2[0] = lo;
+        fm2[1] = hi > lo ? 1.0 / (hi - lo) : 0.0;
+    }
+}
+
+// Feature coordinate (fp64) of a stored word of parameter c: log scale for
+// integer log-uniform, linear for integer uniform and continuous, the index
+// for categoricals (fm2: the offset and scale of feature_map64).  Returns
+// false for a word that has no feature.
+__device__ __forceinline__ bool feature64(const double* sp, const double* fm2, int c, uint32_t w, double* u) {
+    const int kind = (int)sp[c * 4];
     const double v = kind == SCOOT_CONTINUOUS ? (double)__uint_as_float(w) : (double)(int32_t)w;
     if (kind == SCOOT_INT_LOG) {
         if (!(v > 0.0)) return false;
-        *u = (log(v) - log(lo)) / (log(hi) - log(lo));
+        *u = (log(v) - fm2[2 * c]) * fm2[2 * c + 1];
     } else if (kind == SCOOT_INT_UNIFORM || kind == SCOOT_CONTINUOUS) {
-        *u = hi > lo ? (v - lo) / (hi - lo) : 0.0;
+        *u = (v - fm2[2 * c]) * fm2[2 * c + 1];
     } else {
         *u = v;
     }
@@ -225,40 +261,66 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
     const int tid = threadIdx.x;
     if (tid == 0) s_nf = a.ctrl->n_front;
     if (tid < M) s_ref[tid] = okey(h.ref[tid]);
+    if (tid < 4) s_A[tid] = 0;
     __syncthreads();
     for (int e = tid; e < s_nf * M; e += blockDim.x) F[e] = okey(a.front[e]);
     __syncthreads();
-    if (add && tid == 0) {
+    __shared__ int s_wt[32];
+    if (add) {  // (uniform: every thread takes part in the block-wide steps)
         long long zk[M];
-        bool above = true, covered = false;
+        bool above = true;
+#pragma unroll
         for (int m = 0; m < M; ++m) {
             zk[m] = okey(z[m]);
             above &= zk[m] > s_ref[m];
         }
-        for (int k = 0; k < s_nf && !covered; ++k) {
+        const int nf0 = s_nf;
+        int cov = 0;  // some front point weakly dominates z
+        for (int k = tid; k < nf0; k += blockDim.x) {
             bool ge = true;
+#pragma unroll
             for (int m = 0; m < M; ++m) ge &= F[k * M + m] >= zk[m];
-            covered = ge;
+            cov |= ge;
         }
+        const bool covered = __syncthreads_or(cov) != 0;
         if (above && !covered) {
-            int w = 0;
-            for (int k = 0; k < s_nf; ++k) {
-                bool ge = true, gt = false;
-                for (int m = 0; m < M; ++m) {
-                    ge &= zk[m] >= F[k * M + m];
-                    gt |= zk[m] > F[k * M + m];
+            // Keep, in order, the points z does not dominate (a stable compaction
+            // in chunks of the block: a point moves only to a lower position, and
+            // every point of a chunk is read before any is written), then z.
+            int base = 0;
+            for (int c0 = 0; c0 < nf0; c0 += blockDim.x) {
+                const int k = c0 + tid;
+                long long pt[M];
+                bool keep = false;
+                if (k < nf0) {
+                    bool ge = true, gt = false;
+#pragma unroll
+                    for (int m = 0; m < M; ++m) {
+                        pt[m] = F[k * M + m];
+                        ge &= zk[m] >= pt[m];
+                        gt |= zk[m] > pt[m];
+                    }
+                    keep = !(ge && gt);  // not dominated by the fantasy
                 }
-                if (ge && gt) continue;  // dominated by the fantasy
-                for (int m = 0; m < M; ++m) F[w * M + m] = F[k * M + m];
-                ++w;
+                int tot;
+                const int pos = block_flag_prefix(keep, s_wt, &tot);
+                if (keep) {
+#pragma unroll
+                    for (int m = 0; m < M; ++m) F[(base + pos) * M + m] = pt[m];
+                }
+                base += tot;
+                __syncthreads();
             }
-            if (w < fcap) {
-                for (int m = 0; m < M; ++m) F[w * M + m] = zk[m];
-                ++w;
-            } else {
-                atomicOr(a.err, SCOOT_DEVERR_CAPACITY);
+            if (tid == 0) {
+                int w = base;
+                if (w < fcap) {
+                    for (int m = 0; m < M; ++m) F[w * M + m] = zk[m];
+                    ++w;
+                } else {
+                    atomicOr(a.err, SCOOT_DEVERR_CAPACITY);
+                }
+                s_nf = w;
             }
-            s_nf = w;
         }
     }
     __syncthreads();
@@ -282,11 +344,10 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
             for (int u = 0; u <= nf; ++u) below += first[u] && (u == 0 ? s_ref[j] : F[(u - 1) * M + j]) < v;
             axis[j * (fcap + 1) + below] = v;
         }
-        if (tid == 0) {
-            int cnt = 0;
-            for (int t = 0; t <= nf; ++t) cnt += first[t];
-            s_A[j] = cnt;
-        }
+        int cnt = 0;
+        for (int t = tid; t <= nf; t += blockDim.x) cnt += first[t];
+        cnt = __reduce_add_sync(0xffffffffu, cnt);
+        if ((tid & 31) == 0 && cnt) atomicAdd(&s_A[j], cnt);
         __syncthreads();
     }
     int cells = 1;
@@ -321,43 +382,81 @@ __device__ void front_update_and_boxes(const FantArgs& a, const FantHeader& h, b
     }
     __syncthreads();
     // Boxes per row (cells merged while the floor repeats), then their offsets.
-    for (int r = tid; r < rows; r += blockDim.x) {
-        int cnt = 1;
-        for (int kk = 1; kk < A_last; ++kk) cnt += cell[r * A_last + kk] != cell[r * A_last + kk - 1];
-        rowcnt[r + 1] = cnt;
-    }
-    __syncthreads();
-    if (tid == 0) {
-        rowcnt[0] = 0;
-        for (int r = 0; r < rows; ++r) rowcnt[r + 1] += rowcnt[r];
-        s_total = rowcnt[rows];
-        s_ok = s_total <= a.box_cap;
-    }
-    __syncthreads();
-    for (int r = tid; r < rows && s_ok; r += blockDim.x) {
+    const long long* al = axis + (G - 1) * (fcap + 1);
+    if (rows == 1) {
+        // One row (two objectives, or one value on every other axis): a box per
+        // run of equal floors, the cells in parallel; a cell's box is the number
+        // of run starts up to it, less one (a block-wide prefix).
         float lo_pre[G > 1 ? G - 1 : 1], up_pre[G > 1 ? G - 1 : 1];
-        int rest = r;
-        for (int j = G - 2; j >= 0; --j) {
-            const int kj = rest % s_A[j];
-            rest /= s_A[j];
-            lo_pre[j] = (float)okey_value(axis[j * (fcap + 1) + kj]);
-            up_pre[j] = kj + 1 < s_A[j] ? (float)okey_value(axis[j * (fcap + 1) + kj + 1]) : __int_as_float(0x7f800000);
+        for (int j = 0; j < G - 1; ++j) {
+            lo_pre[j] = (float)okey_value(axis[j * (fcap + 1)]);
+            up_pre[j] = 1 < s_A[j] ? (float)okey_value(axis[j * (fcap + 1) + 1]) : __int_as_float(0x7f800000);
         }
-        int b = rowcnt[r] - 1;
-        const long long* al = axis + (G - 1) * (fcap + 1);
-        for (int kk = 0; kk < A_last; ++kk) {
-            const long long fl = cell[r * A_last + kk];
-            if (kk == 0 || fl != cell[r * A_last + kk - 1]) {
-                ++b;
-                for (int j = 0; j < G - 1; ++j) {
-                    a.box_lo[b * M + j] = lo_pre[j];
-                    a.box_hi[b * M + j] = up_pre[j];
+        int base = 0;
+        for (int c0 = 0; c0 < A_last; c0 += blockDim.x) {
+            const int kk = c0 + tid;
+            const bool in = kk < A_last;
+            const bool start = in && (kk == 0 || cell[kk] != cell[kk - 1]);
+            int tot;
+            const int pos = block_flag_prefix(start, s_wt, &tot);
+            const int b = base + pos + (start ? 0 : -1);
+            if (in && b < a.box_cap) {
+                if (start) {
+                    for (int j = 0; j < G - 1; ++j) {
+                        a.box_lo[b * M + j] = lo_pre[j];
+                        a.box_hi[b * M + j] = up_pre[j];
+                    }
+                    a.box_lo[b * M + G - 1] = (float)okey_value(al[kk]);
+                    a.box_lo[b * M + M - 1] = (float)okey_value(cell[kk]);
+                    a.box_hi[b * M + M - 1] = __int_as_float(0x7f800000);
                 }
-                a.box_lo[b * M + G - 1] = (float)okey_value(al[kk]);
-                a.box_lo[b * M + M - 1] = (float)okey_value(fl);
-                a.box_hi[b * M + M - 1] = __int_as_float(0x7f800000);
+                if (kk + 1 == A_last || cell[kk + 1] != cell[kk])  // the run's last cell
+                    a.box_hi[b * M + G - 1] = kk + 1 < A_last ? (float)okey_value(al[kk + 1]) : __int_as_float(0x7f800000);
             }
-            a.box_hi[b * M + G - 1] = kk + 1 < A_last ? (float)okey_value(al[kk + 1]) : __int_as_float(0x7f800000);
+            base += tot;
+        }
+        if (tid == 0) {
+            s_total = base;
+            s_ok = base <= a.box_cap;
+        }
+    } else {
+        for (int r = tid; r < rows; r += blockDim.x) {
+            int cnt = 1;
+            for (int kk = 1; kk < A_last; ++kk) cnt += cell[r * A_last + kk] != cell[r * A_last + kk - 1];
+            rowcnt[r + 1] = cnt;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            rowcnt[0] = 0;
+            for (int r = 0; r < rows; ++r) rowcnt[r + 1] += rowcnt[r];
+            s_total = rowcnt[rows];
+            s_ok = s_total <= a.box_cap;
+        }
+        __syncthreads();
+        for (int r = tid; r < rows && s_ok; r += blockDim.x) {
+            float lo_pre[G > 1 ? G - 1 : 1], up_pre[G > 1 ? G - 1 : 1];
+            int rest = r;
+            for (int j = G - 2; j >= 0; --j) {
+                const int kj = rest % s_A[j];
+                rest /= s_A[j];
+                lo_pre[j] = (float)okey_value(axis[j * (fcap + 1) + kj]);
+                up_pre[j] = kj + 1 < s_A[j] ? (float)okey_value(axis[j * (fcap + 1) + kj + 1]) : __int_as_float(0x7f800000);
+            }
+            int b = rowcnt[r] - 1;
+            for (int kk = 0; kk < A_last; ++kk) {
+                const long long fl = cell[r * A_last + kk];
+                if (kk == 0 || fl != cell[r * A_last + kk - 1]) {
+                    ++b;
+                    for (int j = 0; j < G - 1; ++j) {
+                        a.box_lo[b * M + j] = lo_pre[j];
+                        a.box_hi[b * M + j] = up_pre[j];
+                    }
+                    a.box_lo[b * M + G - 1] = (float)okey_value(al[kk]);
+                    a.box_lo[b * M + M - 1] = (float)okey_value(fl);
+                    a.box_hi[b * M + M - 1] = __int_as_float(0x7f800000);
+                }
+                a.box_hi[b * M + G - 1] = kk + 1 < A_last ? (float)okey_value(al[kk + 1]) : __int_as_float(0x7f800000);
+            }
         }
     }
     __syncthreads();
@@ -444,6 +543,8 @@ __global__ void __launch_bounds__(kPickThreads) fant_init(const __grid_constant_
     if (!ok) return;
     const double* f0 = reinterpret_cast<const double*>(a.fant + h.off_front);
     for (int e = threadIdx.x; e < h.front0 * M; e += blockDim.x) a.front[e] = f0[e];
+    if (threadIdx.x < a.d)
+        feature_map64(reinterpret_cast<const double*>(a.fant + h.off_space), threadIdx.x, a.fmap64 + 2 * threadIdx.x);
     __syncthreads();
     front_update_and_boxes<M>(a, h, false, nullptr, smem);
 }
@@ -647,7 +748,7 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
     __syncthreads();
     if (tid < d) {  // the pick's features (one thread each) ...
         double x = 0.0;
-        if (!feature64(sp, tid, s_words[tid], &x)) s_bad = 1;
+        if (!feature64(sp, a.fmap64, tid, s_words[tid], &x)) s_bad = 1;
         u[tid] = x;
         if (lead) a.upick[(size_t)j * d + tid] = x;
     } else if (tid >= 32 && tid < 32 + d) {  // ... and, in another warp, the length scales
@@ -712,25 +813,29 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
     if (tid == 0) a.ctrl->arrived_m[m] = 0u;
     double* vv = reinterpret_cast<double*>(smem);  // [n] v_p
     double* D = vv + n;                            // [q] v_p . v_{p_t}
-    double* bq = D + q;                            // [q] k(x_p, x_{p_t}) - v_p . v_{p_t}
+    double* bq = D + q;                            // [q] k(x_p, x_{p_t}), then minus v_p . v_{p_t}
     double* cq = bq + q;                           // [q] c_t(x_p)
     double* red = cq + q;                          // [32]
     double* red2 = red + 32;                       // [32]
+    double* Ws = red2 + 32;                        // [j][q] rows of W of the earlier picks
+    // The phase's global reads go out together (an in-order pipe would
+    // otherwise wait for each load before issuing the next): W's rows and
+    // k(x_p, x_{p_t}) into shared memory, each thread's slab parts into registers.
+    const double* W = a.wf + (size_t)m * q * q;
+    for (int e = tid; e < j * q; e += blockDim.x) Ws[e] = W[e];
+    for (int t = tid; t < j; t += blockDim.x) bq[t] = __ldcg(a.kpt + (size_t)m * q + t);
     const double* pm = a.part + (size_t)m * B * n;
     double* vrow = a.vpick + ((size_t)j * M + m) * n;
     double vv_part = 0.0;
     for (int i = tid; i < n; i += blockDim.x) {
-        const int nb = min(B, i / w + 1);  // the slabs with c0 <= i, summed in slab order by fours
-        double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
-        int k = 0;
-        for (; k + 3 < nb; k += 4) {
-            s0 += __ldcg(pm + (size_t)k * n + i);
-            s1 += __ldcg(pm + (size_t)(k + 1) * n + i);
-            s2 += __ldcg(pm + (size_t)(k + 2) * n + i);
-            s3 += __ldcg(pm + (size_t)(k + 3) * n + i);
-        }
-        for (; k < nb; ++k) s0 += __ldcg(pm + (size_t)k * n + i);
-        const double v = (s0 + s1) + (s2 + s3);
+        const int nb = min(B, i / w + 1);  // the slabs with c0 <= i, summed in slab order, k mod 4 apart
+        double pv[kPickSlabMax];
+#pragma unroll
+        for (int k = 0; k < kPickSlabMax; ++k) pv[k] = __ldcg(pm + (size_t)min(k, nb - 1) * n + i);
+        double sk[4] = {0.0, 0.0, 0.0, 0.0};
+#pragma unroll
+        for (int k = 0; k < kPickSlabMax; ++k) sk[k & 3] += k < nb ? pv[k] : 0.0;
+        const double v = (sk[0] + sk[1]) + (sk[2] + sk[3]);
         vv[i] = v;
         vrow[i] = v;
         a.vp[m * a.n_pad + i] = (float)v;
@@ -743,17 +848,28 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         s = warp_sum(s);
         if (tid == 0) a.mupick[(size_t)j * M + m] = s;
     }
-    const double vnorm = block_sum(vv_part, red);  // (its barriers also publish vv)
-    {  // v_p . v_{p_t}: a warp per two earlier picks
+    const double vnorm = block_sum(vv_part, red);  // (its barriers also publish vv, Ws and bq)
+    {  // v_p . v_{p_t}: a warp per two earlier picks, eight rows per lane loaded before use
         const int lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
         for (int t = warp; t < j; t += 2 * nw) {
             const int t2 = t + nw < j ? t + nw : t;
             const double* va = a.vpick + ((size_t)t * M + m) * n;
             const double* vb = a.vpick + ((size_t)t2 * M + m) * n;
             double sa = 0.0, sb = 0.0;
-            for (int i = lane; i < n; i += 32) {
-                sa = fma(vv[i], va[i], sa);
-                sb = fma(vv[i], vb[i], sb);
+            for (int i0 = lane; i0 < n; i0 += 32 * 8) {
+                double xa[8], xb[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int i = min(i0 + 32 * u, n - 1);
+                    xa[u] = va[i];
+                    xb[u] = vb[i];
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    if (i0 + 32 * u < n) {
+                        sa = fma(vv[i0 + 32 * u], xa[u], sa);
+                        sb = fma(vv[i0 + 32 * u], xb[u], sb);
+                    }
             }
             for (int o = 16; o > 0; o >>= 1) {
                 sa += __shfl_xor_sync(0xffffffffu, sa, o);
@@ -766,13 +882,12 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         }
     }
     __syncthreads();
-    for (int t = tid; t < j; t += blockDim.x) bq[t] = __ldcg(a.kpt + (size_t)m * q + t) - D[t];
+    for (int t = tid; t < j; t += blockDim.x) bq[t] -= D[t];
     __syncthreads();
     // c(x_p) = W b: row t of W holds t + 1 entries.
-    const double* W = a.wf + (size_t)m * q * q;
     double csq = 0.0;
     for (int t = tid; t < j; t += blockDim.x) {
-        const double* wt = W + (size_t)t * q;
+        const double* wt = Ws + (size_t)t * q;
         double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
         int k = 0;
         for (; k + 3 <= t; k += 4) {
@@ -801,10 +916,10 @@ __global__ void __launch_bounds__(kPickThreads) fant_pick(const __grid_constant_
         double s0 = 0.0, s1 = 0.0;
         int k = t;
         for (; k + 1 < j; k += 2) {
-            s0 = fma(cq[k], W[(size_t)k * q + t], s0);
-            s1 = fma(cq[k + 1], W[(size_t)(k + 1) * q + t], s1);
+            s0 = fma(cq[k], Ws[(size_t)k * q + t], s0);
+            s1 = fma(cq[k + 1], Ws[(size_t)(k + 1) * q + t], s1);
         }
-        if (k < j) s0 = fma(cq[k], W[(size_t)k * q + t], s0);
+        if (k < j) s0 = fma(cq[k], Ws[(size_t)k * q + t], s0);
         wj[t] = -inv * (s0 + s1);
     }
     for (int t = tid; t < q; t += blockDim.x) a.cxp[m * q + t] = t < j ? (float)cq[t] : 0.0f;
@@ -837,7 +952,7 @@ scatter_var(const int32_t* list, const unsigned int* n_list, int64_t n, int64_t 
 
 struct WorkLayout {
     int64_t mean, var, V, C, ctrl, picked, vp, cxp, inv_s, upick, vpick, wf, part, mupart, kpt, mupick, front,
-        box_lo, box_hi, part_key, part_pos, rec, words, tcb, tcb_bytes, bytes;
+        box_lo, box_hi, part_key, part_pos, rec, words, fmap64, tcb, tcb_bytes, bytes;
 };
 
 int64_t up256(int64_t x) { return (x + 255) / 256 * 256; }
@@ -870,6 +985,7 @@ WorkLayout work_layout(const scoot_gp_layout* L, int64_t n, int q, int box_cap) 
     w.part_pos = o; o = up256(o + kPartMax * 4);
     w.rec = o;      o = up256(o + SCOOT_FANT_REC * 8);
     w.words = o;    o = up256(o + 16 * 4);
+    w.fmap64 = o;   o = up256(o + 16 * 2 * 8);
     // the split copy of L^{-1} for the tensor-core posterior (when n_pad allows it)
     w.tcb_bytes = n_pad <= kMaxNpadTc ? scoot_tc_bsplit_bytes((int)n_pad, (int)M) : 0;
     w.tcb = o;      o = up256(o + w.tcb_bytes);
@@ -897,7 +1013,7 @@ scoot_status set_attributes(scoot_ctx* ctx, Session& ss) {
     const FantArgs& a = ss.a;
     ss.pass_smem = (size_t)(2 * a.box_cap + a.n_mc) * 16 + (size_t)((a.q + 1) & ~1) * 8 + (size_t)M * a.n_pad * 4 +
                    (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4;
-    ss.pick_smem = std::max((size_t)std::max(32 + a.slab_w, a.n_obs + 3 * a.q + 64) * 8,
+    ss.pick_smem = std::max((size_t)std::max(32 + a.slab_w, a.n_obs + 3 * a.q + 64 + a.q * a.q) * 8,
                             boxes_smem(a.front_cap, M, a.box_cap));
     int max_smem = 0;
     SCOOT_CUDA(ctx, cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, ctx->device));
@@ -1011,6 +1127,7 @@ scoot_status scoot_fantasy_begin(scoot_ctx* ctx, const scoot_gp_layout* L, const
     a.part_pos = reinterpret_cast<int32_t*>(wk + w.part_pos);
     a.rec = reinterpret_cast<uint64_t*>(wk + w.rec);
     a.pick_words = reinterpret_cast<uint32_t*>(wk + w.words);
+    a.fmap64 = reinterpret_cast<double*>(wk + w.fmap64);
     a.out_idx = idx;
     a.out_val = val;
     a.out_count = count;
