@@ -45,6 +45,8 @@ namespace {
 using namespace scoot_dev;
 
 constexpr int kPassThreads = 256;
+constexpr int kCullQueue = 512;        // candidates queued for their exact EHVI per pass block
+constexpr int kCullSamplesMax = 256;   // base samples the culling's corners are built from
 constexpr int kPickThreads = 256;
 constexpr int kPartMax = 2048;   // per-block argmax partials of one pass
 constexpr int kPickSlabMax = 32;  // column slabs per objective of the pick's L^{-1} k product
@@ -62,6 +64,7 @@ struct Ctrl {
     int32_t n_front;
     int32_t local_pos;  // list position of this shard's best candidate of the current pass (-1: none)
     uint64_t local_key; // its selection key (global index)
+    uint64_t pass_best; // the largest exact selection key found so far in the current pass (culling)
 };
 
 struct FantArgs {
@@ -493,6 +496,7 @@ __device__ void pass_record(const FantArgs& a) {
     block_keymax(best, pos);
     if (threadIdx.x == 0) {
         a.ctrl->passed = 0u;
+        a.ctrl->pass_best = 0ull;  // for the next pass
         a.ctrl->local_key = best;
         a.ctrl->local_pos = best != 0ull ? pos : -1;
         a.rec[0] = best;
@@ -528,6 +532,7 @@ __global__ void __launch_bounds__(kPickThreads) fant_init(const __grid_constant_
         a.ctrl->arrived = 0u;
         for (int m = 0; m < SCOOT_MAX_OBJ; ++m) a.ctrl->arrived_m[m] = 0u;
         a.ctrl->passed = 0u;
+        a.ctrl->pass_best = 0ull;
         a.ctrl->local_key = 0ull;
         a.ctrl->local_pos = -1;
         a.ctrl->n_boxes = 0;
@@ -595,10 +600,9 @@ __global__ void __launch_bounds__(kPassThreads, M == 2 ? 4 : 1) fant_pass(const 
     uint64_t best = 0ull;
     int32_t best_pos = -1;
     const float inv_mc = 1.0f / (float)a.n_mc;
-    for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < n_live;
-         pos += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
-        float vr[M];
+    // The downdate of the candidate at list position pos (pick j - 1's rank-1
+    // term, stored), and its variances.
+    auto downdate = [&](int64_t pos, int64_t i, float* vr) {
         if (l >= 0) {
             float r2[M];
 #pragma unroll
@@ -649,23 +653,141 @@ __global__ void __launch_bounds__(kPassThreads, M == 2 ? 4 : 1) fant_pass(const 
 #pragma unroll
             for (int m = 0; m < M; ++m) vr[m] = a.var[(int64_t)m * a.ldc + pos];
         }
-        bool taken = false;
-        for (int t = 0; t < j; ++t) taken |= pk[t] == pos;
-        if (taken) continue;
-        float mu[M], sd[M];
-#pragma unroll
-        for (int m = 0; m < M; ++m) {
-            mu[m] = a.mean[(int64_t)m * a.ldc + pos];
-            sd[m] = sqrtf(fmaxf(vr[m], 0.0f));
-        }
-        float v;
+    };
+    auto exact = [&](const float* mu, const float* sd) -> float {
         if constexpr (M <= 3)  // (the saturated form takes two or three objectives)
-            v = fast ? ehvi_partial_sat<M>(mu, sd, blo, nb, epsv, a.n_mc, 0, 1) * inv_mc
-                     : ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
+            return fast ? ehvi_partial_sat<M>(mu, sd, blo, nb, epsv, a.n_mc, 0, 1) * inv_mc
+                        : ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
         else
-            v = ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
-        if (!(v != v) && v != -INFINITY)
-            keymax(best, best_pos, make_key(v, (uint32_t)(a.index_offset + i)), (int32_t)pos);
+            return ehvi_value<M>(mu, sd, blo, bhi, nb, epsv, a.n_mc);
+    };
+    const bool cull = fast && a.n_mc >= 16 && a.n_mc % 8 == 0 && a.n_mc <= kCullSamplesMax;
+    if (!cull) {
+        for (int64_t pos = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; pos < n_live;
+             pos += (int64_t)gridDim.x * blockDim.x) {
+            const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+            float vr[M];
+            downdate(pos, i, vr);
+            bool taken = false;
+            for (int t = 0; t < j; ++t) taken |= pk[t] == pos;
+            if (taken) continue;
+            float mu[M], sd[M];
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                mu[m] = a.mean[(int64_t)m * a.ldc + pos];
+                sd[m] = sqrtf(fmaxf(vr[m], 0.0f));
+            }
+            const float v = exact(mu, sd);
+            if (!(v != v) && v != -INFINITY)
+                keymax(best, best_pos, make_key(v, (uint32_t)(a.index_offset + i)), (int32_t)pos);
+        }
+    } else if constexpr (M <= 3) {
+        // Culling.  The samples, in 8-sample groups by rank of their first
+        // objective, give corners (the group's largest value per objective);
+        // the HVI is monotone in each objective (and its computed form too:
+        // every operation is monotone), so the group size times the HVI at
+        // the corner bounds the group's HVI sum, and the corners' sum bounds
+        // the EHVI.  A candidate whose bound's selection key (the bound
+        // raised by 2^-16 against the sums' roundings) is below the largest
+        // exact key found so far (this block's or any block's) cannot be the
+        // pass's argmax and skips its EHVI; the others queue in shared memory
+        // and are evaluated a block-full at a time, so a warp's lanes all have
+        // work.
+        const int ng = a.n_mc / 8;
+        float4* cornv = reinterpret_cast<float4*>(reinterpret_cast<uintptr_t>(ups + a.d + 3) & ~(uintptr_t)15);  // [ng]
+        int* rk = reinterpret_cast<int*>(cornv + ng);                   // [n_mc]
+        float* qmu = reinterpret_cast<float*>(rk + a.n_mc);              // [M][kCullQueue]
+        float* qsd = qmu + M * kCullQueue;                               // [M][kCullQueue]
+        int32_t* qpos = reinterpret_cast<int32_t*>(qsd + M * kCullQueue); // [kCullQueue]
+        uint32_t* qidx = reinterpret_cast<uint32_t*>(qpos + kCullQueue);  // [kCullQueue]
+        __shared__ unsigned long long s_best;
+        __shared__ int s_qn;
+        for (int s = threadIdx.x; s < a.n_mc; s += blockDim.x) {
+            const float e0 = epsv[s].x;
+            int r = 0;
+            for (int u = 0; u < a.n_mc; ++u) r += epsv[u].x < e0 || (epsv[u].x == e0 && u < s);
+            rk[s] = r;
+        }
+        if (threadIdx.x == 0) {
+            s_best = 0ull;
+            s_qn = 0;
+        }
+        __syncthreads();
+        for (int g = threadIdx.x; g < ng; g += blockDim.x) {
+            float4 c = make_float4(-INFINITY, -INFINITY, -INFINITY, 0.0f);
+            for (int s = 0; s < a.n_mc; ++s)
+                if (rk[s] / 8 == g) {
+                    const float4 e = epsv[s];
+                    c.x = fmaxf(c.x, e.x);
+                    c.y = fmaxf(c.y, e.y);
+                    c.z = fmaxf(c.z, e.z);
+                }
+            if (M < 3) c.z = 0.0f;
+            cornv[g] = c;
+        }
+        __syncthreads();
+        const int64_t first = (int64_t)blockIdx.x * blockDim.x;
+        const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+        const int64_t rounds = first < n_live ? (n_live - first + stride - 1) / stride : 0;  // block-uniform
+        unsigned long long gb = 0ull;
+        for (int64_t rd = 0; rd < rounds; ++rd) {
+            const int64_t pos = first + rd * stride + threadIdx.x;
+            const bool valid = pos < n_live;
+            const unsigned long long gb_next = *(volatile const unsigned long long*)&a.ctrl->pass_best;
+            if (valid) {
+                const int64_t i = a.list ? (int64_t)a.list[pos] : pos;
+                float vr[M];
+                downdate(pos, i, vr);
+                bool taken = false;
+                for (int t = 0; t < j; ++t) taken |= pk[t] == pos;
+                if (!taken) {
+                    float mu[M], sd[M];
+#pragma unroll
+                    for (int m = 0; m < M; ++m) {
+                        mu[m] = a.mean[(int64_t)m * a.ldc + pos];
+                        sd[m] = sqrtf(fmaxf(vr[m], 0.0f));
+                    }
+                    const uint32_t gi = (uint32_t)(a.index_offset + i);
+                    const float ub = ehvi_partial_sat<M>(mu, sd, blo, nb, cornv, ng, 0, 1) * (8.0f * inv_mc);
+                    const unsigned long long th = max(s_best, gb);
+                    if (ub != ub || make_key(ub * (1.0f + 1.0f / 65536.0f), gi) > th) {
+                        const int slot = atomicAdd(&s_qn, 1);
+#pragma unroll
+                        for (int m = 0; m < M; ++m) {
+                            qmu[m * kCullQueue + slot] = mu[m];
+                            qsd[m * kCullQueue + slot] = sd[m];
+                        }
+                        qpos[slot] = (int32_t)pos;
+                        qidx[slot] = gi;
+                    }
+                }
+            }
+            gb = max(gb, gb_next);
+            __syncthreads();
+            const int qn = s_qn;
+            if (qn >= (int)blockDim.x || rd + 1 == rounds) {
+                for (int e = threadIdx.x; e < qn; e += blockDim.x) {
+                    float mu[M], sd[M];
+#pragma unroll
+                    for (int m = 0; m < M; ++m) {
+                        mu[m] = qmu[m * kCullQueue + e];
+                        sd[m] = qsd[m * kCullQueue + e];
+                    }
+                    const float v = exact(mu, sd);
+                    if (!(v != v) && v != -INFINITY) {
+                        const uint64_t key = make_key(v, qidx[e]);
+                        keymax(best, best_pos, key, qpos[e]);
+                        atomicMax(&s_best, (unsigned long long)key);
+                    }
+                }
+                __syncthreads();
+                if (threadIdx.x == 0) {
+                    s_qn = 0;
+                    atomicMax((unsigned long long*)&a.ctrl->pass_best, s_best);
+                }
+                __syncthreads();
+            }
+        }
     }
     block_keymax(best, best_pos);
     if (threadIdx.x == 0) {
@@ -1012,7 +1134,8 @@ template <int M>
 scoot_status set_attributes(scoot_ctx* ctx, Session& ss) {
     const FantArgs& a = ss.a;
     ss.pass_smem = (size_t)(2 * a.box_cap + a.n_mc) * 16 + (size_t)((a.q + 1) & ~1) * 8 + (size_t)M * a.n_pad * 4 +
-                   (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4;
+                   (size_t)M * a.q * 4 + (size_t)M * 4 + (size_t)a.d * 4 + 16 +   // ... + culling:
+                   (size_t)(a.n_mc / 8) * 16 + (size_t)a.n_mc * 4 + (size_t)kCullQueue * (2 * M * 4 + 8);
     ss.pick_smem = std::max((size_t)std::max(32 + a.slab_w, a.n_obs + 3 * a.q + 64 + a.q * a.q) * 8,
                             boxes_smem(a.front_cap, M, a.box_cap));
     int max_smem = 0;
