@@ -150,11 +150,16 @@ def test_score_ehvi_exact_parity(S, ctx, name, k):
     ratio = np.abs(g[idx] - want) / tol
     print(f"[parity] score_ehvi_exact {name}: n={len(idx)} B={len(lo)} max|err|/tol={ratio.max():.3f}")
     assert ratio.max() <= 1.0
-    # fused == posterior + acq_ehvi_exact
+    # fused == posterior + acq_ehvi_exact (the posterior's product in fp32 SIMT, as in the fused
+    # kernel: the same arithmetic; the tensor-core product has its own parity test)
     M = inst.n_obj
     mean = torch.empty((M, n), device="cuda")
     vv = torch.empty((M, n), device="cuda")
-    S.scoot_gp_posterior(ctx, L, state, cand, n, mean, vv, mask)
+    S.scoot_ctx_set_tensor_cores(ctx, 0)
+    try:
+        S.scoot_gp_posterior(ctx, L, state, cand, n, mean, vv, mask)
+    finally:
+        S.scoot_ctx_set_tensor_cores(ctx, 1)
     acq2 = torch.empty(n, device="cuda")
     S.scoot_acq_ehvi_exact(ctx, mean, vv, n, grid, n_grid, corner, acq2, mask)
     g2 = np_(acq2)

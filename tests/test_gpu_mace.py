@@ -139,10 +139,15 @@ def test_score_mace_parity(S, ctx):
         print(f"[parity] score_mace {name} row {r}: n={len(idx)} max|err|/tol={ratio.max():.3f}")
         rows.append(ratio.max())
     assert max(rows) <= 1.0
-    # the fused kernel agrees with posterior + acq_mace
+    # the fused kernel agrees with posterior + acq_mace (the posterior's product in fp32 SIMT, as
+    # in the fused kernel)
     mean = torch.empty((1, n), device="cuda")
     vv = torch.empty((1, n), device="cuda")
-    S.scoot_gp_posterior(ctx, L, state, cand, n, mean, vv, mask)
+    S.scoot_ctx_set_tensor_cores(ctx, 0)
+    try:
+        S.scoot_gp_posterior(ctx, L, state, cand, n, mean, vv, mask)
+    finally:
+        S.scoot_ctx_set_tensor_cores(ctx, 1)
     acq2 = torch.empty((3, n), device="cuda")
     S.scoot_acq_mace(ctx, mean[0], vv[0], n, yb, xi, kappa, acq2, mask)
     g2 = np_(acq2)

@@ -358,7 +358,11 @@ def test_score_ehvi_parity(S, ctx, name, k):
         M = inst.n_obj
         mean = torch.empty((M, n), device="cuda")
         var_d = torch.empty((M, n), device="cuda")
-        S.scoot_gp_posterior(ctx, L, state, cand, n, mean, var_d, mask)
+        S.scoot_ctx_set_tensor_cores(ctx, 0)  # the fused kernel's fp32 SIMT product
+        try:
+            S.scoot_gp_posterior(ctx, L, state, cand, n, mean, var_d, mask)
+        finally:
+            S.scoot_ctx_set_tensor_cores(ctx, 1)
         acq2 = torch.empty(n, device="cuda")
         S.scoot_acq_ehvi(ctx, mean, var_d, n, lo, hi, eps, acq2, mask)
         g2 = np_(acq2)
