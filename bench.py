@@ -46,7 +46,8 @@ FP32_LANES_PER_SM = 128
 # DRAM bytes per launch from ncu (dram__bytes_read.sum + dram__bytes_write.sum),
 # keyed by (kernel, workload), valid only while the kernel's sources are
 # unchanged (sha256 prefix of their contents when the counters were taken).
-KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"], "score": ["score.cu", "device_common.cuh"],
+KERNEL_FILES = {"prune": ["prune_rf.cu"], "rf": ["prune_rf.cu"],
+                "score": ["score.cu", "posterior_tc.cu", "device_common.cuh"],
                 "posterior": ["posterior_tc.cu", "device_common.cuh"], "fant_pass": ["fantasy.cu", "device_common.cuh"],
                 "topq": ["topq.cu", "device_common.cuh"], "pareto": ["pareto.cu"]}
 TRAFFIC = {
@@ -1036,6 +1037,15 @@ def main():
         a = flops_per_launch / (launch_ms / 1e3) / 1e12
         return {"bound": "alu", "achieved": a, "peak": fp32_peak, "unit": "TFLOP/s", "frac": a / fp32_peak,
                 "kernel": name, "work_per_launch": flops_per_launch, "launch_ms": launch_ms}
+
+    def tensor_roof(bf16_flops, launch_ms):
+        bf16 = peaks.get("bf16_tflops") if peaks else None
+        a = bf16_flops / (launch_ms / 1e3) / 1e12
+        return {"bf16_flops_per_launch": bf16_flops, "achieved_tflops": a, "peak_tflops": bf16,
+                "frac": a / bf16 if bf16 else None,
+                "peak_source": "measured (MEASURED_PEAKS.json bf16_tflops, burst)" if bf16 else None,
+                "note": "the work above counts the fp32-equivalent product once; the tensor cores run six bf16 "
+                        "part products of it"}
     kernels = {}
     for s_ in ("prune", "rf"):
         k_, pc = work[s_]
@@ -1051,14 +1061,7 @@ def main():
         init_ms, _ = mean_of("fant_init")
         kernels["posterior"] = alu_roof(posterior_flops(inst) * n_feasible, post_ms, "posterior (whitened rows)")
         if 64 * ((inst.n_obs + 63) // 64) <= 256:  # the L^{-1} k product runs on the tensor cores
-            tf = posterior_tensor_flops(inst) * n_feasible
-            bf16 = peaks.get("bf16_tflops") if peaks else None
-            kernels["posterior"]["tensor"] = {
-                "bf16_flops_per_launch": tf, "achieved_tflops": tf / (post_ms / 1e3) / 1e12,
-                "peak_tflops": bf16, "frac": (tf / (post_ms / 1e3) / 1e12) / bf16 if bf16 else None,
-                "peak_source": "measured (MEASURED_PEAKS.json bf16_tflops, burst)" if bf16 else None,
-                "note": "the work above counts the fp32-equivalent product once; the tensor cores run six bf16 "
-                        "part products of it"}
+            kernels["posterior"]["tensor"] = tensor_roof(posterior_tensor_flops(inst) * n_feasible, post_ms)
         pb = fantasy_pass_bytes(inst, inp.q, n_feasible)[:n_pass]
         kernels["fant_pass"] = hbm_roof(statistics.mean(pb), pass_ms / n_pass, "fant_pass")
         kernels["fant_pass"]["launches_per_step"] = n_pass
@@ -1067,6 +1070,9 @@ def main():
     else:
         k_, pc = work["score"]
         kernels["score"] = alu_roof(pc * n_feasible, stage_ms["score"], "score")
+        if inp.acq in ("ei", "mace") and 64 * ((inst.n_obs + 63) // 64) <= 256:
+            # posterior and acquisition in the tensor-core kernel (objective 0)
+            kernels["score"]["tensor"] = tensor_roof(posterior_tensor_flops(inst, 1) * n_feasible, stage_ms["score"])
         last = "pareto" if inp.acq == "mace" else "topq"
         kernels[last] = hbm_roof(work[last][1] * N, stage_ms[last], last)
         kernel_ms = {k: stage_ms[k] for k in stage_names}

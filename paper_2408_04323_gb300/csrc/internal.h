@@ -175,6 +175,13 @@ struct ScootTcArgs {
     int32_t by_index; // mean / var at the candidate's index (else at its list position)
     uint8_t* bsplit;  // [M][n_pad / 32][3][n_pad * 64 bytes]
     uint32_t* err;
+    // Acquisition epilogue (objective 0 only, acq at the candidate's index;
+    // mean / var then unused): 0 none, 1 EI (Eq. 6) into acq[i], 2 MACE's
+    // UCB, PI and EI (Section 4.5) into acq[i], acq[lda + i], acq[2 lda + i].
+    int32_t acq_kind;
+    float* acq;
+    int64_t lda;
+    float xi, kappa;
 };
 int64_t scoot_tc_bsplit_bytes(int n_pad, int M);
 bool scoot_tc_supported(scoot_ctx* ctx, const ScootTcArgs& a, int DO);

@@ -34,7 +34,8 @@
 //     g (2 K-steps x 6 part products) and commits them to mbarrier g mod 2.
 // After the last k-block the threads read D back (tcgen05.ld), write V in the
 // tiled float4-group layout of the fantasy pass (vtile_index), and finish mu
-// and sigma^2.
+// and sigma^2, or in their place the acquisition (EI, or MACE's UCB, PI and
+// EI) when V is not wanted.
 //
 // Operand layout in shared memory: the canonical no-swizzle K-major form of
 // a 32-wide k-block: 8-row x 16-byte core matrices, 128 bytes apart along K
@@ -496,9 +497,23 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 }
                 if (qd == 0 && live) {
                     const float* rs = red + r;
-                    const int64_t o = (int64_t)m * a.ldo + (a.by_index ? i : pos);
-                    a.mean[o] = (rs[4 * kTM] + rs[5 * kTM]) + (rs[6 * kTM] + rs[7 * kTM]);
-                    a.var[o] = fmaxf(sf2 - ((rs[0] + rs[kTM]) + (rs[2 * kTM] + rs[3 * kTM])), 0.0f);
+                    const float mean = (rs[4 * kTM] + rs[5 * kTM]) + (rs[6 * kTM] + rs[7 * kTM]);
+                    const float var = fmaxf(sf2 - ((rs[0] + rs[kTM]) + (rs[2 * kTM] + rs[3 * kTM])), 0.0f);
+                    if (a.acq_kind == 0) {
+                        const int64_t o = (int64_t)m * a.ldo + (a.by_index ? i : pos);
+                        a.mean[o] = mean;
+                        a.var[o] = var;
+                    } else {
+                        const float ybest = gscal[2];
+                        const float ei = ei_value(mean, var, ybest, a.xi);
+                        if (a.acq_kind == 1) {
+                            a.acq[i] = ei;
+                        } else {
+                            a.acq[i] = ucb_value(mean, var, a.kappa);
+                            a.acq[a.lda + i] = pi_value(mean, var, ybest, a.xi);
+                            a.acq[2 * a.lda + i] = ei;
+                        }
+                    }
                 }
             }
             i_cur = i_nxt;

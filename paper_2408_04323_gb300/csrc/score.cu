@@ -680,8 +680,9 @@ scoot_status dispatch_m(scoot_ctx* ctx, const ScoreArgs& a, int M, cudaStream_t 
     }
 }
 
-// The state part of the tensor-core posterior's arguments.
-ScootTcArgs tc_args(scoot_ctx* ctx, const ScoreArgs& a) {
+// The state part of the tensor-core posterior's arguments, for the first
+// nobj objectives.
+ScootTcArgs tc_args(scoot_ctx* ctx, const ScoreArgs& a, int nobj) {
     ScootTcArgs t;
     std::memset(&t, 0, sizeof(t));
     t.state = a.state;
@@ -695,13 +696,13 @@ ScootTcArgs tc_args(scoot_ctx* ctx, const ScoreArgs& a) {
     t.off_linv = a.off_linv;
     t.n_obs = a.n_obs;
     t.d = a.d;
-    t.n_obj = a.n_obj;
+    t.n_obj = nobj;
     t.kernel = a.kernel;
     t.n_pad = a.n_rb * kRB;
     t.n_ord = a.n_ord;
     t.n_pat = a.n_pat;
     t.n_tiles = a.n_tiles;
-    const int64_t cat = (int64_t)a.n_obj * a.n_obs * a.n_pat;
+    const int64_t cat = (int64_t)nobj * a.n_obs * a.n_pat;
     t.cat_smem = (a.n_ord < a.d && cat <= kCatSmemMax) ? (int32_t)cat : 0;
     t.err = ctx->d_err;
     return t;
@@ -709,6 +710,40 @@ ScootTcArgs tc_args(scoot_ctx* ctx, const ScoreArgs& a) {
 
 // Padded ordinal feature count of the kernels (DO).
 int tc_do(const ScoreArgs& a) { return a.n_ord <= 4 ? 4 : a.n_ord <= 8 ? 8 : a.n_ord <= 12 ? 12 : 16; }
+
+// The tensor-core route of the entry points that take moments or an
+// acquisition straight from the posterior, without V: t carries the outputs
+// (mean / var, or the acquisition epilogue) and a.cand / n / ld the pool.
+// Workspace: the compacted list (when masked), then the split copy of
+// L^{-1}, reserved whole before the compaction writes the list; where the
+// mask is 0 the compaction writes -inf into the fill_rows rows of the
+// acquisition.  *used is false (nothing launched) when the context has the
+// tensor cores off or the model does not fit the tensor-core kernel.
+scoot_status tc_direct(scoot_ctx* ctx, const ScoreArgs& a, const uint8_t* mask, ScootTcArgs t, int fill_rows,
+                       cudaStream_t st, bool* used) {
+    *used = false;
+    if (!ctx->tensor_cores || a.n_rb * kRB > kMaxNpadTc) return SCOOT_OK;
+    const int DO = tc_do(a);
+    if (!scoot_tc_supported(ctx, t, DO)) return SCOOT_OK;
+    *used = true;
+    const size_t list_bytes = mask ? ((256 + (size_t)a.n * 4 + 255) & ~(size_t)255) : 0;
+    scoot_status s = scoot_workspace(ctx, list_bytes + (size_t)scoot_tc_bsplit_bytes(t.n_pad, t.n_obj));
+    if (s != SCOOT_OK) return s;
+    if (mask) {
+        ScootList lst;
+        uint32_t* fill = t.acq_kind ? reinterpret_cast<uint32_t*>(t.acq) : nullptr;
+        if ((s = scoot_compact(ctx, mask, a.n, fill, 0xFF800000u, st, &lst, fill_rows, t.lda)) != SCOOT_OK) return s;
+        t.list = lst.list;
+        t.n_list = lst.count;
+    }
+    t.cand = a.cand;
+    t.n = a.n;
+    t.ld = a.ld;
+    t.vout = nullptr;
+    t.by_index = 1;
+    t.bsplit = static_cast<uint8_t*>(ctx->ws) + list_bytes;
+    return scoot_posterior_tc(ctx, t, DO, st);
+}
 
 }  // namespace
 
@@ -720,7 +755,7 @@ scoot_status scoot_posterior_whitened(scoot_ctx* ctx, const scoot_gp_layout* L, 
     scoot_status s = fill_state_args(ctx, L, state, a);
     if (s != SCOOT_OK) return s;
     if (tc_work && ctx->tensor_cores) {
-        ScootTcArgs t = tc_args(ctx, a);
+        ScootTcArgs t = tc_args(ctx, a, a.n_obj);
         t.cand = cand;
         t.n = n;
         t.ld = ld;
@@ -767,33 +802,13 @@ scoot_status scoot_gp_posterior(scoot_ctx* ctx, const scoot_gp_layout* L, const 
     a.var = var;
     a.ldo = ldo;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (ctx->tensor_cores && a.n_rb * kRB <= kMaxNpadTc) {
-        // Workspace: the compacted list (when masked), then the split copy of
-        // L^{-1}; reserved whole before the compaction writes the list.
-        ScootTcArgs t = tc_args(ctx, a);
-        const int DO = tc_do(a);
-        if (scoot_tc_supported(ctx, t, DO)) {
-            const size_t list_bytes = mask ? ((256 + (size_t)n * 4 + 255) & ~(size_t)255) : 0;
-            if ((s = scoot_workspace(ctx, list_bytes + (size_t)scoot_tc_bsplit_bytes(t.n_pad, t.n_obj))) != SCOOT_OK)
-                return s;
-            if (mask) {
-                ScootList lst;
-                if ((s = scoot_compact(ctx, mask, n, nullptr, 0u, st, &lst)) != SCOOT_OK) return s;
-                t.list = lst.list;
-                t.n_list = lst.count;
-            }
-            t.cand = cand;
-            t.n = n;
-            t.ld = ld;
-            t.mean = mean;
-            t.var = var;
-            t.ldo = ldo;
-            t.vout = nullptr;
-            t.by_index = 1;
-            t.bsplit = static_cast<uint8_t*>(ctx->ws) + list_bytes;
-            return scoot_posterior_tc(ctx, t, DO, st);
-        }
-    }
+    ScootTcArgs t = tc_args(ctx, a, a.n_obj);
+    t.mean = mean;
+    t.var = var;
+    t.ldo = ldo;
+    bool used = false;
+    s = tc_direct(ctx, a, mask, t, 0, st, &used);
+    if (used || s != SCOOT_OK) return s;
     return launch_score<kWriteMoments, 1>(ctx, a, st);
 }
 
@@ -962,7 +977,16 @@ scoot_status scoot_score_ei(scoot_ctx* ctx, const scoot_gp_layout* L, const void
     a.mask = mask;
     a.acq = acq;
     a.xi = xi;
-    return launch_score<kEI, 1>(ctx, a, static_cast<cudaStream_t>(stream));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    ScootTcArgs t = tc_args(ctx, a, 1);
+    t.acq_kind = 1;
+    t.acq = acq;
+    t.lda = n;
+    t.xi = xi;
+    bool used = false;
+    s = tc_direct(ctx, a, mask, t, 1, st, &used);
+    if (used || s != SCOOT_OK) return s;
+    return launch_score<kEI, 1>(ctx, a, st);
 }
 
 scoot_status scoot_score_mace(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,
@@ -984,7 +1008,17 @@ scoot_status scoot_score_mace(scoot_ctx* ctx, const scoot_gp_layout* L, const vo
     a.lda = lda;
     a.xi = xi;
     a.kappa = kappa;
-    return launch_score<kMACE, 1>(ctx, a, static_cast<cudaStream_t>(stream));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    ScootTcArgs t = tc_args(ctx, a, 1);
+    t.acq_kind = 2;
+    t.acq = acq;
+    t.lda = lda;
+    t.xi = xi;
+    t.kappa = kappa;
+    bool used = false;
+    s = tc_direct(ctx, a, mask, t, 3, st, &used);
+    if (used || s != SCOOT_OK) return s;
+    return launch_score<kMACE, 1>(ctx, a, st);
 }
 
 scoot_status scoot_score_ehvi(scoot_ctx* ctx, const scoot_gp_layout* L, const void* state,

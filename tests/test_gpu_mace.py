@@ -110,8 +110,10 @@ def _gp(S, inst):
     return L, dev(blob)
 
 
-def test_score_mace_parity(S, ctx):
-    """Fused posterior + (UCB, PI, EI) against the oracle's fp64 posterior."""
+@pytest.mark.parametrize("tc", [1, 0], ids=["tensor", "simt"])
+def test_score_mace_parity(S, ctx, tc):
+    """Fused posterior + (UCB, PI, EI) against the oracle's fp64 posterior,
+    with either product of L^{-1} k (tensor cores or fp32 SIMT)."""
     name = "d10-ei"
     n = 8192 + 77
     inst = make_instance(name, seeds(name)[1], n_cand=n)
@@ -121,8 +123,12 @@ def test_score_mace_parity(S, ctx):
     S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
     kappa, xi = 6.31, 1e-4
     acq = torch.full((3, n), 5.0, device="cuda")
-    S.scoot_score_mace(ctx, L, state, cand, n, xi, kappa, acq, mask)
-    g = np_(acq)
+    S.scoot_ctx_set_tensor_cores(ctx, tc)
+    try:
+        S.scoot_score_mace(ctx, L, state, cand, n, xi, kappa, acq, mask)
+        g = np_(acq)
+    finally:
+        S.scoot_ctx_set_tensor_cores(ctx, 1)
     known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
     assert np.all(g[:, ~known] == -np.inf) and np.all(np.isfinite(g[:, known]))
     idx = np.nonzero(known)[0]
@@ -136,14 +142,13 @@ def test_score_mace_parity(S, ctx):
         want, tol = propagated_tol(f, mu, var, e_mu, e_var)
         tol = tol + rounding_tol(mu[:, 0], var[:, 0], yb, xi, kappa)[r]
         ratio = np.abs(g[r, idx] - want) / tol
-        print(f"[parity] score_mace {name} row {r}: n={len(idx)} max|err|/tol={ratio.max():.3f}")
+        print(f"[parity] score_mace {name} tc={tc} row {r}: n={len(idx)} max|err|/tol={ratio.max():.3f}")
         rows.append(ratio.max())
     assert max(rows) <= 1.0
-    # the fused kernel agrees with posterior + acq_mace (the posterior's product in fp32 SIMT, as
-    # in the fused kernel)
+    # the fused kernel agrees with posterior + acq_mace (the posterior with the same product)
     mean = torch.empty((1, n), device="cuda")
     vv = torch.empty((1, n), device="cuda")
-    S.scoot_ctx_set_tensor_cores(ctx, 0)
+    S.scoot_ctx_set_tensor_cores(ctx, tc)
     try:
         S.scoot_gp_posterior(ctx, L, state, cand, n, mean, vv, mask)
     finally:

@@ -446,7 +446,11 @@ def test_score_ehvi_four_objectives_at_large_scale(S, ctx):
     assert report_tol(f"score_ehvi M=4 at scale 1e3 (P={fs}, B={len(lo)})", g[idx], want, tol).max() <= 1.0
 
 
-def test_score_ei_parity(S, ctx):
+@pytest.mark.parametrize("tc", [1, 0], ids=["tensor", "simt"])
+def test_score_ei_parity(S, ctx, tc):
+    """Posterior + EI in one launch, at the full d10-ei pool, with either
+    product of L^{-1} k (the tensor-core kernel's EI epilogue, the fused SIMT
+    kernel)."""
     name = "d10-ei"
     inst = make_instance(name, seeds(name)[0])
     n = inst.n_cand
@@ -454,9 +458,13 @@ def test_score_ei_parity(S, ctx):
     cand = cand_dev(inst)
     mask = torch.empty(n, dtype=torch.uint8, device="cuda")
     S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
-    acq = torch.empty(n, device="cuda")
-    S.scoot_score_ei(ctx, L, state, cand, n, 1e-4, acq, mask)
-    g = np_(acq)
+    acq = torch.full((n,), 5.0, device="cuda")
+    S.scoot_ctx_set_tensor_cores(ctx, tc)
+    try:
+        S.scoot_score_ei(ctx, L, state, cand, n, 1e-4, acq, mask)
+        g = np_(acq)
+    finally:
+        S.scoot_ctx_set_tensor_cores(ctx, 1)
     known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
     assert np.array_equal(np.isfinite(g), known)
     top = np.argsort(-np.where(known, g, -np.inf))[:64]
@@ -466,7 +474,7 @@ def test_score_ei_parity(S, ctx):
     yb = float(inst.y_obs[0].max())
     f = lambda a, b: O.expected_improvement(a[:, 0], b[:, 0], yb, 1e-4)
     want, tol = propagated_tol(f, mu, var, e_mu, e_var)
-    assert report_tol("score_ei d10-ei", g[idx], want, tol).max() <= 1.0
+    assert report_tol(f"score_ei d10-ei {'tensor' if tc else 'simt'}", g[idx], want, tol).max() <= 1.0
 
 
 # ------------------------------------------------------------------ top-q (Section 4.7)

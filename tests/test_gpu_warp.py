@@ -80,8 +80,10 @@ def test_warped_posterior_parity(S, ctx, name, kernel):
         assert np.abs(mu0 - mu).max() > 1e-2
 
 
-def test_warped_score_ei_matern32(S, ctx):
-    """The paper's kernel: Matérn-3/2 with input warping, fused with EI."""
+@pytest.mark.parametrize("tc", [1, 0], ids=["tensor", "simt"])
+def test_warped_score_ei_matern32(S, ctx, tc):
+    """The paper's kernel: Matérn-3/2 with input warping, fused with EI
+    (either product of L^{-1} k)."""
     name = "d10-ei"
     n = 8192 + 5
     inst = make_instance(name, seeds(name)[2], n_cand=n)
@@ -91,8 +93,12 @@ def test_warped_score_ei_matern32(S, ctx):
     mask = torch.empty(n, dtype=torch.uint8, device="cuda")
     S.scoot_prune(ctx, inst.space, inst.clauses, cand, n, mask)
     acq = torch.empty(n, device="cuda")
-    S.scoot_score_ei(ctx, L, state, cand, n, 1e-4, acq, mask)
-    g = np_(acq)
+    S.scoot_ctx_set_tensor_cores(ctx, tc)
+    try:
+        S.scoot_score_ei(ctx, L, state, cand, n, 1e-4, acq, mask)
+        g = np_(acq)
+    finally:
+        S.scoot_ctx_set_tensor_cores(ctx, 1)
     known = O.prune_mask(inst.space, inst.clauses, inst.cand, n)
     idx = np.nonzero(known)[0][::3]
     mu, var, e_mu, e_var = posterior_tols(oracle_gps(inst, warp, 1), np.ascontiguousarray(inst.cand[:, idx]))
@@ -100,7 +106,7 @@ def test_warped_score_ei_matern32(S, ctx):
     f = lambda a, b: O.expected_improvement(a[:, 0], b[:, 0], yb, 1e-4)
     want, tol = propagated_tol(f, mu, var, e_mu, e_var)
     ratio = np.abs(g[idx] - want) / tol
-    print(f"[parity] warped Matérn-3/2 score_ei: n={len(idx)} max|err|/tol={ratio.max():.3f}")
+    print(f"[parity] warped Matérn-3/2 score_ei tc={tc}: n={len(idx)} max|err|/tol={ratio.max():.3f}")
     assert ratio.max() <= 1.0
 
 
