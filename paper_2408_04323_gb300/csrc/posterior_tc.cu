@@ -131,6 +131,28 @@ __device__ __forceinline__ bool mbar_wait(uint32_t addr, uint32_t parity) {
     }
 }
 
+// The covariance's square root and exponential on the MUFU unit: sqrt.approx
+// and ex2.approx (relative error of order 2^-22 each; exp(-a) = 2^(-a log2 e),
+// the product's rounding adding a relative 2^-24 a), a few instructions fewer
+// per covariance than the IEEE-rounded sqrtf and expf.  At a > 20, where the
+// product's rounding weighs most, k < 4e-7 s_f^2.
+constexpr float kLog2e = 1.4426950408889634f;
+__device__ __forceinline__ float sqrt_hw(float x) {
+    float y;
+    asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float ex2_hw(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+// The Matérn polynomial factor at a = sqrt(2 nu) r: 1 + a (nu = 3/2) or
+// 1 + a + a^2 / 3 (nu = 5/2).
+__device__ __forceinline__ float matern_poly(float a, bool m32) {
+    return m32 ? 1.0f + a : fmaf(a, fmaf(a, 0.33333333333333333f, 1.0f), 1.0f);
+}
+
 // B = L^{-1} of every objective, split into bf16 parts, per k-block of 32
 // columns in the canonical layout: [M][n_pad / 32][3][n_pad rows x 64 bytes].
 // One thread per (objective, k-block, row, group of 8 columns).
@@ -359,6 +381,8 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                 const float* alm = al + (size_t)m * a.n_pad;
                 const float sf2 = gscal[m * 4 + 0];
                 const bool warped = gscal[m * 4 + 3] != 0.0f;
+                const bool m32 = a.kernel == SCOOT_MATERN32;
+                const float kc = m32 ? 1.7320508075688772f : 2.2360679774997896f;
                 const float* catrow = (a.cat_smem ? cat_s : gcat) + (size_t)m * a.n_obs * a.n_pat + pid;
                 float ut[DO];
 #pragma unroll
@@ -411,11 +435,14 @@ __global__ void __launch_bounds__(kThr + 32, 1) posterior_tc_kernel(const __grid
                             r2v[e + h] = r2;
                         }
                     }
-                    float kv[8];
+                    float kv[8], ex[8];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) kv[e] = sqrtf(r2v[e]);
+                    for (int e = 0; e < 8; ++e) kv[e] = sqrt_hw(r2v[e]) * kc;  // a = sqrt(2 nu) r
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) kv[e] = (live && c0 + e < a.n_obs) ? sf2 * matern(kv[e], a.kernel) : 0.0f;
+                    for (int e = 0; e < 8; ++e) ex[e] = ex2_hw(kv[e] * -kLog2e);  // exp(-a)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        kv[e] = (live && c0 + e < a.n_obs) ? sf2 * matern_poly(kv[e], m32) * ex[e] : 0.0f;
 #pragma unroll
                     for (int e = 0; e < 8; ++e) mu_part = fmaf(kv[e], alm[c0 + e], mu_part);
                     if (kb + 1 < KB) {
