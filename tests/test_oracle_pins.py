@@ -944,6 +944,27 @@ def test_sobol_skip_and_configs():
     assert f.min() >= 0.5 and f.max() < 0.95
 
 
+def test_sobol_configs_mapping_values():
+    """The mappings of the shortfall fill (Section 4.6) at the first eight
+    points of the first dimension (the van der Corput points k / 8, pinned
+    above), worked by hand: integer log-uniform on [1, 1024] is 1024^u =
+    2^(10 u) rounded (2^1.25 = 2.38, 2^2.5 = 5.66, 2^3.75 = 13.45, 2^6.25 =
+    76.1, 2^7.5 = 181.02, 2^8.75 = 430.5 + 0.04); integer uniform on [3, 9]
+    is 3 + floor(7 u); a categorical of 5 choices floor(5 u); continuous on
+    [0.5, 0.95] is 0.5 + 0.45 u."""
+    u = [0.0, 0.5, 0.25, 0.75, 0.125, 0.625, 0.375, 0.875]  # points 0 .. 7
+    log_at = {0.0: 1, 0.125: 2, 0.25: 6, 0.375: 13, 0.5: 32, 0.625: 76, 0.75: 181, 0.875: 431}
+    uni_at = {0.0: 3, 0.125: 3, 0.25: 4, 0.375: 5, 0.5: 6, 0.625: 7, 0.75: 8, 0.875: 9}
+    cat_at = {0.0: 0, 0.125: 0, 0.25: 1, 0.375: 1, 0.5: 2, 0.625: 3, 0.75: 3, 0.875: 4}
+    for kind, lo, hi, want in ((INT_LOG, 1, 1024, log_at), (INT_UNIFORM, 3, 9, uni_at)):
+        w = O.sobol_configs(_space((kind, 0, lo, hi)), 8).view(np.int32)[0]
+        assert w.tolist() == [want[x] for x in u], kind
+    w = O.sobol_configs(_space((CATEGORICAL, 5, 0, 0)), 8).view(np.int32)[0]
+    assert w.tolist() == [cat_at[x] for x in u]
+    f = O.sobol_configs(_space((CONTINUOUS, 0, 0.5, 0.95)), 8).view(np.float32)[0]
+    assert f.tolist() == [float(np.float32(0.5 + 0.45 * x)) for x in u]
+
+
 def test_delta_controller_trajectory():
     """Worked by hand from Algorithm 1 with k = 2 and step 0.05."""
     d, c = 0.5, 0
