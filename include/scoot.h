@@ -11,7 +11,7 @@
  *   scoot_gp_mle         GP hyperparameters by maximum likelihood (Section 4.3)
  *   scoot_acq_ei         expected improvement, Eq. (6)
  *   scoot_acq_ehvi       Monte-Carlo expected hypervolume improvement, Eq. (7)
- *   scoot_score_ei       posterior + EI in one kernel
+ *   scoot_score_ei       posterior + EI in one pass
  *   scoot_score_ehvi     posterior + EHVI in one kernel
  *   scoot_score_ehvi_exact  posterior + exact EHVI (independent Gaussians)
  *   scoot_select_topq    top-q for parallel suggestion (Section 4.7)
@@ -399,9 +399,13 @@ scoot_status scoot_acq_ehvi(scoot_ctx* ctx, const float* mean, const float* var,
                             const float* box_lo, const float* box_hi, int32_t n_boxes,
                             const float* eps, int32_t n_mc, float* acq, void* stream);
 
-/* scoot_gp_posterior followed by scoot_acq_ei, in one kernel, without
+/* scoot_gp_posterior followed by scoot_acq_ei, in one pass, without
  * writing mean or variance (objective 0; y_best is the state's best
- * observed value of objective 0). */
+ * observed value of objective 0).  With the context's tensor cores on and
+ * at most 256 observations the pass is the tensor-core posterior with an EI
+ * epilogue (after a small kernel that splits L^{-1} into bf16 parts in the
+ * context workspace), else one fused fp32 kernel; where mask[i] == 0,
+ * acq[i] = -inf. */
 scoot_status scoot_score_ei(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
                             const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
                             float xi, float* acq, void* stream);
@@ -715,8 +719,9 @@ scoot_status scoot_acq_mace(scoot_ctx* ctx, const float* mean, const float* var,
                             int64_t n, float y_best, float xi, float kappa, float* acq, int64_t lda,
                             void* stream);
 
-/* scoot_gp_posterior followed by scoot_acq_mace, in one kernel (objective 0;
- * y_best is the state's best observed value of objective 0). */
+/* scoot_gp_posterior followed by scoot_acq_mace, in one pass (objective 0;
+ * y_best is the state's best observed value of objective 0), on the tensor
+ * cores or in one fused fp32 kernel as scoot_score_ei. */
 scoot_status scoot_score_mace(scoot_ctx* ctx, const scoot_gp_layout* layout, const void* state,
                               const uint32_t* cand, int64_t n, int64_t ld, const uint8_t* mask,
                               float xi, float kappa, float* acq, int64_t lda, void* stream);
