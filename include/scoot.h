@@ -154,8 +154,9 @@ scoot_status scoot_ctx_workspace_bytes(const scoot_ctx* ctx, int64_t* bytes);
 #define SCOOT_PHASE_SCATTER        5   /* variances scattered to var_out */
 scoot_status scoot_ctx_set_timing(scoot_ctx* ctx, int32_t enable);
 
-/* Tensor cores for the whitened posterior (on by default).  With enable != 0
- * the posterior of scoot_suggest_fantasy / scoot_fantasy_begin computes
+/* Tensor cores for the posterior (on by default).  With enable != 0 the
+ * posterior of scoot_gp_posterior, scoot_score_ei, scoot_score_mace and
+ * scoot_suggest_fantasy / scoot_fantasy_begin computes
  * V = L^{-1} k(X, x) on the tcgen05 tensor cores when the padded observation
  * count is at most 256 and the state fits a block's shared memory: each fp32
  * operand split into three bf16 parts, six part products accumulated in fp32
