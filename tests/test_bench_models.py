@@ -94,3 +94,18 @@ def test_scoring_work_model(name):
     assert wm["topq"] == ("hbm", 5)
     mace = bench.work_model(inst, B, "mace")["score"][1]
     assert mace == n * (3 * d + 12) + 2 * n + n * (n + 1) + 2 * n + 47
+
+
+@pytest.mark.parametrize("name", ["d8-ehvi2", "d10-ei", "d12-fantasy"])
+def test_tensor_flops_count_the_issued_part_products(name):
+    """bf16 flops per candidate of the tensor-core posterior: every (row i,
+    column c) pair the MMAs touch (rows from the first row of c's 32-column
+    k-block on, the rest of the triangle skipped), six part products of two
+    flops each, per objective; enumerated pair by pair here."""
+    inst = make_instance(name, seeds(name)[0], n_cand=16)
+    n_pad = 64 * ((inst.n_obs + 63) // 64)
+    pairs = sum(1 for i in range(n_pad) for c in range(n_pad) if i >= 32 * (c // 32))
+    assert bench.posterior_tensor_flops(inst) == inst.n_obj * 6 * 2 * pairs
+    assert bench.posterior_tensor_flops(inst, 1) == 6 * 2 * pairs
+    # at least the triangle, at most the square
+    assert n_pad * (n_pad + 1) // 2 <= pairs <= n_pad * n_pad
